@@ -1,0 +1,76 @@
+/*
+ * oracle.h — plain, single-threaded CPU statement of the lineage expand /
+ * ready-queue batch / gather-commit / assemble semantics of RayOrch
+ * (arXiv 2609.18703, Sections 4.2-4.5).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the test suite, the smoke check and the
+ * benchmark's CPU-baseline leg may load or call this code.  It shares no
+ * code, header, table or helper with the GPU library; both follow the paper.
+ *
+ * Every array is host memory.  Sizes are element counts.  Status and code
+ * numbering is the same as the GPU library's so that outputs compare
+ * directly; the numbers are restated here, not included from there.
+ */
+#ifndef RO_ORACLE_H
+#define RO_ORACLE_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* call status */
+enum { OR_OK = 0, OR_E_INVAL = 1, OR_E_CAPACITY = 2, OR_E_OVERFLOW = 3, OR_E_STATE = 4,
+       OR_E_OOM = 5 };
+/* Item outcomes of Eq. (1) as carried by reports and assembled parents */
+enum { OR_PENDING = 0, OR_PRESENT = 1, OR_DROPPED = 2, OR_FAILED = 3, OR_SUPPRESSED = 4 };
+/* per-report verdicts of the generation fence, Eq. (3) */
+enum { OR_ACCEPT = 0, OR_REJ_INVALID = 1, OR_REJ_NOT_INFLIGHT = 2, OR_REJ_STALE_GEN = 3,
+       OR_REJ_DUPLICATE = 4 };
+/* Grain phases of Eq. (2) */
+enum { OR_WAITING = 0, OR_READY = 1, OR_IN_FLIGHT = 2, OR_SEALED = 3 };
+
+typedef struct or_ctx or_ctx;
+
+typedef struct {
+  uint64_t accepted, rej_invalid, rej_not_inflight, rej_stale_gen, rej_duplicate;
+  uint64_t ready_bad_candidates;    /* candidates naming no child of the expansion */
+  uint64_t assemble_incomplete;     /* listed parents that were not complete */
+} or_stats;
+
+or_ctx* or_ctx_create(uint32_t n_calls);
+void    or_ctx_destroy(or_ctx* ctx);
+void    or_ctx_reset(or_ctx* ctx);
+void    or_ctx_stats(const or_ctx* ctx, or_stats* out);
+
+/* Expansion (Section 4.2): offsets = exclusive prefix sum of counts, one
+ * child per (parent, ordinal) numbered parent-major; empty expansions are
+ * terminal at once and listed (ascending) in empty_parents. */
+int or_expand(or_ctx* ctx, int32_t parent_xid, const uint32_t* counts, uint64_t n_parents,
+              const uint8_t* parent_call, uint64_t* offsets, uint32_t* child_parent,
+              uint32_t* child_ordinal, uint64_t child_cap, uint32_t* empty_parents,
+              uint64_t* n_children, uint64_t* n_empty, int32_t* xid);
+
+/* Per-Call FIFO Ready Queue with elastic reservation (Section 4.3, Eq. 2). */
+int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand,
+                   uint64_t n_cand, uint32_t batch_size, int32_t flush, uint32_t* batched,
+                   uint64_t batched_cap, uint64_t* n_batched, uint64_t* n_batches);
+
+/* Generation-fenced commit (Section 4.4, Eq. 3) and parent completion
+ * (Section 4.2, Reduce); completed parents listed ascending. */
+int or_gather_commit(or_ctx* ctx, int32_t xid, uint64_t n, const uint32_t* child,
+                     const uint8_t* state, const uint32_t* len, const uint64_t* off,
+                     const uint32_t* gen, uint64_t arena_bytes, uint8_t* code,
+                     uint32_t* done_parents, uint64_t done_cap, uint64_t* n_done);
+
+/* Ordered Reduce output (Section 4.2): parents == NULL assembles the parents
+ * completed by the latest commit on xid. */
+int or_assemble(or_ctx* ctx, int32_t xid, const uint8_t* arena, uint64_t arena_bytes,
+                const uint32_t* parents, uint64_t n_parents, uint8_t* status,
+                uint64_t* out_off, uint32_t* out_len, uint8_t* out, uint64_t out_cap,
+                uint64_t* out_cursor, uint64_t* out_bytes, uint64_t* n_assembled);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

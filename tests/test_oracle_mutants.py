@@ -1,0 +1,47 @@
+"""The oracle's pins must catch plausible mistakes.  Each case plants one
+mistake in a private copy of the oracle's C source (on the CPU), builds it,
+and runs the pin suite against it; the suite has to fail."""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+MUTANTS = {
+    "ordinal_off_by_one": ("child_ordinal[c] = j;", "child_ordinal[c] = j + 1;"),
+    "flush_ignored": ("uint64_t take = flush ? queued : (queued / batch_size) * batch_size;",
+                      "uint64_t take = (queued / batch_size) * batch_size;"),
+    "readmits_queued": ("if (x->phase[c] != OR_WAITING) continue;", ";"),
+    "fence_ignores_generation": ("} else if (g != x->gen[c]) {", "} else if (0) {"),
+    "completion_off_by_one": ("if (x->terminal[p] == member_count(x, p)) x->last_done[k++] = p;",
+                              "if (x->terminal[p] + 1 == member_count(x, p)) x->last_done[k++] = p;"),
+    "dropped_suppresses": ("if (s == OR_FAILED || s == OR_SUPPRESSED) x->bad[p] = 1;",
+                           "if (s != OR_PRESENT) x->bad[p] = 1;"),
+    "source_index_shift": ("memcpy(out + pos, arena + x->off[c], x->len[c]);",
+                           "memcpy(out + pos, arena + x->off[c] + 1, x->len[c]);"),
+    "done_list_unsorted": ("qsort(x->last_done, k, sizeof(uint32_t), cmp_u32);", "(void)cmp_u32;"),
+    "len_off_transposed": ("x->off[c] = (s == OR_PRESENT) ? off[r] : 0;",
+                           "x->off[c] = (s == OR_PRESENT) ? len[r] : 0;"),
+    "scan_extra_term": ("offsets[p + 1] = offsets[p] + counts[p];",
+                        "offsets[p + 1] = offsets[p] + counts[p] + (p == 1);"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_catch_planted_mistake(name, tmp_path):
+    before, after = MUTANTS[name]
+    src = open(os.path.join(ROOT, "oracle", "oracle.c")).read()
+    assert src.count(before) == 1, f"mutation site for {name} not unique"
+    (tmp_path / "oracle.c").write_text(src.replace(before, after))
+    shutil.copy(os.path.join(ROOT, "oracle", "oracle.h"), tmp_path / "oracle.h")
+    so = tmp_path / "libmutant.so"
+    subprocess.run(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-w", "-o", str(so),
+                    str(tmp_path / "oracle.c")], check=True)
+    env = dict(os.environ, ORACLE_LIB=str(so))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle.py")],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode != 0, f"pins did not catch mutant {name}:\n{r.stdout[-2000:]}"

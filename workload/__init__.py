@@ -1,0 +1,14 @@
+"""Seeded synthetic inputs shared by the oracle checks, the GPU tests and the bench.
+
+Holds no lineage arithmetic: it draws counts, per-child results, arrival and
+readiness orders, and fills result payload bytes from a counter-based hash.
+"""
+from .configs import (CONFIGS, FAILED, DROPPED, PRESENT, SUPPRESSED, Level, Workload,
+                      docpage, skew, streaming, tiny, video)
+from .payload import fill_host_arena, mix64, record_bytes, records_concat
+
+__all__ = [
+    "CONFIGS", "PRESENT", "DROPPED", "FAILED", "SUPPRESSED", "Level", "Workload",
+    "tiny", "docpage", "video", "skew", "streaming",
+    "fill_host_arena", "mix64", "record_bytes", "records_concat",
+]
