@@ -1,0 +1,475 @@
+#!/usr/bin/env python
+"""Benchmark of the lineage expand -> FIFO batch -> gather-commit -> assemble
+pass on GB300 (one JSON line on stdout from rank 0).
+
+Workload (default): the document->page configuration — 1,000,000 parents,
+pages per parent lognormal(2.3, 1.0) in [1, 2000] (about 16.4M children),
+payload lognormal(7.5, 0.8) bytes in [256 B, 64 KB], 5 % FAILED, results
+arriving in 256 random waves, batch size 256.  Synthetic, seeded inputs
+(workload/) stand in for the paper's corpora.
+
+One step = ro_expand + ro_batch_ready (all children, flush) + 256 x
+(ro_gather_commit + ro_assemble of the parents that wave completed), with the
+inputs and the 39 GB result arena resident in HBM.  The wave loop is replayed
+from a CUDA graph (it is launch-bound: 5 kernels per wave).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Multi-GPU (torchrun): every rank runs its own source microbatch (weak
+scaling, no collective on the data path); the step time is the max over
+ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "children/sec expand->gather->assemble at 1 GB300; payload GB/s as % of HBM peak"
+K_ACOPY = 8
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--parents", type=int, default=1_000_000)
+    ap.add_argument("--waves", type=int, default=256)
+    ap.add_argument("--no-graph", action="store_true", help="launch the wave loop eagerly")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--cpu-parents", type=int, default=40_000,
+                    help="parents in the oracle's bounded CPU sample")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ----------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples (200 ms) while the timed region runs."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.t = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        if self.t:
+            self.t.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ CPU oracle
+def cpu_oracle_sample(parents: int, waves: int):
+    """Time the oracle (single-threaded C) on a bounded sample of the same
+    workload: the first `parents` documents of the same distribution."""
+    from oracle import OracleCtx
+    from tests.pipeline import host_arena
+    from workload import docpage
+    lv = docpage(parents=parents, waves=waves, salt=1).top
+    arena = host_arena(lv)
+    o = OracleCtx()
+    t0 = time.perf_counter()
+    x = o.expand(lv.counts)["xid"]
+    o.batch_ready(x, 0, None, lv.batch_size, flush=True)
+    total = 0
+    for w in range(lv.n_waves):
+        ch, st, ln, of = lv.reports(lv.wave(w))
+        cm = o.gather_commit(x, ch, st, ln, of, arena_bytes=lv.arena_bytes)
+        a = o.assemble(x, arena, parents=None, n_parents=max(cm["n_done"], 1))
+        total += a["out_bytes"]
+    dt = time.perf_counter() - t0
+    o.close()
+    return lv.n_children / dt, dt, lv.n_children, total
+
+
+def run_reference(args, rank):
+    if rank != 0:
+        return
+    v, dt, n, _ = cpu_oracle_sample(args.cpu_parents, args.waves)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(v, 1), "unit": "children/s",
+        "n_gpus": args.gpus, "steps": 1, "warmup": 0, "ms_per_step": round(dt * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8/u32/u64",
+        "data": "synthetic",
+        "config": {"workload": f"document->page, {args.cpu_parents} of 1,000,000 parents "
+                               f"(bounded CPU sample), {args.waves} waves",
+                   "global_batch": n, "parallelism": "single-threaded oracle"},
+        "cpu_baseline": {"value": round(v, 1), "unit": "children/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{args.cpu_parents} parents / {n} children, full pass"},
+        "e2e": {"value": round(v, 1), "unit": "children/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------ GPU
+class Pass:
+    """Device-resident inputs and outputs of one document->page microbatch."""
+
+    def __init__(self, lv, device, stream):
+        import torch
+        from workload.device import fill_payload
+        self.torch = torch
+        self.lv = lv
+        self.P, self.N, self.W, self.B = lv.n_parents, lv.n_children, lv.n_waves, lv.batch_size
+        dev = torch.device("cuda", device)
+        self.stream = stream
+        i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).to(dev)
+        i64 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int64)).to(dev)
+        u8 = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+        arr = lv.arrival
+        self.counts = i32(lv.counts)
+        # reports, in arrival order; wave w = [bounds[w], bounds[w+1])
+        self.child = i32(arr)
+        self.state = u8(lv.state[arr])
+        self.length = i32(lv.length[arr])
+        self.off = i64(lv.arena_off[arr])
+        self.bounds = lv.wave_bounds.astype(np.int64)
+        self.arena_bytes = int(lv.arena_bytes)
+        self.arena = torch.empty(max(self.arena_bytes, 16), dtype=torch.uint8, device=dev)
+        off_c, len_c = i64(lv.arena_off), i32(lv.length)
+        fill_payload(self.arena, off_c, len_c, lv.payload_seed, stream)
+        torch.cuda.synchronize(dev)
+        del off_c, len_c
+        self.out_cap = self.arena_bytes + 64
+        self.out = torch.empty(self.out_cap, dtype=torch.uint8, device=dev)
+        self.offsets = torch.empty(self.P + 1, dtype=torch.int64, device=dev)
+        self.cp = torch.empty(self.N, dtype=torch.int32, device=dev)
+        self.co = torch.empty(self.N, dtype=torch.int32, device=dev)
+        self.batched = torch.empty(self.N + self.B, dtype=torch.int32, device=dev)
+        self.n_batched = torch.zeros(1, dtype=torch.int64, device=dev)
+        self.status = torch.empty(self.P, dtype=torch.uint8, device=dev)
+        self.out_off = torch.empty(self.P + 1, dtype=torch.int64, device=dev)
+        self.out_len = torch.empty(self.P, dtype=torch.int32, device=dev)
+        self.cursor = torch.zeros(1, dtype=torch.int64, device=dev)
+        self.out_bytes = torch.zeros(self.W, dtype=torch.int64, device=dev)
+
+    def expand(self, ro, ctx):
+        st, n, ne, xid = ro.ro_expand(ctx, -1, self.counts, self.P, None, self.offsets, self.cp,
+                                      self.co, self.N, None)
+        if st != 0:
+            raise RuntimeError(f"ro_expand: {st} {ro.ro_last_error(ctx)}")
+        assert n == self.N
+        return xid
+
+    def waves(self, ro, ctx, xid):
+        """batch_ready + every wave's commit and assemble; asynchronous."""
+        L = ro.load()
+        st = L.ro_batch_ready(ctx, xid, 0, None, 0, self.B, 1, self.batched.data_ptr(),
+                              self.N + self.B, self.n_batched.data_ptr(), None, None)
+        bad = st
+        self.cursor.zero_()
+        cb, sb, lb, ob = (self.child.data_ptr(), self.state.data_ptr(), self.length.data_ptr(),
+                          self.off.data_ptr())
+        ar, st_p, oo, ol, out = (self.arena.data_ptr(), self.status.data_ptr(),
+                                 self.out_off.data_ptr(), self.out_len.data_ptr(),
+                                 self.out.data_ptr())
+        cur, obw = self.cursor.data_ptr(), self.out_bytes.data_ptr()
+        for w in range(self.W):
+            s, e = int(self.bounds[w]), int(self.bounds[w + 1])
+            bad |= L.ro_gather_commit(ctx, xid, e - s, None, cb + 4 * s, sb + s, lb + 4 * s,
+                                      ob + 8 * s, None, self.arena_bytes, None, None, 0, None, None)
+            bad |= L.ro_assemble(ctx, xid, ar, self.arena_bytes, None, self.P, None, st_p, oo, ol,
+                                 out, self.out_cap, cur, obw + 8 * w, None)
+        if bad:
+            raise RuntimeError(f"wave loop: status {bad}: {ro.ro_last_error(ctx)}")
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import __graft_entry__
+    import paper_2609_18703_gb300 as ro
+    from workload import docpage
+
+    torch.cuda.set_device(local_rank)
+    __graft_entry__.build()
+    hbm_peak, peak_kind = peaks()
+    lv = docpage(parents=args.parents, waves=args.waves, salt=rank).top
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
+    ps = Pass(lv, local_rank, stream)
+    ctx = ro.ro_ctx_create(local_rank, stream, 1)
+
+    def step_eager():
+        ro.ro_ctx_reset(ctx)
+        xid = ps.expand(ro, ctx)
+        ps.waves(ro, ctx, xid)
+
+    graph = None
+    per_replay = 0
+
+    def step_graph():
+        ro.ro_ctx_reset(ctx)
+        ps.expand(ro, ctx)
+        graph.replay()
+
+    # warm-up (sizes every buffer), then capture the wave loop once
+    for _ in range(max(1, args.warmup)):
+        step_eager()
+    stream.synchronize()
+    if ro.ro_ctx_sync(ctx) != 0:
+        raise RuntimeError(ro.ro_last_error(ctx))
+    if not args.no_graph:
+        ro.ro_ctx_reset(ctx)
+        xid = ps.expand(ro, ctx)
+        ro.ro_ctx_profile_read(ctx)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            ps.waves(ro, ctx, xid)
+        per_replay = sum(v[0] for v in ro.ro_ctx_profile_read(ctx).values())   # captured launches
+        for _ in range(args.warmup):
+            step_graph()
+    step = step_eager if graph is None else step_graph
+    stream.synchronize()
+    ro.ro_ctx_profile_read(ctx)   # reset launch counters
+
+    # ---- timed region
+    dist = world > 1
+    if dist:
+        import torch.distributed as td
+        td.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for _ in range(args.steps):
+        step()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        td.barrier()
+    clk = clocks.stop()
+    ms_total = t_start.elapsed_time(t_end)
+    prof = ro.ro_ctx_profile_read(ctx)
+    launches_timed = sum(v[0] for v in prof.values())
+    if graph is not None:   # replays launch the kernels captured once
+        launches_timed += args.steps * per_replay
+    st = ro.ro_ctx_sync(ctx)
+    if st != 0:
+        raise RuntimeError(f"device reported {st}: {ro.ro_last_error(ctx)}")
+    S = int(ps.out_bytes.sum().item())
+    if dist:
+        t = torch.tensor([ms_total], dtype=torch.float64)
+        td.all_reduce(t, op=td.ReduceOp.MAX)
+        ms_total = float(t.item())
+    ms_step = ms_total / args.steps
+    value = world * ps.N / (ms_step * 1e-3)
+
+    # ---- per-kernel timing of the copy kernel (events on its launch stream)
+    ro.ro_ctx_profile(ctx, 1 << K_ACOPY)
+    kt_steps = max(2, min(args.steps, 5))
+    for _ in range(kt_steps):
+        step_eager()
+    stream.synchronize()
+    prof = ro.ro_ctx_profile_read(ctx)
+    ro.ro_ctx_profile(ctx, 0)
+    n_copy, _, copy_ms = prof["asm_copy"][0], prof["asm_copy"][1], prof["asm_copy"][2]
+    copy_bytes = 2.0 * S * kt_steps   # payload read + write, algorithmic
+    achieved = copy_bytes / (copy_ms * 1e-3) / 1e9 if copy_ms > 0 else 0.0
+    pass_alg = 33.0 * ps.N + 25.0 * ps.P + 2.0 * S
+    kernel_ms = {k: round(v[2] / kt_steps, 4) for k, v in prof.items() if v[1]}
+
+    # ---- end to end through the C ABI with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, ps, ro, ctx, stream, world)
+
+    cpu = None
+    if rank == 0 and not args.no_cpu:
+        v_cpu, dt_cpu, n_cpu, _ = cpu_oracle_sample(args.cpu_parents, args.waves)
+        cpu = {"value": round(v_cpu, 1), "unit": "children/s", "cores": 1, "kind": "oracle",
+               "sample": f"document->page, first {args.cpu_parents} parents ({n_cpu} children) "
+                         f"of the same distributions, {args.waves} waves, full pass in {dt_cpu:.2f} s"}
+
+    if rank == 0:
+        payload_gbs = 2.0 * S / (ms_step * 1e-3) / 1e9
+        line = {
+            "metric": METRIC, "value": round(value, 1), "unit": "children/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "u8/u32/u64", "data": "synthetic",
+            "config": {"workload": f"document->page: {ps.P} parents, {ps.N} children, "
+                                   f"{args.waves} arrival waves, batch {ps.B}",
+                       "parents": ps.P, "children": ps.N, "waves": args.waves,
+                       "arena_bytes": ps.arena_bytes, "assembled_bytes": S,
+                       "cuda_graph": graph is not None,
+                       "l2": "inputs larger than L2 (39 GB arena)",
+                       "parallelism": f"replicas x{world} (one microbatch per GPU)"},
+            "payload_gbs": round(payload_gbs, 1),
+            "payload_frac_of_hbm": round(payload_gbs / hbm_peak, 4),
+            "algorithmic_gbs": round(pass_alg / (ms_step * 1e-3) / 1e9, 1),
+            "algorithmic_frac_of_hbm": round(pass_alg / (ms_step * 1e-3) / 1e9 / hbm_peak, 4),
+            "roofline": {"kernel": "asm_copy", "bound": "hbm", "achieved": round(achieved, 1),
+                         "peak": hbm_peak, "peak_kind": peak_kind, "unit": "GB/s",
+                         "frac": round(achieved / hbm_peak, 4), "traffic": None,
+                         "launches": n_copy, "avg_launch_ms": round(copy_ms / max(n_copy, 1), 5)},
+            "kernel_ms_per_step": kernel_ms,
+            "gpu_launches": int(launches_timed),
+            "clocks": clk,
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    ro.ro_ctx_destroy(ctx)
+
+
+def run_e2e(args, ps, ro, ctx, stream, world):
+    """Same pass through the public API with pinned host buffers: each step
+    copies its inputs (counts, reports, result payloads) to the device and the
+    assembled outputs back to the host inside the timed region."""
+    import torch
+    P, N, W = ps.P, ps.N, ps.W
+    pin = lambda t: t.cpu().pin_memory()
+    h_counts, h_child, h_state, h_len, h_off = (pin(ps.counts), pin(ps.child), pin(ps.state),
+                                               pin(ps.length), pin(ps.off))
+    # the arena is laid out in arrival order: wave w's payloads are one contiguous range
+    off_np = ps.lv.arena_off[ps.lv.arrival]
+    len_np = ps.lv.length[ps.lv.arrival]
+    wave_lo, wave_hi = [], []
+    for w in range(W):
+        s, e = int(ps.bounds[w]), int(ps.bounds[w + 1])
+        m = len_np[s:e] > 0
+        lo = int(off_np[s:e][m].min()) if m.any() else 0
+        hi = int((off_np[s:e][m] + len_np[s:e][m]).max()) if m.any() else 0
+        wave_lo.append(lo)
+        wave_hi.append(hi)
+    try:
+        h_arena = torch.empty(ps.arena_bytes, dtype=torch.uint8).pin_memory()
+        h_out = torch.empty(ps.out_cap, dtype=torch.uint8).pin_memory()
+    except Exception as exc:   # host memory
+        return {"value": None, "unit": "children/s", "note": f"pinned host buffers unavailable: {exc}"}
+    _d2h_chunks(ps.arena, h_arena)
+    L = ro.load()
+
+    def step():
+        ps.counts.copy_(h_counts, non_blocking=True)
+        ro.ro_ctx_reset(ctx)
+        xid = ps.expand(ro, ctx)
+        L.ro_batch_ready(ctx, xid, 0, None, 0, ps.B, 1, ps.batched.data_ptr(), N + ps.B,
+                         ps.n_batched.data_ptr(), None, None)
+        ps.cursor.zero_()
+        for w in range(W):
+            s, e = int(ps.bounds[w]), int(ps.bounds[w + 1])
+            for d, h in ((ps.child, h_child), (ps.state, h_state), (ps.length, h_len), (ps.off, h_off)):
+                d[s:e].copy_(h[s:e], non_blocking=True)
+            lo, hi = wave_lo[w], wave_hi[w]
+            if hi > lo:
+                ps.arena[lo:hi].copy_(h_arena[lo:hi], non_blocking=True)
+            L.ro_gather_commit(ctx, xid, e - s, None, ps.child.data_ptr() + 4 * s,
+                               ps.state.data_ptr() + s, ps.length.data_ptr() + 4 * s,
+                               ps.off.data_ptr() + 8 * s, None, ps.arena_bytes, None, None, 0, None,
+                               None)
+            L.ro_assemble(ctx, xid, ps.arena.data_ptr(), ps.arena_bytes, None, P, None,
+                          ps.status.data_ptr(), ps.out_off.data_ptr(), ps.out_len.data_ptr(),
+                          ps.out.data_ptr(), ps.out_cap, ps.cursor.data_ptr(),
+                          ps.out_bytes.data_ptr() + 8 * w, None)
+        torch.cuda.current_stream().synchronize()
+        S = int(ps.cursor.item())
+        h_out[:S].copy_(ps.out[:S])
+        return S
+
+    step()
+    torch.cuda.synchronize()
+    steps = max(1, min(args.steps, 3))
+    t0 = time.perf_counter()
+    S = 0
+    for _ in range(steps):
+        S = step()
+    torch.cuda.synchronize()
+    dt = (time.perf_counter() - t0) / steps
+    h2d = 4 * P + N * (4 + 1 + 4 + 8) + sum(h - l for l, h in zip(wave_lo, wave_hi))
+    return {"value": round(world * N / dt, 1), "unit": "children/s", "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(S), "ms_per_step": round(dt * 1e3, 3)}
+
+
+def _d2h_chunks(src, dst):
+    chunk = 1 << 30
+    for s in range(0, src.numel(), chunk):
+        dst[s:s + chunk].copy_(src[s:s + chunk])
+    return dst
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as td
+        td.init_process_group("gloo")
+    if args.impl == "reference":
+        run_reference(args, rank)
+    else:
+        run_ours(args, rank, world, local_rank)
+    if world > 1:
+        import torch.distributed as td
+        td.barrier()
+        td.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

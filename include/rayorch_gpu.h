@@ -1,0 +1,251 @@
+/*
+ * rayorch_gpu.h — C ABI of the GB300 (sm_103a) lineage expand / gather path.
+ *
+ * The library keeps, on one GPU, the structural lineage state that RayOrch
+ * (arXiv 2609.18703) maintains for an ordered, variable-cardinality
+ * parent -> child expansion and its matching ordered gather:
+ *
+ *   ro_expand         Section 4.2, Table 2, Eq. (1): child offsets, each
+ *                     child's immediate parent and immutable ordinal.
+ *   ro_batch_ready    Section 4.3, Eq. (2): per-Call FIFO Ready Queue and
+ *                     elastic reservation into fixed-size batches.
+ *   ro_gather_commit  Section 4.4, Eq. (3) and Section 4.2 (Reduce):
+ *                     generation-fenced commit of out-of-order child results,
+ *                     per-parent terminal counting, completed-parent list.
+ *   ro_assemble       Section 4.2 (Reduce): each completed parent's Present
+ *                     child payloads concatenated in ordinal order.
+ *
+ * Conventions for every entry point
+ * ---------------------------------
+ * - Pointers prefixed d_ are device memory of the context's GPU; h_ are host
+ *   memory.  The caller allocates and owns every pointer it passes; the
+ *   library never keeps a caller pointer beyond the call (except the arena,
+ *   see ro_gather_commit).  A context owns its internal lineage state
+ *   (phase words, result slots, parent counters, queues, scratch).
+ * - All work is issued on the context's stream, in call order.  Calls return
+ *   without waiting for the GPU unless an h_ output is requested: a non-NULL
+ *   h_ pointer makes the call synchronise the stream and fill it in.  The
+ *   d_ count outputs are written by the GPU in stream order, so a following
+ *   call can consume them (the d_n inputs) without a host round trip.
+ * - Errors are returned as ro_status; nothing throws across the ABI.
+ *   Argument errors the host can see are RO_E_INVAL with no side effects.
+ *   Conditions only the GPU can see (an output too small, a wait that timed
+ *   out) are recorded in the context and returned by the next call that
+ *   synchronises (any call with an h_ output, or ro_ctx_sync); the call that
+ *   hit them leaves lineage state as it was.  CUDA runtime errors give
+ *   RO_E_CUDA and stick to the context.
+ * - Limits: fewer than 2^32 parents and 2^32 children per expansion; arena
+ *   offsets and sizes below 2^48; at most 256 Calls per context; payload
+ *   lengths are uint32.
+ */
+#ifndef RAYORCH_GPU_H
+#define RAYORCH_GPU_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct ro_ctx ro_ctx;
+typedef int32_t ro_status;
+
+/* call status */
+enum {
+  RO_OK = 0,
+  RO_E_INVAL = 1,     /* bad argument; nothing changed */
+  RO_E_CAPACITY = 2,  /* an output buffer is too small; nothing changed, retry */
+  RO_E_OVERFLOW = 3,  /* a count or size exceeds the limits above */
+  RO_E_STATE = 4,     /* the call does not fit the lineage state (unknown xid, ...) */
+  RO_E_OOM = 5,       /* device memory for internal state could not be allocated */
+  RO_E_CUDA = 6,      /* a CUDA runtime error; sticky until ro_ctx_destroy */
+  RO_E_TIMEOUT = 7    /* a bounded device-side wait gave up; results of that call are void */
+};
+
+/* Item outcomes of Eq. (1), as carried by reports and by assembled parents */
+enum {
+  RO_PENDING = 0,     /* not (yet) complete */
+  RO_PRESENT = 1,
+  RO_DROPPED = 2,
+  RO_FAILED = 3,
+  RO_SUPPRESSED = 4
+};
+
+/* per-report verdict of the generation fence, Eq. (3) */
+enum {
+  RO_ACCEPT = 0,
+  RO_REJ_INVALID = 1,       /* no such child, unknown outcome, or payload outside the arena */
+  RO_REJ_NOT_INFLIGHT = 2,  /* the child's Grain is WAITING or READY */
+  RO_REJ_STALE_GEN = 3,     /* generation differs from the Grain's current one */
+  RO_REJ_DUPLICATE = 4      /* the Grain is already SEALED (earlier report, or an earlier
+                               report of the same call) */
+};
+
+/* cumulative counters of a context (since create or the last reset) */
+typedef struct {
+  uint64_t accepted, rej_invalid, rej_not_inflight, rej_stale_gen, rej_duplicate;
+  uint64_t ready_bad_candidates;  /* batch_ready candidates naming no child */
+  uint64_t assemble_incomplete;   /* assembled list entries that were not complete */
+} ro_stats;
+
+/* ------------------------------------------------------------------------
+ * Context = one source microbatch (Sections 1 and 4.3: Ready Queues and
+ * ordered gathering are scoped to one input microbatch).  `stream` is a
+ * cudaStream_t (NULL = legacy default stream) on device `device`; n_calls in
+ * [1, 256] is the number of Calls whose Ready Queues the context keeps.
+ */
+ro_status ro_ctx_create(ro_ctx** ctx, int32_t device, void* stream, uint32_t n_calls);
+ro_status ro_ctx_destroy(ro_ctx* ctx);
+/* Forget every expansion (start the next microbatch).  Device memory is kept
+ * and reused by later expansions of the same or smaller size. */
+ro_status ro_ctx_reset(ro_ctx* ctx);
+/* Wait for the stream and return (then clear) any condition recorded by the GPU. */
+ro_status ro_ctx_sync(ro_ctx* ctx);
+/* Synchronise and copy the cumulative counters. */
+ro_status ro_ctx_stats(ro_ctx* ctx, ro_stats* out);
+/* Text of the last error on this context ("" if none).  Valid until the next call. */
+const char* ro_last_error(const ro_ctx* ctx);
+
+/* Kernel ids for the profiling calls below, in launch order of the path. */
+enum {
+  RO_K_EXPAND_SCAN = 0, RO_K_EXPAND_FILL = 1, RO_K_READY_COUNT = 2, RO_K_READY_SCATTER = 3,
+  RO_K_COMMIT_SCATTER = 4, RO_K_COMMIT_FINISH = 5, RO_K_ASM_PARENTS = 6, RO_K_ASM_MEMBERS = 7,
+  RO_K_ASM_COPY = 8, RO_K_COUNT = 9
+};
+/* Tracing (no counterpart in the paper; it instruments the path).  Every
+ * kernel launch is counted; kernels whose bit (1 << RO_K_*) is set in
+ * kernel_mask are also bracketed by a pair of CUDA events on the context's
+ * stream.  Recording events costs host time per launch, so time few kernels. */
+ro_status ro_ctx_profile(ro_ctx* ctx, uint32_t kernel_mask);
+/* Synchronise, then copy per kernel (arrays of n_kernels entries, any may be
+ * NULL): launches since the last read, launches timed, and their summed
+ * device milliseconds.  Resets the counters. */
+ro_status ro_ctx_profile_read(ro_ctx* ctx, uint64_t* launches, uint64_t* timed, double* ms,
+                              uint32_t n_kernels);
+
+/* ------------------------------------------------------------------------
+ * ro_expand — materialise one Expansion (Section 4.2; Table 2 gives the child
+ * key (parent, ordinal); Eq. (1) makes an empty child list terminal).
+ *
+ *   parent_xid    -1 for a root expansion, else the xid whose children are
+ *                 the parents here (nested levels); n_parents must then equal
+ *                 that expansion's child count.
+ *   d_counts      uint32[n_parents]  children of each parent (read only).
+ *   d_parent_call uint8[n_parents] or NULL: the Call that consumes each
+ *                 parent's children (NULL: Call 0).
+ *   d_offsets     uint64[n_parents+1] out: exclusive prefix sum of counts;
+ *                 d_offsets[n_parents] = number of children N.
+ *   d_child_parent, d_child_ordinal  uint32[child_cap] out: for child c
+ *                 (numbered parent-major, c = d_offsets[p] + ordinal) its
+ *                 immediate parent and zero-based ordinal.
+ *   d_empty_parents uint32[n_parents] out or NULL: ascending ids of parents
+ *                 with no children; they are complete at once and can be
+ *                 assembled (Present, empty).
+ *   h_n_children, h_n_empty  out (required / optional): N and the number
+ *                 of empty parents.  This call always synchronises.
+ *   xid           out: handle of the new expansion.
+ * Errors: RO_E_CAPACITY if N > child_cap (h_n_children holds N, no expansion
+ * is created); RO_E_OVERFLOW if N >= 2^32.
+ */
+ro_status ro_expand(ro_ctx* ctx, int32_t parent_xid, const uint32_t* d_counts,
+                    uint64_t n_parents, const uint8_t* d_parent_call, uint64_t* d_offsets,
+                    uint32_t* d_child_parent, uint32_t* d_child_ordinal, uint64_t child_cap,
+                    uint32_t* d_empty_parents, uint64_t* h_n_children, uint64_t* h_n_empty,
+                    int32_t* xid);
+
+/* ------------------------------------------------------------------------
+ * ro_batch_ready — admission into the per-Call FIFO Ready Queue and elastic
+ * reservation (Section 4.3, Eq. 2).
+ *
+ * Candidates are taken in order; a candidate enters Call `call`'s queue of
+ * expansion xid (WAITING -> READY) when it names a child of xid whose Grain
+ * is WAITING and which belongs to that Call.  A child named twice enters once,
+ * at its first position.  Then whole batches of batch_size are taken from the
+ * head of the queue (READY -> IN-FLIGHT); with flush != 0 the trailing partial
+ * batch is taken too.  Entries left in the queue stay READY for the next call.
+ *
+ *   d_cand      uint32[n_cand] child ids in readiness order, or NULL for all
+ *               children of xid in id order (n_cand ignored).  n_cand < 2^30.
+ *   d_batched   uint32[batched_cap] out: the reserved children; batch k is
+ *               d_batched[k*batch_size ...].  Batches mix parents freely.
+ *   d_n_batched uint64 out (device) or NULL: number reserved.
+ *   h_n_batched, h_n_batches out (host) or NULL: number reserved and number of
+ *               batches; either makes the call synchronise.
+ * Errors: RO_E_CAPACITY when more would be reserved than batched_cap (reported
+ * when the context next synchronises; queue and phases unchanged).
+ */
+ro_status ro_batch_ready(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* d_cand,
+                         uint64_t n_cand, uint32_t batch_size, int32_t flush,
+                         uint32_t* d_batched, uint64_t batched_cap, uint64_t* d_n_batched,
+                         uint64_t* h_n_batched, uint64_t* h_n_batches);
+
+/* ------------------------------------------------------------------------
+ * ro_gather_commit — generation-fenced commit of child results (Section 4.4,
+ * Eq. 3) and per-parent completion (Section 4.2, Reduce).
+ *
+ * Report r names child d_child[r] with outcome d_state[r] (RO_PRESENT,
+ * RO_DROPPED, RO_FAILED or RO_SUPPRESSED); a Present report's value is the
+ * d_len[r] bytes at arena offset d_arena_off[r] (ignored for other outcomes).
+ * A report is accepted when the child's Grain is IN-FLIGHT and d_gen[r] is
+ * its current generation; the Grain becomes SEALED and the outcome is
+ * published for good.  Reports of one call are applied as if one after
+ * another in array order (the first of several reports for one Grain wins).
+ * A parent completes when all of its children are sealed.
+ *
+ *   n, d_n      report count (host), or a device uint64 count (d_n != NULL;
+ *               n is then an upper bound used for launch sizing).
+ *   d_gen       uint32[n] or NULL (generation 0).
+ *   arena_bytes size of the result arena the offsets refer to.  The arena
+ *               bytes of accepted Present reports must stay unchanged until
+ *               their parents are assembled.
+ *   d_code      uint8[n] out or NULL: RO_ACCEPT or an RO_REJ_* verdict.
+ *               Rejected reports change nothing.
+ *   d_done_parents uint32[done_cap] out or NULL: parents completed by this
+ *               call, ascending.  done_cap must be >= min(n, parents of xid).
+ *   d_n_done (device) / h_n_done (host, synchronises) out or NULL.
+ */
+ro_status ro_gather_commit(ro_ctx* ctx, int32_t xid, uint64_t n, const uint64_t* d_n,
+                           const uint32_t* d_child, const uint8_t* d_state,
+                           const uint32_t* d_len, const uint64_t* d_arena_off,
+                           const uint32_t* d_gen, uint64_t arena_bytes, uint8_t* d_code,
+                           uint32_t* d_done_parents, uint64_t done_cap, uint64_t* d_n_done,
+                           uint64_t* h_n_done);
+
+/* ------------------------------------------------------------------------
+ * ro_assemble — ordered Reduce output (Section 4.2).
+ *
+ * For each listed parent: if it is not complete, status RO_PENDING and no
+ * bytes; if a child Failed or was Suppressed, RO_SUPPRESSED and no bytes;
+ * otherwise RO_PRESENT and the Present children's payloads concatenated in
+ * ordinal order (Dropped children add nothing; no survivors give 0 bytes).
+ * Parents are written back to back, in list order, starting at d_out + base
+ * where base = *d_out_cursor (if given) or 0; the cursor then advances.
+ *
+ *   d_arena      the result arena the committed reports referred to.
+ *   d_parents    uint32[n_parents] parent ids, or NULL for the parents
+ *                completed by the latest ro_gather_commit on xid (in its
+ *                ascending order); n_parents is then the capacity of the
+ *                per-parent outputs.  d_n_parents (device count) may replace
+ *                n_parents for an explicit list.
+ *   d_status     uint8[n] out; d_out_off uint64[n+1] out: byte offsets into
+ *                d_out (entry n = end); d_out_len uint32[n] out or NULL.
+ *                With d_out_len, RO_E_OVERFLOW if a parent exceeds 2^32-1 bytes.
+ *   d_out        uint8[out_cap] out.  Byte-exact, no padding; any alignment.
+ *   d_out_bytes (device) / h_out_bytes (host, synchronises) out or NULL:
+ *                bytes written by this call.
+ * Together, (d_parents or the commit's list, d_status, d_out_len, d_out_off)
+ * have the layout of a report array, so an assembled level can be committed
+ * as the results of the level above (nested expansions).
+ * Errors: RO_E_CAPACITY when base + bytes > out_cap or the list is longer
+ * than n_parents (nothing is copied).
+ */
+ro_status ro_assemble(ro_ctx* ctx, int32_t xid, const uint8_t* d_arena, uint64_t arena_bytes,
+                      const uint32_t* d_parents, uint64_t n_parents, const uint64_t* d_n_parents,
+                      uint8_t* d_status, uint64_t* d_out_off, uint32_t* d_out_len,
+                      uint8_t* d_out, uint64_t out_cap, uint64_t* d_out_cursor,
+                      uint64_t* d_out_bytes, uint64_t* h_out_bytes);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* RAYORCH_GPU_H */

@@ -340,7 +340,9 @@ int or_assemble(or_ctx* ctx, int32_t xid, const uint8_t* arena, uint64_t arena_b
   if (out_bytes) *out_bytes = total;
   if (base + total > out_cap) return OR_E_CAPACITY;
   if (out_len && len_overflow) return OR_E_OVERFLOW;
-  if (total && (!out || !arena)) return OR_E_INVAL;
+  /* arena and out both NULL: outcomes and offsets only, no bytes copied */
+  const int sizes_only = !out && !arena;
+  if (total && !sizes_only && (!out || !arena)) return OR_E_INVAL;
 
   uint64_t pos = base;
   for (uint64_t i = 0; i < n; ++i) {
@@ -355,7 +357,7 @@ int or_assemble(or_ctx* ctx, int32_t xid, const uint8_t* arena, uint64_t arena_b
       status[i] = OR_PRESENT;
       for (uint64_t c = x->offsets[p]; c < x->offsets[p + 1]; ++c) {
         if (x->st[c] != OR_PRESENT) continue;   /* Dropped members are excluded */
-        memcpy(out + pos, arena + x->off[c], x->len[c]);
+        if (!sizes_only) memcpy(out + pos, arena + x->off[c], x->len[c]);
         pos += x->len[c];
       }
     }

@@ -64,7 +64,8 @@ int or_gather_commit(or_ctx* ctx, int32_t xid, uint64_t n, const uint32_t* child
                      uint32_t* done_parents, uint64_t done_cap, uint64_t* n_done);
 
 /* Ordered Reduce output (Section 4.2): parents == NULL assembles the parents
- * completed by the latest commit on xid. */
+ * completed by the latest commit on xid.  With arena and out both NULL only
+ * the outcomes and offsets are produced (no bytes copied). */
 int or_assemble(or_ctx* ctx, int32_t xid, const uint8_t* arena, uint64_t arena_bytes,
                 const uint32_t* parents, uint64_t n_parents, uint8_t* status,
                 uint64_t* out_off, uint32_t* out_len, uint8_t* out, uint64_t out_cap,

@@ -185,6 +185,8 @@ class OracleCtx:
     def assemble(self, xid: int, arena: Optional[np.ndarray], parents=None,
                  n_parents: Optional[int] = None, out_cap: Optional[int] = None,
                  cursor: Optional[int] = None, want_len: bool = True, check: bool = True):
+        """Assemble ``parents`` (None: the latest commit's completed parents).
+        With ``arena=None`` only outcomes and offsets are computed (no bytes)."""
         parents = _arr(parents, np.uint32)
         if parents is not None:
             n = parents.size
@@ -195,17 +197,21 @@ class OracleCtx:
         out_len = np.zeros(max(n, 1), dtype=np.uint32) if want_len else None
         arena_u8 = None if arena is None else _arr(arena, np.uint8)
         arena_bytes = 0 if arena_u8 is None else arena_u8.size
+        sizes_only = arena_u8 is None
         if out_cap is None:
-            # first ask for the size (capacity 0 returns E_CAPACITY with the byte count)
-            ob = C.c_uint64(0)
-            na = C.c_uint64(0)
-            cur0 = C.c_uint64(cursor or 0)
-            lib().or_assemble(self._h, xid, _ptr(arena_u8, _u8p), arena_bytes,
-                              _ptr(parents, _u32p), n, _ptr(status, _u8p),
-                              _ptr(out_off, _u64p), None, None, 0,
-                              C.byref(cur0), C.byref(ob), C.byref(na))
-            out_cap = (cursor or 0) + ob.value
-        out = np.zeros(max(out_cap, 1), dtype=np.uint8)
+            if sizes_only:
+                out_cap = (1 << 62)
+            else:
+                # ask for the size first (capacity 0 reports the byte count)
+                ob = C.c_uint64(0)
+                na = C.c_uint64(0)
+                cur0 = C.c_uint64(cursor or 0)
+                lib().or_assemble(self._h, xid, _ptr(arena_u8, _u8p), arena_bytes,
+                                  _ptr(parents, _u32p), n, _ptr(status, _u8p),
+                                  _ptr(out_off, _u64p), None, None, 0,
+                                  C.byref(cur0), C.byref(ob), C.byref(na))
+                out_cap = (cursor or 0) + ob.value
+        out = None if sizes_only else np.zeros(max(out_cap, 1), dtype=np.uint8)
         ob = C.c_uint64(0)
         na = C.c_uint64(0)
         cur = C.c_uint64(cursor) if cursor is not None else None
@@ -219,5 +225,5 @@ class OracleCtx:
         k = na.value
         return dict(status=st, parent_status=status[:k].copy(), out_off=out_off[:k + 1].copy(),
                     out_len=None if out_len is None else out_len[:k].copy(),
-                    out=out[:out_cap], out_bytes=ob.value, n_assembled=k,
-                    cursor=None if cur is None else cur.value)
+                    out=None if out is None else out[:out_cap], out_bytes=ob.value,
+                    n_assembled=k, cursor=None if cur is None else cur.value)

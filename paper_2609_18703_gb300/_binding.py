@@ -1,0 +1,210 @@
+"""Thin ctypes binding of the C ABI in include/rayorch_gpu.h.
+
+Function names and argument order follow the C entry points.  Pointer
+arguments accept a torch tensor (its data_ptr), a raw integer address or
+None; host outputs (the h_ pointers) are returned instead of passed.  A
+``want_host=False`` keeps a call asynchronous (no h_ outputs, no sync).
+
+Nothing here computes: every step runs in libro_gb300.so.  If the library
+is missing the import of a function raises instead of falling back.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from typing import Optional
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libro_gb300.so")
+
+# call status
+RO_OK, RO_E_INVAL, RO_E_CAPACITY, RO_E_OVERFLOW, RO_E_STATE, RO_E_OOM, RO_E_CUDA, RO_E_TIMEOUT = range(8)
+# Item outcomes (Eq. 1)
+RO_PENDING, RO_PRESENT, RO_DROPPED, RO_FAILED, RO_SUPPRESSED = range(5)
+# report verdicts (Eq. 3)
+RO_ACCEPT, RO_REJ_INVALID, RO_REJ_NOT_INFLIGHT, RO_REJ_STALE_GEN, RO_REJ_DUPLICATE = range(5)
+
+STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFLOW",
+                4: "RO_E_STATE", 5: "RO_E_OOM", 6: "RO_E_CUDA", 7: "RO_E_TIMEOUT"}
+
+EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro_ctx_stats",
+           "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
+           "ro_gather_commit", "ro_assemble")
+
+# kernel ids (RO_K_*), in launch order of the path
+KERNELS = ("expand_scan", "expand_fill", "ready_count", "ready_scatter", "commit_scatter",
+           "commit_finish", "asm_parents", "asm_members", "asm_copy")
+
+
+class RoError(RuntimeError):
+    def __init__(self, fn: str, status: int, msg: str = ""):
+        super().__init__(f"{fn}: {STATUS_NAMES.get(status, status)} {msg}".rstrip())
+        self.status = status
+
+
+class _Stats(C.Structure):
+    _fields_ = [(n, C.c_uint64) for n in (
+        "accepted", "rej_invalid", "rej_not_inflight", "rej_stale_gen", "rej_duplicate",
+        "ready_bad_candidates", "assemble_incomplete")]
+
+
+_lib = None
+_vp = C.c_void_p
+_u64 = C.c_uint64
+_u32 = C.c_uint32
+_i32 = C.c_int32
+_pu64 = C.POINTER(C.c_uint64)
+_pi32 = C.POINTER(C.c_int32)
+
+
+def load(path: Optional[str] = None):
+    """Load libro_gb300.so (built in-tree by ``paper_2609_18703_gb300.build``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = path or LIB_PATH
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with "
+                           "`python -m paper_2609_18703_gb300.build` (needs nvcc)")
+    L = C.CDLL(path)
+    L.ro_ctx_create.argtypes = [C.POINTER(_vp), _i32, _vp, _u32]
+    L.ro_ctx_destroy.argtypes = [_vp]
+    L.ro_ctx_reset.argtypes = [_vp]
+    L.ro_ctx_sync.argtypes = [_vp]
+    L.ro_ctx_stats.argtypes = [_vp, C.POINTER(_Stats)]
+    L.ro_last_error.argtypes = [_vp]
+    L.ro_last_error.restype = C.c_char_p
+    L.ro_ctx_profile.argtypes = [_vp, _u32]
+    L.ro_ctx_profile_read.argtypes = [_vp, _pu64, _pu64, C.POINTER(C.c_double), _u32]
+    L.ro_expand.argtypes = [_vp, _i32, _vp, _u64, _vp, _vp, _vp, _vp, _u64, _vp, _pu64, _pu64, _pi32]
+    L.ro_batch_ready.argtypes = [_vp, _i32, _u32, _vp, _u64, _u32, _i32, _vp, _u64, _vp, _pu64, _pu64]
+    L.ro_gather_commit.argtypes = [_vp, _i32, _u64, _vp, _vp, _vp, _vp, _vp, _vp, _u64, _vp, _vp, _u64,
+                                   _vp, _pu64]
+    L.ro_assemble.argtypes = [_vp, _i32, _vp, _u64, _vp, _u64, _vp, _vp, _vp, _vp, _vp, _u64, _vp, _vp,
+                              _pu64]
+    for f in EXPORTS:
+        if f != "ro_last_error":
+            getattr(L, f).restype = C.c_int32
+    _lib = L
+    return L
+
+
+def _ptr(x):
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        if hasattr(x, "is_cuda") and not x.is_cuda:
+            raise ValueError("device argument is a CPU tensor")
+        return x.data_ptr()
+    raise TypeError(f"cannot pass {type(x)!r} as a pointer")
+
+
+def _stream_handle(stream) -> Optional[int]:
+    if stream is None:
+        return None
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def ro_last_error(ctx) -> str:
+    s = load().ro_last_error(ctx)
+    return s.decode() if s else ""
+
+
+def _check(fn, st, ctx=None, allow=()):
+    if st != RO_OK and st not in allow:
+        raise RoError(fn, st, ro_last_error(ctx) if ctx else "")
+    return st
+
+
+def ro_ctx_create(device: int = 0, stream=None, n_calls: int = 1) -> int:
+    h = _vp()
+    st = load().ro_ctx_create(C.byref(h), device, _stream_handle(stream), n_calls)
+    _check("ro_ctx_create", st)
+    return h.value
+
+
+def ro_ctx_destroy(ctx) -> int:
+    return load().ro_ctx_destroy(ctx)
+
+
+def ro_ctx_reset(ctx) -> int:
+    return load().ro_ctx_reset(ctx)
+
+
+def ro_ctx_sync(ctx) -> int:
+    return load().ro_ctx_sync(ctx)
+
+
+def ro_ctx_stats(ctx) -> dict:
+    s = _Stats()
+    st = load().ro_ctx_stats(ctx, C.byref(s))
+    out = {n: int(getattr(s, n)) for n, _ in _Stats._fields_}
+    out["status"] = st
+    return out
+
+
+def ro_ctx_profile(ctx, kernel_mask: int) -> int:
+    return load().ro_ctx_profile(ctx, kernel_mask)
+
+
+def ro_ctx_profile_read(ctx) -> dict:
+    """{kernel name: (launches, launches timed, summed device ms)} since the last read."""
+    k = len(KERNELS)
+    la = (C.c_uint64 * k)()
+    ti = (C.c_uint64 * k)()
+    ms = (C.c_double * k)()
+    st = load().ro_ctx_profile_read(ctx, la, ti, ms, k)
+    _check("ro_ctx_profile_read", st, ctx)
+    return {name: (int(la[i]), int(ti[i]), float(ms[i])) for i, name in enumerate(KERNELS)}
+
+
+def ro_expand(ctx, parent_xid, d_counts, n_parents, d_parent_call, d_offsets, d_child_parent,
+              d_child_ordinal, child_cap, d_empty_parents=None):
+    """Returns (status, n_children, n_empty, xid)."""
+    n = _u64(0)
+    ne = _u64(0)
+    xid = _i32(-1)
+    st = load().ro_expand(ctx, parent_xid, _ptr(d_counts), n_parents, _ptr(d_parent_call),
+                          _ptr(d_offsets), _ptr(d_child_parent), _ptr(d_child_ordinal), child_cap,
+                          _ptr(d_empty_parents), C.byref(n), C.byref(ne), C.byref(xid))
+    return st, n.value, ne.value, xid.value
+
+
+def ro_batch_ready(ctx, xid, call, d_cand, n_cand, batch_size, flush, d_batched, batched_cap,
+                   d_n_batched=None, want_host: bool = True):
+    """Returns (status, n_batched, n_batches); the counts are None without want_host."""
+    nb = _u64(0)
+    nbt = _u64(0)
+    st = load().ro_batch_ready(ctx, xid, call, _ptr(d_cand), n_cand, batch_size, int(flush),
+                               _ptr(d_batched), batched_cap, _ptr(d_n_batched),
+                               C.byref(nb) if want_host else None,
+                               C.byref(nbt) if want_host else None)
+    return (st, nb.value, nbt.value) if want_host else (st, None, None)
+
+
+def ro_gather_commit(ctx, xid, n, d_n, d_child, d_state, d_len, d_arena_off, d_gen, arena_bytes,
+                     d_code=None, d_done_parents=None, done_cap=0, d_n_done=None,
+                     want_host: bool = True):
+    """Returns (status, n_done); n_done is None without want_host."""
+    nd = _u64(0)
+    st = load().ro_gather_commit(ctx, xid, n, _ptr(d_n), _ptr(d_child), _ptr(d_state), _ptr(d_len),
+                                 _ptr(d_arena_off), _ptr(d_gen), arena_bytes, _ptr(d_code),
+                                 _ptr(d_done_parents), done_cap, _ptr(d_n_done),
+                                 C.byref(nd) if want_host else None)
+    return (st, nd.value) if want_host else (st, None)
+
+
+def ro_assemble(ctx, xid, d_arena, arena_bytes, d_parents, n_parents, d_n_parents, d_status,
+                d_out_off, d_out_len, d_out, out_cap, d_out_cursor=None, d_out_bytes=None,
+                want_host: bool = True):
+    """Returns (status, out_bytes); out_bytes is None without want_host."""
+    ob = _u64(0)
+    st = load().ro_assemble(ctx, xid, _ptr(d_arena), arena_bytes, _ptr(d_parents), n_parents,
+                            _ptr(d_n_parents), _ptr(d_status), _ptr(d_out_off), _ptr(d_out_len),
+                            _ptr(d_out), out_cap, _ptr(d_out_cursor), _ptr(d_out_bytes),
+                            C.byref(ob) if want_host else None)
+    return (st, ob.value) if want_host else (st, None)

@@ -1,0 +1,273 @@
+// k_commit.cu — ro_gather_commit kernels (Section 4.4, Eq. 3; Section 4.2, Reduce).
+//
+// commit_scatter  one thread per report.  The fence of Eq. (3) is a single
+//                 compare-and-swap of the child's phase word from
+//                 IN-FLIGHT(gen) to SEALED(gen); the winner publishes the
+//                 outcome into the child's 16-byte record (one sector) and
+//                 counts the member down at its parent with one 64-bit atomic
+//                 add on (remaining | bad << 32).  Lanes of a warp that hit
+//                 the same parent are merged first (__match_any_sync), so a
+//                 hot parent sees one atomic per warp.  The add that takes
+//                 `remaining` to zero completes the parent and sets its bit in
+//                 a completion bitmap.
+// commit_finish   turns the bitmap into the ascending list of completed
+//                 parents (popcount + single-pass scan over bitmap words) and
+//                 clears it.  When the scatter saw two reports for one Grain
+//                 in the same call (rare), CTA 0 first makes the lowest-index
+//                 report the accepted one, so the result equals applying the
+//                 reports one by one in array order.
+#include <algorithm>
+
+#include "ro_internal.h"
+
+namespace ro {
+
+constexpr uint8_t V_WIN_SEALER = 6, V_WIN_CAND = 7, V_LOSE_SEALER = 8, V_LOSE_CAND = 9;
+
+// record word read past L1 (other threads update it with atomics at L2)
+__device__ __forceinline__ uint64_t ld_w(const Rec* rc) {
+  return __ldcg((const unsigned long long*)&rc->w);
+}
+
+__device__ __forceinline__ uint64_t commit_count(const CommitArgs& a) {
+  if (!a.d_n) return a.n_host;
+  const uint64_t n = *a.d_n;
+  return n < a.n_host ? n : a.n_host;
+}
+
+__global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a) {
+  __shared__ unsigned long long s_cnt[6];
+  DevScalars* ds = a.ds;
+  if (threadIdx.x < 6) s_cnt[threadIdx.x] = 0;
+  __syncthreads();
+  const uint64_t n = commit_count(a);
+  if (a.d_n && *a.d_n > a.n_host && blockIdx.x == 0 && threadIdx.x == 0)
+    atomicOr(&ds->err, ERR_INVAL);
+  const int lane = threadIdx.x & 31;
+  const uint64_t warp_global = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
+  uint32_t cnt[6] = {0, 0, 0, 0, 0, 0};
+  for (uint64_t base = warp_global * 32; base < n; base += n_warps * 32) {
+    const uint64_t r = base + lane;
+    uint8_t v = 255;   // inactive lane
+    uint32_t p = 0;
+    bool bad = false;
+    if (r < n) {
+      const uint64_t c = a.child[r];
+      const uint8_t s = a.state[r];
+      const uint32_t l = a.len[r];
+      const uint64_t o = a.off[r];
+      const uint32_t g = a.gen ? a.gen[r] : 0u;
+      const bool valid_state = s >= ST_PRESENT && s <= ST_SUPPRESSED;
+      const bool in_bounds = s != ST_PRESENT || (o <= a.arena_bytes && (uint64_t)l <= a.arena_bytes - o);
+      if (c >= a.N || !valid_state || !in_bounds) {
+        v = V_INVALID;
+      } else {
+        // Eq. (3): accept iff IN-FLIGHT at the report's generation
+        const uint32_t want = ph_make(PH_INFLIGHT, g);
+        uint32_t cur;
+        bool won = false;
+        if (g >> 30) {
+          cur = a.phase[c];   // no Grain ever reaches such a generation
+        } else {
+          cur = atomicCAS(a.phase + c, want, ph_make(PH_SEALED, g));
+          won = cur == want;
+        }
+        if (won) {
+          v = V_ACCEPT;
+          const bool present = s == ST_PRESENT;
+          Rec* rc = a.rec + c;
+          rc->len = present ? l : 0u;
+          atomicOr((unsigned long long*)&rc->w,
+                   (unsigned long long)((present ? (o & W_OFF_MASK) : 0ull) |
+                                        ((uint64_t)s << W_STATE_SHIFT)));
+          p = rc->parent;
+          bad = (s == ST_FAILED || s == ST_SUPPRESSED);
+        } else if ((cur & 3u) == PH_WAITING || (cur & 3u) == PH_READY) {
+          v = V_NOT_INFLIGHT;
+        } else if ((cur >> 2) != g) {
+          v = V_STALE;
+        } else {
+          // SEALED at this generation: a duplicate, possibly of a report of
+          // this same call with a higher index (ordered by commit_finish)
+          v = V_DUP_CANDIDATE;
+          atomicOr((unsigned long long*)&a.rec[c].w, (unsigned long long)W_CONFLICT_BIT);
+        }
+      }
+      a.code[r] = v;
+    }
+    // merge the accepted lanes of this warp by parent, one atomic per parent
+    const unsigned acc = __ballot_sync(0xffffffffu, v == V_ACCEPT);
+    const unsigned badm = __ballot_sync(0xffffffffu, v == V_ACCEPT && bad);
+    if (v == V_ACCEPT) {
+      const unsigned grp = __match_any_sync(acc, p);
+      if (lane == __ffs(grp) - 1) {
+        const unsigned n_tot = __popc(grp), n_bad = __popc(grp & badm);
+        const unsigned long long delta =
+            ((unsigned long long)n_bad << 32) - (unsigned long long)n_tot;
+        const unsigned long long old = atomicAdd(a.pw + p, delta);
+        if ((uint32_t)old == n_tot) atomicOr(a.bitmap + (p >> 5), 1u << (p & 31));
+      }
+    }
+    if (v < 6) cnt[v == V_DUP_CANDIDATE ? 5 : v] += 1;
+  }
+  // statistics: accepted, invalid, not in flight, stale (duplicates are
+  // counted by the finish pass), candidates for ordering
+#pragma unroll
+  for (int k = 0; k < 6; ++k) {
+    uint32_t x = cnt[k];
+    for (int d = 16; d > 0; d >>= 1) x += __shfl_down_sync(0xffffffffu, x, d);
+    if (lane == 0 && x) atomicAdd(&s_cnt[k], (unsigned long long)x);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int k = 0; k < 4; ++k)
+      if (s_cnt[k]) atomicAdd(&ds->stats[k], s_cnt[k]);
+    if (s_cnt[5]) atomicAdd(&ds->cm_conflicts, s_cnt[5]);
+  }
+}
+
+// Make the lowest-index report of each Grain that was reported more than once
+// in this call the accepted one.  Run by one CTA, only when the scatter saw
+// such reports.
+__device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
+  DevScalars* ds = a.ds;
+  __shared__ unsigned long long s_dups;
+  if (threadIdx.x == 0) s_dups = 0;
+  __syncthreads();
+  // A: this call's sealer of a conflicted Grain marks itself and opens the
+  //    minimum-index election in the record's len field
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    if (a.code[r] != V_ACCEPT) continue;
+    Rec* rc = a.rec + a.child[r];
+    if (ld_w(rc) & W_CONFLICT_BIT) {
+      rc->len = 0xFFFFFFFFu;
+      atomicOr((unsigned long long*)&rc->w, (unsigned long long)W_SEALER_BIT);
+    }
+  }
+  __syncthreads();
+  // B: candidates of Grains sealed in this call vote; the others are plain
+  //    duplicates of an earlier call's publication
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    if (a.code[r] != V_DUP_CANDIDATE) continue;
+    Rec* rc = a.rec + a.child[r];
+    if (ld_w(rc) & W_SEALER_BIT) {
+      atomicMin(&rc->len, (uint32_t)r);
+    } else {
+      a.code[r] = V_DUPLICATE;
+      atomicAnd((unsigned long long*)&rc->w, ~(unsigned long long)W_CONFLICT_BIT);
+      atomicAdd(&s_dups, 1ull);
+    }
+  }
+  __syncthreads();
+  // C: every contender learns whether it won
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    const uint8_t v = a.code[r];
+    if (v != V_ACCEPT && v != V_DUP_CANDIDATE) continue;
+    const Rec* rc = a.rec + a.child[r];
+    if (!(ld_w(rc) & W_SEALER_BIT)) continue;
+    const bool win = __ldcg(&rc->len) == (uint32_t)r;
+    a.code[r] = (v == V_ACCEPT) ? (win ? V_WIN_SEALER : V_LOSE_SEALER)
+                                : (win ? V_WIN_CAND : V_LOSE_CAND);
+  }
+  __syncthreads();
+  // D: the winner writes the record; outcome classes move with it
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    const uint8_t v = a.code[r];
+    if (v < V_WIN_SEALER || v > V_LOSE_CAND) continue;
+    const uint8_t s = a.state[r];
+    const bool bad = (s == ST_FAILED || s == ST_SUPPRESSED);
+    Rec* rc = a.rec + a.child[r];
+    const uint32_t p = rc->parent;
+    if (v == V_WIN_SEALER || v == V_WIN_CAND) {
+      const bool present = s == ST_PRESENT;
+      const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK | W_SEALER_BIT | W_CONFLICT_BIT);
+      rc->len = present ? a.len[r] : 0u;
+      rc->w = keep | (present ? (a.off[r] & W_OFF_MASK) : 0ull) | ((uint64_t)s << W_STATE_SHIFT);
+      if (v == V_WIN_CAND && bad) atomicAdd(a.pw + p, 1ull << 32);
+      a.code[r] = V_ACCEPT;
+    } else {
+      if (v == V_LOSE_SEALER && bad) atomicAdd(a.pw + p, ~((1ull << 32) - 1));   // -(1 << 32)
+      a.code[r] = V_DUPLICATE;
+      atomicAdd(&s_dups, 1ull);
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    atomicAdd(&ds->stats[4], s_dups);
+    ds->cm_conflicts = 0;
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a) {
+  __shared__ unsigned long long s_scan[33];
+  __shared__ uint32_t s_tile;
+  __shared__ unsigned long long s_prefix;
+  DevScalars* ds = a.ds;
+  if (blockIdx.x == 0 && ds->cm_conflicts != 0) resolve_duplicates(a, commit_count(a));
+
+  const uint64_t n_words = ceil_div(a.P, 32);
+  const uint64_t TILE = (uint64_t)CF_THREADS * CF_WORDS;
+  const uint64_t n_tiles = ceil_div(n_words, TILE);
+  for (;;) {
+    if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_COMMIT]);
+    __syncthreads();
+    const uint32_t tile = s_tile;
+    __syncthreads();
+    if (tile >= n_tiles) break;
+    const uint64_t w0 = tile * TILE + (uint64_t)threadIdx.x * CF_WORDS;
+    uint32_t words[CF_WORDS];
+    unsigned long long cnt = 0;
+#pragma unroll
+    for (int k = 0; k < CF_WORDS; ++k) {
+      words[k] = (w0 + k < n_words) ? a.bitmap[w0 + k] : 0u;
+      cnt += __popc(words[k]);
+    }
+    unsigned long long total;
+    unsigned long long excl = block_excl_scan(cnt, s_scan, &total);
+    if (threadIdx.x == 0) s_prefix = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_COMMIT], &ds->err);
+    __syncthreads();
+    unsigned long long pos = s_prefix + excl;
+#pragma unroll
+    for (int k = 0; k < CF_WORDS; ++k) {
+      uint32_t bits = words[k];
+      if (!bits) continue;
+      a.bitmap[w0 + k] = 0u;
+      while (bits) {
+        const int b = __ffs(bits) - 1;
+        bits &= bits - 1;
+        const uint32_t parent = (uint32_t)((w0 + k) * 32 + b);
+        a.done_int[pos] = parent;
+        if (a.done_user) a.done_user[pos] = parent;
+        ++pos;
+      }
+    }
+    if (tile == n_tiles - 1 && threadIdx.x == CF_THREADS - 1) {
+      ds->cm_n_done = pos;
+      if (a.n_done_out) *a.n_done_out = pos;
+    }
+  }
+  if (threadIdx.x == 0) {
+    if (n_tiles == 0 && blockIdx.x == 0) {
+      ds->cm_n_done = 0;
+      if (a.n_done_out) *a.n_done_out = 0;
+    }
+    retire_cta(ds, TS_COMMIT);
+  }
+}
+
+void launch_commit(const LaunchCfg& L, const CommitArgs& a) {
+  const uint64_t warps = ceil_div(a.n_host, 32);
+  const int grid =
+      (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(warps, CM_THREADS / 32),
+                                                    (uint64_t)L.grid_commit));
+  RO_LAUNCH(L, K_COMMIT, (commit_scatter_kernel<<<grid, CM_THREADS, 0, L.stream>>>(a)));
+  RO_LAUNCH(L, K_CFINISH, (commit_finish_kernel<<<L.grid_cfinish, CF_THREADS, 0, L.stream>>>(a)));
+}
+
+const void* kernel_ptr_commit(int which) {
+  return which == K_COMMIT ? (const void*)commit_scatter_kernel : (const void*)commit_finish_kernel;
+}
+
+}  // namespace ro

@@ -1,0 +1,202 @@
+// k_ready.cu — ro_batch_ready kernels (Section 4.3, Eq. 2).
+//
+// Admission into a per-Call FIFO Ready Queue is an ordered stream compaction
+// of the candidate list; elastic reservation then takes whole batches from
+// the queue head.  Two passes:
+//   ready_count   decides admission.  A candidate list may name a child more
+//                 than once; the lowest position wins, through a CAS on the
+//                 child's WAITING phase word that keeps the smallest claim.
+//                 Counting the transitions out of "unclaimed" gives the exact
+//                 number admitted.  The last CTA turns that count into the
+//                 reservation (how many leave the queue), checks the output
+//                 capacity and advances the queue's head and tail.
+//   ready_scatter recomputes the admission flags, ranks them with a
+//                 single-pass scan (decoupled look-back) and writes every
+//                 admitted child either into the reserved batches (IN-FLIGHT)
+//                 or behind the queue's tail (READY).  Queued entries from
+//                 earlier calls leave first.
+// With the capacity check in the first pass, a call that cannot fit changes
+// nothing but the claims, which the second pass then releases.
+#include <algorithm>
+
+#include "ro_internal.h"
+
+namespace ro {
+
+__device__ __forceinline__ bool call_ok(const ReadyArgs& a, uint64_t c) {
+  return !a.check_call || w_call(a.rec[c].w) == a.call;
+}
+
+__global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
+  __shared__ unsigned long long s_red[2][RB_THREADS / 32];
+  DevScalars* ds = a.ds;
+  unsigned long long kept = 0, bad = 0;
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < a.n_cand; i += stride) {
+    const uint64_t c = a.cand ? (uint64_t)a.cand[i] : i;
+    if (c >= a.N) {
+      ++bad;
+      continue;
+    }
+    uint32_t w = a.phase[c];
+    if ((w & 3u) != PH_WAITING || !call_ok(a, c)) continue;
+    if (!a.cand) {
+      ++kept;   // ids are distinct: every WAITING child of this Call enters
+      continue;
+    }
+    const uint32_t mine = (uint32_t)i << 2;
+    for (;;) {
+      if ((w & 3u) != PH_WAITING || (w >> 2) <= (uint32_t)i) break;
+      const uint32_t old = atomicCAS(a.phase + c, w, mine);
+      if (old == w) {
+        if ((w >> 2) == CLAIM_NONE) ++kept;   // first claim of this child
+        break;
+      }
+      w = old;
+    }
+  }
+  // block reduction
+  for (int d = 16; d > 0; d >>= 1) {
+    kept += __shfl_down_sync(0xffffffffu, kept, d);
+    bad += __shfl_down_sync(0xffffffffu, bad, d);
+  }
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  if (lane == 0) {
+    s_red[0][wid] = kept;
+    s_red[1][wid] = bad;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long k = 0, b = 0;
+    for (int j = 0; j < RB_THREADS / 32; ++j) {
+      k += s_red[0][j];
+      b += s_red[1][j];
+    }
+    if (k) atomicAdd(&ds->rb_kept, k);
+    if (b) atomicAdd(&ds->rb_bad, b);
+    __threadfence();
+    if (atomicAdd(&ds->rb_ticket, 1u) == gridDim.x - 1) {
+      // last CTA: plan the reservation
+      __threadfence();
+      const unsigned long long K = ld_relaxed_u64(&ds->rb_kept);
+      const unsigned long long head = a.qstate[0], tail = a.qstate[1];
+      const unsigned long long L = tail - head, T = L + K;
+      const unsigned long long npop = a.flush ? T : (T / a.batch_size) * a.batch_size;
+      ds->rb_npop = npop;
+      ds->rb_n_batches = (npop + a.batch_size - 1) / a.batch_size;
+      if (a.n_batched_out) *a.n_batched_out = npop;
+      if (npop > a.cap) {
+        ds->rb_err = 1u;
+        atomicOr(&ds->err, ERR_CAPACITY);
+      } else {
+        ds->rb_err = 0u;
+        ds->rb_L = L;
+        ds->rb_k = K;
+        ds->rb_head = head;
+        ds->rb_tail = tail;
+        a.qstate[0] = head + npop;
+        a.qstate[1] = tail + K;
+        ds->stats[5] += ld_relaxed_u64(&ds->rb_bad);
+      }
+      ds->rb_kept = 0;
+      ds->rb_bad = 0;
+      ds->rb_ticket = 0u;
+      __threadfence();
+    }
+  }
+}
+
+__global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) {
+  __shared__ unsigned long long s_scan[33];
+  __shared__ uint32_t s_tile;
+  __shared__ unsigned long long s_prefix;
+  DevScalars* ds = a.ds;
+  const bool failed = ds->rb_err != 0u;
+  const unsigned long long L = ds->rb_L, npop = ds->rb_npop, head = ds->rb_head;
+
+  if (failed) {
+    // release the claims taken by the first pass; nothing else changes
+    if (a.cand) {
+      const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+      for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < a.n_cand; i += stride) {
+        const uint64_t c = a.cand[i];
+        if (c < a.N && a.phase[c] == ((uint32_t)i << 2)) a.phase[c] = WAIT_UNCLAIMED;
+      }
+    }
+    return;   // no tile counter was touched
+  }
+
+  // entries queued by earlier calls leave first
+  {
+    const unsigned long long n_old = L < npop ? L : npop;
+    const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+    for (uint64_t j = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n_old; j += stride) {
+      const uint32_t c = a.queue[head + j];
+      a.batched[j] = c;
+      a.phase[c] = (a.phase[c] & ~3u) | PH_INFLIGHT;
+    }
+  }
+
+  const uint64_t TILE = (uint64_t)RB_THREADS * RB_ITEMS;
+  const uint64_t n_tiles = ceil_div(a.n_cand, TILE);
+  for (;;) {
+    if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_READY]);
+    __syncthreads();
+    const uint32_t tile = s_tile;
+    __syncthreads();
+    if (tile >= n_tiles) break;
+    const uint64_t i0 = tile * TILE + (uint64_t)threadIdx.x * RB_ITEMS;
+    uint32_t cs[RB_ITEMS];
+    uint32_t flags = 0;
+    unsigned long long cnt = 0;
+#pragma unroll
+    for (int k = 0; k < RB_ITEMS; ++k) {
+      const uint64_t i = i0 + k;
+      cs[k] = 0;
+      if (i >= a.n_cand) continue;
+      const uint64_t c = a.cand ? (uint64_t)a.cand[i] : i;
+      if (c >= a.N) continue;
+      const uint32_t w = a.phase[c];
+      const bool keep = a.cand ? (w == ((uint32_t)i << 2)) : (w == WAIT_UNCLAIMED && call_ok(a, c));
+      if (keep) {
+        flags |= 1u << k;
+        cs[k] = (uint32_t)c;
+        ++cnt;
+      }
+    }
+    unsigned long long total;
+    unsigned long long excl = block_excl_scan(cnt, s_scan, &total);
+    if (threadIdx.x == 0) s_prefix = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_READY], &ds->err);
+    __syncthreads();
+    unsigned long long rank = s_prefix + excl;
+#pragma unroll
+    for (int k = 0; k < RB_ITEMS; ++k) {
+      if (!(flags & (1u << k))) continue;
+      const uint32_t c = cs[k];
+      const unsigned long long j = L + rank;   // position in the logical queue
+      if (j < npop) {
+        a.batched[j] = c;
+        a.phase[c] = ph_make(PH_INFLIGHT, 0u);
+      } else {
+        a.queue[head + j] = c;
+        a.phase[c] = ph_make(PH_READY, 0u);
+      }
+      ++rank;
+    }
+  }
+  if (threadIdx.x == 0) retire_cta(ds, TS_READY);
+}
+
+void launch_ready(const LaunchCfg& L, const ReadyArgs& a) {
+  const uint64_t per = (uint64_t)RB_THREADS;
+  const int grid_count =
+      (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(a.n_cand, per), (uint64_t)L.grid_rb));
+  RO_LAUNCH(L, K_RB_COUNT, (ready_count_kernel<<<grid_count, RB_THREADS, 0, L.stream>>>(a)));
+  RO_LAUNCH(L, K_RB_SCATTER, (ready_scatter_kernel<<<L.grid_rb, RB_THREADS, 0, L.stream>>>(a)));
+}
+
+const void* kernel_ptr_ready(int which) {
+  return which == K_RB_COUNT ? (const void*)ready_count_kernel : (const void*)ready_scatter_kernel;
+}
+
+}  // namespace ro

@@ -1,0 +1,624 @@
+// ro_api.cu — host side of the C ABI declared in include/rayorch_gpu.h:
+// argument checks, ownership of the per-expansion device state, scratch,
+// kernel launches and the mapping of device-recorded conditions to statuses.
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/rayorch_gpu.h"
+#include "ro_internal.h"
+
+namespace ro {
+const void* kernel_ptr_expand(int which);
+const void* kernel_ptr_ready(int which);
+const void* kernel_ptr_commit(int which);
+const void* kernel_ptr_assemble(int which);
+}  // namespace ro
+
+using namespace ro;
+
+namespace {
+
+constexpr int MAX_EXPANSIONS = 64;
+constexpr int N_TS = 6;   // tile-status slots (TS_* in ro_common.cuh)
+
+struct DevBuf {
+  void* p = nullptr;
+  size_t cap = 0;
+};
+
+struct QueueBufs {
+  DevBuf q, state;
+  bool ready = false;   // state zeroed for the current expansion
+};
+
+// Device buffers of one expansion slot, kept across ro_ctx_reset and reused.
+struct ExpSlot {
+  DevBuf offsets, pw, phase, rec, bitmap, done, tfp;
+  std::vector<QueueBufs> queues;
+};
+
+struct Expansion {
+  int32_t parent_xid = -1;
+  uint64_t P = 0, N = 0;
+  bool committed = false;   // a commit produced a completed-parent list
+};
+
+struct TsBuf {
+  DevBuf flag, agg, inc;
+};
+
+}  // namespace
+
+namespace ro {
+// Launch counts always; CUDA-event pairs around the kernels selected by mask.
+struct Profiler {
+  uint32_t mask = 0;
+  std::vector<cudaEvent_t> pool;
+  size_t used = 0;
+  std::vector<std::pair<int, size_t>> marks;   // (kernel, index of its start event)
+  uint64_t launches[K_COUNT] = {};
+  uint64_t timed[K_COUNT] = {};
+  double ms[K_COUNT] = {};
+  int pending = -1;
+};
+
+void prof_begin(Profiler* p, cudaStream_t s, int kid) {
+  if (!p) return;
+  p->launches[kid] += 1;
+  p->pending = -1;
+  if (!(p->mask & (1u << kid))) return;
+  if (p->used + 2 > p->pool.size()) {
+    const size_t add = std::max<size_t>(p->pool.size(), 256);
+    for (size_t i = 0; i < add; ++i) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) {
+        cudaGetLastError();
+        return;
+      }
+      p->pool.push_back(e);
+    }
+  }
+  cudaEventRecord(p->pool[p->used], s);
+  p->pending = (int)p->used;
+  p->used += 2;
+}
+
+void prof_end(Profiler* p, cudaStream_t s, int kid) {
+  if (!p || p->pending < 0) return;
+  cudaEventRecord(p->pool[p->pending + 1], s);
+  p->marks.emplace_back(kid, (size_t)p->pending);
+  p->pending = -1;
+}
+}  // namespace ro
+
+struct ro_ctx {
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  uint32_t n_calls = 1;
+  int num_sms = 0;
+  LaunchCfg L{};
+  DevScalars* ds = nullptr;
+  DevScalars* hs = nullptr;   // pinned mirror
+  std::vector<ExpSlot> slots;
+  std::vector<Expansion> exps;
+  TsBuf ts[N_TS];
+  DevBuf code, mb, mtfp, cpos, csrc, ctfp;
+  Profiler prof;
+  ro_status sticky = RO_OK;
+  std::string err;
+};
+
+namespace {
+
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    int cur = -1;
+    if (cudaGetDevice(&cur) == cudaSuccess && cur != dev) {
+      prev = cur;
+      cudaSetDevice(dev);
+    }
+  }
+  ~DeviceGuard() {
+    if (prev >= 0) cudaSetDevice(prev);
+  }
+};
+
+ro_status fail(ro_ctx* c, ro_status st, const char* fmt, ...) __attribute__((format(printf, 3, 4)));
+ro_status fail(ro_ctx* c, ro_status st, const char* fmt, ...) {
+  if (c) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    c->err = buf;
+  }
+  return st;
+}
+
+ro_status cuda_fail(ro_ctx* c, cudaError_t e, const char* what) {
+  c->sticky = RO_E_CUDA;
+  return fail(c, RO_E_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Grow-only device buffer.  New memory is zeroed on the context's stream.
+ro_status ensure(ro_ctx* c, DevBuf& b, size_t bytes, const char* what) {
+  if (bytes == 0) bytes = 16;
+  if (b.cap >= bytes) return RO_OK;
+  if (b.p) {
+    cudaStreamSynchronize(c->stream);
+    cudaFree(b.p);
+    b.p = nullptr;
+    b.cap = 0;
+  }
+  size_t want = bytes + bytes / 8;   // a little headroom for the next, larger call
+  want = (want + 255) & ~(size_t)255;
+  cudaError_t e = cudaMalloc(&b.p, want);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(c, RO_E_OOM, "cannot allocate %zu bytes for %s", want, what);
+  }
+  b.cap = want;
+  e = cudaMemsetAsync(b.p, 0, want, c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "cudaMemsetAsync");
+  return RO_OK;
+}
+
+#define RO_TRY(x)                 \
+  do {                            \
+    ro_status _s = (x);           \
+    if (_s != RO_OK) return _s;   \
+  } while (0)
+
+// Tile-status arrays of one scan slot (flags start zeroed: epoch 0, nothing
+// published; kernels keep their epochs on the device).
+template <class T>
+ro_status tile_status(ro_ctx* c, int slot, size_t tiles, TileStatus<T>* out) {
+  TsBuf& t = c->ts[slot];
+  tiles = std::max<size_t>(tiles, 1);
+  RO_TRY(ensure(c, t.flag, tiles * sizeof(unsigned long long), "scan flags"));
+  RO_TRY(ensure(c, t.agg, tiles * sizeof(Pair64), "scan aggregates"));
+  RO_TRY(ensure(c, t.inc, tiles * sizeof(Pair64), "scan prefixes"));
+  out->flag = (unsigned long long*)t.flag.p;
+  out->agg = (T*)t.agg.p;
+  out->inc = (T*)t.inc.p;
+  return RO_OK;
+}
+
+ro_status check_launch(ro_ctx* c, const char* what) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(c, e, what);
+  return RO_OK;
+}
+
+// Wait for the stream, mirror the device scalars and turn recorded
+// conditions into a status (clearing them).
+ro_status sync_and_check(ro_ctx* c) {
+  cudaError_t e = cudaMemcpyAsync(c->hs, c->ds, sizeof(DevScalars), cudaMemcpyDeviceToHost, c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "synchronise");
+  const uint32_t err = c->hs->err;
+  if (!err) return RO_OK;
+  cudaMemsetAsync(&c->ds->err, 0, sizeof(uint32_t), c->stream);
+  if (err & ERR_TIMEOUT) return fail(c, RO_E_TIMEOUT, "a device-side wait timed out");
+  if (err & ERR_OVERFLOW) return fail(c, RO_E_OVERFLOW, "an assembled parent exceeds 2^32-1 bytes");
+  if (err & ERR_CAPACITY) return fail(c, RO_E_CAPACITY, "an output buffer is too small");
+  return fail(c, RO_E_INVAL, "a device count exceeded its host bound");
+}
+
+ro_status enter(ro_ctx* c) {
+  if (!c) return RO_E_INVAL;
+  if (c->sticky != RO_OK) return c->sticky;
+  c->err.clear();
+  return RO_OK;
+}
+
+Expansion* get_exp(ro_ctx* c, int32_t xid) {
+  if (xid < 0 || xid >= (int32_t)c->exps.size()) return nullptr;
+  return &c->exps[xid];
+}
+
+int grid_for(const void* k, int threads, int sms, int cap_per_sm) {
+  int per = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k, threads, 0) != cudaSuccess || per < 1)
+    per = 1;
+  per = std::min(per, cap_per_sm);
+  return per * sms;
+}
+
+}  // namespace
+
+extern "C" {
+
+ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_calls) {
+  if (!out) return RO_E_INVAL;
+  *out = nullptr;
+  if (n_calls == 0 || n_calls > 256) return RO_E_INVAL;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
+    cudaGetLastError();
+    return RO_E_CUDA;
+  }
+  DeviceGuard g(device);
+  ro_ctx* c = new ro_ctx();
+  c->device = device;
+  c->stream = (cudaStream_t)stream;
+  c->n_calls = n_calls;
+  cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
+  if (cudaMalloc(&c->ds, sizeof(DevScalars)) != cudaSuccess ||
+      cudaMallocHost(&c->hs, sizeof(DevScalars)) != cudaSuccess) {
+    cudaGetLastError();
+    if (c->ds) cudaFree(c->ds);
+    delete c;
+    return RO_E_OOM;
+  }
+  cudaMemsetAsync(c->ds, 0, sizeof(DevScalars), c->stream);
+  std::memset(c->hs, 0, sizeof(DevScalars));
+  const int s = c->num_sms;
+  c->L.stream = c->stream;
+  c->L.prof = &c->prof;
+  c->L.grid_expand_scan = grid_for(kernel_ptr_expand(K_EXPAND_SCAN), EXP_THREADS, s, 4);
+  c->L.grid_fill = grid_for(kernel_ptr_expand(K_FILL), FILL_THREADS, s, 8);
+  c->L.grid_rb = grid_for(kernel_ptr_ready(K_RB_SCATTER), RB_THREADS, s, 8);
+  c->L.grid_commit = grid_for(kernel_ptr_commit(K_COMMIT), CM_THREADS, s, 8);
+  c->L.grid_cfinish = grid_for(kernel_ptr_commit(K_CFINISH), CF_THREADS, s, 4);
+  c->L.grid_aparents = grid_for(kernel_ptr_assemble(K_APARENTS), AP_THREADS, s, 4);
+  c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 8);
+  c->L.grid_acopy = grid_for(kernel_ptr_assemble(K_ACOPY), AC_THREADS, s, 8);
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) {
+    cudaFree(c->ds);
+    cudaFreeHost(c->hs);
+    delete c;
+    return RO_E_CUDA;
+  }
+  *out = c;
+  return RO_OK;
+}
+
+ro_status ro_ctx_destroy(ro_ctx* c) {
+  if (!c) return RO_E_INVAL;
+  DeviceGuard g(c->device);
+  cudaStreamSynchronize(c->stream);
+  auto fr = [](DevBuf& b) {
+    if (b.p) cudaFree(b.p);
+    b.p = nullptr;
+    b.cap = 0;
+  };
+  for (auto& s : c->slots) {
+    fr(s.offsets); fr(s.pw); fr(s.phase); fr(s.rec); fr(s.bitmap); fr(s.done); fr(s.tfp);
+    for (auto& q : s.queues) {
+      fr(q.q);
+      fr(q.state);
+    }
+  }
+  for (auto& t : c->ts) {
+    fr(t.flag); fr(t.agg); fr(t.inc);
+  }
+  fr(c->code); fr(c->mb); fr(c->mtfp); fr(c->cpos); fr(c->csrc); fr(c->ctfp);
+  for (cudaEvent_t e : c->prof.pool) cudaEventDestroy(e);
+  cudaFree(c->ds);
+  cudaFreeHost(c->hs);
+  delete c;
+  return RO_OK;
+}
+
+ro_status ro_ctx_reset(ro_ctx* c) {
+  if (!c) return RO_E_INVAL;
+  c->exps.clear();
+  c->err.clear();
+  return RO_OK;
+}
+
+ro_status ro_ctx_sync(ro_ctx* c) {
+  RO_TRY(enter(c));
+  DeviceGuard g(c->device);
+  return sync_and_check(c);
+}
+
+ro_status ro_ctx_stats(ro_ctx* c, ro_stats* out) {
+  RO_TRY(enter(c));
+  if (!out) return fail(c, RO_E_INVAL, "stats output is NULL");
+  DeviceGuard g(c->device);
+  ro_status st = sync_and_check(c);
+  uint64_t* o = &out->accepted;
+  for (int k = 0; k < 7; ++k) o[k] = c->hs->stats[k];
+  return st;
+}
+
+const char* ro_last_error(const ro_ctx* c) { return c ? c->err.c_str() : "no context"; }
+
+ro_status ro_ctx_profile(ro_ctx* c, uint32_t kernel_mask) {
+  RO_TRY(enter(c));
+  c->prof.mask = kernel_mask & ((1u << K_COUNT) - 1u);
+  return RO_OK;
+}
+
+ro_status ro_ctx_profile_read(ro_ctx* c, uint64_t* launches, uint64_t* timed, double* ms,
+                              uint32_t n_kernels) {
+  RO_TRY(enter(c));
+  DeviceGuard g(c->device);
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "synchronise");
+  Profiler& p = c->prof;
+  for (const auto& m : p.marks) {
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, p.pool[m.second], p.pool[m.second + 1]) == cudaSuccess) {
+      p.ms[m.first] += t;
+      p.timed[m.first] += 1;
+    } else {
+      cudaGetLastError();
+    }
+  }
+  p.marks.clear();
+  p.used = 0;
+  const uint32_t k = std::min<uint32_t>(n_kernels, K_COUNT);
+  for (uint32_t i = 0; i < k; ++i) {
+    if (launches) launches[i] = p.launches[i];
+    if (timed) timed[i] = p.timed[i];
+    if (ms) ms[i] = p.ms[i];
+    p.launches[i] = 0;
+    p.timed[i] = 0;
+    p.ms[i] = 0.0;
+  }
+  return RO_OK;
+}
+
+// ---------------------------------------------------------------------------
+ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uint64_t n_parents,
+                    const uint8_t* d_parent_call, uint64_t* d_offsets, uint32_t* d_child_parent,
+                    uint32_t* d_child_ordinal, uint64_t child_cap, uint32_t* d_empty_parents,
+                    uint64_t* h_n_children, uint64_t* h_n_empty, int32_t* xid) {
+  RO_TRY(enter(c));
+  if (!xid || !h_n_children || !d_offsets || (n_parents && !d_counts))
+    return fail(c, RO_E_INVAL, "ro_expand: NULL argument");
+  if (n_parents >= (1ull << 32)) return fail(c, RO_E_OVERFLOW, "ro_expand: 2^32 parents or more");
+  if ((int)c->exps.size() >= MAX_EXPANSIONS)
+    return fail(c, RO_E_STATE, "ro_expand: more than %d expansions in one context", MAX_EXPANSIONS);
+  if (parent_xid != -1) {
+    Expansion* px = get_exp(c, parent_xid);
+    if (!px) return fail(c, RO_E_STATE, "ro_expand: unknown parent expansion %d", parent_xid);
+    if (px->N != n_parents)
+      return fail(c, RO_E_INVAL, "ro_expand: %llu parents but parent expansion has %llu children",
+                  (unsigned long long)n_parents, (unsigned long long)px->N);
+  }
+  DeviceGuard g(c->device);
+  const size_t slot = c->exps.size();
+  if (c->slots.size() <= slot) c->slots.resize(slot + 1);
+  ExpSlot& S = c->slots[slot];
+  const uint64_t P = n_parents;
+  const uint64_t cap_children = std::min<uint64_t>(child_cap, (1ull << 32));
+  const uint64_t tfp_entries = ceil_div(cap_children, FILL_TILE) + 1;
+  RO_TRY(ensure(c, S.offsets, (P + 1) * sizeof(uint64_t), "offsets"));
+  RO_TRY(ensure(c, S.pw, P * sizeof(uint64_t), "parent counters"));
+  RO_TRY(ensure(c, S.tfp, tfp_entries * sizeof(uint32_t), "fill tiles"));
+  ExpandScanArgs sa{};
+  sa.counts = d_counts;
+  sa.P = P;
+  sa.offsets_user = d_offsets;
+  sa.offsets = (uint64_t*)S.offsets.p;
+  sa.pw = (unsigned long long*)S.pw.p;
+  sa.empty_out = d_empty_parents;
+  sa.tfp = (uint32_t*)S.tfp.p;
+  sa.tfp_cap = tfp_entries;
+  sa.ds = c->ds;
+  RO_TRY(tile_status(c, TS_EXPAND, ceil_div(P, (uint64_t)EXP_THREADS * EXP_ITEMS), &sa.ts));
+  launch_expand_scan(c->L, sa);
+  RO_TRY(check_launch(c, "expand_scan"));
+  RO_TRY(sync_and_check(c));
+  const uint64_t N = c->hs->n_children;
+  *h_n_children = N;
+  if (h_n_empty) *h_n_empty = c->hs->n_empty;
+  if (N >= (1ull << 32)) return fail(c, RO_E_OVERFLOW, "ro_expand: 2^32 children or more");
+  if (N > child_cap)
+    return fail(c, RO_E_CAPACITY, "ro_expand: %llu children exceed child_cap %llu",
+                (unsigned long long)N, (unsigned long long)child_cap);
+  if (N && (!d_child_parent || !d_child_ordinal))
+    return fail(c, RO_E_INVAL, "ro_expand: NULL child arrays");
+
+  RO_TRY(ensure(c, S.phase, N * sizeof(uint32_t), "phase words"));
+  RO_TRY(ensure(c, S.rec, N * sizeof(Rec), "result records"));
+  RO_TRY(ensure(c, S.bitmap, ceil_div(P, 32) * sizeof(uint32_t), "completion bitmap"));
+  RO_TRY(ensure(c, S.done, P * sizeof(uint32_t), "completed parents"));
+  cudaMemsetAsync(S.bitmap.p, 0, ceil_div(P, 32) * sizeof(uint32_t), c->stream);
+  ExpandFillArgs fa{};
+  fa.offsets = (const uint64_t*)S.offsets.p;
+  fa.P = P;
+  fa.N = N;
+  fa.tfp = (const uint32_t*)S.tfp.p;
+  fa.parent_call = d_parent_call;
+  fa.child_parent = d_child_parent;
+  fa.child_ordinal = d_child_ordinal;
+  fa.phase = (uint32_t*)S.phase.p;
+  fa.rec = (Rec*)S.rec.p;
+  launch_expand_fill(c->L, fa);
+  RO_TRY(check_launch(c, "expand_fill"));
+  if (S.queues.size() < c->n_calls) S.queues.resize(c->n_calls);
+  for (auto& q : S.queues) q.ready = false;
+
+  Expansion x;
+  x.parent_xid = parent_xid;
+  x.P = P;
+  x.N = N;
+  c->exps.push_back(x);
+  *xid = (int32_t)slot;
+  return RO_OK;
+}
+
+// ---------------------------------------------------------------------------
+ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* d_cand,
+                         uint64_t n_cand, uint32_t batch_size, int32_t flush, uint32_t* d_batched,
+                         uint64_t batched_cap, uint64_t* d_n_batched, uint64_t* h_n_batched,
+                         uint64_t* h_n_batches) {
+  RO_TRY(enter(c));
+  Expansion* x = get_exp(c, xid);
+  if (!x) return fail(c, RO_E_STATE, "ro_batch_ready: unknown expansion %d", xid);
+  if (call >= c->n_calls) return fail(c, RO_E_INVAL, "ro_batch_ready: call %u out of range", call);
+  if (batch_size == 0) return fail(c, RO_E_INVAL, "ro_batch_ready: batch_size is 0");
+  if (batched_cap && !d_batched) return fail(c, RO_E_INVAL, "ro_batch_ready: NULL d_batched");
+  if (d_cand && n_cand > MAX_CAND)
+    return fail(c, RO_E_INVAL, "ro_batch_ready: more than 2^30-2 candidates in one call");
+  DeviceGuard g(c->device);
+  ExpSlot& S = c->slots[xid];
+  QueueBufs& Q = S.queues[call];
+  if (!Q.ready) {
+    RO_TRY(ensure(c, Q.q, x->N * sizeof(uint32_t), "ready queue"));
+    RO_TRY(ensure(c, Q.state, 2 * sizeof(unsigned long long), "queue state"));
+    cudaMemsetAsync(Q.state.p, 0, 2 * sizeof(unsigned long long), c->stream);
+    Q.ready = true;
+  }
+  ReadyArgs ra{};
+  ra.cand = d_cand;
+  ra.n_cand = d_cand ? n_cand : x->N;
+  ra.N = x->N;
+  ra.phase = (uint32_t*)S.phase.p;
+  ra.rec = (const Rec*)S.rec.p;
+  ra.check_call = c->n_calls > 1;
+  ra.call = call;
+  ra.batch_size = batch_size;
+  ra.flush = flush != 0;
+  ra.cap = batched_cap;
+  ra.queue = (uint32_t*)Q.q.p;
+  ra.qstate = (unsigned long long*)Q.state.p;
+  ra.batched = d_batched;
+  ra.n_batched_out = d_n_batched;
+  ra.ds = c->ds;
+  RO_TRY(tile_status(c, TS_READY, ceil_div(ra.n_cand, (uint64_t)RB_THREADS * RB_ITEMS), &ra.ts));
+  launch_ready(c->L, ra);
+  RO_TRY(check_launch(c, "batch_ready"));
+  if (h_n_batched || h_n_batches) {
+    ro_status st = sync_and_check(c);
+    if (h_n_batched) *h_n_batched = c->hs->rb_npop;
+    if (h_n_batches) *h_n_batches = c->hs->rb_n_batches;
+    return st;
+  }
+  return RO_OK;
+}
+
+// ---------------------------------------------------------------------------
+ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d_n,
+                           const uint32_t* d_child, const uint8_t* d_state, const uint32_t* d_len,
+                           const uint64_t* d_arena_off, const uint32_t* d_gen, uint64_t arena_bytes,
+                           uint8_t* d_code, uint32_t* d_done_parents, uint64_t done_cap,
+                           uint64_t* d_n_done, uint64_t* h_n_done) {
+  RO_TRY(enter(c));
+  Expansion* x = get_exp(c, xid);
+  if (!x) return fail(c, RO_E_STATE, "ro_gather_commit: unknown expansion %d", xid);
+  if (n >= (1ull << 32)) return fail(c, RO_E_OVERFLOW, "ro_gather_commit: 2^32 reports or more");
+  if (n && (!d_child || !d_state || !d_len || !d_arena_off))
+    return fail(c, RO_E_INVAL, "ro_gather_commit: NULL report array");
+  if (arena_bytes >= MAX_ARENA) return fail(c, RO_E_OVERFLOW, "ro_gather_commit: arena of 2^48 bytes or more");
+  if (d_done_parents && done_cap < std::min<uint64_t>(n, x->P))
+    return fail(c, RO_E_INVAL, "ro_gather_commit: done_cap below min(n, parents)");
+  DeviceGuard g(c->device);
+  ExpSlot& S = c->slots[xid];
+  CommitArgs ca{};
+  ca.n_host = n;
+  ca.d_n = d_n;
+  ca.child = d_child;
+  ca.state = d_state;
+  ca.len = d_len;
+  ca.off = d_arena_off;
+  ca.gen = d_gen;
+  ca.arena_bytes = arena_bytes;
+  ca.N = x->N;
+  ca.P = x->P;
+  ca.phase = (uint32_t*)S.phase.p;
+  ca.rec = (Rec*)S.rec.p;
+  ca.pw = (unsigned long long*)S.pw.p;
+  ca.bitmap = (uint32_t*)S.bitmap.p;
+  if (d_code) {
+    ca.code = d_code;
+  } else {
+    RO_TRY(ensure(c, c->code, n, "report verdicts"));
+    ca.code = (uint8_t*)c->code.p;
+  }
+  ca.done_user = d_done_parents;
+  ca.done_int = (uint32_t*)S.done.p;
+  ca.n_done_out = d_n_done;
+  ca.ds = c->ds;
+  RO_TRY(tile_status(c, TS_COMMIT, ceil_div(ceil_div(x->P, 32), (uint64_t)CF_THREADS * CF_WORDS),
+                     &ca.ts));
+  launch_commit(c->L, ca);
+  RO_TRY(check_launch(c, "gather_commit"));
+  x->committed = true;
+  if (h_n_done) {
+    ro_status st = sync_and_check(c);
+    *h_n_done = c->hs->cm_n_done;
+    return st;
+  }
+  return RO_OK;
+}
+
+// ---------------------------------------------------------------------------
+ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t arena_bytes,
+                      const uint32_t* d_parents, uint64_t n_parents, const uint64_t* d_n_parents,
+                      uint8_t* d_status, uint64_t* d_out_off, uint32_t* d_out_len, uint8_t* d_out,
+                      uint64_t out_cap, uint64_t* d_out_cursor, uint64_t* d_out_bytes,
+                      uint64_t* h_out_bytes) {
+  RO_TRY(enter(c));
+  Expansion* x = get_exp(c, xid);
+  if (!x) return fail(c, RO_E_STATE, "ro_assemble: unknown expansion %d", xid);
+  if (!d_arena || !d_status || !d_out_off)
+    return fail(c, RO_E_INVAL, "ro_assemble: NULL arena, status or offsets");
+  if (out_cap && !d_out) return fail(c, RO_E_INVAL, "ro_assemble: NULL output");
+  if (!d_parents && !x->committed)
+    return fail(c, RO_E_STATE, "ro_assemble: no commit on expansion %d to take parents from", xid);
+  if (n_parents >= (1ull << 32)) return fail(c, RO_E_OVERFLOW, "ro_assemble: list of 2^32 or more");
+  DeviceGuard g(c->device);
+  ExpSlot& S = c->slots[xid];
+  const uint64_t member_cap = std::max<uint64_t>(x->N, 1);
+  const uint64_t mtfp_cap = ceil_div(member_cap, AM_TILE) + 2;
+  const uint64_t ctfp_cap = ceil_div(out_cap + 32, AC_CHUNK) + 2;
+  RO_TRY(ensure(c, c->mb, (n_parents + 1) * sizeof(uint32_t), "member bases"));
+  RO_TRY(ensure(c, c->mtfp, mtfp_cap * sizeof(uint32_t), "member tiles"));
+  RO_TRY(ensure(c, c->cpos, member_cap * sizeof(uint64_t), "member positions"));
+  RO_TRY(ensure(c, c->csrc, member_cap * sizeof(uint64_t), "member sources"));
+  RO_TRY(ensure(c, c->ctfp, ctfp_cap * sizeof(uint32_t), "copy chunks"));
+  AssembleArgs aa{};
+  aa.list = d_parents ? d_parents : (const uint32_t*)S.done.p;
+  aa.n_host = n_parents;
+  aa.d_n = d_parents ? d_n_parents : nullptr;
+  aa.list_is_commit = d_parents ? 0 : 1;
+  aa.P = x->P;
+  aa.N = x->N;
+  aa.offsets = (const uint64_t*)S.offsets.p;
+  aa.pw = (const unsigned long long*)S.pw.p;
+  aa.rec = (const Rec*)S.rec.p;
+  aa.arena = d_arena;
+  aa.arena_bytes = arena_bytes;
+  aa.status = d_status;
+  aa.out_off = d_out_off;
+  aa.out_len = d_out_len;
+  aa.out = d_out;
+  aa.out_cap = out_cap;
+  aa.cursor = d_out_cursor;
+  aa.out_bytes = d_out_bytes;
+  aa.mb = (uint32_t*)c->mb.p;
+  aa.mtfp = (uint32_t*)c->mtfp.p;
+  aa.mtfp_cap = mtfp_cap;
+  aa.cpos = (uint64_t*)c->cpos.p;
+  aa.csrc = (uint64_t*)c->csrc.p;
+  aa.member_cap = member_cap;
+  aa.ctfp = (uint32_t*)c->ctfp.p;
+  aa.ctfp_cap = ctfp_cap;
+  aa.ds = c->ds;
+  RO_TRY(tile_status(c, TS_ASM_PARENTS, ceil_div(n_parents, (uint64_t)AP_THREADS * AP_ITEMS),
+                     &aa.ts_parents));
+  RO_TRY(tile_status(c, TS_ASM_MEMBERS, ceil_div(member_cap, (uint64_t)AM_TILE), &aa.ts_members));
+  launch_assemble(c->L, aa);
+  RO_TRY(check_launch(c, "assemble"));
+  if (h_out_bytes) {
+    ro_status st = sync_and_check(c);
+    *h_out_bytes = c->hs->as_bytes;
+    return st;
+  }
+  return RO_OK;
+}
+
+}  // extern "C"

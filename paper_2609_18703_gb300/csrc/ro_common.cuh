@@ -1,0 +1,288 @@
+// ro_common.cuh — layouts and device helpers shared by the lineage kernels.
+//
+// Per-child state of an expansion lives in two arrays:
+//   phase[c]  uint32 Grain phase word (Eq. 2): bits 0-1 phase; for WAITING the
+//             upper 30 bits hold the admission claim of the current
+//             ro_batch_ready call (all ones = unclaimed), otherwise the
+//             attempt generation (Eq. 3).
+//   rec[c]    16-byte record: immediate parent, payload length and one word
+//             packing the arena offset (48 bits), the published outcome
+//             (3 bits), two commit bookkeeping flags and the Call (8 bits).
+// Per-parent state: pw[p] = remaining unsealed members (low 32 bits) plus the
+// number of Failed/Suppressed members (high 32 bits), so one 64-bit atomic add
+// both counts a member down and records its outcome class.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace ro {
+
+// ---- Grain phases (Eq. 2) -------------------------------------------------
+constexpr uint32_t PH_WAITING = 0u, PH_READY = 1u, PH_INFLIGHT = 2u, PH_SEALED = 3u;
+constexpr uint32_t CLAIM_NONE = 0x3FFFFFFFu;              // unclaimed WAITING
+constexpr uint32_t WAIT_UNCLAIMED = (CLAIM_NONE << 2) | PH_WAITING;
+constexpr uint64_t MAX_CAND = (uint64_t)CLAIM_NONE - 1;   // candidates per call
+
+__host__ __device__ constexpr uint32_t ph_make(uint32_t phase, uint32_t gen) {
+  return (gen << 2) | phase;
+}
+
+// ---- Item outcomes (Eq. 1) and report verdicts (Eq. 3) --------------------
+constexpr uint8_t ST_PENDING = 0, ST_PRESENT = 1, ST_DROPPED = 2, ST_FAILED = 3,
+                  ST_SUPPRESSED = 4;
+constexpr uint8_t V_ACCEPT = 0, V_INVALID = 1, V_NOT_INFLIGHT = 2, V_STALE = 3,
+                  V_DUPLICATE = 4;
+// internal verdict: the Grain was SEALED at the same generation; resolved to
+// ACCEPT or DUPLICATE by the commit's ordering pass
+constexpr uint8_t V_DUP_CANDIDATE = 5;
+
+// ---- result record ----------------------------------------------------------
+struct __align__(16) Rec {
+  uint32_t parent;
+  uint32_t len;
+  uint64_t w;   // off (0-47) | state (48-50) | sealer-seen (54) | conflict (55) | call (56-63)
+};
+constexpr uint64_t W_OFF_MASK = (1ull << 48) - 1;
+constexpr int W_STATE_SHIFT = 48;
+constexpr uint64_t W_STATE_MASK = 7ull << W_STATE_SHIFT;
+constexpr uint64_t W_SEALER_BIT = 1ull << 54;
+constexpr uint64_t W_CONFLICT_BIT = 1ull << 55;
+constexpr int W_CALL_SHIFT = 56;
+constexpr uint64_t MAX_ARENA = 1ull << 48;
+
+__device__ __forceinline__ uint8_t w_state(uint64_t w) {
+  return (uint8_t)((w >> W_STATE_SHIFT) & 7u);
+}
+__device__ __forceinline__ uint64_t w_off(uint64_t w) { return w & W_OFF_MASK; }
+__device__ __forceinline__ uint32_t w_call(uint64_t w) { return (uint32_t)(w >> W_CALL_SHIFT); }
+
+// ---- per-parent word ----------------------------------------------------------
+__device__ __forceinline__ uint32_t pw_remaining(uint64_t v) { return (uint32_t)v; }
+__device__ __forceinline__ uint32_t pw_bad(uint64_t v) { return (uint32_t)(v >> 32); }
+
+// ---- errors recorded by kernels (sticky in DevScalars::err) --------------------
+enum : uint32_t {
+  ERR_CAPACITY = 1u,
+  ERR_TIMEOUT = 2u,
+  ERR_OVERFLOW = 4u,
+  ERR_INVAL = 8u,
+};
+
+// Counters and small results that kernels hand to later kernels and to the
+// host.  One instance per context, in device memory, mirrored to pinned host
+// memory when a call synchronises.
+struct DevScalars {
+  uint32_t err;
+  uint32_t pad0;
+  unsigned long long stats[7];   // same order as ro_stats
+  // ro_expand
+  unsigned long long n_children, n_empty, last_nonempty_parent;
+  // ro_batch_ready
+  unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
+  uint32_t rb_ticket, rb_err;
+  // ro_gather_commit
+  unsigned long long cm_n, cm_conflicts, cm_n_done;
+  // ro_assemble
+  unsigned long long as_n, as_M, as_Mnz, as_bytes, as_base, as_origin;
+  uint32_t as_err, pad1;
+  // dynamic tile counters / exit tickets / scan epochs, one per look-back kernel
+  uint32_t tile_ctr[8];
+  uint32_t exit_ctr[8];
+  unsigned long long epoch[8];
+};
+enum TileSlot { TS_EXPAND = 0, TS_READY = 1, TS_COMMIT = 2, TS_ASM_PARENTS = 3, TS_ASM_MEMBERS = 4 };
+
+// ---- memory-order helpers --------------------------------------------------------
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// ---- values carried by decoupled look-back scans ------------------------------------
+struct Pair64 {
+  unsigned long long a, b;
+  __device__ __forceinline__ Pair64 operator+(const Pair64& o) const { return {a + o.a, b + o.b}; }
+};
+
+__device__ __forceinline__ unsigned long long load_cg(const unsigned long long* p) {
+  return __ldcg(p);
+}
+__device__ __forceinline__ Pair64 load_cg(const Pair64* p) {
+  return Pair64{__ldcg(&p->a), __ldcg(&p->b)};
+}
+
+// Spin limit of every device-side wait: ~2^22 polls with a short sleep each
+// (well under a second).  A wait that runs out records ERR_TIMEOUT and the
+// kernel carries on with what it has, so the context stays usable.
+constexpr uint32_t SPIN_LIMIT = 1u << 22;
+
+// Tile status for a single-pass scan: flag[t] = (epoch << 2) | kind with
+// kind 1 = aggregate of tile t published, 2 = inclusive prefix published.
+// The epoch is read from device memory at kernel start and advanced by the
+// kernel's last CTA, so flags of earlier launches (or of earlier replays of
+// a captured CUDA graph) never look current; nothing needs clearing.
+template <class T>
+struct TileStatus {
+  unsigned long long* flag;
+  T* agg;
+  T* inc;
+};
+
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_u64(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+template <class T>
+__device__ __forceinline__ void ts_publish(const TileStatus<T>& ts, uint32_t tile, const T& v,
+                                           unsigned long long kind, unsigned long long epoch) {
+  if (kind == 1ull)
+    ts.agg[tile] = v;
+  else
+    ts.inc[tile] = v;
+  __threadfence();
+  st_release_u64(ts.flag + tile, (epoch << 2) | kind);
+}
+
+// Exclusive prefix of tile `tile` given its local aggregate (decoupled
+// look-back, one thread).  Tiles are claimed in increasing order by running
+// CTAs, so every predecessor is resident or done and each wait ends; the
+// waits are bounded anyway (SPIN_LIMIT) and record ERR_TIMEOUT.
+template <class T>
+__device__ T lookback_exclusive(const TileStatus<T>& ts, uint32_t tile, const T& local,
+                                unsigned long long epoch, uint32_t* err) {
+  if (tile == 0) {
+    ts_publish(ts, 0, local, 2ull, epoch);
+    return T{};
+  }
+  ts_publish(ts, tile, local, 1ull, epoch);
+  T excl{};
+  int64_t j = (int64_t)tile - 1;
+  while (j >= 0) {
+    unsigned long long f = 0;
+    uint32_t spins = 0;
+    for (;;) {
+      f = ld_acquire_u64(ts.flag + j);
+      if ((f >> 2) == epoch && (f & 3ull) != 0ull) break;
+      if (++spins > SPIN_LIMIT) break;
+      // once any wait of this context has given up, stop waiting at once
+      if ((spins & 1023u) == 0u && (ld_acquire(err) & ERR_TIMEOUT)) spins = SPIN_LIMIT + 1;
+      if (spins > SPIN_LIMIT) break;
+      __nanosleep(64);
+    }
+    if (spins > SPIN_LIMIT) {
+      atomicOr(err, ERR_TIMEOUT);
+      break;
+    }
+    if ((f & 3ull) == 2ull) {
+      excl = load_cg(ts.inc + j) + excl;
+      break;
+    }
+    excl = load_cg(ts.agg + j) + excl;
+    --j;
+  }
+  ts_publish(ts, tile, excl + local, 2ull, epoch);
+  return excl;
+}
+
+// Claim the next tile of a dynamically scheduled (persistent) kernel.
+__device__ __forceinline__ uint32_t claim_tile(uint32_t* ctr) { return atomicAdd(ctr, 1u); }
+
+// Called by thread 0 of every CTA on exit; the last CTA out resets the tile
+// counter and advances the epoch for the next launch of this kernel.
+__device__ __forceinline__ void retire_cta(DevScalars* ds, int slot) {
+  __threadfence();
+  if (atomicAdd(&ds->exit_ctr[slot], 1u) == gridDim.x - 1) {
+    ds->tile_ctr[slot] = 0u;
+    ds->exit_ctr[slot] = 0u;
+    ds->epoch[slot] += 1ull;
+    __threadfence();
+  }
+}
+
+// ---- block-wide scans ---------------------------------------------------------------
+template <class T>
+__device__ __forceinline__ T warp_incl_scan(T v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    T u = __shfl_up_sync(0xffffffffu, v, d);
+    if (lane >= d) v += u;
+  }
+  return v;
+}
+
+// Block exclusive scan of one value per thread.  `smem` holds >= 33 T.
+// Returns the exclusive prefix; *total receives the block sum.
+template <class T>
+__device__ T block_excl_scan(T v, T* smem, T* total) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  T inc = warp_incl_scan(v);
+  if (lane == 31) smem[wid] = inc;
+  __syncthreads();
+  if (wid == 0) {
+    T s = (lane < nw) ? smem[lane] : T(0);
+    s = warp_incl_scan(s);
+    if (lane < nw) smem[lane] = s;   // inclusive warp totals
+  }
+  __syncthreads();
+  T base = (wid > 0) ? smem[wid - 1] : T(0);
+  *total = smem[nw - 1];
+  __syncthreads();
+  return base + inc - v;
+}
+
+__device__ __forceinline__ unsigned long long shfl_up_u64(unsigned long long v, int d) {
+  return __shfl_up_sync(0xffffffffu, v, d);
+}
+
+// Block exclusive scan of a pair of 64-bit values.
+__device__ __forceinline__ Pair64 block_excl_scan_pair(Pair64 v, Pair64* smem, Pair64* total) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  Pair64 inc = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    unsigned long long ua = shfl_up_u64(inc.a, d), ub = shfl_up_u64(inc.b, d);
+    if (lane >= d) {
+      inc.a += ua;
+      inc.b += ub;
+    }
+  }
+  if (lane == 31) smem[wid] = inc;
+  __syncthreads();
+  if (wid == 0) {
+    Pair64 s = (lane < nw) ? smem[lane] : Pair64{0, 0};
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      unsigned long long ua = shfl_up_u64(s.a, d), ub = shfl_up_u64(s.b, d);
+      if (lane >= d) {
+        s.a += ua;
+        s.b += ub;
+      }
+    }
+    if (lane < nw) smem[lane] = s;
+  }
+  __syncthreads();
+  Pair64 base = (wid > 0) ? smem[wid - 1] : Pair64{0, 0};
+  *total = smem[nw - 1];
+  __syncthreads();
+  return Pair64{base.a + inc.a - v.a, base.b + inc.b - v.b};
+}
+
+__host__ __device__ constexpr uint64_t ceil_div(uint64_t a, uint64_t b) { return (a + b - 1) / b; }
+
+}  // namespace ro

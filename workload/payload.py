@@ -53,15 +53,42 @@ def records_concat(seed: int, children, lengths) -> bytes:
     return b"".join(record_bytes(seed, int(c), int(n)) for c, n in zip(children, lengths))
 
 
+def _host_lib():
+    import ctypes as C
+    import os
+    from .build import HOST_LIB, build_host
+    if not os.path.exists(HOST_LIB):
+        build_host()
+    L = C.CDLL(HOST_LIB)
+    L.wl_fill_host.argtypes = [C.c_void_p, C.c_uint64, C.c_void_p, C.c_void_p, C.c_void_p,
+                               C.c_uint64, C.c_uint64]
+    L.wl_fill_host.restype = C.c_int
+    return L
+
+
 def fill_host_arena(seed: int, children: np.ndarray, offsets: np.ndarray,
-                    lengths: np.ndarray, arena_bytes: int,
+                    lengths: np.ndarray, arena_bytes: int, use_c: bool = True,
                     chunk_bytes: int = 1 << 26) -> np.ndarray:
     """Build a host arena (uint8) holding each listed child's record at its offset.
 
-    Vectorised over children in chunks of about ``chunk_bytes`` payload bytes.
+    Uses the C filler (``csrc/payload_host.c``) when gcc is available, else a
+    numpy version vectorised over children in chunks of ``chunk_bytes``.
     Children with length 0 are skipped.
     """
-    arena = np.zeros(arena_bytes, dtype=np.uint8)
+    arena = np.zeros(max(arena_bytes, 1), dtype=np.uint8)[:arena_bytes]
+    if use_c:
+        try:
+            L = _host_lib()
+        except Exception:
+            L = None
+        if L is not None:
+            c = np.ascontiguousarray(children, dtype=np.uint64)
+            o = np.ascontiguousarray(offsets, dtype=np.uint64)
+            ln = np.ascontiguousarray(lengths, dtype=np.uint64)
+            if L.wl_fill_host(arena.ctypes.data, arena_bytes, c.ctypes.data, o.ctypes.data,
+                              ln.ctypes.data, c.size, seed & ((1 << 64) - 1)) != 0:
+                raise ValueError("record outside the arena")
+            return arena
     children = np.asarray(children, dtype=np.uint64)
     offsets = np.asarray(offsets, dtype=np.uint64)
     lengths = np.asarray(lengths, dtype=np.int64)
