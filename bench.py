@@ -120,6 +120,16 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+# ------------------------------------------------------------------ ranks
+def max_over_ranks(x: float) -> float:
+    """Largest value of x over all ranks (gloo; host tensors only)."""
+    import torch
+    import torch.distributed as td
+    t = torch.tensor([float(x)], dtype=torch.float64)
+    td.all_reduce(t, op=td.ReduceOp.MAX)
+    return float(t.item())
+
+
 # ------------------------------------------------------------------ CPU oracle
 def cpu_oracle_sample(parents: int, waves: int):
     """Time the oracle (single-threaded C) on a bounded sample of the same
@@ -313,9 +323,7 @@ def run_ours(args, rank, world, local_rank):
         raise RuntimeError(f"device reported {st}: {ro.ro_last_error(ctx)}")
     S = int(ps.out_bytes.sum().item())
     if dist:
-        t = torch.tensor([ms_total], dtype=torch.float64)
-        td.all_reduce(t, op=td.ReduceOp.MAX)
-        ms_total = float(t.item())
+        ms_total = max_over_ranks(ms_total)
     ms_step = ms_total / args.steps
     value = world * ps.N / (ms_step * 1e-3)
 

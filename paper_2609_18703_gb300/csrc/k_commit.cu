@@ -136,12 +136,12 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
   if (threadIdx.x == 0) s_dups = 0;
   __syncthreads();
   // A: this call's sealer of a conflicted Grain marks itself and opens the
-  //    minimum-index election in the record's len field
+  //    minimum-index election in the record's len field with its own index
   for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
     if (a.code[r] != V_ACCEPT) continue;
     Rec* rc = a.rec + a.child[r];
     if (ld_w(rc) & W_CONFLICT_BIT) {
-      rc->len = 0xFFFFFFFFu;
+      rc->len = (uint32_t)r;
       atomicOr((unsigned long long*)&rc->w, (unsigned long long)W_SEALER_BIT);
     }
   }
