@@ -245,6 +245,39 @@ ro_status ro_assemble(ro_ctx* ctx, int32_t xid, const uint8_t* d_arena, uint64_t
                       uint8_t* d_out, uint64_t out_cap, uint64_t* d_out_cursor,
                       uint64_t* d_out_bytes, uint64_t* h_out_bytes);
 
+/* ------------------------------------------------------------------------
+ * ro_expand_noalloc — the offsets, parents and ordinals of ro_expand, for
+ * callers that cannot allocate device memory.  The paper has no counterpart;
+ * this is a deployment variant.
+ *
+ * Some callers cannot call cudaMalloc: code that runs inside a memory budget
+ * owned by another allocator, code that must not synchronise the device the
+ * way cudaMalloc/cudaFree may, or embedders that forbid allocation after
+ * start-up.  This call needs no context and allocates nothing.  Its scratch
+ * (scan tile status, fill-tile table, counters) is one fixed array of about
+ * 292 KB in the library's device memory, which every GPU that loads the
+ * library holds until the process exits.  It keeps no lineage state, so the
+ * result cannot be committed or assembled against.
+ *
+ *   Arguments as in ro_expand (d_counts, n_parents, d_offsets uint64[P+1],
+ *   d_child_parent / d_child_ordinal uint32[child_cap], d_empty_parents
+ *   uint32[P] or NULL), on `stream` (a cudaStream_t, NULL = legacy default
+ *   stream) of the current device.  h_n_children (required) and h_n_empty
+ *   (optional) receive N and the number of empty parents; the call
+ *   synchronises the stream.
+ *   Limits: at most 16,777,216 parents and 134,217,728 children, else
+ *   RO_E_CAPACITY (beyond the static scratch; nothing is launched when the
+ *   parent count is too large).  RO_E_CAPACITY also when N > child_cap.
+ *   The first call on a device looks up the scratch's device address; make
+ *   that first call before any stream capture.  All calls share the one
+ *   scratch array: calls that overlap on the GPU (other streams, other host
+ *   threads) race and must be serialised by the caller.
+ */
+ro_status ro_expand_noalloc(const uint32_t* d_counts, uint64_t n_parents, uint64_t* d_offsets,
+                            uint32_t* d_child_parent, uint32_t* d_child_ordinal,
+                            uint64_t child_cap, uint32_t* d_empty_parents, void* stream,
+                            uint64_t* h_n_children, uint64_t* h_n_empty);
+
 #ifdef __cplusplus
 }
 #endif

@@ -29,7 +29,7 @@ STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFL
 
 EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro_ctx_stats",
            "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
-           "ro_gather_commit", "ro_assemble")
+           "ro_gather_commit", "ro_assemble", "ro_expand_noalloc")
 
 # kernel ids (RO_K_*), in launch order of the path
 KERNELS = ("expand_scan", "expand_fill", "ready_count", "ready_scatter", "commit_scatter",
@@ -82,6 +82,7 @@ def load(path: Optional[str] = None):
                                    _vp, _pu64]
     L.ro_assemble.argtypes = [_vp, _i32, _vp, _u64, _vp, _u64, _vp, _vp, _vp, _vp, _vp, _u64, _vp, _vp,
                               _pu64]
+    L.ro_expand_noalloc.argtypes = [_vp, _u64, _vp, _vp, _vp, _u64, _vp, _vp, _pu64, _pu64]
     for f in EXPORTS:
         if f != "ro_last_error":
             getattr(L, f).restype = C.c_int32
@@ -208,3 +209,15 @@ def ro_assemble(ctx, xid, d_arena, arena_bytes, d_parents, n_parents, d_n_parent
                             _ptr(d_out), out_cap, _ptr(d_out_cursor), _ptr(d_out_bytes),
                             C.byref(ob) if want_host else None)
     return (st, ob.value) if want_host else (st, None)
+
+
+def ro_expand_noalloc(d_counts, n_parents, d_offsets, d_child_parent, d_child_ordinal, child_cap,
+                      d_empty_parents=None, stream=None):
+    """Context-free expansion that allocates nothing (static device scratch).
+    Returns (status, n_children, n_empty)."""
+    n = _u64(0)
+    ne = _u64(0)
+    st = load().ro_expand_noalloc(_ptr(d_counts), n_parents, _ptr(d_offsets), _ptr(d_child_parent),
+                                  _ptr(d_child_ordinal), child_cap, _ptr(d_empty_parents),
+                                  _stream_handle(stream), C.byref(n), C.byref(ne))
+    return st, n.value, ne.value
