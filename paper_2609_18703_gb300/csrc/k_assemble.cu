@@ -3,23 +3,25 @@
 // A completed parent is Suppressed if a member Failed or was Suppressed,
 // otherwise Present with the Present members' payloads concatenated by
 // ordinal (Dropped members add nothing).  The work is a segmented byte gather
-// from the result arena, done in three passes:
-//   asm_parents  per listed parent: outcome, number of members to gather
-//                (0 unless Present), exclusive scan of those counts (member
-//                bases), and for every 2048-member tile the parent that
-//                contains its first member.
+// from the result arena:
+//   asm_parents  (explicit lists only) per listed parent: outcome, number of
+//                members to gather (0 unless Present), exclusive scan of those
+//                counts (member bases), and for every 2048-member tile the
+//                parent containing its first member.  For the latest commit's
+//                own list, commit_finish has already produced this plan.
 //   asm_members  per member (load-balanced over tiles of 2048 members, so a
 //                100k-member parent is spread over many CTAs): read its
 //                record, scan the Present bytes (single-pass look-back) and
 //                emit, for every member that contributes bytes, its output
 //                position and arena offset, plus each parent's output offset
-//                and, for every 16 KB output chunk, the first member in it.
-//   asm_copy     per 16 KB output chunk: stage the chunk's members in shared
-//                memory and write the chunk as aligned 16-byte stores.  Each
-//                store takes its bytes from one member with two aligned
-//                16-byte loads and a funnel shift (source and destination
-//                alignments differ arbitrarily); words that straddle members
-//                or the ends of the output are assembled byte by byte.
+//                and, for every 32 KB output chunk, the first member in it.
+//   asm_copy     per 32 KB output chunk: stage the chunk's members in shared
+//                memory; every thread then writes 8 aligned 16-byte words,
+//                four in flight at a time.  A word's bytes come from at most
+//                two members (more only for records under 16 bytes): each
+//                piece is read as the one or two aligned 16-byte blocks that
+//                hold it and shifted into place with funnel shifts, so source
+//                and destination alignments may differ arbitrarily.
 #include <algorithm>
 
 #include "ro_internal.h"
@@ -68,9 +70,19 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
     }
     return;   // no tile claimed
   }
-  if (threadIdx.x == 0) s_incomplete = 0;
   const uint64_t TILE = (uint64_t)AP_THREADS * AP_ITEMS;
   const uint64_t n_tiles = ceil_div(n, TILE);
+  if (n_tiles == 0) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      a.mb[0] = 0;
+      ds->as_M = 0;
+      ds->as_n = 0;
+    }
+    return;
+  }
+  const uint32_t n_part = participants(n_tiles);
+  if (blockIdx.x >= n_part) return;
+  if (threadIdx.x == 0) s_incomplete = 0;
   for (;;) {
     if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_ASM_PARENTS]);
     __syncthreads();
@@ -133,12 +145,7 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
   __syncthreads();
   if (threadIdx.x == 0) {
     if (s_incomplete) atomicAdd(&ds->stats[6], s_incomplete);
-    if (n_tiles == 0 && blockIdx.x == 0) {
-      a.mb[0] = 0;
-      ds->as_M = 0;
-      ds->as_n = 0;
-    }
-    retire_cta(ds, TS_ASM_PARENTS);
+    retire_cta(ds, TS_ASM_PARENTS, n_part);
   }
 }
 
@@ -150,8 +157,23 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
   __shared__ uint32_t s_tile;
   __shared__ Pair64 s_prefix;
   DevScalars* ds = a.ds;
-  if (ds->as_err) return;   // nothing claimed
-  const uint64_t n = ds->as_n, M = ds->as_M;
+  uint64_t n, M;
+  if (a.list_is_commit) {
+    n = ds->cm_n_done;
+    M = ds->cm_M;
+    if (n > a.n_host) {   // the commit completed more parents than the outputs hold
+      if (blockIdx.x == 0 && threadIdx.x == 0) {
+        ds->as_err = 1u;
+        atomicOr(&ds->err, ERR_CAPACITY);
+      }
+      return;
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) ds->as_n = n;
+  } else {
+    if (ds->as_err) return;   // nothing claimed
+    n = ds->as_n;
+    M = ds->as_M;
+  }
   const uint64_t base = a.cursor ? *a.cursor : 0ull;
   const uint64_t out_addr = (uint64_t)(uintptr_t)a.out;
   const uint64_t origin = (out_addr + base) & ~15ull;
@@ -173,6 +195,8 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
     return;
   }
 
+  const uint32_t n_part = participants(n_tiles);
+  if (blockIdx.x >= n_part) return;
   for (;;) {
     if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_ASM_MEMBERS]);
     __syncthreads();
@@ -292,19 +316,12 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
     }
     __syncthreads();
   }
-  if (threadIdx.x == 0) retire_cta(ds, TS_ASM_MEMBERS);
+  if (threadIdx.x == 0) retire_cta(ds, TS_ASM_MEMBERS, n_part);
 }
 
 // ---------------------------------------------------------------------------
-// 16 bytes starting at any address, from the one or two aligned 16-byte
-// blocks that hold them (both lie inside the record being read).
-__device__ __forceinline__ uint4 load16_any(const uint8_t* p) {
-  const uintptr_t addr = (uintptr_t)p;
-  const uint32_t sh = (uint32_t)(addr & 15u);
-  const uint4* q = reinterpret_cast<const uint4*>(addr & ~(uintptr_t)15);
-  const uint4 x = __ldg(q);
-  if (sh == 0) return x;
-  const uint4 y = __ldg(q + 1);
+// Bytes sh .. sh+15 of the 32-byte window (x, y), sh in [0, 15].
+__device__ __forceinline__ uint4 window16(const uint4 x, const uint4 y, uint32_t sh) {
   const uint32_t b = (sh & 3u) * 8u;
   uint32_t a0, a1, a2, a3, a4;
   switch (sh >> 2) {
@@ -321,110 +338,383 @@ __device__ __forceinline__ uint4 load16_any(const uint8_t* p) {
   return r;
 }
 
-__global__ void __launch_bounds__(AC_THREADS) asm_copy_kernel(AssembleArgs a) {
-  __shared__ uint64_t s_pos[AC_SMEM_CAP + 1];
-  __shared__ uint64_t s_src[AC_SMEM_CAP];
+__device__ __forceinline__ uint4 shfl_down4(const uint4 v, int d) {
+  return make_uint4(__shfl_down_sync(0xffffffffu, v.x, d), __shfl_down_sync(0xffffffffu, v.y, d),
+                    __shfl_down_sync(0xffffffffu, v.z, d), __shfl_down_sync(0xffffffffu, v.w, d));
+}
+__device__ __forceinline__ uint4 shfl_idx4(const uint4 v, int l) {
+  return make_uint4(__shfl_sync(0xffffffffu, v.x, l), __shfl_sync(0xffffffffu, v.y, l),
+                    __shfl_sync(0xffffffffu, v.z, l), __shfl_sync(0xffffffffu, v.w, l));
+}
+
+// 32-bit lane mask selecting bytes [lo, hi) of word q (0..3) of a 16-byte word.
+__device__ __forceinline__ uint32_t byte_mask(uint32_t lo, uint32_t hi, int q) {
+  const uint32_t m16 = ((1u << hi) - 1u) & ~((1u << lo) - 1u);   // hi <= 16
+  const uint32_t nib = (m16 >> (4 * q)) & 0xFu;
+  return ((nib & 1u) * 0xFFu) | ((nib & 2u) * 0x7F80u) | ((nib & 4u) * 0x3FC000u) |
+         ((nib & 8u) * 0x1FE00000u);
+}
+
+// acc with bytes [lo, hi) replaced by those of v
+__device__ __forceinline__ uint4 merge_piece(uint4 acc, const uint4 v, uint32_t lo, uint32_t hi) {
+  uint32_t m;
+  m = byte_mask(lo, hi, 0); acc.x = (acc.x & ~m) | (v.x & m);
+  m = byte_mask(lo, hi, 1); acc.y = (acc.y & ~m) | (v.y & m);
+  m = byte_mask(lo, hi, 2); acc.z = (acc.z & ~m) | (v.z & m);
+  m = byte_mask(lo, hi, 3); acc.w = (acc.w & ~m) | (v.w & m);
+  return acc;
+}
+
+constexpr int CP_UNROLL = 4;   // groups of 32 words in flight per warp
+
+// One warp copies `len` bytes from src to dst (both any alignment).  Whole
+// destination words are written with 16-byte stores, each lane's word built
+// from its own aligned source block and its right neighbour's (shuffled in,
+// or loaded by the lane at a group's edge); the partial first and last words
+// are written byte by byte, so the bytes of neighbouring pieces are never
+// touched.  Every block read holds at least one byte of the source range.
+// (Used for chunks whose pieces do not fit the shared-memory stage.)
+__device__ __forceinline__ void warp_copy(uint8_t* dst, const uint8_t* src, uint64_t len, int lane) {
+  const uint64_t d = (uint64_t)(uintptr_t)dst, d_end = d + len;
+  const uint64_t head_end = ((d + 15) & ~15ull) < d_end ? ((d + 15) & ~15ull) : d_end;
+  if ((uint64_t)lane < head_end - d) dst[lane] = __ldg(src + lane);
+  if (head_end == d_end) return;
+  const uint64_t full_lo = head_end, full_hi = d_end & ~15ull;
+  if (full_hi > full_lo) {
+    const uint64_t nw = (full_hi - full_lo) >> 4;
+    const uint8_t* s_full = src + (full_lo - d);
+    const uint32_t sig = (uint32_t)((uintptr_t)s_full & 15u);
+    const uint4* A0 = reinterpret_cast<const uint4*>((uintptr_t)s_full & ~(uintptr_t)15);
+    uint4* D0 = reinterpret_cast<uint4*>((uintptr_t)full_lo);
+    for (uint64_t g0 = 0; g0 < nw; g0 += 32 * CP_UNROLL) {
+      uint4 x[CP_UNROLL], y[CP_UNROLL];
+#pragma unroll
+      for (int u = 0; u < CP_UNROLL; ++u) {
+        const uint64_t k = g0 + (uint64_t)u * 32 + lane;
+        x[u] = make_uint4(0u, 0u, 0u, 0u);
+        y[u] = x[u];
+        if (k < nw) {
+          x[u] = __ldg(A0 + k);
+          const bool edge = (lane == 31 && (u == CP_UNROLL - 1 || k + 1 >= nw)) || k + 1 >= nw;
+          if (sig && edge) y[u] = __ldg(A0 + k + 1);
+        }
+      }
+      if (sig) {
+#pragma unroll
+        for (int u = 0; u < CP_UNROLL; ++u) {
+          const uint64_t k = g0 + (uint64_t)u * 32 + lane;
+          const uint4 nb = shfl_down4(x[u], 1);
+          const uint4 nx = (u + 1 < CP_UNROLL) ? shfl_idx4(x[(u + 1) % CP_UNROLL], 0) : nb;
+          const bool edge = (lane == 31 && (u == CP_UNROLL - 1 || k + 1 >= nw)) || k + 1 >= nw;
+          if (!edge) y[u] = (lane == 31) ? nx : nb;
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < CP_UNROLL; ++u) {
+        const uint64_t k = g0 + (uint64_t)u * 32 + lane;
+        if (k < nw) D0[k] = sig ? window16(x[u], y[u], sig) : x[u];
+      }
+    }
+  }
+  const uint64_t tail_lo = full_hi > head_end ? full_hi : head_end;
+  if ((uint64_t)lane < d_end - tail_lo) dst[(tail_lo - d) + lane] = __ldg(src + (tail_lo - d) + lane);
+}
+
+// ---- TMA staging --------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0u;
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// bulk copy of `bytes` (multiple of 16) from 16-byte aligned global memory
+// into 16-byte aligned shared memory, completing on `bar`
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
+// Bounded wait on a stage barrier; false (and ERR_TIMEOUT) if it gave up.
+__device__ __forceinline__ bool stage_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
+  for (uint32_t i = 0; i < (1u << 20); ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 255u) == 255u && (ld_acquire(err) & ERR_TIMEOUT)) break;
+  }
+  atomicOr(err, ERR_TIMEOUT);
+  return false;
+}
+
+// One pipeline stage: the source bytes of one 16 KB output chunk, laid out
+// piece by piece (each piece = the part of one member inside the chunk, read
+// as the aligned 16-byte blocks that hold it).
+struct CopyStage {
+  uint32_t np;                    // pieces staged, or AC_FALLBACK
+  uint32_t vbeg, vend;            // valid output bytes of the chunk, chunk-relative
+  uint32_t pad;
+  uint32_t pstart[AC_PIECES + 1]; // chunk-relative output start of each piece (+ end)
+  int32_t qbase[AC_PIECES];       // buffer offset of output byte 0 of the chunk, per piece
+  __align__(16) unsigned char buf[AC_BUF + 64];
+};
+constexpr uint32_t AC_FALLBACK = 0xFFFFFFFFu;
+
+size_t asm_copy_smem() { return 2 * sizeof(CopyStage); }
+
+struct CopyCtx {
+  const AssembleArgs* a;
+  uint64_t out_addr, start, end, origin, n_chunks, Mnz, end_rel;
+};
+
+__device__ __forceinline__ uint64_t cpos_at(const CopyCtx& c, uint64_t j) {
+  return j < c.Mnz ? c.a->cpos[j] : c.end_rel;
+}
+
+// Warp 0 stages chunk b: piece table, then one bulk copy per piece.
+__device__ void stage_chunk(const CopyCtx& c, uint64_t b, CopyStage* st, uint64_t* bar, int lane) {
+  const AssembleArgs& a = *c.a;
+  const uint64_t cs = c.origin + b * AC_CHUNK;
+  const uint64_t ce = cs + AC_CHUNK;
+  const uint64_t vb = cs > c.start ? cs : c.start;
+  const uint64_t ve = ce < c.end ? ce : c.end;
+  const uint64_t j_lo = a.ctfp[b];
+  const uint64_t j_hi = (b + 1 < c.n_chunks) ? a.ctfp[b + 1] : c.Mnz - 1;
+  const uint64_t np = j_hi - j_lo + 1;
+  if (lane == 0) {
+    st->vbeg = (uint32_t)(vb - cs);
+    st->vend = (uint32_t)(ve - cs);
+  }
+  bool fits = np <= AC_PIECES;
+  uint32_t roff = 0;   // running buffer offset (uniform)
+  if (fits) {
+    for (uint64_t g = 0; g < np; g += 32) {
+      const uint64_t i = g + lane;
+      uint32_t size = 0, sh = 0, ps = 0;
+      if (i < np) {
+        const uint64_t j = j_lo + i;
+        const uint64_t p0 = c.out_addr + a.cpos[j], p1 = c.out_addr + cpos_at(c, j + 1);
+        const uint64_t ob = p0 > vb ? p0 : vb, oe = p1 < ve ? p1 : ve;
+        const uint64_t src = (uint64_t)(uintptr_t)a.arena + a.csrc[j] + (ob - p0);
+        const uint64_t a0 = src & ~15ull, a1 = (src + (oe - ob) + 15) & ~15ull;
+        size = (uint32_t)(a1 - a0);
+        sh = (uint32_t)(src & 15u);
+        ps = (uint32_t)(ob - cs);
+      }
+      uint32_t inc = size;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const uint32_t t = __shfl_up_sync(0xffffffffu, inc, d);
+        if (lane >= d) inc += t;
+      }
+      const uint32_t my_off = roff + inc - size;
+      if (i < np) {
+        st->pstart[i] = ps;
+        st->qbase[i] = (int32_t)(my_off + sh) - (int32_t)ps;
+      }
+      roff += __shfl_sync(0xffffffffu, inc, 31);
+    }
+    fits = roff <= AC_BUF;
+  }
+  if (!fits) {
+    if (lane == 0) {
+      st->np = AC_FALLBACK;
+      mbar_arrive(bar);   // completes the phase; consumers copy from global
+    }
+    __syncwarp();
+    return;
+  }
+  if (lane == 0) {
+    st->np = (uint32_t)np;
+    st->pstart[np] = (uint32_t)(ve - cs);
+  }
+  __syncwarp();
+  fence_proxy_async_smem();   // earlier generic reads of this buffer before async writes
+  if (lane == 0) mbar_arrive_tx(bar, roff);
+  __syncwarp();
+  for (uint64_t i = lane; i < np; i += 32) {
+    const uint64_t j = j_lo + i;
+    const uint64_t p0 = c.out_addr + a.cpos[j];
+    const uint64_t ob = cs + st->pstart[i];
+    const uint64_t oe = cs + st->pstart[i + 1];
+    const uint64_t src = (uint64_t)(uintptr_t)a.arena + a.csrc[j] + (ob - p0);
+    const uint64_t a0 = src & ~15ull, a1 = (src + (oe - ob) + 15) & ~15ull;
+    const uint32_t off = (uint32_t)(st->qbase[i] + (int32_t)st->pstart[i]) - (uint32_t)(src & 15u);
+    if (a1 > a0)   // a member that starts exactly at the chunk's end stages nothing
+      bulk_g2s(st->buf + off, reinterpret_cast<const void*>((uintptr_t)a0), (uint32_t)(a1 - a0), bar);
+  }
+}
+
+// All threads: write chunk b from its staged pieces.
+__device__ void emit_chunk(const CopyCtx& c, uint64_t b, const CopyStage* st) {
+  const uint64_t cs = c.origin + b * AC_CHUNK;
+  const uint32_t np = st->np;
+  const uint32_t vbeg = st->vbeg, vend = st->vend;
+  const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll 1
+  for (uint32_t wr = threadIdx.x * 16u; wr < (uint32_t)AC_CHUNK; wr += AC_THREADS * 16u) {
+    const uint32_t vlo = wr > vbeg ? wr : vbeg;
+    const uint32_t vhi = (wr + 16u < vend) ? wr + 16u : vend;
+    if (vlo >= vhi) continue;
+    // piece holding chunk byte vlo
+    uint32_t lo_i = 0, hi_i = np;
+    while (hi_i - lo_i > 1) {
+      const uint32_t mid = (lo_i + hi_i) >> 1;
+      if (st->pstart[mid] <= vlo) lo_i = mid; else hi_i = mid;
+    }
+    uint32_t i = lo_i;
+    uint32_t lo = vlo - wr;
+    const uint32_t hiw = vhi - wr;
+    uint4 acc = zero;
+    for (;;) {
+      const uint32_t pe = st->pstart[i + 1] - wr;   // piece end, word-relative (may exceed 16)
+      const uint32_t hi = pe < hiw ? pe : hiw;
+      const int32_t q = st->qbase[i] + (int32_t)wr;
+      const int32_t A = (q + (int32_t)lo) & ~15;
+      const int32_t dl = q - A;
+      const uint4 x = *reinterpret_cast<const uint4*>(st->buf + A);
+      const uint4 y = *reinterpret_cast<const uint4*>(st->buf + A + 16);
+      const uint4 v = dl >= 0 ? window16(x, y, (uint32_t)dl) : window16(zero, x, (uint32_t)(16 + dl));
+      acc = (lo == 0u && hi == 16u) ? v : merge_piece(acc, v, lo, hi);
+      if (hi >= hiw) break;
+      lo = hi;
+      ++i;
+    }
+    const uint64_t W = cs + wr;
+    if (vlo == wr && vhi == wr + 16u) {
+      *reinterpret_cast<uint4*>((uintptr_t)W) = acc;
+    } else {
+      const uint32_t vv[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+      for (int t = 0; t < 16; ++t)
+        if ((uint32_t)t >= vlo - wr && (uint32_t)t < vhi - wr)
+          *reinterpret_cast<uint8_t*>((uintptr_t)(W + t)) = (uint8_t)(vv[t >> 2] >> (8 * (t & 3)));
+    }
+  }
+}
+
+// Chunk b copied from global memory by warps (pieces did not fit a stage).
+__device__ void emit_chunk_direct(const CopyCtx& c, uint64_t b) {
+  const AssembleArgs& a = *c.a;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr uint64_t SLICE = AC_CHUNK / (AC_THREADS / 32);
+  const uint64_t cs = c.origin + b * AC_CHUNK;
+  const uint64_t j_lo = a.ctfp[b];
+  const uint64_t j_hi = (b + 1 < c.n_chunks) ? a.ctfp[b + 1] : c.Mnz - 1;
+  const uint64_t sl = cs + (uint64_t)warp * SLICE, sh = sl + SLICE;
+  uint64_t ra = (sl > c.start ? sl : c.start) - c.out_addr;
+  const uint64_t rb = (sh < c.end ? sh : c.end) - c.out_addr;
+  if (ra >= rb) return;
+  uint64_t lo = j_lo, hi = j_hi + 1;
+  while (hi - lo > 1) {
+    const uint64_t mid = lo + ((hi - lo) >> 1);
+    if (a.cpos[mid] <= ra) lo = mid; else hi = mid;
+  }
+  for (uint64_t k = lo; ra < rb; ++k) {
+    const uint64_t pk = a.cpos[k], pn = cpos_at(c, k + 1);
+    const uint64_t e = pn < rb ? pn : rb;
+    warp_copy(a.out + ra, a.arena + a.csrc[k] + (ra - pk), e - ra, lane);
+    ra = e;
+  }
+}
+
+__global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a) {
+  extern __shared__ __align__(128) unsigned char ac_smem[];
+  __shared__ __align__(8) uint64_t bars[2];
+  CopyStage* stages = reinterpret_cast<CopyStage*>(ac_smem);
   DevScalars* ds = a.ds;
   const bool failed = ds->as_err != 0u;
   const uint64_t n = ds->as_n, S = ds->as_bytes, Mnz = ds->as_Mnz, base = ds->as_base;
-  const uint64_t out_addr = (uint64_t)(uintptr_t)a.out;
+  CopyCtx c;
+  c.a = &a;
+  c.out_addr = (uint64_t)(uintptr_t)a.out;
+  c.start = c.out_addr + base;
+  c.end = c.start + S;
+  c.origin = c.start & ~15ull;
+  c.n_chunks = (!failed && S) ? ceil_div(c.end - c.origin, AC_CHUNK) : 0;
+  c.Mnz = Mnz;
+  c.end_rel = base + S;
+  const uint64_t par_units = failed ? 0 : ceil_div(n, (uint64_t)AC_THREADS * 8);
+  uint64_t units = c.n_chunks > par_units ? c.n_chunks : par_units;
+  if (units == 0) units = 1;   // one CTA still finishes the call
+  const uint32_t n_part = participants(units);
+  if (blockIdx.x >= n_part) return;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   if (!failed) {
-    // per-parent byte counts
-    if (a.out_len) {
-      const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+    // per-parent outputs that need the whole scan: status (plan lists) and lengths
+    if (a.out_len || a.plan_status) {
+      const uint64_t stride = (uint64_t)n_part * blockDim.x;
       for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
-        const uint64_t len = a.out_off[i + 1] - a.out_off[i];
-        if (len > 0xFFFFFFFFull) atomicOr(&ds->err, ERR_OVERFLOW);
-        a.out_len[i] = (uint32_t)len;
+        if (a.plan_status) a.status[i] = a.plan_status[i];
+        if (a.out_len) {
+          const uint64_t len = a.out_off[i + 1] - a.out_off[i];
+          if (len > 0xFFFFFFFFull) atomicOr(&ds->err, ERR_OVERFLOW);
+          a.out_len[i] = (uint32_t)len;
+        }
       }
     }
-    const uint64_t start = out_addr + base, end = start + S;
-    const uint64_t origin = start & ~15ull;
-    const uint64_t n_chunks = S ? ceil_div(end - origin, AC_CHUNK) : 0;
-    const uint64_t stop = (end + 15) & ~15ull;
-    for (uint64_t b = blockIdx.x; b < n_chunks; b += gridDim.x) {
-      const uint64_t cs = origin + b * AC_CHUNK;
-      const uint64_t ce = (cs + AC_CHUNK < stop) ? cs + AC_CHUNK : stop;
-      const uint64_t j_lo = a.ctfp[b];
-      const uint64_t j_hi = (b + 1 < n_chunks) ? a.ctfp[b + 1] : Mnz - 1;
-      const uint64_t Rm = j_hi - j_lo + 1;
-      const bool staged = Rm + 1 <= AC_SMEM_CAP;
-      const uint64_t end_rel = base + S;
-      if (staged) {
-        for (uint64_t k = threadIdx.x; k <= Rm; k += blockDim.x) {
-          const uint64_t j = j_lo + k;
-          s_pos[k] = (j < Mnz) ? a.cpos[j] : end_rel;
-          if (k < Rm) s_src[k] = a.csrc[j];
-        }
+    if (threadIdx.x == 0) {
+      mbar_init(&bars[0], 1);
+      mbar_init(&bars[1], 1);
+      mbar_fence_init();
+    }
+    __syncthreads();
+    uint32_t phase[2] = {0u, 0u};
+    bool pending[2] = {false, false};
+    bool ok = true;
+    uint64_t b = blockIdx.x;
+    if (b < c.n_chunks) {
+      if (warp == 0) stage_chunk(c, b, &stages[0], &bars[0], lane);
+      pending[0] = true;
+    }
+    for (uint32_t it = 0; b < c.n_chunks && ok; b += n_part, ++it) {
+      const uint32_t s = it & 1u;
+      const uint64_t bn = b + n_part;
+      if (bn < c.n_chunks) {   // next chunk's loads overlap this chunk's writes
+        if (warp == 0) stage_chunk(c, bn, &stages[s ^ 1u], &bars[s ^ 1u], lane);
+        pending[s ^ 1u] = true;
       }
-      __syncthreads();
-      // position (relative to out) where member j_lo + k starts; k == Rm: end
-      auto pos_of = [&](uint64_t k) -> uint64_t {
-        if (staged) return s_pos[k];
-        const uint64_t j = j_lo + k;
-        return (j < Mnz) ? a.cpos[j] : end_rel;
-      };
-      auto src_of = [&](uint64_t k) -> uint64_t { return staged ? s_src[k] : a.csrc[j_lo + k]; };
-      auto find = [&](uint64_t rel) -> uint64_t {   // member holding relative byte rel
-        uint64_t lo = 0, hi = Rm;
-        while (hi - lo > 1) {
-          const uint64_t mid = lo + ((hi - lo) >> 1);
-          if (pos_of(mid) <= rel)
-            lo = mid;
-          else
-            hi = mid;
-        }
-        return lo;
-      };
-      const uint64_t n_words = (ce - cs) >> 4;
-      for (uint64_t wi = threadIdx.x; wi < n_words; wi += blockDim.x) {
-        const uint64_t W = cs + (wi << 4);
-        const uint64_t lo_v = W > start ? W : start;
-        const uint64_t hi_v = (W + 16 < end) ? W + 16 : end;
-        if (lo_v >= hi_v) continue;
-        uint64_t k = find(lo_v - out_addr);
-        const uint64_t p0 = pos_of(k), p1 = pos_of(k + 1);
-        const uint64_t wrel = W - out_addr;
-        if (lo_v == W && hi_v == W + 16 && p0 <= wrel && wrel + 16 <= p1) {
-          const uint4 v = load16_any(a.arena + src_of(k) + (wrel - p0));
-          *reinterpret_cast<uint4*>((uintptr_t)W) = v;
-          continue;
-        }
-        // the word straddles members or an end of the output
-        uint32_t wv[4] = {0u, 0u, 0u, 0u};
-        uint64_t kk = k, kp0 = p0, kp1 = p1, ksrc = src_of(k);
-#pragma unroll
-        for (int t = 0; t < 16; ++t) {
-          const uint64_t addr = W + t;
-          if (addr < lo_v || addr >= hi_v) continue;
-          const uint64_t rel = addr - out_addr;
-          while (rel >= kp1) {
-            ++kk;
-            kp0 = kp1;
-            kp1 = pos_of(kk + 1);
-            ksrc = src_of(kk);
-          }
-          const uint8_t byte = __ldg(a.arena + ksrc + (rel - kp0));
-          wv[t >> 2] |= (uint32_t)byte << (8 * (t & 3));
-        }
-        if (lo_v == W && hi_v == W + 16) {
-          *reinterpret_cast<uint4*>((uintptr_t)W) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
-        } else {
-#pragma unroll
-          for (int t = 0; t < 16; ++t) {
-            const uint64_t addr = W + t;
-            if (addr >= lo_v && addr < hi_v)
-              *reinterpret_cast<uint8_t*>((uintptr_t)addr) = (uint8_t)(wv[t >> 2] >> (8 * (t & 3)));
-          }
-        }
+      ok = stage_wait(&bars[s], phase[s], &ds->err);
+      phase[s] ^= 1u;
+      pending[s] = false;
+      if (ok) {
+        if (stages[s].np == AC_FALLBACK)
+          emit_chunk_direct(c, b);
+        else
+          emit_chunk(c, b, &stages[s]);
       }
       __syncthreads();
     }
+    // a wait that gave up: give outstanding copies a bounded chance to land
+    for (int s = 0; s < 2; ++s)
+      if (pending[s]) stage_wait(&bars[s], phase[s], &ds->err);
   }
   if (threadIdx.x == 0) {
     __threadfence();
-    if (atomicAdd(&ds->exit_ctr[TS_ASM_COPY], 1u) == gridDim.x - 1) {
+    if (atomicAdd(&ds->exit_ctr[TS_ASM_COPY], 1u) == n_part - 1) {
       if (!failed && a.cursor) *a.cursor = base + S;
       if (a.out_bytes) *a.out_bytes = S;
       ds->as_err = 0u;
@@ -435,9 +725,19 @@ __global__ void __launch_bounds__(AC_THREADS) asm_copy_kernel(AssembleArgs a) {
 }
 
 void launch_assemble(const LaunchCfg& L, const AssembleArgs& a) {
-  RO_LAUNCH(L, K_APARENTS, (asm_parents_kernel<<<L.grid_aparents, AP_THREADS, 0, L.stream>>>(a)));
+  if (!a.list_is_commit) {
+    const uint64_t tiles = ceil_div(a.n_host, (uint64_t)AP_THREADS * AP_ITEMS);
+    const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(tiles, (uint64_t)L.grid_aparents));
+    RO_LAUNCH(L, K_APARENTS, (asm_parents_kernel<<<grid, AP_THREADS, 0, L.stream>>>(a)));
+  }
   RO_LAUNCH(L, K_AMEMBERS, (asm_members_kernel<<<L.grid_amembers, AM_THREADS, 0, L.stream>>>(a)));
-  RO_LAUNCH(L, K_ACOPY, (asm_copy_kernel<<<L.grid_acopy, AC_THREADS, 0, L.stream>>>(a)));
+  RO_LAUNCH(L, K_ACOPY, (asm_copy_kernel<<<L.grid_acopy, AC_THREADS, asm_copy_smem(), L.stream>>>(a)));
+}
+
+// opt in to the copy kernel's dynamic shared memory (two pipeline stages)
+cudaError_t prepare_assemble_kernels() {
+  return cudaFuncSetAttribute(asm_copy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)asm_copy_smem());
 }
 
 const void* kernel_ptr_assemble(int which) {

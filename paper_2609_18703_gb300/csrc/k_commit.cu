@@ -193,23 +193,69 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
     }
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    atomicAdd(&ds->stats[4], s_dups);
-    ds->cm_conflicts = 0;
-  }
+  if (threadIdx.x == 0) atomicAdd(&ds->stats[4], s_dups);
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a) {
-  __shared__ unsigned long long s_scan[33];
-  __shared__ uint32_t s_tile;
-  __shared__ unsigned long long s_prefix;
-  DevScalars* ds = a.ds;
-  if (blockIdx.x == 0 && ds->cm_conflicts != 0) resolve_duplicates(a, commit_count(a));
+__device__ __forceinline__ uint32_t plan_members(const CommitArgs& a, uint32_t p, uint8_t* st) {
+  const unsigned long long v = __ldcg(a.pw + p);
+  if (pw_bad(v) != 0u) {
+    *st = ST_SUPPRESSED;
+    return 0u;
+  }
+  *st = ST_PRESENT;
+  return (uint32_t)(a.offsets[p + 1] - a.offsets[p]);
+}
 
+// Completed-parent list, ascending (popcount + single-pass scan over bitmap
+// words), plus the assembly plan of those parents: outcome, members to
+// gather and member bases, i.e. what ro_assemble's first pass would compute
+// for this list.
+__global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a) {
+  __shared__ Pair64 s_scan[33];
+  __shared__ uint32_t s_tile;
+  __shared__ Pair64 s_prefix;
+  __shared__ uint32_t s_fix;
+  DevScalars* ds = a.ds;
   const uint64_t n_words = ceil_div(a.P, 32);
   const uint64_t TILE = (uint64_t)CF_THREADS * CF_WORDS;
   const uint64_t n_tiles = ceil_div(n_words, TILE);
+  if (n_tiles == 0) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      ds->cm_n_done = 0;
+      ds->cm_M = 0;
+      a.plan_mb[0] = 0;
+      if (a.n_done_out) *a.n_done_out = 0;
+    }
+    return;
+  }
+  const uint32_t n_part = participants(n_tiles);
+  if (blockIdx.x >= n_part) return;
+
+  // Reports of one Grain that met in this call: the first CTA here orders
+  // them; the others wait for it before reading outcome classes.
+  if (ds->cm_conflicts != 0) {
+    if (threadIdx.x == 0) s_fix = atomicAdd(&ds->cm_fix_ticket, 1u);
+    __syncthreads();
+    if (s_fix == 0u) {
+      resolve_duplicates(a, commit_count(a));
+      if (threadIdx.x == 0) {
+        __threadfence();
+        st_release(&ds->cm_fix_done, 1u);
+      }
+    } else if (threadIdx.x == 0) {
+      uint32_t spins = 0;
+      while (ld_acquire(&ds->cm_fix_done) == 0u) {
+        if (++spins > SPIN_LIMIT) {
+          atomicOr(&ds->err, ERR_TIMEOUT);
+          break;
+        }
+        __nanosleep(128);
+      }
+    }
+    __syncthreads();
+  }
+
   for (;;) {
     if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_COMMIT]);
     __syncthreads();
@@ -218,17 +264,25 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
     if (tile >= n_tiles) break;
     const uint64_t w0 = tile * TILE + (uint64_t)threadIdx.x * CF_WORDS;
     uint32_t words[CF_WORDS];
-    unsigned long long cnt = 0;
+    Pair64 mine{0, 0};   // (completed parents, members to gather)
 #pragma unroll
     for (int k = 0; k < CF_WORDS; ++k) {
       words[k] = (w0 + k < n_words) ? a.bitmap[w0 + k] : 0u;
-      cnt += __popc(words[k]);
+      uint32_t bits = words[k];
+      mine.a += __popc(bits);
+      while (bits) {
+        const int b = __ffs(bits) - 1;
+        bits &= bits - 1;
+        uint8_t st;
+        mine.b += plan_members(a, (uint32_t)((w0 + k) * 32 + b), &st);
+      }
     }
-    unsigned long long total;
-    unsigned long long excl = block_excl_scan(cnt, s_scan, &total);
-    if (threadIdx.x == 0) s_prefix = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_COMMIT], &ds->err);
+    Pair64 total;
+    Pair64 excl = block_excl_scan_pair(mine, s_scan, &total);
+    if (threadIdx.x == 0)
+      s_prefix = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_COMMIT], &ds->err);
     __syncthreads();
-    unsigned long long pos = s_prefix + excl;
+    Pair64 run = s_prefix + excl;
 #pragma unroll
     for (int k = 0; k < CF_WORDS; ++k) {
       uint32_t bits = words[k];
@@ -238,22 +292,36 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
         const int b = __ffs(bits) - 1;
         bits &= bits - 1;
         const uint32_t parent = (uint32_t)((w0 + k) * 32 + b);
-        a.done_int[pos] = parent;
-        if (a.done_user) a.done_user[pos] = parent;
-        ++pos;
+        uint8_t st;
+        const uint32_t m = plan_members(a, parent, &st);
+        a.done_int[run.a] = parent;
+        if (a.done_user) a.done_user[run.a] = parent;
+        a.plan_status[run.a] = st;
+        a.plan_mb[run.a] = (uint32_t)run.b;
+        for (uint64_t t = ceil_div(run.b, AM_TILE); t * AM_TILE < run.b + m && t < a.plan_mtfp_cap; ++t)
+          a.plan_mtfp[t] = (uint32_t)run.a;
+        run.a += 1;
+        run.b += m;
       }
     }
     if (tile == n_tiles - 1 && threadIdx.x == CF_THREADS - 1) {
-      ds->cm_n_done = pos;
-      if (a.n_done_out) *a.n_done_out = pos;
+      ds->cm_n_done = run.a;
+      ds->cm_M = run.b;
+      a.plan_mb[run.a] = (uint32_t)run.b;
+      if (a.n_done_out) *a.n_done_out = run.a;
     }
   }
   if (threadIdx.x == 0) {
-    if (n_tiles == 0 && blockIdx.x == 0) {
-      ds->cm_n_done = 0;
-      if (a.n_done_out) *a.n_done_out = 0;
+    __threadfence();
+    if (atomicAdd(&ds->exit_ctr[TS_COMMIT], 1u) == n_part - 1) {
+      ds->tile_ctr[TS_COMMIT] = 0u;
+      ds->exit_ctr[TS_COMMIT] = 0u;
+      ds->epoch[TS_COMMIT] += 1ull;
+      ds->cm_conflicts = 0ull;
+      ds->cm_fix_ticket = 0u;
+      ds->cm_fix_done = 0u;
+      __threadfence();
     }
-    retire_cta(ds, TS_COMMIT);
   }
 }
 
@@ -263,7 +331,9 @@ void launch_commit(const LaunchCfg& L, const CommitArgs& a) {
       (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(warps, CM_THREADS / 32),
                                                     (uint64_t)L.grid_commit));
   RO_LAUNCH(L, K_COMMIT, (commit_scatter_kernel<<<grid, CM_THREADS, 0, L.stream>>>(a)));
-  RO_LAUNCH(L, K_CFINISH, (commit_finish_kernel<<<L.grid_cfinish, CF_THREADS, 0, L.stream>>>(a)));
+  const uint64_t n_tiles = ceil_div(ceil_div(a.P, 32), (uint64_t)CF_THREADS * CF_WORDS);
+  const int grid_f = (int)std::max<uint64_t>(1, std::min<uint64_t>(n_tiles, (uint64_t)L.grid_cfinish));
+  RO_LAUNCH(L, K_CFINISH, (commit_finish_kernel<<<grid_f, CF_THREADS, 0, L.stream>>>(a)));
 }
 
 const void* kernel_ptr_commit(int which) {

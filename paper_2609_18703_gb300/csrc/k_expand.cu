@@ -25,6 +25,17 @@ __global__ void __launch_bounds__(EXP_THREADS) expand_scan_kernel(ExpandScanArgs
   const uint64_t TILE = (uint64_t)EXP_THREADS * EXP_ITEMS;
   const uint64_t n_tiles = ceil_div(a.P, TILE);
   DevScalars* ds = a.ds;
+  if (n_tiles == 0) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      a.offsets_user[0] = 0;
+      a.offsets[0] = 0;
+      ds->n_children = 0;
+      ds->n_empty = 0;
+    }
+    return;
+  }
+  const uint32_t n_part = participants(n_tiles);
+  if (blockIdx.x >= n_part) return;
 
   for (;;) {
     if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_EXPAND]);
@@ -73,15 +84,7 @@ __global__ void __launch_bounds__(EXP_THREADS) expand_scan_kernel(ExpandScanArgs
       ds->n_empty = run.b;
     }
   }
-  if (threadIdx.x == 0) {
-    if (n_tiles == 0 && blockIdx.x == 0) {
-      a.offsets_user[0] = 0;
-      a.offsets[0] = 0;
-      ds->n_children = 0;
-      ds->n_empty = 0;
-    }
-    retire_cta(ds, TS_EXPAND);
-  }
+  if (threadIdx.x == 0) retire_cta(ds, TS_EXPAND, n_part);
 }
 
 // Largest index k in [lo, hi) with v[k] <= x (v non-decreasing, v[lo] <= x).

@@ -126,10 +126,16 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
     return;   // no tile counter was touched
   }
 
+  const uint64_t TILE = (uint64_t)RB_THREADS * RB_ITEMS;
+  const uint64_t n_tiles = ceil_div(a.n_cand, TILE);
+  const unsigned long long n_old = L < npop ? L : npop;
+  const uint64_t units = n_tiles > ceil_div(n_old, TILE) ? n_tiles : ceil_div(n_old, TILE);
+  const uint32_t n_part = participants(units);
+  if (blockIdx.x >= n_part) return;
+
   // entries queued by earlier calls leave first
   {
-    const unsigned long long n_old = L < npop ? L : npop;
-    const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+    const uint64_t stride = (uint64_t)n_part * blockDim.x;
     for (uint64_t j = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n_old; j += stride) {
       const uint32_t c = a.queue[head + j];
       a.batched[j] = c;
@@ -137,8 +143,6 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
     }
   }
 
-  const uint64_t TILE = (uint64_t)RB_THREADS * RB_ITEMS;
-  const uint64_t n_tiles = ceil_div(a.n_cand, TILE);
   for (;;) {
     if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_READY]);
     __syncthreads();
@@ -184,7 +188,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
       ++rank;
     }
   }
-  if (threadIdx.x == 0) retire_cta(ds, TS_READY);
+  if (threadIdx.x == 0) retire_cta(ds, TS_READY, n_part);
 }
 
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a) {

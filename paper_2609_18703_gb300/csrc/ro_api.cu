@@ -12,6 +12,8 @@
 #include "ro_internal.h"
 
 namespace ro {
+cudaError_t prepare_assemble_kernels();
+size_t asm_copy_smem();
 const void* kernel_ptr_expand(int which);
 const void* kernel_ptr_ready(int which);
 const void* kernel_ptr_commit(int which);
@@ -38,6 +40,7 @@ struct QueueBufs {
 // Device buffers of one expansion slot, kept across ro_ctx_reset and reused.
 struct ExpSlot {
   DevBuf offsets, pw, phase, rec, bitmap, done, tfp;
+  DevBuf plan_status, plan_mb, plan_mtfp;   // assembly plan of the latest commit
   std::vector<QueueBufs> queues;
 };
 
@@ -223,10 +226,12 @@ Expansion* get_exp(ro_ctx* c, int32_t xid) {
   return &c->exps[xid];
 }
 
-int grid_for(const void* k, int threads, int sms, int cap_per_sm) {
+int grid_for(const void* k, int threads, int sms, int cap_per_sm, size_t dyn_smem = 0) {
   int per = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k, threads, 0) != cudaSuccess || per < 1)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k, threads, dyn_smem) != cudaSuccess || per < 1) {
+    cudaGetLastError();
     per = 1;
+  }
   per = std::min(per, cap_per_sm);
   return per * sms;
 }
@@ -269,7 +274,14 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_cfinish = grid_for(kernel_ptr_commit(K_CFINISH), CF_THREADS, s, 4);
   c->L.grid_aparents = grid_for(kernel_ptr_assemble(K_APARENTS), AP_THREADS, s, 4);
   c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 8);
-  c->L.grid_acopy = grid_for(kernel_ptr_assemble(K_ACOPY), AC_THREADS, s, 8);
+  if (prepare_assemble_kernels() != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(c->ds);
+    cudaFreeHost(c->hs);
+    delete c;
+    return RO_E_CUDA;
+  }
+  c->L.grid_acopy = grid_for(kernel_ptr_assemble(K_ACOPY), AC_THREADS, s, 8, asm_copy_smem());
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) {
     cudaFree(c->ds);
@@ -292,6 +304,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   };
   for (auto& s : c->slots) {
     fr(s.offsets); fr(s.pw); fr(s.phase); fr(s.rec); fr(s.bitmap); fr(s.done); fr(s.tfp);
+    fr(s.plan_status); fr(s.plan_mb); fr(s.plan_mtfp);
     for (auto& q : s.queues) {
       fr(q.q);
       fr(q.state);
@@ -425,6 +438,9 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   RO_TRY(ensure(c, S.rec, N * sizeof(Rec), "result records"));
   RO_TRY(ensure(c, S.bitmap, ceil_div(P, 32) * sizeof(uint32_t), "completion bitmap"));
   RO_TRY(ensure(c, S.done, P * sizeof(uint32_t), "completed parents"));
+  RO_TRY(ensure(c, S.plan_status, P, "assembly plan"));
+  RO_TRY(ensure(c, S.plan_mb, (P + 1) * sizeof(uint32_t), "assembly plan"));
+  RO_TRY(ensure(c, S.plan_mtfp, (ceil_div(N, AM_TILE) + 2) * sizeof(uint32_t), "assembly plan"));
   cudaMemsetAsync(S.bitmap.p, 0, ceil_div(P, 32) * sizeof(uint32_t), c->stream);
   ExpandFillArgs fa{};
   fa.offsets = (const uint64_t*)S.offsets.p;
@@ -541,6 +557,11 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.done_user = d_done_parents;
   ca.done_int = (uint32_t*)S.done.p;
   ca.n_done_out = d_n_done;
+  ca.offsets = (const uint64_t*)S.offsets.p;
+  ca.plan_status = (uint8_t*)S.plan_status.p;
+  ca.plan_mb = (uint32_t*)S.plan_mb.p;
+  ca.plan_mtfp = (uint32_t*)S.plan_mtfp.p;
+  ca.plan_mtfp_cap = ceil_div(x->N, AM_TILE) + 2;
   ca.ds = c->ds;
   RO_TRY(tile_status(c, TS_COMMIT, ceil_div(ceil_div(x->P, 32), (uint64_t)CF_THREADS * CF_WORDS),
                      &ca.ts));
@@ -575,8 +596,10 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   const uint64_t member_cap = std::max<uint64_t>(x->N, 1);
   const uint64_t mtfp_cap = ceil_div(member_cap, AM_TILE) + 2;
   const uint64_t ctfp_cap = ceil_div(out_cap + 32, AC_CHUNK) + 2;
-  RO_TRY(ensure(c, c->mb, (n_parents + 1) * sizeof(uint32_t), "member bases"));
-  RO_TRY(ensure(c, c->mtfp, mtfp_cap * sizeof(uint32_t), "member tiles"));
+  if (d_parents) {
+    RO_TRY(ensure(c, c->mb, (n_parents + 1) * sizeof(uint32_t), "member bases"));
+    RO_TRY(ensure(c, c->mtfp, mtfp_cap * sizeof(uint32_t), "member tiles"));
+  }
   RO_TRY(ensure(c, c->cpos, member_cap * sizeof(uint64_t), "member positions"));
   RO_TRY(ensure(c, c->csrc, member_cap * sizeof(uint64_t), "member sources"));
   RO_TRY(ensure(c, c->ctfp, ctfp_cap * sizeof(uint32_t), "copy chunks"));
@@ -585,6 +608,7 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   aa.n_host = n_parents;
   aa.d_n = d_parents ? d_n_parents : nullptr;
   aa.list_is_commit = d_parents ? 0 : 1;
+  aa.plan_status = d_parents ? nullptr : (const uint8_t*)S.plan_status.p;
   aa.P = x->P;
   aa.N = x->N;
   aa.offsets = (const uint64_t*)S.offsets.p;
@@ -599,8 +623,8 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   aa.out_cap = out_cap;
   aa.cursor = d_out_cursor;
   aa.out_bytes = d_out_bytes;
-  aa.mb = (uint32_t*)c->mb.p;
-  aa.mtfp = (uint32_t*)c->mtfp.p;
+  aa.mb = d_parents ? (uint32_t*)c->mb.p : (uint32_t*)S.plan_mb.p;
+  aa.mtfp = d_parents ? (uint32_t*)c->mtfp.p : (uint32_t*)S.plan_mtfp.p;
   aa.mtfp_cap = mtfp_cap;
   aa.cpos = (uint64_t*)c->cpos.p;
   aa.csrc = (uint64_t*)c->csrc.p;

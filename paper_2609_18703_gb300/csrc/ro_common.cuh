@@ -82,7 +82,8 @@ struct DevScalars {
   unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
   uint32_t rb_ticket, rb_err;
   // ro_gather_commit
-  unsigned long long cm_n, cm_conflicts, cm_n_done;
+  unsigned long long cm_n, cm_conflicts, cm_n_done, cm_M;
+  uint32_t cm_fix_ticket, cm_fix_done;
   // ro_assemble
   unsigned long long as_n, as_M, as_Mnz, as_bytes, as_base, as_origin;
   uint32_t as_err, pad1;
@@ -202,11 +203,17 @@ __device__ T lookback_exclusive(const TileStatus<T>& ts, uint32_t tile, const T&
 // Claim the next tile of a dynamically scheduled (persistent) kernel.
 __device__ __forceinline__ uint32_t claim_tile(uint32_t* ctr) { return atomicAdd(ctr, 1u); }
 
-// Called by thread 0 of every CTA on exit; the last CTA out resets the tile
-// counter and advances the epoch for the next launch of this kernel.
-__device__ __forceinline__ void retire_cta(DevScalars* ds, int slot) {
+// CTAs that take part in a persistent kernel: never more than there are work
+// units, so small launches cost few atomics.  The others return at once.
+__device__ __forceinline__ uint32_t participants(uint64_t units) {
+  return (uint32_t)(units < (uint64_t)gridDim.x ? units : (uint64_t)gridDim.x);
+}
+
+// Called by thread 0 of every participating CTA on exit; the last one out
+// resets the tile counter and advances the epoch for the next launch.
+__device__ __forceinline__ void retire_cta(DevScalars* ds, int slot, uint32_t n_part) {
   __threadfence();
-  if (atomicAdd(&ds->exit_ctr[slot], 1u) == gridDim.x - 1) {
+  if (atomicAdd(&ds->exit_ctr[slot], 1u) == n_part - 1) {
     ds->tile_ctr[slot] = 0u;
     ds->exit_ctr[slot] = 0u;
     ds->epoch[slot] += 1ull;

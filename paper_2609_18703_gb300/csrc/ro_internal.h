@@ -22,7 +22,8 @@ constexpr uint32_t AM_TILE = AM_THREADS * AM_ITEMS;
 constexpr uint32_t AM_SMEM_CAP = 4096;                        // listed parents staged per tile
 constexpr int AC_THREADS = 256;
 constexpr uint64_t AC_CHUNK = 16384;                          // output bytes per copy chunk
-constexpr uint32_t AC_SMEM_CAP = 1536;                        // members staged per chunk
+constexpr uint32_t AC_BUF = 26624;                            // staged source bytes per chunk
+constexpr uint32_t AC_PIECES = 640;                           // member pieces staged per chunk
 
 // kernel entry points for occupancy queries and per-kernel timing
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CFINISH, K_APARENTS,
@@ -115,8 +116,14 @@ struct CommitArgs {
   uint32_t* done_user;        // optional
   uint32_t* done_int;
   uint64_t* n_done_out;       // optional device output
+  // assembly plan of the completed parents (consumed by ro_assemble(NULL))
+  const uint64_t* offsets;
+  uint8_t* plan_status;       // P
+  uint32_t* plan_mb;          // P+1 member bases
+  uint32_t* plan_mtfp;        // member tile -> containing listed parent
+  uint64_t plan_mtfp_cap;
   DevScalars* ds;
-  TileStatus<unsigned long long> ts;
+  TileStatus<Pair64> ts;
 };
 void launch_commit(const LaunchCfg& L, const CommitArgs& a);
 
@@ -124,8 +131,9 @@ void launch_commit(const LaunchCfg& L, const CommitArgs& a);
 struct AssembleArgs {
   const uint32_t* list;       // user's list or the latest commit's
   uint64_t n_host;            // list length, or capacity of the outputs
-  const uint64_t* d_n;        // device list length (optional)
-  int list_is_commit;         // list is the commit's internal list (count in ds->cm_n_done)
+  const uint64_t* d_n;        // device list length (optional, user list only)
+  int list_is_commit;         // plan of the latest commit (counts in ds->cm_n_done / cm_M)
+  const uint8_t* plan_status; // that plan's statuses (copied to status), or NULL
   uint64_t P, N;
   const uint64_t* offsets;
   const unsigned long long* pw;
@@ -139,7 +147,7 @@ struct AssembleArgs {
   uint64_t out_cap;
   uint64_t* cursor;           // optional (device)
   uint64_t* out_bytes;        // optional (device)
-  // scratch
+  // member bases / member-tile table: scratch (user list) or the commit's plan
   uint32_t* mb;               // member base per listed parent (n+1)
   uint32_t* mtfp;             // member tile -> containing listed parent
   uint64_t mtfp_cap;
