@@ -3,25 +3,23 @@
 // A completed parent is Suppressed if a member Failed or was Suppressed,
 // otherwise Present with the Present members' payloads concatenated by
 // ordinal (Dropped members add nothing).  The work is a segmented byte gather
-// from the result arena:
-//   asm_parents  (explicit lists only) per listed parent: outcome, number of
-//                members to gather (0 unless Present), exclusive scan of those
-//                counts (member bases), and for every 2048-member tile the
-//                parent containing its first member.  For the latest commit's
-//                own list, commit_finish has already produced this plan.
+// from the result arena, driven by an assembly plan: per listed parent its
+// relative output offset, per contributing member its relative position and
+// arena offset.  For the parents completed by the latest commit,
+// commit_finish has built the plan already; for an explicit list:
+//   asm_parents  per listed parent: outcome, number of members to gather
+//                (0 unless Present), exclusive scan of those counts (member
+//                bases), and for every 2048-member tile the parent holding its
+//                first member;
 //   asm_members  per member (load-balanced over tiles of 2048 members, so a
 //                100k-member parent is spread over many CTAs): read its
-//                record, scan the Present bytes (single-pass look-back) and
-//                emit, for every member that contributes bytes, its output
-//                position and arena offset, plus each parent's output offset
-//                and, for every 32 KB output chunk, the first member in it.
-//   asm_copy     per 32 KB output chunk: stage the chunk's members in shared
-//                memory; every thread then writes 8 aligned 16-byte words,
-//                four in flight at a time.  A word's bytes come from at most
-//                two members (more only for records under 16 bytes): each
-//                piece is read as the one or two aligned 16-byte blocks that
-//                hold it and shifted into place with funnel shifts, so source
-//                and destination alignments may differ arbitrarily.
+//                record and scan the Present bytes (single-pass look-back).
+// Then asm_copy writes the output in 16 KB chunks of the call's output: one
+// warp finds the chunk's members (32-ary warp search over the positions) and
+// stages their source bytes in shared memory with cp.async.bulk (two stages,
+// mbarrier completion, bounded waits) while all warps turn the previous chunk
+// into aligned 16-byte stores; source and destination alignments may differ
+// arbitrarily.
 #include <algorithm>
 
 #include "ro_internal.h"
@@ -31,13 +29,7 @@ namespace ro {
 constexpr int TS_ASM_COPY = 5;
 
 __device__ __forceinline__ uint64_t asm_list_count(const AssembleArgs& a, bool* over) {
-  uint64_t n;
-  if (a.list_is_commit)
-    n = a.ds->cm_n_done;
-  else if (a.d_n)
-    n = *a.d_n;
-  else
-    n = a.n_host;
+  const uint64_t n = a.d_n ? *a.d_n : a.n_host;
   *over = n > a.n_host;
   return n > a.n_host ? a.n_host : n;
 }
@@ -56,6 +48,7 @@ __device__ __forceinline__ uint32_t last_le_u(const V* v, uint32_t lo, uint32_t 
 
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a) {
+  wait_predecessor();
   __shared__ unsigned long long s_scan[33];
   __shared__ uint32_t s_tile;
   __shared__ unsigned long long s_prefix;
@@ -76,7 +69,7 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
     if (blockIdx.x == 0 && threadIdx.x == 0) {
       a.mb[0] = 0;
       ds->as_M = 0;
-      ds->as_n = 0;
+      ds->as_hdr.n = 0;
     }
     return;
   }
@@ -135,7 +128,7 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
     if (tile == n_tiles - 1 && threadIdx.x == AP_THREADS - 1) {
       a.mb[n] = (uint32_t)run;
       ds->as_M = run;
-      ds->as_n = n;
+      ds->as_hdr.n = n;
       if (run > a.member_cap) {
         ds->as_err = 1u;
         atomicOr(&ds->err, ERR_CAPACITY);
@@ -151,52 +144,31 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
 
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a) {
+  wait_predecessor();
   __shared__ uint32_t s_mb[AM_SMEM_CAP];
   __shared__ uint32_t s_coff[AM_SMEM_CAP];
   __shared__ Pair64 s_scan[33];
   __shared__ uint32_t s_tile;
   __shared__ Pair64 s_prefix;
   DevScalars* ds = a.ds;
-  uint64_t n, M;
-  if (a.list_is_commit) {
-    n = ds->cm_n_done;
-    M = ds->cm_M;
-    if (n > a.n_host) {   // the commit completed more parents than the outputs hold
-      if (blockIdx.x == 0 && threadIdx.x == 0) {
-        ds->as_err = 1u;
-        atomicOr(&ds->err, ERR_CAPACITY);
-      }
-      return;
-    }
-    if (blockIdx.x == 0 && threadIdx.x == 0) ds->as_n = n;
-  } else {
-    if (ds->as_err) return;   // nothing claimed
-    n = ds->as_n;
-    M = ds->as_M;
-  }
-  const uint64_t base = a.cursor ? *a.cursor : 0ull;
-  const uint64_t out_addr = (uint64_t)(uintptr_t)a.out;
-  const uint64_t origin = (out_addr + base) & ~15ull;
+  const PlanBufs& pl = a.plan;
+  if (ds->as_err) return;   // nothing claimed
+  const uint64_t n = ds->as_hdr.n, M = ds->as_M;
   const uint64_t n_tiles = ceil_div(M, AM_TILE);
 
-  if (M == 0) {
+  if (M == 0) {   // nothing to gather: every listed parent starts at 0
     if (blockIdx.x == 0) {
-      for (uint64_t i = threadIdx.x; i <= n; i += blockDim.x) a.out_off[i] = base;
+      for (uint64_t i = threadIdx.x; i <= n; i += blockDim.x) pl.off[i] = 0;
       if (threadIdx.x == 0) {
-        ds->as_bytes = 0;
-        ds->as_Mnz = 0;
-        ds->as_base = base;
-        if (base > a.out_cap) {
-          ds->as_err = 1u;
-          atomicOr(&ds->err, ERR_CAPACITY);
-        }
+        pl.hdr->bytes = 0;
+        pl.hdr->nnz = 0;
       }
     }
     return;
   }
-
   const uint32_t n_part = participants(n_tiles);
   if (blockIdx.x >= n_part) return;
+
   for (;;) {
     if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_ASM_MEMBERS]);
     __syncthreads();
@@ -241,10 +213,7 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
         uint64_t lo = i_lo, hi = i_hi + 1;
         while (hi - lo > 1) {
           const uint64_t mid = lo + ((hi - lo) >> 1);
-          if (a.mb[mid] <= g)
-            lo = mid;
-          else
-            hi = mid;
+          if (a.mb[mid] <= g) lo = mid; else hi = mid;
         }
         i = lo;
         mbi = a.mb[lo];
@@ -275,44 +244,34 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
     for (int k = 0; k < AM_ITEMS; ++k) {
       const uint64_t g = gt + k;
       if (g >= M) break;
-      const uint64_t pos = base + run.a;
+      const uint64_t pos = run.a;
       if (first[k]) {
         // the parent starts here, and so do the member-less parents listed just before it
-        a.out_off[par[k]] = pos;
+        pl.off[par[k]] = pos;
         for (int64_t q = (int64_t)par[k] - 1; q >= 0; --q) {
           const uint32_t mbq = (staged && (uint64_t)q >= i_lo) ? s_mb[q - i_lo] : a.mb[q];
           if (mbq != g) break;
-          a.out_off[q] = pos;
+          pl.off[q] = pos;
         }
       }
       if (contrib[k]) {
         const uint64_t j = run.b;
         if (j < a.member_cap) {
-          a.cpos[j] = pos;
-          a.csrc[j] = src[k];
+          pl.cpos[j] = pos;
+          pl.csrc[j] = src[k];
         }
-        const uint64_t A = out_addr + pos, E = A + contrib[k];
-        if (j == 0 && a.ctfp_cap) a.ctfp[0] = 0u;
-        for (uint64_t b = ceil_div(A - origin, AC_CHUNK); origin + b * AC_CHUNK < E && b < a.ctfp_cap; ++b)
-          a.ctfp[b] = (uint32_t)j;
         run.b += 1;
         run.a += contrib[k];
       }
     }
     if (tile == n_tiles - 1 && threadIdx.x == AM_THREADS - 1) {
-      const uint64_t end = base + run.a;
-      a.out_off[n] = end;
+      pl.off[n] = run.a;
       for (int64_t q = (int64_t)n - 1; q >= 0; --q) {
         if ((uint64_t)a.mb[q] != M) break;   // member-less parents at the very end
-        a.out_off[q] = end;
+        pl.off[q] = run.a;
       }
-      ds->as_bytes = run.a;
-      ds->as_Mnz = run.b;
-      ds->as_base = base;
-      if (end > a.out_cap || ceil_div(out_addr + end - origin, AC_CHUNK) > a.ctfp_cap) {
-        ds->as_err = 1u;
-        atomicOr(&ds->err, ERR_CAPACITY);
-      }
+      pl.hdr->bytes = run.a;
+      pl.hdr->nnz = run.b;
     }
     __syncthreads();
   }
@@ -471,13 +430,17 @@ __device__ __forceinline__ bool stage_wait(uint64_t* bar, uint32_t parity, uint3
 
 // One pipeline stage: the source bytes of one 16 KB output chunk, laid out
 // piece by piece (each piece = the part of one member inside the chunk, read
-// as the aligned 16-byte blocks that hold it).
+// as the aligned 16-byte blocks that hold it).  Offsets inside the chunk are
+// taken from wbase, the aligned word at or before the chunk's first byte.
 struct CopyStage {
   uint32_t np;                    // pieces staged, or AC_FALLBACK
-  uint32_t vbeg, vend;            // valid output bytes of the chunk, chunk-relative
+  uint32_t vbeg, vend;            // the chunk's bytes, relative to wbase
   uint32_t pad;
-  uint32_t pstart[AC_PIECES + 1]; // chunk-relative output start of each piece (+ end)
-  int32_t qbase[AC_PIECES];       // buffer offset of output byte 0 of the chunk, per piece
+  unsigned long long wbase;       // absolute address of the chunk's first word
+  unsigned long long rel_s, rel_e;   // the chunk's bytes, relative to the call's output
+  unsigned long long j_lo;        // first member of the chunk
+  uint32_t pstart[AC_PIECES + 1]; // output start of each piece (+ end), relative to wbase
+  int32_t qbase[AC_PIECES];       // buffer offset of output byte wbase, per piece
   __align__(16) unsigned char buf[AC_BUF + 64];
 };
 constexpr uint32_t AC_FALLBACK = 0xFFFFFFFFu;
@@ -486,42 +449,64 @@ size_t asm_copy_smem() { return 2 * sizeof(CopyStage); }
 
 struct CopyCtx {
   const AssembleArgs* a;
-  uint64_t out_addr, start, end, origin, n_chunks, Mnz, end_rel;
+  const uint64_t* cpos;
+  const uint64_t* csrc;
+  uint64_t out_base;   // absolute address of the call's first output byte
+  uint64_t S, Mnz;
 };
 
 __device__ __forceinline__ uint64_t cpos_at(const CopyCtx& c, uint64_t j) {
-  return j < c.Mnz ? c.a->cpos[j] : c.end_rel;
+  return j < c.Mnz ? c.cpos[j] : c.S;
 }
 
-// Warp 0 stages chunk b: piece table, then one bulk copy per piece.
-__device__ void stage_chunk(const CopyCtx& c, uint64_t b, CopyStage* st, uint64_t* bar, int lane) {
-  const AssembleArgs& a = *c.a;
-  const uint64_t cs = c.origin + b * AC_CHUNK;
-  const uint64_t ce = cs + AC_CHUNK;
-  const uint64_t vb = cs > c.start ? cs : c.start;
-  const uint64_t ve = ce < c.end ? ce : c.end;
-  const uint64_t j_lo = a.ctfp[b];
-  const uint64_t j_hi = (b + 1 < c.n_chunks) ? a.ctfp[b + 1] : c.Mnz - 1;
-  const uint64_t np = j_hi - j_lo + 1;
-  if (lane == 0) {
-    st->vbeg = (uint32_t)(vb - cs);
-    st->vend = (uint32_t)(ve - cs);
+// Largest j in [0, n) with pos[j] <= x (pos[0] = 0 <= x): 32 probes a round.
+__device__ __forceinline__ uint64_t warp_search(const uint64_t* pos, uint64_t n, uint64_t x, int lane) {
+  uint64_t lo = 0, hi = n;
+  while (hi - lo > 1) {
+    const uint64_t step = (hi - lo + 31) / 32;
+    const uint64_t probe = lo + step * (uint64_t)lane;
+    const bool le = probe < hi && pos[probe] <= x;
+    const unsigned m = __ballot_sync(0xffffffffu, le);
+    const uint64_t last = (uint64_t)(31 - __clz((int)m));
+    lo = lo + step * last;
+    hi = (lo + step < hi) ? lo + step : hi;
   }
+  return lo;
+}
+
+// Warp 0 stages chunk k: finds its members, builds the piece table and issues
+// one bulk copy per piece.
+__device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_t* bar, int lane) {
+  const uint64_t rs = k * AC_CHUNK;
+  const uint64_t re = (rs + AC_CHUNK < c.S) ? rs + AC_CHUNK : c.S;
+  const uint64_t j_lo = warp_search(c.cpos, c.Mnz, rs, lane);
+  const uint64_t j_hi = warp_search(c.cpos, c.Mnz, re - 1, lane);
+  const uint64_t np = j_hi - j_lo + 1;
+  const uint64_t wbase = (c.out_base + rs) & ~15ull;
+  if (lane == 0) {
+    st->wbase = wbase;
+    st->rel_s = rs;
+    st->rel_e = re;
+    st->j_lo = j_lo;
+    st->vbeg = (uint32_t)(c.out_base + rs - wbase);
+    st->vend = (uint32_t)(c.out_base + re - wbase);
+  }
+  const uint64_t arena = (uint64_t)(uintptr_t)c.a->arena;
   bool fits = np <= AC_PIECES;
-  uint32_t roff = 0;   // running buffer offset (uniform)
+  uint32_t roff = 0;   // running buffer offset (warp-uniform)
   if (fits) {
     for (uint64_t g = 0; g < np; g += 32) {
       const uint64_t i = g + lane;
       uint32_t size = 0, sh = 0, ps = 0;
       if (i < np) {
         const uint64_t j = j_lo + i;
-        const uint64_t p0 = c.out_addr + a.cpos[j], p1 = c.out_addr + cpos_at(c, j + 1);
-        const uint64_t ob = p0 > vb ? p0 : vb, oe = p1 < ve ? p1 : ve;
-        const uint64_t src = (uint64_t)(uintptr_t)a.arena + a.csrc[j] + (ob - p0);
+        const uint64_t p0 = c.cpos[j], p1 = cpos_at(c, j + 1);
+        const uint64_t ob = p0 > rs ? p0 : rs, oe = p1 < re ? p1 : re;
+        const uint64_t src = arena + c.csrc[j] + (ob - p0);
         const uint64_t a0 = src & ~15ull, a1 = (src + (oe - ob) + 15) & ~15ull;
         size = (uint32_t)(a1 - a0);
         sh = (uint32_t)(src & 15u);
-        ps = (uint32_t)(ob - cs);
+        ps = (uint32_t)(c.out_base + ob - wbase);
       }
       uint32_t inc = size;
 #pragma unroll
@@ -548,7 +533,7 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t b, CopyStage* st, uint64_
   }
   if (lane == 0) {
     st->np = (uint32_t)np;
-    st->pstart[np] = (uint32_t)(ve - cs);
+    st->pstart[np] = (uint32_t)(c.out_base + re - wbase);
   }
   __syncwarp();
   fence_proxy_async_smem();   // earlier generic reads of this buffer before async writes
@@ -556,10 +541,10 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t b, CopyStage* st, uint64_
   __syncwarp();
   for (uint64_t i = lane; i < np; i += 32) {
     const uint64_t j = j_lo + i;
-    const uint64_t p0 = c.out_addr + a.cpos[j];
-    const uint64_t ob = cs + st->pstart[i];
-    const uint64_t oe = cs + st->pstart[i + 1];
-    const uint64_t src = (uint64_t)(uintptr_t)a.arena + a.csrc[j] + (ob - p0);
+    const uint64_t p0 = c.cpos[j];
+    const uint64_t ob = wbase + st->pstart[i] - c.out_base;      // relative
+    const uint64_t oe = wbase + st->pstart[i + 1] - c.out_base;
+    const uint64_t src = arena + c.csrc[j] + (ob - p0);
     const uint64_t a0 = src & ~15ull, a1 = (src + (oe - ob) + 15) & ~15ull;
     const uint32_t off = (uint32_t)(st->qbase[i] + (int32_t)st->pstart[i]) - (uint32_t)(src & 15u);
     if (a1 > a0)   // a member that starts exactly at the chunk's end stages nothing
@@ -567,18 +552,18 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t b, CopyStage* st, uint64_
   }
 }
 
-// All threads: write chunk b from its staged pieces.
-__device__ void emit_chunk(const CopyCtx& c, uint64_t b, const CopyStage* st) {
-  const uint64_t cs = c.origin + b * AC_CHUNK;
+// All threads: write the staged chunk as aligned 16-byte words.
+__device__ void emit_chunk(const CopyStage* st) {
   const uint32_t np = st->np;
   const uint32_t vbeg = st->vbeg, vend = st->vend;
+  const uint64_t wbase = st->wbase;
   const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll 1
-  for (uint32_t wr = threadIdx.x * 16u; wr < (uint32_t)AC_CHUNK; wr += AC_THREADS * 16u) {
+  for (uint32_t wr = threadIdx.x * 16u; wr < vend; wr += AC_THREADS * 16u) {
     const uint32_t vlo = wr > vbeg ? wr : vbeg;
     const uint32_t vhi = (wr + 16u < vend) ? wr + 16u : vend;
     if (vlo >= vhi) continue;
-    // piece holding chunk byte vlo
+    // piece holding byte vlo
     uint32_t lo_i = 0, hi_i = np;
     while (hi_i - lo_i > 1) {
       const uint32_t mid = (lo_i + hi_i) >> 1;
@@ -602,10 +587,11 @@ __device__ void emit_chunk(const CopyCtx& c, uint64_t b, const CopyStage* st) {
       lo = hi;
       ++i;
     }
-    const uint64_t W = cs + wr;
+    const uint64_t W = wbase + wr;
     if (vlo == wr && vhi == wr + 16u) {
       *reinterpret_cast<uint4*>((uintptr_t)W) = acc;
     } else {
+      // the chunk's first or last word: only its own bytes
       const uint32_t vv[4] = {acc.x, acc.y, acc.z, acc.w};
 #pragma unroll
       for (int t = 0; t < 16; ++t)
@@ -615,62 +601,68 @@ __device__ void emit_chunk(const CopyCtx& c, uint64_t b, const CopyStage* st) {
   }
 }
 
-// Chunk b copied from global memory by warps (pieces did not fit a stage).
-__device__ void emit_chunk_direct(const CopyCtx& c, uint64_t b) {
-  const AssembleArgs& a = *c.a;
+// A chunk whose pieces do not fit a stage: warps copy slices straight from
+// global memory.
+__device__ void emit_chunk_direct(const CopyCtx& c, const CopyStage* st) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   constexpr uint64_t SLICE = AC_CHUNK / (AC_THREADS / 32);
-  const uint64_t cs = c.origin + b * AC_CHUNK;
-  const uint64_t j_lo = a.ctfp[b];
-  const uint64_t j_hi = (b + 1 < c.n_chunks) ? a.ctfp[b + 1] : c.Mnz - 1;
-  const uint64_t sl = cs + (uint64_t)warp * SLICE, sh = sl + SLICE;
-  uint64_t ra = (sl > c.start ? sl : c.start) - c.out_addr;
-  const uint64_t rb = (sh < c.end ? sh : c.end) - c.out_addr;
+  const uint64_t rs = st->rel_s, re = st->rel_e;
+  uint64_t ra = rs + (uint64_t)warp * SLICE;
+  const uint64_t rb = (ra + SLICE < re) ? ra + SLICE : re;
   if (ra >= rb) return;
-  uint64_t lo = j_lo, hi = j_hi + 1;
-  while (hi - lo > 1) {
-    const uint64_t mid = lo + ((hi - lo) >> 1);
-    if (a.cpos[mid] <= ra) lo = mid; else hi = mid;
-  }
-  for (uint64_t k = lo; ra < rb; ++k) {
-    const uint64_t pk = a.cpos[k], pn = cpos_at(c, k + 1);
+  uint64_t k = warp_search(c.cpos, c.Mnz, ra, lane);
+  for (; ra < rb; ++k) {
+    const uint64_t pk = c.cpos[k], pn = cpos_at(c, k + 1);
     const uint64_t e = pn < rb ? pn : rb;
-    warp_copy(a.out + ra, a.arena + a.csrc[k] + (ra - pk), e - ra, lane);
+    warp_copy(c.a->out + (c.out_base - (uint64_t)(uintptr_t)c.a->out) + ra,
+              c.a->arena + c.csrc[k] + (ra - pk), e - ra, lane);
     ra = e;
   }
 }
 
 __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a) {
+  wait_predecessor();
   extern __shared__ __align__(128) unsigned char ac_smem[];
   __shared__ __align__(8) uint64_t bars[2];
   CopyStage* stages = reinterpret_cast<CopyStage*>(ac_smem);
   DevScalars* ds = a.ds;
-  const bool failed = ds->as_err != 0u;
-  const uint64_t n = ds->as_n, S = ds->as_bytes, Mnz = ds->as_Mnz, base = ds->as_base;
+  const PlanHdr hdr = *a.plan.hdr;
+  const uint64_t n = hdr.n, S = hdr.bytes;
+  const uint64_t base = a.cursor ? *a.cursor : 0ull;
+  // conditions every CTA sees the same way
+  bool failed = ds->as_err != 0u;
+  const bool too_many = a.from_commit && n > a.n_host;   // outputs hold fewer parents
+  const bool too_big = base + S > a.out_cap;
+  if (!failed && (too_many || too_big)) {
+    failed = true;
+    if (threadIdx.x == 0) atomicOr(&ds->err, ERR_CAPACITY);
+  }
   CopyCtx c;
   c.a = &a;
-  c.out_addr = (uint64_t)(uintptr_t)a.out;
-  c.start = c.out_addr + base;
-  c.end = c.start + S;
-  c.origin = c.start & ~15ull;
-  c.n_chunks = (!failed && S) ? ceil_div(c.end - c.origin, AC_CHUNK) : 0;
-  c.Mnz = Mnz;
-  c.end_rel = base + S;
-  const uint64_t par_units = failed ? 0 : ceil_div(n, (uint64_t)AC_THREADS * 8);
-  uint64_t units = c.n_chunks > par_units ? c.n_chunks : par_units;
+  c.cpos = a.plan.cpos;
+  c.csrc = a.plan.csrc;
+  c.out_base = (uint64_t)(uintptr_t)a.out + base;
+  c.S = S;
+  c.Mnz = hdr.nnz;
+  const uint64_t n_chunks = (!failed && S) ? ceil_div(S, AC_CHUNK) : 0;
+  const uint64_t par_units = failed ? 0 : ceil_div(n + 1, (uint64_t)AC_THREADS * 8);
+  uint64_t units = n_chunks > par_units ? n_chunks : par_units;
   if (units == 0) units = 1;   // one CTA still finishes the call
   const uint32_t n_part = participants(units);
   if (blockIdx.x >= n_part) return;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   if (!failed) {
-    // per-parent outputs that need the whole scan: status (plan lists) and lengths
-    if (a.out_len || a.plan_status) {
+    // per-parent outputs: status (commit plans), offsets, lengths
+    {
       const uint64_t stride = (uint64_t)n_part * blockDim.x;
-      for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
-        if (a.plan_status) a.status[i] = a.plan_status[i];
+      for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i <= n; i += stride) {
+        const uint64_t o = a.plan.off[i];
+        a.out_off[i] = base + o;
+        if (i == n) break;
+        if (a.st_src) a.status[i] = a.st_src[i];
         if (a.out_len) {
-          const uint64_t len = a.out_off[i + 1] - a.out_off[i];
+          const uint64_t len = a.plan.off[i + 1] - o;
           if (len > 0xFFFFFFFFull) atomicOr(&ds->err, ERR_OVERFLOW);
           a.out_len[i] = (uint32_t)len;
         }
@@ -685,16 +677,16 @@ __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a)
     uint32_t phase[2] = {0u, 0u};
     bool pending[2] = {false, false};
     bool ok = true;
-    uint64_t b = blockIdx.x;
-    if (b < c.n_chunks) {
-      if (warp == 0) stage_chunk(c, b, &stages[0], &bars[0], lane);
+    uint64_t k = blockIdx.x;
+    if (k < n_chunks) {
+      if (warp == 0) stage_chunk(c, k, &stages[0], &bars[0], lane);
       pending[0] = true;
     }
-    for (uint32_t it = 0; b < c.n_chunks && ok; b += n_part, ++it) {
+    for (uint32_t it = 0; k < n_chunks && ok; k += n_part, ++it) {
       const uint32_t s = it & 1u;
-      const uint64_t bn = b + n_part;
-      if (bn < c.n_chunks) {   // next chunk's loads overlap this chunk's writes
-        if (warp == 0) stage_chunk(c, bn, &stages[s ^ 1u], &bars[s ^ 1u], lane);
+      const uint64_t kn = k + n_part;
+      if (kn < n_chunks) {   // next chunk's loads overlap this chunk's writes
+        if (warp == 0) stage_chunk(c, kn, &stages[s ^ 1u], &bars[s ^ 1u], lane);
         pending[s ^ 1u] = true;
       }
       ok = stage_wait(&bars[s], phase[s], &ds->err);
@@ -702,9 +694,9 @@ __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a)
       pending[s] = false;
       if (ok) {
         if (stages[s].np == AC_FALLBACK)
-          emit_chunk_direct(c, b);
+          emit_chunk_direct(c, &stages[s]);
         else
-          emit_chunk(c, b, &stages[s]);
+          emit_chunk(&stages[s]);
       }
       __syncthreads();
     }
@@ -717,6 +709,7 @@ __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a)
     if (atomicAdd(&ds->exit_ctr[TS_ASM_COPY], 1u) == n_part - 1) {
       if (!failed && a.cursor) *a.cursor = base + S;
       if (a.out_bytes) *a.out_bytes = S;
+      ds->as_bytes = S;
       ds->as_err = 0u;
       ds->exit_ctr[TS_ASM_COPY] = 0u;
       __threadfence();
@@ -725,13 +718,13 @@ __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a)
 }
 
 void launch_assemble(const LaunchCfg& L, const AssembleArgs& a) {
-  if (!a.list_is_commit) {
+  if (!a.from_commit) {
     const uint64_t tiles = ceil_div(a.n_host, (uint64_t)AP_THREADS * AP_ITEMS);
     const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(tiles, (uint64_t)L.grid_aparents));
-    RO_LAUNCH(L, K_APARENTS, (asm_parents_kernel<<<grid, AP_THREADS, 0, L.stream>>>(a)));
+    launch_k(L, K_APARENTS, asm_parents_kernel, grid, AP_THREADS, 0, a);
+    launch_k(L, K_AMEMBERS, asm_members_kernel, L.grid_amembers, AM_THREADS, 0, a);
   }
-  RO_LAUNCH(L, K_AMEMBERS, (asm_members_kernel<<<L.grid_amembers, AM_THREADS, 0, L.stream>>>(a)));
-  RO_LAUNCH(L, K_ACOPY, (asm_copy_kernel<<<L.grid_acopy, AC_THREADS, asm_copy_smem(), L.stream>>>(a)));
+  launch_k(L, K_ACOPY, asm_copy_kernel, L.grid_acopy, AC_THREADS, asm_copy_smem(), a);
 }
 
 // opt in to the copy kernel's dynamic shared memory (two pipeline stages)

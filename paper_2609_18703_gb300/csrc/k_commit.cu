@@ -10,12 +10,18 @@
 //                 hot parent sees one atomic per warp.  The add that takes
 //                 `remaining` to zero completes the parent and sets its bit in
 //                 a completion bitmap.
+//                 That add also tells whether a member Failed or was
+//                 Suppressed, so the same thread records how many members the
+//                 parent will gather (0 if Suppressed).
 // commit_finish   turns the bitmap into the ascending list of completed
 //                 parents (popcount + single-pass scan over bitmap words) and
-//                 clears it.  When the scatter saw two reports for one Grain
-//                 in the same call (rare), CTA 0 first makes the lowest-index
-//                 report the accepted one, so the result equals applying the
-//                 reports one by one in array order.
+//                 clears it, then plans their assembly: per parent its
+//                 relative output offset, per contributing member its
+//                 relative position and arena offset (a second single-pass
+//                 scan).  When the scatter saw two reports for one Grain in
+//                 the same call (rare), the first CTA in orders them first, so
+//                 the result equals applying the reports one by one in array
+//                 order.
 #include <algorithm>
 
 #include "ro_internal.h"
@@ -36,6 +42,7 @@ __device__ __forceinline__ uint64_t commit_count(const CommitArgs& a) {
 }
 
 __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a) {
+  wait_predecessor();
   __shared__ unsigned long long s_cnt[6];
   DevScalars* ds = a.ds;
   if (threadIdx.x < 6) s_cnt[threadIdx.x] = 0;
@@ -63,6 +70,7 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
       if (c >= a.N || !valid_state || !in_bounds) {
         v = V_INVALID;
       } else {
+        const uint32_t par = a.rec[c].parent;   // immutable: read alongside the fence
         // Eq. (3): accept iff IN-FLIGHT at the report's generation
         const uint32_t want = ph_make(PH_INFLIGHT, g);
         uint32_t cur;
@@ -81,7 +89,7 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
           atomicOr((unsigned long long*)&rc->w,
                    (unsigned long long)((present ? (o & W_OFF_MASK) : 0ull) |
                                         ((uint64_t)s << W_STATE_SHIFT)));
-          p = rc->parent;
+          p = par;
           bad = (s == ST_FAILED || s == ST_SUPPRESSED);
         } else if ((cur & 3u) == PH_WAITING || (cur & 3u) == PH_READY) {
           v = V_NOT_INFLIGHT;
@@ -106,7 +114,11 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
         const unsigned long long delta =
             ((unsigned long long)n_bad << 32) - (unsigned long long)n_tot;
         const unsigned long long old = atomicAdd(a.pw + p, delta);
-        if ((uint32_t)old == n_tot) atomicOr(a.bitmap + (p >> 5), 1u << (p & 31));
+        if ((uint32_t)old == n_tot) {   // the last members: the parent is complete
+          const uint32_t m = (pw_bad(old) + n_bad) ? 0u : (uint32_t)(a.offsets[p + 1] - a.offsets[p]);
+          a.pm[p] = m;
+          atomicOr(a.bitmap + (p >> 5), 1u << (p & 31));
+        }
       }
     }
     if (v < 6) cnt[v == V_DUP_CANDIDATE ? 5 : v] += 1;
@@ -185,46 +197,82 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
       rc->len = present ? a.len[r] : 0u;
       rc->w = keep | (present ? (a.off[r] & W_OFF_MASK) : 0ull) | ((uint64_t)s << W_STATE_SHIFT);
       if (v == V_WIN_CAND && bad) atomicAdd(a.pw + p, 1ull << 32);
-      a.code[r] = V_ACCEPT;
     } else {
       if (v == V_LOSE_SEALER && bad) atomicAdd(a.pw + p, ~((1ull << 32) - 1));   // -(1 << 32)
-      a.code[r] = V_DUPLICATE;
       atomicAdd(&s_dups, 1ull);
     }
+  }
+  __syncthreads();
+  // E: a parent whose outcome class moved and that is complete gets its
+  //    member count to gather redone; then the verdicts become final
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    const uint8_t v = a.code[r];
+    if (v < V_WIN_SEALER || v > V_LOSE_CAND) continue;
+    const uint32_t p = a.rec[a.child[r]].parent;
+    const unsigned long long pv = __ldcg(a.pw + p);
+    if (pw_remaining(pv) == 0u) {
+      const uint32_t m = pw_bad(pv) ? 0u : (uint32_t)(a.offsets[p + 1] - a.offsets[p]);
+      atomicExch(a.pm + p, m);
+    }
+    a.code[r] = (v == V_WIN_SEALER || v == V_WIN_CAND) ? V_ACCEPT : V_DUPLICATE;
   }
   __syncthreads();
   if (threadIdx.x == 0) atomicAdd(&ds->stats[4], s_dups);
   __syncthreads();
 }
 
-__device__ __forceinline__ uint32_t plan_members(const CommitArgs& a, uint32_t p, uint8_t* st) {
-  const unsigned long long v = __ldcg(a.pw + p);
-  if (pw_bad(v) != 0u) {
-    *st = ST_SUPPRESSED;
-    return 0u;
+// Warp `lane`'s share of parent p's members, MB_ITEMS consecutive records
+// per lane per step: calls f(k, contrib, src) for every member k of the step
+// in order (contrib 0 for members that add no bytes).
+template <class F>
+__device__ __forceinline__ void for_members(const CommitArgs& a, uint64_t c0, uint64_t m, int lane,
+                                            F&& f) {
+  for (uint64_t g = 0; g < m; g += 32 * MB_ITEMS) {
+    uint32_t len[MB_ITEMS];
+    uint64_t src[MB_ITEMS];
+#pragma unroll
+    for (int t = 0; t < MB_ITEMS; ++t) {
+      const uint64_t k = g + (uint64_t)lane * MB_ITEMS + t;
+      len[t] = 0;
+      src[t] = 0;
+      if (k < m) {
+        const Rec r = a.rec[c0 + k];
+        if (w_state(r.w) == ST_PRESENT) {
+          len[t] = r.len;
+          src[t] = w_off(r.w);
+        }
+      }
+    }
+    f(g, len, src);
   }
-  *st = ST_PRESENT;
-  return (uint32_t)(a.offsets[p + 1] - a.offsets[p]);
 }
 
-// Completed-parent list, ascending (popcount + single-pass scan over bitmap
-// words), plus the assembly plan of those parents: outcome, members to
-// gather and member bases, i.e. what ro_assemble's first pass would compute
-// for this list.
+// Completed-parent list, ascending (popcount + look-back scan over bitmap
+// words), and the assembly plan of those parents: each parent's outcome and
+// relative output offset, and for every member that contributes bytes its
+// relative output position and arena offset (a second look-back scan, of
+// (bytes, contributing members), in the same tile order).
 __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a) {
-  __shared__ Pair64 s_scan[33];
+  wait_predecessor();
+  __shared__ unsigned long long s_scan[33];
+  __shared__ Pair64 s_scan2[33];
   __shared__ uint32_t s_tile;
-  __shared__ Pair64 s_prefix;
+  __shared__ unsigned long long s_nb, s_ne;
+  __shared__ Pair64 s_base, s_carry;
   __shared__ uint32_t s_fix;
   DevScalars* ds = a.ds;
+  const PlanBufs& pl = a.plan;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr int N_WARPS = CF_THREADS / 32;
   const uint64_t n_words = ceil_div(a.P, 32);
-  const uint64_t TILE = (uint64_t)CF_THREADS * CF_WORDS;
-  const uint64_t n_tiles = ceil_div(n_words, TILE);
+  const uint64_t n_tiles = ceil_div(n_words, (uint64_t)CF_THREADS);
   if (n_tiles == 0) {
     if (blockIdx.x == 0 && threadIdx.x == 0) {
       ds->cm_n_done = 0;
-      ds->cm_M = 0;
-      a.plan_mb[0] = 0;
+      pl.hdr->n = 0;
+      pl.hdr->bytes = 0;
+      pl.hdr->nnz = 0;
+      pl.off[0] = 0;
       if (a.n_done_out) *a.n_done_out = 0;
     }
     return;
@@ -262,54 +310,134 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
     const uint32_t tile = s_tile;
     __syncthreads();
     if (tile >= n_tiles) break;
-    const uint64_t w0 = tile * TILE + (uint64_t)threadIdx.x * CF_WORDS;
-    uint32_t words[CF_WORDS];
-    Pair64 mine{0, 0};   // (completed parents, members to gather)
-#pragma unroll
-    for (int k = 0; k < CF_WORDS; ++k) {
-      words[k] = (w0 + k < n_words) ? a.bitmap[w0 + k] : 0u;
-      uint32_t bits = words[k];
-      mine.a += __popc(bits);
-      while (bits) {
-        const int b = __ffs(bits) - 1;
-        bits &= bits - 1;
-        uint8_t st;
-        mine.b += plan_members(a, (uint32_t)((w0 + k) * 32 + b), &st);
-      }
+
+    // ---- scan 1: completed parents of this tile's 256 bitmap words
+    const uint64_t w = (uint64_t)tile * CF_THREADS + threadIdx.x;
+    const uint32_t bits = (w < n_words) ? a.bitmap[w] : 0u;
+    unsigned long long total;
+    const unsigned long long excl = block_excl_scan((unsigned long long)__popc(bits), s_scan, &total);
+    if (threadIdx.x == 0) {
+      const unsigned long long nb =
+          lookback_exclusive(a.ts_done, tile, total, ds->epoch[TS_COMMIT], &ds->err);
+      s_nb = nb;
+      s_ne = nb + total;
     }
-    Pair64 total;
-    Pair64 excl = block_excl_scan_pair(mine, s_scan, &total);
-    if (threadIdx.x == 0)
-      s_prefix = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_COMMIT], &ds->err);
     __syncthreads();
-    Pair64 run = s_prefix + excl;
+    const unsigned long long nb = s_nb, ne = s_ne;
+    if (bits) {
+      unsigned long long i = nb + excl;
+      uint32_t b = bits;
+      while (b) {
+        const uint32_t parent = (uint32_t)(w * 32 + (__ffs(b) - 1));
+        b &= b - 1;
+        a.done_int[i] = parent;
+        if (a.done_user) a.done_user[i] = parent;
+        pl.status[i] = __ldcg(a.pm + parent) ? ST_PRESENT : ST_SUPPRESSED;
+        ++i;
+      }
+      a.bitmap[w] = 0u;
+    }
+    __syncthreads();
+
+    // ---- bytes and contributing members of each completed parent (a warp each)
+    for (unsigned long long i = nb + warp; i < ne; i += N_WARPS) {
+      const uint32_t p = a.done_int[i];
+      unsigned long long bytes = 0, nz = 0;
+      if (pl.status[i] == ST_PRESENT) {
+        const uint64_t c0 = a.offsets[p], m = a.offsets[p + 1] - c0;
+        for_members(a, c0, m, lane, [&](uint64_t, const uint32_t* len, const uint64_t*) {
 #pragma unroll
-    for (int k = 0; k < CF_WORDS; ++k) {
-      uint32_t bits = words[k];
-      if (!bits) continue;
-      a.bitmap[w0 + k] = 0u;
-      while (bits) {
-        const int b = __ffs(bits) - 1;
-        bits &= bits - 1;
-        const uint32_t parent = (uint32_t)((w0 + k) * 32 + b);
-        uint8_t st;
-        const uint32_t m = plan_members(a, parent, &st);
-        a.done_int[run.a] = parent;
-        if (a.done_user) a.done_user[run.a] = parent;
-        a.plan_status[run.a] = st;
-        a.plan_mb[run.a] = (uint32_t)run.b;
-        for (uint64_t t = ceil_div(run.b, AM_TILE); t * AM_TILE < run.b + m && t < a.plan_mtfp_cap; ++t)
-          a.plan_mtfp[t] = (uint32_t)run.a;
-        run.a += 1;
-        run.b += m;
+          for (int t = 0; t < MB_ITEMS; ++t) {
+            bytes += len[t];
+            nz += len[t] ? 1u : 0u;
+          }
+        });
+#pragma unroll
+        for (int d = 16; d > 0; d >>= 1) {
+          bytes += __shfl_down_sync(0xffffffffu, bytes, d);
+          nz += __shfl_down_sync(0xffffffffu, nz, d);
+        }
+      }
+      if (lane == 0) {
+        pl.pbytes[i] = bytes;
+        pl.pnz[i] = (uint32_t)nz;
       }
     }
-    if (tile == n_tiles - 1 && threadIdx.x == CF_THREADS - 1) {
-      ds->cm_n_done = run.a;
-      ds->cm_M = run.b;
-      a.plan_mb[run.a] = (uint32_t)run.b;
-      if (a.n_done_out) *a.n_done_out = run.a;
+    __syncthreads();
+
+    // ---- tile-local exclusive prefix of (bytes, contributing members)
+    if (threadIdx.x == 0) s_carry = Pair64{0, 0};
+    __syncthreads();
+    for (unsigned long long i0 = nb; i0 < ne; i0 += CF_THREADS) {
+      const unsigned long long i = i0 + threadIdx.x;
+      const Pair64 v = (i < ne) ? Pair64{pl.pbytes[i], pl.pnz[i]} : Pair64{0, 0};
+      Pair64 tot;
+      const Pair64 ex = block_excl_scan_pair(v, s_scan2, &tot);
+      const Pair64 carry = s_carry;
+      if (i < ne) {
+        pl.pbytes[i] = carry.a + ex.a;
+        pl.pnz[i] = (uint32_t)(carry.b + ex.b);
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) s_carry = carry + tot;
+      __syncthreads();
     }
+    if (threadIdx.x == 0)
+      s_base = lookback_exclusive(a.ts_bytes, tile, s_carry, ds->epoch[TS_COMMIT], &ds->err);
+    __syncthreads();
+    const Pair64 base = s_base;
+
+    // ---- relative offsets and member positions
+    for (unsigned long long i = nb + warp; i < ne; i += N_WARPS) {
+      const uint64_t off = base.a + pl.pbytes[i];
+      uint64_t nzb = base.b + pl.pnz[i];
+      if (lane == 0) pl.off[i] = off;
+      if (pl.status[i] != ST_PRESENT) continue;
+      const uint32_t p = a.done_int[i];
+      const uint64_t c0 = a.offsets[p], m = a.offsets[p + 1] - c0;
+      uint64_t run = off;
+      for_members(a, c0, m, lane, [&](uint64_t, const uint32_t* len, const uint64_t* src) {
+        unsigned long long mine = 0, mine_nz = 0;
+#pragma unroll
+        for (int t = 0; t < MB_ITEMS; ++t) {
+          mine += len[t];
+          mine_nz += len[t] ? 1u : 0u;
+        }
+        unsigned long long inc = mine, inc_nz = mine_nz;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+          const unsigned long long u = __shfl_up_sync(0xffffffffu, inc, d);
+          const unsigned long long un = __shfl_up_sync(0xffffffffu, inc_nz, d);
+          if (lane >= d) {
+            inc += u;
+            inc_nz += un;
+          }
+        }
+        uint64_t pos = run + (inc - mine);
+        uint64_t j = nzb + (inc_nz - mine_nz);
+#pragma unroll
+        for (int t = 0; t < MB_ITEMS; ++t) {
+          if (len[t]) {
+            pl.cpos[j] = pos;
+            pl.csrc[j] = src[t];
+            ++j;
+            pos += len[t];
+          }
+        }
+        run += __shfl_sync(0xffffffffu, inc, 31);
+        nzb += __shfl_sync(0xffffffffu, inc_nz, 31);
+      });
+    }
+    if (tile == n_tiles - 1 && threadIdx.x == 0) {
+      const Pair64 end = base + s_carry;
+      ds->cm_n_done = ne;
+      pl.hdr->n = ne;
+      pl.hdr->bytes = end.a;
+      pl.hdr->nnz = end.b;
+      pl.off[ne] = end.a;
+      if (a.n_done_out) *a.n_done_out = ne;
+    }
+    __syncthreads();
   }
   if (threadIdx.x == 0) {
     __threadfence();
@@ -330,10 +458,10 @@ void launch_commit(const LaunchCfg& L, const CommitArgs& a) {
   const int grid =
       (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(warps, CM_THREADS / 32),
                                                     (uint64_t)L.grid_commit));
-  RO_LAUNCH(L, K_COMMIT, (commit_scatter_kernel<<<grid, CM_THREADS, 0, L.stream>>>(a)));
-  const uint64_t n_tiles = ceil_div(ceil_div(a.P, 32), (uint64_t)CF_THREADS * CF_WORDS);
+  launch_k(L, K_COMMIT, commit_scatter_kernel, grid, CM_THREADS, 0, a);
+  const uint64_t n_tiles = ceil_div(ceil_div(a.P, 32), (uint64_t)CF_THREADS);
   const int grid_f = (int)std::max<uint64_t>(1, std::min<uint64_t>(n_tiles, (uint64_t)L.grid_cfinish));
-  RO_LAUNCH(L, K_CFINISH, (commit_finish_kernel<<<grid_f, CF_THREADS, 0, L.stream>>>(a)));
+  launch_k(L, K_CFINISH, commit_finish_kernel, grid_f, CF_THREADS, 0, a);
 }
 
 const void* kernel_ptr_commit(int which) {

@@ -19,6 +19,7 @@
 namespace ro {
 
 __global__ void __launch_bounds__(EXP_THREADS) expand_scan_kernel(ExpandScanArgs a) {
+  wait_predecessor();
   __shared__ Pair64 s_scan[33];
   __shared__ uint32_t s_tile;
   __shared__ Pair64 s_prefix;
@@ -101,6 +102,7 @@ __device__ __forceinline__ uint32_t last_le(const V* v, uint32_t lo, uint32_t hi
 }
 
 __global__ void __launch_bounds__(FILL_THREADS) expand_fill_kernel(ExpandFillArgs a) {
+  wait_predecessor();
   __shared__ uint64_t s_off[FILL_SMEM_CAP];
   const uint64_t n_tiles = ceil_div(a.N, FILL_TILE);
   for (uint64_t t = blockIdx.x; t < n_tiles; t += gridDim.x) {
@@ -147,14 +149,14 @@ __global__ void __launch_bounds__(FILL_THREADS) expand_fill_kernel(ExpandFillArg
 }
 
 void launch_expand_scan(const LaunchCfg& L, const ExpandScanArgs& a) {
-  RO_LAUNCH(L, K_EXPAND_SCAN, (expand_scan_kernel<<<L.grid_expand_scan, EXP_THREADS, 0, L.stream>>>(a)));
+  launch_k(L, K_EXPAND_SCAN, expand_scan_kernel, L.grid_expand_scan, EXP_THREADS, 0, a);
 }
 
 void launch_expand_fill(const LaunchCfg& L, const ExpandFillArgs& a) {
   const uint64_t n_tiles = ceil_div(a.N, FILL_TILE);
   if (n_tiles == 0) return;
   const int grid = (int)std::min<uint64_t>(n_tiles, (uint64_t)L.grid_fill);
-  RO_LAUNCH(L, K_FILL, (expand_fill_kernel<<<grid, FILL_THREADS, 0, L.stream>>>(a)));
+  launch_k(L, K_FILL, expand_fill_kernel, grid, FILL_THREADS, 0, a);
 }
 
 const void* kernel_ptr_expand(int which) {

@@ -28,6 +28,7 @@ __device__ __forceinline__ bool call_ok(const ReadyArgs& a, uint64_t c) {
 }
 
 __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
+  wait_predecessor();
   __shared__ unsigned long long s_red[2][RB_THREADS / 32];
   DevScalars* ds = a.ds;
   unsigned long long kept = 0, bad = 0;
@@ -107,6 +108,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
 }
 
 __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) {
+  wait_predecessor();
   __shared__ unsigned long long s_scan[33];
   __shared__ uint32_t s_tile;
   __shared__ unsigned long long s_prefix;
@@ -195,8 +197,8 @@ void launch_ready(const LaunchCfg& L, const ReadyArgs& a) {
   const uint64_t per = (uint64_t)RB_THREADS;
   const int grid_count =
       (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(a.n_cand, per), (uint64_t)L.grid_rb));
-  RO_LAUNCH(L, K_RB_COUNT, (ready_count_kernel<<<grid_count, RB_THREADS, 0, L.stream>>>(a)));
-  RO_LAUNCH(L, K_RB_SCATTER, (ready_scatter_kernel<<<L.grid_rb, RB_THREADS, 0, L.stream>>>(a)));
+  launch_k(L, K_RB_COUNT, ready_count_kernel, grid_count, RB_THREADS, 0, a);
+  launch_k(L, K_RB_SCATTER, ready_scatter_kernel, L.grid_rb, RB_THREADS, 0, a);
 }
 
 const void* kernel_ptr_ready(int which) {

@@ -25,7 +25,8 @@ using namespace ro;
 namespace {
 
 constexpr int MAX_EXPANSIONS = 64;
-constexpr int N_TS = 6;   // tile-status slots (TS_* in ro_common.cuh)
+constexpr int N_TS = 8;   // tile-status slots (TS_* in ro_common.cuh)
+constexpr int TS_COMMIT_BYTES = 6;   // commit_finish's second scan (flags only; shares TS_COMMIT's epoch)
 
 struct DevBuf {
   void* p = nullptr;
@@ -39,8 +40,9 @@ struct QueueBufs {
 
 // Device buffers of one expansion slot, kept across ro_ctx_reset and reused.
 struct ExpSlot {
-  DevBuf offsets, pw, phase, rec, bitmap, done, tfp;
-  DevBuf plan_status, plan_mb, plan_mtfp;   // assembly plan of the latest commit
+  DevBuf offsets, pw, phase, rec, bitmap, done, tfp, pm;
+  // assembly plan of the latest commit
+  DevBuf plan_status, plan_off, plan_pbytes, plan_pnz, plan_cpos, plan_csrc, plan_hdr;
   std::vector<QueueBufs> queues;
 };
 
@@ -109,7 +111,7 @@ struct ro_ctx {
   std::vector<ExpSlot> slots;
   std::vector<Expansion> exps;
   TsBuf ts[N_TS];
-  DevBuf code, mb, mtfp, cpos, csrc, ctfp;
+  DevBuf code, mb, mtfp, cpos, csrc, as_off;
   Profiler prof;
   ro_status sticky = RO_OK;
   std::string err;
@@ -226,6 +228,18 @@ Expansion* get_exp(ro_ctx* c, int32_t xid) {
   return &c->exps[xid];
 }
 
+PlanBufs slot_plan(ExpSlot& S) {
+  PlanBufs pl;
+  pl.status = (uint8_t*)S.plan_status.p;
+  pl.off = (uint64_t*)S.plan_off.p;
+  pl.pbytes = (uint64_t*)S.plan_pbytes.p;
+  pl.pnz = (uint32_t*)S.plan_pnz.p;
+  pl.cpos = (uint64_t*)S.plan_cpos.p;
+  pl.csrc = (uint64_t*)S.plan_csrc.p;
+  pl.hdr = (PlanHdr*)S.plan_hdr.p;
+  return pl;
+}
+
 int grid_for(const void* k, int threads, int sms, int cap_per_sm, size_t dyn_smem = 0) {
   int per = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k, threads, dyn_smem) != cudaSuccess || per < 1) {
@@ -304,7 +318,8 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   };
   for (auto& s : c->slots) {
     fr(s.offsets); fr(s.pw); fr(s.phase); fr(s.rec); fr(s.bitmap); fr(s.done); fr(s.tfp);
-    fr(s.plan_status); fr(s.plan_mb); fr(s.plan_mtfp);
+    fr(s.pm); fr(s.plan_status); fr(s.plan_off); fr(s.plan_pbytes); fr(s.plan_pnz);
+    fr(s.plan_cpos); fr(s.plan_csrc); fr(s.plan_hdr);
     for (auto& q : s.queues) {
       fr(q.q);
       fr(q.state);
@@ -313,7 +328,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   for (auto& t : c->ts) {
     fr(t.flag); fr(t.agg); fr(t.inc);
   }
-  fr(c->code); fr(c->mb); fr(c->mtfp); fr(c->cpos); fr(c->csrc); fr(c->ctfp);
+  fr(c->code); fr(c->mb); fr(c->mtfp); fr(c->cpos); fr(c->csrc); fr(c->as_off);
   for (cudaEvent_t e : c->prof.pool) cudaEventDestroy(e);
   cudaFree(c->ds);
   cudaFreeHost(c->hs);
@@ -439,8 +454,13 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   RO_TRY(ensure(c, S.bitmap, ceil_div(P, 32) * sizeof(uint32_t), "completion bitmap"));
   RO_TRY(ensure(c, S.done, P * sizeof(uint32_t), "completed parents"));
   RO_TRY(ensure(c, S.plan_status, P, "assembly plan"));
-  RO_TRY(ensure(c, S.plan_mb, (P + 1) * sizeof(uint32_t), "assembly plan"));
-  RO_TRY(ensure(c, S.plan_mtfp, (ceil_div(N, AM_TILE) + 2) * sizeof(uint32_t), "assembly plan"));
+  RO_TRY(ensure(c, S.plan_off, (P + 1) * sizeof(uint64_t), "assembly plan"));
+  RO_TRY(ensure(c, S.plan_pbytes, P * sizeof(uint64_t), "assembly plan"));
+  RO_TRY(ensure(c, S.plan_pnz, P * sizeof(uint32_t), "assembly plan"));
+  RO_TRY(ensure(c, S.plan_cpos, N * sizeof(uint64_t), "assembly plan"));
+  RO_TRY(ensure(c, S.plan_csrc, N * sizeof(uint64_t), "assembly plan"));
+  RO_TRY(ensure(c, S.plan_hdr, sizeof(PlanHdr), "assembly plan"));
+  RO_TRY(ensure(c, S.pm, P * sizeof(uint32_t), "parent member counts"));
   cudaMemsetAsync(S.bitmap.p, 0, ceil_div(P, 32) * sizeof(uint32_t), c->stream);
   ExpandFillArgs fa{};
   fa.offsets = (const uint64_t*)S.offsets.p;
@@ -548,6 +568,7 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.rec = (Rec*)S.rec.p;
   ca.pw = (unsigned long long*)S.pw.p;
   ca.bitmap = (uint32_t*)S.bitmap.p;
+  ca.pm = (uint32_t*)S.pm.p;
   if (d_code) {
     ca.code = d_code;
   } else {
@@ -558,13 +579,11 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.done_int = (uint32_t*)S.done.p;
   ca.n_done_out = d_n_done;
   ca.offsets = (const uint64_t*)S.offsets.p;
-  ca.plan_status = (uint8_t*)S.plan_status.p;
-  ca.plan_mb = (uint32_t*)S.plan_mb.p;
-  ca.plan_mtfp = (uint32_t*)S.plan_mtfp.p;
-  ca.plan_mtfp_cap = ceil_div(x->N, AM_TILE) + 2;
+  ca.plan = slot_plan(S);
   ca.ds = c->ds;
-  RO_TRY(tile_status(c, TS_COMMIT, ceil_div(ceil_div(x->P, 32), (uint64_t)CF_THREADS * CF_WORDS),
-                     &ca.ts));
+  const uint64_t cf_tiles = ceil_div(ceil_div(x->P, 32), (uint64_t)CF_THREADS);
+  RO_TRY(tile_status(c, TS_COMMIT, cf_tiles, &ca.ts_done));
+  RO_TRY(tile_status(c, TS_COMMIT_BYTES, cf_tiles, &ca.ts_bytes));
   launch_commit(c->L, ca);
   RO_TRY(check_launch(c, "gather_commit"));
   x->committed = true;
@@ -595,20 +614,29 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   ExpSlot& S = c->slots[xid];
   const uint64_t member_cap = std::max<uint64_t>(x->N, 1);
   const uint64_t mtfp_cap = ceil_div(member_cap, AM_TILE) + 2;
-  const uint64_t ctfp_cap = ceil_div(out_cap + 32, AC_CHUNK) + 2;
+  AssembleArgs aa{};
+  aa.from_commit = d_parents ? 0 : 1;
   if (d_parents) {
     RO_TRY(ensure(c, c->mb, (n_parents + 1) * sizeof(uint32_t), "member bases"));
     RO_TRY(ensure(c, c->mtfp, mtfp_cap * sizeof(uint32_t), "member tiles"));
+    RO_TRY(ensure(c, c->as_off, (n_parents + 1) * sizeof(uint64_t), "assembly offsets"));
+    RO_TRY(ensure(c, c->cpos, member_cap * sizeof(uint64_t), "member positions"));
+    RO_TRY(ensure(c, c->csrc, member_cap * sizeof(uint64_t), "member sources"));
+    aa.plan.status = nullptr;
+    aa.plan.off = (uint64_t*)c->as_off.p;
+    aa.plan.pbytes = nullptr;
+    aa.plan.pnz = nullptr;
+    aa.plan.cpos = (uint64_t*)c->cpos.p;
+    aa.plan.csrc = (uint64_t*)c->csrc.p;
+    aa.plan.hdr = &c->ds->as_hdr;
+    aa.st_src = nullptr;
+  } else {
+    aa.plan = slot_plan(S);
+    aa.st_src = (const uint8_t*)S.plan_status.p;
   }
-  RO_TRY(ensure(c, c->cpos, member_cap * sizeof(uint64_t), "member positions"));
-  RO_TRY(ensure(c, c->csrc, member_cap * sizeof(uint64_t), "member sources"));
-  RO_TRY(ensure(c, c->ctfp, ctfp_cap * sizeof(uint32_t), "copy chunks"));
-  AssembleArgs aa{};
-  aa.list = d_parents ? d_parents : (const uint32_t*)S.done.p;
+  aa.list = d_parents;
   aa.n_host = n_parents;
   aa.d_n = d_parents ? d_n_parents : nullptr;
-  aa.list_is_commit = d_parents ? 0 : 1;
-  aa.plan_status = d_parents ? nullptr : (const uint8_t*)S.plan_status.p;
   aa.P = x->P;
   aa.N = x->N;
   aa.offsets = (const uint64_t*)S.offsets.p;
@@ -623,18 +651,16 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   aa.out_cap = out_cap;
   aa.cursor = d_out_cursor;
   aa.out_bytes = d_out_bytes;
-  aa.mb = d_parents ? (uint32_t*)c->mb.p : (uint32_t*)S.plan_mb.p;
-  aa.mtfp = d_parents ? (uint32_t*)c->mtfp.p : (uint32_t*)S.plan_mtfp.p;
+  aa.mb = (uint32_t*)c->mb.p;
+  aa.mtfp = (uint32_t*)c->mtfp.p;
   aa.mtfp_cap = mtfp_cap;
-  aa.cpos = (uint64_t*)c->cpos.p;
-  aa.csrc = (uint64_t*)c->csrc.p;
   aa.member_cap = member_cap;
-  aa.ctfp = (uint32_t*)c->ctfp.p;
-  aa.ctfp_cap = ctfp_cap;
   aa.ds = c->ds;
-  RO_TRY(tile_status(c, TS_ASM_PARENTS, ceil_div(n_parents, (uint64_t)AP_THREADS * AP_ITEMS),
-                     &aa.ts_parents));
-  RO_TRY(tile_status(c, TS_ASM_MEMBERS, ceil_div(member_cap, (uint64_t)AM_TILE), &aa.ts_members));
+  if (d_parents) {
+    RO_TRY(tile_status(c, TS_ASM_PARENTS, ceil_div(n_parents, (uint64_t)AP_THREADS * AP_ITEMS),
+                       &aa.ts_parents));
+    RO_TRY(tile_status(c, TS_ASM_MEMBERS, ceil_div(member_cap, (uint64_t)AM_TILE), &aa.ts_members));
+  }
   launch_assemble(c->L, aa);
   RO_TRY(check_launch(c, "assemble"));
   if (h_out_bytes) {

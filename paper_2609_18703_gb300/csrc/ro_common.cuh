@@ -69,6 +69,14 @@ enum : uint32_t {
   ERR_INVAL = 8u,
 };
 
+// Header of an assembly plan (see PlanBufs).
+struct PlanHdr {
+  unsigned long long n;      // listed parents
+  unsigned long long bytes;  // bytes to assemble
+  unsigned long long nnz;    // members that contribute bytes
+  unsigned long long pad;
+};
+
 // Counters and small results that kernels hand to later kernels and to the
 // host.  One instance per context, in device memory, mirrored to pinned host
 // memory when a call synchronises.
@@ -85,7 +93,9 @@ struct DevScalars {
   unsigned long long cm_n, cm_conflicts, cm_n_done, cm_M;
   uint32_t cm_fix_ticket, cm_fix_done;
   // ro_assemble
-  unsigned long long as_n, as_M, as_Mnz, as_bytes, as_base, as_origin;
+  PlanHdr as_hdr;                 // plan of an explicit list
+  unsigned long long as_M;        // members of an explicit list's Present parents
+  unsigned long long as_bytes;    // bytes of the latest assemble (host read-back)
   uint32_t as_err, pad1;
   // dynamic tile counters / exit tickets / scan epochs, one per look-back kernel
   uint32_t tile_ctr[8];
@@ -93,6 +103,12 @@ struct DevScalars {
   unsigned long long epoch[8];
 };
 enum TileSlot { TS_EXPAND = 0, TS_READY = 1, TS_COMMIT = 2, TS_ASM_PARENTS = 3, TS_ASM_MEMBERS = 4 };
+
+// Wait until the grid this launch depends on (programmatic dependent launch)
+// has completed and its memory is visible; a no-op without a dependency.
+__device__ __forceinline__ void wait_predecessor() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
 
 // ---- memory-order helpers --------------------------------------------------------
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {

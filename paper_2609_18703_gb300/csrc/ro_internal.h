@@ -15,13 +15,14 @@ constexpr int FILL_THREADS = 256;
 constexpr uint32_t FILL_SMEM_CAP = FILL_TILE + 256;           // offsets staged per fill tile
 constexpr int RB_THREADS = 256, RB_ITEMS = 8;                 // candidates per tile: 2048
 constexpr int CM_THREADS = 256;
-constexpr int CF_THREADS = 256, CF_WORDS = 4;                 // bitmap words per tile: 1024
+constexpr int CF_THREADS = 256;                               // bitmap words per tile (1 each)
+constexpr int MB_ITEMS = 8;                                   // members per lane per step
 constexpr int AP_THREADS = 256, AP_ITEMS = 4;                 // listed parents per tile: 1024
 constexpr int AM_THREADS = 256, AM_ITEMS = 8;                 // members per tile: 2048
 constexpr uint32_t AM_TILE = AM_THREADS * AM_ITEMS;
 constexpr uint32_t AM_SMEM_CAP = 4096;                        // listed parents staged per tile
 constexpr int AC_THREADS = 256;
-constexpr uint64_t AC_CHUNK = 16384;                          // output bytes per copy chunk
+constexpr uint64_t AC_CHUNK = 16384;                          // output bytes per copy chunk (relative)
 constexpr uint32_t AC_BUF = 26624;                            // staged source bytes per chunk
 constexpr uint32_t AC_PIECES = 640;                           // member pieces staged per chunk
 
@@ -42,13 +43,27 @@ struct LaunchCfg {
       grid_amembers, grid_acopy;
 };
 
-// launch one kernel between the profiler's marks
-#define RO_LAUNCH(L, kid, ...)              \
-  do {                                      \
-    prof_begin((L).prof, (L).stream, kid);  \
-    __VA_ARGS__;                            \
-    prof_end((L).prof, (L).stream, kid);    \
-  } while (0)
+// Launch one kernel between the profiler's marks, with programmatic
+// dependent launch: the kernel may be scheduled while its predecessor on the
+// stream drains, and waits (griddepcontrol.wait, first statement of every
+// kernel here) until the predecessor has finished and its writes are visible.
+template <typename Arg>
+inline void launch_k(const LaunchCfg& L, int kid, void (*kern)(Arg), int grid, int block,
+                     size_t smem, const Arg& a) {
+  prof_begin(L.prof, L.stream, kid);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3((unsigned)block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = L.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, kern, a);
+  prof_end(L.prof, L.stream, kid);
+}
 
 // ---- ro_expand ----------------------------------------------------------------
 struct ExpandScanArgs {
@@ -97,6 +112,19 @@ struct ReadyArgs {
 };
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a);
 
+// ---- assembly plans ------------------------------------------------------------------
+// The plan of one list of completed parents: everything the copy needs, with
+// positions relative to the start of that call's output (header: PlanHdr).
+struct PlanBufs {
+  uint8_t* status;    // per listed parent
+  uint64_t* off;      // per listed parent: relative output offset; [n] = bytes
+  uint64_t* pbytes;   // scratch per listed parent: bytes, then their tile-local prefix
+  uint32_t* pnz;      // scratch per listed parent: contributing members, then prefix
+  uint64_t* cpos;     // per contributing member: relative output position
+  uint64_t* csrc;     // per contributing member: arena offset
+  PlanHdr* hdr;
+};
+
 // ---- ro_gather_commit ----------------------------------------------------------------
 struct CommitArgs {
   uint64_t n_host;
@@ -112,28 +140,26 @@ struct CommitArgs {
   Rec* rec;
   unsigned long long* pw;
   uint32_t* bitmap;
+  uint32_t* pm;               // per parent: members to gather once complete (0: Suppressed)
   uint8_t* code;              // user's or internal
   uint32_t* done_user;        // optional
   uint32_t* done_int;
   uint64_t* n_done_out;       // optional device output
   // assembly plan of the completed parents (consumed by ro_assemble(NULL))
   const uint64_t* offsets;
-  uint8_t* plan_status;       // P
-  uint32_t* plan_mb;          // P+1 member bases
-  uint32_t* plan_mtfp;        // member tile -> containing listed parent
-  uint64_t plan_mtfp_cap;
+  PlanBufs plan;
   DevScalars* ds;
-  TileStatus<Pair64> ts;
+  TileStatus<unsigned long long> ts_done;   // scan 1: completed parents
+  TileStatus<Pair64> ts_bytes;              // scan 2: (bytes, contributing members)
 };
 void launch_commit(const LaunchCfg& L, const CommitArgs& a);
 
 // ---- ro_assemble ---------------------------------------------------------------------
 struct AssembleArgs {
-  const uint32_t* list;       // user's list or the latest commit's
-  uint64_t n_host;            // list length, or capacity of the outputs
-  const uint64_t* d_n;        // device list length (optional, user list only)
-  int list_is_commit;         // plan of the latest commit (counts in ds->cm_n_done / cm_M)
-  const uint8_t* plan_status; // that plan's statuses (copied to status), or NULL
+  const uint32_t* list;       // explicit list of parents (asm_parents / asm_members only)
+  uint64_t n_host;            // list length, or capacity of the per-parent outputs
+  const uint64_t* d_n;        // device list length (optional, explicit list only)
+  int from_commit;            // 1: copy the latest commit's plan (no planning kernels)
   uint64_t P, N;
   const uint64_t* offsets;
   const unsigned long long* pw;
@@ -147,15 +173,13 @@ struct AssembleArgs {
   uint64_t out_cap;
   uint64_t* cursor;           // optional (device)
   uint64_t* out_bytes;        // optional (device)
-  // member bases / member-tile table: scratch (user list) or the commit's plan
-  uint32_t* mb;               // member base per listed parent (n+1)
-  uint32_t* mtfp;             // member tile -> containing listed parent
+  PlanBufs plan;              // the commit's plan, or scratch filled by the planning kernels
+  const uint8_t* st_src;      // statuses to copy into status (commit plan), or NULL
+  // explicit lists: member bases and member-tile table
+  uint32_t* mb;
+  uint32_t* mtfp;
   uint64_t mtfp_cap;
-  uint64_t* cpos;             // nonzero member output positions (relative to out)
-  uint64_t* csrc;             // nonzero member arena offsets
-  uint64_t member_cap;        // capacity of cpos/csrc
-  uint32_t* ctfp;             // copy chunk -> first member
-  uint64_t ctfp_cap;
+  uint64_t member_cap;        // capacity of plan.cpos / plan.csrc
   DevScalars* ds;
   TileStatus<unsigned long long> ts_parents;
   TileStatus<Pair64> ts_members;
