@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--parents", type=int, default=1_000_000)
     ap.add_argument("--waves", type=int, default=256)
     ap.add_argument("--no-graph", action="store_true", help="launch the wave loop eagerly")
+    ap.add_argument("--one-stream", action="store_true",
+                    help="plan and copy on the context's stream (no overlap across waves)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-parents", type=int, default=40_000,
@@ -243,6 +245,7 @@ class Pass:
                                       ob + 8 * s, None, self.arena_bytes, None, None, 0, None, None)
             bad |= L.ro_assemble(ctx, xid, ar, self.arena_bytes, None, self.P, None, st_p, oo, ol,
                                  out, self.out_cap, cur, obw + 8 * w, None)
+        bad |= L.ro_ctx_join(ctx)   # the copies of the last waves, back into the context's stream
         if bad:
             raise RuntimeError(f"wave loop: status {bad}: {ro.ro_last_error(ctx)}")
 
@@ -261,6 +264,9 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.set_stream(stream)
     ps = Pass(lv, local_rank, stream)
     ctx = ro.ro_ctx_create(local_rank, stream, 1)
+    if not args.one_stream:   # assembly planning and copies overlap later waves' commits
+        plan_stream, copy_stream = torch.cuda.Stream(), torch.cuda.Stream()
+        ro.ro_ctx_set_streams(ctx, plan_stream, copy_stream)
 
     def step_eager():
         ro.ro_ctx_reset(ctx)
@@ -365,6 +371,7 @@ def run_ours(args, rank, world, local_rank):
                        "parents": ps.P, "children": ps.N, "waves": args.waves,
                        "arena_bytes": ps.arena_bytes, "assembled_bytes": S,
                        "cuda_graph": graph is not None,
+                       "streams": 1 if args.one_stream else 3,
                        "l2": "inputs larger than L2 (39 GB arena)",
                        "parallelism": f"replicas x{world} (one microbatch per GPU)"},
             "payload_gbs": round(payload_gbs, 1),
@@ -435,6 +442,7 @@ def run_e2e(args, ps, ro, ctx, stream, world):
                           ps.status.data_ptr(), ps.out_off.data_ptr(), ps.out_len.data_ptr(),
                           ps.out.data_ptr(), ps.out_cap, ps.cursor.data_ptr(),
                           ps.out_bytes.data_ptr() + 8 * w, None)
+        L.ro_ctx_join(ctx)
         torch.cuda.current_stream().synchronize()
         S = int(ps.cursor.item())
         h_out[:S].copy_(ps.out[:S])

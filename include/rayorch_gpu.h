@@ -22,11 +22,17 @@
  *   library never keeps a caller pointer beyond the call (except the arena,
  *   see ro_gather_commit).  A context owns its internal lineage state
  *   (phase words, result slots, parent counters, queues, scratch).
- * - All work is issued on the context's stream, in call order.  Calls return
- *   without waiting for the GPU unless an h_ output is requested: a non-NULL
- *   h_ pointer makes the call synchronise the stream and fill it in.  The
- *   d_ count outputs are written by the GPU in stream order, so a following
- *   call can consume them (the d_n inputs) without a host round trip.
+ * - Work is issued on the context's stream, in call order, except assembly:
+ *   ro_assemble plans on the context's plan stream and copies on its copy
+ *   stream (both the context's stream unless ro_ctx_set_streams names
+ *   others).  Each assembly is ordered after all work the caller issued on
+ *   the context before it; the caller's ro_assemble outputs are complete
+ *   once ro_ctx_join has made the context's stream wait for the other two
+ *   (or once any call synchronises).  Calls return without waiting for the
+ *   GPU unless an h_ output is requested: a non-NULL h_ pointer makes the
+ *   call synchronise every stream and fill it in.  The d_ count outputs are
+ *   written by the GPU in stream order, so a following call can consume
+ *   them (the d_n inputs) without a host round trip.
  * - Errors are returned as ro_status; nothing throws across the ABI.
  *   Argument errors the host can see are RO_E_INVAL with no side effects.
  *   Conditions only the GPU can see (an output too small, a wait that timed
@@ -99,8 +105,25 @@ ro_status ro_ctx_destroy(ro_ctx* ctx);
 /* Forget every expansion (start the next microbatch).  Device memory is kept
  * and reused by later expansions of the same or smaller size. */
 ro_status ro_ctx_reset(ro_ctx* ctx);
-/* Wait for the stream and return (then clear) any condition recorded by the GPU. */
+/* Wait for every stream of the context and return (then clear) any condition
+ * recorded by the GPU. */
 ro_status ro_ctx_sync(ro_ctx* ctx);
+/* Streams for assembly (no counterpart in the paper; it schedules the path).
+ * plan_stream and copy_stream are cudaStream_t handles on the context's
+ * device, NULL for the context's stream.  With separate streams the planning
+ * and copy of one wave's completed parents overlap the next waves' admission
+ * and commits; up to three commits and assemblies per expansion may be in
+ * flight at once (the context keeps three list and plan slots per expansion
+ * and orders their reuse with events).  The context's stream first waits for
+ * the old streams.  The caller keeps the streams alive until ro_ctx_destroy
+ * or the next ro_ctx_set_streams. */
+ro_status ro_ctx_set_streams(ro_ctx* ctx, void* plan_stream, void* copy_stream);
+/* Make the context's stream wait (on the GPU) for all work issued so far on
+ * the plan and copy streams.  Call it before reading assembly outputs in
+ * stream order, before starting a capture of the context's stream, and
+ * before ending one (a captured assembly forks onto the other streams, and a
+ * capture must join them back).  Nothing waits on the host. */
+ro_status ro_ctx_join(ro_ctx* ctx);
 /* Synchronise and copy the cumulative counters. */
 ro_status ro_ctx_stats(ro_ctx* ctx, ro_stats* out);
 /* Text of the last error on this context ("" if none).  Valid until the next call. */
@@ -221,7 +244,11 @@ ro_status ro_gather_commit(ro_ctx* ctx, int32_t xid, uint64_t n, const uint64_t*
  * Parents are written back to back, in list order, starting at d_out + base
  * where base = *d_out_cursor (if given) or 0; the cursor then advances.
  *
- *   d_arena      the result arena the committed reports referred to.
+ *   d_arena      the result arena the committed reports referred to.  It
+ *                is read in aligned 16-byte blocks, so the memory from
+ *                d_arena up to the next 16-byte boundary at or after
+ *                d_arena + arena_bytes must be readable (true of any
+ *                cudaMalloc allocation that holds the arena).
  *   d_parents    uint32[n_parents] parent ids, or NULL for the parents
  *                completed by the latest ro_gather_commit on xid (in its
  *                ascending order); n_parents is then the capacity of the
@@ -238,6 +265,10 @@ ro_status ro_gather_commit(ro_ctx* ctx, int32_t xid, uint64_t n, const uint64_t*
  * as the results of the level above (nested expansions).
  * Errors: RO_E_CAPACITY when base + bytes > out_cap or the list is longer
  * than n_parents (nothing is copied).
+ * Streams: planning runs on the plan stream and the copy on the copy stream
+ * (see ro_ctx_set_streams); the outputs (d_status, d_out_off, d_out_len,
+ * d_out, the cursor, d_out_bytes) are written there.  Read them after
+ * ro_ctx_join in stream order, or after any synchronising call.
  */
 ro_status ro_assemble(ro_ctx* ctx, int32_t xid, const uint8_t* d_arena, uint64_t arena_bytes,
                       const uint32_t* d_parents, uint64_t n_parents, const uint64_t* d_n_parents,

@@ -28,7 +28,7 @@ STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFL
                 4: "RO_E_STATE", 5: "RO_E_OOM", 6: "RO_E_CUDA", 7: "RO_E_TIMEOUT"}
 
 EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro_ctx_stats",
-           "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
+           "ro_ctx_set_streams", "ro_ctx_join", "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
            "ro_gather_commit", "ro_assemble", "ro_expand_noalloc")
 
 # kernel ids (RO_K_*), in launch order of the path
@@ -72,6 +72,8 @@ def load(path: Optional[str] = None):
     L.ro_ctx_reset.argtypes = [_vp]
     L.ro_ctx_sync.argtypes = [_vp]
     L.ro_ctx_stats.argtypes = [_vp, C.POINTER(_Stats)]
+    L.ro_ctx_set_streams.argtypes = [_vp, _vp, _vp]
+    L.ro_ctx_join.argtypes = [_vp]
     L.ro_last_error.argtypes = [_vp]
     L.ro_last_error.restype = C.c_char_p
     L.ro_ctx_profile.argtypes = [_vp, _u32]
@@ -138,6 +140,17 @@ def ro_ctx_reset(ctx) -> int:
 
 def ro_ctx_sync(ctx) -> int:
     return load().ro_ctx_sync(ctx)
+
+
+def ro_ctx_set_streams(ctx, plan_stream=None, copy_stream=None) -> int:
+    """Assembly planning / copy streams (torch.cuda.Stream, raw handle or None)."""
+    st = load().ro_ctx_set_streams(ctx, _stream_handle(plan_stream), _stream_handle(copy_stream))
+    return _check("ro_ctx_set_streams", st, ctx)
+
+
+def ro_ctx_join(ctx) -> int:
+    """The context's stream waits (on the GPU) for the plan and copy streams."""
+    return _check("ro_ctx_join", load().ro_ctx_join(ctx), ctx)
 
 
 def ro_ctx_stats(ctx) -> dict:

@@ -3,23 +3,26 @@
 // A completed parent is Suppressed if a member Failed or was Suppressed,
 // otherwise Present with the Present members' payloads concatenated by
 // ordinal (Dropped members add nothing).  The work is a segmented byte gather
-// from the result arena, driven by an assembly plan: per listed parent its
-// relative output offset, per contributing member its relative position and
-// arena offset.  For the parents completed by the latest commit,
-// commit_finish has built the plan already; for an explicit list:
-//   asm_parents  per listed parent: outcome, number of members to gather
-//                (0 unless Present), exclusive scan of those counts (member
-//                bases), and for every 2048-member tile the parent holding its
-//                first member;
-//   asm_members  per member (load-balanced over tiles of 2048 members, so a
-//                100k-member parent is spread over many CTAs): read its
-//                record and scan the Present bytes (single-pass look-back).
-// Then asm_copy writes the output in 16 KB chunks of the call's output: one
-// warp finds the chunk's members (32-ary warp search over the positions) and
-// stages their source bytes in shared memory with cp.async.bulk (two stages,
-// mbarrier completion, bounded waits) while all warps turn the previous chunk
-// into aligned 16-byte stores; source and destination alignments may differ
-// arbitrarily.
+// from the result arena in three steps:
+//   asm_parents  (caller's lists only; commit_finish does this for the
+//                parents a commit completed) per listed parent: outcome,
+//                members to gather (0 unless Present), their exclusive scan
+//                (member bases), and for every 2048-member tile the parent
+//                holding its first member;
+//   asm_members  per member, load-balanced over 2048-member tiles so a
+//                100k-member parent spreads over many CTAs: read the record,
+//                scan the Present bytes (single-pass look-back) and write the
+//                plan — each parent's relative output offset, each
+//                contributing member's relative position and arena offset, and
+//                for every 16 KB chunk of the output the member holding its
+//                first byte;
+//   asm_copy     per chunk: one warp stages the chunk's member pieces in
+//                shared memory with cp.async.bulk (two stages, mbarrier
+//                completion, bounded waits) while all warps turn the previous
+//                chunk into aligned 16-byte stores; source and destination
+//                alignments may differ arbitrarily.
+// The plan is independent of where the output starts, so planning (on the
+// context's plan stream) can run ahead of the copies (copy stream).
 #include <algorithm>
 
 #include "ro_internal.h"
@@ -27,12 +30,6 @@
 namespace ro {
 
 constexpr int TS_ASM_COPY = 5;
-
-__device__ __forceinline__ uint64_t asm_list_count(const AssembleArgs& a, bool* over) {
-  const uint64_t n = a.d_n ? *a.d_n : a.n_host;
-  *over = n > a.n_host;
-  return n > a.n_host ? a.n_host : n;
-}
 
 template <class V>
 __device__ __forceinline__ uint32_t last_le_u(const V* v, uint32_t lo, uint32_t hi, uint64_t x) {
@@ -47,6 +44,7 @@ __device__ __forceinline__ uint32_t last_le_u(const V* v, uint32_t lo, uint32_t 
 }
 
 // ---------------------------------------------------------------------------
+// asm_parents: a caller's list -> outcomes, member bases, member-tile table.
 __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a) {
   wait_predecessor();
   __shared__ unsigned long long s_scan[33];
@@ -54,22 +52,25 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
   __shared__ unsigned long long s_prefix;
   __shared__ unsigned long long s_incomplete;
   DevScalars* ds = a.ds;
-  bool over = false;
-  const uint64_t n = asm_list_count(a, &over);
-  if (over) {
-    if (threadIdx.x == 0) {
-      ds->as_err = 1u;
-      atomicOr(&ds->err, ERR_CAPACITY);
+  const ListBufs& L = a.list;
+  const uint64_t n_req = a.d_n ? *a.d_n : a.n_host;
+  if (n_req > a.n_host) {   // a device count beyond the arrays' length
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      L.hdr->err = 1u;
+      L.hdr->n = 0;
+      atomicOr(&ds->err, ERR_INVAL);
     }
-    return;   // no tile claimed
+    return;
   }
+  const uint64_t n = n_req;
   const uint64_t TILE = (uint64_t)AP_THREADS * AP_ITEMS;
   const uint64_t n_tiles = ceil_div(n, TILE);
   if (n_tiles == 0) {
     if (blockIdx.x == 0 && threadIdx.x == 0) {
-      a.mb[0] = 0;
-      ds->as_M = 0;
-      ds->as_hdr.n = 0;
+      L.mb[0] = 0;
+      L.hdr->n = 0;
+      L.hdr->M = 0;
+      L.hdr->err = 0u;
     }
     return;
   }
@@ -83,18 +84,20 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
     __syncthreads();
     if (tile >= n_tiles) break;
     const uint64_t i0 = tile * TILE + (uint64_t)threadIdx.x * AP_ITEMS;
-    uint32_t m[AP_ITEMS];
+    uint32_t m[AP_ITEMS], cf[AP_ITEMS];
     unsigned long long mine = 0;
     uint32_t incomplete = 0;
 #pragma unroll
     for (int k = 0; k < AP_ITEMS; ++k) {
       const uint64_t i = i0 + k;
       m[k] = 0;
+      cf[k] = 0;
       if (i >= n) continue;
-      const uint64_t p = a.list[i];
+      const uint64_t p = L.parents[i];
       uint8_t st = ST_PENDING;
       if (p < a.P) {
         const unsigned long long v = a.pw[p];
+        cf[k] = (uint32_t)a.offsets[p];
         if (pw_remaining(v) == 0u) {
           if (pw_bad(v) != 0u) {
             st = ST_SUPPRESSED;
@@ -105,34 +108,35 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
         }
       }
       if (st == ST_PENDING) ++incomplete;
-      a.status[i] = st;
+      L.status[i] = st;
       mine += m[k];
     }
     if (incomplete) atomicAdd(&s_incomplete, (unsigned long long)incomplete);
     unsigned long long total;
     unsigned long long excl = block_excl_scan(mine, s_scan, &total);
-    if (threadIdx.x == 0) s_prefix = lookback_exclusive(a.ts_parents, tile, total, ds->epoch[TS_ASM_PARENTS], &ds->err);
+    if (threadIdx.x == 0)
+      s_prefix = lookback_exclusive(a.ts_parents, tile, total, ds->epoch[TS_ASM_PARENTS], &ds->err);
     __syncthreads();
     unsigned long long run = s_prefix + excl;
 #pragma unroll
     for (int k = 0; k < AP_ITEMS; ++k) {
       const uint64_t i = i0 + k;
       if (i >= n) break;
-      a.mb[i] = (uint32_t)run;
+      L.mb[i] = (uint32_t)run;
+      L.coff[i] = cf[k];
       if (m[k]) {
-        for (uint64_t b = ceil_div(run, AM_TILE); b * AM_TILE < run + m[k] && b < a.mtfp_cap; ++b)
-          a.mtfp[b] = (uint32_t)i;
+        for (uint64_t b = ceil_div(run, AM_TILE); b * AM_TILE < run + m[k] && b < L.mtfp_cap; ++b)
+          L.mtfp[b] = (uint32_t)i;
       }
       run += m[k];
     }
     if (tile == n_tiles - 1 && threadIdx.x == AP_THREADS - 1) {
-      a.mb[n] = (uint32_t)run;
-      ds->as_M = run;
-      ds->as_hdr.n = n;
-      if (run > a.member_cap) {
-        ds->as_err = 1u;
-        atomicOr(&ds->err, ERR_CAPACITY);
-      }
+      L.mb[n] = (uint32_t)run;
+      L.hdr->n = n;
+      L.hdr->M = run;
+      // more members than the plan holds (a parent listed many times)
+      L.hdr->err = run > a.plan.member_cap ? 1u : 0u;
+      if (run > a.plan.member_cap) atomicOr(&ds->err, ERR_CAPACITY);
     }
   }
   __syncthreads();
@@ -143,6 +147,7 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
 }
 
 // ---------------------------------------------------------------------------
+// asm_members: list -> plan (relative offsets and member positions).
 __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a) {
   wait_predecessor();
   __shared__ uint32_t s_mb[AM_SMEM_CAP];
@@ -151,23 +156,43 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
   __shared__ uint32_t s_tile;
   __shared__ Pair64 s_prefix;
   DevScalars* ds = a.ds;
+  const ListBufs& L = a.list;
   const PlanBufs& pl = a.plan;
-  if (ds->as_err) return;   // nothing claimed
-  const uint64_t n = ds->as_hdr.n, M = ds->as_M;
-  const uint64_t n_tiles = ceil_div(M, AM_TILE);
-
-  if (M == 0) {   // nothing to gather: every listed parent starts at 0
-    if (blockIdx.x == 0) {
-      for (uint64_t i = threadIdx.x; i <= n; i += blockDim.x) pl.off[i] = 0;
-      if (threadIdx.x == 0) {
-        pl.hdr->bytes = 0;
-        pl.hdr->nnz = 0;
-      }
+  const ListHdr lh = *L.hdr;
+  const uint64_t n = lh.n, M = lh.M;
+  if (lh.err) {   // nothing to plan
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      pl.hdr->n = n;
+      pl.hdr->bytes = 0;
+      pl.hdr->nnz = 0;
+      pl.hdr->err = 1u;
     }
     return;
   }
-  const uint32_t n_part = participants(n_tiles);
+  const uint64_t n_tiles = ceil_div(M, AM_TILE);
+  const uint64_t par_units = ceil_div(n, (uint64_t)AM_TILE);
+  const uint32_t n_part = participants((n_tiles > par_units ? n_tiles : par_units) + 1);
   if (blockIdx.x >= n_part) return;
+
+  // outcomes travel with the plan (the list's slot may be reused meanwhile)
+  if (pl.status) {
+    const uint64_t stride = (uint64_t)n_part * blockDim.x;
+    for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
+      pl.status[i] = L.status[i];
+  }
+  if (M == 0) {   // nothing to gather: every listed parent starts at 0
+    const uint64_t stride = (uint64_t)n_part * blockDim.x;
+    for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i <= n; i += stride)
+      pl.off[i] = 0;
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      pl.hdr->n = n;
+      pl.hdr->bytes = 0;
+      pl.hdr->nnz = 0;
+      pl.hdr->err = 0u;
+      pl.hdr->chunks_ok = 1u;
+    }
+    return;
+  }
 
   for (;;) {
     if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_ASM_MEMBERS]);
@@ -176,15 +201,14 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
     __syncthreads();
     if (tile >= n_tiles) break;
     const uint64_t g0 = (uint64_t)tile * AM_TILE;
-    const uint64_t i_lo = a.mtfp[tile];
-    const uint64_t i_hi = (tile + 1 < n_tiles) ? a.mtfp[tile + 1] : n - 1;
+    const uint64_t i_lo = L.mtfp[tile];
+    const uint64_t i_hi = (tile + 1 < n_tiles) ? L.mtfp[tile + 1] : n - 1;
     const uint64_t R = i_hi - i_lo + 1;
     const bool staged = R <= AM_SMEM_CAP;
     if (staged) {
       for (uint64_t k = threadIdx.x; k < R; k += blockDim.x) {
-        s_mb[k] = a.mb[i_lo + k];
-        const uint64_t p = a.list[i_lo + k];   // listed ids may name no parent
-        s_coff[k] = p < a.P ? (uint32_t)a.offsets[p] : 0u;
+        s_mb[k] = L.mb[i_lo + k];
+        s_coff[k] = L.coff[i_lo + k];
       }
     }
     __syncthreads();
@@ -213,11 +237,11 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
         uint64_t lo = i_lo, hi = i_hi + 1;
         while (hi - lo > 1) {
           const uint64_t mid = lo + ((hi - lo) >> 1);
-          if (a.mb[mid] <= g) lo = mid; else hi = mid;
+          if (L.mb[mid] <= g) lo = mid; else hi = mid;
         }
         i = lo;
-        mbi = a.mb[lo];
-        coff = a.offsets[a.list[lo]];
+        mbi = L.mb[lo];
+        coff = L.coff[lo];
       }
       const Rec r = a.rec[coff + (g - mbi)];
       if (w_state(r.w) == ST_PRESENT && r.len) {
@@ -226,7 +250,7 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
         // the arena passed here must hold what the commit accepted
         if (src[k] > a.arena_bytes || (uint64_t)r.len > a.arena_bytes - src[k]) {
           atomicOr(&ds->err, ERR_INVAL);
-          ds->as_err = 1u;
+          pl.hdr->err = 1u;
         }
       }
       par[k] = (uint32_t)i;
@@ -249,17 +273,20 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
         // the parent starts here, and so do the member-less parents listed just before it
         pl.off[par[k]] = pos;
         for (int64_t q = (int64_t)par[k] - 1; q >= 0; --q) {
-          const uint32_t mbq = (staged && (uint64_t)q >= i_lo) ? s_mb[q - i_lo] : a.mb[q];
+          const uint32_t mbq = (staged && (uint64_t)q >= i_lo) ? s_mb[q - i_lo] : L.mb[q];
           if (mbq != g) break;
           pl.off[q] = pos;
         }
       }
       if (contrib[k]) {
         const uint64_t j = run.b;
-        if (j < a.member_cap) {
+        if (j < pl.member_cap) {
           pl.cpos[j] = pos;
           pl.csrc[j] = src[k];
         }
+        const uint64_t e = pos + contrib[k];
+        for (uint64_t t = ceil_div(pos, AC_CHUNK); t * AC_CHUNK < e && t < pl.ctfp_cap; ++t)
+          pl.ctfp[t] = (uint32_t)j;
         run.b += 1;
         run.a += contrib[k];
       }
@@ -267,11 +294,13 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
     if (tile == n_tiles - 1 && threadIdx.x == AM_THREADS - 1) {
       pl.off[n] = run.a;
       for (int64_t q = (int64_t)n - 1; q >= 0; --q) {
-        if ((uint64_t)a.mb[q] != M) break;   // member-less parents at the very end
+        if ((uint64_t)L.mb[q] != M) break;   // member-less parents at the very end
         pl.off[q] = run.a;
       }
+      pl.hdr->n = n;
       pl.hdr->bytes = run.a;
       pl.hdr->nnz = run.b;
+      pl.hdr->chunks_ok = ceil_div(run.a, AC_CHUNK) <= pl.ctfp_cap ? 1u : 0u;
     }
     __syncthreads();
   }
@@ -451,8 +480,9 @@ struct CopyCtx {
   const AssembleArgs* a;
   const uint64_t* cpos;
   const uint64_t* csrc;
-  uint64_t out_base;   // absolute address of the call's first output byte
-  uint64_t S, Mnz;
+  const uint32_t* ctfp;   // chunk table, or NULL (search instead)
+  uint64_t out_base;      // absolute address of the call's first output byte
+  uint64_t S, Mnz, n_chunks;
 };
 
 __device__ __forceinline__ uint64_t cpos_at(const CopyCtx& c, uint64_t j) {
@@ -479,8 +509,14 @@ __device__ __forceinline__ uint64_t warp_search(const uint64_t* pos, uint64_t n,
 __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_t* bar, int lane) {
   const uint64_t rs = k * AC_CHUNK;
   const uint64_t re = (rs + AC_CHUNK < c.S) ? rs + AC_CHUNK : c.S;
-  const uint64_t j_lo = warp_search(c.cpos, c.Mnz, rs, lane);
-  const uint64_t j_hi = warp_search(c.cpos, c.Mnz, re - 1, lane);
+  uint64_t j_lo, j_hi;
+  if (c.ctfp) {
+    j_lo = c.ctfp[k];
+    j_hi = (k + 1 < c.n_chunks) ? c.ctfp[k + 1] : c.Mnz - 1;
+  } else {
+    j_lo = warp_search(c.cpos, c.Mnz, rs, lane);
+    j_hi = warp_search(c.cpos, c.Mnz, re - 1, lane);
+  }
   const uint64_t np = j_hi - j_lo + 1;
   const uint64_t wbase = (c.out_base + rs) & ~15ull;
   if (lane == 0) {
@@ -630,8 +666,8 @@ __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a)
   const uint64_t n = hdr.n, S = hdr.bytes;
   const uint64_t base = a.cursor ? *a.cursor : 0ull;
   // conditions every CTA sees the same way
-  bool failed = ds->as_err != 0u;
-  const bool too_many = a.from_commit && n > a.n_host;   // outputs hold fewer parents
+  bool failed = hdr.err != 0u;
+  const bool too_many = !a.user_list && n > a.n_host;   // outputs hold fewer parents
   const bool too_big = base + S > a.out_cap;
   if (!failed && (too_many || too_big)) {
     failed = true;
@@ -641,10 +677,12 @@ __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a)
   c.a = &a;
   c.cpos = a.plan.cpos;
   c.csrc = a.plan.csrc;
+  c.ctfp = hdr.chunks_ok ? a.plan.ctfp : nullptr;
   c.out_base = (uint64_t)(uintptr_t)a.out + base;
   c.S = S;
   c.Mnz = hdr.nnz;
   const uint64_t n_chunks = (!failed && S) ? ceil_div(S, AC_CHUNK) : 0;
+  c.n_chunks = n_chunks;
   const uint64_t par_units = failed ? 0 : ceil_div(n + 1, (uint64_t)AC_THREADS * 8);
   uint64_t units = n_chunks > par_units ? n_chunks : par_units;
   if (units == 0) units = 1;   // one CTA still finishes the call
@@ -660,7 +698,7 @@ __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a)
         const uint64_t o = a.plan.off[i];
         a.out_off[i] = base + o;
         if (i == n) break;
-        if (a.st_src) a.status[i] = a.st_src[i];
+        if (a.plan.status) a.status[i] = a.plan.status[i];
         if (a.out_len) {
           const uint64_t len = a.plan.off[i + 1] - o;
           if (len > 0xFFFFFFFFull) atomicOr(&ds->err, ERR_OVERFLOW);
@@ -710,20 +748,23 @@ __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a)
       if (!failed && a.cursor) *a.cursor = base + S;
       if (a.out_bytes) *a.out_bytes = S;
       ds->as_bytes = S;
-      ds->as_err = 0u;
+      a.plan.hdr->err = 0u;   // the plan is consumed
       ds->exit_ctr[TS_ASM_COPY] = 0u;
       __threadfence();
     }
   }
 }
 
-void launch_assemble(const LaunchCfg& L, const AssembleArgs& a) {
-  if (!a.from_commit) {
+void launch_assemble_plan(const LaunchCfg& L, const AssembleArgs& a) {
+  if (a.user_list) {
     const uint64_t tiles = ceil_div(a.n_host, (uint64_t)AP_THREADS * AP_ITEMS);
     const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(tiles, (uint64_t)L.grid_aparents));
     launch_k(L, K_APARENTS, asm_parents_kernel, grid, AP_THREADS, 0, a);
-    launch_k(L, K_AMEMBERS, asm_members_kernel, L.grid_amembers, AM_THREADS, 0, a);
   }
+  launch_k(L, K_AMEMBERS, asm_members_kernel, L.grid_amembers, AM_THREADS, 0, a);
+}
+
+void launch_assemble_copy(const LaunchCfg& L, const AssembleArgs& a) {
   launch_k(L, K_ACOPY, asm_copy_kernel, L.grid_acopy, AC_THREADS, asm_copy_smem(), a);
 }
 

@@ -12,16 +12,15 @@
 //                 a completion bitmap.
 //                 That add also tells whether a member Failed or was
 //                 Suppressed, so the same thread records how many members the
-//                 parent will gather (0 if Suppressed).
+//                 parent will gather (0 if Suppressed) and adds it to its
+//                 bitmap word's total.
 // commit_finish   turns the bitmap into the ascending list of completed
-//                 parents (popcount + single-pass scan over bitmap words) and
-//                 clears it, then plans their assembly: per parent its
-//                 relative output offset, per contributing member its
-//                 relative position and arena offset (a second single-pass
-//                 scan).  When the scatter saw two reports for one Grain in
-//                 the same call (rare), the first CTA in orders them first, so
-//                 the result equals applying the reports one by one in array
-//                 order.
+//                 parents and their member bases (one single-pass scan over
+//                 bitmap words of (popcount, word total)) and clears it; the
+//                 list is what ro_assemble(NULL) plans and copies.  When the
+//                 scatter saw two reports for one Grain in the same call
+//                 (rare), the first CTA in orders them first, so the result
+//                 equals applying the reports one by one in array order.
 #include <algorithm>
 
 #include "ro_internal.h"
@@ -117,6 +116,7 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
         if ((uint32_t)old == n_tot) {   // the last members: the parent is complete
           const uint32_t m = (pw_bad(old) + n_bad) ? 0u : (uint32_t)(a.offsets[p + 1] - a.offsets[p]);
           a.pm[p] = m;
+          if (m) atomicAdd(a.wm + (p >> 5), m);
           atomicOr(a.bitmap + (p >> 5), 1u << (p & 31));
         }
       }
@@ -212,7 +212,8 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
     const unsigned long long pv = __ldcg(a.pw + p);
     if (pw_remaining(pv) == 0u) {
       const uint32_t m = pw_bad(pv) ? 0u : (uint32_t)(a.offsets[p + 1] - a.offsets[p]);
-      atomicExch(a.pm + p, m);
+      const uint32_t old = atomicExch(a.pm + p, m);
+      if (old != m) atomicAdd(a.wm + (p >> 5), m - old);
     }
     a.code[r] = (v == V_WIN_SEALER || v == V_WIN_CAND) ? V_ACCEPT : V_DUPLICATE;
   }
@@ -221,58 +222,25 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
   __syncthreads();
 }
 
-// Warp `lane`'s share of parent p's members, MB_ITEMS consecutive records
-// per lane per step: calls f(k, contrib, src) for every member k of the step
-// in order (contrib 0 for members that add no bytes).
-template <class F>
-__device__ __forceinline__ void for_members(const CommitArgs& a, uint64_t c0, uint64_t m, int lane,
-                                            F&& f) {
-  for (uint64_t g = 0; g < m; g += 32 * MB_ITEMS) {
-    uint32_t len[MB_ITEMS];
-    uint64_t src[MB_ITEMS];
-#pragma unroll
-    for (int t = 0; t < MB_ITEMS; ++t) {
-      const uint64_t k = g + (uint64_t)lane * MB_ITEMS + t;
-      len[t] = 0;
-      src[t] = 0;
-      if (k < m) {
-        const Rec r = a.rec[c0 + k];
-        if (w_state(r.w) == ST_PRESENT) {
-          len[t] = r.len;
-          src[t] = w_off(r.w);
-        }
-      }
-    }
-    f(g, len, src);
-  }
-}
-
-// Completed-parent list, ascending (popcount + look-back scan over bitmap
-// words), and the assembly plan of those parents: each parent's outcome and
-// relative output offset, and for every member that contributes bytes its
-// relative output position and arena offset (a second look-back scan, of
-// (bytes, contributing members), in the same tile order).
+// Completed-parent list, ascending, with each parent's outcome, first child
+// and member base, and the member-tile table asm_members works from.
 __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a) {
   wait_predecessor();
-  __shared__ unsigned long long s_scan[33];
-  __shared__ Pair64 s_scan2[33];
+  __shared__ Pair64 s_scan[33];
   __shared__ uint32_t s_tile;
-  __shared__ unsigned long long s_nb, s_ne;
-  __shared__ Pair64 s_base, s_carry;
+  __shared__ Pair64 s_prefix;
   __shared__ uint32_t s_fix;
   DevScalars* ds = a.ds;
-  const PlanBufs& pl = a.plan;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  constexpr int N_WARPS = CF_THREADS / 32;
+  const ListBufs& L = a.list;
   const uint64_t n_words = ceil_div(a.P, 32);
   const uint64_t n_tiles = ceil_div(n_words, (uint64_t)CF_THREADS);
   if (n_tiles == 0) {
     if (blockIdx.x == 0 && threadIdx.x == 0) {
       ds->cm_n_done = 0;
-      pl.hdr->n = 0;
-      pl.hdr->bytes = 0;
-      pl.hdr->nnz = 0;
-      pl.off[0] = 0;
+      L.hdr->n = 0;
+      L.hdr->M = 0;
+      L.hdr->err = 0u;
+      L.mb[0] = 0;
       if (a.n_done_out) *a.n_done_out = 0;
     }
     return;
@@ -310,134 +278,43 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
     const uint32_t tile = s_tile;
     __syncthreads();
     if (tile >= n_tiles) break;
-
-    // ---- scan 1: completed parents of this tile's 256 bitmap words
     const uint64_t w = (uint64_t)tile * CF_THREADS + threadIdx.x;
     const uint32_t bits = (w < n_words) ? a.bitmap[w] : 0u;
-    unsigned long long total;
-    const unsigned long long excl = block_excl_scan((unsigned long long)__popc(bits), s_scan, &total);
-    if (threadIdx.x == 0) {
-      const unsigned long long nb =
-          lookback_exclusive(a.ts_done, tile, total, ds->epoch[TS_COMMIT], &ds->err);
-      s_nb = nb;
-      s_ne = nb + total;
-    }
+    const uint32_t wsum = bits ? __ldcg(a.wm + w) : 0u;
+    Pair64 total;
+    const Pair64 excl = block_excl_scan_pair(Pair64{(unsigned long long)__popc(bits), wsum}, s_scan, &total);
+    if (threadIdx.x == 0)
+      s_prefix = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_COMMIT], &ds->err);
     __syncthreads();
-    const unsigned long long nb = s_nb, ne = s_ne;
+    Pair64 run = s_prefix + excl;   // (completed parents, members) before my word
     if (bits) {
-      unsigned long long i = nb + excl;
       uint32_t b = bits;
       while (b) {
         const uint32_t parent = (uint32_t)(w * 32 + (__ffs(b) - 1));
         b &= b - 1;
+        const uint32_t m = __ldcg(a.pm + parent);
+        const unsigned long long i = run.a;
         a.done_int[i] = parent;
         if (a.done_user) a.done_user[i] = parent;
-        pl.status[i] = __ldcg(a.pm + parent) ? ST_PRESENT : ST_SUPPRESSED;
-        ++i;
+        L.status[i] = m ? ST_PRESENT : ST_SUPPRESSED;
+        L.mb[i] = (uint32_t)run.b;
+        L.coff[i] = (uint32_t)a.offsets[parent];
+        for (uint64_t t = ceil_div(run.b, AM_TILE); t * AM_TILE < run.b + m && t < L.mtfp_cap; ++t)
+          L.mtfp[t] = (uint32_t)i;
+        run.a += 1;
+        run.b += m;
       }
       a.bitmap[w] = 0u;
+      a.wm[w] = 0u;
     }
-    __syncthreads();
-
-    // ---- bytes and contributing members of each completed parent (a warp each)
-    for (unsigned long long i = nb + warp; i < ne; i += N_WARPS) {
-      const uint32_t p = a.done_int[i];
-      unsigned long long bytes = 0, nz = 0;
-      if (pl.status[i] == ST_PRESENT) {
-        const uint64_t c0 = a.offsets[p], m = a.offsets[p + 1] - c0;
-        for_members(a, c0, m, lane, [&](uint64_t, const uint32_t* len, const uint64_t*) {
-#pragma unroll
-          for (int t = 0; t < MB_ITEMS; ++t) {
-            bytes += len[t];
-            nz += len[t] ? 1u : 0u;
-          }
-        });
-#pragma unroll
-        for (int d = 16; d > 0; d >>= 1) {
-          bytes += __shfl_down_sync(0xffffffffu, bytes, d);
-          nz += __shfl_down_sync(0xffffffffu, nz, d);
-        }
-      }
-      if (lane == 0) {
-        pl.pbytes[i] = bytes;
-        pl.pnz[i] = (uint32_t)nz;
-      }
+    if (tile == n_tiles - 1 && threadIdx.x == CF_THREADS - 1) {
+      ds->cm_n_done = run.a;
+      L.hdr->n = run.a;
+      L.hdr->M = run.b;
+      L.hdr->err = 0u;
+      L.mb[run.a] = (uint32_t)run.b;
+      if (a.n_done_out) *a.n_done_out = run.a;
     }
-    __syncthreads();
-
-    // ---- tile-local exclusive prefix of (bytes, contributing members)
-    if (threadIdx.x == 0) s_carry = Pair64{0, 0};
-    __syncthreads();
-    for (unsigned long long i0 = nb; i0 < ne; i0 += CF_THREADS) {
-      const unsigned long long i = i0 + threadIdx.x;
-      const Pair64 v = (i < ne) ? Pair64{pl.pbytes[i], pl.pnz[i]} : Pair64{0, 0};
-      Pair64 tot;
-      const Pair64 ex = block_excl_scan_pair(v, s_scan2, &tot);
-      const Pair64 carry = s_carry;
-      if (i < ne) {
-        pl.pbytes[i] = carry.a + ex.a;
-        pl.pnz[i] = (uint32_t)(carry.b + ex.b);
-      }
-      __syncthreads();
-      if (threadIdx.x == 0) s_carry = carry + tot;
-      __syncthreads();
-    }
-    if (threadIdx.x == 0)
-      s_base = lookback_exclusive(a.ts_bytes, tile, s_carry, ds->epoch[TS_COMMIT], &ds->err);
-    __syncthreads();
-    const Pair64 base = s_base;
-
-    // ---- relative offsets and member positions
-    for (unsigned long long i = nb + warp; i < ne; i += N_WARPS) {
-      const uint64_t off = base.a + pl.pbytes[i];
-      uint64_t nzb = base.b + pl.pnz[i];
-      if (lane == 0) pl.off[i] = off;
-      if (pl.status[i] != ST_PRESENT) continue;
-      const uint32_t p = a.done_int[i];
-      const uint64_t c0 = a.offsets[p], m = a.offsets[p + 1] - c0;
-      uint64_t run = off;
-      for_members(a, c0, m, lane, [&](uint64_t, const uint32_t* len, const uint64_t* src) {
-        unsigned long long mine = 0, mine_nz = 0;
-#pragma unroll
-        for (int t = 0; t < MB_ITEMS; ++t) {
-          mine += len[t];
-          mine_nz += len[t] ? 1u : 0u;
-        }
-        unsigned long long inc = mine, inc_nz = mine_nz;
-#pragma unroll
-        for (int d = 1; d < 32; d <<= 1) {
-          const unsigned long long u = __shfl_up_sync(0xffffffffu, inc, d);
-          const unsigned long long un = __shfl_up_sync(0xffffffffu, inc_nz, d);
-          if (lane >= d) {
-            inc += u;
-            inc_nz += un;
-          }
-        }
-        uint64_t pos = run + (inc - mine);
-        uint64_t j = nzb + (inc_nz - mine_nz);
-#pragma unroll
-        for (int t = 0; t < MB_ITEMS; ++t) {
-          if (len[t]) {
-            pl.cpos[j] = pos;
-            pl.csrc[j] = src[t];
-            ++j;
-            pos += len[t];
-          }
-        }
-        run += __shfl_sync(0xffffffffu, inc, 31);
-        nzb += __shfl_sync(0xffffffffu, inc_nz, 31);
-      });
-    }
-    if (tile == n_tiles - 1 && threadIdx.x == 0) {
-      const Pair64 end = base + s_carry;
-      ds->cm_n_done = ne;
-      pl.hdr->n = ne;
-      pl.hdr->bytes = end.a;
-      pl.hdr->nnz = end.b;
-      pl.off[ne] = end.a;
-      if (a.n_done_out) *a.n_done_out = ne;
-    }
-    __syncthreads();
   }
   if (threadIdx.x == 0) {
     __threadfence();

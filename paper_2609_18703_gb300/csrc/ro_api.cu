@@ -1,6 +1,14 @@
 // ro_api.cu — host side of the C ABI declared in include/rayorch_gpu.h:
 // argument checks, ownership of the per-expansion device state, scratch,
-// kernel launches and the mapping of device-recorded conditions to statuses.
+// kernel launches on the context's streams, and the mapping of
+// device-recorded conditions to statuses.
+//
+// Streams.  Expansion, admission and commit run on the context's stream.
+// Assembly planning (asm_parents, asm_members) runs on the plan stream and
+// the copy on the copy stream; both default to the context's stream.  With
+// separate streams the work of consecutive waves overlaps: the lists of
+// completed parents and the assembly plans live in rings of slots per
+// expansion, handed from stream to stream with events.
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
@@ -25,12 +33,19 @@ using namespace ro;
 namespace {
 
 constexpr int MAX_EXPANSIONS = 64;
-constexpr int N_TS = 8;   // tile-status slots (TS_* in ro_common.cuh)
-constexpr int TS_COMMIT_BYTES = 6;   // commit_finish's second scan (flags only; shares TS_COMMIT's epoch)
+constexpr int N_TS = 8;    // tile-status slots (TS_* in ro_common.cuh)
+constexpr int RING = 3;    // list / plan slots per expansion
 
 struct DevBuf {
   void* p = nullptr;
   size_t cap = 0;
+};
+
+// An event with the stream capture it was recorded under (0: none).
+struct Ev {
+  cudaEvent_t e = nullptr;
+  unsigned long long cap_id = 0;
+  bool recorded = false;
 };
 
 struct QueueBufs {
@@ -38,18 +53,31 @@ struct QueueBufs {
   bool ready = false;   // state zeroed for the current expansion
 };
 
+// A list of completed parents (written by a commit, read by planning).
+struct ListSlot {
+  DevBuf done, status, mb, coff, mtfp, hdr;
+  Ev freed;   // the planning that read it is done
+};
+// An assembly plan (written by planning, read by the copy).
+struct PlanSlot {
+  DevBuf status, off, cpos, csrc, ctfp, hdr;
+  uint64_t ctfp_cap = 0;
+  Ev ready, freed;
+};
+
 // Device buffers of one expansion slot, kept across ro_ctx_reset and reused.
 struct ExpSlot {
-  DevBuf offsets, pw, phase, rec, bitmap, done, tfp, pm;
-  // assembly plan of the latest commit
-  DevBuf plan_status, plan_off, plan_pbytes, plan_pnz, plan_cpos, plan_csrc, plan_hdr;
+  DevBuf offsets, pw, phase, rec, bitmap, tfp, pm, wm;
+  ListSlot lists[RING];
+  PlanSlot plans[RING];
   std::vector<QueueBufs> queues;
 };
 
 struct Expansion {
   int32_t parent_xid = -1;
   uint64_t P = 0, N = 0;
-  bool committed = false;   // a commit produced a completed-parent list
+  uint64_t commits = 0, assembles = 0;
+  int last_list = -1;   // list slot written by the latest commit
 };
 
 struct TsBuf {
@@ -102,16 +130,20 @@ void prof_end(Profiler* p, cudaStream_t s, int kid) {
 
 struct ro_ctx {
   int device = 0;
-  cudaStream_t stream = nullptr;
+  cudaStream_t stream = nullptr;        // expansion, admission, commit
+  cudaStream_t plan_stream = nullptr;   // assembly planning
+  cudaStream_t copy_stream = nullptr;   // assembly copies
   uint32_t n_calls = 1;
   int num_sms = 0;
-  LaunchCfg L{};
+  LaunchCfg L{}, Lp{}, Lc{};
   DevScalars* ds = nullptr;
   DevScalars* hs = nullptr;   // pinned mirror
   std::vector<ExpSlot> slots;
   std::vector<Expansion> exps;
   TsBuf ts[N_TS];
-  DevBuf code, mb, mtfp, cpos, csrc, as_off;
+  DevBuf code;
+  DevBuf x_mb, x_coff, x_mtfp, x_hdr;   // explicit-list assembly scratch
+  Ev fork, x_planned, join_plan, join_copy;
   Profiler prof;
   ro_status sticky = RO_OK;
   std::string err;
@@ -151,12 +183,37 @@ ro_status cuda_fail(ro_ctx* c, cudaError_t e, const char* what) {
   return fail(c, RO_E_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
-// Grow-only device buffer.  New memory is zeroed on the context's stream.
+#define RO_TRY(x)                 \
+  do {                            \
+    ro_status _s = (x);           \
+    if (_s != RO_OK) return _s;   \
+  } while (0)
+
+unsigned long long capture_id(cudaStream_t s) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  unsigned long long id = 0;
+  if (cudaStreamGetCaptureInfo(s, &st, &id) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return st == cudaStreamCaptureStatusActive ? id : 0;
+}
+
+void sync_all_streams(ro_ctx* c) {
+  cudaStreamSynchronize(c->stream);
+  if (c->plan_stream != c->stream) cudaStreamSynchronize(c->plan_stream);
+  if (c->copy_stream != c->stream) cudaStreamSynchronize(c->copy_stream);
+}
+
+// Grow-only device buffer, zeroed when (re)allocated.  Growth needs a
+// synchronisation, so it is refused while the context's stream is captured.
 ro_status ensure(ro_ctx* c, DevBuf& b, size_t bytes, const char* what) {
   if (bytes == 0) bytes = 16;
   if (b.cap >= bytes) return RO_OK;
+  if (capture_id(c->stream))
+    return fail(c, RO_E_STATE, "%s must grow during stream capture: run the call once uncaptured first", what);
   if (b.p) {
-    cudaStreamSynchronize(c->stream);
+    sync_all_streams(c);   // the old buffer may be in use on any stream
     cudaFree(b.p);
     b.p = nullptr;
     b.cap = 0;
@@ -170,15 +227,57 @@ ro_status ensure(ro_ctx* c, DevBuf& b, size_t bytes, const char* what) {
   }
   b.cap = want;
   e = cudaMemsetAsync(b.p, 0, want, c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);   // zero before any stream uses it
   if (e != cudaSuccess) return cuda_fail(c, e, "cudaMemsetAsync");
   return RO_OK;
 }
 
-#define RO_TRY(x)                 \
-  do {                            \
-    ro_status _s = (x);           \
-    if (_s != RO_OK) return _s;   \
-  } while (0)
+ro_status ev_record(ro_ctx* c, Ev& ev, cudaStream_t s) {
+  if (!ev.e) {
+    cudaError_t e = cudaEventCreateWithFlags(&ev.e, cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(c, e, "cudaEventCreate");
+  }
+  cudaError_t e = cudaEventRecord(ev.e, s);
+  if (e != cudaSuccess) return cuda_fail(c, e, "cudaEventRecord");
+  ev.cap_id = capture_id(s);
+  ev.recorded = true;
+  return RO_OK;
+}
+
+// Make s wait for ev.  An event recorded in the capture that is now active on
+// the context's stream is waited on (pulling s into that capture if it is
+// not in it yet); an event recorded outside any capture is waited on only by
+// a stream that is not being captured; an event from a finished capture is
+// skipped.  What is skipped is ordered through the context's stream: a
+// captured graph joins its streams back into it, and the caller joins the
+// streams before it starts a capture.
+ro_status ev_wait(ro_ctx* c, const Ev& ev, cudaStream_t s) {
+  if (!ev.recorded) return RO_OK;
+  const unsigned long long cs = capture_id(s);
+  if (ev.cap_id == 0) {
+    if (cs != 0) return RO_OK;
+  } else {
+    const unsigned long long active = capture_id(c->stream);
+    if (ev.cap_id != active || (cs != 0 && cs != active)) return RO_OK;
+  }
+  cudaError_t e = cudaStreamWaitEvent(s, ev.e, 0);
+  if (e != cudaSuccess) return cuda_fail(c, e, "cudaStreamWaitEvent");
+  return RO_OK;
+}
+
+// from -> to: `to` waits for everything enqueued on `from` so far
+ro_status order(ro_ctx* c, Ev& ev, cudaStream_t from, cudaStream_t to) {
+  if (from == to) return RO_OK;
+  RO_TRY(ev_record(c, ev, from));
+  return ev_wait(c, ev, to);
+}
+
+// The context's stream waits for the plan and copy streams.
+ro_status join(ro_ctx* c) {
+  RO_TRY(order(c, c->join_plan, c->plan_stream, c->stream));
+  if (c->copy_stream != c->plan_stream) RO_TRY(order(c, c->join_copy, c->copy_stream, c->stream));
+  return RO_OK;
+}
 
 // Tile-status arrays of one scan slot (flags start zeroed: epoch 0, nothing
 // published; kernels keep their epochs on the device).
@@ -201,9 +300,10 @@ ro_status check_launch(ro_ctx* c, const char* what) {
   return RO_OK;
 }
 
-// Wait for the stream, mirror the device scalars and turn recorded
+// Wait for every stream, mirror the device scalars and turn recorded
 // conditions into a status (clearing them).
 ro_status sync_and_check(ro_ctx* c) {
+  RO_TRY(join(c));
   cudaError_t e = cudaMemcpyAsync(c->hs, c->ds, sizeof(DevScalars), cudaMemcpyDeviceToHost, c->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) return cuda_fail(c, e, "synchronise");
@@ -213,7 +313,7 @@ ro_status sync_and_check(ro_ctx* c) {
   if (err & ERR_TIMEOUT) return fail(c, RO_E_TIMEOUT, "a device-side wait timed out");
   if (err & ERR_OVERFLOW) return fail(c, RO_E_OVERFLOW, "an assembled parent exceeds 2^32-1 bytes");
   if (err & ERR_CAPACITY) return fail(c, RO_E_CAPACITY, "an output buffer is too small");
-  return fail(c, RO_E_INVAL, "a device count exceeded its host bound");
+  return fail(c, RO_E_INVAL, "a device count or arena offset exceeded its bound");
 }
 
 ro_status enter(ro_ctx* c) {
@@ -228,18 +328,6 @@ Expansion* get_exp(ro_ctx* c, int32_t xid) {
   return &c->exps[xid];
 }
 
-PlanBufs slot_plan(ExpSlot& S) {
-  PlanBufs pl;
-  pl.status = (uint8_t*)S.plan_status.p;
-  pl.off = (uint64_t*)S.plan_off.p;
-  pl.pbytes = (uint64_t*)S.plan_pbytes.p;
-  pl.pnz = (uint32_t*)S.plan_pnz.p;
-  pl.cpos = (uint64_t*)S.plan_cpos.p;
-  pl.csrc = (uint64_t*)S.plan_csrc.p;
-  pl.hdr = (PlanHdr*)S.plan_hdr.p;
-  return pl;
-}
-
 int grid_for(const void* k, int threads, int sms, int cap_per_sm, size_t dyn_smem = 0) {
   int per = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k, threads, dyn_smem) != cudaSuccess || per < 1) {
@@ -248,6 +336,41 @@ int grid_for(const void* k, int threads, int sms, int cap_per_sm, size_t dyn_sme
   }
   per = std::min(per, cap_per_sm);
   return per * sms;
+}
+
+void free_buf(DevBuf& b) {
+  if (b.p) cudaFree(b.p);
+  b.p = nullptr;
+  b.cap = 0;
+}
+void free_ev(Ev& e) {
+  if (e.e) cudaEventDestroy(e.e);
+  e = Ev{};
+}
+
+ListBufs list_bufs(ListSlot& s, uint64_t mtfp_cap) {
+  ListBufs l;
+  l.parents = (const uint32_t*)s.done.p;
+  l.status = (uint8_t*)s.status.p;
+  l.mb = (uint32_t*)s.mb.p;
+  l.coff = (uint32_t*)s.coff.p;
+  l.mtfp = (uint32_t*)s.mtfp.p;
+  l.mtfp_cap = mtfp_cap;
+  l.hdr = (ListHdr*)s.hdr.p;
+  return l;
+}
+
+PlanBufs plan_bufs(PlanSlot& s, uint64_t member_cap, bool with_status) {
+  PlanBufs p;
+  p.status = with_status ? (uint8_t*)s.status.p : nullptr;
+  p.off = (uint64_t*)s.off.p;
+  p.cpos = (uint64_t*)s.cpos.p;
+  p.csrc = (uint64_t*)s.csrc.p;
+  p.member_cap = member_cap;
+  p.ctfp = (uint32_t*)s.ctfp.p;
+  p.ctfp_cap = s.ctfp_cap;
+  p.hdr = (PlanHdr*)s.hdr.p;
+  return p;
 }
 
 }  // namespace
@@ -267,6 +390,8 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   ro_ctx* c = new ro_ctx();
   c->device = device;
   c->stream = (cudaStream_t)stream;
+  c->plan_stream = c->stream;
+  c->copy_stream = c->stream;
   c->n_calls = n_calls;
   cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
   if (cudaMalloc(&c->ds, sizeof(DevScalars)) != cudaSuccess ||
@@ -278,6 +403,13 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   }
   cudaMemsetAsync(c->ds, 0, sizeof(DevScalars), c->stream);
   std::memset(c->hs, 0, sizeof(DevScalars));
+  if (prepare_assemble_kernels() != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(c->ds);
+    cudaFreeHost(c->hs);
+    delete c;
+    return RO_E_CUDA;
+  }
   const int s = c->num_sms;
   c->L.stream = c->stream;
   c->L.prof = &c->prof;
@@ -288,14 +420,9 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_cfinish = grid_for(kernel_ptr_commit(K_CFINISH), CF_THREADS, s, 4);
   c->L.grid_aparents = grid_for(kernel_ptr_assemble(K_APARENTS), AP_THREADS, s, 4);
   c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 8);
-  if (prepare_assemble_kernels() != cudaSuccess) {
-    cudaGetLastError();
-    cudaFree(c->ds);
-    cudaFreeHost(c->hs);
-    delete c;
-    return RO_E_CUDA;
-  }
   c->L.grid_acopy = grid_for(kernel_ptr_assemble(K_ACOPY), AC_THREADS, s, 8, asm_copy_smem());
+  c->Lp = c->L;
+  c->Lc = c->L;
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) {
     cudaFree(c->ds);
@@ -310,25 +437,28 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
 ro_status ro_ctx_destroy(ro_ctx* c) {
   if (!c) return RO_E_INVAL;
   DeviceGuard g(c->device);
-  cudaStreamSynchronize(c->stream);
-  auto fr = [](DevBuf& b) {
-    if (b.p) cudaFree(b.p);
-    b.p = nullptr;
-    b.cap = 0;
-  };
+  sync_all_streams(c);
   for (auto& s : c->slots) {
-    fr(s.offsets); fr(s.pw); fr(s.phase); fr(s.rec); fr(s.bitmap); fr(s.done); fr(s.tfp);
-    fr(s.pm); fr(s.plan_status); fr(s.plan_off); fr(s.plan_pbytes); fr(s.plan_pnz);
-    fr(s.plan_cpos); fr(s.plan_csrc); fr(s.plan_hdr);
+    free_buf(s.offsets); free_buf(s.pw); free_buf(s.phase); free_buf(s.rec); free_buf(s.bitmap);
+    free_buf(s.tfp); free_buf(s.pm); free_buf(s.wm);
+    for (auto& l : s.lists) {
+      free_buf(l.done); free_buf(l.status); free_buf(l.mb); free_buf(l.coff); free_buf(l.mtfp);
+      free_buf(l.hdr); free_ev(l.freed);
+    }
+    for (auto& p : s.plans) {
+      free_buf(p.status); free_buf(p.off); free_buf(p.cpos); free_buf(p.csrc); free_buf(p.ctfp);
+      free_buf(p.hdr); free_ev(p.ready); free_ev(p.freed);
+    }
     for (auto& q : s.queues) {
-      fr(q.q);
-      fr(q.state);
+      free_buf(q.q);
+      free_buf(q.state);
     }
   }
   for (auto& t : c->ts) {
-    fr(t.flag); fr(t.agg); fr(t.inc);
+    free_buf(t.flag); free_buf(t.agg); free_buf(t.inc);
   }
-  fr(c->code); fr(c->mb); fr(c->mtfp); fr(c->cpos); fr(c->csrc); fr(c->as_off);
+  free_buf(c->code); free_buf(c->x_mb); free_buf(c->x_coff); free_buf(c->x_mtfp); free_buf(c->x_hdr);
+  free_ev(c->fork); free_ev(c->x_planned); free_ev(c->join_plan); free_ev(c->join_copy);
   for (cudaEvent_t e : c->prof.pool) cudaEventDestroy(e);
   cudaFree(c->ds);
   cudaFreeHost(c->hs);
@@ -338,9 +468,28 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
 
 ro_status ro_ctx_reset(ro_ctx* c) {
   if (!c) return RO_E_INVAL;
+  DeviceGuard g(c->device);
+  RO_TRY(join(c));   // the next expansion reuses buffers the other streams may still read
   c->exps.clear();
   c->err.clear();
   return RO_OK;
+}
+
+ro_status ro_ctx_set_streams(ro_ctx* c, void* plan_stream, void* copy_stream) {
+  RO_TRY(enter(c));
+  DeviceGuard g(c->device);
+  RO_TRY(join(c));
+  c->plan_stream = plan_stream ? (cudaStream_t)plan_stream : c->stream;
+  c->copy_stream = copy_stream ? (cudaStream_t)copy_stream : c->stream;
+  c->Lp.stream = c->plan_stream;
+  c->Lc.stream = c->copy_stream;
+  return RO_OK;
+}
+
+ro_status ro_ctx_join(ro_ctx* c) {
+  RO_TRY(enter(c));
+  DeviceGuard g(c->device);
+  return join(c);
 }
 
 ro_status ro_ctx_sync(ro_ctx* c) {
@@ -371,6 +520,7 @@ ro_status ro_ctx_profile_read(ro_ctx* c, uint64_t* launches, uint64_t* timed, do
                               uint32_t n_kernels) {
   RO_TRY(enter(c));
   DeviceGuard g(c->device);
+  RO_TRY(join(c));
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) return cuda_fail(c, e, "synchronise");
   Profiler& p = c->prof;
@@ -449,19 +599,29 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   if (N && (!d_child_parent || !d_child_ordinal))
     return fail(c, RO_E_INVAL, "ro_expand: NULL child arrays");
 
+  const uint64_t mtfp_cap = ceil_div(N, AM_TILE) + 2;
   RO_TRY(ensure(c, S.phase, N * sizeof(uint32_t), "phase words"));
   RO_TRY(ensure(c, S.rec, N * sizeof(Rec), "result records"));
   RO_TRY(ensure(c, S.bitmap, ceil_div(P, 32) * sizeof(uint32_t), "completion bitmap"));
-  RO_TRY(ensure(c, S.done, P * sizeof(uint32_t), "completed parents"));
-  RO_TRY(ensure(c, S.plan_status, P, "assembly plan"));
-  RO_TRY(ensure(c, S.plan_off, (P + 1) * sizeof(uint64_t), "assembly plan"));
-  RO_TRY(ensure(c, S.plan_pbytes, P * sizeof(uint64_t), "assembly plan"));
-  RO_TRY(ensure(c, S.plan_pnz, P * sizeof(uint32_t), "assembly plan"));
-  RO_TRY(ensure(c, S.plan_cpos, N * sizeof(uint64_t), "assembly plan"));
-  RO_TRY(ensure(c, S.plan_csrc, N * sizeof(uint64_t), "assembly plan"));
-  RO_TRY(ensure(c, S.plan_hdr, sizeof(PlanHdr), "assembly plan"));
   RO_TRY(ensure(c, S.pm, P * sizeof(uint32_t), "parent member counts"));
+  RO_TRY(ensure(c, S.wm, ceil_div(P, 32) * sizeof(uint32_t), "word member counts"));
+  for (auto& l : S.lists) {
+    RO_TRY(ensure(c, l.done, P * sizeof(uint32_t), "completed parents"));
+    RO_TRY(ensure(c, l.status, P, "completed parents"));
+    RO_TRY(ensure(c, l.mb, (P + 1) * sizeof(uint32_t), "member bases"));
+    RO_TRY(ensure(c, l.coff, P * sizeof(uint32_t), "member bases"));
+    RO_TRY(ensure(c, l.mtfp, mtfp_cap * sizeof(uint32_t), "member tiles"));
+    RO_TRY(ensure(c, l.hdr, sizeof(ListHdr), "list header"));
+  }
+  for (auto& p : S.plans) {
+    RO_TRY(ensure(c, p.status, P, "assembly plan"));
+    RO_TRY(ensure(c, p.off, (P + 1) * sizeof(uint64_t), "assembly plan"));
+    RO_TRY(ensure(c, p.cpos, N * sizeof(uint64_t), "assembly plan"));
+    RO_TRY(ensure(c, p.csrc, N * sizeof(uint64_t), "assembly plan"));
+    RO_TRY(ensure(c, p.hdr, sizeof(PlanHdr), "assembly plan"));
+  }
   cudaMemsetAsync(S.bitmap.p, 0, ceil_div(P, 32) * sizeof(uint32_t), c->stream);
+  cudaMemsetAsync(S.wm.p, 0, ceil_div(P, 32) * sizeof(uint32_t), c->stream);
   ExpandFillArgs fa{};
   fa.offsets = (const uint64_t*)S.offsets.p;
   fa.P = P;
@@ -553,6 +713,8 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
     return fail(c, RO_E_INVAL, "ro_gather_commit: done_cap below min(n, parents)");
   DeviceGuard g(c->device);
   ExpSlot& S = c->slots[xid];
+  const int ls = (int)(x->commits % RING);
+  ListSlot& LS = S.lists[ls];
   CommitArgs ca{};
   ca.n_host = n;
   ca.d_n = d_n;
@@ -569,6 +731,7 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.pw = (unsigned long long*)S.pw.p;
   ca.bitmap = (uint32_t*)S.bitmap.p;
   ca.pm = (uint32_t*)S.pm.p;
+  ca.wm = (uint32_t*)S.wm.p;
   if (d_code) {
     ca.code = d_code;
   } else {
@@ -576,17 +739,18 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
     ca.code = (uint8_t*)c->code.p;
   }
   ca.done_user = d_done_parents;
-  ca.done_int = (uint32_t*)S.done.p;
+  ca.done_int = (uint32_t*)LS.done.p;
   ca.n_done_out = d_n_done;
   ca.offsets = (const uint64_t*)S.offsets.p;
-  ca.plan = slot_plan(S);
+  ca.list = list_bufs(LS, ceil_div(x->N, AM_TILE) + 2);
   ca.ds = c->ds;
-  const uint64_t cf_tiles = ceil_div(ceil_div(x->P, 32), (uint64_t)CF_THREADS);
-  RO_TRY(tile_status(c, TS_COMMIT, cf_tiles, &ca.ts_done));
-  RO_TRY(tile_status(c, TS_COMMIT_BYTES, cf_tiles, &ca.ts_bytes));
+  RO_TRY(tile_status(c, TS_COMMIT, ceil_div(ceil_div(x->P, 32), (uint64_t)CF_THREADS), &ca.ts));
+  // the slot is free once the planning that read it (RING commits ago) is done
+  RO_TRY(ev_wait(c, LS.freed, c->stream));
   launch_commit(c->L, ca);
   RO_TRY(check_launch(c, "gather_commit"));
-  x->committed = true;
+  x->last_list = ls;
+  x->commits += 1;
   if (h_n_done) {
     ro_status st = sync_and_check(c);
     *h_n_done = c->hs->cm_n_done;
@@ -607,34 +771,23 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   if (!d_arena || !d_status || !d_out_off)
     return fail(c, RO_E_INVAL, "ro_assemble: NULL arena, status or offsets");
   if (out_cap && !d_out) return fail(c, RO_E_INVAL, "ro_assemble: NULL output");
-  if (!d_parents && !x->committed)
+  if (!d_parents && x->last_list < 0)
     return fail(c, RO_E_STATE, "ro_assemble: no commit on expansion %d to take parents from", xid);
   if (n_parents >= (1ull << 32)) return fail(c, RO_E_OVERFLOW, "ro_assemble: list of 2^32 or more");
+  if (arena_bytes >= MAX_ARENA) return fail(c, RO_E_OVERFLOW, "ro_assemble: arena of 2^48 bytes or more");
   DeviceGuard g(c->device);
   ExpSlot& S = c->slots[xid];
   const uint64_t member_cap = std::max<uint64_t>(x->N, 1);
   const uint64_t mtfp_cap = ceil_div(member_cap, AM_TILE) + 2;
-  AssembleArgs aa{};
-  aa.from_commit = d_parents ? 0 : 1;
-  if (d_parents) {
-    RO_TRY(ensure(c, c->mb, (n_parents + 1) * sizeof(uint32_t), "member bases"));
-    RO_TRY(ensure(c, c->mtfp, mtfp_cap * sizeof(uint32_t), "member tiles"));
-    RO_TRY(ensure(c, c->as_off, (n_parents + 1) * sizeof(uint64_t), "assembly offsets"));
-    RO_TRY(ensure(c, c->cpos, member_cap * sizeof(uint64_t), "member positions"));
-    RO_TRY(ensure(c, c->csrc, member_cap * sizeof(uint64_t), "member sources"));
-    aa.plan.status = nullptr;
-    aa.plan.off = (uint64_t*)c->as_off.p;
-    aa.plan.pbytes = nullptr;
-    aa.plan.pnz = nullptr;
-    aa.plan.cpos = (uint64_t*)c->cpos.p;
-    aa.plan.csrc = (uint64_t*)c->csrc.p;
-    aa.plan.hdr = &c->ds->as_hdr;
-    aa.st_src = nullptr;
-  } else {
-    aa.plan = slot_plan(S);
-    aa.st_src = (const uint8_t*)S.plan_status.p;
+  PlanSlot& PS = S.plans[x->assembles % RING];
+  // chunk table: one entry per 16 KB of output (the copy searches beyond it)
+  const uint64_t want_chunks = std::min<uint64_t>(ceil_div(out_cap, AC_CHUNK) + 2, 1ull << 31);
+  if (PS.ctfp_cap < want_chunks) {
+    RO_TRY(ensure(c, PS.ctfp, want_chunks * sizeof(uint32_t), "chunk table"));
+    PS.ctfp_cap = PS.ctfp.cap / sizeof(uint32_t);
   }
-  aa.list = d_parents;
+  AssembleArgs aa{};
+  aa.user_list = d_parents;
   aa.n_host = n_parents;
   aa.d_n = d_parents ? d_n_parents : nullptr;
   aa.P = x->P;
@@ -651,18 +804,52 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   aa.out_cap = out_cap;
   aa.cursor = d_out_cursor;
   aa.out_bytes = d_out_bytes;
-  aa.mb = (uint32_t*)c->mb.p;
-  aa.mtfp = (uint32_t*)c->mtfp.p;
-  aa.mtfp_cap = mtfp_cap;
-  aa.member_cap = member_cap;
+  aa.plan = plan_bufs(PS, member_cap, d_parents == nullptr);
   aa.ds = c->ds;
+  ListSlot* LS = nullptr;
   if (d_parents) {
+    // a caller's list may be longer than the expansion's parents (repeats)
+    RO_TRY(ensure(c, PS.off, (n_parents + 1) * sizeof(uint64_t), "assembly plan"));
+    aa.plan.off = (uint64_t*)PS.off.p;
+    RO_TRY(ensure(c, c->x_mb, (n_parents + 1) * sizeof(uint32_t), "member bases"));
+    RO_TRY(ensure(c, c->x_coff, std::max<uint64_t>(n_parents, 1) * sizeof(uint32_t), "member bases"));
+    RO_TRY(ensure(c, c->x_mtfp, mtfp_cap * sizeof(uint32_t), "member tiles"));
+    RO_TRY(ensure(c, c->x_hdr, sizeof(ListHdr), "list header"));
+    aa.list.parents = d_parents;
+    aa.list.status = d_status;
+    aa.list.mb = (uint32_t*)c->x_mb.p;
+    aa.list.coff = (uint32_t*)c->x_coff.p;
+    aa.list.mtfp = (uint32_t*)c->x_mtfp.p;
+    aa.list.mtfp_cap = mtfp_cap;
+    aa.list.hdr = (ListHdr*)c->x_hdr.p;
     RO_TRY(tile_status(c, TS_ASM_PARENTS, ceil_div(n_parents, (uint64_t)AP_THREADS * AP_ITEMS),
                        &aa.ts_parents));
-    RO_TRY(tile_status(c, TS_ASM_MEMBERS, ceil_div(member_cap, (uint64_t)AM_TILE), &aa.ts_members));
+  } else {
+    LS = &S.lists[x->last_list];
+    aa.list = list_bufs(*LS, mtfp_cap);
   }
-  launch_assemble(c->L, aa);
-  RO_TRY(check_launch(c, "assemble"));
+  RO_TRY(tile_status(c, TS_ASM_MEMBERS, ceil_div(member_cap, (uint64_t)AM_TILE), &aa.ts_members));
+
+  // planning follows everything enqueued on the context's stream so far,
+  // and the copy that last read this plan slot
+  RO_TRY(order(c, c->fork, c->stream, c->plan_stream));
+  RO_TRY(ev_wait(c, PS.freed, c->plan_stream));
+  launch_assemble_plan(c->Lp, aa);
+  RO_TRY(check_launch(c, "assemble (plan)"));
+  if (c->plan_stream != c->stream) {
+    if (LS) {
+      RO_TRY(ev_record(c, LS->freed, c->plan_stream));
+    } else {
+      // a caller's list is classified against the parents' counters as they
+      // are now: later commits wait for that
+      RO_TRY(order(c, c->x_planned, c->plan_stream, c->stream));
+    }
+  }
+  RO_TRY(order(c, PS.ready, c->plan_stream, c->copy_stream));
+  launch_assemble_copy(c->Lc, aa);
+  RO_TRY(check_launch(c, "assemble (copy)"));
+  if (c->copy_stream != c->plan_stream) RO_TRY(ev_record(c, PS.freed, c->copy_stream));
+  x->assembles += 1;
   if (h_out_bytes) {
     ro_status st = sync_and_check(c);
     *h_out_bytes = c->hs->as_bytes;

@@ -69,12 +69,21 @@ enum : uint32_t {
   ERR_INVAL = 8u,
 };
 
+// Header of a list of completed parents to assemble (see ListBufs).
+struct ListHdr {
+  unsigned long long n;      // listed parents
+  unsigned long long M;      // members of the listed Present parents
+  uint32_t err;              // the list cannot be planned (capacity)
+  uint32_t pad;
+  unsigned long long pad2;
+};
 // Header of an assembly plan (see PlanBufs).
 struct PlanHdr {
   unsigned long long n;      // listed parents
   unsigned long long bytes;  // bytes to assemble
   unsigned long long nnz;    // members that contribute bytes
-  unsigned long long pad;
+  uint32_t err;              // the plan is void (a capacity or arena check failed)
+  uint32_t chunks_ok;        // the chunk table covers every chunk
 };
 
 // Counters and small results that kernels hand to later kernels and to the
@@ -90,13 +99,10 @@ struct DevScalars {
   unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
   uint32_t rb_ticket, rb_err;
   // ro_gather_commit
-  unsigned long long cm_n, cm_conflicts, cm_n_done, cm_M;
+  unsigned long long cm_n, cm_conflicts, cm_n_done;
   uint32_t cm_fix_ticket, cm_fix_done;
   // ro_assemble
-  PlanHdr as_hdr;                 // plan of an explicit list
-  unsigned long long as_M;        // members of an explicit list's Present parents
   unsigned long long as_bytes;    // bytes of the latest assemble (host read-back)
-  uint32_t as_err, pad1;
   // dynamic tile counters / exit tickets / scan epochs, one per look-back kernel
   uint32_t tile_ctr[8];
   uint32_t exit_ctr[8];

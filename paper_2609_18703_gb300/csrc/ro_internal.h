@@ -112,16 +112,30 @@ struct ReadyArgs {
 };
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a);
 
-// ---- assembly plans ------------------------------------------------------------------
-// The plan of one list of completed parents: everything the copy needs, with
-// positions relative to the start of that call's output (header: PlanHdr).
+// ---- lists and plans -------------------------------------------------------------------
+// A list of parents to assemble with its member bases: produced by
+// commit_finish (the parents a commit completed) or by asm_parents (a
+// caller's list), consumed by asm_members.
+struct ListBufs {
+  const uint32_t* parents;    // listed parent ids
+  uint8_t* status;            // outcome per listed parent
+  uint32_t* mb;               // member base per listed parent (+ total at [n])
+  uint32_t* coff;             // first child of each listed parent
+  uint32_t* mtfp;             // member tile -> listed parent holding its first member
+  uint64_t mtfp_cap;
+  ListHdr* hdr;
+};
+// The assembly plan of a list: everything the copy needs, with positions
+// relative to the start of that call's output.  Produced by asm_members,
+// consumed by asm_copy.
 struct PlanBufs {
-  uint8_t* status;    // per listed parent
-  uint64_t* off;      // per listed parent: relative output offset; [n] = bytes
-  uint64_t* pbytes;   // scratch per listed parent: bytes, then their tile-local prefix
-  uint32_t* pnz;      // scratch per listed parent: contributing members, then prefix
-  uint64_t* cpos;     // per contributing member: relative output position
-  uint64_t* csrc;     // per contributing member: arena offset
+  uint8_t* status;            // outcome per listed parent, copied for asm_copy (or NULL)
+  uint64_t* off;              // relative output offset per listed parent (+ total at [n])
+  uint64_t* cpos;             // relative output position of each contributing member
+  uint64_t* csrc;             // arena offset of each contributing member
+  uint64_t member_cap;        // capacity of cpos / csrc
+  uint32_t* ctfp;             // relative 16 KB chunk -> member holding its first byte
+  uint64_t ctfp_cap;
   PlanHdr* hdr;
 };
 
@@ -141,25 +155,23 @@ struct CommitArgs {
   unsigned long long* pw;
   uint32_t* bitmap;
   uint32_t* pm;               // per parent: members to gather once complete (0: Suppressed)
+  uint32_t* wm;               // per bitmap word: sum of pm of the parents completed in this call
   uint8_t* code;              // user's or internal
   uint32_t* done_user;        // optional
-  uint32_t* done_int;
+  uint32_t* done_int;         // the list (a ring slot)
   uint64_t* n_done_out;       // optional device output
-  // assembly plan of the completed parents (consumed by ro_assemble(NULL))
   const uint64_t* offsets;
-  PlanBufs plan;
+  ListBufs list;              // written: the completed parents with member bases
   DevScalars* ds;
-  TileStatus<unsigned long long> ts_done;   // scan 1: completed parents
-  TileStatus<Pair64> ts_bytes;              // scan 2: (bytes, contributing members)
+  TileStatus<Pair64> ts;
 };
 void launch_commit(const LaunchCfg& L, const CommitArgs& a);
 
 // ---- ro_assemble ---------------------------------------------------------------------
 struct AssembleArgs {
-  const uint32_t* list;       // explicit list of parents (asm_parents / asm_members only)
+  const uint32_t* user_list;  // explicit list (asm_parents), or NULL: the commit's list
   uint64_t n_host;            // list length, or capacity of the per-parent outputs
   const uint64_t* d_n;        // device list length (optional, explicit list only)
-  int from_commit;            // 1: copy the latest commit's plan (no planning kernels)
   uint64_t P, N;
   const uint64_t* offsets;
   const unsigned long long* pw;
@@ -173,18 +185,17 @@ struct AssembleArgs {
   uint64_t out_cap;
   uint64_t* cursor;           // optional (device)
   uint64_t* out_bytes;        // optional (device)
-  PlanBufs plan;              // the commit's plan, or scratch filled by the planning kernels
-  const uint8_t* st_src;      // statuses to copy into status (commit plan), or NULL
-  // explicit lists: member bases and member-tile table
-  uint32_t* mb;
-  uint32_t* mtfp;
-  uint64_t mtfp_cap;
-  uint64_t member_cap;        // capacity of plan.cpos / plan.csrc
+  ListBufs list;
+  PlanBufs plan;
   DevScalars* ds;
   TileStatus<unsigned long long> ts_parents;
   TileStatus<Pair64> ts_members;
 };
-void launch_assemble(const LaunchCfg& L, const AssembleArgs& a);
+// the planning kernels (explicit lists: asm_parents then asm_members) and
+// the copy, each on its own stream
+void launch_assemble_plan(const LaunchCfg& L, const AssembleArgs& a);
+void launch_assemble_copy(const LaunchCfg& L, const AssembleArgs& a);
+
 
 
 }  // namespace ro

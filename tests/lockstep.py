@@ -36,10 +36,13 @@ def host(t: torch.Tensor, dtype, n: Optional[int] = None) -> np.ndarray:
 
 
 class Lockstep:
-    def __init__(self, n_calls: int = 1):
+    def __init__(self, n_calls: int = 1, streams: bool = False):
         self.o = OracleCtx(n_calls)
         self.stream = torch.cuda.current_stream()
         self.ctx = ro.ro_ctx_create(0, self.stream, n_calls)
+        if streams:   # assembly planning and copies on streams of their own
+            self.side = (torch.cuda.Stream(), torch.cuda.Stream())
+            ro.ro_ctx_set_streams(self.ctx, *self.side)
         self.N = {}
         self.P = {}
 

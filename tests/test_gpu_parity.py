@@ -122,11 +122,11 @@ def test_pipeline_tiny_config():
         ls.check_stats()
 
 
-@pytest.mark.parametrize("device_count", [False, True])
-def test_pipeline_docpage_small(device_count):
+@pytest.mark.parametrize("device_count,streams", [(False, False), (True, False), (False, True)])
+def test_pipeline_docpage_small(device_count, streams):
     lv = docpage(parents=2500, waves=16).top
     a = host_arena(lv)
-    with Lockstep() as ls:
+    with Lockstep(streams=streams) as ls:
         run_level(ls, lv, a, _arena_dev(a), device_count=device_count)
         ls.check_stats()
 
@@ -223,11 +223,12 @@ def test_duplicate_reports_first_in_array_order_wins(seed):
 
 
 # ------------------------------------------------------------ assemble corners
-def test_assemble_lists_cursor_capacity_and_alignment():
+@pytest.mark.parametrize("streams", [False, True])
+def test_assemble_lists_cursor_capacity_and_alignment(streams):
     rng = np.random.default_rng(9)
     P = 3000
     counts = rng.integers(0, 8, P).astype(np.uint32)
-    with Lockstep() as ls:
+    with Lockstep(streams=streams) as ls:
         ex = ls.expand(counts)
         x = ex["xid"]
         N = ls.N[x]
