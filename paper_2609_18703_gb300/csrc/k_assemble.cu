@@ -114,8 +114,10 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
     if (incomplete) atomicAdd(&s_incomplete, (unsigned long long)incomplete);
     unsigned long long total;
     unsigned long long excl = block_excl_scan(mine, s_scan, &total);
-    if (threadIdx.x == 0)
-      s_prefix = lookback_exclusive(a.ts_parents, tile, total, ds->epoch[TS_ASM_PARENTS], &ds->err);
+    if (threadIdx.x < 32) {  // one warp looks back
+      const auto pfx = lookback_exclusive(a.ts_parents, tile, total, ds->epoch[TS_ASM_PARENTS], &ds->err);
+      if (threadIdx.x == 0) s_prefix = pfx;
+    }
     __syncthreads();
     unsigned long long run = s_prefix + excl;
 #pragma unroll
@@ -213,37 +215,59 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
     }
     __syncthreads();
 
+    // my members gt .. gt+AM_ITEMS-1 are consecutive: one search finds the
+    // list entry holding the first, a walk over the member bases the rest
     const uint64_t gt = g0 + (uint64_t)threadIdx.x * AM_ITEMS;
+    constexpr uint64_t NONE = ~0ull;
+    uint64_t ridx[AM_ITEMS];
+    uint32_t par[AM_ITEMS];
+    uint32_t firsts = 0;   // bit k: member gt+k is its parent's first
+    {
+      uint64_t i = i_lo;
+      if (gt < M) {
+        if (staged) {
+          i = i_lo + last_le_u(s_mb, 0u, (uint32_t)R, gt);
+        } else {
+          uint64_t lo = i_lo, hi = i_hi + 1;
+          while (hi - lo > 1) {
+            const uint64_t mid = lo + ((hi - lo) >> 1);
+            if (L.mb[mid] <= gt) lo = mid; else hi = mid;
+          }
+          i = lo;
+        }
+      }
+      // no member of this tile lies past entry i_hi
+      auto mb_at = [&](uint64_t x) -> uint64_t { return staged ? s_mb[x - i_lo] : L.mb[x]; };
+      uint64_t mbi = gt < M ? mb_at(i) : 0;
+      uint64_t mbn = (gt < M && i < i_hi) ? mb_at(i + 1) : NONE;
+      uint64_t cof = gt < M ? (staged ? s_coff[i - i_lo] : L.coff[i]) : 0;
+#pragma unroll
+      for (int k = 0; k < AM_ITEMS; ++k) {
+        const uint64_t g = gt + k;
+        ridx[k] = NONE;
+        par[k] = (uint32_t)i;
+        if (g < M) {
+          while (g >= mbn) {   // member-less entries have equal bases and are passed over
+            ++i;
+            mbi = mbn;
+            mbn = (i < i_hi) ? mb_at(i + 1) : NONE;
+            cof = staged ? s_coff[i - i_lo] : L.coff[i];
+          }
+          par[k] = (uint32_t)i;
+          if (g == mbi) firsts |= 1u << k;
+          ridx[k] = cof + (g - mbi);
+        }
+      }
+    }
     uint32_t contrib[AM_ITEMS];
     uint64_t src[AM_ITEMS];
-    uint32_t par[AM_ITEMS];
-    bool first[AM_ITEMS];
     Pair64 mine{0, 0};
 #pragma unroll
     for (int k = 0; k < AM_ITEMS; ++k) {
-      const uint64_t g = gt + k;
       contrib[k] = 0;
       src[k] = 0;
-      par[k] = 0;
-      first[k] = false;
-      if (g >= M) continue;
-      uint64_t i, mbi, coff;
-      if (staged) {
-        const uint32_t kk = last_le_u(s_mb, 0u, (uint32_t)R, g);
-        i = i_lo + kk;
-        mbi = s_mb[kk];
-        coff = s_coff[kk];
-      } else {
-        uint64_t lo = i_lo, hi = i_hi + 1;
-        while (hi - lo > 1) {
-          const uint64_t mid = lo + ((hi - lo) >> 1);
-          if (L.mb[mid] <= g) lo = mid; else hi = mid;
-        }
-        i = lo;
-        mbi = L.mb[lo];
-        coff = L.coff[lo];
-      }
-      const Rec r = a.rec[coff + (g - mbi)];
+      if (ridx[k] == NONE) continue;
+      const Rec r = a.rec[ridx[k]];
       if (w_state(r.w) == ST_PRESENT && r.len) {
         contrib[k] = r.len;
         src[k] = w_off(r.w);
@@ -253,15 +277,15 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
           pl.hdr->err = 1u;
         }
       }
-      par[k] = (uint32_t)i;
-      first[k] = (g == mbi);
       mine.a += contrib[k];
       mine.b += contrib[k] ? 1ull : 0ull;
     }
     Pair64 total;
     Pair64 excl = block_excl_scan_pair(mine, s_scan, &total);
-    if (threadIdx.x == 0)
-      s_prefix = lookback_exclusive(a.ts_members, tile, total, ds->epoch[TS_ASM_MEMBERS], &ds->err);
+    if (threadIdx.x < 32) {  // one warp looks back
+      const auto pfx = lookback_exclusive(a.ts_members, tile, total, ds->epoch[TS_ASM_MEMBERS], &ds->err);
+      if (threadIdx.x == 0) s_prefix = pfx;
+    }
     __syncthreads();
     Pair64 run = s_prefix + excl;   // (bytes, contributing members) before my first item
 #pragma unroll
@@ -269,7 +293,7 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
       const uint64_t g = gt + k;
       if (g >= M) break;
       const uint64_t pos = run.a;
-      if (first[k]) {
+      if (firsts & (1u << k)) {
         // the parent starts here, and so do the member-less parents listed just before it
         pl.off[par[k]] = pos;
         for (int64_t q = (int64_t)par[k] - 1; q >= 0; --q) {
@@ -447,13 +471,20 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
-// Bounded wait on a stage barrier; false (and ERR_TIMEOUT) if it gave up.
-__device__ __forceinline__ bool stage_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
+// Bounded wait on a stage barrier for the phase of parity `parity`; false
+// (recording ERR_TIMEOUT and raising the CTA's abort flag) if it gave up or
+// another warp of the CTA already did.
+__device__ __forceinline__ bool stage_wait2(uint64_t* bar, uint32_t parity, uint32_t* err,
+                                            volatile uint32_t* abort) {
   for (uint32_t i = 0; i < (1u << 20); ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 255u && (ld_acquire(err) & ERR_TIMEOUT)) break;
+    if ((i & 255u) == 255u && (*abort || (ld_acquire(err) & ERR_TIMEOUT))) {
+      *abort = 1u;
+      return false;
+    }
   }
   atomicOr(err, ERR_TIMEOUT);
+  *abort = 1u;
   return false;
 }
 
@@ -470,11 +501,14 @@ struct CopyStage {
   unsigned long long j_lo;        // first member of the chunk
   uint32_t pstart[AC_PIECES + 1]; // output start of each piece (+ end), relative to wbase
   int32_t qbase[AC_PIECES];       // buffer offset of output byte wbase, per piece
-  __align__(16) unsigned char buf[AC_BUF + 64];
+  uint32_t pad2[3];
+  // the 16 bytes before buf (the end of qbase) may be read and ignored: a
+  // piece's first word can start before the piece's first staged block
+  __align__(16) unsigned char buf[AC_BUF + 32];
 };
 constexpr uint32_t AC_FALLBACK = 0xFFFFFFFFu;
 
-size_t asm_copy_smem() { return 2 * sizeof(CopyStage); }
+size_t asm_copy_smem() { return AC_STAGES * sizeof(CopyStage); }
 
 struct CopyCtx {
   const AssembleArgs* a;
@@ -504,8 +538,8 @@ __device__ __forceinline__ uint64_t warp_search(const uint64_t* pos, uint64_t n,
   return lo;
 }
 
-// Warp 0 stages chunk k: finds its members, builds the piece table and issues
-// one bulk copy per piece.
+// A producer warp stages chunk k: finds its members, builds the piece table
+// and issues one bulk copy per piece, completing on `bar`.
 __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_t* bar, int lane) {
   const uint64_t rs = k * AC_CHUNK;
   const uint64_t re = (rs + AC_CHUNK < c.S) ? rs + AC_CHUNK : c.S;
@@ -528,7 +562,7 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_
     st->vend = (uint32_t)(c.out_base + re - wbase);
   }
   const uint64_t arena = (uint64_t)(uintptr_t)c.a->arena;
-  bool fits = np <= AC_PIECES;
+  const bool fits = np <= AC_PIECES;   // then the aligned blocks fit AC_BUF too
   uint32_t roff = 0;   // running buffer offset (warp-uniform)
   if (fits) {
     for (uint64_t g = 0; g < np; g += 32) {
@@ -557,7 +591,6 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_
       }
       roff += __shfl_sync(0xffffffffu, inc, 31);
     }
-    fits = roff <= AC_BUF;
   }
   if (!fits) {
     if (lane == 0) {
@@ -572,7 +605,7 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_
     st->pstart[np] = (uint32_t)(c.out_base + re - wbase);
   }
   __syncwarp();
-  fence_proxy_async_smem();   // earlier generic reads of this buffer before async writes
+  fence_proxy_async_smem();   // earlier generic accesses of this stage before async writes
   if (lane == 0) mbar_arrive_tx(bar, roff);
   __syncwarp();
   for (uint64_t i = lane; i < np; i += 32) {
@@ -588,62 +621,78 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_
   }
 }
 
-// All threads: write the staged chunk as aligned 16-byte words.
-__device__ void emit_chunk(const CopyStage* st) {
-  const uint32_t np = st->np;
-  const uint32_t vbeg = st->vbeg, vend = st->vend;
+__device__ __forceinline__ uint4 lds128(const unsigned char* p) {
+  return *reinterpret_cast<const uint4*>(p);
+}
+// bytes A .. A+15 of the stage buffer (A may be down to -15)
+__device__ __forceinline__ uint4 stage_word(const CopyStage* st, int32_t A) {
+  const int32_t Aa = A & ~15;
+  return window16(lds128(st->buf + Aa), lds128(st->buf + Aa + 16), (uint32_t)(A & 15));
+}
+
+// Consumer warp cw writes words [w0, w1) of a staged chunk, a lane per
+// 16-byte word.  A word inside one piece is one shifted 16-byte read of the
+// stage; a word that meets a piece boundary merges its pieces' bytes.  The
+// chunk's first and last words may hold bytes of neighbouring chunks: only
+// the chunk's own bytes of them are written, byte by byte.
+__device__ void emit_range(const CopyStage* st, uint32_t cw, int lane) {
+  const uint32_t np = st->np, vbeg = st->vbeg, vend = st->vend;
   const uint64_t wbase = st->wbase;
+  const uint32_t nW = (vend + 15u) >> 4;
+  const uint32_t w0 = (nW * cw) / AC_CONSUMERS, w1 = (nW * (cw + 1)) / AC_CONSUMERS;
+  if (w0 >= w1) return;
+  const uint32_t first = (w0 * 16u > vbeg) ? w0 * 16u : vbeg;
+  uint32_t a = 0, b = np;   // the piece holding byte `first` (pstart[0] = vbeg)
+  while (b - a > 1) {
+    const uint32_t m = (a + b) >> 1;
+    if (st->pstart[m] <= first) a = m; else b = m;
+  }
+  uint32_t icur = a;
   const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll 1
-  for (uint32_t wr = threadIdx.x * 16u; wr < vend; wr += AC_THREADS * 16u) {
-    const uint32_t vlo = wr > vbeg ? wr : vbeg;
-    const uint32_t vhi = (wr + 16u < vend) ? wr + 16u : vend;
-    if (vlo >= vhi) continue;
-    // piece holding byte vlo
-    uint32_t lo_i = 0, hi_i = np;
-    while (hi_i - lo_i > 1) {
-      const uint32_t mid = (lo_i + hi_i) >> 1;
-      if (st->pstart[mid] <= vlo) lo_i = mid; else hi_i = mid;
-    }
-    uint32_t i = lo_i;
-    uint32_t lo = vlo - wr;
-    const uint32_t hiw = vhi - wr;
-    uint4 acc = zero;
-    for (;;) {
-      const uint32_t pe = st->pstart[i + 1] - wr;   // piece end, word-relative (may exceed 16)
-      const uint32_t hi = pe < hiw ? pe : hiw;
-      const int32_t q = st->qbase[i] + (int32_t)wr;
-      const int32_t A = (q + (int32_t)lo) & ~15;
-      const int32_t dl = q - A;
-      const uint4 x = *reinterpret_cast<const uint4*>(st->buf + A);
-      const uint4 y = *reinterpret_cast<const uint4*>(st->buf + A + 16);
-      const uint4 v = dl >= 0 ? window16(x, y, (uint32_t)dl) : window16(zero, x, (uint32_t)(16 + dl));
-      acc = (lo == 0u && hi == 16u) ? v : merge_piece(acc, v, lo, hi);
-      if (hi >= hiw) break;
-      lo = hi;
-      ++i;
-    }
-    const uint64_t W = wbase + wr;
-    if (vlo == wr && vhi == wr + 16u) {
-      *reinterpret_cast<uint4*>((uintptr_t)W) = acc;
-    } else {
-      // the chunk's first or last word: only its own bytes
-      const uint32_t vv[4] = {acc.x, acc.y, acc.z, acc.w};
+  for (uint32_t g = w0; g < w1; g += 32) {
+    const uint32_t w = g + (uint32_t)lane;
+    uint32_t i = icur;
+    if (w < w1) {
+      const uint32_t wr = w * 16u;
+      const uint32_t lo = wr > vbeg ? wr : vbeg;
+      const uint32_t hi = (wr + 16u < vend) ? wr + 16u : vend;
+      while (st->pstart[i + 1] <= lo) ++i;
+      uint4* dst = reinterpret_cast<uint4*>((uintptr_t)(wbase + wr));
+      if (lo == wr && hi == wr + 16u && st->pstart[i + 1] >= hi) {
+        *dst = stage_word(st, st->qbase[i] + (int32_t)wr);
+      } else {
+        uint4 acc = zero;
+        uint32_t l2 = lo;
+        for (;;) {
+          const uint32_t pe = st->pstart[i + 1];
+          const uint32_t h2 = pe < hi ? pe : hi;
+          acc = merge_piece(acc, stage_word(st, st->qbase[i] + (int32_t)wr), l2 - wr, h2 - wr);
+          if (h2 >= hi) break;
+          l2 = h2;
+          ++i;
+        }
+        if (lo == wr && hi == wr + 16u) {
+          *dst = acc;
+        } else {
+          const uint32_t vv[4] = {acc.x, acc.y, acc.z, acc.w};
+          uint8_t* d8 = reinterpret_cast<uint8_t*>(dst);
 #pragma unroll
-      for (int t = 0; t < 16; ++t)
-        if ((uint32_t)t >= vlo - wr && (uint32_t)t < vhi - wr)
-          *reinterpret_cast<uint8_t*>((uintptr_t)(W + t)) = (uint8_t)(vv[t >> 2] >> (8 * (t & 3)));
+          for (int t = 0; t < 16; ++t)
+            if ((uint32_t)t >= lo - wr && (uint32_t)t < hi - wr) d8[t] = (uint8_t)(vv[t >> 2] >> (8 * (t & 3)));
+        }
+      }
     }
+    icur = __shfl_sync(0xffffffffu, i, 31);
   }
 }
 
-// A chunk whose pieces do not fit a stage: warps copy slices straight from
-// global memory.
-__device__ void emit_chunk_direct(const CopyCtx& c, const CopyStage* st) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  constexpr uint64_t SLICE = AC_CHUNK / (AC_THREADS / 32);
+// A chunk whose pieces do not fit a stage: consumer warps copy slices of it
+// straight from global memory.
+__device__ void emit_direct(const CopyCtx& c, const CopyStage* st, uint32_t cw, int lane) {
+  constexpr uint64_t SLICE = (AC_CHUNK + AC_CONSUMERS - 1) / AC_CONSUMERS;
   const uint64_t rs = st->rel_s, re = st->rel_e;
-  uint64_t ra = rs + (uint64_t)warp * SLICE;
+  uint64_t ra = rs + (uint64_t)cw * SLICE;
   const uint64_t rb = (ra + SLICE < re) ? ra + SLICE : re;
   if (ra >= rb) return;
   uint64_t k = warp_search(c.cpos, c.Mnz, ra, lane);
@@ -656,10 +705,18 @@ __device__ void emit_chunk_direct(const CopyCtx& c, const CopyStage* st) {
   }
 }
 
-__global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a) {
+// The copy: per-parent outputs, then the chunks of the call's output, each
+// CTA taking every n_part-th chunk.  Warps 0..AC_PRODUCERS-1 stage chunks
+// into a ring of AC_STAGES stages (producer p takes the CTA's chunks i with
+// i % AC_PRODUCERS == p), the other warps write them out in order; full
+// and empty mbarriers per stage hand the stages back and forth.
+__global__ void __launch_bounds__(AC_THREADS, 2) asm_copy_kernel(AssembleArgs a) {
   wait_predecessor();
   extern __shared__ __align__(128) unsigned char ac_smem[];
-  __shared__ __align__(8) uint64_t bars[2];
+  __shared__ __align__(8) uint64_t full_bar[AC_STAGES];
+  __shared__ __align__(8) uint64_t empty_bar[AC_STAGES];
+  __shared__ uint32_t s_issued[AC_STAGES];
+  __shared__ uint32_t s_abort;
   CopyStage* stages = reinterpret_cast<CopyStage*>(ac_smem);
   DevScalars* ds = a.ds;
   const PlanHdr hdr = *a.plan.hdr;
@@ -707,50 +764,58 @@ __global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a)
       }
     }
     if (threadIdx.x == 0) {
-      mbar_init(&bars[0], 1);
-      mbar_init(&bars[1], 1);
+      for (int s = 0; s < AC_STAGES; ++s) {
+        mbar_init(&full_bar[s], 1);
+        mbar_init(&empty_bar[s], AC_CONSUMERS);
+        s_issued[s] = 0u;
+      }
+      s_abort = 0u;
       mbar_fence_init();
     }
     __syncthreads();
-    uint32_t phase[2] = {0u, 0u};
-    bool pending[2] = {false, false};
-    bool ok = true;
-    uint64_t k = blockIdx.x;
-    if (k < n_chunks) {
-      if (warp == 0) stage_chunk(c, k, &stages[0], &bars[0], lane);
-      pending[0] = true;
-    }
-    for (uint32_t it = 0; k < n_chunks && ok; k += n_part, ++it) {
-      const uint32_t s = it & 1u;
-      const uint64_t kn = k + n_part;
-      if (kn < n_chunks) {   // next chunk's loads overlap this chunk's writes
-        if (warp == 0) stage_chunk(c, kn, &stages[s ^ 1u], &bars[s ^ 1u], lane);
-        pending[s ^ 1u] = true;
+    volatile uint32_t* abort = &s_abort;
+    if (warp < AC_PRODUCERS) {
+      for (uint32_t i = (uint32_t)warp;; i += AC_PRODUCERS) {
+        const uint64_t k = blockIdx.x + (uint64_t)i * n_part;
+        if (k >= n_chunks) break;
+        const uint32_t s = i % AC_STAGES, u = i / AC_STAGES;
+        if (u > 0 && !stage_wait2(&empty_bar[s], (u - 1u) & 1u, &ds->err, abort)) break;
+        stage_chunk(c, k, &stages[s], &full_bar[s], lane);
+        if (lane == 0) s_issued[s] = u + 1u;
       }
-      ok = stage_wait(&bars[s], phase[s], &ds->err);
-      phase[s] ^= 1u;
-      pending[s] = false;
-      if (ok) {
+    } else {
+      const uint32_t cw = (uint32_t)(warp - AC_PRODUCERS);
+      for (uint32_t i = 0;; ++i) {
+        const uint64_t k = blockIdx.x + (uint64_t)i * n_part;
+        if (k >= n_chunks) break;
+        const uint32_t s = i % AC_STAGES, u = i / AC_STAGES;
+        if (!stage_wait2(&full_bar[s], u & 1u, &ds->err, abort)) break;
         if (stages[s].np == AC_FALLBACK)
-          emit_chunk_direct(c, &stages[s]);
+          emit_direct(c, &stages[s], cw, lane);
         else
-          emit_chunk(&stages[s]);
+          emit_range(&stages[s], cw, lane);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty_bar[s]);
       }
-      __syncthreads();
     }
-    // a wait that gave up: give outstanding copies a bounded chance to land
-    for (int s = 0; s < 2; ++s)
-      if (pending[s]) stage_wait(&bars[s], phase[s], &ds->err);
+    __syncthreads();
+    // a wait that gave up: give the copies still in flight a bounded chance
+    // to land before the CTA's shared memory is released
+    if (s_abort && threadIdx.x == 0) {
+      for (int s = 0; s < AC_STAGES; ++s) {
+        if (!s_issued[s]) continue;
+        for (uint32_t t = 0; t < (1u << 20); ++t)
+          if (mbar_try_wait(&full_bar[s], (s_issued[s] - 1u) & 1u)) break;
+      }
+    }
   }
   if (threadIdx.x == 0) {
-    __threadfence();
-    if (atomicAdd(&ds->exit_ctr[TS_ASM_COPY], 1u) == n_part - 1) {
+    if (ticket(&ds->exit_ctr[TS_ASM_COPY]) == n_part - 1) {
       if (!failed && a.cursor) *a.cursor = base + S;
       if (a.out_bytes) *a.out_bytes = S;
       ds->as_bytes = S;
       a.plan.hdr->err = 0u;   // the plan is consumed
       ds->exit_ctr[TS_ASM_COPY] = 0u;
-      __threadfence();
     }
   }
 }

@@ -42,6 +42,7 @@ __device__ __forceinline__ uint64_t commit_count(const CommitArgs& a) {
 
 __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a) {
   wait_predecessor();
+  allow_successor();
   __shared__ unsigned long long s_cnt[6];
   DevScalars* ds = a.ds;
   if (threadIdx.x < 6) s_cnt[threadIdx.x] = 0;
@@ -112,9 +113,11 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
         const unsigned n_tot = __popc(grp), n_bad = __popc(grp & badm);
         const unsigned long long delta =
             ((unsigned long long)n_bad << 32) - (unsigned long long)n_tot;
+        // the parent's size, loaded alongside the count (used if it completes)
+        const uint32_t size = (uint32_t)(__ldg(a.offsets + p + 1) - __ldg(a.offsets + p));
         const unsigned long long old = atomicAdd(a.pw + p, delta);
         if ((uint32_t)old == n_tot) {   // the last members: the parent is complete
-          const uint32_t m = (pw_bad(old) + n_bad) ? 0u : (uint32_t)(a.offsets[p + 1] - a.offsets[p]);
+          const uint32_t m = (pw_bad(old) + n_bad) ? 0u : size;
           a.pm[p] = m;
           if (m) atomicAdd(a.wm + (p >> 5), m);
           atomicOr(a.bitmap + (p >> 5), 1u << (p & 31));
@@ -279,12 +282,15 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
     __syncthreads();
     if (tile >= n_tiles) break;
     const uint64_t w = (uint64_t)tile * CF_THREADS + threadIdx.x;
-    const uint32_t bits = (w < n_words) ? a.bitmap[w] : 0u;
-    const uint32_t wsum = bits ? __ldcg(a.wm + w) : 0u;
+    const uint32_t bits = (w < n_words) ? __ldcg(a.bitmap + w) : 0u;
+    const uint32_t wsum0 = (w < n_words) ? __ldcg(a.wm + w) : 0u;   // loaded alongside the bits
+    const uint32_t wsum = bits ? wsum0 : 0u;
     Pair64 total;
     const Pair64 excl = block_excl_scan_pair(Pair64{(unsigned long long)__popc(bits), wsum}, s_scan, &total);
-    if (threadIdx.x == 0)
-      s_prefix = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_COMMIT], &ds->err);
+    if (threadIdx.x < 32) {  // one warp looks back
+      const auto pfx = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_COMMIT], &ds->err);
+      if (threadIdx.x == 0) s_prefix = pfx;
+    }
     __syncthreads();
     Pair64 run = s_prefix + excl;   // (completed parents, members) before my word
     if (bits) {
@@ -317,15 +323,13 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
     }
   }
   if (threadIdx.x == 0) {
-    __threadfence();
-    if (atomicAdd(&ds->exit_ctr[TS_COMMIT], 1u) == n_part - 1) {
+    if (ticket(&ds->exit_ctr[TS_COMMIT]) == n_part - 1) {
       ds->tile_ctr[TS_COMMIT] = 0u;
       ds->exit_ctr[TS_COMMIT] = 0u;
       ds->epoch[TS_COMMIT] += 1ull;
       ds->cm_conflicts = 0ull;
       ds->cm_fix_ticket = 0u;
       ds->cm_fix_done = 0u;
-      __threadfence();
     }
   }
 }

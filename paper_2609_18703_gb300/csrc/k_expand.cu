@@ -57,7 +57,10 @@ __global__ void __launch_bounds__(EXP_THREADS) expand_scan_kernel(ExpandScanArgs
     }
     Pair64 total;
     Pair64 excl = block_excl_scan_pair(mine, s_scan, &total);
-    if (threadIdx.x == 0) s_prefix = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_EXPAND], &ds->err);
+    if (threadIdx.x < 32) {  // one warp looks back
+      const auto pfx = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_EXPAND], &ds->err);
+      if (threadIdx.x == 0) s_prefix = pfx;
+    }
     __syncthreads();
     Pair64 run = s_prefix + excl;
 #pragma unroll

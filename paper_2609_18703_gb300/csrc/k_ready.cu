@@ -75,10 +75,8 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
     }
     if (k) atomicAdd(&ds->rb_kept, k);
     if (b) atomicAdd(&ds->rb_bad, b);
-    __threadfence();
-    if (atomicAdd(&ds->rb_ticket, 1u) == gridDim.x - 1) {
+    if (ticket(&ds->rb_ticket) == gridDim.x - 1) {
       // last CTA: plan the reservation
-      __threadfence();
       const unsigned long long K = ld_relaxed_u64(&ds->rb_kept);
       const unsigned long long head = a.qstate[0], tail = a.qstate[1];
       const unsigned long long L = tail - head, T = L + K;
@@ -102,7 +100,6 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
       ds->rb_kept = 0;
       ds->rb_bad = 0;
       ds->rb_ticket = 0u;
-      __threadfence();
     }
   }
 }
@@ -172,7 +169,10 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
     }
     unsigned long long total;
     unsigned long long excl = block_excl_scan(cnt, s_scan, &total);
-    if (threadIdx.x == 0) s_prefix = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_READY], &ds->err);
+    if (threadIdx.x < 32) {  // one warp looks back
+      const auto pfx = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_READY], &ds->err);
+      if (threadIdx.x == 0) s_prefix = pfx;
+    }
     __syncthreads();
     unsigned long long rank = s_prefix + excl;
 #pragma unroll

@@ -115,6 +115,12 @@ enum TileSlot { TS_EXPAND = 0, TS_READY = 1, TS_COMMIT = 2, TS_ASM_PARENTS = 3, 
 __device__ __forceinline__ void wait_predecessor() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
 }
+// Let the next kernel on the stream be scheduled now: it starts, and then
+// waits in wait_predecessor() until this grid has finished and its memory is
+// visible, so its launch overlaps this grid instead of following it.
+__device__ __forceinline__ void allow_successor() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 // ---- memory-order helpers --------------------------------------------------------
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
@@ -177,48 +183,80 @@ __device__ __forceinline__ void ts_publish(const TileStatus<T>& ts, uint32_t til
     ts.agg[tile] = v;
   else
     ts.inc[tile] = v;
-  __threadfence();
-  st_release_u64(ts.flag + tile, (epoch << 2) | kind);
+  st_release_u64(ts.flag + tile, (epoch << 2) | kind);   // orders the value before the flag
+}
+
+__device__ __forceinline__ unsigned long long warp_sum(unsigned long long v) {
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) v += __shfl_xor_sync(0xffffffffu, v, d);
+  return v;
+}
+__device__ __forceinline__ Pair64 warp_sum(Pair64 v) {
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) {
+    v.a += __shfl_xor_sync(0xffffffffu, v.a, d);
+    v.b += __shfl_xor_sync(0xffffffffu, v.b, d);
+  }
+  return v;
 }
 
 // Exclusive prefix of tile `tile` given its local aggregate (decoupled
-// look-back, one thread).  Tiles are claimed in increasing order by running
-// CTAs, so every predecessor is resident or done and each wait ends; the
-// waits are bounded anyway (SPIN_LIMIT) and record ERR_TIMEOUT.
+// look-back), computed by one whole warp: each step inspects the 32 nearest
+// predecessors not yet summed at once (lane l the l-th nearest), adds the
+// aggregates up to the nearest inclusive prefix and stops there, else moves
+// 32 tiles back.  Tiles are claimed in increasing order by running CTAs, so
+// every predecessor is resident or done and each wait ends; the waits are
+// bounded anyway (SPIN_LIMIT) and record ERR_TIMEOUT.  Every lane returns
+// the prefix.
 template <class T>
 __device__ T lookback_exclusive(const TileStatus<T>& ts, uint32_t tile, const T& local,
                                 unsigned long long epoch, uint32_t* err) {
+  const int lane = threadIdx.x & 31;
   if (tile == 0) {
-    ts_publish(ts, 0, local, 2ull, epoch);
+    if (lane == 0) ts_publish(ts, 0, local, 2ull, epoch);
+    __syncwarp();
     return T{};
   }
-  ts_publish(ts, tile, local, 1ull, epoch);
+  if (lane == 0) ts_publish(ts, tile, local, 1ull, epoch);
   T excl{};
-  int64_t j = (int64_t)tile - 1;
-  while (j >= 0) {
+  int64_t j = (int64_t)tile - 1;   // nearest predecessor not summed yet
+  for (;;) {
+    const int64_t mine = j - lane;
     unsigned long long f = 0;
     uint32_t spins = 0;
+    bool gave_up = false;
     for (;;) {
-      f = ld_acquire_u64(ts.flag + j);
-      if ((f >> 2) == epoch && (f & 3ull) != 0ull) break;
-      if (++spins > SPIN_LIMIT) break;
+      const bool ready = mine < 0 || (((f = ld_acquire_u64(ts.flag + mine)) >> 2) == epoch && (f & 3ull) != 0ull);
+      if (__all_sync(0xffffffffu, ready)) break;
+      ++spins;
+      bool stop = spins > SPIN_LIMIT;
       // once any wait of this context has given up, stop waiting at once
-      if ((spins & 1023u) == 0u && (ld_acquire(err) & ERR_TIMEOUT)) spins = SPIN_LIMIT + 1;
-      if (spins > SPIN_LIMIT) break;
+      if ((spins & 1023u) == 0u && lane == 0 && (ld_acquire(err) & ERR_TIMEOUT)) stop = true;
+      if (__any_sync(0xffffffffu, stop)) {
+        gave_up = true;
+        break;
+      }
       __nanosleep(64);
     }
-    if (spins > SPIN_LIMIT) {
-      atomicOr(err, ERR_TIMEOUT);
+    if (gave_up) {
+      if (lane == 0) atomicOr(err, ERR_TIMEOUT);
       break;
     }
-    if ((f & 3ull) == 2ull) {
-      excl = load_cg(ts.inc + j) + excl;
-      break;
+    // lanes past tile 0 count as an inclusive prefix of zero
+    const bool inclusive = mine < 0 || (f & 3ull) == 2ull;
+    const unsigned im = __ballot_sync(0xffffffffu, inclusive);
+    const int stop = im ? __ffs(im) - 1 : 32;
+    T v{};
+    if (mine >= 0) {
+      if (lane < stop) v = load_cg(ts.agg + mine);
+      else if (lane == stop) v = load_cg(ts.inc + mine);
     }
-    excl = load_cg(ts.agg + j) + excl;
-    --j;
+    excl = excl + warp_sum(v);
+    if (stop < 32) break;
+    j -= 32;
   }
-  ts_publish(ts, tile, excl + local, 2ull, epoch);
+  if (lane == 0) ts_publish(ts, tile, excl + local, 2ull, epoch);
+  __syncwarp();
   return excl;
 }
 
@@ -231,15 +269,23 @@ __device__ __forceinline__ uint32_t participants(uint64_t units) {
   return (uint32_t)(units < (uint64_t)gridDim.x ? units : (uint64_t)gridDim.x);
 }
 
+// Exit ticket: an add with acquire-release semantics at GPU scope, so
+// everything the CTA did before it (its thread 0 after a CTA barrier) is
+// visible to whoever draws the last ticket, and that CTA sees it all.
+__device__ __forceinline__ uint32_t ticket(uint32_t* ctr) {
+  uint32_t old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(ctr) : "memory");
+  return old;
+}
+
 // Called by thread 0 of every participating CTA on exit; the last one out
-// resets the tile counter and advances the epoch for the next launch.
+// resets the tile counter and advances the epoch for the next launch (the
+// end of the grid publishes them).
 __device__ __forceinline__ void retire_cta(DevScalars* ds, int slot, uint32_t n_part) {
-  __threadfence();
-  if (atomicAdd(&ds->exit_ctr[slot], 1u) == n_part - 1) {
+  if (ticket(&ds->exit_ctr[slot]) == n_part - 1) {
     ds->tile_ctr[slot] = 0u;
     ds->exit_ctr[slot] = 0u;
     ds->epoch[slot] += 1ull;
-    __threadfence();
   }
 }
 

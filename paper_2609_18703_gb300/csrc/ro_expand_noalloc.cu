@@ -73,7 +73,10 @@ expand_scan_noalloc_kernel(const uint32_t* counts, uint64_t P, uint64_t* offsets
     }
     Pair64 total;
     Pair64 excl = block_excl_scan_pair(mine, s_scan, &total);
-    if (threadIdx.x == 0) s_prefix = lookback_exclusive(ts, tile, total, epoch, &h->err);
+    if (threadIdx.x < 32) {  // one warp looks back
+      const auto pfx = lookback_exclusive(ts, tile, total, epoch, &h->err);
+      if (threadIdx.x == 0) s_prefix = pfx;
+    }
     __syncthreads();
     Pair64 run = s_prefix + excl;
 #pragma unroll
@@ -103,12 +106,10 @@ expand_scan_noalloc_kernel(const uint32_t* counts, uint64_t P, uint64_t* offsets
       h->n_children = 0;
       h->n_empty = 0;
     }
-    __threadfence();
-    if (atomicAdd(&h->exit_ctr, 1u) == gridDim.x - 1) {
+    if (ticket(&h->exit_ctr) == gridDim.x - 1) {
       h->tile_ctr = 0u;
       h->exit_ctr = 0u;
       h->epoch = epoch + 1ull;
-      __threadfence();
     }
   }
 }

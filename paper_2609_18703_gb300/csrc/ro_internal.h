@@ -21,10 +21,13 @@ constexpr int AP_THREADS = 256, AP_ITEMS = 4;                 // listed parents 
 constexpr int AM_THREADS = 256, AM_ITEMS = 8;                 // members per tile: 2048
 constexpr uint32_t AM_TILE = AM_THREADS * AM_ITEMS;
 constexpr uint32_t AM_SMEM_CAP = 4096;                        // listed parents staged per tile
-constexpr int AC_THREADS = 256;
+constexpr int AC_THREADS = 256;                               // 2 producer + 6 consumer warps
+constexpr int AC_PRODUCERS = 2, AC_CONSUMERS = AC_THREADS / 32 - AC_PRODUCERS;
+constexpr int AC_STAGES = 4;                                  // chunks staged per CTA
 constexpr uint64_t AC_CHUNK = 16384;                          // output bytes per copy chunk (relative)
-constexpr uint32_t AC_BUF = 26624;                            // staged source bytes per chunk
-constexpr uint32_t AC_PIECES = 640;                           // member pieces staged per chunk
+constexpr uint32_t AC_PIECES = 256;                           // member pieces staged per chunk
+constexpr uint32_t AC_BUF = 16384 + 32 * AC_PIECES;           // staged source bytes per chunk (fits any
+                                                              // AC_PIECES pieces: each adds < 32)
 
 // kernel entry points for occupancy queries and per-kernel timing
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CFINISH, K_APARENTS,
