@@ -334,20 +334,32 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
 // ---------------------------------------------------------------------------
 // Bytes sh .. sh+15 of the 32-byte window (x, y), sh in [0, 15].
 __device__ __forceinline__ uint4 window16(const uint4 x, const uint4 y, uint32_t sh) {
+  // branch-free: move the window by 8 bytes, then by 4, then funnel-shift
+  // the remaining 0..3 bytes (lanes with different shifts do not diverge)
+  const bool h8 = (sh & 8u) != 0u, h4 = (sh & 4u) != 0u;
+  const uint32_t b0 = h8 ? x.z : x.x, b1 = h8 ? x.w : x.y, b2 = h8 ? y.x : x.z;
+  const uint32_t b3 = h8 ? y.y : x.w, b4 = h8 ? y.z : y.x, b5 = h8 ? y.w : y.y;
+  const uint32_t a0 = h4 ? b1 : b0, a1 = h4 ? b2 : b1, a2 = h4 ? b3 : b2;
+  const uint32_t a3 = h4 ? b4 : b3, a4 = h4 ? b5 : b4;
   const uint32_t b = (sh & 3u) * 8u;
-  uint32_t a0, a1, a2, a3, a4;
-  switch (sh >> 2) {
-    case 0: a0 = x.x; a1 = x.y; a2 = x.z; a3 = x.w; a4 = y.x; break;
-    case 1: a0 = x.y; a1 = x.z; a2 = x.w; a3 = y.x; a4 = y.y; break;
-    case 2: a0 = x.z; a1 = x.w; a2 = y.x; a3 = y.y; a4 = y.z; break;
-    default: a0 = x.w; a1 = y.x; a2 = y.y; a3 = y.z; a4 = y.w; break;
-  }
   uint4 r;
   r.x = __funnelshift_r(a0, a1, b);
   r.y = __funnelshift_r(a1, a2, b);
   r.z = __funnelshift_r(a2, a3, b);
   r.w = __funnelshift_r(a3, a4, b);
   return r;
+}
+
+// v with its bytes from position b (0..16) on replaced by those of u
+__device__ __forceinline__ uint32_t keep_low(uint32_t v, uint32_t u, int b) {
+  const int c = b < 0 ? 0 : (b > 4 ? 4 : b);
+  const uint32_t m = (uint32_t)((1ull << (8 * c)) - 1ull);
+  return (v & m) | (u & ~m);
+}
+__device__ __forceinline__ uint4 take_from(const uint4 v, const uint4 u, uint32_t b) {
+  const int bi = (int)b;
+  return make_uint4(keep_low(v.x, u.x, bi), keep_low(v.y, u.y, bi - 4), keep_low(v.z, u.z, bi - 8),
+                    keep_low(v.w, u.w, bi - 12));
 }
 
 __device__ __forceinline__ uint4 shfl_down4(const uint4 v, int d) {
@@ -357,24 +369,6 @@ __device__ __forceinline__ uint4 shfl_down4(const uint4 v, int d) {
 __device__ __forceinline__ uint4 shfl_idx4(const uint4 v, int l) {
   return make_uint4(__shfl_sync(0xffffffffu, v.x, l), __shfl_sync(0xffffffffu, v.y, l),
                     __shfl_sync(0xffffffffu, v.z, l), __shfl_sync(0xffffffffu, v.w, l));
-}
-
-// 32-bit lane mask selecting bytes [lo, hi) of word q (0..3) of a 16-byte word.
-__device__ __forceinline__ uint32_t byte_mask(uint32_t lo, uint32_t hi, int q) {
-  const uint32_t m16 = ((1u << hi) - 1u) & ~((1u << lo) - 1u);   // hi <= 16
-  const uint32_t nib = (m16 >> (4 * q)) & 0xFu;
-  return ((nib & 1u) * 0xFFu) | ((nib & 2u) * 0x7F80u) | ((nib & 4u) * 0x3FC000u) |
-         ((nib & 8u) * 0x1FE00000u);
-}
-
-// acc with bytes [lo, hi) replaced by those of v
-__device__ __forceinline__ uint4 merge_piece(uint4 acc, const uint4 v, uint32_t lo, uint32_t hi) {
-  uint32_t m;
-  m = byte_mask(lo, hi, 0); acc.x = (acc.x & ~m) | (v.x & m);
-  m = byte_mask(lo, hi, 1); acc.y = (acc.y & ~m) | (v.y & m);
-  m = byte_mask(lo, hi, 2); acc.z = (acc.z & ~m) | (v.z & m);
-  m = byte_mask(lo, hi, 3); acc.w = (acc.w & ~m) | (v.w & m);
-  return acc;
 }
 
 constexpr int CP_UNROLL = 4;   // groups of 32 words in flight per warp
@@ -458,6 +452,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0u;
 }
+// The same wait, but the thread may sleep until the phase completes (or
+// about `ns` nanoseconds pass) instead of returning at once.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity), "r"(ns)
+      : "memory");
+  return ok != 0u;
+}
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -476,8 +481,9 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
 // another warp of the CTA already did.
 __device__ __forceinline__ bool stage_wait2(uint64_t* bar, uint32_t parity, uint32_t* err,
                                             volatile uint32_t* abort) {
+  // at most 2^20 polls of up to ~1 us each
   for (uint32_t i = 0; i < (1u << 20); ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait_sleep(bar, parity, 1000u)) return true;
     if ((i & 255u) == 255u && (*abort || (ld_acquire(err) & ERR_TIMEOUT))) {
       *abort = 1u;
       return false;
@@ -621,6 +627,83 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_
   }
 }
 
+// A chunk's pieces as a producer warp finds them.  With at most 32 pieces
+// each lane keeps one piece's source block range in registers, so the
+// chunk can be described (its global loads paid) before a stage is free and
+// staged later without touching global memory again.
+struct ChunkDesc {
+  uint64_t k, rs, re, j_lo, np, wbase;
+  bool inreg;                // np <= 32: the lane's piece below is valid if lane < np
+  uint64_t a0;               // the lane's piece: first aligned source block
+  uint32_t size, sh, ps;     // its staged bytes, source misalignment, output start (wbase-relative)
+};
+
+__device__ __forceinline__ void describe_chunk(const CopyCtx& c, uint64_t k, ChunkDesc& d, int lane) {
+  d.k = k;
+  d.rs = k * AC_CHUNK;
+  d.re = (d.rs + AC_CHUNK < c.S) ? d.rs + AC_CHUNK : c.S;
+  uint64_t j_hi;
+  if (c.ctfp) {
+    d.j_lo = c.ctfp[k];
+    j_hi = (k + 1 < c.n_chunks) ? c.ctfp[k + 1] : c.Mnz - 1;
+  } else {
+    d.j_lo = warp_search(c.cpos, c.Mnz, d.rs, lane);
+    j_hi = warp_search(c.cpos, c.Mnz, d.re - 1, lane);
+  }
+  d.np = j_hi - d.j_lo + 1;
+  d.wbase = (c.out_base + d.rs) & ~15ull;
+  d.inreg = d.np <= 32;
+  d.a0 = 0;
+  d.size = d.sh = d.ps = 0;
+  if (d.inreg && (uint64_t)lane < d.np) {
+    const uint64_t j = d.j_lo + lane;
+    const uint64_t p0 = c.cpos[j], p1 = cpos_at(c, j + 1);
+    const uint64_t ob = p0 > d.rs ? p0 : d.rs, oe = p1 < d.re ? p1 : d.re;
+    const uint64_t src = (uint64_t)(uintptr_t)c.a->arena + c.csrc[j] + (ob - p0);
+    d.a0 = src & ~15ull;
+    d.size = (uint32_t)(((src + (oe - ob) + 15) & ~15ull) - d.a0);
+    d.sh = (uint32_t)(src & 15u);
+    d.ps = (uint32_t)(c.out_base + ob - d.wbase);
+  }
+}
+
+// Stage a described chunk: piece table, expected bytes, one bulk copy per
+// piece.  Chunks of more than 32 pieces take stage_chunk's general path.
+__device__ void issue_chunk(const CopyCtx& c, const ChunkDesc& d, CopyStage* st, uint64_t* bar, int lane) {
+  if (!d.inreg) {
+    stage_chunk(c, d.k, st, bar, lane);
+    return;
+  }
+  uint32_t inc = d.size;
+#pragma unroll
+  for (int s = 1; s < 32; s <<= 1) {
+    const uint32_t t = __shfl_up_sync(0xffffffffu, inc, s);
+    if (lane >= s) inc += t;
+  }
+  const uint32_t my_off = inc - d.size;
+  const uint32_t roff = __shfl_sync(0xffffffffu, inc, 31);
+  if ((uint64_t)lane < d.np) {
+    st->pstart[lane] = d.ps;
+    st->qbase[lane] = (int32_t)(my_off + d.sh) - (int32_t)d.ps;
+  }
+  if (lane == 0) {
+    st->wbase = d.wbase;
+    st->rel_s = d.rs;
+    st->rel_e = d.re;
+    st->j_lo = d.j_lo;
+    st->vbeg = (uint32_t)(c.out_base + d.rs - d.wbase);
+    st->vend = (uint32_t)(c.out_base + d.re - d.wbase);
+    st->np = (uint32_t)d.np;
+    st->pstart[d.np] = (uint32_t)(c.out_base + d.re - d.wbase);
+  }
+  __syncwarp();
+  fence_proxy_async_smem();   // earlier generic accesses of this stage before async writes
+  if (lane == 0) mbar_arrive_tx(bar, roff);
+  __syncwarp();
+  if ((uint64_t)lane < d.np && d.size)
+    bulk_g2s(st->buf + my_off, reinterpret_cast<const void*>((uintptr_t)d.a0), d.size, bar);
+}
+
 __device__ __forceinline__ uint4 lds128(const unsigned char* p) {
   return *reinterpret_cast<const uint4*>(p);
 }
@@ -648,7 +731,6 @@ __device__ void emit_range(const CopyStage* st, uint32_t cw, int lane) {
     if (st->pstart[m] <= first) a = m; else b = m;
   }
   uint32_t icur = a;
-  const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll 1
   for (uint32_t g = w0; g < w1; g += 32) {
     const uint32_t w = g + (uint32_t)lane;
@@ -657,30 +739,29 @@ __device__ void emit_range(const CopyStage* st, uint32_t cw, int lane) {
       const uint32_t wr = w * 16u;
       const uint32_t lo = wr > vbeg ? wr : vbeg;
       const uint32_t hi = (wr + 16u < vend) ? wr + 16u : vend;
-      while (st->pstart[i + 1] <= lo) ++i;
+      uint32_t pe = st->pstart[i + 1];
+      while (pe <= lo) {
+        ++i;
+        pe = st->pstart[i + 1];
+      }
+      // bytes [lo, pe) come from piece i; a word that reaches further takes
+      // the rest from the following pieces, one boundary at a time
+      uint4 v = stage_word(st, st->qbase[i] + (int32_t)wr);
+      while (pe < hi) {
+        ++i;
+        v = take_from(v, stage_word(st, st->qbase[i] + (int32_t)wr), pe - wr);
+        pe = st->pstart[i + 1];
+      }
       uint4* dst = reinterpret_cast<uint4*>((uintptr_t)(wbase + wr));
-      if (lo == wr && hi == wr + 16u && st->pstart[i + 1] >= hi) {
-        *dst = stage_word(st, st->qbase[i] + (int32_t)wr);
+      if (lo == wr && hi == wr + 16u) {
+        *dst = v;
       } else {
-        uint4 acc = zero;
-        uint32_t l2 = lo;
-        for (;;) {
-          const uint32_t pe = st->pstart[i + 1];
-          const uint32_t h2 = pe < hi ? pe : hi;
-          acc = merge_piece(acc, stage_word(st, st->qbase[i] + (int32_t)wr), l2 - wr, h2 - wr);
-          if (h2 >= hi) break;
-          l2 = h2;
-          ++i;
-        }
-        if (lo == wr && hi == wr + 16u) {
-          *dst = acc;
-        } else {
-          const uint32_t vv[4] = {acc.x, acc.y, acc.z, acc.w};
-          uint8_t* d8 = reinterpret_cast<uint8_t*>(dst);
+        // the chunk's first or last word: only the chunk's own bytes
+        const uint32_t vv[4] = {v.x, v.y, v.z, v.w};
+        uint8_t* d8 = reinterpret_cast<uint8_t*>(dst);
 #pragma unroll
-          for (int t = 0; t < 16; ++t)
-            if ((uint32_t)t >= lo - wr && (uint32_t)t < hi - wr) d8[t] = (uint8_t)(vv[t >> 2] >> (8 * (t & 3)));
-        }
+        for (int t = 0; t < 16; ++t)
+          if ((uint32_t)t >= lo - wr && (uint32_t)t < hi - wr) d8[t] = (uint8_t)(vv[t >> 2] >> (8 * (t & 3)));
       }
     }
     icur = __shfl_sync(0xffffffffu, i, 31);
@@ -775,13 +856,20 @@ __global__ void __launch_bounds__(AC_THREADS, 2) asm_copy_kernel(AssembleArgs a)
     __syncthreads();
     volatile uint32_t* abort = &s_abort;
     if (warp < AC_PRODUCERS) {
-      for (uint32_t i = (uint32_t)warp;; i += AC_PRODUCERS) {
-        const uint64_t k = blockIdx.x + (uint64_t)i * n_part;
-        if (k >= n_chunks) break;
+      // each chunk is described before its stage frees up: the loads of
+      // chunk i+AC_PRODUCERS overlap the copies and the writing of chunk i
+      ChunkDesc d;
+      uint32_t i = (uint32_t)warp;
+      uint64_t k = blockIdx.x + (uint64_t)i * n_part;
+      if (k < n_chunks) describe_chunk(c, k, d, lane);
+      while (k < n_chunks) {
         const uint32_t s = i % AC_STAGES, u = i / AC_STAGES;
         if (u > 0 && !stage_wait2(&empty_bar[s], (u - 1u) & 1u, &ds->err, abort)) break;
-        stage_chunk(c, k, &stages[s], &full_bar[s], lane);
+        issue_chunk(c, d, &stages[s], &full_bar[s], lane);
         if (lane == 0) s_issued[s] = u + 1u;
+        i += AC_PRODUCERS;
+        k = blockIdx.x + (uint64_t)i * n_part;
+        if (k < n_chunks) describe_chunk(c, k, d, lane);
       }
     } else {
       const uint32_t cw = (uint32_t)(warp - AC_PRODUCERS);
