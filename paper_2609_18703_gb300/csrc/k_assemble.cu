@@ -176,12 +176,6 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
   const uint32_t n_part = participants((n_tiles > par_units ? n_tiles : par_units) + 1);
   if (blockIdx.x >= n_part) return;
 
-  // outcomes travel with the plan (the list's slot may be reused meanwhile)
-  if (pl.status) {
-    const uint64_t stride = (uint64_t)n_part * blockDim.x;
-    for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
-      pl.status[i] = L.status[i];
-  }
   if (M == 0) {   // nothing to gather: every listed parent starts at 0
     const uint64_t stride = (uint64_t)n_part * blockDim.x;
     for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i <= n; i += stride)
@@ -208,9 +202,10 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
     const uint64_t R = i_hi - i_lo + 1;
     const bool staged = R <= AM_SMEM_CAP;
     if (staged) {
-      for (uint64_t k = threadIdx.x; k < R; k += blockDim.x) {
-        s_mb[k] = L.mb[i_lo + k];
-        s_coff[k] = L.coff[i_lo + k];
+#pragma unroll 4
+      for (uint32_t k = threadIdx.x; k < (uint32_t)R; k += AM_THREADS) {
+        s_mb[k] = __ldcg(L.mb + i_lo + k);
+        s_coff[k] = __ldcg(L.coff + i_lo + k);
       }
     }
     __syncthreads();
@@ -836,7 +831,7 @@ __global__ void __launch_bounds__(AC_THREADS, 2) asm_copy_kernel(AssembleArgs a)
         const uint64_t o = a.plan.off[i];
         a.out_off[i] = base + o;
         if (i == n) break;
-        if (a.plan.status) a.status[i] = a.plan.status[i];
+        if (!a.user_list) a.status[i] = a.list.status[i];   // a caller's list has them already
         if (a.out_len) {
           const uint64_t len = a.plan.off[i + 1] - o;
           if (len > 0xFFFFFFFFull) atomicOr(&ds->err, ERR_OVERFLOW);

@@ -56,11 +56,11 @@ struct QueueBufs {
 // A list of completed parents (written by a commit, read by planning).
 struct ListSlot {
   DevBuf done, status, mb, coff, mtfp, hdr;
-  Ev freed;   // the planning that read it is done
+  Ev freed;   // the assembly that read it is done
 };
 // An assembly plan (written by planning, read by the copy).
 struct PlanSlot {
-  DevBuf status, off, cpos, csrc, ctfp, hdr;
+  DevBuf off, cpos, csrc, ctfp, hdr;
   uint64_t ctfp_cap = 0;
   Ev ready, freed;
 };
@@ -360,9 +360,8 @@ ListBufs list_bufs(ListSlot& s, uint64_t mtfp_cap) {
   return l;
 }
 
-PlanBufs plan_bufs(PlanSlot& s, uint64_t member_cap, bool with_status) {
+PlanBufs plan_bufs(PlanSlot& s, uint64_t member_cap) {
   PlanBufs p;
-  p.status = with_status ? (uint8_t*)s.status.p : nullptr;
   p.off = (uint64_t*)s.off.p;
   p.cpos = (uint64_t*)s.cpos.p;
   p.csrc = (uint64_t*)s.csrc.p;
@@ -419,7 +418,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_commit = grid_for(kernel_ptr_commit(K_COMMIT), CM_THREADS, s, 8);
   c->L.grid_cfinish = grid_for(kernel_ptr_commit(K_CFINISH), CF_THREADS, s, 4);
   c->L.grid_aparents = grid_for(kernel_ptr_assemble(K_APARENTS), AP_THREADS, s, 4);
-  c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 8);
+  c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 1);
   c->L.grid_acopy = grid_for(kernel_ptr_assemble(K_ACOPY), AC_THREADS, s, 8, asm_copy_smem());
   c->Lp = c->L;
   c->Lc = c->L;
@@ -446,7 +445,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
       free_buf(l.hdr); free_ev(l.freed);
     }
     for (auto& p : s.plans) {
-      free_buf(p.status); free_buf(p.off); free_buf(p.cpos); free_buf(p.csrc); free_buf(p.ctfp);
+      free_buf(p.off); free_buf(p.cpos); free_buf(p.csrc); free_buf(p.ctfp);
       free_buf(p.hdr); free_ev(p.ready); free_ev(p.freed);
     }
     for (auto& q : s.queues) {
@@ -614,7 +613,6 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
     RO_TRY(ensure(c, l.hdr, sizeof(ListHdr), "list header"));
   }
   for (auto& p : S.plans) {
-    RO_TRY(ensure(c, p.status, P, "assembly plan"));
     RO_TRY(ensure(c, p.off, (P + 1) * sizeof(uint64_t), "assembly plan"));
     RO_TRY(ensure(c, p.cpos, N * sizeof(uint64_t), "assembly plan"));
     RO_TRY(ensure(c, p.csrc, N * sizeof(uint64_t), "assembly plan"));
@@ -804,7 +802,7 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   aa.out_cap = out_cap;
   aa.cursor = d_out_cursor;
   aa.out_bytes = d_out_bytes;
-  aa.plan = plan_bufs(PS, member_cap, d_parents == nullptr);
+  aa.plan = plan_bufs(PS, member_cap);
   aa.ds = c->ds;
   ListSlot* LS = nullptr;
   if (d_parents) {
@@ -836,19 +834,17 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   RO_TRY(ev_wait(c, PS.freed, c->plan_stream));
   launch_assemble_plan(c->Lp, aa);
   RO_TRY(check_launch(c, "assemble (plan)"));
-  if (c->plan_stream != c->stream) {
-    if (LS) {
-      RO_TRY(ev_record(c, LS->freed, c->plan_stream));
-    } else {
-      // a caller's list is classified against the parents' counters as they
-      // are now: later commits wait for that
-      RO_TRY(order(c, c->x_planned, c->plan_stream, c->stream));
-    }
+  if (!LS && c->plan_stream != c->stream) {
+    // a caller's list is classified against the parents' counters as they
+    // are now: later commits wait for that
+    RO_TRY(order(c, c->x_planned, c->plan_stream, c->stream));
   }
   RO_TRY(order(c, PS.ready, c->plan_stream, c->copy_stream));
   launch_assemble_copy(c->Lc, aa);
   RO_TRY(check_launch(c, "assemble (copy)"));
   if (c->copy_stream != c->plan_stream) RO_TRY(ev_record(c, PS.freed, c->copy_stream));
+  // the copy reads the list's outcomes: the slot is free once it is done
+  if (LS && c->copy_stream != c->stream) RO_TRY(ev_record(c, LS->freed, c->copy_stream));
   x->assembles += 1;
   if (h_out_bytes) {
     ro_status st = sync_and_check(c);

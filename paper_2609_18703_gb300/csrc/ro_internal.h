@@ -132,7 +132,6 @@ struct ListBufs {
 // relative to the start of that call's output.  Produced by asm_members,
 // consumed by asm_copy.
 struct PlanBufs {
-  uint8_t* status;            // outcome per listed parent, copied for asm_copy (or NULL)
   uint64_t* off;              // relative output offset per listed parent (+ total at [n])
   uint64_t* cpos;             // relative output position of each contributing member
   uint64_t* csrc;             // arena offset of each contributing member
