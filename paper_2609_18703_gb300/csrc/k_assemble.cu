@@ -254,6 +254,17 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
         }
       }
     }
+    // all record loads first (no store in between), so they overlap
+    Rec rr[AM_ITEMS];
+#pragma unroll
+    for (int k = 0; k < AM_ITEMS; ++k) {
+      if (ridx[k] != NONE) {
+        rr[k] = a.rec[ridx[k]];
+      } else {
+        rr[k].len = 0;
+        rr[k].w = 0;
+      }
+    }
     uint32_t contrib[AM_ITEMS];
     uint64_t src[AM_ITEMS];
     Pair64 mine{0, 0};
@@ -261,8 +272,7 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
     for (int k = 0; k < AM_ITEMS; ++k) {
       contrib[k] = 0;
       src[k] = 0;
-      if (ridx[k] == NONE) continue;
-      const Rec r = a.rec[ridx[k]];
+      const Rec r = rr[k];
       if (w_state(r.w) == ST_PRESENT && r.len) {
         contrib[k] = r.len;
         src[k] = w_off(r.w);

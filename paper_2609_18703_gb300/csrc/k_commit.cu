@@ -296,19 +296,40 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
     if (bits) {
       uint32_t b = bits;
       while (b) {
-        const uint32_t parent = (uint32_t)(w * 32 + (__ffs(b) - 1));
-        b &= b - 1;
-        const uint32_t m = __ldcg(a.pm + parent);
-        const unsigned long long i = run.a;
-        a.done_int[i] = parent;
-        if (a.done_user) a.done_user[i] = parent;
-        L.status[i] = m ? ST_PRESENT : ST_SUPPRESSED;
-        L.mb[i] = (uint32_t)run.b;
-        L.coff[i] = (uint32_t)a.offsets[parent];
-        for (uint64_t t = ceil_div(run.b, AM_TILE); t * AM_TILE < run.b + m && t < L.mtfp_cap; ++t)
-          L.mtfp[t] = (uint32_t)i;
-        run.a += 1;
-        run.b += m;
+        // up to four completed parents at a time: their loads first, then
+        // the writes (a load after a store would wait for it)
+        constexpr int G = 4;
+        uint32_t par[G], m[G], cf[G];
+        int cnt = 0;
+#pragma unroll
+        for (int u = 0; u < G; ++u) {
+          if (b) {
+            par[u] = (uint32_t)(w * 32 + (__ffs(b) - 1));
+            b &= b - 1;
+            cnt = u + 1;
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < G; ++u) {
+          if (u < cnt) {
+            m[u] = __ldcg(a.pm + par[u]);
+            cf[u] = (uint32_t)__ldg(a.offsets + par[u]);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < G; ++u) {
+          if (u >= cnt) break;
+          const unsigned long long i = run.a;
+          a.done_int[i] = par[u];
+          if (a.done_user) a.done_user[i] = par[u];
+          L.status[i] = m[u] ? ST_PRESENT : ST_SUPPRESSED;
+          L.mb[i] = (uint32_t)run.b;
+          L.coff[i] = cf[u];
+          for (uint64_t t = ceil_div(run.b, AM_TILE); t * AM_TILE < run.b + m[u] && t < L.mtfp_cap; ++t)
+            L.mtfp[t] = (uint32_t)i;
+          run.a += 1;
+          run.b += m[u];
+        }
       }
       a.bitmap[w] = 0u;
       a.wm[w] = 0u;
