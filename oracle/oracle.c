@@ -31,8 +31,10 @@ typedef struct {
   uint8_t* st;              /* N: published outcome (Eq. 1) */
   uint32_t* len;            /* N: payload length of a Present value */
   uint64_t* off;            /* N: arena offset of a Present value */
+  uint8_t* by_barrier;      /* N: sealed by a sibling's GroupFailure */
   uint64_t* terminal;       /* P: members whose outcome has been published */
   uint8_t* bad;             /* P: a member is Failed or Suppressed */
+  uint8_t* barrier;         /* P: a GroupFailure suppressed the parent's open members */
   uint32_t** q;             /* per Call: FIFO Ready Queue storage (N slots) */
   uint64_t* qhead;
   uint64_t* qtail;
@@ -51,7 +53,7 @@ static void exp_free(or_exp* x) {
   if (!x) return;
   free(x->offsets); free(x->child_parent); free(x->child_call); free(x->phase);
   free(x->gen); free(x->st); free(x->len); free(x->off); free(x->terminal); free(x->bad);
-  free(x->last_done);
+  free(x->by_barrier); free(x->barrier); free(x->last_done);
   free(x);
 }
 
@@ -146,13 +148,15 @@ int or_expand(or_ctx* ctx, int32_t parent_xid, const uint32_t* counts, uint64_t 
   x->off = (uint64_t*)malloc((N ? N : 1) * sizeof(uint64_t));
   x->terminal = (uint64_t*)calloc(n_parents ? n_parents : 1, sizeof(uint64_t));
   x->bad = (uint8_t*)calloc(n_parents ? n_parents : 1, 1);
+  x->barrier = (uint8_t*)calloc(n_parents ? n_parents : 1, 1);
+  x->by_barrier = (uint8_t*)calloc(N ? N : 1, 1);
   x->last_done = (uint32_t*)malloc((n_parents ? n_parents : 1) * sizeof(uint32_t));
   x->q = (uint32_t**)calloc(ctx->n_calls, sizeof(uint32_t*));
   x->qhead = (uint64_t*)calloc(ctx->n_calls, sizeof(uint64_t));
   x->qtail = (uint64_t*)calloc(ctx->n_calls, sizeof(uint64_t));
   if (!x->offsets || !x->child_parent || !x->child_call || !x->phase || !x->gen || !x->st ||
-      !x->len || !x->off || !x->terminal || !x->bad || !x->last_done || !x->q || !x->qhead ||
-      !x->qtail) {
+      !x->len || !x->off || !x->terminal || !x->bad || !x->barrier || !x->by_barrier ||
+      !x->last_done || !x->q || !x->qhead || !x->qtail) {
     free(x->q); free(x->qhead); free(x->qtail);
     exp_free(x);
     return OR_E_OOM;
@@ -207,6 +211,16 @@ int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand
     if (!x->q[call]) return OR_E_OOM;
   }
   uint32_t* q = x->q[call];
+
+  /* queued Grains a GroupFailure sealed leave the queue undispatched */
+  uint64_t kept = x->qhead[call];
+  for (uint64_t t = x->qhead[call]; t < x->qtail[call]; ++t) {
+    if (x->phase[q[t]] == OR_READY)
+      q[kept++] = q[t];
+    else
+      ctx->stats.queue_dropped++;
+  }
+  x->qtail[call] = kept;
   uint64_t old_tail = x->qtail[call];
 
   /* admission: candidates in order; only WAITING Grains of this Call enter */
@@ -252,7 +266,10 @@ static int cmp_u32(const void* a, const void* b) {
  * an admitted report moves the Grain to SEALED and records its outcome
  * (Eq. 1), after which nothing can change it.  A parent is complete once all
  * of its children have a recorded outcome (Section 4.2, Reduce).  Reports
- * are applied one after another in array order.                            */
+ * are applied one after another in array order.  A GroupFailure report
+ * (Section 4.4, Figure 5) fails its own Grain and then suppresses the
+ * parent's other open Grains: queued ones will never be dispatched, and the
+ * later reports of in-flight ones are rejected.                            */
 int or_gather_commit(or_ctx* ctx, int32_t xid, uint64_t n, const uint32_t* child,
                      const uint8_t* state, const uint32_t* len, const uint64_t* off,
                      const uint32_t* gen, uint64_t arena_bytes, uint8_t* code,
@@ -269,7 +286,7 @@ int or_gather_commit(or_ctx* ctx, int32_t xid, uint64_t n, const uint32_t* child
     uint32_t g = gen ? gen[r] : 0;
     uint8_t v;
     int valid_state = (s == OR_PRESENT || s == OR_DROPPED || s == OR_FAILED ||
-                       s == OR_SUPPRESSED);
+                       s == OR_SUPPRESSED || s == OR_GROUP_FAILURE);
     int in_bounds = (s != OR_PRESENT) || (off[r] <= arena_bytes && len[r] <= arena_bytes - off[r]);
     if (c >= x->N || !valid_state || !in_bounds) {
       v = OR_REJ_INVALID;
@@ -278,17 +295,38 @@ int or_gather_commit(or_ctx* ctx, int32_t xid, uint64_t n, const uint32_t* child
     } else if (g != x->gen[c]) {
       v = OR_REJ_STALE_GEN;
     } else if (x->phase[c] == OR_SEALED) {
-      v = OR_REJ_DUPLICATE;
+      v = x->by_barrier[c] ? OR_REJ_BARRIER : OR_REJ_DUPLICATE;
     } else {
       v = OR_ACCEPT;
       x->phase[c] = OR_SEALED;
-      x->st[c] = s;
+      x->st[c] = (s == OR_GROUP_FAILURE) ? OR_FAILED : s;   /* the reporting Grain failed */
       x->len[c] = (s == OR_PRESENT) ? len[r] : 0;
       x->off[c] = (s == OR_PRESENT) ? off[r] : 0;
       uint32_t p = x->child_parent[c];
       x->terminal[p] += 1;
-      if (s == OR_FAILED || s == OR_SUPPRESSED) x->bad[p] = 1;
+      if (s == OR_FAILED || s == OR_SUPPRESSED || s == OR_GROUP_FAILURE) x->bad[p] = 1;
       if (x->terminal[p] == member_count(x, p)) x->last_done[k++] = p;
+      if (s == OR_GROUP_FAILURE && !x->barrier[p]) {
+        /* the barrier for (Call, parent): every sibling not yet sealed is
+           suppressed now, queued or in flight; sealed ones keep their facts */
+        x->barrier[p] = 1;
+        uint64_t sealed_now = 0;
+        for (uint64_t d = x->offsets[p]; d < x->offsets[p + 1]; ++d) {
+          if (x->phase[d] == OR_SEALED) continue;
+          if (x->phase[d] == OR_IN_FLIGHT)
+            ctx->stats.barrier_in_flight++;
+          else
+            ctx->stats.barrier_not_dispatched++;
+          x->phase[d] = OR_SEALED;
+          x->st[d] = OR_SUPPRESSED;
+          x->len[d] = 0;
+          x->off[d] = 0;
+          x->by_barrier[d] = 1;
+          x->terminal[p] += 1;
+          ++sealed_now;
+        }
+        if (sealed_now && x->terminal[p] == member_count(x, p)) x->last_done[k++] = p;
+      }
     }
     if (code) code[r] = v;
     switch (v) {
@@ -296,6 +334,7 @@ int or_gather_commit(or_ctx* ctx, int32_t xid, uint64_t n, const uint32_t* child
       case OR_REJ_INVALID: ctx->stats.rej_invalid++; break;
       case OR_REJ_NOT_INFLIGHT: ctx->stats.rej_not_inflight++; break;
       case OR_REJ_STALE_GEN: ctx->stats.rej_stale_gen++; break;
+      case OR_REJ_BARRIER: ctx->stats.rej_barrier++; break;
       default: ctx->stats.rej_duplicate++; break;
     }
   }

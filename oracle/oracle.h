@@ -24,9 +24,14 @@ enum { OR_OK = 0, OR_E_INVAL = 1, OR_E_CAPACITY = 2, OR_E_OVERFLOW = 3, OR_E_STA
        OR_E_OOM = 5 };
 /* Item outcomes of Eq. (1) as carried by reports and assembled parents */
 enum { OR_PENDING = 0, OR_PRESENT = 1, OR_DROPPED = 2, OR_FAILED = 3, OR_SUPPRESSED = 4 };
-/* per-report verdicts of the generation fence, Eq. (3) */
+/* A report kind, not an outcome (Section 4.4, typed GroupFailure): the
+ * reporting Grain Failed and its siblings under the same (Call, parent)
+ * are to be suppressed. */
+enum { OR_GROUP_FAILURE = 5 };
+/* per-report verdicts of the generation fence, Eq. (3); BARRIER: the Grain
+ * was sealed by a GroupFailure of a sibling */
 enum { OR_ACCEPT = 0, OR_REJ_INVALID = 1, OR_REJ_NOT_INFLIGHT = 2, OR_REJ_STALE_GEN = 3,
-       OR_REJ_DUPLICATE = 4 };
+       OR_REJ_DUPLICATE = 4, OR_REJ_BARRIER = 5 };
 /* Grain phases of Eq. (2) */
 enum { OR_WAITING = 0, OR_READY = 1, OR_IN_FLIGHT = 2, OR_SEALED = 3 };
 
@@ -36,6 +41,10 @@ typedef struct {
   uint64_t accepted, rej_invalid, rej_not_inflight, rej_stale_gen, rej_duplicate;
   uint64_t ready_bad_candidates;    /* candidates naming no child of the expansion */
   uint64_t assemble_incomplete;     /* listed parents that were not complete */
+  uint64_t rej_barrier;             /* reports for Grains a GroupFailure suppressed */
+  uint64_t barrier_not_dispatched;  /* siblings suppressed while WAITING or READY */
+  uint64_t barrier_in_flight;       /* siblings suppressed while IN-FLIGHT */
+  uint64_t queue_dropped;           /* suppressed Grains removed from a Ready Queue */
 } or_stats;
 
 or_ctx* or_ctx_create(uint32_t n_calls);
@@ -51,13 +60,17 @@ int or_expand(or_ctx* ctx, int32_t parent_xid, const uint32_t* counts, uint64_t 
               uint32_t* child_ordinal, uint64_t child_cap, uint32_t* empty_parents,
               uint64_t* n_children, uint64_t* n_empty, int32_t* xid);
 
-/* Per-Call FIFO Ready Queue with elastic reservation (Section 4.3, Eq. 2). */
+/* Per-Call FIFO Ready Queue with elastic reservation (Section 4.3, Eq. 2).
+ * Queued Grains that a GroupFailure suppressed leave the queue at the next
+ * reservation without being dispatched (Section 4.4). */
 int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand,
                    uint64_t n_cand, uint32_t batch_size, int32_t flush, uint32_t* batched,
                    uint64_t batched_cap, uint64_t* n_batched, uint64_t* n_batches);
 
 /* Generation-fenced commit (Section 4.4, Eq. 3) and parent completion
- * (Section 4.2, Reduce); completed parents listed ascending. */
+ * (Section 4.2, Reduce); completed parents listed ascending.  An accepted
+ * OR_GROUP_FAILURE report seals its Grain Failed and then suppresses every
+ * sibling not yet sealed (Section 4.4, Figure 5). */
 int or_gather_commit(or_ctx* ctx, int32_t xid, uint64_t n, const uint32_t* child,
                      const uint8_t* state, const uint32_t* len, const uint64_t* off,
                      const uint32_t* gen, uint64_t arena_bytes, uint8_t* code,

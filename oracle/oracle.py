@@ -19,7 +19,8 @@ from .build import LIB, build
 
 OK, E_INVAL, E_CAPACITY, E_OVERFLOW, E_STATE, E_OOM = range(6)
 PENDING, PRESENT, DROPPED, FAILED, SUPPRESSED = range(5)
-ACCEPT, REJ_INVALID, REJ_NOT_INFLIGHT, REJ_STALE_GEN, REJ_DUPLICATE = range(5)
+GROUP_FAILURE = 5   # report kind (Section 4.4): the Grain failed and its open siblings are suppressed
+ACCEPT, REJ_INVALID, REJ_NOT_INFLIGHT, REJ_STALE_GEN, REJ_DUPLICATE, REJ_BARRIER = range(6)
 
 _u8p = C.POINTER(C.c_uint8)
 _u32p = C.POINTER(C.c_uint32)
@@ -36,7 +37,8 @@ class OracleError(RuntimeError):
 class _Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in (
         "accepted", "rej_invalid", "rej_not_inflight", "rej_stale_gen", "rej_duplicate",
-        "ready_bad_candidates", "assemble_incomplete")]
+        "ready_bad_candidates", "assemble_incomplete", "rej_barrier", "barrier_not_dispatched",
+        "barrier_in_flight", "queue_dropped")]
 
 
 _lib = None

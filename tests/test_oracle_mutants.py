@@ -18,7 +18,7 @@ MUTANTS = {
     "fence_ignores_generation": ("} else if (g != x->gen[c]) {", "} else if (0) {"),
     "completion_off_by_one": ("if (x->terminal[p] == member_count(x, p)) x->last_done[k++] = p;",
                               "if (x->terminal[p] + 1 == member_count(x, p)) x->last_done[k++] = p;"),
-    "dropped_suppresses": ("if (s == OR_FAILED || s == OR_SUPPRESSED) x->bad[p] = 1;",
+    "dropped_suppresses": ("if (s == OR_FAILED || s == OR_SUPPRESSED || s == OR_GROUP_FAILURE) x->bad[p] = 1;",
                            "if (s != OR_PRESENT) x->bad[p] = 1;"),
     "source_index_shift": ("memcpy(out + pos, arena + x->off[c], x->len[c]);",
                            "memcpy(out + pos, arena + x->off[c] + 1, x->len[c]);"),
@@ -27,6 +27,15 @@ MUTANTS = {
                            "x->off[c] = (s == OR_PRESENT) ? len[r] : 0;"),
     "scan_extra_term": ("offsets[p + 1] = offsets[p] + counts[p];",
                         "offsets[p + 1] = offsets[p] + counts[p] + (p == 1);"),
+    # GroupFailure containment (Section 4.4)
+    "barrier_spares_queued": ("if (x->phase[d] == OR_SEALED) continue;",
+                              "if (x->phase[d] != OR_IN_FLIGHT) continue;"),
+    "barrier_reseals_committed": ("if (x->phase[d] == OR_SEALED) continue;", "if (d == c) continue;"),
+    "queue_keeps_suppressed": ("if (x->phase[q[t]] == OR_READY)", "if (1)"),
+    "barrier_verdict_lost": ("v = x->by_barrier[c] ? OR_REJ_BARRIER : OR_REJ_DUPLICATE;",
+                             "v = OR_REJ_DUPLICATE;"),
+    "barrier_completion_missed": ("if (sealed_now && x->terminal[p] == member_count(x, p)) x->last_done[k++] = p;",
+                                  "(void)sealed_now;"),
 }
 
 
@@ -42,6 +51,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
                     str(tmp_path / "oracle.c")], check=True)
     env = dict(os.environ, ORACLE_LIB=str(so))
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
-                        os.path.join(ROOT, "tests", "test_oracle.py")],
+                        os.path.join(ROOT, "tests", "test_oracle.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_group_failure.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode != 0, f"pins did not catch mutant {name}:\n{r.stdout[-2000:]}"
