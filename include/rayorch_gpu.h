@@ -76,6 +76,14 @@ enum {
   RO_FAILED = 3,
   RO_SUPPRESSED = 4
 };
+/* A report kind that is not an outcome (Section 4.4, typed GroupFailure):
+ * the reporting Grain failed (it is sealed RO_FAILED) and a barrier is
+ * installed for its (Call, parent): every sibling not yet sealed is sealed
+ * RO_SUPPRESSED at once.  Queued siblings then leave the Ready Queue at the
+ * next reservation without being dispatched, later reports of in-flight
+ * siblings are rejected (RO_REJ_BARRIER), siblings sealed earlier keep their
+ * facts and other parents are unaffected. */
+enum { RO_GROUP_FAILURE = 5 };
 
 /* per-report verdict of the generation fence, Eq. (3) */
 enum {
@@ -83,8 +91,9 @@ enum {
   RO_REJ_INVALID = 1,       /* no such child, unknown outcome, or payload outside the arena */
   RO_REJ_NOT_INFLIGHT = 2,  /* the child's Grain is WAITING or READY */
   RO_REJ_STALE_GEN = 3,     /* generation differs from the Grain's current one */
-  RO_REJ_DUPLICATE = 4      /* the Grain is already SEALED (earlier report, or an earlier
+  RO_REJ_DUPLICATE = 4,     /* the Grain is already SEALED (earlier report, or an earlier
                                report of the same call) */
+  RO_REJ_BARRIER = 5        /* the Grain was sealed by a sibling's GroupFailure */
 };
 
 /* cumulative counters of a context (since create or the last reset) */
@@ -92,6 +101,10 @@ typedef struct {
   uint64_t accepted, rej_invalid, rej_not_inflight, rej_stale_gen, rej_duplicate;
   uint64_t ready_bad_candidates;  /* batch_ready candidates naming no child */
   uint64_t assemble_incomplete;   /* assembled list entries that were not complete */
+  uint64_t rej_barrier;           /* reports rejected with RO_REJ_BARRIER */
+  uint64_t barrier_not_dispatched;/* siblings a GroupFailure sealed while WAITING or READY */
+  uint64_t barrier_in_flight;     /* siblings a GroupFailure sealed while IN-FLIGHT */
+  uint64_t queue_dropped;         /* sealed Grains removed from a Ready Queue undispatched */
 } ro_stats;
 
 /* ------------------------------------------------------------------------
@@ -207,12 +220,14 @@ ro_status ro_batch_ready(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t
  * Eq. 3) and per-parent completion (Section 4.2, Reduce).
  *
  * Report r names child d_child[r] with outcome d_state[r] (RO_PRESENT,
- * RO_DROPPED, RO_FAILED or RO_SUPPRESSED); a Present report's value is the
+ * RO_DROPPED, RO_FAILED or RO_SUPPRESSED) or the kind RO_GROUP_FAILURE
+ * (Section 4.4, see above); a Present report's value is the
  * d_len[r] bytes at arena offset d_arena_off[r] (ignored for other outcomes).
  * A report is accepted when the child's Grain is IN-FLIGHT and d_gen[r] is
  * its current generation; the Grain becomes SEALED and the outcome is
  * published for good.  Reports of one call are applied as if one after
- * another in array order (the first of several reports for one Grain wins).
+ * another in array order (the first of several reports for one Grain wins;
+ * a GroupFailure's barrier applies to the reports after it, not before).
  * A parent completes when all of its children are sealed.
  *
  *   n, d_n      report count (host), or a device uint64 count (d_n != NULL;

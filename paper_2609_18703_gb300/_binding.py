@@ -21,8 +21,10 @@ LIB_PATH = os.path.join(HERE, "libro_gb300.so")
 RO_OK, RO_E_INVAL, RO_E_CAPACITY, RO_E_OVERFLOW, RO_E_STATE, RO_E_OOM, RO_E_CUDA, RO_E_TIMEOUT = range(8)
 # Item outcomes (Eq. 1)
 RO_PENDING, RO_PRESENT, RO_DROPPED, RO_FAILED, RO_SUPPRESSED = range(5)
+# report kind (Section 4.4): the Grain failed and its open siblings are suppressed
+RO_GROUP_FAILURE = 5
 # report verdicts (Eq. 3)
-RO_ACCEPT, RO_REJ_INVALID, RO_REJ_NOT_INFLIGHT, RO_REJ_STALE_GEN, RO_REJ_DUPLICATE = range(5)
+RO_ACCEPT, RO_REJ_INVALID, RO_REJ_NOT_INFLIGHT, RO_REJ_STALE_GEN, RO_REJ_DUPLICATE, RO_REJ_BARRIER = range(6)
 
 STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFLOW",
                 4: "RO_E_STATE", 5: "RO_E_OOM", 6: "RO_E_CUDA", 7: "RO_E_TIMEOUT"}
@@ -45,7 +47,8 @@ class RoError(RuntimeError):
 class _Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in (
         "accepted", "rej_invalid", "rej_not_inflight", "rej_stale_gen", "rej_duplicate",
-        "ready_bad_candidates", "assemble_incomplete")]
+        "ready_bad_candidates", "assemble_incomplete", "rej_barrier", "barrier_not_dispatched",
+        "barrier_in_flight", "queue_dropped")]
 
 
 _lib = None

@@ -27,7 +27,8 @@
 
 namespace ro {
 
-constexpr uint8_t V_WIN_SEALER = 6, V_WIN_CAND = 7, V_LOSE_SEALER = 8, V_LOSE_CAND = 9;
+constexpr uint8_t V_WIN_SEALER = 7, V_WIN_CAND = 8, V_LOSE_SEALER = 9, V_LOSE_CAND = 10;
+constexpr uint32_t GB_NONE = 0xFFFFFFFFu;
 
 // record word read past L1 (other threads update it with atomics at L2)
 __device__ __forceinline__ uint64_t ld_w(const Rec* rc) {
@@ -43,9 +44,11 @@ __device__ __forceinline__ uint64_t commit_count(const CommitArgs& a) {
 __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a) {
   wait_predecessor();
   allow_successor();
-  __shared__ unsigned long long s_cnt[6];
+  // verdict counts: accept, invalid, not in flight, stale, -, barrier,
+  // duplicate candidates, accepted GroupFailures
+  __shared__ unsigned long long s_cnt[8];
   DevScalars* ds = a.ds;
-  if (threadIdx.x < 6) s_cnt[threadIdx.x] = 0;
+  if (threadIdx.x < 8) s_cnt[threadIdx.x] = 0;
   __syncthreads();
   const uint64_t n = commit_count(a);
   if (a.d_n && *a.d_n > a.n_host && blockIdx.x == 0 && threadIdx.x == 0)
@@ -53,7 +56,7 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
   const int lane = threadIdx.x & 31;
   const uint64_t warp_global = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
-  uint32_t cnt[6] = {0, 0, 0, 0, 0, 0};
+  uint32_t cnt[8] = {0, 0, 0, 0, 0, 0, 0, 0};
   for (uint64_t base = warp_global * 32; base < n; base += n_warps * 32) {
     const uint64_t r = base + lane;
     uint8_t v = 255;   // inactive lane
@@ -65,7 +68,7 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
       const uint32_t l = a.len[r];
       const uint64_t o = a.off[r];
       const uint32_t g = a.gen ? a.gen[r] : 0u;
-      const bool valid_state = s >= ST_PRESENT && s <= ST_SUPPRESSED;
+      const bool valid_state = s >= ST_PRESENT && s <= ST_GROUP_FAILURE;
       const bool in_bounds = s != ST_PRESENT || (o <= a.arena_bytes && (uint64_t)l <= a.arena_bytes - o);
       if (c >= a.N || !valid_state || !in_bounds) {
         v = V_INVALID;
@@ -84,17 +87,22 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
         if (won) {
           v = V_ACCEPT;
           const bool present = s == ST_PRESENT;
+          // a GroupFailure's own Grain failed
+          const uint8_t outcome = (s == ST_GROUP_FAILURE) ? ST_FAILED : s;
           Rec* rc = a.rec + c;
           rc->len = present ? l : 0u;
           atomicOr((unsigned long long*)&rc->w,
                    (unsigned long long)((present ? (o & W_OFF_MASK) : 0ull) |
-                                        ((uint64_t)s << W_STATE_SHIFT)));
+                                        ((uint64_t)outcome << W_STATE_SHIFT)));
           p = par;
-          bad = (s == ST_FAILED || s == ST_SUPPRESSED);
+          bad = (s == ST_FAILED || s == ST_SUPPRESSED || s == ST_GROUP_FAILURE);
+          if (s == ST_GROUP_FAILURE) atomicMin(a.gb + par, (uint32_t)r);   // barrier: commit_finish
         } else if ((cur & 3u) == PH_WAITING || (cur & 3u) == PH_READY) {
           v = V_NOT_INFLIGHT;
         } else if ((cur >> 2) != g) {
           v = V_STALE;
+        } else if (ld_w(a.rec + c) & W_BARRIER_BIT) {
+          v = V_BARRIER;   // suppressed by a sibling's GroupFailure in an earlier call
         } else {
           // SEALED at this generation: a duplicate, possibly of a report of
           // this same call with a higher index (ordered by commit_finish)
@@ -124,12 +132,14 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
         }
       }
     }
-    if (v < 6) cnt[v == V_DUP_CANDIDATE ? 5 : v] += 1;
+    if (v <= V_DUP_CANDIDATE) cnt[v] += 1;
+    // any GroupFailure report (it may still win an ordering of duplicates)
+    if (r < n && v != V_INVALID && a.state[r] == ST_GROUP_FAILURE) cnt[7] += 1;
   }
-  // statistics: accepted, invalid, not in flight, stale (duplicates are
-  // counted by the finish pass), candidates for ordering
+  // statistics: accepted, invalid, not in flight, stale, barrier (duplicates
+  // are counted by the finish pass), candidates for ordering, GroupFailures
 #pragma unroll
-  for (int k = 0; k < 6; ++k) {
+  for (int k = 0; k < 8; ++k) {
     uint32_t x = cnt[k];
     for (int d = 16; d > 0; d >>= 1) x += __shfl_down_sync(0xffffffffu, x, d);
     if (lane == 0 && x) atomicAdd(&s_cnt[k], (unsigned long long)x);
@@ -138,7 +148,9 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
   if (threadIdx.x == 0) {
     for (int k = 0; k < 4; ++k)
       if (s_cnt[k]) atomicAdd(&ds->stats[k], s_cnt[k]);
-    if (s_cnt[5]) atomicAdd(&ds->cm_conflicts, s_cnt[5]);
+    if (s_cnt[5]) atomicAdd(&ds->stats[7], s_cnt[5]);
+    if (s_cnt[6]) atomicAdd(&ds->cm_conflicts, s_cnt[6]);
+    if (s_cnt[7]) atomicAdd(&ds->cm_gf, s_cnt[7]);
   }
 }
 
@@ -191,14 +203,15 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
     const uint8_t v = a.code[r];
     if (v < V_WIN_SEALER || v > V_LOSE_CAND) continue;
     const uint8_t s = a.state[r];
-    const bool bad = (s == ST_FAILED || s == ST_SUPPRESSED);
+    const bool bad = (s == ST_FAILED || s == ST_SUPPRESSED || s == ST_GROUP_FAILURE);
     Rec* rc = a.rec + a.child[r];
     const uint32_t p = rc->parent;
     if (v == V_WIN_SEALER || v == V_WIN_CAND) {
       const bool present = s == ST_PRESENT;
+      const uint8_t outcome = (s == ST_GROUP_FAILURE) ? ST_FAILED : s;
       const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK | W_SEALER_BIT | W_CONFLICT_BIT);
       rc->len = present ? a.len[r] : 0u;
-      rc->w = keep | (present ? (a.off[r] & W_OFF_MASK) : 0ull) | ((uint64_t)s << W_STATE_SHIFT);
+      rc->w = keep | (present ? (a.off[r] & W_OFF_MASK) : 0ull) | ((uint64_t)outcome << W_STATE_SHIFT);
       if (v == V_WIN_CAND && bad) atomicAdd(a.pw + p, 1ull << 32);
     } else {
       if (v == V_LOSE_SEALER && bad) atomicAdd(a.pw + p, ~((1ull << 32) - 1));   // -(1 << 32)
@@ -222,6 +235,166 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
   }
   __syncthreads();
   if (threadIdx.x == 0) atomicAdd(&ds->stats[4], s_dups);
+  __syncthreads();
+}
+
+__device__ __forceinline__ void stat_add(unsigned long long* s, unsigned long long d) {
+  if (d) atomicAdd(s, d);   // d may be a negative delta in two's complement
+}
+
+// GroupFailure barriers (Section 4.4) of this call, applied as if the
+// reports were taken one by one in array order.  Run by one CTA, after the
+// duplicate ordering and only when the scatter accepted a GroupFailure.
+// For each parent, the lowest accepted GroupFailure report b installs the
+// barrier: sibling reports before b stand; those after b see their Grain
+// sealed by the barrier; every sibling still unsealed is sealed Suppressed.
+__device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
+  DevScalars* ds = a.ds;
+  // accepted, not in flight, stale, duplicate, barrier, suppressed while
+  // waiting/ready, suppressed while in flight
+  __shared__ unsigned long long s_d[7];   // signed deltas, two's complement
+  if (threadIdx.x < 7) s_d[threadIdx.x] = 0;
+  __syncthreads();
+  auto parent_of = [&](uint64_t r, uint32_t* p) -> bool {
+    const uint64_t c = a.child[r];
+    if (c >= a.N) return false;
+    *p = a.rec[c].parent;
+    return true;
+  };
+  // 1: barrier indices from the final verdicts (a GroupFailure can have lost
+  //    to an earlier duplicate of its Grain)
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    uint32_t p;
+    if (a.state[r] == ST_GROUP_FAILURE && parent_of(r, &p)) a.gb[p] = GB_NONE;
+  }
+  __syncthreads();
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    uint32_t p;
+    if (a.state[r] == ST_GROUP_FAILURE && a.code[r] == V_ACCEPT && parent_of(r, &p))
+      atomicMin(a.gb + p, (uint32_t)r);
+  }
+  __syncthreads();
+  // 2: sibling reports after the barrier that the scatter accepted: their
+  //    Grain was in flight when the barrier sealed it
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    uint32_t p;
+    if (a.code[r] != V_ACCEPT || !parent_of(r, &p)) continue;
+    const uint32_t b = __ldcg(a.gb + p);
+    if (b == GB_NONE || r <= b) continue;
+    Rec* rc = a.rec + a.child[r];
+    const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
+    rc->len = 0u;
+    rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
+    const uint8_t s = a.state[r];
+    if (!(s == ST_FAILED || s == ST_SUPPRESSED || s == ST_GROUP_FAILURE))
+      atomicAdd(a.pw + p, 1ull << 32);   // its outcome class is now bad
+    a.code[r] = V_BARRIER;
+    atomicAdd(&s_d[0], ~0ull);
+    atomicAdd(&s_d[4], 1ull);
+    atomicAdd(&s_d[6], 1ull);
+  }
+  __syncthreads();
+  // 3: other reports after the barrier whose Grain the barrier sealed
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    uint32_t p;
+    const uint8_t v = a.code[r];
+    if ((v != V_DUPLICATE && v != V_NOT_INFLIGHT) || !parent_of(r, &p)) continue;
+    const uint32_t b = __ldcg(a.gb + p);
+    if (b == GB_NONE || r <= b) continue;
+    const uint64_t c = a.child[r];
+    if (v == V_DUPLICATE) {
+      if (!(ld_w(a.rec + c) & W_BARRIER_BIT)) continue;   // sealed before the barrier
+      a.code[r] = V_BARRIER;
+      atomicAdd(&s_d[3], ~0ull);
+      atomicAdd(&s_d[4], 1ull);
+    } else {
+      // WAITING or READY at scatter time, sealed by the barrier before this
+      // report: the fence now compares generations
+      const uint32_t ph = __ldcg(a.phase + c);
+      const uint32_t gen_c = ((ph & 3u) == PH_WAITING) ? 0u : (ph >> 2);
+      const uint32_t g = a.gen ? a.gen[r] : 0u;
+      const bool same = g == gen_c;
+      a.code[r] = same ? V_BARRIER : V_STALE;
+      atomicAdd(&s_d[1], ~0ull);
+      atomicAdd(&s_d[same ? 4 : 2], 1ull);
+    }
+  }
+  __syncthreads();
+  // 4: a parent that completed in the scatter and whose class moved in (2):
+  //    its member count to gather is redone
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    uint32_t p;
+    if (a.code[r] != V_BARRIER || a.state[r] == ST_GROUP_FAILURE || !parent_of(r, &p)) continue;
+    const uint32_t b = __ldcg(a.gb + p);
+    if (b == GB_NONE || r <= b) continue;
+    const unsigned long long pv = __ldcg(a.pw + p);
+    if (pw_remaining(pv) != 0u) continue;
+    const uint32_t old = atomicExch(a.pm + p, 0u);   // Suppressed: nothing to gather
+    if (old) atomicAdd(a.wm + (p >> 5), 0u - old);
+  }
+  __syncthreads();
+  // 5: the barrier seals every sibling that is still open; one warp per
+  //    triggering report
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  for (uint64_t base = (uint64_t)warp * 32; base < n; base += (uint64_t)nw * 32) {
+    const uint64_t r = base + lane;
+    uint32_t p = 0;
+    const bool trig = r < n && a.state[r] == ST_GROUP_FAILURE && a.code[r] == V_ACCEPT &&
+                      parent_of(r, &p) && __ldcg(a.gb + p) == (uint32_t)r;
+    unsigned m = __ballot_sync(0xffffffffu, trig);
+    while (m) {
+      const int src = __ffs(m) - 1;
+      m &= m - 1;
+      const uint32_t pp = __shfl_sync(0xffffffffu, p, src);
+      const uint64_t c0 = a.offsets[pp], c1 = a.offsets[pp + 1];
+      uint32_t k_wait = 0, k_fly = 0;
+      for (uint64_t d = c0 + lane; d < c1; d += 32) {
+        const uint32_t ph = __ldcg(a.phase + d);
+        const uint32_t f = ph & 3u;
+        if (f == PH_SEALED) continue;
+        const uint32_t gen_d = (f == PH_WAITING) ? 0u : (ph >> 2);
+        a.phase[d] = ph_make(PH_SEALED, gen_d);
+        Rec* rc = a.rec + d;
+        const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
+        rc->len = 0u;
+        rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
+        if (f == PH_INFLIGHT) ++k_fly; else ++k_wait;
+      }
+      for (int s = 16; s > 0; s >>= 1) {
+        k_wait += __shfl_down_sync(0xffffffffu, k_wait, s);
+        k_fly += __shfl_down_sync(0xffffffffu, k_fly, s);
+      }
+      if (lane == 0) {
+        const unsigned long long k = (unsigned long long)k_wait + k_fly;
+        if (k) {
+          const unsigned long long old = atomicAdd(a.pw + pp, (k << 32) - k);
+          if ((uint32_t)old == k) {   // the barrier completes the parent
+            a.pm[pp] = 0u;
+            atomicOr(a.bitmap + (pp >> 5), 1u << (pp & 31));
+          }
+        }
+        atomicAdd(&s_d[5], (unsigned long long)k_wait);
+        atomicAdd(&s_d[6], (unsigned long long)k_fly);
+      }
+      __syncwarp();
+    }
+  }
+  __syncthreads();
+  // 6: this call's barrier indices are spent
+  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    uint32_t p;
+    if (a.state[r] == ST_GROUP_FAILURE && parent_of(r, &p)) a.gb[p] = GB_NONE;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    stat_add(&ds->stats[0], s_d[0]);
+    stat_add(&ds->stats[2], s_d[1]);
+    stat_add(&ds->stats[3], s_d[2]);
+    stat_add(&ds->stats[4], s_d[3]);
+    stat_add(&ds->stats[7], s_d[4]);
+    stat_add(&ds->stats[8], s_d[5]);
+    stat_add(&ds->stats[9], s_d[6]);
+  }
   __syncthreads();
 }
 
@@ -253,11 +426,12 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
 
   // Reports of one Grain that met in this call: the first CTA here orders
   // them; the others wait for it before reading outcome classes.
-  if (ds->cm_conflicts != 0) {
+  if (ds->cm_conflicts != 0 || ds->cm_gf != 0) {
     if (threadIdx.x == 0) s_fix = atomicAdd(&ds->cm_fix_ticket, 1u);
     __syncthreads();
     if (s_fix == 0u) {
-      resolve_duplicates(a, commit_count(a));
+      if (ds->cm_conflicts != 0) resolve_duplicates(a, commit_count(a));
+      if (ds->cm_gf != 0) resolve_barriers(a, commit_count(a));
       if (threadIdx.x == 0) {
         __threadfence();
         st_release(&ds->cm_fix_done, 1u);
@@ -349,6 +523,7 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
       ds->exit_ctr[TS_COMMIT] = 0u;
       ds->epoch[TS_COMMIT] += 1ull;
       ds->cm_conflicts = 0ull;
+      ds->cm_gf = 0ull;
       ds->cm_fix_ticket = 0u;
       ds->cm_fix_done = 0u;
     }

@@ -30,6 +30,8 @@ __device__ __forceinline__ bool call_ok(const ReadyArgs& a, uint64_t c) {
 __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
   wait_predecessor();
   __shared__ unsigned long long s_red[2][RB_THREADS / 32];
+  __shared__ unsigned long long s_scan[33];
+  __shared__ uint32_t s_last;
   DevScalars* ds = a.ds;
   unsigned long long kept = 0, bad = 0;
   const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
@@ -75,10 +77,35 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
     }
     if (k) atomicAdd(&ds->rb_kept, k);
     if (b) atomicAdd(&ds->rb_bad, b);
-    if (ticket(&ds->rb_ticket) == gridDim.x - 1) {
-      // last CTA: plan the reservation
+    s_last = ticket(&ds->rb_ticket) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  // last CTA.  Queued Grains that a GroupFailure has sealed since they were
+  // queued leave the queue now, undispatched (Section 4.4): stable in-place
+  // compaction of the queue window (fewer than one batch is ever left over).
+  const unsigned long long head = a.qstate[0], tail0 = a.qstate[1];
+  unsigned long long tail = head;
+  for (unsigned long long base = head; base < tail0; base += RB_THREADS) {
+    const unsigned long long i = base + threadIdx.x;
+    uint32_t c = 0;
+    bool live = false;
+    if (i < tail0) {
+      c = a.queue[i];
+      live = (a.phase[c] & 3u) == PH_READY;
+    }
+    unsigned long long total;
+    const unsigned long long pos = block_excl_scan((unsigned long long)live, s_scan, &total);
+    if (live) a.queue[tail + pos] = c;   // never ahead of an entry not yet read
+    tail += total;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    {
+      // plan the reservation
+      if (tail0 != tail) ds->stats[10] += tail0 - tail;
+      a.qstate[1] = tail;
       const unsigned long long K = ld_relaxed_u64(&ds->rb_kept);
-      const unsigned long long head = a.qstate[0], tail = a.qstate[1];
       const unsigned long long L = tail - head, T = L + K;
       const unsigned long long npop = a.flush ? T : (T / a.batch_size) * a.batch_size;
       ds->rb_npop = npop;

@@ -67,7 +67,7 @@ struct PlanSlot {
 
 // Device buffers of one expansion slot, kept across ro_ctx_reset and reused.
 struct ExpSlot {
-  DevBuf offsets, pw, phase, rec, bitmap, tfp, pm, wm;
+  DevBuf offsets, pw, phase, rec, bitmap, tfp, pm, wm, gb;
   ListSlot lists[RING];
   PlanSlot plans[RING];
   std::vector<QueueBufs> queues;
@@ -439,7 +439,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   sync_all_streams(c);
   for (auto& s : c->slots) {
     free_buf(s.offsets); free_buf(s.pw); free_buf(s.phase); free_buf(s.rec); free_buf(s.bitmap);
-    free_buf(s.tfp); free_buf(s.pm); free_buf(s.wm);
+    free_buf(s.tfp); free_buf(s.pm); free_buf(s.wm); free_buf(s.gb);
     for (auto& l : s.lists) {
       free_buf(l.done); free_buf(l.status); free_buf(l.mb); free_buf(l.coff); free_buf(l.mtfp);
       free_buf(l.hdr); free_ev(l.freed);
@@ -503,7 +503,7 @@ ro_status ro_ctx_stats(ro_ctx* c, ro_stats* out) {
   DeviceGuard g(c->device);
   ro_status st = sync_and_check(c);
   uint64_t* o = &out->accepted;
-  for (int k = 0; k < 7; ++k) o[k] = c->hs->stats[k];
+  for (int k = 0; k < 11; ++k) o[k] = c->hs->stats[k];
   return st;
 }
 
@@ -604,6 +604,7 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   RO_TRY(ensure(c, S.bitmap, ceil_div(P, 32) * sizeof(uint32_t), "completion bitmap"));
   RO_TRY(ensure(c, S.pm, P * sizeof(uint32_t), "parent member counts"));
   RO_TRY(ensure(c, S.wm, ceil_div(P, 32) * sizeof(uint32_t), "word member counts"));
+  RO_TRY(ensure(c, S.gb, P * sizeof(uint32_t), "GroupFailure barriers"));
   for (auto& l : S.lists) {
     RO_TRY(ensure(c, l.done, P * sizeof(uint32_t), "completed parents"));
     RO_TRY(ensure(c, l.status, P, "completed parents"));
@@ -620,6 +621,7 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   }
   cudaMemsetAsync(S.bitmap.p, 0, ceil_div(P, 32) * sizeof(uint32_t), c->stream);
   cudaMemsetAsync(S.wm.p, 0, ceil_div(P, 32) * sizeof(uint32_t), c->stream);
+  cudaMemsetAsync(S.gb.p, 0xFF, P * sizeof(uint32_t), c->stream);   // no barrier pending
   ExpandFillArgs fa{};
   fa.offsets = (const uint64_t*)S.offsets.p;
   fa.P = P;
@@ -730,6 +732,7 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.bitmap = (uint32_t*)S.bitmap.p;
   ca.pm = (uint32_t*)S.pm.p;
   ca.wm = (uint32_t*)S.wm.p;
+  ca.gb = (uint32_t*)S.gb.p;
   if (d_code) {
     ca.code = d_code;
   } else {

@@ -31,21 +31,24 @@ __host__ __device__ constexpr uint32_t ph_make(uint32_t phase, uint32_t gen) {
 // ---- Item outcomes (Eq. 1) and report verdicts (Eq. 3) --------------------
 constexpr uint8_t ST_PENDING = 0, ST_PRESENT = 1, ST_DROPPED = 2, ST_FAILED = 3,
                   ST_SUPPRESSED = 4;
+// report kind (Section 4.4): the Grain failed and its open siblings are suppressed
+constexpr uint8_t ST_GROUP_FAILURE = 5;
 constexpr uint8_t V_ACCEPT = 0, V_INVALID = 1, V_NOT_INFLIGHT = 2, V_STALE = 3,
-                  V_DUPLICATE = 4;
+                  V_DUPLICATE = 4, V_BARRIER = 5;
 // internal verdict: the Grain was SEALED at the same generation; resolved to
 // ACCEPT or DUPLICATE by the commit's ordering pass
-constexpr uint8_t V_DUP_CANDIDATE = 5;
+constexpr uint8_t V_DUP_CANDIDATE = 6;
 
 // ---- result record ----------------------------------------------------------
 struct __align__(16) Rec {
   uint32_t parent;
   uint32_t len;
-  uint64_t w;   // off (0-47) | state (48-50) | sealer-seen (54) | conflict (55) | call (56-63)
+  uint64_t w;   // off (0-47) | state (48-50) | barrier (53) | sealer-seen (54) | conflict (55) | call (56-63)
 };
 constexpr uint64_t W_OFF_MASK = (1ull << 48) - 1;
 constexpr int W_STATE_SHIFT = 48;
 constexpr uint64_t W_STATE_MASK = 7ull << W_STATE_SHIFT;
+constexpr uint64_t W_BARRIER_BIT = 1ull << 53;   // sealed by a sibling's GroupFailure
 constexpr uint64_t W_SEALER_BIT = 1ull << 54;
 constexpr uint64_t W_CONFLICT_BIT = 1ull << 55;
 constexpr int W_CALL_SHIFT = 56;
@@ -92,14 +95,14 @@ struct PlanHdr {
 struct DevScalars {
   uint32_t err;
   uint32_t pad0;
-  unsigned long long stats[7];   // same order as ro_stats
+  unsigned long long stats[11];  // same order as ro_stats
   // ro_expand
   unsigned long long n_children, n_empty, last_nonempty_parent;
   // ro_batch_ready
   unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
   uint32_t rb_ticket, rb_err;
   // ro_gather_commit
-  unsigned long long cm_n, cm_conflicts, cm_n_done;
+  unsigned long long cm_n, cm_conflicts, cm_n_done, cm_gf;
   uint32_t cm_fix_ticket, cm_fix_done;
   // ro_assemble
   unsigned long long as_bytes;    // bytes of the latest assemble (host read-back)

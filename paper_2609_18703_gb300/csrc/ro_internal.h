@@ -158,6 +158,8 @@ struct CommitArgs {
   uint32_t* bitmap;
   uint32_t* pm;               // per parent: members to gather once complete (0: Suppressed)
   uint32_t* wm;               // per bitmap word: sum of pm of the parents completed in this call
+  uint32_t* gb;               // per parent: lowest accepted GroupFailure report of this call
+                              // (all ones: none); reset by commit_finish
   uint8_t* code;              // user's or internal
   uint32_t* done_user;        // optional
   uint32_t* done_int;         // the list (a ring slot)
