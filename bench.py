@@ -55,6 +55,10 @@ def parse():
     ap.add_argument("--parents", type=int, default=1_000_000)
     ap.add_argument("--waves", type=int, default=256)
     ap.add_argument("--no-graph", action="store_true", help="launch the wave loop eagerly")
+    ap.add_argument("--rq4", action="store_true",
+                    help="failure-containment pass (GroupFailure at ordinal 0 of the largest parents)")
+    ap.add_argument("--rq4-waves", type=int, default=64)
+    ap.add_argument("--rq4-parents", type=int, default=99)
     ap.add_argument("--one-stream", action="store_true",
                     help="plan and copy on the context's stream (no overlap across waves)")
     ap.add_argument("--no-e2e", action="store_true")
@@ -487,8 +491,112 @@ def _d2h_chunks(src, dst):
     return dst
 
 
+def run_rq4(args, local_rank):
+    """Failure containment on the GPU path (Section 4.4; the paper's RQ4 set-up,
+    Section 6): the document->page level is dispatched over `--rq4-waves`
+    readiness waves (each wave: admit its children, reserve batches of 256,
+    commit the dispatched children's reports in FIFO order, assemble the
+    parents they complete).  A poisoned pass reports GroupFailure at ordinal 0
+    of the `--rq4-parents` largest parents; a clean pass does not.  Prints one
+    JSON line with both pass times and the suppressed-sibling counts."""
+    import torch
+    import __graft_entry__
+    import paper_2609_18703_gb300 as ro
+    from workload import docpage
+    from workload.device import fill_payload
+    torch.cuda.set_device(local_rank)
+    __graft_entry__.build()
+    lv = docpage(parents=args.parents, waves=1).top
+    dev = torch.device("cuda", local_rank)
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
+    P, N, W, B = lv.n_parents, lv.n_children, args.rq4_waves, 256
+    rng = np.random.default_rng(0x52415934)
+    ready = rng.permutation(N).astype(np.int64)                 # readiness order
+    bounds = np.linspace(0, N, W + 1).astype(np.int64)
+    off_p = np.concatenate([[0], np.cumsum(lv.counts.astype(np.int64))])
+    big = np.argsort(-lv.counts.astype(np.int64), kind="stable")[:args.rq4_parents]
+    triggers = off_p[big]
+    t = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a).view(dt)).to(dev)
+    counts = t(lv.counts, np.int32)
+    cand = t(ready.astype(np.uint32), np.int32)
+    st_clean = t(lv.state, np.uint8)
+    st_pois_np = lv.state.copy()
+    st_pois_np[triggers] = ro.RO_GROUP_FAILURE
+    st_pois = t(st_pois_np, np.uint8)
+    length = t(lv.length, np.int32)
+    aoff = t(lv.arena_off, np.int64)
+    arena = torch.empty(max(int(lv.arena_bytes), 16), dtype=torch.uint8, device=dev)
+    fill_payload(arena, aoff, length, lv.payload_seed, stream)
+    offsets = torch.empty(P + 1, dtype=torch.int64, device=dev)
+    cp = torch.empty(N, dtype=torch.int32, device=dev)
+    co = torch.empty(N, dtype=torch.int32, device=dev)
+    cap = int(np.max(np.diff(bounds))) + B
+    batched = torch.zeros(cap, dtype=torch.int32, device=dev)
+    nb = torch.zeros(1, dtype=torch.int64, device=dev)
+    status = torch.empty(P, dtype=torch.uint8, device=dev)
+    out_off = torch.empty(P + 1, dtype=torch.int64, device=dev)
+    out = torch.empty(int(lv.arena_bytes) + 64, dtype=torch.uint8, device=dev)
+    cursor = torch.zeros(1, dtype=torch.int64, device=dev)
+    ctx = ro.ro_ctx_create(local_rank, stream, 1)
+    L = ro.load()
+
+    def one_pass(states):
+        ro.ro_ctx_reset(ctx)
+        st, n, _, x = ro.ro_expand(ctx, -1, counts, P, None, offsets, cp, co, N, None)
+        assert st == 0 and n == N
+        cursor.zero_()
+        for w in range(W):
+            s0, s1 = int(bounds[w]), int(bounds[w + 1])
+            L.ro_batch_ready(ctx, x, 0, cand.data_ptr() + 4 * s0, s1 - s0, B, 1,
+                             batched.data_ptr(), cap, nb.data_ptr(), None, None)
+            idx = batched.long()
+            # the dispatched children's reports (the executor's side of the protocol)
+            r_st, r_len, r_off = states[idx], length[idx], aoff[idx]
+            L.ro_gather_commit(ctx, x, cap, nb.data_ptr(), batched.data_ptr(), r_st.data_ptr(),
+                               r_len.data_ptr(), r_off.data_ptr(), None, int(lv.arena_bytes),
+                               None, None, 0, None, None)
+            L.ro_assemble(ctx, x, arena.data_ptr(), int(lv.arena_bytes), None, P, None,
+                          status.data_ptr(), out_off.data_ptr(), None, out.data_ptr(), out.numel(),
+                          cursor.data_ptr(), None, None)
+        L.ro_ctx_join(ctx)
+
+    res = {}
+    for name, states in (("clean", st_clean), ("poisoned", st_pois)):
+        one_pass(states)                       # warm-up
+        ro.ro_ctx_stats(ctx)                   # clears nothing; read below as deltas
+        before = ro.ro_ctx_stats(ctx)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        one_pass(states)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        after = ro.ro_ctx_stats(ctx)
+        assert after.pop("status") == 0, ro.ro_last_error(ctx)
+        before.pop("status")
+        d = {k: after[k] - before[k] for k in after}
+        res[name] = {"ms_per_pass": round(e0.elapsed_time(e1), 3),
+                     "children_per_s": round(N / (e0.elapsed_time(e1) * 1e-3), 1),
+                     "accepted": d["accepted"], "rej_barrier": d["rej_barrier"],
+                     "siblings_not_dispatched": d["barrier_not_dispatched"],
+                     "siblings_suppressed_in_flight": d["barrier_in_flight"],
+                     "queue_dropped": d["queue_dropped"], "bytes_assembled": int(cursor.item())}
+    siblings = int(lv.counts[big].astype(np.int64).sum()) - len(big)
+    print(json.dumps({"rq4": {
+        "workload": f"document->page: {P} parents, {N} children, dispatched over {W} readiness "
+                    f"waves, batches of {B}; GroupFailure at ordinal 0 of the {len(big)} largest parents",
+        "poisoned_parents": int(len(big)), "poisoned_parent_siblings": siblings,
+        "share_of_children_in_poisoned_parents": round(int(lv.counts[big].sum()) / N, 4),
+        **res}}), flush=True)
+    ro.ro_ctx_destroy(ctx)
+
+
 def main():
     args = parse()
+    if args.rq4:
+        run_rq4(args, int(os.environ.get("LOCAL_RANK", "0")))
+        return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

@@ -244,16 +244,34 @@ __device__ __forceinline__ void stat_add(unsigned long long* s, unsigned long lo
 
 // GroupFailure barriers (Section 4.4) of this call, applied as if the
 // reports were taken one by one in array order.  Run by one CTA, after the
-// duplicate ordering and only when the scatter accepted a GroupFailure.
+// duplicate ordering and only when the call carries a GroupFailure report.
 // For each parent, the lowest accepted GroupFailure report b installs the
 // barrier: sibling reports before b stand; those after b see their Grain
 // sealed by the barrier; every sibling still unsealed is sealed Suppressed.
+// The GroupFailure reports and the barrier parents (few) are kept in shared
+// memory; the barriers sorted by first child, so a report's barrier is a
+// search there on its child id.  The two passes over all reports load 16
+// reports' fields per thread before acting on any.  Past GF_CAP
+// GroupFailure reports in one call, a report's parent and barrier are read
+// from global memory instead (slower, same result).
+constexpr int GF_CAP = 128;
+constexpr int RB_GROUP = 16;
 __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
   DevScalars* ds = a.ds;
-  // accepted, not in flight, stale, duplicate, barrier, suppressed while
-  // waiting/ready, suppressed while in flight
-  __shared__ unsigned long long s_d[7];   // signed deltas, two's complement
+  // counter deltas: accepted, not in flight, stale, duplicate, barrier,
+  // suppressed while waiting/ready, suppressed while in flight
+  __shared__ unsigned long long s_d[7];   // two's complement
+  __shared__ uint32_t s_gr[GF_CAP], s_gp[GF_CAP];   // GroupFailure reports and their parents
+  __shared__ uint32_t s_nf, s_ng;
+  __shared__ uint32_t s_p[GF_CAP], s_b[GF_CAP];     // barriers: parent, report
+  __shared__ unsigned long long s_c0[GF_CAP], s_c1[GF_CAP];
+  __shared__ uint32_t s_sp[GF_CAP], s_sb[GF_CAP];   // the same, sorted by first child
+  __shared__ unsigned long long s_sc0[GF_CAP], s_sc1[GF_CAP];
   if (threadIdx.x < 7) s_d[threadIdx.x] = 0;
+  if (threadIdx.x == 0) {
+    s_nf = 0;
+    s_ng = 0;
+  }
   __syncthreads();
   auto parent_of = [&](uint64_t r, uint32_t* p) -> bool {
     const uint64_t c = a.child[r];
@@ -261,129 +279,216 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
     *p = a.rec[c].parent;
     return true;
   };
-  // 1: barrier indices from the final verdicts (a GroupFailure can have lost
-  //    to an earlier duplicate of its Grain)
-  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
-    uint32_t p;
-    if (a.state[r] == ST_GROUP_FAILURE && parent_of(r, &p)) a.gb[p] = GB_NONE;
+  // 0: the call's GroupFailure reports (with a valid child)
+  for (uint64_t base = (uint64_t)threadIdx.x * RB_GROUP; base < n; base += (uint64_t)blockDim.x * RB_GROUP) {
+    uint8_t sv[RB_GROUP];
+#pragma unroll
+    for (int j = 0; j < RB_GROUP; ++j) sv[j] = (base + j < n) ? a.state[base + j] : 0;
+#pragma unroll
+    for (int j = 0; j < RB_GROUP; ++j) {
+      uint32_t p;
+      if (sv[j] != ST_GROUP_FAILURE || !parent_of(base + j, &p)) continue;
+      const uint32_t k = atomicAdd(&s_nf, 1u);
+      if (k < GF_CAP) {
+        s_gr[k] = (uint32_t)(base + j);
+        s_gp[k] = p;
+      }
+    }
   }
   __syncthreads();
-  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
-    uint32_t p;
-    if (a.state[r] == ST_GROUP_FAILURE && a.code[r] == V_ACCEPT && parent_of(r, &p))
-      atomicMin(a.gb + p, (uint32_t)r);
+  const uint32_t nf = s_nf;
+  const bool fast = nf <= GF_CAP;
+  // 1: barrier index per parent from the final verdicts (a GroupFailure can
+  //    have lost to an earlier duplicate of its Grain)
+  if (fast) {
+    for (uint32_t i = threadIdx.x; i < nf; i += blockDim.x) a.gb[s_gp[i]] = GB_NONE;
+    __syncthreads();
+    for (uint32_t i = threadIdx.x; i < nf; i += blockDim.x)
+      if (a.code[s_gr[i]] == V_ACCEPT) atomicMin(a.gb + s_gp[i], s_gr[i]);
+    __syncthreads();
+    for (uint32_t i = threadIdx.x; i < nf; i += blockDim.x) {
+      const uint32_t r = s_gr[i], p = s_gp[i];
+      if (a.code[r] != V_ACCEPT || __ldcg(a.gb + p) != r) continue;
+      const uint32_t k = atomicAdd(&s_ng, 1u);
+      s_p[k] = p;
+      s_b[k] = r;
+      s_c0[k] = a.offsets[p];
+      s_c1[k] = a.offsets[p + 1];
+    }
+  } else {
+    for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+      uint32_t p;
+      if (a.state[r] == ST_GROUP_FAILURE && parent_of(r, &p)) a.gb[p] = GB_NONE;
+    }
+    __syncthreads();
+    for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+      uint32_t p;
+      if (a.state[r] == ST_GROUP_FAILURE && a.code[r] == V_ACCEPT && parent_of(r, &p))
+        atomicMin(a.gb + p, (uint32_t)r);
+    }
   }
   __syncthreads();
-  // 2: sibling reports after the barrier that the scatter accepted: their
-  //    Grain was in flight when the barrier sealed it
-  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
-    uint32_t p;
-    if (a.code[r] != V_ACCEPT || !parent_of(r, &p)) continue;
-    const uint32_t b = __ldcg(a.gb + p);
-    if (b == GB_NONE || r <= b) continue;
-    Rec* rc = a.rec + a.child[r];
-    const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
-    rc->len = 0u;
-    rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
-    const uint8_t s = a.state[r];
-    if (!(s == ST_FAILED || s == ST_SUPPRESSED || s == ST_GROUP_FAILURE))
-      atomicAdd(a.pw + p, 1ull << 32);   // its outcome class is now bad
-    a.code[r] = V_BARRIER;
-    atomicAdd(&s_d[0], ~0ull);
-    atomicAdd(&s_d[4], 1ull);
-    atomicAdd(&s_d[6], 1ull);
+  const uint32_t ng = s_ng;
+  if (fast) {   // sort the barriers by first child (rank sort; ranges are disjoint)
+    for (uint32_t i = threadIdx.x; i < ng; i += blockDim.x) {
+      uint32_t rank = 0;
+      for (uint32_t j = 0; j < ng; ++j) rank += s_c0[j] < s_c0[i];
+      s_sp[rank] = s_p[i];
+      s_sb[rank] = s_b[i];
+      s_sc0[rank] = s_c0[i];
+      s_sc1[rank] = s_c1[i];
+    }
   }
   __syncthreads();
-  // 3: other reports after the barrier whose Grain the barrier sealed
-  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
-    uint32_t p;
-    const uint8_t v = a.code[r];
-    if ((v != V_DUPLICATE && v != V_NOT_INFLIGHT) || !parent_of(r, &p)) continue;
-    const uint32_t b = __ldcg(a.gb + p);
-    if (b == GB_NONE || r <= b) continue;
-    const uint64_t c = a.child[r];
-    if (v == V_DUPLICATE) {
+  if (fast && ng == 0) return;   // every GroupFailure was rejected
+  // the barrier (parent, report) a child falls under, if any
+  auto barrier_of = [&](uint64_t c, uint32_t* p, uint32_t* b) -> bool {
+    if (c >= a.N) return false;
+    if (fast) {
+      if (c < s_sc0[0]) return false;
+      uint32_t lo = 0, hi = ng;
+      while (hi - lo > 1) {
+        const uint32_t mid = (lo + hi) >> 1;
+        if (s_sc0[mid] <= c) lo = mid; else hi = mid;
+      }
+      if (c >= s_sc1[lo]) return false;
+      const uint32_t pp = s_sp[lo];
+      *p = pp;
+      *b = s_sb[lo];
+      return true;
+    }
+    const uint32_t pp = a.rec[c].parent;
+    const uint32_t bb = __ldcg(a.gb + pp);
+    if (bb == GB_NONE) return false;
+    *p = pp;
+    *b = bb;
+    return true;
+  };
+  // 2: reports after a barrier whose Grain the barrier found open: those the
+  //    scatter accepted were in flight; those it found WAITING or READY now
+  //    meet a sealed Grain and the fence compares generations
+  for (uint64_t base = (uint64_t)threadIdx.x * RB_GROUP; base < n; base += (uint64_t)blockDim.x * RB_GROUP) {
+    uint8_t cv[RB_GROUP];
+    uint32_t chv[RB_GROUP];
+#pragma unroll
+    for (int j = 0; j < RB_GROUP; ++j) cv[j] = (base + j < n) ? a.code[base + j] : V_INVALID;
+#pragma unroll
+    for (int j = 0; j < RB_GROUP; ++j)
+      chv[j] = (cv[j] == V_ACCEPT || cv[j] == V_NOT_INFLIGHT) ? a.child[base + j] : 0u;
+#pragma unroll 1
+    for (int j = 0; j < RB_GROUP; ++j) {
+      const uint8_t v = cv[j];
+      if (v != V_ACCEPT && v != V_NOT_INFLIGHT) continue;
+      const uint64_t r = base + j, c = chv[j];
+      uint32_t p, b;
+      if (!barrier_of(c, &p, &b) || r <= b) continue;
+      if (v == V_ACCEPT) {
+        Rec* rc = a.rec + c;
+        const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
+        rc->len = 0u;
+        rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
+        const uint8_t st = a.state[r];
+        if (!(st == ST_FAILED || st == ST_SUPPRESSED || st == ST_GROUP_FAILURE))
+          atomicAdd(a.pw + p, 1ull << 32);   // its outcome class is now bad
+        a.code[r] = V_BARRIER;
+        atomicAdd(&s_d[0], ~0ull);
+        atomicAdd(&s_d[4], 1ull);
+        atomicAdd(&s_d[6], 1ull);
+      } else {
+        const uint32_t ph = __ldcg(a.phase + c);
+        const uint32_t gen_c = ((ph & 3u) == PH_WAITING) ? 0u : (ph >> 2);
+        const uint32_t g = a.gen ? a.gen[r] : 0u;
+        const bool same = g == gen_c;
+        a.code[r] = same ? V_BARRIER : V_STALE;
+        atomicAdd(&s_d[1], ~0ull);
+        atomicAdd(&s_d[same ? 4 : 2], 1ull);
+      }
+    }
+  }
+  __syncthreads();
+  // 3: duplicates after a barrier of a Grain whose accepted report (2) just
+  //    turned into a barrier rejection (only if this call had duplicates)
+  const bool had_dups = ds->cm_conflicts != 0;
+  for (uint64_t base = (uint64_t)threadIdx.x * RB_GROUP; had_dups && base < n;
+       base += (uint64_t)blockDim.x * RB_GROUP) {
+    uint8_t cv[RB_GROUP];
+#pragma unroll
+    for (int j = 0; j < RB_GROUP; ++j) cv[j] = (base + j < n) ? a.code[base + j] : V_INVALID;
+#pragma unroll 1
+    for (int j = 0; j < RB_GROUP; ++j) {
+      if (cv[j] != V_DUPLICATE) continue;
+      const uint64_t r = base + j, c = a.child[r];
+      uint32_t p, b;
+      if (!barrier_of(c, &p, &b) || r <= b) continue;
       if (!(ld_w(a.rec + c) & W_BARRIER_BIT)) continue;   // sealed before the barrier
       a.code[r] = V_BARRIER;
       atomicAdd(&s_d[3], ~0ull);
       atomicAdd(&s_d[4], 1ull);
-    } else {
-      // WAITING or READY at scatter time, sealed by the barrier before this
-      // report: the fence now compares generations
-      const uint32_t ph = __ldcg(a.phase + c);
-      const uint32_t gen_c = ((ph & 3u) == PH_WAITING) ? 0u : (ph >> 2);
-      const uint32_t g = a.gen ? a.gen[r] : 0u;
-      const bool same = g == gen_c;
-      a.code[r] = same ? V_BARRIER : V_STALE;
-      atomicAdd(&s_d[1], ~0ull);
-      atomicAdd(&s_d[same ? 4 : 2], 1ull);
     }
   }
   __syncthreads();
-  // 4: a parent that completed in the scatter and whose class moved in (2):
-  //    its member count to gather is redone
-  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
-    uint32_t p;
-    if (a.code[r] != V_BARRIER || a.state[r] == ST_GROUP_FAILURE || !parent_of(r, &p)) continue;
-    const uint32_t b = __ldcg(a.gb + p);
-    if (b == GB_NONE || r <= b) continue;
-    const unsigned long long pv = __ldcg(a.pw + p);
-    if (pw_remaining(pv) != 0u) continue;
-    const uint32_t old = atomicExch(a.pm + p, 0u);   // Suppressed: nothing to gather
-    if (old) atomicAdd(a.wm + (p >> 5), 0u - old);
-  }
-  __syncthreads();
-  // 5: the barrier seals every sibling that is still open; one warp per
-  //    triggering report
+  // 4: the barrier seals every sibling that is still open; one warp per
+  //    barrier (the parent then completes; it has a failed member, so it
+  //    gathers nothing)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  for (uint64_t base = (uint64_t)warp * 32; base < n; base += (uint64_t)nw * 32) {
-    const uint64_t r = base + lane;
-    uint32_t p = 0;
-    const bool trig = r < n && a.state[r] == ST_GROUP_FAILURE && a.code[r] == V_ACCEPT &&
-                      parent_of(r, &p) && __ldcg(a.gb + p) == (uint32_t)r;
-    unsigned m = __ballot_sync(0xffffffffu, trig);
-    while (m) {
-      const int src = __ffs(m) - 1;
-      m &= m - 1;
-      const uint32_t pp = __shfl_sync(0xffffffffu, p, src);
-      const uint64_t c0 = a.offsets[pp], c1 = a.offsets[pp + 1];
-      uint32_t k_wait = 0, k_fly = 0;
-      for (uint64_t d = c0 + lane; d < c1; d += 32) {
-        const uint32_t ph = __ldcg(a.phase + d);
-        const uint32_t f = ph & 3u;
-        if (f == PH_SEALED) continue;
-        const uint32_t gen_d = (f == PH_WAITING) ? 0u : (ph >> 2);
-        a.phase[d] = ph_make(PH_SEALED, gen_d);
-        Rec* rc = a.rec + d;
-        const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
-        rc->len = 0u;
-        rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
-        if (f == PH_INFLIGHT) ++k_fly; else ++k_wait;
-      }
-      for (int s = 16; s > 0; s >>= 1) {
-        k_wait += __shfl_down_sync(0xffffffffu, k_wait, s);
-        k_fly += __shfl_down_sync(0xffffffffu, k_fly, s);
-      }
-      if (lane == 0) {
-        const unsigned long long k = (unsigned long long)k_wait + k_fly;
-        if (k) {
-          const unsigned long long old = atomicAdd(a.pw + pp, (k << 32) - k);
-          if ((uint32_t)old == k) {   // the barrier completes the parent
-            a.pm[pp] = 0u;
-            atomicOr(a.bitmap + (pp >> 5), 1u << (pp & 31));
-          }
+  auto seal_open = [&](uint32_t pp) {
+    const uint64_t c0 = a.offsets[pp], c1 = a.offsets[pp + 1];
+    uint32_t k_wait = 0, k_fly = 0;
+    for (uint64_t d = c0 + lane; d < c1; d += 32) {
+      const uint32_t ph = __ldcg(a.phase + d);
+      const uint32_t f = ph & 3u;
+      if (f == PH_SEALED) continue;
+      const uint32_t gen_d = (f == PH_WAITING) ? 0u : (ph >> 2);
+      a.phase[d] = ph_make(PH_SEALED, gen_d);
+      Rec* rc = a.rec + d;
+      const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
+      rc->len = 0u;
+      rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
+      if (f == PH_INFLIGHT) ++k_fly; else ++k_wait;
+    }
+    for (int sh = 16; sh > 0; sh >>= 1) {
+      k_wait += __shfl_down_sync(0xffffffffu, k_wait, sh);
+      k_fly += __shfl_down_sync(0xffffffffu, k_fly, sh);
+    }
+    if (lane == 0) {
+      const unsigned long long k = (unsigned long long)k_wait + k_fly;
+      if (k) {
+        const unsigned long long old = atomicAdd(a.pw + pp, (k << 32) - k);
+        if ((uint32_t)old == k) {   // the barrier completes the parent
+          a.pm[pp] = 0u;
+          atomicOr(a.bitmap + (pp >> 5), 1u << (pp & 31));
         }
-        atomicAdd(&s_d[5], (unsigned long long)k_wait);
-        atomicAdd(&s_d[6], (unsigned long long)k_fly);
       }
-      __syncwarp();
+      atomicAdd(&s_d[5], (unsigned long long)k_wait);
+      atomicAdd(&s_d[6], (unsigned long long)k_fly);
+    }
+    __syncwarp();
+  };
+  if (fast) {
+    for (uint32_t i = warp; i < ng; i += nw) seal_open(s_sp[i]);
+  } else {
+    for (uint64_t base = (uint64_t)warp * 32; base < n; base += (uint64_t)nw * 32) {
+      const uint64_t r = base + lane;
+      uint32_t p = 0;
+      const bool trig = r < n && a.state[r] == ST_GROUP_FAILURE && a.code[r] == V_ACCEPT &&
+                        parent_of(r, &p) && __ldcg(a.gb + p) == (uint32_t)r;
+      unsigned m = __ballot_sync(0xffffffffu, trig);
+      while (m) {
+        const int src = __ffs(m) - 1;
+        m &= m - 1;
+        seal_open(__shfl_sync(0xffffffffu, p, src));
+      }
     }
   }
   __syncthreads();
-  // 6: this call's barrier indices are spent
-  for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
-    uint32_t p;
-    if (a.state[r] == ST_GROUP_FAILURE && parent_of(r, &p)) a.gb[p] = GB_NONE;
+  // 5: this call's barrier indices are spent
+  if (fast) {
+    for (uint32_t i = threadIdx.x; i < nf; i += blockDim.x) a.gb[s_gp[i]] = GB_NONE;
+  } else {
+    for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
+      uint32_t p;
+      if (a.state[r] == ST_GROUP_FAILURE && parent_of(r, &p)) a.gb[p] = GB_NONE;
+    }
   }
   __syncthreads();
   if (threadIdx.x == 0) {
