@@ -38,6 +38,8 @@ typedef struct {
   uint32_t** q;             /* per Call: FIFO Ready Queue storage (N slots) */
   uint64_t* qhead;
   uint64_t* qtail;
+  uint32_t** rq;            /* per Call: recovery queue (retried Grains, N slots) */
+  uint64_t* rlen;
   uint32_t* last_done;      /* parents completed by the latest commit */
   uint64_t n_last_done;
 } or_exp;
@@ -72,6 +74,10 @@ void or_ctx_reset(or_ctx* ctx) {
     if (x && x->q) {
       for (uint32_t c = 0; c < ctx->n_calls; ++c) free(x->q[c]);
       free(x->q); free(x->qhead); free(x->qtail);
+    }
+    if (x && x->rq) {
+      for (uint32_t c = 0; c < ctx->n_calls; ++c) free(x->rq[c]);
+      free(x->rq); free(x->rlen);
     }
     exp_free(x);
     ctx->exp[i] = NULL;
@@ -154,10 +160,12 @@ int or_expand(or_ctx* ctx, int32_t parent_xid, const uint32_t* counts, uint64_t 
   x->q = (uint32_t**)calloc(ctx->n_calls, sizeof(uint32_t*));
   x->qhead = (uint64_t*)calloc(ctx->n_calls, sizeof(uint64_t));
   x->qtail = (uint64_t*)calloc(ctx->n_calls, sizeof(uint64_t));
+  x->rq = (uint32_t**)calloc(ctx->n_calls, sizeof(uint32_t*));
+  x->rlen = (uint64_t*)calloc(ctx->n_calls, sizeof(uint64_t));
   if (!x->offsets || !x->child_parent || !x->child_call || !x->phase || !x->gen || !x->st ||
       !x->len || !x->off || !x->terminal || !x->bad || !x->barrier || !x->by_barrier ||
-      !x->last_done || !x->q || !x->qhead || !x->qtail) {
-    free(x->q); free(x->qhead); free(x->qtail);
+      !x->last_done || !x->q || !x->qhead || !x->qtail || !x->rq || !x->rlen) {
+    free(x->q); free(x->qhead); free(x->qtail); free(x->rq); free(x->rlen);
     exp_free(x);
     return OR_E_OOM;
   }
@@ -212,6 +220,17 @@ int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand
   }
   uint32_t* q = x->q[call];
 
+  /* recovery groups go first: they are placed ahead of the queue's entries
+     (the slots before the head are free: every retried Grain was taken out
+     of this queue once) */
+  if (x->rlen[call]) {
+    uint64_t nr = x->rlen[call];
+    if (nr > x->qhead[call]) return OR_E_STATE;   /* cannot happen: see above */
+    x->qhead[call] -= nr;
+    memcpy(q + x->qhead[call], x->rq[call], nr * sizeof(uint32_t));
+    x->rlen[call] = 0;
+  }
+
   /* queued Grains a GroupFailure sealed leave the queue undispatched */
   uint64_t kept = x->qhead[call];
   for (uint64_t t = x->qhead[call]; t < x->qtail[call]; ++t) {
@@ -252,6 +271,37 @@ int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand
   x->qhead[call] += take;
   if (n_batches) *n_batches = (take + batch_size - 1) / batch_size;
   ctx->stats.ready_bad_candidates += bad_cand;
+  return OR_OK;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Retry (Section 4.4; Eq. 2's IN-FLIGHT -> READY edge).  A physical attempt
+ * failed: its Grains keep their identity, return to READY with the next
+ * generation (so reports of the failed attempt are stale), and re-enter as
+ * one group of the Call's recovery queue, ahead of normal entries
+ * (Section 4.3).                                                           */
+int or_retry(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* children, uint64_t n,
+             uint64_t* n_retried) {
+  or_exp* x = get_exp(ctx, xid);
+  if (!x || call >= ctx->n_calls || (n && !children)) return OR_E_INVAL;
+  if (!x->rq[call]) {
+    x->rq[call] = (uint32_t*)malloc((x->N ? x->N : 1) * sizeof(uint32_t));
+    if (!x->rq[call]) return OR_E_OOM;
+  }
+  uint64_t k = 0;
+  for (uint64_t i = 0; i < n; ++i) {
+    uint64_t c = children[i];
+    if (c >= x->N || x->phase[c] != OR_IN_FLIGHT || x->child_call[c] != call) {
+      ctx->stats.retry_skipped++;
+      continue;
+    }
+    x->phase[c] = OR_READY;
+    x->gen[c] += 1;
+    x->rq[call][x->rlen[call]++] = (uint32_t)c;
+    ++k;
+  }
+  ctx->stats.retried += k;
+  if (n_retried) *n_retried = k;
   return OR_OK;
 }
 

@@ -45,6 +45,8 @@ typedef struct {
   uint64_t barrier_not_dispatched;  /* siblings suppressed while WAITING or READY */
   uint64_t barrier_in_flight;       /* siblings suppressed while IN-FLIGHT */
   uint64_t queue_dropped;           /* suppressed Grains removed from a Ready Queue */
+  uint64_t retried;                 /* Grains moved back to READY at a new generation */
+  uint64_t retry_skipped;           /* retry entries naming no in-flight Grain of the Call */
 } or_stats;
 
 or_ctx* or_ctx_create(uint32_t n_calls);
@@ -66,6 +68,15 @@ int or_expand(or_ctx* ctx, int32_t parent_xid, const uint32_t* counts, uint64_t 
 int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand,
                    uint64_t n_cand, uint32_t batch_size, int32_t flush, uint32_t* batched,
                    uint64_t batched_cap, uint64_t* n_batched, uint64_t* n_batches);
+
+/* Retry of a failed physical attempt (Section 4.4; Eq. 2 IN-FLIGHT -> READY;
+ * Section 4.3 recovery queues): each listed Grain of this Call that is
+ * IN-FLIGHT (first occurrence in the list) goes back to READY with its
+ * generation + 1, and the listed Grains, in list order, form one group in
+ * the Call's recovery queue.  The next reservation takes recovery groups,
+ * oldest first, before the Ready Queue's entries. */
+int or_retry(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* children, uint64_t n,
+             uint64_t* n_retried);
 
 /* Generation-fenced commit (Section 4.4, Eq. 3) and parent completion
  * (Section 4.2, Reduce); completed parents listed ascending.  An accepted

@@ -38,7 +38,7 @@ class _Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in (
         "accepted", "rej_invalid", "rej_not_inflight", "rej_stale_gen", "rej_duplicate",
         "ready_bad_candidates", "assemble_incomplete", "rej_barrier", "barrier_not_dispatched",
-        "barrier_in_flight", "queue_dropped")]
+        "barrier_in_flight", "queue_dropped", "retried", "retry_skipped")]
 
 
 _lib = None
@@ -68,7 +68,8 @@ def lib():
                                        _u64p, _u32p, C.c_uint64, _u8p, _u32p, C.c_uint64, _u64p]
         L.or_assemble.argtypes = [C.c_void_p, C.c_int32, _u8p, C.c_uint64, _u32p, C.c_uint64,
                                   _u8p, _u64p, _u32p, _u8p, C.c_uint64, _u64p, _u64p, _u64p]
-        for f in ("or_expand", "or_batch_ready", "or_gather_commit", "or_assemble"):
+        L.or_retry.argtypes = [C.c_void_p, C.c_int32, C.c_uint32, _u32p, C.c_uint64, _u64p]
+        for f in ("or_expand", "or_batch_ready", "or_gather_commit", "or_assemble", "or_retry"):
             getattr(L, f).restype = C.c_int
         _lib = L
     return _lib
@@ -150,8 +151,8 @@ class OracleCtx:
         cand = _arr(cand, np.uint32)
         n_cand = 0 if cand is None else cand.size
         if cap is None:
-            # at most the queued leftovers (< batch_size) plus every candidate come out
-            cap = (n_cand if cand is not None else self._n_children[xid]) + batch_size
+            # never more than the expansion's children (plus a batch of slack)
+            cap = self._n_children[xid] + batch_size
         out = np.zeros(max(cap, 1), dtype=np.uint32)
         nb = C.c_uint64(0)
         nbt = C.c_uint64(0)
@@ -161,6 +162,17 @@ class OracleCtx:
             raise OracleError("or_batch_ready", st)
         return dict(status=st, batched=out[:nb.value].copy() if st == OK else None,
                     n_batched=nb.value, n_batches=nbt.value)
+
+    def retry(self, xid: int, call: int, children, check: bool = True):
+        """Failed attempt: IN-FLIGHT Grains back to READY at generation + 1, as one
+        recovery group taken before the Ready Queue at the next reservation."""
+        children = _arr(children, np.uint32)
+        n = 0 if children is None else children.size
+        k = C.c_uint64(0)
+        st = lib().or_retry(self._h, xid, call, _ptr(children, _u32p), n, C.byref(k))
+        if check and st != OK:
+            raise OracleError("or_retry", st)
+        return dict(status=st, n_retried=k.value)
 
     def gather_commit(self, xid: int, child, state, length, off, gen=None,
                       arena_bytes: int = (1 << 48) - 1, n_parents_hint: Optional[int] = None,

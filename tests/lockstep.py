@@ -97,7 +97,7 @@ class Lockstep:
         cand_np = None if cand is None else np.asarray(cand, dtype=np.uint32)
         n_cand = self.N[xid] if cand_np is None else cand_np.size
         if cap is None:
-            cap = n_cand + batch_size
+            cap = self.N[xid] + batch_size
         r = self.o.batch_ready(xid, call, cand_np, batch_size, flush, cap=cap, check=False)
         d_cand = None if cand_np is None else dev(cand_np, np.uint32)
         d_b = empty(cap, np.uint32)

@@ -34,6 +34,13 @@ MUTANTS = {
     "queue_keeps_suppressed": ("if (x->phase[q[t]] == OR_READY)", "if (1)"),
     "barrier_verdict_lost": ("v = x->by_barrier[c] ? OR_REJ_BARRIER : OR_REJ_DUPLICATE;",
                              "v = OR_REJ_DUPLICATE;"),
+    # retry and recovery queues (Section 4.4, Eq. 2; Section 4.3)
+    "retry_keeps_generation": ("    x->gen[c] += 1;\n", "    (void)0;\n"),
+    "recovery_never_reinserted": ("  if (x->rlen[call]) {", "  if (0) {"),
+    "recovery_behind_queue": ("    memcpy(q + x->qhead[call], x->rq[call], nr * sizeof(uint32_t));",
+                              "    for (uint64_t i = 0; i < nr; ++i) q[x->qhead[call] + i] = x->rq[call][nr - 1 - i];"),
+    "retry_ignores_call": ("if (c >= x->N || x->phase[c] != OR_IN_FLIGHT || x->child_call[c] != call) {",
+                           "if (c >= x->N || x->phase[c] != OR_IN_FLIGHT) {"),
     "barrier_completion_missed": ("if (sealed_now && x->terminal[p] == member_count(x, p)) x->last_done[k++] = p;",
                                   "(void)sealed_now;"),
 }
@@ -52,6 +59,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     env = dict(os.environ, ORACLE_LIB=str(so))
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
                         os.path.join(ROOT, "tests", "test_oracle.py"),
-                        os.path.join(ROOT, "tests", "test_oracle_group_failure.py")],
+                        os.path.join(ROOT, "tests", "test_oracle_group_failure.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_retry.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode != 0, f"pins did not catch mutant {name}:\n{r.stdout[-2000:]}"
