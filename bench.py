@@ -55,6 +55,7 @@ def parse():
     ap.add_argument("--parents", type=int, default=1_000_000)
     ap.add_argument("--waves", type=int, default=256)
     ap.add_argument("--no-graph", action="store_true", help="launch the wave loop eagerly")
+    ap.add_argument("--retry", action="store_true", help="ro_retry throughput (failed attempts)")
     ap.add_argument("--rq4", action="store_true",
                     help="failure-containment pass (GroupFailure at ordinal 0 of the largest parents)")
     ap.add_argument("--rq4-waves", type=int, default=64)
@@ -592,8 +593,72 @@ def run_rq4(args, local_rank):
     ro.ro_ctx_destroy(ctx)
 
 
+def run_retry_bench(args, local_rank):
+    """Throughput of ro_retry (Section 4.4, Eq. 2's retry edge): every child of
+    the document->page level is dispatched, then a seeded random 1/16 of them
+    (one failed attempt of ~1M Grains, in random order) is retried; between
+    repetitions the recovery group is reserved again (READY -> IN-FLIGHT).
+    Only the ro_retry calls are timed (CUDA events on the context's stream)."""
+    import torch
+    import __graft_entry__
+    import paper_2609_18703_gb300 as ro
+    from workload import docpage
+    torch.cuda.set_device(local_rank)
+    __graft_entry__.build()
+    hbm_peak, peak_kind = peaks()
+    lv = docpage(parents=args.parents, waves=1).top
+    dev = torch.device("cuda", local_rank)
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
+    P, N = lv.n_parents, lv.n_children
+    rng = np.random.default_rng(0x52415935)
+    pick = rng.permutation(N)[: N // 16].astype(np.uint32)
+    counts = torch.from_numpy(lv.counts.view(np.int32)).to(dev)
+    lst = torch.from_numpy(pick.view(np.int32)).to(dev)
+    offsets = torch.empty(P + 1, dtype=torch.int64, device=dev)
+    cp = torch.empty(N, dtype=torch.int32, device=dev)
+    co = torch.empty(N, dtype=torch.int32, device=dev)
+    batched = torch.empty(N + 256, dtype=torch.int32, device=dev)
+    ctx = ro.ro_ctx_create(local_rank, stream, 1)
+    st, n, _, x = ro.ro_expand(ctx, -1, counts, P, None, offsets, cp, co, N, None)
+    assert st == 0
+    st, nb, _ = ro.ro_batch_ready(ctx, x, 0, None, 0, 256, 1, batched, N + 256)
+    assert st == 0 and nb == N
+    L = ro.load()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    for i in range(args.warmup + args.steps):
+        if i >= args.warmup:
+            ev[i - args.warmup][0].record(stream)
+        L.ro_retry(ctx, x, 0, lst.data_ptr(), lst.numel(), None)
+        if i >= args.warmup:
+            ev[i - args.warmup][1].record(stream)
+        L.ro_batch_ready(ctx, x, 0, None, 0, 256, 1, batched.data_ptr(), N + 256, None, None, None)
+    torch.cuda.synchronize()
+    stats = ro.ro_ctx_stats(ctx)
+    assert stats.pop("status") == 0, ro.ro_last_error(ctx)
+    assert stats["retried"] == (args.warmup + args.steps) * lst.numel()
+    ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
+    k = lst.numel()
+    # algorithmic bytes per retried Grain: list entry 4 read, phase word read
+    # and rewritten (8), record word read for the Call (8) and len claimed and
+    # cleared (12), recovery-queue entry 4 written
+    alg = 36.0 * k
+    print(json.dumps({"retry": {
+        "workload": f"document->page: {N} children in flight; one failed attempt of {k} Grains "
+                    f"(random order) retried per call",
+        "ms_per_call": round(ms, 4), "grains_per_s": round(k / (ms * 1e-3), 1),
+        "algorithmic_gbs": round(alg / (ms * 1e-3) / 1e9, 1), "peak_gbs": hbm_peak,
+        "peak_kind": peak_kind, "frac": round(alg / (ms * 1e-3) / 1e9 / hbm_peak, 4),
+        "steps": args.steps, "warmup": args.warmup}}), flush=True)
+    ro.ro_ctx_destroy(ctx)
+
+
 def main():
     args = parse()
+    if args.retry:
+        run_retry_bench(args, int(os.environ.get("LOCAL_RANK", "0")))
+        return
     if args.rq4:
         run_rq4(args, int(os.environ.get("LOCAL_RANK", "0")))
         return

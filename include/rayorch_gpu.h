@@ -105,6 +105,8 @@ typedef struct {
   uint64_t barrier_not_dispatched;/* siblings a GroupFailure sealed while WAITING or READY */
   uint64_t barrier_in_flight;     /* siblings a GroupFailure sealed while IN-FLIGHT */
   uint64_t queue_dropped;         /* sealed Grains removed from a Ready Queue undispatched */
+  uint64_t retried;               /* Grains ro_retry moved back to READY */
+  uint64_t retry_skipped;         /* ro_retry entries naming no IN-FLIGHT Grain of the Call */
 } ro_stats;
 
 /* ------------------------------------------------------------------------
@@ -146,7 +148,7 @@ const char* ro_last_error(const ro_ctx* ctx);
 enum {
   RO_K_EXPAND_SCAN = 0, RO_K_EXPAND_FILL = 1, RO_K_READY_COUNT = 2, RO_K_READY_SCATTER = 3,
   RO_K_COMMIT_SCATTER = 4, RO_K_COMMIT_FINISH = 5, RO_K_ASM_PARENTS = 6, RO_K_ASM_MEMBERS = 7,
-  RO_K_ASM_COPY = 8, RO_K_COUNT = 9
+  RO_K_ASM_COPY = 8, RO_K_RETRY_CLAIM = 9, RO_K_RETRY_SCATTER = 10, RO_K_COUNT = 11
 };
 /* Tracing (no counterpart in the paper; it instruments the path).  Every
  * kernel launch is counted; kernels whose bit (1 << RO_K_*) is set in
@@ -214,6 +216,26 @@ ro_status ro_batch_ready(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t
                          uint64_t n_cand, uint32_t batch_size, int32_t flush,
                          uint32_t* d_batched, uint64_t batched_cap, uint64_t* d_n_batched,
                          uint64_t* h_n_batched, uint64_t* h_n_batches);
+
+/* ------------------------------------------------------------------------
+ * ro_retry — a failed physical attempt is tried again (Section 4.4: the
+ * runtime may retry a Grain at a higher generation; Eq. 2's IN-FLIGHT ->
+ * READY edge; Section 4.3: recovery queues reinsert the Grain group).
+ *
+ *   d_children  uint32[n] the Grains of the failed attempt (a batch), in
+ *               the order they are to run again.
+ * Every listed Grain of Call `call` that is IN-FLIGHT (first occurrence in
+ * the list) goes back to READY with its generation + 1, so reports of the
+ * failed attempt are rejected (RO_REJ_NOT_INFLIGHT while READY,
+ * RO_REJ_STALE_GEN once dispatched again).  Those Grains, in list order,
+ * form one group of the Call's recovery queue; the next ro_batch_ready for
+ * the Call reserves recovery groups, oldest first, before the Ready Queue's
+ * entries (a retried Grain that a GroupFailure has sealed meanwhile is
+ * dropped).  Entries naming no IN-FLIGHT Grain of the Call are skipped and
+ * counted.  h_n_retried (host, synchronises) out or NULL: Grains retried.
+ */
+ro_status ro_retry(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* d_children, uint64_t n,
+                   uint64_t* h_n_retried);
 
 /* ------------------------------------------------------------------------
  * ro_gather_commit — generation-fenced commit of child results (Section 4.4,

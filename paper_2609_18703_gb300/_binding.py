@@ -31,11 +31,11 @@ STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFL
 
 EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro_ctx_stats",
            "ro_ctx_set_streams", "ro_ctx_join", "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
-           "ro_gather_commit", "ro_assemble", "ro_expand_noalloc")
+           "ro_retry", "ro_gather_commit", "ro_assemble", "ro_expand_noalloc")
 
 # kernel ids (RO_K_*), in launch order of the path
 KERNELS = ("expand_scan", "expand_fill", "ready_count", "ready_scatter", "commit_scatter",
-           "commit_finish", "asm_parents", "asm_members", "asm_copy")
+           "commit_finish", "asm_parents", "asm_members", "asm_copy", "retry_claim", "retry_scatter")
 
 
 class RoError(RuntimeError):
@@ -48,7 +48,7 @@ class _Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in (
         "accepted", "rej_invalid", "rej_not_inflight", "rej_stale_gen", "rej_duplicate",
         "ready_bad_candidates", "assemble_incomplete", "rej_barrier", "barrier_not_dispatched",
-        "barrier_in_flight", "queue_dropped")]
+        "barrier_in_flight", "queue_dropped", "retried", "retry_skipped")]
 
 
 _lib = None
@@ -83,6 +83,7 @@ def load(path: Optional[str] = None):
     L.ro_ctx_profile_read.argtypes = [_vp, _pu64, _pu64, C.POINTER(C.c_double), _u32]
     L.ro_expand.argtypes = [_vp, _i32, _vp, _u64, _vp, _vp, _vp, _vp, _u64, _vp, _pu64, _pu64, _pi32]
     L.ro_batch_ready.argtypes = [_vp, _i32, _u32, _vp, _u64, _u32, _i32, _vp, _u64, _vp, _pu64, _pu64]
+    L.ro_retry.argtypes = [_vp, _i32, _u32, _vp, _u64, _pu64]
     L.ro_gather_commit.argtypes = [_vp, _i32, _u64, _vp, _vp, _vp, _vp, _vp, _vp, _u64, _vp, _vp, _u64,
                                    _vp, _pu64]
     L.ro_assemble.argtypes = [_vp, _i32, _vp, _u64, _vp, _u64, _vp, _vp, _vp, _vp, _vp, _u64, _vp, _vp,
@@ -201,6 +202,13 @@ def ro_batch_ready(ctx, xid, call, d_cand, n_cand, batch_size, flush, d_batched,
                                C.byref(nb) if want_host else None,
                                C.byref(nbt) if want_host else None)
     return (st, nb.value, nbt.value) if want_host else (st, None, None)
+
+
+def ro_retry(ctx, xid, call, d_children, n, want_host: bool = True):
+    """Returns (status, n_retried); n_retried is None without want_host."""
+    k = _u64(0)
+    st = load().ro_retry(ctx, xid, call, _ptr(d_children), n, C.byref(k) if want_host else None)
+    return (st, k.value) if want_host else (st, None)
 
 
 def ro_gather_commit(ctx, xid, n, d_n, d_child, d_state, d_len, d_arena_off, d_gen, arena_bytes,

@@ -81,10 +81,18 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
   }
   __syncthreads();
   if (!s_last) return;
-  // last CTA.  Queued Grains that a GroupFailure has sealed since they were
-  // queued leave the queue now, undispatched (Section 4.4): stable in-place
-  // compaction of the queue window (fewer than one batch is ever left over).
-  const unsigned long long head = a.qstate[0], tail0 = a.qstate[1];
+  // last CTA.  Recovery groups (ro_retry) go ahead of the queue's entries,
+  // into the slots before the head: each retried Grain was taken out of this
+  // queue once, so there are at least as many such slots.
+  const unsigned long long nr = a.qstate[2], h0 = a.qstate[0];
+  const unsigned long long mv = nr < h0 ? nr : h0;
+  for (unsigned long long j = threadIdx.x; j < mv; j += RB_THREADS) a.queue[h0 - mv + j] = a.rq[j];
+  if (mv != nr && threadIdx.x == 0) atomicOr(&ds->err, ERR_INVAL);   // cannot happen
+  __syncthreads();
+  // Queued Grains that a GroupFailure has sealed since they were queued
+  // leave the queue now, undispatched (Section 4.4): stable in-place
+  // compaction of the queue window (fewer than one batch is usually left over).
+  const unsigned long long head = h0 - mv, tail0 = a.qstate[1];
   unsigned long long tail = head;
   for (unsigned long long base = head; base < tail0; base += RB_THREADS) {
     const unsigned long long i = base + threadIdx.x;
@@ -104,7 +112,9 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
     {
       // plan the reservation
       if (tail0 != tail) ds->stats[10] += tail0 - tail;
+      a.qstate[0] = head;
       a.qstate[1] = tail;
+      a.qstate[2] = 0;
       const unsigned long long K = ld_relaxed_u64(&ds->rb_kept);
       const unsigned long long L = tail - head, T = L + K;
       const unsigned long long npop = a.flush ? T : (T / a.batch_size) * a.batch_size;

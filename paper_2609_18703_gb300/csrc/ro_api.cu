@@ -26,6 +26,7 @@ const void* kernel_ptr_expand(int which);
 const void* kernel_ptr_ready(int which);
 const void* kernel_ptr_commit(int which);
 const void* kernel_ptr_assemble(int which);
+const void* kernel_ptr_retry(int which);
 }  // namespace ro
 
 using namespace ro;
@@ -49,7 +50,7 @@ struct Ev {
 };
 
 struct QueueBufs {
-  DevBuf q, state;
+  DevBuf q, rq, state;  // Ready Queue, recovery queue, [head, tail, recovery length]
   bool ready = false;   // state zeroed for the current expansion
 };
 
@@ -372,6 +373,17 @@ PlanBufs plan_bufs(PlanSlot& s, uint64_t member_cap) {
   return p;
 }
 
+// The (expansion, Call) queues, empty at the expansion's first use.
+ro_status queue_ready(ro_ctx* c, QueueBufs& Q, uint64_t N) {
+  if (Q.ready) return RO_OK;
+  RO_TRY(ensure(c, Q.q, N * sizeof(uint32_t), "ready queue"));
+  RO_TRY(ensure(c, Q.rq, N * sizeof(uint32_t), "recovery queue"));
+  RO_TRY(ensure(c, Q.state, 3 * sizeof(unsigned long long), "queue state"));
+  cudaMemsetAsync(Q.state.p, 0, 3 * sizeof(unsigned long long), c->stream);
+  Q.ready = true;
+  return RO_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -420,6 +432,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_aparents = grid_for(kernel_ptr_assemble(K_APARENTS), AP_THREADS, s, 4);
   c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 1);
   c->L.grid_acopy = grid_for(kernel_ptr_assemble(K_ACOPY), AC_THREADS, s, 8, asm_copy_smem());
+  c->L.grid_retry = grid_for(kernel_ptr_retry(K_RT_SCATTER), RT_THREADS, s, 4);
   c->Lp = c->L;
   c->Lc = c->L;
   cudaError_t e = cudaStreamSynchronize(c->stream);
@@ -450,6 +463,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
     }
     for (auto& q : s.queues) {
       free_buf(q.q);
+      free_buf(q.rq);
       free_buf(q.state);
     }
   }
@@ -503,7 +517,7 @@ ro_status ro_ctx_stats(ro_ctx* c, ro_stats* out) {
   DeviceGuard g(c->device);
   ro_status st = sync_and_check(c);
   uint64_t* o = &out->accepted;
-  for (int k = 0; k < 11; ++k) o[k] = c->hs->stats[k];
+  for (int k = 0; k < 13; ++k) o[k] = c->hs->stats[k];
   return st;
 }
 
@@ -662,12 +676,7 @@ ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* 
   DeviceGuard g(c->device);
   ExpSlot& S = c->slots[xid];
   QueueBufs& Q = S.queues[call];
-  if (!Q.ready) {
-    RO_TRY(ensure(c, Q.q, x->N * sizeof(uint32_t), "ready queue"));
-    RO_TRY(ensure(c, Q.state, 2 * sizeof(unsigned long long), "queue state"));
-    cudaMemsetAsync(Q.state.p, 0, 2 * sizeof(unsigned long long), c->stream);
-    Q.ready = true;
-  }
+  RO_TRY(queue_ready(c, Q, x->N));
   ReadyArgs ra{};
   ra.cand = d_cand;
   ra.n_cand = d_cand ? n_cand : x->N;
@@ -681,6 +690,7 @@ ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* 
   ra.cap = batched_cap;
   ra.queue = (uint32_t*)Q.q.p;
   ra.qstate = (unsigned long long*)Q.state.p;
+  ra.rq = (const uint32_t*)Q.rq.p;
   ra.batched = d_batched;
   ra.n_batched_out = d_n_batched;
   ra.ds = c->ds;
@@ -691,6 +701,43 @@ ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* 
     ro_status st = sync_and_check(c);
     if (h_n_batched) *h_n_batched = c->hs->rb_npop;
     if (h_n_batches) *h_n_batches = c->hs->rb_n_batches;
+    return st;
+  }
+  return RO_OK;
+}
+
+// ---------------------------------------------------------------------------
+ro_status ro_retry(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* d_children, uint64_t n,
+                   uint64_t* h_n_retried) {
+  RO_TRY(enter(c));
+  Expansion* x = get_exp(c, xid);
+  if (!x) return fail(c, RO_E_STATE, "ro_retry: unknown expansion %d", xid);
+  if (call >= c->n_calls) return fail(c, RO_E_INVAL, "ro_retry: call %u out of range", call);
+  if (n && !d_children) return fail(c, RO_E_INVAL, "ro_retry: NULL d_children");
+  if (n >= 0xFFFFFFFFull) return fail(c, RO_E_OVERFLOW, "ro_retry: 2^32-1 entries or more");
+  DeviceGuard g(c->device);
+  ExpSlot& S = c->slots[xid];
+  if (h_n_retried) *h_n_retried = 0;
+  if (n == 0) return RO_OK;
+  QueueBufs& Q = S.queues[call];
+  RO_TRY(queue_ready(c, Q, x->N));
+  RetryArgs ta{};
+  ta.children = d_children;
+  ta.n = n;
+  ta.N = x->N;
+  ta.phase = (uint32_t*)S.phase.p;
+  ta.rec = (Rec*)S.rec.p;
+  ta.check_call = c->n_calls > 1;
+  ta.call = call;
+  ta.rq = (uint32_t*)Q.rq.p;
+  ta.qstate = (unsigned long long*)Q.state.p;
+  ta.ds = c->ds;
+  RO_TRY(tile_status(c, TS_RETRY, ceil_div(n, (uint64_t)RT_THREADS * RT_ITEMS), &ta.ts));
+  launch_retry(c->L, ta);
+  RO_TRY(check_launch(c, "retry"));
+  if (h_n_retried) {
+    ro_status st = sync_and_check(c);
+    *h_n_retried = c->hs->rt_done;
     return st;
   }
   return RO_OK;

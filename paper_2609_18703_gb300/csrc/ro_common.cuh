@@ -95,7 +95,7 @@ struct PlanHdr {
 struct DevScalars {
   uint32_t err;
   uint32_t pad0;
-  unsigned long long stats[11];  // same order as ro_stats
+  unsigned long long stats[13];  // same order as ro_stats
   // ro_expand
   unsigned long long n_children, n_empty, last_nonempty_parent;
   // ro_batch_ready
@@ -103,6 +103,8 @@ struct DevScalars {
   uint32_t rb_ticket, rb_err;
   // ro_gather_commit
   unsigned long long cm_n, cm_conflicts, cm_n_done, cm_gf;
+  // ro_retry
+  unsigned long long rt_done;
   uint32_t cm_fix_ticket, cm_fix_done;
   // ro_assemble
   unsigned long long as_bytes;    // bytes of the latest assemble (host read-back)
@@ -111,7 +113,8 @@ struct DevScalars {
   uint32_t exit_ctr[8];
   unsigned long long epoch[8];
 };
-enum TileSlot { TS_EXPAND = 0, TS_READY = 1, TS_COMMIT = 2, TS_ASM_PARENTS = 3, TS_ASM_MEMBERS = 4 };
+enum TileSlot { TS_EXPAND = 0, TS_READY = 1, TS_COMMIT = 2, TS_ASM_PARENTS = 3, TS_ASM_MEMBERS = 4,
+                TS_RETRY = 6 };   // 5: asm_copy's exit ticket
 
 // Wait until the grid this launch depends on (programmatic dependent launch)
 // has completed and its memory is visible; a no-op without a dependency.

@@ -31,7 +31,7 @@ constexpr uint32_t AC_BUF = 16384 + 32 * AC_PIECES;           // staged source b
 
 // kernel entry points for occupancy queries and per-kernel timing
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CFINISH, K_APARENTS,
-                K_AMEMBERS, K_ACOPY, K_COUNT };
+                K_AMEMBERS, K_ACOPY, K_RT_CLAIM, K_RT_SCATTER, K_COUNT };
 
 // Launch counter and optional CUDA-event timing of selected kernels, on the
 // stream they are launched on (see ro_ctx_profile in the C ABI).
@@ -43,7 +43,7 @@ struct LaunchCfg {
   cudaStream_t stream;
   Profiler* prof;
   int grid_expand_scan, grid_fill, grid_rb, grid_commit, grid_cfinish, grid_aparents,
-      grid_amembers, grid_acopy;
+      grid_amembers, grid_acopy, grid_retry;
 };
 
 // Launch one kernel between the profiler's marks, with programmatic
@@ -107,13 +107,31 @@ struct ReadyArgs {
   int flush;
   uint64_t cap;
   uint32_t* queue;            // this (expansion, Call) queue storage
-  unsigned long long* qstate; // [head, tail]
+  unsigned long long* qstate; // [head, tail, recovery length]
+  const uint32_t* rq;         // this (expansion, Call) recovery queue storage
   uint32_t* batched;
   uint64_t* n_batched_out;    // optional device output
   DevScalars* ds;
   TileStatus<unsigned long long> ts;
 };
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a);
+
+// ---- ro_retry ----------------------------------------------------------------------
+constexpr int RT_THREADS = 256, RT_ITEMS = 8;                 // retry entries per tile: 2048
+struct RetryArgs {
+  const uint32_t* children;
+  uint64_t n;
+  uint64_t N;
+  uint32_t* phase;
+  Rec* rec;                   // len of an IN-FLIGHT Grain holds the claim (~index) meanwhile
+  int check_call;
+  uint32_t call;
+  uint32_t* rq;               // recovery queue storage
+  unsigned long long* qstate; // [head, tail, recovery length]
+  DevScalars* ds;
+  TileStatus<unsigned long long> ts;
+};
+void launch_retry(const LaunchCfg& L, const RetryArgs& a);
 
 // ---- lists and plans -------------------------------------------------------------------
 // A list of parents to assemble with its member bases: produced by

@@ -113,6 +113,15 @@ class Lockstep:
             assert np.array_equal(got, r["batched"])
         return dict(status=st, batched=r["batched"], n_batched=nb)
 
+    # ------------------------------------------------------------- retry
+    def retry(self, xid: int, call: int, children) -> dict:
+        ch = np.asarray(children, np.uint32)
+        r = self.o.retry(xid, call, ch, check=False)
+        st, k = ro.ro_retry(self.ctx, xid, call, dev(ch, np.uint32), ch.size)
+        assert st == r["status"], (st, r["status"], ro.ro_last_error(self.ctx))
+        assert k == r["n_retried"], (k, r["n_retried"])
+        return r
+
     # ------------------------------------------------------------ commit
     def commit(self, xid: int, child, state, length, off, gen=None,
                arena_bytes: int = (1 << 48) - 1, device_count: bool = False,
