@@ -458,3 +458,57 @@ int or_assemble(or_ctx* ctx, int32_t xid, const uint8_t* arena, uint64_t arena_b
   (void)arena_bytes;
   return OR_OK;
 }
+
+/* ------------------------------------------------------------------------ */
+/* List-structured Reduce output (Section 4.2): the parent's value is the
+ * list of its present members' values in ordinal order; the entries below
+ * let a reader split the concatenated bytes back into that list.  Dropped
+ * members are listed with their outcome and no bytes.                      */
+int or_assemble_list(or_ctx* ctx, int32_t xid, const uint8_t* arena, uint64_t arena_bytes,
+                     const uint32_t* parents, uint64_t n_parents, uint8_t* status,
+                     uint64_t* out_off, uint32_t* out_len, uint8_t* out, uint64_t out_cap,
+                     uint64_t* out_cursor, uint64_t* out_bytes, uint64_t* n_assembled,
+                     uint64_t* elem_base, uint8_t* elem_state, uint64_t* elem_off,
+                     uint32_t* elem_len, uint64_t elem_cap, uint64_t* n_elems) {
+  or_exp* x = get_exp(ctx, xid);
+  if (!x || !elem_base) return OR_E_INVAL;
+  const uint32_t* list = parents ? parents : x->last_done;
+  uint64_t n = parents ? n_parents : x->n_last_done;
+  uint64_t base = out_cursor ? *out_cursor : 0;
+  /* entries first: the members of every listed parent that is complete and
+     not suppressed */
+  uint64_t ne = 0;
+  for (uint64_t i = 0; i < n; ++i) {
+    uint64_t p = list[i];
+    if (p >= x->P || x->terminal[p] != member_count(x, p) || x->bad[p]) continue;
+    ne += member_count(x, p);
+  }
+  if (n_elems) *n_elems = ne;
+  if (ne > elem_cap) return OR_E_CAPACITY;
+  if (ne && (!elem_state || !elem_off || !elem_len)) return OR_E_INVAL;
+  int st = or_assemble(ctx, xid, arena, arena_bytes, parents, n_parents, status, out_off, out_len,
+                       out, out_cap, out_cursor, out_bytes, n_assembled);
+  if (st != OR_OK) return st;
+  uint64_t e = 0, pos = base;
+  for (uint64_t i = 0; i < n; ++i) {
+    uint64_t p = list[i];
+    elem_base[i] = e;
+    if (p >= x->P || x->terminal[p] != member_count(x, p) || x->bad[p]) continue;
+    for (uint64_t c = x->offsets[p]; c < x->offsets[p + 1]; ++c) {
+      elem_state[e] = x->st[c];
+      elem_off[e] = pos;
+      elem_len[e] = (x->st[c] == OR_PRESENT) ? x->len[c] : 0;
+      pos += elem_len[e];
+      ++e;
+    }
+  }
+  elem_base[n] = e;
+  return OR_OK;
+}
+
+/* F.filter (Table 3): pass on true, drop on false; inputs that failed or
+ * were suppressed keep their state (Section 4.2's propagation precedence). */
+void or_filter_reports(uint8_t* state, const uint8_t* keep, uint64_t n) {
+  for (uint64_t r = 0; r < n; ++r)
+    if (state[r] == OR_PRESENT && !keep[r]) state[r] = OR_DROPPED;
+}

@@ -95,6 +95,25 @@ int or_assemble(or_ctx* ctx, int32_t xid, const uint8_t* arena, uint64_t arena_b
                 uint64_t* out_off, uint32_t* out_len, uint8_t* out, uint64_t out_cap,
                 uint64_t* out_cursor, uint64_t* out_bytes, uint64_t* n_assembled);
 
+/* List-structured Reduce output (Section 4.2: present values in ordinal
+ * order; Table 3's F.reduce gathers a list).  Same as or_assemble, plus for
+ * every listed parent that is assembled Present the entries of its members
+ * in ordinal order: elem_base[i] .. elem_base[i+1] (elem_base has n+1
+ * entries); for each entry its outcome (PRESENT or DROPPED), the output
+ * offset of its bytes and their length (0 if Dropped).  Suppressed and
+ * incomplete parents have no entries.  elem_cap bounds the entries. */
+int or_assemble_list(or_ctx* ctx, int32_t xid, const uint8_t* arena, uint64_t arena_bytes,
+                     const uint32_t* parents, uint64_t n_parents, uint8_t* status,
+                     uint64_t* out_off, uint32_t* out_len, uint8_t* out, uint64_t out_cap,
+                     uint64_t* out_cursor, uint64_t* out_bytes, uint64_t* n_assembled,
+                     uint64_t* elem_base, uint8_t* elem_state, uint64_t* elem_off,
+                     uint32_t* elem_len, uint64_t elem_cap, uint64_t* n_elems);
+
+/* F.filter (Table 3; Section 4.2's propagation rule) applied to a batch of
+ * reports: a Present report whose mask is 0 becomes Dropped; every other
+ * report keeps its state (a failed or suppressed input stays so). */
+void or_filter_reports(uint8_t* state, const uint8_t* keep, uint64_t n);
+
 #ifdef __cplusplus
 }
 #endif

@@ -69,7 +69,13 @@ def lib():
         L.or_assemble.argtypes = [C.c_void_p, C.c_int32, _u8p, C.c_uint64, _u32p, C.c_uint64,
                                   _u8p, _u64p, _u32p, _u8p, C.c_uint64, _u64p, _u64p, _u64p]
         L.or_retry.argtypes = [C.c_void_p, C.c_int32, C.c_uint32, _u32p, C.c_uint64, _u64p]
-        for f in ("or_expand", "or_batch_ready", "or_gather_commit", "or_assemble", "or_retry"):
+        L.or_assemble_list.argtypes = [C.c_void_p, C.c_int32, _u8p, C.c_uint64, _u32p, C.c_uint64,
+                                       _u8p, _u64p, _u32p, _u8p, C.c_uint64, _u64p, _u64p, _u64p,
+                                       _u64p, _u8p, _u64p, _u32p, C.c_uint64, _u64p]
+        L.or_filter_reports.argtypes = [_u8p, _u8p, C.c_uint64]
+        L.or_filter_reports.restype = None
+        for f in ("or_expand", "or_batch_ready", "or_gather_commit", "or_assemble", "or_retry",
+                  "or_assemble_list"):
             getattr(L, f).restype = C.c_int
         _lib = L
     return _lib
@@ -162,6 +168,53 @@ class OracleCtx:
             raise OracleError("or_batch_ready", st)
         return dict(status=st, batched=out[:nb.value].copy() if st == OK else None,
                     n_batched=nb.value, n_batches=nbt.value)
+
+    def assemble_list(self, xid: int, arena: Optional[np.ndarray], parents=None,
+                      n_parents: Optional[int] = None, out_cap: Optional[int] = None,
+                      cursor: Optional[int] = None, elem_cap: Optional[int] = None,
+                      check: bool = True):
+        """Assemble plus the list structure: per listed parent its member
+        entries (outcome, output offset, length) in ordinal order."""
+        parents = _arr(parents, np.uint32)
+        n = parents.size if parents is not None else (n_parents if n_parents is not None else (1 << 22))
+        arena_u8 = _arr(arena, np.uint8)
+        arena_bytes = arena_u8.size
+        if out_cap is None:
+            sz = self.assemble(xid, None, parents=parents, n_parents=n_parents, check=False)
+            out_cap = (cursor or 0) + sz["out_bytes"]
+        if elem_cap is None:
+            elem_cap = self._n_children[xid]
+        status = np.zeros(max(n, 1), np.uint8)
+        out_off = np.zeros(n + 1, np.uint64)
+        out_len = np.zeros(max(n, 1), np.uint32)
+        out = np.zeros(max(out_cap, 1), np.uint8)
+        eb = np.zeros(n + 1, np.uint64)
+        es = np.zeros(max(elem_cap, 1), np.uint8)
+        eo = np.zeros(max(elem_cap, 1), np.uint64)
+        el = np.zeros(max(elem_cap, 1), np.uint32)
+        ob, na, ne = C.c_uint64(0), C.c_uint64(0), C.c_uint64(0)
+        cur = C.c_uint64(cursor) if cursor is not None else None
+        st = lib().or_assemble_list(self._h, xid, _ptr(arena_u8, _u8p), arena_bytes, _ptr(parents, _u32p),
+                                    n, _ptr(status, _u8p), _ptr(out_off, _u64p), _ptr(out_len, _u32p),
+                                    _ptr(out, _u8p), out_cap, C.byref(cur) if cur is not None else None,
+                                    C.byref(ob), C.byref(na), _ptr(eb, _u64p), _ptr(es, _u8p),
+                                    _ptr(eo, _u64p), _ptr(el, _u32p), elem_cap, C.byref(ne))
+        if check and st != OK:
+            raise OracleError("or_assemble_list", st)
+        k, m = na.value, ne.value
+        return dict(status=st, parent_status=status[:k].copy(), out_off=out_off[:k + 1].copy(),
+                    out_len=out_len[:k].copy(), out=out[:out_cap], out_bytes=ob.value,
+                    n_assembled=k, cursor=None if cur is None else cur.value,
+                    elem_base=eb[:k + 1].copy(), elem_state=es[:m].copy(), elem_off=eo[:m].copy(),
+                    elem_len=el[:m].copy(), n_elems=m)
+
+    @staticmethod
+    def filter_reports(state, keep):
+        """F.filter on a report batch (returns the new states)."""
+        st = np.ascontiguousarray(np.asarray(state, np.uint8)).copy()
+        kp = np.ascontiguousarray(np.asarray(keep, np.uint8))
+        lib().or_filter_reports(_ptr(st, _u8p), _ptr(kp, _u8p), st.size)
+        return st
 
     def retry(self, xid: int, call: int, children, check: bool = True):
         """Failed attempt: IN-FLIGHT Grains back to READY at generation + 1, as one

@@ -41,6 +41,11 @@ MUTANTS = {
                               "    for (uint64_t i = 0; i < nr; ++i) q[x->qhead[call] + i] = x->rq[call][nr - 1 - i];"),
     "retry_ignores_call": ("if (c >= x->N || x->phase[c] != OR_IN_FLIGHT || x->child_call[c] != call) {",
                            "if (c >= x->N || x->phase[c] != OR_IN_FLIGHT) {"),
+    # list-structured output and F.filter (Section 4.2, Table 3)
+    "list_state_lost": ("      elem_state[e] = x->st[c];", "      elem_state[e] = OR_PRESENT;"),
+    "list_base_off_by_one": ("  elem_base[n] = e;", "  elem_base[n] = e + 1;"),
+    "filter_drops_failed": ("if (state[r] == OR_PRESENT && !keep[r]) state[r] = OR_DROPPED;",
+                            "if (!keep[r]) state[r] = OR_DROPPED;"),
     "barrier_completion_missed": ("if (sealed_now && x->terminal[p] == member_count(x, p)) x->last_done[k++] = p;",
                                   "(void)sealed_now;"),
 }
@@ -60,6 +65,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
                         os.path.join(ROOT, "tests", "test_oracle.py"),
                         os.path.join(ROOT, "tests", "test_oracle_group_failure.py"),
-                        os.path.join(ROOT, "tests", "test_oracle_retry.py")],
+                        os.path.join(ROOT, "tests", "test_oracle_retry.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_lists.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode != 0, f"pins did not catch mutant {name}:\n{r.stdout[-2000:]}"
