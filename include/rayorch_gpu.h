@@ -314,6 +314,48 @@ ro_status ro_assemble(ro_ctx* ctx, int32_t xid, const uint8_t* d_arena, uint64_t
                       uint64_t* d_out_bytes, uint64_t* h_out_bytes);
 
 /* ------------------------------------------------------------------------
+ * ro_assemble_list — ro_assemble plus the list structure of each assembled
+ * parent (Section 4.2: the Reduce emits the present values in immutable
+ * ordinal order; Table 3's F.reduce gathers a list), so a reader can split
+ * each parent's concatenated bytes back into its ordered list.
+ *
+ * All arguments of ro_assemble, then:
+ *   d_elem_base  uint64[n+1] out: listed parent i's entries are
+ *                d_elem_base[i] .. d_elem_base[i+1]-1 (none unless it is
+ *                assembled Present).
+ *   d_elem_state uint8[elem_cap] out: per entry, in ordinal order, the
+ *                member's outcome (RO_PRESENT or RO_DROPPED).
+ *   d_elem_off   uint64[elem_cap] out: the offset in d_out of the member's
+ *                bytes (a Dropped member: where it would have been).
+ *   d_elem_len   uint32[elem_cap] out: the member's bytes (0 if Dropped).
+ *   elem_cap     entries the three arrays hold: every member of every listed
+ *                Present parent is an entry.
+ *   d_n_elems (device) / h_n_elems (host, synchronises) out or NULL: entries.
+ * Errors: those of ro_assemble; RO_E_CAPACITY also when the entries exceed
+ * elem_cap (then nothing is copied and the entry arrays are undefined).
+ * A parent whose members were all Dropped is Present with 0 bytes and its
+ * entries all RO_DROPPED: a present empty list.
+ */
+ro_status ro_assemble_list(ro_ctx* ctx, int32_t xid, const uint8_t* d_arena, uint64_t arena_bytes,
+                           const uint32_t* d_parents, uint64_t n_parents,
+                           const uint64_t* d_n_parents, uint8_t* d_status, uint64_t* d_out_off,
+                           uint32_t* d_out_len, uint8_t* d_out, uint64_t out_cap,
+                           uint64_t* d_out_cursor, uint64_t* d_out_bytes, uint64_t* h_out_bytes,
+                           uint64_t* d_elem_base, uint8_t* d_elem_state, uint64_t* d_elem_off,
+                           uint32_t* d_elem_len, uint64_t elem_cap, uint64_t* d_n_elems,
+                           uint64_t* h_n_elems);
+
+/* ------------------------------------------------------------------------
+ * ro_filter_reports — F.filter (Table 3: pass on true, drop on false) on a
+ * batch of reports before they are committed, with Section 4.2's
+ * propagation precedence: a RO_PRESENT report whose d_keep byte is 0
+ * becomes RO_DROPPED; every other report keeps its state (a failed or
+ * suppressed input stays so).  d_state uint8[n] in/out, d_keep uint8[n];
+ * runs on the context's stream.
+ */
+ro_status ro_filter_reports(ro_ctx* ctx, uint8_t* d_state, const uint8_t* d_keep, uint64_t n);
+
+/* ------------------------------------------------------------------------
  * ro_expand_noalloc — the offsets, parents and ordinals of ro_expand, for
  * callers that cannot allocate device memory.  The paper has no counterpart;
  * this is a deployment variant.

@@ -512,3 +512,22 @@ void or_filter_reports(uint8_t* state, const uint8_t* keep, uint64_t n) {
   for (uint64_t r = 0; r < n; ++r)
     if (state[r] == OR_PRESENT && !keep[r]) state[r] = OR_DROPPED;
 }
+
+int or_assemble_size(or_ctx* ctx, int32_t xid, const uint32_t* parents, uint64_t n_parents,
+                     uint64_t* bytes, uint64_t* elems) {
+  or_exp* x = get_exp(ctx, xid);
+  if (!x) return OR_E_INVAL;
+  const uint32_t* list = parents ? parents : x->last_done;
+  uint64_t n = parents ? n_parents : x->n_last_done;
+  uint64_t b = 0, e = 0;
+  for (uint64_t i = 0; i < n; ++i) {
+    uint64_t p = list[i];
+    if (p >= x->P || x->terminal[p] != member_count(x, p) || x->bad[p]) continue;
+    e += member_count(x, p);
+    for (uint64_t c = x->offsets[p]; c < x->offsets[p + 1]; ++c)
+      if (x->st[c] == OR_PRESENT) b += x->len[c];
+  }
+  if (bytes) *bytes = b;
+  if (elems) *elems = e;
+  return OR_OK;
+}

@@ -109,6 +109,11 @@ int or_assemble_list(or_ctx* ctx, int32_t xid, const uint8_t* arena, uint64_t ar
                      uint64_t* elem_base, uint8_t* elem_state, uint64_t* elem_off,
                      uint32_t* elem_len, uint64_t elem_cap, uint64_t* n_elems);
 
+/* Bytes and list entries an assembly of `parents` (NULL: the latest commit's
+ * completed parents) would produce; changes nothing (no counters). */
+int or_assemble_size(or_ctx* ctx, int32_t xid, const uint32_t* parents, uint64_t n_parents,
+                     uint64_t* bytes, uint64_t* elems);
+
 /* F.filter (Table 3; Section 4.2's propagation rule) applied to a batch of
  * reports: a Present report whose mask is 0 becomes Dropped; every other
  * report keeps its state (a failed or suppressed input stays so). */

@@ -72,6 +72,8 @@ def lib():
         L.or_assemble_list.argtypes = [C.c_void_p, C.c_int32, _u8p, C.c_uint64, _u32p, C.c_uint64,
                                        _u8p, _u64p, _u32p, _u8p, C.c_uint64, _u64p, _u64p, _u64p,
                                        _u64p, _u8p, _u64p, _u32p, C.c_uint64, _u64p]
+        L.or_assemble_size.argtypes = [C.c_void_p, C.c_int32, _u32p, C.c_uint64, _u64p, _u64p]
+        L.or_assemble_size.restype = C.c_int
         L.or_filter_reports.argtypes = [_u8p, _u8p, C.c_uint64]
         L.or_filter_reports.restype = None
         for f in ("or_expand", "or_batch_ready", "or_gather_commit", "or_assemble", "or_retry",
@@ -180,8 +182,7 @@ class OracleCtx:
         arena_u8 = _arr(arena, np.uint8)
         arena_bytes = arena_u8.size
         if out_cap is None:
-            sz = self.assemble(xid, None, parents=parents, n_parents=n_parents, check=False)
-            out_cap = (cursor or 0) + sz["out_bytes"]
+            out_cap = (cursor or 0) + self.assemble_size(xid, parents, n)[0]
         if elem_cap is None:
             elem_cap = self._n_children[xid]
         status = np.zeros(max(n, 1), np.uint8)
@@ -207,6 +208,12 @@ class OracleCtx:
                     n_assembled=k, cursor=None if cur is None else cur.value,
                     elem_base=eb[:k + 1].copy(), elem_state=es[:m].copy(), elem_off=eo[:m].copy(),
                     elem_len=el[:m].copy(), n_elems=m)
+
+    def assemble_size(self, xid: int, parents, n: int):
+        """(bytes, list entries) of an assembly, without changing anything."""
+        b, e = C.c_uint64(0), C.c_uint64(0)
+        lib().or_assemble_size(self._h, xid, _ptr(parents, _u32p), n, C.byref(b), C.byref(e))
+        return b.value, e.value
 
     @staticmethod
     def filter_reports(state, keep):
@@ -269,15 +276,7 @@ class OracleCtx:
             if sizes_only:
                 out_cap = (1 << 62)
             else:
-                # ask for the size first (capacity 0 reports the byte count)
-                ob = C.c_uint64(0)
-                na = C.c_uint64(0)
-                cur0 = C.c_uint64(cursor or 0)
-                lib().or_assemble(self._h, xid, _ptr(arena_u8, _u8p), arena_bytes,
-                                  _ptr(parents, _u32p), n, _ptr(status, _u8p),
-                                  _ptr(out_off, _u64p), None, None, 0,
-                                  C.byref(cur0), C.byref(ob), C.byref(na))
-                out_cap = (cursor or 0) + ob.value
+                out_cap = (cursor or 0) + self.assemble_size(xid, parents, n)[0]
         out = None if sizes_only else np.zeros(max(out_cap, 1), dtype=np.uint8)
         ob = C.c_uint64(0)
         na = C.c_uint64(0)

@@ -31,7 +31,8 @@ STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFL
 
 EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro_ctx_stats",
            "ro_ctx_set_streams", "ro_ctx_join", "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
-           "ro_retry", "ro_gather_commit", "ro_assemble", "ro_expand_noalloc")
+           "ro_retry", "ro_gather_commit", "ro_assemble", "ro_assemble_list", "ro_filter_reports",
+           "ro_expand_noalloc")
 
 # kernel ids (RO_K_*), in launch order of the path
 KERNELS = ("expand_scan", "expand_fill", "ready_count", "ready_scatter", "commit_scatter",
@@ -88,6 +89,9 @@ def load(path: Optional[str] = None):
                                    _vp, _pu64]
     L.ro_assemble.argtypes = [_vp, _i32, _vp, _u64, _vp, _u64, _vp, _vp, _vp, _vp, _vp, _u64, _vp, _vp,
                               _pu64]
+    L.ro_assemble_list.argtypes = [_vp, _i32, _vp, _u64, _vp, _u64, _vp, _vp, _vp, _vp, _vp, _u64, _vp,
+                                   _vp, _pu64, _vp, _vp, _vp, _vp, _u64, _vp, _pu64]
+    L.ro_filter_reports.argtypes = [_vp, _vp, _vp, _u64]
     L.ro_expand_noalloc.argtypes = [_vp, _u64, _vp, _vp, _vp, _u64, _vp, _vp, _pu64, _pu64]
     for f in EXPORTS:
         if f != "ro_last_error":
@@ -233,6 +237,27 @@ def ro_assemble(ctx, xid, d_arena, arena_bytes, d_parents, n_parents, d_n_parent
                             _ptr(d_out), out_cap, _ptr(d_out_cursor), _ptr(d_out_bytes),
                             C.byref(ob) if want_host else None)
     return (st, ob.value) if want_host else (st, None)
+
+
+def ro_assemble_list(ctx, xid, d_arena, arena_bytes, d_parents, n_parents, d_n_parents, d_status,
+                     d_out_off, d_out_len, d_out, out_cap, d_out_cursor, d_out_bytes, d_elem_base,
+                     d_elem_state, d_elem_off, d_elem_len, elem_cap, d_n_elems=None,
+                     want_host: bool = True):
+    """Returns (status, out_bytes, n_elems); the counts are None without want_host."""
+    ob = _u64(0)
+    ne = _u64(0)
+    st = load().ro_assemble_list(ctx, xid, _ptr(d_arena), arena_bytes, _ptr(d_parents), n_parents,
+                                 _ptr(d_n_parents), _ptr(d_status), _ptr(d_out_off), _ptr(d_out_len),
+                                 _ptr(d_out), out_cap, _ptr(d_out_cursor), _ptr(d_out_bytes),
+                                 C.byref(ob) if want_host else None, _ptr(d_elem_base),
+                                 _ptr(d_elem_state), _ptr(d_elem_off), _ptr(d_elem_len), elem_cap,
+                                 _ptr(d_n_elems), C.byref(ne) if want_host else None)
+    return (st, ob.value, ne.value) if want_host else (st, None, None)
+
+
+def ro_filter_reports(ctx, d_state, d_keep, n) -> int:
+    """F.filter on a report batch (in place, on the context's stream)."""
+    return load().ro_filter_reports(ctx, _ptr(d_state), _ptr(d_keep), n)
 
 
 def ro_expand_noalloc(d_counts, n_parents, d_offsets, d_child_parent, d_child_ordinal, child_cap,

@@ -143,7 +143,8 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    if (s_incomplete) atomicAdd(&ds->stats[6], s_incomplete);
+    // counted once the assembly succeeds (asm_copy)
+    if (s_incomplete) atomicAdd(&L.hdr->incomplete, s_incomplete);
     retire_cta(ds, TS_ASM_PARENTS, n_part);
   }
 }
@@ -162,12 +163,18 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
   const PlanBufs& pl = a.plan;
   const ListHdr lh = *L.hdr;
   const uint64_t n = lh.n, M = lh.M;
-  if (lh.err) {   // nothing to plan
+  // the list's entries must fit the caller's list-structure outputs
+  const bool elems_too_many = a.elem_base && M > a.elem_cap;
+  if (lh.err || elems_too_many) {   // nothing to plan
     if (blockIdx.x == 0 && threadIdx.x == 0) {
       pl.hdr->n = n;
       pl.hdr->bytes = 0;
       pl.hdr->nnz = 0;
+      pl.hdr->M = M;
+      pl.hdr->incomplete = 0;
       pl.hdr->err = 1u;
+      L.hdr->incomplete = 0;   // spent (asm_parents adds to it)
+      if (elems_too_many) atomicOr(&ds->err, ERR_CAPACITY);
     }
     return;
   }
@@ -175,6 +182,11 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
   const uint64_t par_units = ceil_div(n, (uint64_t)AM_TILE);
   const uint32_t n_part = participants((n_tiles > par_units ? n_tiles : par_units) + 1);
   if (blockIdx.x >= n_part) return;
+  if (a.elem_base) {   // each listed parent's first list entry (its member base)
+    const uint64_t stride = (uint64_t)n_part * blockDim.x;
+    for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i <= n; i += stride)
+      a.elem_base[i] = L.mb[i];
+  }
 
   if (M == 0) {   // nothing to gather: every listed parent starts at 0
     const uint64_t stride = (uint64_t)n_part * blockDim.x;
@@ -184,8 +196,11 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
       pl.hdr->n = n;
       pl.hdr->bytes = 0;
       pl.hdr->nnz = 0;
+      pl.hdr->M = 0;
+      pl.hdr->incomplete = lh.incomplete;
       pl.hdr->err = 0u;
       pl.hdr->chunks_ok = 1u;
+      L.hdr->incomplete = 0;   // spent (asm_parents adds to it)
     }
     return;
   }
@@ -307,6 +322,11 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
           pl.off[q] = pos;
         }
       }
+      if (a.elem_base) {   // the member's list entry (offset relative until the copy)
+        a.elem_state[g] = w_state(rr[k].w) == ST_PRESENT ? ST_PRESENT : ST_DROPPED;
+        a.elem_len[g] = contrib[k];
+        a.elem_off[g] = pos;
+      }
       if (contrib[k]) {
         const uint64_t j = run.b;
         if (j < pl.member_cap) {
@@ -329,11 +349,18 @@ __global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a)
       pl.hdr->n = n;
       pl.hdr->bytes = run.a;
       pl.hdr->nnz = run.b;
+      pl.hdr->M = M;
+      pl.hdr->incomplete = lh.incomplete;
       pl.hdr->chunks_ok = ceil_div(run.a, AC_CHUNK) <= pl.ctfp_cap ? 1u : 0u;
     }
     __syncthreads();
   }
-  if (threadIdx.x == 0) retire_cta(ds, TS_ASM_MEMBERS, n_part);
+  if (threadIdx.x == 0 && ticket(&ds->exit_ctr[TS_ASM_MEMBERS]) == n_part - 1) {
+    ds->tile_ctr[TS_ASM_MEMBERS] = 0u;
+    ds->exit_ctr[TS_ASM_MEMBERS] = 0u;
+    ds->epoch[TS_ASM_MEMBERS] += 1ull;
+    L.hdr->incomplete = 0;   // spent (asm_parents adds to it)
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -834,10 +861,14 @@ __global__ void __launch_bounds__(AC_THREADS, 2) asm_copy_kernel(AssembleArgs a)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   if (!failed) {
-    // per-parent outputs: status (commit plans), offsets, lengths
+    // per-parent outputs: status (commit plans), offsets, lengths, and the
+    // list structure's entry offsets made absolute
     {
       const uint64_t stride = (uint64_t)n_part * blockDim.x;
-      for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i <= n; i += stride) {
+      const uint64_t gt0 = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+      if (a.elem_base)
+        for (uint64_t g = gt0; g < hdr.M; g += stride) a.elem_off[g] += base;
+      for (uint64_t i = gt0; i <= n; i += stride) {
         const uint64_t o = a.plan.off[i];
         a.out_off[i] = base + o;
         if (i == n) break;
@@ -905,8 +936,11 @@ __global__ void __launch_bounds__(AC_THREADS, 2) asm_copy_kernel(AssembleArgs a)
   if (threadIdx.x == 0) {
     if (ticket(&ds->exit_ctr[TS_ASM_COPY]) == n_part - 1) {
       if (!failed && a.cursor) *a.cursor = base + S;
+      if (!failed && hdr.incomplete) ds->stats[6] += hdr.incomplete;
       if (a.out_bytes) *a.out_bytes = S;
+      if (a.n_elems_out) *a.n_elems_out = hdr.M;
       ds->as_bytes = S;
+      ds->as_elems = hdr.M;
       a.plan.hdr->err = 0u;   // the plan is consumed
       ds->exit_ctr[TS_ASM_COPY] = 0u;
     }
@@ -930,6 +964,19 @@ void launch_assemble_copy(const LaunchCfg& L, const AssembleArgs& a) {
 cudaError_t prepare_assemble_kernels() {
   return cudaFuncSetAttribute(asm_copy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)asm_copy_smem());
+}
+
+// F.filter (Table 3) on a report batch: Present with a false mask -> Dropped
+__global__ void filter_kernel(uint8_t* state, const uint8_t* keep, uint64_t n) {
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t r = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n; r += stride)
+    if (state[r] == ST_PRESENT && !keep[r]) state[r] = ST_DROPPED;
+}
+
+void launch_filter(cudaStream_t s, uint8_t* state, const uint8_t* keep, uint64_t n, int grid) {
+  const uint64_t need = ceil_div(n, 256);
+  const int g = (int)(need < (uint64_t)grid ? (need ? need : 1) : grid);
+  filter_kernel<<<g, 256, 0, s>>>(state, keep, n);
 }
 
 const void* kernel_ptr_assemble(int which) {

@@ -521,6 +521,7 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
       L.hdr->n = 0;
       L.hdr->M = 0;
       L.hdr->err = 0u;
+      L.hdr->incomplete = 0;
       L.mb[0] = 0;
       if (a.n_done_out) *a.n_done_out = 0;
     }
@@ -618,6 +619,7 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
       L.hdr->n = run.a;
       L.hdr->M = run.b;
       L.hdr->err = 0u;
+      L.hdr->incomplete = 0;
       L.mb[run.a] = (uint32_t)run.b;
       if (a.n_done_out) *a.n_done_out = run.a;
     }

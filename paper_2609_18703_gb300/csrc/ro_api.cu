@@ -808,11 +808,67 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
 }
 
 // ---------------------------------------------------------------------------
+namespace {
+struct ElemOut {
+  uint64_t* base;
+  uint8_t* state;
+  uint64_t* off;
+  uint32_t* len;
+  uint64_t cap;
+  uint64_t* d_n;
+  uint64_t* h_n;
+};
+ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t arena_bytes,
+                        const uint32_t* d_parents, uint64_t n_parents, const uint64_t* d_n_parents,
+                        uint8_t* d_status, uint64_t* d_out_off, uint32_t* d_out_len, uint8_t* d_out,
+                        uint64_t out_cap, uint64_t* d_out_cursor, uint64_t* d_out_bytes,
+                        uint64_t* h_out_bytes, const ElemOut* eo);
+}  // namespace
+
 ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t arena_bytes,
                       const uint32_t* d_parents, uint64_t n_parents, const uint64_t* d_n_parents,
                       uint8_t* d_status, uint64_t* d_out_off, uint32_t* d_out_len, uint8_t* d_out,
                       uint64_t out_cap, uint64_t* d_out_cursor, uint64_t* d_out_bytes,
                       uint64_t* h_out_bytes) {
+  return assemble_impl(c, xid, d_arena, arena_bytes, d_parents, n_parents, d_n_parents, d_status,
+                       d_out_off, d_out_len, d_out, out_cap, d_out_cursor, d_out_bytes, h_out_bytes,
+                       nullptr);
+}
+
+ro_status ro_assemble_list(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t arena_bytes,
+                           const uint32_t* d_parents, uint64_t n_parents,
+                           const uint64_t* d_n_parents, uint8_t* d_status, uint64_t* d_out_off,
+                           uint32_t* d_out_len, uint8_t* d_out, uint64_t out_cap,
+                           uint64_t* d_out_cursor, uint64_t* d_out_bytes, uint64_t* h_out_bytes,
+                           uint64_t* d_elem_base, uint8_t* d_elem_state, uint64_t* d_elem_off,
+                           uint32_t* d_elem_len, uint64_t elem_cap, uint64_t* d_n_elems,
+                           uint64_t* h_n_elems) {
+  RO_TRY(enter(c));
+  if (!d_elem_base || (elem_cap && (!d_elem_state || !d_elem_off || !d_elem_len)))
+    return fail(c, RO_E_INVAL, "ro_assemble_list: NULL list-structure output");
+  const ElemOut eo{d_elem_base, d_elem_state, d_elem_off, d_elem_len, elem_cap, d_n_elems, h_n_elems};
+  return assemble_impl(c, xid, d_arena, arena_bytes, d_parents, n_parents, d_n_parents, d_status,
+                       d_out_off, d_out_len, d_out, out_cap, d_out_cursor, d_out_bytes, h_out_bytes,
+                       &eo);
+}
+
+ro_status ro_filter_reports(ro_ctx* c, uint8_t* d_state, const uint8_t* d_keep, uint64_t n) {
+  RO_TRY(enter(c));
+  if (n && (!d_state || !d_keep)) return fail(c, RO_E_INVAL, "ro_filter_reports: NULL argument");
+  if (!n) return RO_OK;
+  DeviceGuard g(c->device);
+  launch_filter(c->stream, d_state, d_keep, n, c->num_sms * 8);
+  return check_launch(c, "filter_reports");
+}
+
+}  // extern "C"
+
+namespace {
+ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t arena_bytes,
+                        const uint32_t* d_parents, uint64_t n_parents, const uint64_t* d_n_parents,
+                        uint8_t* d_status, uint64_t* d_out_off, uint32_t* d_out_len, uint8_t* d_out,
+                        uint64_t out_cap, uint64_t* d_out_cursor, uint64_t* d_out_bytes,
+                        uint64_t* h_out_bytes, const ElemOut* eo) {
   RO_TRY(enter(c));
   Expansion* x = get_exp(c, xid);
   if (!x) return fail(c, RO_E_STATE, "ro_assemble: unknown expansion %d", xid);
@@ -852,6 +908,14 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   aa.out_cap = out_cap;
   aa.cursor = d_out_cursor;
   aa.out_bytes = d_out_bytes;
+  if (eo) {
+    aa.elem_base = eo->base;
+    aa.elem_state = eo->state;
+    aa.elem_off = eo->off;
+    aa.elem_len = eo->len;
+    aa.elem_cap = eo->cap;
+    aa.n_elems_out = eo->d_n;
+  }
   aa.plan = plan_bufs(PS, member_cap);
   aa.ds = c->ds;
   ListSlot* LS = nullptr;
@@ -896,12 +960,12 @@ ro_status ro_assemble(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t a
   // the copy reads the list's outcomes: the slot is free once it is done
   if (LS && c->copy_stream != c->stream) RO_TRY(ev_record(c, LS->freed, c->copy_stream));
   x->assembles += 1;
-  if (h_out_bytes) {
+  if (h_out_bytes || (eo && eo->h_n)) {
     ro_status st = sync_and_check(c);
-    *h_out_bytes = c->hs->as_bytes;
+    if (h_out_bytes) *h_out_bytes = c->hs->as_bytes;
+    if (eo && eo->h_n) *eo->h_n = c->hs->as_elems;
     return st;
   }
   return RO_OK;
 }
-
-}  // extern "C"
+}  // namespace

@@ -78,7 +78,7 @@ struct ListHdr {
   unsigned long long M;      // members of the listed Present parents
   uint32_t err;              // the list cannot be planned (capacity)
   uint32_t pad;
-  unsigned long long pad2;
+  unsigned long long incomplete;   // listed entries that are not complete parents
 };
 // Header of an assembly plan (see PlanBufs).
 struct PlanHdr {
@@ -87,6 +87,8 @@ struct PlanHdr {
   unsigned long long nnz;    // members that contribute bytes
   uint32_t err;              // the plan is void (a capacity or arena check failed)
   uint32_t chunks_ok;        // the chunk table covers every chunk
+  unsigned long long M;      // list entries (members of the listed Present parents)
+  unsigned long long incomplete;   // listed entries that are not complete parents
 };
 
 // Counters and small results that kernels hand to later kernels and to the
@@ -108,6 +110,7 @@ struct DevScalars {
   uint32_t cm_fix_ticket, cm_fix_done;
   // ro_assemble
   unsigned long long as_bytes;    // bytes of the latest assemble (host read-back)
+  unsigned long long as_elems;    // list entries of the latest assemble (host read-back)
   // dynamic tile counters / exit tickets / scan epochs, one per look-back kernel
   uint32_t tile_ctr[8];
   uint32_t exit_ctr[8];

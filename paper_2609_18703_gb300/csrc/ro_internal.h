@@ -207,6 +207,14 @@ struct AssembleArgs {
   uint64_t out_cap;
   uint64_t* cursor;           // optional (device)
   uint64_t* out_bytes;        // optional (device)
+  // list structure (optional; ro_assemble_list): per listed parent its first
+  // entry, per entry (member of a Present parent) outcome, offset, length
+  uint64_t* elem_base;
+  uint8_t* elem_state;
+  uint64_t* elem_off;
+  uint32_t* elem_len;
+  uint64_t elem_cap;
+  uint64_t* n_elems_out;      // optional (device)
   ListBufs list;
   PlanBufs plan;
   DevScalars* ds;
@@ -217,6 +225,8 @@ struct AssembleArgs {
 // the copy, each on its own stream
 void launch_assemble_plan(const LaunchCfg& L, const AssembleArgs& a);
 void launch_assemble_copy(const LaunchCfg& L, const AssembleArgs& a);
+// F.filter on a report batch (context-free)
+void launch_filter(cudaStream_t s, uint8_t* state, const uint8_t* keep, uint64_t n, int grid);
 
 
 

@@ -191,6 +191,57 @@ class Lockstep:
                 raise AssertionError(f"assembled bytes differ at {bad.size} positions, first {bad[:8]}")
         return dict(status=st, out_bytes=ob, out=out_dev, r=r)
 
+    def assemble_list(self, xid: int, arena_np: np.ndarray, arena_dev: torch.Tensor, parents=None,
+                      n_parents: Optional[int] = None, out_cap: Optional[int] = None,
+                      cursor: Optional[int] = None, elem_cap: Optional[int] = None) -> dict:
+        parents_np = None if parents is None else np.asarray(parents, np.uint32)
+        if elem_cap is None:
+            elem_cap = self.N[xid]
+        r = self.o.assemble_list(xid, arena_np, parents=parents_np, n_parents=n_parents,
+                                 out_cap=out_cap, cursor=cursor, elem_cap=elem_cap, check=False)
+        n_host = parents_np.size if parents_np is not None else n_parents
+        if out_cap is None:
+            out_cap = (cursor or 0) + r["out_bytes"]
+        out_dev = torch.zeros(max(out_cap, 1), dtype=torch.uint8, device="cuda")
+        d_par = None if parents_np is None else dev(parents_np, np.uint32)
+        d_status = empty(max(n_host, 1), np.uint8)
+        d_off = empty(max(n_host, 1) + 1, np.uint64)
+        d_len = empty(max(n_host, 1), np.uint32)
+        d_cur = dev(np.array([cursor], np.uint64), np.uint64) if cursor is not None else None
+        d_eb = empty(max(n_host, 1) + 1, np.uint64)
+        d_es = empty(max(elem_cap, 1), np.uint8)
+        d_eo = empty(max(elem_cap, 1), np.uint64)
+        d_el = empty(max(elem_cap, 1), np.uint32)
+        d_ne = empty(1, np.uint64)
+        st, ob, ne = ro.ro_assemble_list(self.ctx, xid, arena_dev, arena_dev.numel(), d_par, n_host, None,
+                                         d_status, d_off, d_len, out_dev, out_cap, d_cur, None, d_eb,
+                                         d_es, d_eo, d_el, elem_cap, d_ne)
+        assert st == r["status"], (st, r["status"], ro.ro_last_error(self.ctx))
+        if st != ro.RO_OK:
+            return r
+        k, m = r["n_assembled"], r["n_elems"]
+        assert ob == r["out_bytes"] and ne == m and int(host(d_ne, np.uint64, 1)[0]) == m
+        assert np.array_equal(host(d_status, np.uint8, k), r["parent_status"])
+        assert np.array_equal(host(d_off, np.uint64, k + 1), r["out_off"])
+        assert np.array_equal(host(d_len, np.uint32, k), r["out_len"])
+        assert np.array_equal(host(d_eb, np.uint64, k + 1), r["elem_base"])
+        assert np.array_equal(host(d_es, np.uint8, m), r["elem_state"])
+        assert np.array_equal(host(d_eo, np.uint64, m), r["elem_off"])
+        assert np.array_equal(host(d_el, np.uint32, m), r["elem_len"])
+        base = cursor or 0
+        if ob:
+            assert np.array_equal(out_dev[base:base + ob].cpu().numpy(), r["out"][base:base + ob])
+        return r
+
+    def filter(self, state, keep) -> np.ndarray:
+        want = self.o.filter_reports(state, keep)
+        d_s = dev(np.asarray(state, np.uint8), np.uint8)
+        d_k = dev(np.asarray(keep, np.uint8), np.uint8)
+        assert ro.ro_filter_reports(self.ctx, d_s, d_k, len(want)) == ro.RO_OK
+        got = host(d_s, np.uint8, len(want))
+        assert np.array_equal(got, want)
+        return want
+
     def check_stats(self):
         g = ro.ro_ctx_stats(self.ctx)
         assert g.pop("status") == ro.RO_OK
