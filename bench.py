@@ -60,6 +60,10 @@ def parse():
                     help="failure-containment pass (GroupFailure at ordinal 0 of the largest parents)")
     ap.add_argument("--rq4-waves", type=int, default=64)
     ap.add_argument("--rq4-parents", type=int, default=99)
+    ap.add_argument("--lists", action="store_true",
+                    help="assemble with ro_assemble_list (per-member list entries, Section 4.2)")
+    ap.add_argument("--filter-drop", type=float, default=0.0,
+                    help="F.filter each wave's reports first; fraction the predicate rejects")
     ap.add_argument("--one-stream", action="store_true",
                     help="plan and copy on the context's stream (no overlap across waves)")
     ap.add_argument("--no-e2e", action="store_true")
@@ -199,7 +203,7 @@ def run_reference(args, rank):
 class Pass:
     """Device-resident inputs and outputs of one document->page microbatch."""
 
-    def __init__(self, lv, device, stream):
+    def __init__(self, lv, device, stream, lists=False, filter_drop=0.0):
         import torch
         from workload.device import fill_payload
         self.torch = torch
@@ -236,6 +240,30 @@ class Pass:
         self.out_len = torch.empty(self.P, dtype=torch.int32, device=dev)
         self.cursor = torch.zeros(1, dtype=torch.int64, device=dev)
         self.out_bytes = torch.zeros(self.W, dtype=torch.int64, device=dev)
+        self.lists = lists
+        if lists:
+            # wave w's list entries and entry ranges go to windows of their own,
+            # sized by the parents whose last report arrives in that wave
+            wave_of = np.empty(self.N, np.int64)
+            for w in range(self.W):
+                wave_of[arr[self.bounds[w]:self.bounds[w + 1]]] = w
+            off = np.concatenate([[0], np.cumsum(lv.counts.astype(np.int64))])
+            nz = np.flatnonzero(lv.counts > 0)
+            last = np.maximum.reduceat(wave_of, off[nz]) if nz.size else np.zeros(0, np.int64)
+            ent = np.bincount(last, weights=lv.counts[nz].astype(np.int64), minlength=self.W)
+            par = np.bincount(last, minlength=self.W)
+            self.ent_cap = ent.astype(np.int64)
+            self.ent_at = np.concatenate([[0], np.cumsum(self.ent_cap)])
+            self.base_at = np.concatenate([[0], np.cumsum(par + 1)])
+            self.elem_base = torch.empty(int(self.base_at[-1]), dtype=torch.int64, device=dev)
+            self.elem_state = torch.empty(max(self.N, 1), dtype=torch.uint8, device=dev)
+            self.elem_off = torch.empty(max(self.N, 1), dtype=torch.int64, device=dev)
+            self.elem_len = torch.empty(max(self.N, 1), dtype=torch.int32, device=dev)
+            self.n_elems = torch.zeros(self.W, dtype=torch.int64, device=dev)
+        self.keep = None
+        if filter_drop > 0:
+            rng = np.random.default_rng([0x46494C54, int(lv.payload_seed) & 0xFFFFFFFF])
+            self.keep = u8((rng.random(self.N) >= filter_drop).astype(np.uint8))
 
     def expand(self, ro, ctx):
         st, n, ne, xid = ro.ro_expand(ctx, -1, self.counts, self.P, None, self.offsets, self.cp,
@@ -260,8 +288,19 @@ class Pass:
         cur, obw = self.cursor.data_ptr(), self.out_bytes.data_ptr()
         for w in range(self.W):
             s, e = int(self.bounds[w]), int(self.bounds[w + 1])
+            if self.keep is not None:
+                bad |= L.ro_filter_reports(ctx, sb + s, self.keep.data_ptr() + s, e - s)
             bad |= L.ro_gather_commit(ctx, xid, e - s, None, cb + 4 * s, sb + s, lb + 4 * s,
                                       ob + 8 * s, None, self.arena_bytes, None, None, 0, None, None)
+            if self.lists:
+                a0, b0 = int(self.ent_at[w]), int(self.base_at[w])
+                bad |= L.ro_assemble_list(
+                    ctx, xid, ar, self.arena_bytes, None, self.P, None, st_p, oo, ol, out,
+                    self.out_cap, cur, obw + 8 * w, None, self.elem_base.data_ptr() + 8 * b0,
+                    self.elem_state.data_ptr() + a0, self.elem_off.data_ptr() + 8 * a0,
+                    self.elem_len.data_ptr() + 4 * a0, int(self.ent_cap[w]),
+                    self.n_elems.data_ptr() + 8 * w, None)
+                continue
             bad |= L.ro_assemble(ctx, xid, ar, self.arena_bytes, None, self.P, None, st_p, oo, ol,
                                  out, self.out_cap, cur, obw + 8 * w, None)
         bad |= L.ro_ctx_join(ctx)   # the copies of the last waves, back into the context's stream
@@ -281,7 +320,7 @@ def run_ours(args, rank, world, local_rank):
     lv = docpage(parents=args.parents, waves=args.waves, salt=rank).top
     stream = torch.cuda.Stream()
     torch.cuda.set_stream(stream)
-    ps = Pass(lv, local_rank, stream)
+    ps = Pass(lv, local_rank, stream, lists=args.lists, filter_drop=args.filter_drop)
     ctx = ro.ro_ctx_create(local_rank, stream, 1)
     if not args.one_stream:   # assembly planning and copies overlap later waves' commits
         plan_stream, copy_stream = torch.cuda.Stream(), torch.cuda.Stream()
@@ -364,6 +403,11 @@ def run_ours(args, rank, world, local_rank):
     copy_bytes = 2.0 * S * kt_steps   # payload read + write, algorithmic
     achieved = copy_bytes / (copy_ms * 1e-3) / 1e9 if copy_ms > 0 else 0.0
     pass_alg = 33.0 * ps.N + 25.0 * ps.P + 2.0 * S
+    n_entries = int(ps.n_elems.sum().item()) if ps.lists else 0
+    if ps.lists:   # per entry: state, offset, length; per listed parent: its range start
+        pass_alg += 13.0 * n_entries + 8.0 * (ps.P + ps.W)
+    if ps.keep is not None:   # F.filter reads state and predicate, writes state
+        pass_alg += 3.0 * ps.N
     kernel_ms = {k: round(v[2] / kt_steps, 4) for k, v in prof.items() if v[1]}
 
     # ---- end to end through the C ABI with host buffers
@@ -390,6 +434,9 @@ def run_ours(args, rank, world, local_rank):
                                    f"{args.waves} arrival waves, batch {ps.B}",
                        "parents": ps.P, "children": ps.N, "waves": args.waves,
                        "arena_bytes": ps.arena_bytes, "assembled_bytes": S,
+                       "output": "list entries per member" if ps.lists else "bytes",
+                       "list_entries": n_entries if ps.lists else None,
+                       "filter_drop": args.filter_drop,
                        "cuda_graph": graph is not None,
                        "streams": 1 if args.one_stream else 3,
                        "l2": "inputs larger than L2 (39 GB arena)",

@@ -9,6 +9,8 @@
  *                     child's immediate parent and immutable ordinal.
  *   ro_batch_ready    Section 4.3, Eq. (2): per-Call FIFO Ready Queue and
  *                     elastic reservation into fixed-size batches.
+ *   ro_batch_ready_parent  Section 4.3: the same queue with parent-bound
+ *                     reservation (each batch holds siblings of one parent).
  *   ro_gather_commit  Section 4.4, Eq. (3) and Section 4.2 (Reduce):
  *                     generation-fenced commit of out-of-order child results,
  *                     per-parent terminal counting, completed-parent list.
@@ -148,7 +150,9 @@ const char* ro_last_error(const ro_ctx* ctx);
 enum {
   RO_K_EXPAND_SCAN = 0, RO_K_EXPAND_FILL = 1, RO_K_READY_COUNT = 2, RO_K_READY_SCATTER = 3,
   RO_K_COMMIT_SCATTER = 4, RO_K_COMMIT_FINISH = 5, RO_K_ASM_PARENTS = 6, RO_K_ASM_MEMBERS = 7,
-  RO_K_ASM_COPY = 8, RO_K_RETRY_CLAIM = 9, RO_K_RETRY_SCATTER = 10, RO_K_COUNT = 11
+  RO_K_ASM_COPY = 8, RO_K_RETRY_CLAIM = 9, RO_K_RETRY_SCATTER = 10, RO_K_PB_KEYS = 11,
+  RO_K_PB_HIST = 12, RO_K_PB_ROWSCAN = 13, RO_K_PB_SORT = 14, RO_K_PB_BOUNDS = 15,
+  RO_K_PB_RANK = 16, RO_K_PB_SCAN = 17, RO_K_PB_EMIT = 18, RO_K_COUNT = 19
 };
 /* Tracing (no counterpart in the paper; it instruments the path).  Every
  * kernel launch is counted; kernels whose bit (1 << RO_K_*) is set in
@@ -216,6 +220,42 @@ ro_status ro_batch_ready(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t
                          uint64_t n_cand, uint32_t batch_size, int32_t flush,
                          uint32_t* d_batched, uint64_t batched_cap, uint64_t* d_n_batched,
                          uint64_t* h_n_batched, uint64_t* h_n_batches);
+
+/* ------------------------------------------------------------------------
+ * ro_batch_ready_parent — admission into the per-Call FIFO Ready Queue and
+ * parent-bound reservation (Section 4.3, Eq. 2).
+ *
+ * Admission is that of ro_batch_ready.  Then reservations are made one after
+ * another: each takes up to batch_size queued siblings of the parent of the
+ * queue's first entry, in queue order (READY -> IN-FLIGHT), and every entry
+ * it leaves keeps its place relative to the others.  Without flush a
+ * reservation that would hold fewer than batch_size siblings is not made and
+ * the queue waits for more of that parent's siblings (as ro_batch_ready waits
+ * for a whole batch); with flush != 0 reservations repeat until the queue is
+ * empty.  Recovery groups (ro_retry) enter ahead of the queue's entries first.
+ *
+ *   d_cand, n_cand, batch_size, flush   as in ro_batch_ready.
+ *   d_batched    uint32[batched_cap] out: the batches back to back; each
+ *                holds children of one parent.
+ *   d_batch_off  uint64[batch_off_cap] out or NULL: n_batches + 1 batch
+ *                boundaries; batch k is d_batched[d_batch_off[k] ..
+ *                d_batch_off[k+1]).
+ *   d_n_batched, d_n_batches  uint64 out (device) or NULL.
+ *   h_n_batched, h_n_batches  out (host) or NULL; either makes the call
+ *                synchronise.
+ * Errors: RO_E_CAPACITY when more would be reserved than batched_cap, or
+ * d_batch_off cannot hold n_batches + 1 entries (reported when the context
+ * next synchronises; the admission is undone, the outputs are undefined).
+ * Device scratch of about 44 bytes per child and 8 per parent of the
+ * expansion is allocated at the first call (like ro_batch_ready, this call
+ * cannot be the first to size it inside a stream capture).
+ */
+ro_status ro_batch_ready_parent(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* d_cand,
+                                uint64_t n_cand, uint32_t batch_size, int32_t flush,
+                                uint32_t* d_batched, uint64_t batched_cap, uint64_t* d_batch_off,
+                                uint64_t batch_off_cap, uint64_t* d_n_batched,
+                                uint64_t* d_n_batches, uint64_t* h_n_batched,
+                                uint64_t* h_n_batches);
 
 /* ------------------------------------------------------------------------
  * ro_retry — a failed physical attempt is tried again (Section 4.4: the

@@ -204,15 +204,13 @@ int or_expand(or_ctx* ctx, int32_t parent_xid, const uint32_t* counts, uint64_t 
 
 /* ------------------------------------------------------------------------ */
 /* Per-Call FIFO Ready Queue (Section 4.3, Eq. 2).  Candidates are admitted
- * in the order given, WAITING -> READY, if they belong to this Call; the
- * elastic policy then takes up to B queued Grains at a time from the front,
- * whatever their parents, READY -> IN-FLIGHT.  Only whole batches are taken,
- * except on flush, which also takes the last partial batch.                */
-int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand,
-                   uint64_t n_cand, uint32_t batch_size, int32_t flush, uint32_t* batched,
-                   uint64_t batched_cap, uint64_t* n_batched, uint64_t* n_batches) {
-  or_exp* x = get_exp(ctx, xid);
-  if (!x || call >= ctx->n_calls || batch_size == 0) return OR_E_INVAL;
+ * in the order given, WAITING -> READY, if they belong to this Call.  What
+ * precedes a reservation of either policy: recovery groups move ahead of the
+ * queue's entries, queued Grains sealed since (GroupFailure) leave, and the
+ * candidates are admitted behind the tail.  *old_tail gets the tail before
+ * admission (to undo it), *bad_cand the candidates naming no child.        */
+static int ready_admit(or_ctx* ctx, or_exp* x, uint32_t call, const uint32_t* cand,
+                       uint64_t n_cand, uint64_t* old_tail, uint64_t* bad_cand) {
   if (!cand) n_cand = x->N;
   if (!x->q[call]) {
     x->q[call] = (uint32_t*)malloc((x->N ? x->N : 1) * sizeof(uint32_t));
@@ -240,27 +238,49 @@ int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand
       ctx->stats.queue_dropped++;
   }
   x->qtail[call] = kept;
-  uint64_t old_tail = x->qtail[call];
+  *old_tail = x->qtail[call];
 
   /* admission: candidates in order; only WAITING Grains of this Call enter */
-  uint64_t bad_cand = 0;
+  uint64_t bad = 0;
   for (uint64_t i = 0; i < n_cand; ++i) {
     uint64_t c = cand ? cand[i] : i;
-    if (c >= x->N) { ++bad_cand; continue; }
+    if (c >= x->N) { ++bad; continue; }
     if (x->phase[c] != OR_WAITING) continue;
     if (x->child_call[c] != call) continue;
     x->phase[c] = OR_READY;
     q[x->qtail[call]++] = (uint32_t)c;
   }
+  *bad_cand = bad;
+  return OR_OK;
+}
+
+/* Undo an admission (a reservation that did not fit): the call can be
+ * repeated with more room. */
+static void ready_unadmit(or_exp* x, uint32_t call, uint64_t old_tail) {
+  uint32_t* q = x->q[call];
+  for (uint64_t t = old_tail; t < x->qtail[call]; ++t) x->phase[q[t]] = OR_WAITING;
+  x->qtail[call] = old_tail;
+}
+
+/* Elastic reservation takes up to B queued Grains at a time from the front,
+ * whatever their parents, READY -> IN-FLIGHT.  Only whole batches are taken,
+ * except on flush, which also takes the last partial batch.                */
+int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand,
+                   uint64_t n_cand, uint32_t batch_size, int32_t flush, uint32_t* batched,
+                   uint64_t batched_cap, uint64_t* n_batched, uint64_t* n_batches) {
+  or_exp* x = get_exp(ctx, xid);
+  if (!x || call >= ctx->n_calls || batch_size == 0) return OR_E_INVAL;
+  uint64_t old_tail, bad_cand;
+  int rc = ready_admit(ctx, x, call, cand, n_cand, &old_tail, &bad_cand);
+  if (rc != OR_OK) return rc;
+  uint32_t* q = x->q[call];
 
   /* reservation: whole batches of B from the head (all on flush) */
   uint64_t queued = x->qtail[call] - x->qhead[call];
   uint64_t take = flush ? queued : (queued / batch_size) * batch_size;
   if (n_batched) *n_batched = take;
   if (take > batched_cap || (take && !batched)) {
-    /* undo the admission so that the call can be retried */
-    for (uint64_t t = old_tail; t < x->qtail[call]; ++t) x->phase[q[t]] = OR_WAITING;
-    x->qtail[call] = old_tail;
+    ready_unadmit(x, call, old_tail);
     return take > batched_cap ? OR_E_CAPACITY : OR_E_INVAL;
   }
   for (uint64_t i = 0; i < take; ++i) {
@@ -272,6 +292,94 @@ int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand
   if (n_batches) *n_batches = (take + batch_size - 1) / batch_size;
   ctx->stats.ready_bad_candidates += bad_cand;
   return OR_OK;
+}
+
+/* Parent-bound reservation (Section 4.3): one reservation takes up to B
+ * queued siblings of the parent of the queue's first entry, in queue order;
+ * every entry it leaves keeps its place relative to the others.
+ * Reservations repeat while they can be made.  Without flush a reservation
+ * that would hold fewer than B siblings is not made, and the queue waits
+ * for more of that parent's siblings (as elastic reservation waits for a
+ * whole batch); with flush reservations repeat until the queue is empty.
+ * Kept as the steps read: the queue is a doubly linked list in queue order
+ * and each parent's queued entries a singly linked list in queue order.   */
+int or_batch_ready_parent(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand,
+                          uint64_t n_cand, uint32_t batch_size, int32_t flush,
+                          uint32_t* batched, uint64_t batched_cap, uint64_t* batch_off,
+                          uint64_t batch_off_cap, uint64_t* n_batched, uint64_t* n_batches) {
+  or_exp* x = get_exp(ctx, xid);
+  if (!x || call >= ctx->n_calls || batch_size == 0) return OR_E_INVAL;
+  uint64_t old_tail, bad_cand;
+  int rc = ready_admit(ctx, x, call, cand, n_cand, &old_tail, &bad_cand);
+  if (rc != OR_OK) return rc;
+  uint32_t* q = x->q[call];
+  const uint64_t h = x->qhead[call], n = x->qtail[call] - h;
+
+  int64_t* prev = (int64_t*)malloc((n ? n : 1) * sizeof(int64_t));
+  int64_t* next = (int64_t*)malloc((n ? n : 1) * sizeof(int64_t));
+  int64_t* sib = (int64_t*)malloc((n ? n : 1) * sizeof(int64_t));
+  int64_t* first = (int64_t*)malloc((x->P ? x->P : 1) * sizeof(int64_t));
+  int64_t* last = (int64_t*)malloc((x->P ? x->P : 1) * sizeof(int64_t));
+  uint32_t* out = (uint32_t*)malloc((n ? n : 1) * sizeof(uint32_t));
+  uint64_t* bo = (uint64_t*)malloc((n + 1) * sizeof(uint64_t));
+  const uint64_t pick_cap = batch_size < n ? batch_size : n;   /* a batch never exceeds the queue */
+  int64_t* pick = (int64_t*)malloc((pick_cap ? pick_cap : 1) * sizeof(int64_t));
+  if (!prev || !next || !sib || !first || !last || !out || !bo || !pick) {
+    free(prev); free(next); free(sib); free(first); free(last); free(out); free(bo); free(pick);
+    ready_unadmit(x, call, old_tail);
+    return OR_E_OOM;
+  }
+  for (uint64_t p = 0; p < x->P; ++p) first[p] = last[p] = -1;
+  for (uint64_t i = 0; i < n; ++i) {
+    prev[i] = (int64_t)i - 1;
+    next[i] = i + 1 < n ? (int64_t)i + 1 : -1;
+    sib[i] = -1;
+    uint32_t p = x->child_parent[q[h + i]];
+    if (first[p] < 0) first[p] = (int64_t)i; else sib[last[p]] = (int64_t)i;
+    last[p] = (int64_t)i;
+  }
+  int64_t front = n ? 0 : -1;
+  uint64_t take = 0, nb = 0;
+  while (front >= 0) {
+    /* the first ready parent: the parent of the queue's first entry */
+    uint32_t p = x->child_parent[q[h + front]];
+    uint64_t k = 0;
+    int64_t e = first[p];
+    while (e >= 0 && k < batch_size) { pick[k++] = e; e = sib[e]; }
+    if (k < batch_size && !flush) break;   /* short of B: wait for more siblings */
+    bo[nb++] = take;
+    for (uint64_t j = 0; j < k; ++j) {
+      int64_t t = pick[j];
+      out[take++] = q[h + t];
+      if (prev[t] >= 0) next[prev[t]] = next[t]; else front = next[t];
+      if (next[t] >= 0) prev[next[t]] = prev[t];
+    }
+    first[p] = e;
+  }
+  bo[nb] = take;
+
+  if (n_batched) *n_batched = take;
+  if (n_batches) *n_batches = nb;
+  int bad = take > batched_cap ? OR_E_CAPACITY
+          : (batch_off && nb + 1 > batch_off_cap) ? OR_E_CAPACITY
+          : (take && !batched) ? OR_E_INVAL : OR_OK;
+  if (bad != OR_OK) {
+    ready_unadmit(x, call, old_tail);
+  } else {
+    for (uint64_t i = 0; i < take; ++i) {
+      batched[i] = out[i];
+      x->phase[out[i]] = OR_IN_FLIGHT;
+    }
+    if (batch_off) memcpy(batch_off, bo, (nb + 1) * sizeof(uint64_t));
+    /* the entries left, in queue order, behind the new head */
+    uint64_t r = 0;
+    for (int64_t t = front; t >= 0; t = next[t]) out[r++] = q[h + t];
+    memcpy(q + h + take, out, r * sizeof(uint32_t));
+    x->qhead[call] = h + take;
+    ctx->stats.ready_bad_candidates += bad_cand;
+  }
+  free(prev); free(next); free(sib); free(first); free(last); free(out); free(bo); free(pick);
+  return bad;
 }
 
 /* ------------------------------------------------------------------------ */

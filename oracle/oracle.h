@@ -69,6 +69,19 @@ int or_batch_ready(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand
                    uint64_t n_cand, uint32_t batch_size, int32_t flush, uint32_t* batched,
                    uint64_t batched_cap, uint64_t* n_batched, uint64_t* n_batches);
 
+/* Parent-bound reservation (Section 4.3): admission as or_batch_ready, then
+ * reservations that each take up to B queued siblings of the parent of the
+ * queue's first entry (queue order), leaving the other entries in order;
+ * repeated while a whole batch of B siblings is at hand (flush: until the
+ * queue is empty).  batched gets the batches back to back; batch_off (or
+ * NULL) n_batches + 1 boundaries, batch k = batched[batch_off[k] ..
+ * batch_off[k+1]).  OR_E_CAPACITY (nothing changes but the queue prelude)
+ * when batched_cap or batch_off_cap is too small. */
+int or_batch_ready_parent(or_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* cand,
+                          uint64_t n_cand, uint32_t batch_size, int32_t flush,
+                          uint32_t* batched, uint64_t batched_cap, uint64_t* batch_off,
+                          uint64_t batch_off_cap, uint64_t* n_batched, uint64_t* n_batches);
+
 /* Retry of a failed physical attempt (Section 4.4; Eq. 2 IN-FLIGHT -> READY;
  * Section 4.3 recovery queues): each listed Grain of this Call that is
  * IN-FLIGHT (first occurrence in the list) goes back to READY with its

@@ -62,6 +62,10 @@ def lib():
         L.or_ctx_stats.argtypes = [C.c_void_p, C.POINTER(_Stats)]
         L.or_expand.argtypes = [C.c_void_p, C.c_int32, _u32p, C.c_uint64, _u8p, _u64p, _u32p,
                                 _u32p, C.c_uint64, _u32p, _u64p, _u64p, _i32p]
+        L.or_batch_ready_parent.argtypes = [C.c_void_p, C.c_int32, C.c_uint32, _u32p, C.c_uint64,
+                                            C.c_uint32, C.c_int32, _u32p, C.c_uint64, _u64p,
+                                            C.c_uint64, _u64p, _u64p]
+        L.or_batch_ready_parent.restype = C.c_int
         L.or_batch_ready.argtypes = [C.c_void_p, C.c_int32, C.c_uint32, _u32p, C.c_uint64,
                                      C.c_uint32, C.c_int32, _u32p, C.c_uint64, _u64p, _u64p]
         L.or_gather_commit.argtypes = [C.c_void_p, C.c_int32, C.c_uint64, _u32p, _u8p, _u32p,
@@ -93,7 +97,9 @@ def _ptr(a: Optional[np.ndarray], ctype):
 def _arr(a, dtype) -> Optional[np.ndarray]:
     if a is None:
         return None
-    return np.ascontiguousarray(np.asarray(a), dtype=dtype)
+    a = np.ascontiguousarray(np.asarray(a), dtype=dtype)
+    # an empty list stays a list (a valid pointer), unlike NULL ("all")
+    return a if a.size else np.zeros(1, dtype)[:0]
 
 
 class OracleCtx:
@@ -169,6 +175,31 @@ class OracleCtx:
         if check and st != OK:
             raise OracleError("or_batch_ready", st)
         return dict(status=st, batched=out[:nb.value].copy() if st == OK else None,
+                    n_batched=nb.value, n_batches=nbt.value)
+
+    def batch_ready_parent(self, xid: int, call: int = 0, cand=None, batch_size: int = 1,
+                           flush: bool = False, cap: Optional[int] = None,
+                           off_cap: Optional[int] = None, check: bool = True):
+        """Admission plus parent-bound reservation (Section 4.3); the batches
+        are batched[batch_off[k]:batch_off[k+1]]."""
+        cand = _arr(cand, np.uint32)
+        n_cand = 0 if cand is None else cand.size
+        if cap is None:
+            cap = self._n_children[xid]
+        if off_cap is None:
+            off_cap = cap + 1
+        out = np.zeros(max(cap, 1), dtype=np.uint32)
+        offs = np.zeros(max(off_cap, 1), dtype=np.uint64)
+        nb = C.c_uint64(0)
+        nbt = C.c_uint64(0)
+        st = lib().or_batch_ready_parent(self._h, xid, call, _ptr(cand, _u32p), n_cand, batch_size,
+                                         int(flush), _ptr(out, _u32p), cap, _ptr(offs, _u64p),
+                                         off_cap, C.byref(nb), C.byref(nbt))
+        if check and st != OK:
+            raise OracleError("or_batch_ready_parent", st)
+        ok = st == OK
+        return dict(status=st, batched=out[:nb.value].copy() if ok else None,
+                    batch_off=offs[:nbt.value + 1].copy() if ok else None,
                     n_batched=nb.value, n_batches=nbt.value)
 
     def assemble_list(self, xid: int, arena: Optional[np.ndarray], parents=None,

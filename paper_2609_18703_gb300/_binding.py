@@ -31,12 +31,14 @@ STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFL
 
 EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro_ctx_stats",
            "ro_ctx_set_streams", "ro_ctx_join", "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
-           "ro_retry", "ro_gather_commit", "ro_assemble", "ro_assemble_list", "ro_filter_reports",
+           "ro_retry", "ro_batch_ready_parent", "ro_gather_commit", "ro_assemble", "ro_assemble_list", "ro_filter_reports",
            "ro_expand_noalloc")
 
 # kernel ids (RO_K_*), in launch order of the path
 KERNELS = ("expand_scan", "expand_fill", "ready_count", "ready_scatter", "commit_scatter",
-           "commit_finish", "asm_parents", "asm_members", "asm_copy", "retry_claim", "retry_scatter")
+           "commit_finish", "asm_parents", "asm_members", "asm_copy", "retry_claim", "retry_scatter",
+           "pb_keys", "pb_hist", "pb_rowscan", "pb_sort", "pb_bounds", "pb_rank", "pb_scan",
+           "pb_emit")
 
 
 class RoError(RuntimeError):
@@ -92,6 +94,8 @@ def load(path: Optional[str] = None):
     L.ro_assemble_list.argtypes = [_vp, _i32, _vp, _u64, _vp, _u64, _vp, _vp, _vp, _vp, _vp, _u64, _vp,
                                    _vp, _pu64, _vp, _vp, _vp, _vp, _u64, _vp, _pu64]
     L.ro_filter_reports.argtypes = [_vp, _vp, _vp, _u64]
+    L.ro_batch_ready_parent.argtypes = [_vp, _i32, C.c_uint32, _vp, _u64, C.c_uint32, _i32, _vp,
+                                        _u64, _vp, _u64, _vp, _vp, _pu64, _pu64]
     L.ro_expand_noalloc.argtypes = [_vp, _u64, _vp, _vp, _vp, _u64, _vp, _vp, _pu64, _pu64]
     for f in EXPORTS:
         if f != "ro_last_error":
@@ -253,6 +257,20 @@ def ro_assemble_list(ctx, xid, d_arena, arena_bytes, d_parents, n_parents, d_n_p
                                  _ptr(d_elem_state), _ptr(d_elem_off), _ptr(d_elem_len), elem_cap,
                                  _ptr(d_n_elems), C.byref(ne) if want_host else None)
     return (st, ob.value, ne.value) if want_host else (st, None, None)
+
+
+def ro_batch_ready_parent(ctx, xid, call, d_cand, n_cand, batch_size, flush, d_batched,
+                          batched_cap, d_batch_off=None, batch_off_cap=0, d_n_batched=None,
+                          d_n_batches=None, want_host: bool = True):
+    """Admission plus parent-bound reservation.  Returns (status, n_batched,
+    n_batches); the counts are None without want_host (no synchronisation)."""
+    nb, nbt = _u64(0), _u64(0)
+    st = load().ro_batch_ready_parent(ctx, xid, call, _ptr(d_cand), n_cand, batch_size, int(flush),
+                                      _ptr(d_batched), batched_cap, _ptr(d_batch_off), batch_off_cap,
+                                      _ptr(d_n_batched), _ptr(d_n_batches),
+                                      C.byref(nb) if want_host else None,
+                                      C.byref(nbt) if want_host else None)
+    return (st, nb.value, nbt.value) if want_host else (st, None, None)
 
 
 def ro_filter_reports(ctx, d_state, d_keep, n) -> int:

@@ -117,7 +117,18 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
       a.qstate[2] = 0;
       const unsigned long long K = ld_relaxed_u64(&ds->rb_kept);
       const unsigned long long L = tail - head, T = L + K;
-      const unsigned long long npop = a.flush ? T : (T / a.batch_size) * a.batch_size;
+      // parent-bound reservation takes nothing here: everything admitted is
+      // queued and the window [head, head + T) goes to launch_parent
+      const unsigned long long npop =
+          a.parent_bound ? 0ull : a.flush ? T : (T / a.batch_size) * a.batch_size;
+      if (a.parent_bound) {
+        ds->pb_Q = T;
+        ds->pb_head = head;
+        ds->pb_old_tail = tail;
+        ds->pb_stop = ~0ull;
+        ds->pb_bad = ld_relaxed_u64(&ds->rb_bad);
+        ds->pb_err = 0u;
+      }
       ds->rb_npop = npop;
       ds->rb_n_batches = (npop + a.batch_size - 1) / a.batch_size;
       if (a.n_batched_out) *a.n_batched_out = npop;
@@ -132,7 +143,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
         ds->rb_tail = tail;
         a.qstate[0] = head + npop;
         a.qstate[1] = tail + K;
-        ds->stats[5] += ld_relaxed_u64(&ds->rb_bad);
+        if (!a.parent_bound) ds->stats[5] += ld_relaxed_u64(&ds->rb_bad);
       }
       ds->rb_kept = 0;
       ds->rb_bad = 0;

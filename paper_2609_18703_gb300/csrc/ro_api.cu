@@ -27,6 +27,7 @@ const void* kernel_ptr_ready(int which);
 const void* kernel_ptr_commit(int which);
 const void* kernel_ptr_assemble(int which);
 const void* kernel_ptr_retry(int which);
+const void* kernel_ptr_parent(int which);
 }  // namespace ro
 
 using namespace ro;
@@ -144,6 +145,9 @@ struct ro_ctx {
   TsBuf ts[N_TS];
   DevBuf code;
   DevBuf x_mb, x_coff, x_mtfp, x_hdr;   // explicit-list assembly scratch
+  // parent-bound reservation scratch (see ParentArgs)
+  DevBuf pb_key[2], pb_val[2], pb_child, pb_hist, pb_dtot, pb_first, pb_endp, pb_rank, pb_spos,
+      pb_head, pb_csize, pb_coff, pb_rem;
   Ev fork, x_planned, join_plan, join_copy;
   Profiler prof;
   ro_status sticky = RO_OK;
@@ -433,6 +437,8 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 1);
   c->L.grid_acopy = grid_for(kernel_ptr_assemble(K_ACOPY), AC_THREADS, s, 8, asm_copy_smem());
   c->L.grid_retry = grid_for(kernel_ptr_retry(K_RT_SCATTER), RT_THREADS, s, 4);
+  c->L.grid_pb = grid_for(kernel_ptr_parent(K_PB_RANK), PB_THREADS, s, 8);
+  c->L.grid_pb_sort = grid_for(kernel_ptr_parent(K_PB_SORT), PB_THREADS, s, 8);
   c->Lp = c->L;
   c->Lc = c->L;
   cudaError_t e = cudaStreamSynchronize(c->stream);
@@ -471,6 +477,10 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
     free_buf(t.flag); free_buf(t.agg); free_buf(t.inc);
   }
   free_buf(c->code); free_buf(c->x_mb); free_buf(c->x_coff); free_buf(c->x_mtfp); free_buf(c->x_hdr);
+  for (DevBuf* b : {&c->pb_key[0], &c->pb_key[1], &c->pb_val[0], &c->pb_val[1], &c->pb_child,
+                    &c->pb_hist, &c->pb_dtot, &c->pb_first, &c->pb_endp, &c->pb_rank, &c->pb_spos,
+                    &c->pb_head, &c->pb_csize, &c->pb_coff, &c->pb_rem})
+    free_buf(*b);
   free_ev(c->fork); free_ev(c->x_planned); free_ev(c->join_plan); free_ev(c->join_copy);
   for (cudaEvent_t e : c->prof.pool) cudaEventDestroy(e);
   cudaFree(c->ds);
@@ -701,6 +711,104 @@ ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* 
     ro_status st = sync_and_check(c);
     if (h_n_batched) *h_n_batched = c->hs->rb_npop;
     if (h_n_batches) *h_n_batches = c->hs->rb_n_batches;
+    return st;
+  }
+  return RO_OK;
+}
+
+// ---------------------------------------------------------------------------
+ro_status ro_batch_ready_parent(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* d_cand,
+                                uint64_t n_cand, uint32_t batch_size, int32_t flush,
+                                uint32_t* d_batched, uint64_t batched_cap, uint64_t* d_batch_off,
+                                uint64_t batch_off_cap, uint64_t* d_n_batched,
+                                uint64_t* d_n_batches, uint64_t* h_n_batched,
+                                uint64_t* h_n_batches) {
+  RO_TRY(enter(c));
+  Expansion* x = get_exp(c, xid);
+  const char* fn = "ro_batch_ready_parent";
+  if (!x) return fail(c, RO_E_STATE, "%s: unknown expansion %d", fn, xid);
+  if (call >= c->n_calls) return fail(c, RO_E_INVAL, "%s: call %u out of range", fn, call);
+  if (batch_size == 0) return fail(c, RO_E_INVAL, "%s: batch_size is 0", fn);
+  if (batched_cap && !d_batched) return fail(c, RO_E_INVAL, "%s: NULL d_batched", fn);
+  if (d_cand && n_cand > MAX_CAND)
+    return fail(c, RO_E_INVAL, "%s: more than 2^30-2 candidates in one call", fn);
+  DeviceGuard g(c->device);
+  ExpSlot& S = c->slots[xid];
+  QueueBufs& Q = S.queues[call];
+  RO_TRY(queue_ready(c, Q, x->N));
+  const uint64_t N = x->N, P = x->P, tiles = std::max<uint64_t>(1, ceil_div(N, (uint64_t)PB_TILE));
+  const size_t n4 = std::max<uint64_t>(N, 1) * sizeof(uint32_t);
+  for (DevBuf* b : {&c->pb_key[0], &c->pb_key[1], &c->pb_val[0], &c->pb_val[1], &c->pb_child,
+                    &c->pb_rank, &c->pb_spos, &c->pb_head, &c->pb_csize, &c->pb_coff, &c->pb_rem})
+    RO_TRY(ensure(c, *b, n4, "parent-bound scratch"));
+  RO_TRY(ensure(c, c->pb_hist, PB_DIGITS * tiles * sizeof(uint32_t), "parent-bound histogram"));
+  RO_TRY(ensure(c, c->pb_dtot, PB_DIGITS * sizeof(uint32_t), "parent-bound digit totals"));
+  RO_TRY(ensure(c, c->pb_first, std::max<uint64_t>(P, 1) * sizeof(uint32_t), "parent-bound ranges"));
+  RO_TRY(ensure(c, c->pb_endp, std::max<uint64_t>(P, 1) * sizeof(uint32_t), "parent-bound ranges"));
+
+  ReadyArgs ra{};
+  ra.cand = d_cand;
+  ra.n_cand = d_cand ? n_cand : N;
+  ra.N = N;
+  ra.phase = (uint32_t*)S.phase.p;
+  ra.rec = (const Rec*)S.rec.p;
+  ra.check_call = c->n_calls > 1;
+  ra.call = call;
+  ra.batch_size = batch_size;
+  ra.flush = flush != 0;
+  ra.cap = batched_cap;
+  ra.queue = (uint32_t*)Q.q.p;
+  ra.qstate = (unsigned long long*)Q.state.p;
+  ra.rq = (const uint32_t*)Q.rq.p;
+  ra.batched = d_batched;
+  ra.n_batched_out = nullptr;
+  ra.parent_bound = 1;
+  ra.ds = c->ds;
+  RO_TRY(tile_status(c, TS_READY, ceil_div(ra.n_cand, (uint64_t)RB_THREADS * RB_ITEMS), &ra.ts));
+
+  ParentArgs pa{};
+  pa.N = N;
+  pa.P = P;
+  pa.B = batch_size;
+  pa.flush = flush != 0;
+  int bits = 0;
+  while (bits < 32 && P > 1 && ((P - 1) >> bits) != 0) ++bits;
+  pa.passes = (bits + 7) / 8;
+  pa.rec = (const Rec*)S.rec.p;
+  pa.phase = (uint32_t*)S.phase.p;
+  pa.queue = (uint32_t*)Q.q.p;
+  pa.qstate = (unsigned long long*)Q.state.p;
+  pa.batched = d_batched;
+  pa.cap = batched_cap;
+  pa.batch_off = d_batch_off;
+  pa.off_cap = batch_off_cap;
+  pa.n_batched_out = d_n_batched;
+  pa.n_batches_out = d_n_batches;
+  for (int k = 0; k < 2; ++k) {
+    pa.key[k] = (uint32_t*)c->pb_key[k].p;
+    pa.val[k] = (uint32_t*)c->pb_val[k].p;
+  }
+  pa.child = (uint32_t*)c->pb_child.p;
+  pa.hist = (uint32_t*)c->pb_hist.p;
+  pa.dtot = (uint32_t*)c->pb_dtot.p;
+  pa.first = (uint32_t*)c->pb_first.p;
+  pa.endp = (uint32_t*)c->pb_endp.p;
+  pa.rank = (uint32_t*)c->pb_rank.p;
+  pa.spos = (uint32_t*)c->pb_spos.p;
+  pa.head = (uint32_t*)c->pb_head.p;
+  pa.csize = (uint32_t*)c->pb_csize.p;
+  pa.coff = (uint32_t*)c->pb_coff.p;
+  pa.rem = (uint32_t*)c->pb_rem.p;
+  pa.ds = c->ds;
+  RO_TRY(tile_status(c, TS_PARENT, tiles, &pa.ts));
+
+  launch_ready(c->L, ra);
+  launch_parent(c->L, pa);
+  RO_TRY(check_launch(c, "batch_ready_parent"));
+  if (h_n_batched || h_n_batches) {
+    ro_status st = sync_and_check(c);
+    if (h_n_batched) *h_n_batched = c->hs->pb_npop;
+    if (h_n_batches) *h_n_batches = c->hs->pb_nb;
     return st;
   }
   return RO_OK;

@@ -107,6 +107,10 @@ struct DevScalars {
   unsigned long long cm_n, cm_conflicts, cm_n_done, cm_gf;
   // ro_retry
   unsigned long long rt_done;
+  // ro_batch_ready_parent: the queue window after admission, the first short
+  // chunk (no flush), totals, the admission's bad candidates, refusal
+  unsigned long long pb_Q, pb_head, pb_old_tail, pb_stop, pb_npop, pb_nb, pb_R, pb_bad;
+  uint32_t pb_err, pb_pad;
   uint32_t cm_fix_ticket, cm_fix_done;
   // ro_assemble
   unsigned long long as_bytes;    // bytes of the latest assemble (host read-back)
@@ -117,7 +121,7 @@ struct DevScalars {
   unsigned long long epoch[8];
 };
 enum TileSlot { TS_EXPAND = 0, TS_READY = 1, TS_COMMIT = 2, TS_ASM_PARENTS = 3, TS_ASM_MEMBERS = 4,
-                TS_RETRY = 6 };   // 5: asm_copy's exit ticket
+                TS_RETRY = 6, TS_PARENT = 7 };   // 5: asm_copy's exit ticket
 
 // Wait until the grid this launch depends on (programmatic dependent launch)
 // has completed and its memory is visible; a no-op without a dependency.

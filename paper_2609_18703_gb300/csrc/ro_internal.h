@@ -31,7 +31,8 @@ constexpr uint32_t AC_BUF = 16384 + 32 * AC_PIECES;           // staged source b
 
 // kernel entry points for occupancy queries and per-kernel timing
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CFINISH, K_APARENTS,
-                K_AMEMBERS, K_ACOPY, K_RT_CLAIM, K_RT_SCATTER, K_COUNT };
+                K_AMEMBERS, K_ACOPY, K_RT_CLAIM, K_RT_SCATTER, K_PB_KEYS, K_PB_HIST,
+                K_PB_ROWSCAN, K_PB_SORT, K_PB_BOUNDS, K_PB_RANK, K_PB_SCAN, K_PB_EMIT, K_COUNT };
 
 // Launch counter and optional CUDA-event timing of selected kernels, on the
 // stream they are launched on (see ro_ctx_profile in the C ABI).
@@ -43,7 +44,7 @@ struct LaunchCfg {
   cudaStream_t stream;
   Profiler* prof;
   int grid_expand_scan, grid_fill, grid_rb, grid_commit, grid_cfinish, grid_aparents,
-      grid_amembers, grid_acopy, grid_retry;
+      grid_amembers, grid_acopy, grid_retry, grid_pb, grid_pb_sort;
 };
 
 // Launch one kernel between the profiler's marks, with programmatic
@@ -111,10 +112,49 @@ struct ReadyArgs {
   const uint32_t* rq;         // this (expansion, Call) recovery queue storage
   uint32_t* batched;
   uint64_t* n_batched_out;    // optional device output
+  int parent_bound;           // admit only: the window is reserved by launch_parent
   DevScalars* ds;
   TileStatus<unsigned long long> ts;
 };
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a);
+// ---- ro_batch_ready_parent ---------------------------------------------------------
+constexpr int PB_THREADS = 256, PB_ITEMS = 8;                 // queue entries per tile: 2048
+constexpr uint32_t PB_TILE = PB_THREADS * PB_ITEMS;
+constexpr int PB_DIGITS = 256;                                // radix of the sort by parent
+struct ParentArgs {
+  uint64_t N, P;
+  uint32_t B;
+  int flush;
+  int passes;                 // 8-bit digit passes covering the largest parent id
+  int pass;                   // the sort pass of this launch
+  const Rec* rec;
+  uint32_t* phase;
+  uint32_t* queue;
+  unsigned long long* qstate;
+  uint32_t* batched;
+  uint64_t cap;
+  uint64_t* batch_off;        // optional
+  uint64_t off_cap;
+  uint64_t* n_batched_out;    // optional
+  uint64_t* n_batches_out;    // optional
+  // scratch; per window entry (at most N of them) unless noted
+  uint32_t* key[2];           // parent of the entry, sorted by passes
+  uint32_t* val[2];           // window position of the entry, permuted alike
+  uint32_t* child;            // the window's children
+  uint32_t* hist;             // PB_DIGITS x tiles, digit-major
+  uint32_t* dtot;             // PB_DIGITS digit totals
+  uint32_t* first;            // per parent: sorted position of its first entry
+  uint32_t* endp;             // per parent: one past its last
+  uint32_t* rank;             // rank among the parent's entries (queue order)
+  uint32_t* spos;             // sorted position
+  uint32_t* head;             // window position of the chunk's first entry
+  uint32_t* csize;            // chunk size (chunk heads only)
+  uint32_t* coff;             // per sorted position of a chunk head: output offset
+  uint32_t* rem;              // entries left in the queue, in order
+  DevScalars* ds;
+  TileStatus<Pair64> ts;
+};
+void launch_parent(const LaunchCfg& L, const ParentArgs& a);
 
 // ---- ro_retry ----------------------------------------------------------------------
 constexpr int RT_THREADS = 256, RT_ITEMS = 8;                 // retry entries per tile: 2048

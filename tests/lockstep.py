@@ -113,6 +113,34 @@ class Lockstep:
             assert np.array_equal(got, r["batched"])
         return dict(status=st, batched=r["batched"], n_batched=nb)
 
+    def batch_ready_parent(self, xid: int, call: int = 0, cand=None, batch_size: int = 1,
+                           flush: bool = False, cap: Optional[int] = None,
+                           off_cap: Optional[int] = None) -> dict:
+        cand_np = None if cand is None else np.asarray(cand, dtype=np.uint32)
+        n_cand = self.N[xid] if cand_np is None else cand_np.size
+        if cap is None:
+            cap = self.N[xid]
+        if off_cap is None:
+            off_cap = cap + 1
+        r = self.o.batch_ready_parent(xid, call, cand_np, batch_size, flush, cap=cap,
+                                      off_cap=off_cap, check=False)
+        d_cand = None if cand_np is None else dev(cand_np, np.uint32)
+        d_b = empty(cap, np.uint32)
+        d_off = empty(off_cap, np.uint64)
+        d_nb = empty(1, np.uint64)
+        d_nbt = empty(1, np.uint64)
+        st, nb, nbt = ro.ro_batch_ready_parent(self.ctx, xid, call, d_cand,
+                                               0 if cand_np is None else n_cand, batch_size, flush,
+                                               d_b, cap, d_off, off_cap, d_nb, d_nbt)
+        assert st == r["status"], (st, r["status"], ro.ro_last_error(self.ctx))
+        assert nb == r["n_batched"] and nbt == r["n_batches"], (nb, nbt, r["n_batched"], r["n_batches"])
+        if st == ro.RO_OK:
+            assert int(host(d_nb, np.uint64, 1)[0]) == nb
+            assert int(host(d_nbt, np.uint64, 1)[0]) == nbt
+            assert np.array_equal(host(d_b, np.uint32, nb), r["batched"])
+            assert np.array_equal(host(d_off, np.uint64, nbt + 1), r["batch_off"])
+        return r
+
     # ------------------------------------------------------------- retry
     def retry(self, xid: int, call: int, children) -> dict:
         ch = np.asarray(children, np.uint32)

@@ -46,6 +46,15 @@ MUTANTS = {
     "list_base_off_by_one": ("  elem_base[n] = e;", "  elem_base[n] = e + 1;"),
     "filter_drops_failed": ("if (state[r] == OR_PRESENT && !keep[r]) state[r] = OR_DROPPED;",
                             "if (!keep[r]) state[r] = OR_DROPPED;"),
+    # parent-bound reservation (Section 4.3)
+    "pb_takes_short_head": ("if (k < batch_size && !flush) break;", "if (0) break;"),
+    "pb_mixes_parents": ("while (e >= 0 && k < batch_size) { pick[k++] = e; e = sib[e]; }",
+                         "while (e >= 0 && k < batch_size) { pick[k++] = e; e = next[e]; }"),
+    "pb_left_reordered": ("for (int64_t t = front; t >= 0; t = next[t]) out[r++] = q[h + t];",
+                          "for (int64_t t = front; t >= 0; t = next[t]) out[r++] = q[h + (t ^ 1) % (int64_t)n];"),
+    "pb_batch_off_shift": ("    bo[nb++] = take;\n", "    bo[nb++] = take + (nb > 0);\n"),
+    "pb_head_from_tail": ("uint32_t p = x->child_parent[q[h + front]];",
+                          "uint32_t p = x->child_parent[q[x->qtail[call] - 1]];"),
     "barrier_completion_missed": ("if (sealed_now && x->terminal[p] == member_count(x, p)) x->last_done[k++] = p;",
                                   "(void)sealed_now;"),
 }
@@ -66,6 +75,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
                         os.path.join(ROOT, "tests", "test_oracle.py"),
                         os.path.join(ROOT, "tests", "test_oracle_group_failure.py"),
                         os.path.join(ROOT, "tests", "test_oracle_retry.py"),
-                        os.path.join(ROOT, "tests", "test_oracle_lists.py")],
+                        os.path.join(ROOT, "tests", "test_oracle_lists.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_parent_bound.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode != 0, f"pins did not catch mutant {name}:\n{r.stdout[-2000:]}"
