@@ -64,6 +64,8 @@ def parse():
                     help="assemble with ro_assemble_list (per-member list entries, Section 4.2)")
     ap.add_argument("--filter-drop", type=float, default=0.0,
                     help="F.filter each wave's reports first; fraction the predicate rejects")
+    ap.add_argument("--parent-bound", action="store_true",
+                    help="reserve with ro_batch_ready_parent (Section 4.3), pages admitted in arrival order")
     ap.add_argument("--one-stream", action="store_true",
                     help="plan and copy on the context's stream (no overlap across waves)")
     ap.add_argument("--no-e2e", action="store_true")
@@ -203,7 +205,7 @@ def run_reference(args, rank):
 class Pass:
     """Device-resident inputs and outputs of one document->page microbatch."""
 
-    def __init__(self, lv, device, stream, lists=False, filter_drop=0.0):
+    def __init__(self, lv, device, stream, lists=False, filter_drop=0.0, parent_bound=False):
         import torch
         from workload.device import fill_payload
         self.torch = torch
@@ -241,6 +243,10 @@ class Pass:
         self.cursor = torch.zeros(1, dtype=torch.int64, device=dev)
         self.out_bytes = torch.zeros(self.W, dtype=torch.int64, device=dev)
         self.lists = lists
+        self.parent_bound = parent_bound
+        if parent_bound:
+            self.batch_off = torch.empty(self.N + 1, dtype=torch.int64, device=dev)
+            self.n_batches = torch.zeros(1, dtype=torch.int64, device=dev)
         if lists:
             # wave w's list entries and entry ranges go to windows of their own,
             # sized by the parents whose last report arrives in that wave
@@ -276,8 +282,15 @@ class Pass:
     def waves(self, ro, ctx, xid):
         """batch_ready + every wave's commit and assemble; asynchronous."""
         L = ro.load()
-        st = L.ro_batch_ready(ctx, xid, 0, None, 0, self.B, 1, self.batched.data_ptr(),
-                              self.N + self.B, self.n_batched.data_ptr(), None, None)
+        if self.parent_bound:   # batches of siblings, pages admitted in arrival order
+            st = L.ro_batch_ready_parent(ctx, xid, 0, self.child.data_ptr(), self.N, self.B, 1,
+                                         self.batched.data_ptr(), self.N + self.B,
+                                         self.batch_off.data_ptr(), self.N + 1,
+                                         self.n_batched.data_ptr(), self.n_batches.data_ptr(),
+                                         None, None)
+        else:
+            st = L.ro_batch_ready(ctx, xid, 0, None, 0, self.B, 1, self.batched.data_ptr(),
+                                  self.N + self.B, self.n_batched.data_ptr(), None, None)
         bad = st
         self.cursor.zero_()
         cb, sb, lb, ob = (self.child.data_ptr(), self.state.data_ptr(), self.length.data_ptr(),
@@ -320,7 +333,8 @@ def run_ours(args, rank, world, local_rank):
     lv = docpage(parents=args.parents, waves=args.waves, salt=rank).top
     stream = torch.cuda.Stream()
     torch.cuda.set_stream(stream)
-    ps = Pass(lv, local_rank, stream, lists=args.lists, filter_drop=args.filter_drop)
+    ps = Pass(lv, local_rank, stream, lists=args.lists, filter_drop=args.filter_drop,
+              parent_bound=args.parent_bound)
     ctx = ro.ro_ctx_create(local_rank, stream, 1)
     if not args.one_stream:   # assembly planning and copies overlap later waves' commits
         plan_stream, copy_stream = torch.cuda.Stream(), torch.cuda.Stream()
@@ -392,7 +406,13 @@ def run_ours(args, rank, world, local_rank):
     value = world * ps.N / (ms_step * 1e-3)
 
     # ---- per-kernel timing of the copy kernel (events on its launch stream)
-    ro.ro_ctx_profile(ctx, 1 << K_ACOPY)
+    # and, with --parent-bound, of the reservation's kernels
+    res_kernels = ("ready_count", "ready_scatter") + tuple(k for k in ro.KERNELS if k.startswith("pb_"))
+    mask = 1 << K_ACOPY
+    if ps.parent_bound:
+        for k in res_kernels:
+            mask |= 1 << ro.KERNELS.index(k)
+    ro.ro_ctx_profile(ctx, mask)
     kt_steps = max(2, min(args.steps, 5))
     for _ in range(kt_steps):
         step_eager()
@@ -409,6 +429,20 @@ def run_ours(args, rank, world, local_rank):
     if ps.keep is not None:   # F.filter reads state and predicate, writes state
         pass_alg += 3.0 * ps.N
     kernel_ms = {k: round(v[2] / kt_steps, 4) for k, v in prof.items() if v[1]}
+    reservation = None
+    if ps.parent_bound:
+        nbt = int(ps.n_batches.item())
+        res_ms = sum(prof[k][2] for k in res_kernels) / kt_steps
+        # admission: candidate, phase read + write, queue entry; reservation:
+        # queue entry, parent, phase read + write, batched entry; boundaries
+        res_bytes = 40.0 * ps.N + 8.0 * (nbt + 1)
+        pass_alg += 4.0 * ps.N + 8.0 * (nbt + 1)   # candidates in arrival order, boundaries
+        res_gbs = res_bytes / (res_ms * 1e-3) / 1e9 if res_ms > 0 else 0.0
+        reservation = {"policy": "parent-bound", "batch": ps.B, "entries": ps.N, "batches": nbt,
+                       "ms": round(res_ms, 4), "entries_per_s": round(ps.N / (res_ms * 1e-3), 1),
+                       "algorithmic_bytes": res_bytes, "achieved_gbs": round(res_gbs, 1),
+                       "frac_of_hbm": round(res_gbs / hbm_peak, 4),
+                       "kernel_ms": {k: round(prof[k][2] / kt_steps, 4) for k in res_kernels}}
 
     # ---- end to end through the C ABI with host buffers
     e2e = None
@@ -434,6 +468,7 @@ def run_ours(args, rank, world, local_rank):
                                    f"{args.waves} arrival waves, batch {ps.B}",
                        "parents": ps.P, "children": ps.N, "waves": args.waves,
                        "arena_bytes": ps.arena_bytes, "assembled_bytes": S,
+                       "reservation": "parent-bound" if ps.parent_bound else "elastic",
                        "output": "list entries per member" if ps.lists else "bytes",
                        "list_entries": n_entries if ps.lists else None,
                        "filter_drop": args.filter_drop,
@@ -453,6 +488,7 @@ def run_ours(args, rank, world, local_rank):
                                            "scaled by bytes assembled per launch",
                          "launches": n_copy, "avg_launch_ms": round(copy_ms / max(n_copy, 1), 5)},
             "kernel_ms_per_step": kernel_ms,
+            "parent_bound_reservation": reservation,
             "gpu_launches": int(launches_timed),
             "clocks": clk,
             "e2e": e2e,

@@ -16,11 +16,12 @@
 //                contributing member's relative position and arena offset, and
 //                for every 16 KB chunk of the output the member holding its
 //                first byte;
-//   asm_copy     per chunk: one warp stages the chunk's member pieces in
-//                shared memory with cp.async.bulk (two stages, mbarrier
-//                completion, bounded waits) while all warps turn the previous
-//                chunk into aligned 16-byte stores; source and destination
-//                alignments may differ arbitrarily.
+//   asm_copy     per chunk: two producer warps stage chunks' member pieces
+//                in shared memory with cp.async.bulk (a ring of AC_STAGES
+//                stages, mbarrier completion, bounded waits) while six
+//                consumer warps turn staged chunks into aligned 16-byte
+//                stores; source and destination alignments may differ
+//                arbitrarily.
 // The plan is independent of where the output starts, so planning (on the
 // context's plan stream) can run ahead of the copies (copy stream).
 #include <algorithm>
@@ -823,7 +824,10 @@ __device__ void emit_direct(const CopyCtx& c, const CopyStage* st, uint32_t cw, 
 // into a ring of AC_STAGES stages (producer p takes the CTA's chunks i with
 // i % AC_PRODUCERS == p), the other warps write them out in order; full
 // and empty mbarriers per stage hand the stages back and forth.
-__global__ void __launch_bounds__(AC_THREADS, 2) asm_copy_kernel(AssembleArgs a) {
+// Sized to leave room beside it: two CTAs per SM take 2 x 256 threads x 80
+// registers and 2 x 3 stages of shared memory, so the commit kernels of later
+// waves (other streams) can be resident on the same SMs while a copy runs.
+__global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a) {
   wait_predecessor();
   extern __shared__ __align__(128) unsigned char ac_smem[];
   __shared__ __align__(8) uint64_t full_bar[AC_STAGES];
@@ -960,7 +964,7 @@ void launch_assemble_copy(const LaunchCfg& L, const AssembleArgs& a) {
   launch_k(L, K_ACOPY, asm_copy_kernel, L.grid_acopy, AC_THREADS, asm_copy_smem(), a);
 }
 
-// opt in to the copy kernel's dynamic shared memory (two pipeline stages)
+// opt in to the copy kernel's dynamic shared memory (AC_STAGES pipeline stages)
 cudaError_t prepare_assemble_kernels() {
   return cudaFuncSetAttribute(asm_copy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)asm_copy_smem());

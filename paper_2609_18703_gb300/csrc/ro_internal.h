@@ -23,7 +23,7 @@ constexpr uint32_t AM_TILE = AM_THREADS * AM_ITEMS;
 constexpr uint32_t AM_SMEM_CAP = 4096;                        // listed parents staged per tile
 constexpr int AC_THREADS = 256;                               // 2 producer + 6 consumer warps
 constexpr int AC_PRODUCERS = 2, AC_CONSUMERS = AC_THREADS / 32 - AC_PRODUCERS;
-constexpr int AC_STAGES = 4;                                  // chunks staged per CTA
+constexpr int AC_STAGES = 3;                                  // chunks staged per CTA
 constexpr uint64_t AC_CHUNK = 16384;                          // output bytes per copy chunk (relative)
 constexpr uint32_t AC_PIECES = 256;                           // member pieces staged per chunk
 constexpr uint32_t AC_BUF = 16384 + 32 * AC_PIECES;           // staged source bytes per chunk (fits any
