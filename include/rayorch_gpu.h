@@ -152,7 +152,7 @@ enum {
   RO_K_COMMIT_SCATTER = 4, RO_K_COMMIT_FINISH = 5, RO_K_ASM_PARENTS = 6, RO_K_ASM_MEMBERS = 7,
   RO_K_ASM_COPY = 8, RO_K_RETRY_CLAIM = 9, RO_K_RETRY_SCATTER = 10, RO_K_PB_KEYS = 11,
   RO_K_PB_HIST = 12, RO_K_PB_ROWSCAN = 13, RO_K_PB_SORT = 14, RO_K_PB_BOUNDS = 15,
-  RO_K_PB_RANK = 16, RO_K_PB_SCAN = 17, RO_K_PB_EMIT = 18, RO_K_COUNT = 19
+  RO_K_PB_HEADS = 16, RO_K_PB_MARK = 17, RO_K_PB_SCAN = 18, RO_K_PB_EMIT = 19, RO_K_COUNT = 20
 };
 /* Tracing (no counterpart in the paper; it instruments the path).  Every
  * kernel launch is counted; kernels whose bit (1 << RO_K_*) is set in
@@ -246,7 +246,7 @@ ro_status ro_batch_ready(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t
  * Errors: RO_E_CAPACITY when more would be reserved than batched_cap, or
  * d_batch_off cannot hold n_batches + 1 entries (reported when the context
  * next synchronises; the admission is undone, the outputs are undefined).
- * Device scratch of about 44 bytes per child and 8 per parent of the
+ * Device scratch of about 37 bytes per child and 8 per parent of the
  * expansion is allocated at the first call (like ro_batch_ready, this call
  * cannot be the first to size it inside a stream capture).
  */

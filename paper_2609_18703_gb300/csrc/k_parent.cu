@@ -9,16 +9,23 @@
 // first entry (without flush, up to the first chunk shorter than B).  The
 // ranks come from a stable sort of the window by parent id.
 //
-//   pb_keys     window copy: child, parent (sort key), position (sort value)
+//   pb_keys     window copy: child, parent (sort key), position (sort value);
+//               clears the per-position chunk sizes and marks
 //   pb_hist     per tile digit counts of one 8-bit digit of the key
 //   pb_rowscan  per digit, exclusive scan over tiles; digit totals
 //   pb_sort     stable scatter of one digit pass (warp match + per-warp counts)
 //   pb_bounds   per parent, sorted range of its entries
-//   pb_rank     per entry: rank, chunk head, chunk size; first short chunk
+//   pb_heads    sorted order: each chunk's first entry records the chunk size
+//               at its queue position; the first short chunk (no flush)
+//   pb_mark     sorted order, no flush only: marks entries of chunks at or
+//               after the first short chunk, which stay queued
 //   pb_scan     queue order, single-pass scan (decoupled look-back): output
 //               offset of each taken chunk, batch boundaries, entries left
-//   pb_emit     writes the batches (IN-FLIGHT) and the queue's remainder, or
-//               on a refusal (capacity) undoes the admission
+//   pb_emit     sorted order: writes each taken chunk's entries contiguously
+//               (IN-FLIGHT) and the queue's remainder, or on a refusal
+//               (capacity) undoes the admission
+// Only chunk heads (about one entry in B) and marked entries are written by
+// queue position; everything else moves in sorted order.
 // The admission itself (ready_count / ready_scatter with parent_bound set)
 // runs first and queues every admitted Grain.
 #include <algorithm>
@@ -29,14 +36,29 @@ namespace ro {
 
 __global__ void __launch_bounds__(PB_THREADS) pb_keys_kernel(ParentArgs a) {
   wait_predecessor();
+  constexpr int U = 4;   // entries per thread per step: their loads first
   const DevScalars* ds = a.ds;
   const uint64_t Q = ds->pb_Q, head = ds->pb_head;
   const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
-  for (uint64_t j = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; j < Q; j += stride) {
-    const uint32_t c = a.queue[head + j];
-    a.child[j] = c;
-    a.key[0][j] = a.rec[c].parent;
-    a.val[0][j] = (uint32_t)j;
+  for (uint64_t j0 = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; j0 < Q; j0 += U * stride) {
+    uint32_t c[U], p[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint64_t j = j0 + u * stride;
+      c[u] = j < Q ? a.queue[head + j] : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) p[u] = j0 + u * stride < Q ? a.rec[c[u]].parent : 0u;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint64_t j = j0 + u * stride;
+      if (j >= Q) break;
+      a.child[j] = c[u];
+      a.key[0][j] = p[u];
+      a.val[0][j] = (uint32_t)j;
+      a.hsz[j] = 0u;
+      a.left[j] = 0u;
+    }
   }
 }
 
@@ -162,7 +184,9 @@ __global__ void __launch_bounds__(PB_THREADS) pb_bounds_kernel(ParentArgs a) {
   }
 }
 
-__global__ void __launch_bounds__(PB_THREADS) pb_rank_kernel(ParentArgs a) {
+// Sorted order: the first entry of each chunk (rank a multiple of B among
+// its parent's entries) records the chunk's size at its queue position.
+__global__ void __launch_bounds__(PB_THREADS) pb_heads_kernel(ParentArgs a) {
   wait_predecessor();
   DevScalars* ds = a.ds;
   const uint64_t Q = ds->pb_Q;
@@ -171,19 +195,33 @@ __global__ void __launch_bounds__(PB_THREADS) pb_rank_kernel(ParentArgs a) {
   const uint32_t B = a.B;
   const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
   for (uint64_t s = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; s < Q; s += stride) {
-    const uint32_t p = key[s], i = val[s];
-    const uint32_t f = a.first[p];
-    const uint32_t r = (uint32_t)s - f, cnt = a.endp[p] - f;
-    const uint32_t k0 = r - r % B;              // rank of the chunk's first entry
-    const uint32_t hw = val[f + k0];            // its queue position
-    a.rank[i] = r;
-    a.spos[i] = (uint32_t)s;
-    a.head[i] = hw;
-    if (r == k0) {
-      const uint32_t sz = min(B, cnt - k0);
-      a.csize[i] = sz;
-      if (!a.flush && sz < B) atomicMin(&ds->pb_stop, (unsigned long long)i);
-    }
+    const uint32_t p = key[s];
+    const uint32_t r = (uint32_t)s - a.first[p];
+    if (r % B != 0u) continue;
+    const uint32_t i = val[s];
+    const uint32_t sz = min(B, a.endp[p] - (uint32_t)s);
+    a.hsz[i] = sz;
+    if (!a.flush && sz < B) atomicMin(&ds->pb_stop, (unsigned long long)i);
+  }
+}
+
+// Sorted order, only when a short chunk stops the reservations: entries of
+// chunks whose first entry is at or after the stop stay queued.
+__global__ void __launch_bounds__(PB_THREADS) pb_mark_kernel(ParentArgs a) {
+  wait_predecessor();
+  const DevScalars* ds = a.ds;
+  const unsigned long long stop = ds->pb_stop;
+  if (stop == ~0ull) return;
+  const uint64_t Q = ds->pb_Q;
+  const uint32_t* key = a.key[a.passes & 1];
+  const uint32_t* val = a.val[a.passes & 1];
+  const uint32_t B = a.B;
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t s = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; s < Q; s += stride) {
+    const uint32_t f = a.first[key[s]];
+    const uint32_t r = (uint32_t)s - f;
+    const uint32_t hw = val[f + (r - r % B)];   // queue position of the chunk's first entry
+    if (hw >= stop) a.left[val[s]] = 1u;
   }
 }
 
@@ -222,18 +260,19 @@ __global__ void __launch_bounds__(PB_THREADS) pb_scan_kernel(ParentArgs a) {
     const uint64_t i0 = (uint64_t)tile * PB_TILE + (uint64_t)threadIdx.x * PB_ITEMS;
     // a: entries of the taken chunks; b: taken chunks << 32 | entries left
     Pair64 mine{0, 0};
-    uint32_t take_head = 0, left = 0;
+    uint32_t take_head = 0, left = 0, sz[PB_ITEMS];
 #pragma unroll
     for (int k = 0; k < PB_ITEMS; ++k) {
       const uint64_t i = i0 + k;
+      sz[k] = 0u;
       if (i >= Q) continue;
-      const bool taken = a.head[i] < stop;
-      if (!taken) {
+      sz[k] = a.hsz[i];
+      if (a.left[i]) {
         left |= 1u << k;
         mine.b += 1;
-      } else if (a.rank[i] % B == 0u) {
+      } else if (sz[k] != 0u && i < stop) {
         take_head |= 1u << k;
-        mine.a += a.csize[i];
+        mine.a += sz[k];
         mine.b += 1ull << 32;
       }
     }
@@ -249,10 +288,10 @@ __global__ void __launch_bounds__(PB_THREADS) pb_scan_kernel(ParentArgs a) {
     for (int k = 0; k < PB_ITEMS; ++k) {
       const uint64_t i = i0 + k;
       if (take_head & (1u << k)) {
-        a.coff[a.spos[i]] = (uint32_t)run.a;
+        a.hoff[i] = (uint32_t)run.a;
         const uint64_t b = run.b >> 32;
         if (a.batch_off && b < a.off_cap) a.batch_off[b] = run.a;
-        run.a += a.csize[i];
+        run.a += sz[k];
         run.b += 1ull << 32;
       } else if (left & (1u << k)) {
         a.rem[run.b & 0xFFFFFFFFull] = a.child[i];
@@ -291,13 +330,18 @@ __global__ void __launch_bounds__(PB_THREADS) pb_emit_kernel(ParentArgs a) {
     return;
   }
   const unsigned long long stop = ds->pb_stop, npop = ds->pb_npop, R = ds->pb_R;
+  const uint32_t* key = a.key[a.passes & 1];
+  const uint32_t* val = a.val[a.passes & 1];
   const uint32_t B = a.B;
-  for (uint64_t i = g; i < Q; i += stride) {
-    if (a.head[i] >= stop) continue;
-    const uint32_t r = a.rank[i] % B;
-    const uint32_t pos = a.coff[a.spos[i] - r] + r;
-    const uint32_t c = a.child[i];
-    a.batched[pos] = c;
+  // sorted order: a taken chunk's entries are consecutive here and in the
+  // output, so the writes to the batches are contiguous
+  for (uint64_t s = g; s < Q; s += stride) {
+    const uint32_t f = a.first[key[s]];
+    const uint32_t r = (uint32_t)s - f, k = r % B;
+    const uint32_t hw = val[f + (r - k)];   // queue position of the chunk's first entry
+    if (hw >= stop) continue;
+    const uint32_t c = a.child[val[s]];
+    a.batched[a.hoff[hw] + k] = c;
     a.phase[c] = (a.phase[c] & ~3u) | PH_INFLIGHT;
   }
   for (uint64_t j = g; j < R; j += stride) a.queue[head + npop + j] = a.rem[j];
@@ -321,7 +365,8 @@ void launch_parent(const LaunchCfg& L, const ParentArgs& a) {
     launch_k(L, K_PB_SORT, pb_sort_kernel, g_tile, PB_THREADS, 0, b);
   }
   launch_k(L, K_PB_BOUNDS, pb_bounds_kernel, g_elem, PB_THREADS, 0, a);
-  launch_k(L, K_PB_RANK, pb_rank_kernel, g_elem, PB_THREADS, 0, a);
+  launch_k(L, K_PB_HEADS, pb_heads_kernel, g_elem, PB_THREADS, 0, a);
+  if (!a.flush) launch_k(L, K_PB_MARK, pb_mark_kernel, g_elem, PB_THREADS, 0, a);
   launch_k(L, K_PB_SCAN, pb_scan_kernel, g_tile, PB_THREADS, 0, a);
   launch_k(L, K_PB_EMIT, pb_emit_kernel, g_elem, PB_THREADS, 0, a);
 }
@@ -330,7 +375,7 @@ const void* kernel_ptr_parent(int which) {
   switch (which) {
     case K_PB_SORT: return (const void*)pb_sort_kernel;
     case K_PB_SCAN: return (const void*)pb_scan_kernel;
-    default: return (const void*)pb_rank_kernel;
+    default: return (const void*)pb_heads_kernel;
   }
 }
 

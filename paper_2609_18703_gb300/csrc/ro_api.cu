@@ -146,8 +146,8 @@ struct ro_ctx {
   DevBuf code;
   DevBuf x_mb, x_coff, x_mtfp, x_hdr;   // explicit-list assembly scratch
   // parent-bound reservation scratch (see ParentArgs)
-  DevBuf pb_key[2], pb_val[2], pb_child, pb_hist, pb_dtot, pb_first, pb_endp, pb_rank, pb_spos,
-      pb_head, pb_csize, pb_coff, pb_rem;
+  DevBuf pb_key[2], pb_val[2], pb_child, pb_hist, pb_dtot, pb_first, pb_endp, pb_hsz, pb_left,
+      pb_hoff, pb_rem;
   Ev fork, x_planned, join_plan, join_copy;
   Profiler prof;
   ro_status sticky = RO_OK;
@@ -437,7 +437,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 1);
   c->L.grid_acopy = grid_for(kernel_ptr_assemble(K_ACOPY), AC_THREADS, s, 2, asm_copy_smem());
   c->L.grid_retry = grid_for(kernel_ptr_retry(K_RT_SCATTER), RT_THREADS, s, 4);
-  c->L.grid_pb = grid_for(kernel_ptr_parent(K_PB_RANK), PB_THREADS, s, 8);
+  c->L.grid_pb = grid_for(kernel_ptr_parent(K_PB_HEADS), PB_THREADS, s, 8);
   c->L.grid_pb_sort = grid_for(kernel_ptr_parent(K_PB_SORT), PB_THREADS, s, 8);
   c->Lp = c->L;
   c->Lc = c->L;
@@ -478,8 +478,8 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   }
   free_buf(c->code); free_buf(c->x_mb); free_buf(c->x_coff); free_buf(c->x_mtfp); free_buf(c->x_hdr);
   for (DevBuf* b : {&c->pb_key[0], &c->pb_key[1], &c->pb_val[0], &c->pb_val[1], &c->pb_child,
-                    &c->pb_hist, &c->pb_dtot, &c->pb_first, &c->pb_endp, &c->pb_rank, &c->pb_spos,
-                    &c->pb_head, &c->pb_csize, &c->pb_coff, &c->pb_rem})
+                    &c->pb_hist, &c->pb_dtot, &c->pb_first, &c->pb_endp, &c->pb_hsz, &c->pb_left,
+                    &c->pb_hoff, &c->pb_rem})
     free_buf(*b);
   free_ev(c->fork); free_ev(c->x_planned); free_ev(c->join_plan); free_ev(c->join_copy);
   for (cudaEvent_t e : c->prof.pool) cudaEventDestroy(e);
@@ -739,8 +739,9 @@ ro_status ro_batch_ready_parent(ro_ctx* c, int32_t xid, uint32_t call, const uin
   const uint64_t N = x->N, P = x->P, tiles = std::max<uint64_t>(1, ceil_div(N, (uint64_t)PB_TILE));
   const size_t n4 = std::max<uint64_t>(N, 1) * sizeof(uint32_t);
   for (DevBuf* b : {&c->pb_key[0], &c->pb_key[1], &c->pb_val[0], &c->pb_val[1], &c->pb_child,
-                    &c->pb_rank, &c->pb_spos, &c->pb_head, &c->pb_csize, &c->pb_coff, &c->pb_rem})
+                    &c->pb_hsz, &c->pb_hoff, &c->pb_rem})
     RO_TRY(ensure(c, *b, n4, "parent-bound scratch"));
+  RO_TRY(ensure(c, c->pb_left, std::max<uint64_t>(N, 1), "parent-bound scratch"));
   RO_TRY(ensure(c, c->pb_hist, PB_DIGITS * tiles * sizeof(uint32_t), "parent-bound histogram"));
   RO_TRY(ensure(c, c->pb_dtot, PB_DIGITS * sizeof(uint32_t), "parent-bound digit totals"));
   RO_TRY(ensure(c, c->pb_first, std::max<uint64_t>(P, 1) * sizeof(uint32_t), "parent-bound ranges"));
@@ -793,11 +794,9 @@ ro_status ro_batch_ready_parent(ro_ctx* c, int32_t xid, uint32_t call, const uin
   pa.dtot = (uint32_t*)c->pb_dtot.p;
   pa.first = (uint32_t*)c->pb_first.p;
   pa.endp = (uint32_t*)c->pb_endp.p;
-  pa.rank = (uint32_t*)c->pb_rank.p;
-  pa.spos = (uint32_t*)c->pb_spos.p;
-  pa.head = (uint32_t*)c->pb_head.p;
-  pa.csize = (uint32_t*)c->pb_csize.p;
-  pa.coff = (uint32_t*)c->pb_coff.p;
+  pa.hsz = (uint32_t*)c->pb_hsz.p;
+  pa.left = (uint8_t*)c->pb_left.p;
+  pa.hoff = (uint32_t*)c->pb_hoff.p;
   pa.rem = (uint32_t*)c->pb_rem.p;
   pa.ds = c->ds;
   RO_TRY(tile_status(c, TS_PARENT, tiles, &pa.ts));

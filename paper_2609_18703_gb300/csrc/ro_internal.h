@@ -32,7 +32,8 @@ constexpr uint32_t AC_BUF = 16384 + 32 * AC_PIECES;           // staged source b
 // kernel entry points for occupancy queries and per-kernel timing
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CFINISH, K_APARENTS,
                 K_AMEMBERS, K_ACOPY, K_RT_CLAIM, K_RT_SCATTER, K_PB_KEYS, K_PB_HIST,
-                K_PB_ROWSCAN, K_PB_SORT, K_PB_BOUNDS, K_PB_RANK, K_PB_SCAN, K_PB_EMIT, K_COUNT };
+                K_PB_ROWSCAN, K_PB_SORT, K_PB_BOUNDS, K_PB_HEADS, K_PB_MARK, K_PB_SCAN, K_PB_EMIT,
+                K_COUNT };
 
 // Launch counter and optional CUDA-event timing of selected kernels, on the
 // stream they are launched on (see ro_ctx_profile in the C ABI).
@@ -145,11 +146,9 @@ struct ParentArgs {
   uint32_t* dtot;             // PB_DIGITS digit totals
   uint32_t* first;            // per parent: sorted position of its first entry
   uint32_t* endp;             // per parent: one past its last
-  uint32_t* rank;             // rank among the parent's entries (queue order)
-  uint32_t* spos;             // sorted position
-  uint32_t* head;             // window position of the chunk's first entry
-  uint32_t* csize;            // chunk size (chunk heads only)
-  uint32_t* coff;             // per sorted position of a chunk head: output offset
+  uint32_t* hsz;              // by queue position: chunk size at a chunk's first entry, else 0
+  uint8_t* left;              // by queue position: 1 if the entry stays queued (no flush)
+  uint32_t* hoff;             // by queue position of a taken chunk's first entry: output offset
   uint32_t* rem;              // entries left in the queue, in order
   DevScalars* ds;
   TileStatus<Pair64> ts;
