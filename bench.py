@@ -70,6 +70,8 @@ def parse():
                     help="plan and copy on the context's stream (no overlap across waves)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--ref-parents", type=int, default=100_000,
+                    help="parents in each --impl reference step (bounded CPU sample)")
     ap.add_argument("--cpu-parents", type=int, default=1_000_000,
                     help="parents in the oracle's bounded CPU sample")
     return ap.parse_args()
@@ -164,37 +166,108 @@ def cpu_oracle_sample(parents: int, waves: int, min_seconds: float = 10.0, max_p
     arena = host_arena(lv)
     reports = [lv.reports(lv.wave(w)) for w in range(lv.n_waves)]
     passes, total, dt = 0, 0, 0.0
-    while passes < max_passes and (passes == 0 or dt < min_seconds):
+    # one core, as a single-threaded baseline; the affinity is restored after
+    prev = os.sched_getaffinity(0) if hasattr(os, "sched_getaffinity") else None
+    core = min(prev) if prev else None
+    if core is not None:
+        os.sched_setaffinity(0, {core})
+    try:
+        while passes < max_passes and (passes == 0 or dt < min_seconds):
+            o = OracleCtx()
+            t0 = time.perf_counter()
+            x = o.expand(lv.counts)["xid"]
+            o.batch_ready(x, 0, None, lv.batch_size, flush=True)
+            total = 0
+            for ch, st, ln, of in reports:
+                cm = o.gather_commit(x, ch, st, ln, of, arena_bytes=lv.arena_bytes)
+                a = o.assemble(x, arena, parents=None, n_parents=max(cm["n_done"], 1))
+                total += a["out_bytes"]
+            dt += time.perf_counter() - t0
+            o.close()
+            passes += 1
+    finally:
+        if prev:
+            os.sched_setaffinity(0, prev)
+    return passes * lv.n_children / dt, dt, lv.n_children, total, passes, core
+
+
+def host_cpu() -> dict:
+    """The host the CPU baseline ran on: model name and logical CPUs."""
+    model = None
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu model")):
+                model = line.split(":", 1)[1].strip()
+                break
+        if model is None:   # Arm hosts name the part elsewhere
+            out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+            for line in out.splitlines():
+                if line.startswith("Model name:"):
+                    model = line.split(":", 1)[1].strip()
+                    break
+    except Exception:
+        pass
+    return {"model": model, "nproc": os.cpu_count()}
+
+
+def run_reference(args, rank):
+    """The oracle as it stands, single-threaded on one host core: W untimed
+    and K timed steps, each one full pass (expand, batch_ready, every wave's
+    commit and assembly with its payload bytes) over a bounded sample of the
+    document->page workload (its first --ref-parents parents)."""
+    if rank != 0:
+        return
+    from oracle import OracleCtx
+    from tests.pipeline import host_arena
+    from workload import docpage
+    lv = docpage(parents=args.ref_parents, waves=args.waves, salt=1).top
+    arena = host_arena(lv)
+    reports = [lv.reports(lv.wave(w)) for w in range(lv.n_waves)]
+
+    def one_pass():
         o = OracleCtx()
-        t0 = time.perf_counter()
         x = o.expand(lv.counts)["xid"]
         o.batch_ready(x, 0, None, lv.batch_size, flush=True)
         total = 0
         for ch, st, ln, of in reports:
             cm = o.gather_commit(x, ch, st, ln, of, arena_bytes=lv.arena_bytes)
-            a = o.assemble(x, arena, parents=None, n_parents=max(cm["n_done"], 1))
-            total += a["out_bytes"]
-        dt += time.perf_counter() - t0
+            total += o.assemble(x, arena, parents=None, n_parents=max(cm["n_done"], 1))["out_bytes"]
         o.close()
-        passes += 1
-    return passes * lv.n_children / dt, dt, lv.n_children, total, passes
+        return total
 
-
-def run_reference(args, rank):
-    if rank != 0:
-        return
-    v, dt, n, _, passes = cpu_oracle_sample(args.cpu_parents, args.waves)
+    prev = os.sched_getaffinity(0) if hasattr(os, "sched_getaffinity") else None
+    core = min(prev) if prev else None
+    if core is not None:
+        os.sched_setaffinity(0, {core})
+    try:
+        for _ in range(args.warmup):
+            one_pass()
+        times = []
+        for _ in range(args.steps):
+            t0 = time.perf_counter()
+            S = one_pass()
+            times.append(time.perf_counter() - t0)
+    finally:
+        if prev:
+            os.sched_setaffinity(0, prev)
+    dt = sum(times)
+    v = args.steps * lv.n_children / dt
     line = {
         "impl": "reference", "metric": METRIC, "value": round(v, 1), "unit": "children/s",
-        "n_gpus": args.gpus, "steps": passes, "warmup": 0, "ms_per_step": round(dt / passes * 1e3, 3),
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(dt / args.steps * 1e3, 3),
+        "ms_per_step_median": round(sorted(times)[len(times) // 2] * 1e3, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8/u32/u64",
         "data": "synthetic",
-        "config": {"workload": f"document->page, {args.cpu_parents} of 1,000,000 parents "
-                               f"(bounded CPU sample), {args.waves} waves",
-                   "global_batch": n, "parallelism": "single-threaded oracle"},
+        "config": {"workload": f"document->page, first {args.ref_parents} of 1,000,000 parents "
+                               f"({lv.n_children} children, bounded CPU sample), {args.waves} waves, "
+                               f"batch {lv.batch_size}",
+                   "parents": args.ref_parents, "children": lv.n_children,
+                   "assembled_bytes": S, "parallelism": "single-threaded oracle, one core"},
         "cpu_baseline": {"value": round(v, 1), "unit": "children/s", "cores": 1, "kind": "oracle",
-                         "sample": f"{args.cpu_parents} parents / {n} children, full pass with "
-                                   f"payload bytes, {passes} passes in {dt:.1f} s"},
+                         "pinned_core": core, "host": host_cpu(),
+                         "sample": f"{args.ref_parents} parents / {lv.n_children} children per step, "
+                                   f"full pass with payload bytes, {args.steps} steps in {dt:.1f} s"},
         "e2e": {"value": round(v, 1), "unit": "children/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -383,11 +456,15 @@ def run_ours(args, rank, world, local_rank):
     clocks.start()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
+    marks = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
     t_start.record(stream)
-    for _ in range(args.steps):
+    marks[0].record(stream)
+    for k in range(args.steps):
         step()
+        marks[k + 1].record(stream)
     t_end.record(stream)
     torch.cuda.synchronize()
+    step_ms = sorted(marks[k].elapsed_time(marks[k + 1]) for k in range(args.steps))
     if dist:
         td.barrier()
     clk = clocks.stop()
@@ -451,8 +528,9 @@ def run_ours(args, rank, world, local_rank):
 
     cpu = None
     if rank == 0 and not args.no_cpu:
-        v_cpu, dt_cpu, n_cpu, _, p_cpu = cpu_oracle_sample(args.cpu_parents, args.waves)
+        v_cpu, dt_cpu, n_cpu, _, p_cpu, core = cpu_oracle_sample(args.cpu_parents, args.waves)
         cpu = {"value": round(v_cpu, 1), "unit": "children/s", "cores": 1, "kind": "oracle",
+               "pinned_core": core, "host": host_cpu(),
                "sample": f"document->page, first {args.cpu_parents} parents ({n_cpu} children) "
                          f"of the same distributions, {args.waves} waves, full pass with payload "
                          f"bytes, {p_cpu} passes in {dt_cpu:.1f} s"}
@@ -462,6 +540,8 @@ def run_ours(args, rank, world, local_rank):
         line = {
             "metric": METRIC, "value": round(value, 1), "unit": "children/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+            "ms_per_step_median": round(step_ms[len(step_ms) // 2], 4),
+            "ms_per_step_best": round(step_ms[0], 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "u8/u32/u64", "data": "synthetic",
             "config": {"workload": f"document->page: {ps.P} parents, {ps.N} children, "
@@ -480,6 +560,7 @@ def run_ours(args, rank, world, local_rank):
             "payload_frac_of_hbm": round(payload_gbs / hbm_peak, 4),
             "algorithmic_gbs": round(pass_alg / (ms_step * 1e-3) / 1e9, 1),
             "algorithmic_frac_of_hbm": round(pass_alg / (ms_step * 1e-3) / 1e9 / hbm_peak, 4),
+            "algorithmic_frac_of_nominal_8tbs": round(pass_alg / (ms_step * 1e-3) / 1e9 / 8000.0, 4),
             "roofline": {"kernel": "asm_copy", "bound": "hbm", "achieved": round(achieved, 1),
                          "peak": hbm_peak, "peak_kind": peak_kind, "unit": "GB/s",
                          "frac": round(achieved / hbm_peak, 4),

@@ -7,9 +7,9 @@
 //   asm_parents  (caller's lists only; commit_finish does this for the
 //                parents a commit completed) per listed parent: outcome,
 //                members to gather (0 unless Present), their exclusive scan
-//                (member bases), and for every 2048-member tile the parent
+//                (member bases), and for every AM_TILE-member tile the parent
 //                holding its first member;
-//   asm_members  per member, load-balanced over 2048-member tiles so a
+//   asm_members  per member, load-balanced over AM_TILE-member tiles so a
 //                100k-member parent spreads over many CTAs: read the record,
 //                scan the Present bytes (single-pass look-back) and write the
 //                plan — each parent's relative output offset, each
