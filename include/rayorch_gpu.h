@@ -24,13 +24,15 @@
  *   library never keeps a caller pointer beyond the call (except the arena,
  *   see ro_gather_commit).  A context owns its internal lineage state
  *   (phase words, result slots, parent counters, queues, scratch).
- * - Work is issued on the context's stream, in call order, except assembly:
- *   ro_assemble plans on the context's plan stream and copies on its copy
- *   stream (both the context's stream unless ro_ctx_set_streams names
- *   others).  Each assembly is ordered after all work the caller issued on
- *   the context before it; the caller's ro_assemble outputs are complete
- *   once ro_ctx_join has made the context's stream wait for the other two
- *   (or once any call synchronises).  Calls return without waiting for the
+ * - Work is issued on the context's stream, in call order, except assembly
+ *   and completion lists: ro_assemble plans on the context's plan stream and
+ *   copies on its copy stream, and with separate streams set
+ *   (ro_ctx_set_streams) ro_gather_commit builds its completed-parent list
+ *   on a stream the context owns.  Each assembly is ordered after all work
+ *   the caller issued on the context before it; the caller's ro_assemble
+ *   outputs and ro_gather_commit's d_done_parents / d_n_done are complete
+ *   once ro_ctx_join has made the context's stream wait for the others (or
+ *   once any call synchronises).  Calls return without waiting for the
  *   GPU unless an h_ output is requested: a non-NULL h_ pointer makes the
  *   call synchronise every stream and fill it in.  The d_ count outputs are
  *   written by the GPU in stream order, so a following call can consume
@@ -131,12 +133,16 @@ ro_status ro_ctx_sync(ro_ctx* ctx);
  * and copy of one wave's completed parents overlap the next waves' admission
  * and commits; up to three commits and assemblies per expansion may be in
  * flight at once (the context keeps three list and plan slots per expansion
- * and orders their reuse with events).  The context's stream first waits for
- * the old streams.  The caller keeps the streams alive until ro_ctx_destroy
+ * and orders their reuse with events).  With a plan stream other than the
+ * context's stream, the context also creates a stream of its own for the
+ * commits' completion scans (destroyed with the context), so one commit's
+ * completed-parent list is built while the next commit's reports are
+ * applied (two completion bitmaps per expansion, alternating).  The
+ * context's stream first waits for the old streams.  The caller keeps the streams alive until ro_ctx_destroy
  * or the next ro_ctx_set_streams. */
 ro_status ro_ctx_set_streams(ro_ctx* ctx, void* plan_stream, void* copy_stream);
 /* Make the context's stream wait (on the GPU) for all work issued so far on
- * the plan and copy streams.  Call it before reading assembly outputs in
+ * the plan and copy streams and the completion-scan stream.  Call it before reading assembly outputs in
  * stream order, before starting a capture of the context's stream, and
  * before ending one (a captured assembly forks onto the other streams, and a
  * capture must join them back).  Nothing waits on the host. */
@@ -303,6 +309,9 @@ ro_status ro_retry(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* d_ch
  *   d_done_parents uint32[done_cap] out or NULL: parents completed by this
  *               call, ascending.  done_cap must be >= min(n, parents of xid).
  *   d_n_done (device) / h_n_done (host, synchronises) out or NULL.
+ *   With separate streams set, d_done_parents and d_n_done are written on
+ *   the context's completion-scan stream (see the conventions above);
+ *   ro_assemble orders itself after them.
  */
 ro_status ro_gather_commit(ro_ctx* ctx, int32_t xid, uint64_t n, const uint64_t* d_n,
                            const uint32_t* d_child, const uint8_t* d_state,

@@ -13,14 +13,17 @@
 //                 That add also tells whether a member Failed or was
 //                 Suppressed, so the same thread records how many members the
 //                 parent will gather (0 if Suppressed) and adds it to its
-//                 bitmap word's total.
+//                 bitmap word's total.  When the call carried two reports for
+//                 one Grain or a GroupFailure (rare), the last CTA to finish
+//                 orders them, so the result equals applying the reports one
+//                 by one in array order, before the call ends.
 // commit_finish   turns the bitmap into the ascending list of completed
 //                 parents and their member bases (one single-pass scan over
 //                 bitmap words of (popcount, word total)) and clears it; the
-//                 list is what ro_assemble(NULL) plans and copies.  When the
-//                 scatter saw two reports for one Grain in the same call
-//                 (rare), the first CTA in orders them first, so the result
-//                 equals applying the reports one by one in array order.
+//                 list is what ro_assemble(NULL) plans and copies.  It reads
+//                 only the bitmap, the per-parent member counts and offsets,
+//                 so with two bitmaps (alternate commits) it can run on its
+//                 own stream while the next commit's scatter runs.
 #include <algorithm>
 
 #include "ro_internal.h"
@@ -41,12 +44,17 @@ __device__ __forceinline__ uint64_t commit_count(const CommitArgs& a) {
   return n < a.n_host ? n : a.n_host;
 }
 
+__device__ void resolve_duplicates(const CommitArgs& a, uint64_t n);
+__device__ void resolve_barriers(const CommitArgs& a, uint64_t n);
+
 __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a) {
   wait_predecessor();
   allow_successor();
   // verdict counts: accept, invalid, not in flight, stale, -, barrier,
   // duplicate candidates, accepted GroupFailures
   __shared__ unsigned long long s_cnt[8];
+  __shared__ unsigned long long s_fix[2];
+  __shared__ uint32_t s_last;
   DevScalars* ds = a.ds;
   if (threadIdx.x < 8) s_cnt[threadIdx.x] = 0;
   __syncthreads();
@@ -151,6 +159,24 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
     if (s_cnt[5]) atomicAdd(&ds->stats[7], s_cnt[5]);
     if (s_cnt[6]) atomicAdd(&ds->cm_conflicts, s_cnt[6]);
     if (s_cnt[7]) atomicAdd(&ds->cm_gf, s_cnt[7]);
+    s_last = ticket(&ds->cm_scatter_ticket) == gridDim.x - 1;
+    if (s_last) {
+      s_fix[0] = ld_relaxed_u64(&ds->cm_conflicts);
+      s_fix[1] = ld_relaxed_u64(&ds->cm_gf);
+    }
+  }
+  __syncthreads();
+  if (!s_last) return;
+  // The last CTA out: reports of one Grain that met in this call are ordered
+  // and GroupFailure barriers are applied before the call ends, so the next
+  // commit (and the completion scan, which may run on another stream) sees
+  // final outcomes.
+  if (s_fix[0]) resolve_duplicates(a, n);
+  if (s_fix[1]) resolve_barriers(a, n);
+  if (threadIdx.x == 0) {
+    ds->cm_conflicts = 0ull;
+    ds->cm_gf = 0ull;
+    ds->cm_scatter_ticket = 0u;
   }
 }
 
@@ -510,7 +536,6 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
   __shared__ Pair64 s_scan[33];
   __shared__ uint32_t s_tile;
   __shared__ Pair64 s_prefix;
-  __shared__ uint32_t s_fix;
   DevScalars* ds = a.ds;
   const ListBufs& L = a.list;
   const uint64_t n_words = ceil_div(a.P, 32);
@@ -529,31 +554,6 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
   }
   const uint32_t n_part = participants(n_tiles);
   if (blockIdx.x >= n_part) return;
-
-  // Reports of one Grain that met in this call: the first CTA here orders
-  // them; the others wait for it before reading outcome classes.
-  if (ds->cm_conflicts != 0 || ds->cm_gf != 0) {
-    if (threadIdx.x == 0) s_fix = atomicAdd(&ds->cm_fix_ticket, 1u);
-    __syncthreads();
-    if (s_fix == 0u) {
-      if (ds->cm_conflicts != 0) resolve_duplicates(a, commit_count(a));
-      if (ds->cm_gf != 0) resolve_barriers(a, commit_count(a));
-      if (threadIdx.x == 0) {
-        __threadfence();
-        st_release(&ds->cm_fix_done, 1u);
-      }
-    } else if (threadIdx.x == 0) {
-      uint32_t spins = 0;
-      while (ld_acquire(&ds->cm_fix_done) == 0u) {
-        if (++spins > SPIN_LIMIT) {
-          atomicOr(&ds->err, ERR_TIMEOUT);
-          break;
-        }
-        __nanosleep(128);
-      }
-    }
-    __syncthreads();
-  }
 
   for (;;) {
     if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_COMMIT]);
@@ -629,20 +629,19 @@ __global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a)
       ds->tile_ctr[TS_COMMIT] = 0u;
       ds->exit_ctr[TS_COMMIT] = 0u;
       ds->epoch[TS_COMMIT] += 1ull;
-      ds->cm_conflicts = 0ull;
-      ds->cm_gf = 0ull;
-      ds->cm_fix_ticket = 0u;
-      ds->cm_fix_done = 0u;
     }
   }
 }
 
-void launch_commit(const LaunchCfg& L, const CommitArgs& a) {
+void launch_commit_scatter(const LaunchCfg& L, const CommitArgs& a) {
   const uint64_t warps = ceil_div(a.n_host, 32);
   const int grid =
       (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(warps, CM_THREADS / 32),
                                                     (uint64_t)L.grid_commit));
   launch_k(L, K_COMMIT, commit_scatter_kernel, grid, CM_THREADS, 0, a);
+}
+
+void launch_commit_finish(const LaunchCfg& L, const CommitArgs& a) {
   const uint64_t n_tiles = ceil_div(ceil_div(a.P, 32), (uint64_t)CF_THREADS);
   const int grid_f = (int)std::max<uint64_t>(1, std::min<uint64_t>(n_tiles, (uint64_t)L.grid_cfinish));
   launch_k(L, K_CFINISH, commit_finish_kernel, grid_f, CF_THREADS, 0, a);

@@ -37,6 +37,7 @@ namespace {
 constexpr int MAX_EXPANSIONS = 64;
 constexpr int N_TS = 8;    // tile-status slots (TS_* in ro_common.cuh)
 constexpr int RING = 3;    // list / plan slots per expansion
+constexpr int BM_SLOTS = 2;   // completion bitmaps per expansion (commits alternate)
 
 struct DevBuf {
   void* p = nullptr;
@@ -69,7 +70,8 @@ struct PlanSlot {
 
 // Device buffers of one expansion slot, kept across ro_ctx_reset and reused.
 struct ExpSlot {
-  DevBuf offsets, pw, phase, rec, bitmap, tfp, pm, wm, gb;
+  DevBuf offsets, pw, phase, rec, bitmap, tfp, pm, wm, gb;   // bitmap, wm: two slots each
+  Ev bm_free[BM_SLOTS];   // the completion scan that read a bitmap slot is done
   ListSlot lists[RING];
   PlanSlot plans[RING];
   std::vector<QueueBufs> queues;
@@ -135,9 +137,11 @@ struct ro_ctx {
   cudaStream_t stream = nullptr;        // expansion, admission, commit
   cudaStream_t plan_stream = nullptr;   // assembly planning
   cudaStream_t copy_stream = nullptr;   // assembly copies
+  cudaStream_t fin_stream = nullptr;    // completion scans (commit_finish)
+  cudaStream_t own_fin = nullptr;       // created for fin_stream, destroyed with the context
   uint32_t n_calls = 1;
   int num_sms = 0;
-  LaunchCfg L{}, Lp{}, Lc{};
+  LaunchCfg L{}, Lp{}, Lc{}, Lf{};
   DevScalars* ds = nullptr;
   DevScalars* hs = nullptr;   // pinned mirror
   std::vector<ExpSlot> slots;
@@ -148,7 +152,7 @@ struct ro_ctx {
   // parent-bound reservation scratch (see ParentArgs)
   DevBuf pb_key[2], pb_val[2], pb_child, pb_hist, pb_dtot, pb_first, pb_endp, pb_hsz, pb_left,
       pb_hoff, pb_rem;
-  Ev fork, x_planned, join_plan, join_copy;
+  Ev fork, x_planned, join_plan, join_copy, fin_fork, fin_join, fin_plan;
   Profiler prof;
   ro_status sticky = RO_OK;
   std::string err;
@@ -208,6 +212,7 @@ void sync_all_streams(ro_ctx* c) {
   cudaStreamSynchronize(c->stream);
   if (c->plan_stream != c->stream) cudaStreamSynchronize(c->plan_stream);
   if (c->copy_stream != c->stream) cudaStreamSynchronize(c->copy_stream);
+  if (c->fin_stream != c->stream) cudaStreamSynchronize(c->fin_stream);
 }
 
 // Grow-only device buffer, zeroed when (re)allocated.  Growth needs a
@@ -279,6 +284,7 @@ ro_status order(ro_ctx* c, Ev& ev, cudaStream_t from, cudaStream_t to) {
 
 // The context's stream waits for the plan and copy streams.
 ro_status join(ro_ctx* c) {
+  RO_TRY(order(c, c->fin_join, c->fin_stream, c->stream));
   RO_TRY(order(c, c->join_plan, c->plan_stream, c->stream));
   if (c->copy_stream != c->plan_stream) RO_TRY(order(c, c->join_copy, c->copy_stream, c->stream));
   return RO_OK;
@@ -407,6 +413,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->stream = (cudaStream_t)stream;
   c->plan_stream = c->stream;
   c->copy_stream = c->stream;
+  c->fin_stream = c->stream;
   c->n_calls = n_calls;
   cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
   if (cudaMalloc(&c->ds, sizeof(DevScalars)) != cudaSuccess ||
@@ -441,6 +448,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_pb_sort = grid_for(kernel_ptr_parent(K_PB_SORT), PB_THREADS, s, 8);
   c->Lp = c->L;
   c->Lc = c->L;
+  c->Lf = c->L;
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) {
     cudaFree(c->ds);
@@ -459,6 +467,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   for (auto& s : c->slots) {
     free_buf(s.offsets); free_buf(s.pw); free_buf(s.phase); free_buf(s.rec); free_buf(s.bitmap);
     free_buf(s.tfp); free_buf(s.pm); free_buf(s.wm); free_buf(s.gb);
+    for (auto& e : s.bm_free) free_ev(e);
     for (auto& l : s.lists) {
       free_buf(l.done); free_buf(l.status); free_buf(l.mb); free_buf(l.coff); free_buf(l.mtfp);
       free_buf(l.hdr); free_ev(l.freed);
@@ -482,6 +491,8 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
                     &c->pb_hoff, &c->pb_rem})
     free_buf(*b);
   free_ev(c->fork); free_ev(c->x_planned); free_ev(c->join_plan); free_ev(c->join_copy);
+  free_ev(c->fin_fork); free_ev(c->fin_join); free_ev(c->fin_plan);
+  if (c->own_fin) cudaStreamDestroy(c->own_fin);
   for (cudaEvent_t e : c->prof.pool) cudaEventDestroy(e);
   cudaFree(c->ds);
   cudaFreeHost(c->hs);
@@ -504,8 +515,24 @@ ro_status ro_ctx_set_streams(ro_ctx* c, void* plan_stream, void* copy_stream) {
   RO_TRY(join(c));
   c->plan_stream = plan_stream ? (cudaStream_t)plan_stream : c->stream;
   c->copy_stream = copy_stream ? (cudaStream_t)copy_stream : c->stream;
+  // with streams of its own for assembly, the context also runs the
+  // completion scans on a stream of its own, so a commit's scan overlaps the
+  // next commit's scatter
+  if (c->plan_stream != c->stream) {
+    if (!c->own_fin) {
+      cudaError_t e = cudaStreamCreateWithFlags(&c->own_fin, cudaStreamNonBlocking);
+      if (e != cudaSuccess) {
+        c->own_fin = nullptr;
+        return cuda_fail(c, e, "cudaStreamCreate");
+      }
+    }
+    c->fin_stream = c->own_fin;
+  } else {
+    c->fin_stream = c->stream;
+  }
   c->Lp.stream = c->plan_stream;
   c->Lc.stream = c->copy_stream;
+  c->Lf.stream = c->fin_stream;
   return RO_OK;
 }
 
@@ -625,9 +652,9 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   const uint64_t mtfp_cap = ceil_div(N, AM_TILE) + 2;
   RO_TRY(ensure(c, S.phase, N * sizeof(uint32_t), "phase words"));
   RO_TRY(ensure(c, S.rec, N * sizeof(Rec), "result records"));
-  RO_TRY(ensure(c, S.bitmap, ceil_div(P, 32) * sizeof(uint32_t), "completion bitmap"));
+  RO_TRY(ensure(c, S.bitmap, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), "completion bitmaps"));
   RO_TRY(ensure(c, S.pm, P * sizeof(uint32_t), "parent member counts"));
-  RO_TRY(ensure(c, S.wm, ceil_div(P, 32) * sizeof(uint32_t), "word member counts"));
+  RO_TRY(ensure(c, S.wm, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), "word member counts"));
   RO_TRY(ensure(c, S.gb, P * sizeof(uint32_t), "GroupFailure barriers"));
   for (auto& l : S.lists) {
     RO_TRY(ensure(c, l.done, P * sizeof(uint32_t), "completed parents"));
@@ -643,8 +670,8 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
     RO_TRY(ensure(c, p.csrc, N * sizeof(uint64_t), "assembly plan"));
     RO_TRY(ensure(c, p.hdr, sizeof(PlanHdr), "assembly plan"));
   }
-  cudaMemsetAsync(S.bitmap.p, 0, ceil_div(P, 32) * sizeof(uint32_t), c->stream);
-  cudaMemsetAsync(S.wm.p, 0, ceil_div(P, 32) * sizeof(uint32_t), c->stream);
+  cudaMemsetAsync(S.bitmap.p, 0, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), c->stream);
+  cudaMemsetAsync(S.wm.p, 0, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), c->stream);
   cudaMemsetAsync(S.gb.p, 0xFF, P * sizeof(uint32_t), c->stream);   // no barrier pending
   ExpandFillArgs fa{};
   fa.offsets = (const uint64_t*)S.offsets.p;
@@ -883,9 +910,11 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.phase = (uint32_t*)S.phase.p;
   ca.rec = (Rec*)S.rec.p;
   ca.pw = (unsigned long long*)S.pw.p;
-  ca.bitmap = (uint32_t*)S.bitmap.p;
+  const int bs = (int)(x->commits % BM_SLOTS);   // bitmap slot of this commit
+  const uint64_t n_words = ceil_div(x->P, 32);
+  ca.bitmap = (uint32_t*)S.bitmap.p + bs * n_words;
   ca.pm = (uint32_t*)S.pm.p;
-  ca.wm = (uint32_t*)S.wm.p;
+  ca.wm = (uint32_t*)S.wm.p + bs * n_words;
   ca.gb = (uint32_t*)S.gb.p;
   if (d_code) {
     ca.code = d_code;
@@ -900,9 +929,16 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.list = list_bufs(LS, ceil_div(x->N, AM_TILE) + 2);
   ca.ds = c->ds;
   RO_TRY(tile_status(c, TS_COMMIT, ceil_div(ceil_div(x->P, 32), (uint64_t)CF_THREADS), &ca.ts));
-  // the slot is free once the planning that read it (RING commits ago) is done
-  RO_TRY(ev_wait(c, LS.freed, c->stream));
-  launch_commit(c->L, ca);
+  // the bitmap slot is free once the completion scan BM_SLOTS commits ago is done
+  RO_TRY(ev_wait(c, S.bm_free[bs], c->stream));
+  launch_commit_scatter(c->L, ca);
+  // the completion scan follows the scatter (on its own stream when the
+  // context has one); the list slot is free once the assembly that read it
+  // (RING commits ago) is done
+  RO_TRY(order(c, c->fin_fork, c->stream, c->fin_stream));
+  RO_TRY(ev_wait(c, LS.freed, c->fin_stream));
+  launch_commit_finish(c->Lf, ca);
+  if (c->fin_stream != c->stream) RO_TRY(ev_record(c, S.bm_free[bs], c->fin_stream));
   RO_TRY(check_launch(c, "gather_commit"));
   x->last_list = ls;
   x->commits += 1;
@@ -1052,6 +1088,7 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   // planning follows everything enqueued on the context's stream so far,
   // and the copy that last read this plan slot
   RO_TRY(order(c, c->fork, c->stream, c->plan_stream));
+  RO_TRY(order(c, c->fin_plan, c->fin_stream, c->plan_stream));   // the commit's completion list
   RO_TRY(ev_wait(c, PS.freed, c->plan_stream));
   launch_assemble_plan(c->Lp, aa);
   RO_TRY(check_launch(c, "assemble (plan)"));

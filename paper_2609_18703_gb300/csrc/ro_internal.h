@@ -229,7 +229,11 @@ struct CommitArgs {
   DevScalars* ds;
   TileStatus<Pair64> ts;
 };
-void launch_commit(const LaunchCfg& L, const CommitArgs& a);
+// the scatter (with the ordering of repeated reports and GroupFailure
+// barriers in its last CTA) and the completion scan, which may run on
+// different streams
+void launch_commit_scatter(const LaunchCfg& L, const CommitArgs& a);
+void launch_commit_finish(const LaunchCfg& L, const CommitArgs& a);
 
 // ---- ro_assemble ---------------------------------------------------------------------
 struct AssembleArgs {
