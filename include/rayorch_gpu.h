@@ -334,7 +334,11 @@ ro_status ro_gather_commit(ro_ctx* ctx, int32_t xid, uint64_t n, const uint64_t*
  *                is read in aligned 16-byte blocks, so the memory from
  *                d_arena up to the next 16-byte boundary at or after
  *                d_arena + arena_bytes must be readable (true of any
- *                cudaMalloc allocation that holds the arena).
+ *                cudaMalloc allocation that holds the arena).  The arena
+ *                may be pinned host memory (cudaHostAlloc / cudaHostRegister):
+ *                the copy then reads the needed payload bytes in place over
+ *                the host link with plain loads (no staging copy of the
+ *                arena).  Pageable host memory is refused (RO_E_INVAL).
  *   d_parents    uint32[n_parents] parent ids, or NULL for the parents
  *                completed by the latest ro_gather_commit on xid (in its
  *                ascending order); n_parents is then the capacity of the
@@ -344,6 +348,7 @@ ro_status ro_gather_commit(ro_ctx* ctx, int32_t xid, uint64_t n, const uint64_t*
  *                d_out (entry n = end); d_out_len uint32[n] out or NULL.
  *                With d_out_len, RO_E_OVERFLOW if a parent exceeds 2^32-1 bytes.
  *   d_out        uint8[out_cap] out.  Byte-exact, no padding; any alignment.
+ *                May be pinned host memory (written in place by the copy).
  *   d_out_bytes (device) / h_out_bytes (host, synchronises) out or NULL:
  *                bytes written by this call.
  * Together, (d_parents or the commit's list, d_status, d_out_len, d_out_off)

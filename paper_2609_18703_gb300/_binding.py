@@ -110,8 +110,10 @@ def _ptr(x):
     if isinstance(x, int):
         return x
     if hasattr(x, "data_ptr"):
-        if hasattr(x, "is_cuda") and not x.is_cuda:
-            raise ValueError("device argument is a CPU tensor")
+        # pinned host tensors are reachable from the GPU (ro_assemble accepts
+        # them for the arena and the output); pageable ones are not
+        if hasattr(x, "is_cuda") and not x.is_cuda and not x.is_pinned():
+            raise ValueError("argument is a pageable CPU tensor (pin it or move it to the GPU)")
         return x.data_ptr()
     raise TypeError(f"cannot pass {type(x)!r} as a pointer")
 

@@ -601,7 +601,9 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_
     st->vend = (uint32_t)(c.out_base + re - wbase);
   }
   const uint64_t arena = (uint64_t)(uintptr_t)c.a->arena;
-  const bool fits = np <= AC_PIECES;   // then the aligned blocks fit AC_BUF too
+  // then the aligned blocks fit AC_BUF too; a host-resident arena is read by
+  // the consumers with plain loads instead of being staged
+  const bool fits = np <= AC_PIECES && !c.a->arena_host;
   uint32_t roff = 0;   // running buffer offset (warp-uniform)
   if (fits) {
     for (uint64_t g = 0; g < np; g += 32) {
@@ -703,7 +705,7 @@ __device__ __forceinline__ void describe_chunk(const CopyCtx& c, uint64_t k, Chu
 // Stage a described chunk: piece table, expected bytes, one bulk copy per
 // piece.  Chunks of more than 32 pieces take stage_chunk's general path.
 __device__ void issue_chunk(const CopyCtx& c, const ChunkDesc& d, CopyStage* st, uint64_t* bar, int lane) {
-  if (!d.inreg) {
+  if (!d.inreg || c.a->arena_host) {
     stage_chunk(c, d.k, st, bar, lane);
     return;
   }

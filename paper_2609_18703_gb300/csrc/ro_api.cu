@@ -383,6 +383,28 @@ PlanBufs plan_bufs(PlanSlot& s, uint64_t member_cap) {
   return p;
 }
 
+// The device's view of a caller pointer: device memory as is; pinned host
+// memory through its device mapping (*host = 1); pageable host memory is an
+// error (the GPU may not reach it).
+template <class T>
+ro_status device_view(ro_ctx* c, T* p, T** out, int* host, const char* what) {
+  cudaPointerAttributes at{};
+  *host = 0;
+  *out = p;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(c, RO_E_INVAL, "ro_assemble: %s pointer is not known to CUDA", what);
+  }
+  if (at.type == cudaMemoryTypeHost) {
+    if (!at.devicePointer) return fail(c, RO_E_INVAL, "ro_assemble: %s host memory is not mapped", what);
+    *out = (T*)at.devicePointer;
+    *host = 1;
+  } else if (at.type == cudaMemoryTypeUnregistered) {
+    return fail(c, RO_E_INVAL, "ro_assemble: %s is pageable host memory (pin it)", what);
+  }
+  return RO_OK;
+}
+
 // The (expansion, Call) queues, empty at the expansion's first use.
 ro_status queue_ready(ro_ctx* c, QueueBufs& Q, uint64_t N) {
   if (Q.ready) return RO_OK;
@@ -1023,6 +1045,18 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   if (n_parents >= (1ull << 32)) return fail(c, RO_E_OVERFLOW, "ro_assemble: list of 2^32 or more");
   if (arena_bytes >= MAX_ARENA) return fail(c, RO_E_OVERFLOW, "ro_assemble: arena of 2^48 bytes or more");
   DeviceGuard g(c->device);
+  // The arena and the output may be pinned host memory (read and written in
+  // place by the copy, no staging copies); pageable host memory is refused.
+  int arena_host = 0;
+  {
+    const uint8_t* dev_arena = nullptr;
+    uint8_t* dev_out = nullptr;
+    RO_TRY(device_view(c, d_arena, &dev_arena, &arena_host, "arena"));
+    int out_host = 0;
+    if (d_out) RO_TRY(device_view(c, d_out, &dev_out, &out_host, "output"));
+    d_arena = dev_arena;
+    d_out = dev_out;
+  }
   ExpSlot& S = c->slots[xid];
   const uint64_t member_cap = std::max<uint64_t>(x->N, 1);
   const uint64_t mtfp_cap = ceil_div(member_cap, AM_TILE) + 2;
@@ -1044,6 +1078,7 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   aa.rec = (const Rec*)S.rec.p;
   aa.arena = d_arena;
   aa.arena_bytes = arena_bytes;
+  aa.arena_host = arena_host;
   aa.status = d_status;
   aa.out_off = d_out_off;
   aa.out_len = d_out_len;

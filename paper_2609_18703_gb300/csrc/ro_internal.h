@@ -246,6 +246,7 @@ struct AssembleArgs {
   const Rec* rec;
   const uint8_t* arena;
   uint64_t arena_bytes;
+  int arena_host;             // the arena is pinned host memory: no bulk (TMA) copies from it
   uint8_t* status;
   uint64_t* out_off;
   uint32_t* out_len;          // optional
