@@ -52,7 +52,12 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="docpage", choices=["docpage", "skew"],
+                    help="docpage: the 1M-document config (default); skew: 10M parents, "
+                         "1,000 of them with 100k children, 32-byte results, one wave")
     ap.add_argument("--parents", type=int, default=1_000_000)
+    ap.add_argument("--profile-all", action="store_true",
+                    help="time every kernel (CUDA events) in the kernel-timing steps")
     ap.add_argument("--waves", type=int, default=256)
     ap.add_argument("--no-graph", action="store_true", help="launch the wave loop eagerly")
     ap.add_argument("--retry", action="store_true", help="ro_retry throughput (failed attempts)")
@@ -403,7 +408,11 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     __graft_entry__.build()
     hbm_peak, peak_kind = peaks()
-    lv = docpage(parents=args.parents, waves=args.waves, salt=rank).top
+    if args.workload == "skew":
+        from workload import skew
+        lv = skew(salt=rank).top
+    else:
+        lv = docpage(parents=args.parents, waves=args.waves, salt=rank).top
     stream = torch.cuda.Stream()
     torch.cuda.set_stream(stream)
     ps = Pass(lv, local_rank, stream, lists=args.lists, filter_drop=args.filter_drop,
@@ -489,6 +498,8 @@ def run_ours(args, rank, world, local_rank):
     if ps.parent_bound:
         for k in res_kernels:
             mask |= 1 << ro.KERNELS.index(k)
+    if args.profile_all:
+        mask = (1 << len(ro.KERNELS)) - 1
     ro.ro_ctx_profile(ctx, mask)
     kt_steps = max(2, min(args.steps, 5))
     for _ in range(kt_steps):
@@ -544,9 +555,13 @@ def run_ours(args, rank, world, local_rank):
             "ms_per_step_best": round(step_ms[0], 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "u8/u32/u64", "data": "synthetic",
-            "config": {"workload": f"document->page: {ps.P} parents, {ps.N} children, "
-                                   f"{args.waves} arrival waves, batch {ps.B}",
-                       "parents": ps.P, "children": ps.N, "waves": args.waves,
+            "config": {"workload": (f"document->page: {ps.P} parents, {ps.N} children, "
+                                    f"{args.waves} arrival waves, batch {ps.B}"
+                                    if args.workload == "docpage" else
+                                    f"extreme skew: {ps.P} parents ({int((ps.lv.counts > 1).sum())} "
+                                    f"with {int(ps.lv.counts.max())} children), {ps.N} children, "
+                                    f"32-byte results, one arrival wave, batch {ps.B}"),
+                       "parents": ps.P, "children": ps.N, "waves": ps.W,
                        "arena_bytes": ps.arena_bytes, "assembled_bytes": S,
                        "reservation": "parent-bound" if ps.parent_bound else "elastic",
                        "output": "list entries per member" if ps.lists else "bytes",

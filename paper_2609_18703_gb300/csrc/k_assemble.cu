@@ -509,6 +509,21 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
+// tx bytes the current phase of `bar` waits for, without arriving
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes) : "memory");
+}
+// 16 bytes from 16-byte aligned global to 16-byte aligned shared memory,
+// asynchronously (no register staging)
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+// the current phase of `bar` also waits for this thread's cp.async copies
+// issued so far (the pending count goes up now and down when they land)
+__device__ __forceinline__ void cp_async_track(uint64_t* bar) {
+  asm volatile("cp.async.mbarrier.arrive.shared::cta.b64 [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+
 // Bounded wait on a stage barrier for the phase of parity `parity`; false
 // (recording ERR_TIMEOUT and raising the CTA's abort flag) if it gave up or
 // another warp of the CTA already did.
@@ -538,8 +553,10 @@ struct CopyStage {
   unsigned long long wbase;       // absolute address of the chunk's first word
   unsigned long long rel_s, rel_e;   // the chunk's bytes, relative to the call's output
   unsigned long long j_lo;        // first member of the chunk
-  uint32_t pstart[AC_PIECES + 1]; // output start of each piece (+ end), relative to wbase
-  int32_t qbase[AC_PIECES];       // buffer offset of output byte wbase, per piece
+  // output start of each piece (+ end), relative to wbase (< 16400), and the
+  // buffer offset of output byte wbase per piece (-16400 .. 24592)
+  uint16_t pstart[AC_PIECES + 1];
+  int16_t qbase[AC_PIECES];
   uint32_t pad2[3];
   // the 16 bytes before buf (the end of qbase) may be read and ignored: a
   // piece's first word can start before the piece's first staged block
@@ -601,38 +618,55 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_
     st->vend = (uint32_t)(c.out_base + re - wbase);
   }
   const uint64_t arena = (uint64_t)(uintptr_t)c.a->arena;
-  // then the aligned blocks fit AC_BUF too; a host-resident arena is read by
-  // the consumers with plain loads instead of being staged
-  const bool fits = np <= AC_PIECES && !c.a->arena_host;
+  // a host-resident arena is read by the consumers with plain loads instead
+  // of being staged; so is a chunk whose aligned blocks do not fit AC_BUF
+  const bool tabled = np <= AC_PIECES && !c.a->arena_host;
   uint32_t roff = 0;   // running buffer offset (warp-uniform)
-  if (fits) {
-    for (uint64_t g = 0; g < np; g += 32) {
-      const uint64_t i = g + lane;
-      uint32_t size = 0, sh = 0, ps = 0;
-      if (i < np) {
-        const uint64_t j = j_lo + i;
-        const uint64_t p0 = c.cpos[j], p1 = cpos_at(c, j + 1);
-        const uint64_t ob = p0 > rs ? p0 : rs, oe = p1 < re ? p1 : re;
-        const uint64_t src = arena + c.csrc[j] + (ob - p0);
-        const uint64_t a0 = src & ~15ull, a1 = (src + (oe - ob) + 15) & ~15ull;
-        size = (uint32_t)(a1 - a0);
-        sh = (uint32_t)(src & 15u);
-        ps = (uint32_t)(c.out_base + ob - wbase);
-      }
-      uint32_t inc = size;
+  uint32_t tx = 0;     // bytes of the pieces staged by bulk copies (per lane)
+  if (tabled) {
+    constexpr int R = 4;   // rounds of 32 pieces whose loads go out together
+    for (uint64_t g0 = 0; g0 < np; g0 += 32 * R) {
+      uint64_t p0[R], p1[R], cs[R];
 #pragma unroll
-      for (int d = 1; d < 32; d <<= 1) {
-        const uint32_t t = __shfl_up_sync(0xffffffffu, inc, d);
-        if (lane >= d) inc += t;
+      for (int u = 0; u < R; ++u) {
+        const uint64_t i = g0 + (uint64_t)u * 32 + lane;
+        p0[u] = p1[u] = cs[u] = 0;
+        if (i < np) {
+          const uint64_t j = j_lo + i;
+          p0[u] = c.cpos[j];
+          p1[u] = cpos_at(c, j + 1);
+          cs[u] = c.csrc[j];
+        }
       }
-      const uint32_t my_off = roff + inc - size;
-      if (i < np) {
-        st->pstart[i] = ps;
-        st->qbase[i] = (int32_t)(my_off + sh) - (int32_t)ps;
+#pragma unroll
+      for (int u = 0; u < R; ++u) {
+        const uint64_t i = g0 + (uint64_t)u * 32 + lane;
+        uint32_t size = 0, sh = 0, ps = 0;
+        if (i < np) {
+          const uint64_t ob = p0[u] > rs ? p0[u] : rs, oe = p1[u] < re ? p1[u] : re;
+          const uint64_t src = arena + cs[u] + (ob - p0[u]);
+          const uint64_t a0 = src & ~15ull, a1 = (src + (oe - ob) + 15) & ~15ull;
+          size = (uint32_t)(a1 - a0);
+          sh = (uint32_t)(src & 15u);
+          ps = (uint32_t)(c.out_base + ob - wbase);
+          if (size > AC_SMALL) tx += size;
+        }
+        uint32_t inc = size;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+          const uint32_t t = __shfl_up_sync(0xffffffffu, inc, d);
+          if (lane >= d) inc += t;
+        }
+        const uint32_t my_off = roff + inc - size;
+        if (i < np) {
+          st->pstart[i] = (uint16_t)ps;
+          st->qbase[i] = (int16_t)((int32_t)(my_off + sh) - (int32_t)ps);
+        }
+        roff += __shfl_sync(0xffffffffu, inc, 31);
       }
-      roff += __shfl_sync(0xffffffffu, inc, 31);
     }
   }
+  const bool fits = tabled && roff <= AC_BUF;
   if (!fits) {
     if (lane == 0) {
       st->np = AC_FALLBACK;
@@ -641,25 +675,52 @@ __device__ void stage_chunk(const CopyCtx& c, uint64_t k, CopyStage* st, uint64_
     __syncwarp();
     return;
   }
+  // the stage completes when the bulk copies' bytes have landed, every
+  // lane's cp.async copies of small pieces too, and lane 0 has arrived
+  for (int d = 16; d > 0; d >>= 1) tx += __shfl_xor_sync(0xffffffffu, tx, d);
   if (lane == 0) {
     st->np = (uint32_t)np;
-    st->pstart[np] = (uint32_t)(c.out_base + re - wbase);
+    st->pstart[np] = (uint16_t)(c.out_base + re - wbase);
+    mbar_expect_tx(bar, tx);
   }
   __syncwarp();
   fence_proxy_async_smem();   // earlier generic accesses of this stage before async writes
-  if (lane == 0) mbar_arrive_tx(bar, roff);
-  __syncwarp();
-  for (uint64_t i = lane; i < np; i += 32) {
-    const uint64_t j = j_lo + i;
-    const uint64_t p0 = c.cpos[j];
-    const uint64_t ob = wbase + st->pstart[i] - c.out_base;      // relative
-    const uint64_t oe = wbase + st->pstart[i + 1] - c.out_base;
-    const uint64_t src = arena + c.csrc[j] + (ob - p0);
-    const uint64_t a0 = src & ~15ull, a1 = (src + (oe - ob) + 15) & ~15ull;
-    const uint32_t off = (uint32_t)(st->qbase[i] + (int32_t)st->pstart[i]) - (uint32_t)(src & 15u);
-    if (a1 > a0)   // a member that starts exactly at the chunk's end stages nothing
-      bulk_g2s(st->buf + off, reinterpret_cast<const void*>((uintptr_t)a0), (uint32_t)(a1 - a0), bar);
+  bool small = false;
+  constexpr int R = 4;
+  for (uint64_t i0 = lane; i0 < np; i0 += 32 * R) {
+    uint64_t p0[R], cs[R];
+#pragma unroll
+    for (int u = 0; u < R; ++u) {
+      const uint64_t i = i0 + (uint64_t)u * 32;
+      p0[u] = cs[u] = 0;
+      if (i < np) {
+        p0[u] = c.cpos[j_lo + i];
+        cs[u] = c.csrc[j_lo + i];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < R; ++u) {
+      const uint64_t i = i0 + (uint64_t)u * 32;
+      if (i >= np) break;
+      const uint64_t ob = wbase + st->pstart[i] - c.out_base;      // relative
+      const uint64_t oe = wbase + st->pstart[i + 1] - c.out_base;
+      const uint64_t src = arena + cs[u] + (ob - p0[u]);
+      const uint64_t a0 = src & ~15ull, a1 = (src + (oe - ob) + 15) & ~15ull;
+      const uint32_t off = (uint32_t)(st->qbase[i] + (int32_t)st->pstart[i]) - (uint32_t)(src & 15u);
+      const uint32_t size = (uint32_t)(a1 - a0);   // 0: a member that starts at the chunk's end
+      if (size > AC_SMALL) {
+        bulk_g2s(st->buf + off, reinterpret_cast<const void*>((uintptr_t)a0), size, bar);
+      } else {
+        // small pieces: one 16-byte asynchronous copy per block, no bulk copy
+        for (uint32_t b = 0; b < size; b += 16)
+          cp_async16(st->buf + off + b, reinterpret_cast<const void*>((uintptr_t)(a0 + b)));
+        small = small || size != 0;
+      }
+    }
   }
+  if (small) cp_async_track(bar);
+  __syncwarp();
+  if (lane == 0) mbar_arrive(bar);
 }
 
 // A chunk's pieces as a producer warp finds them.  With at most 32 pieces
@@ -718,8 +779,8 @@ __device__ void issue_chunk(const CopyCtx& c, const ChunkDesc& d, CopyStage* st,
   const uint32_t my_off = inc - d.size;
   const uint32_t roff = __shfl_sync(0xffffffffu, inc, 31);
   if ((uint64_t)lane < d.np) {
-    st->pstart[lane] = d.ps;
-    st->qbase[lane] = (int32_t)(my_off + d.sh) - (int32_t)d.ps;
+    st->pstart[lane] = (uint16_t)d.ps;
+    st->qbase[lane] = (int16_t)((int32_t)(my_off + d.sh) - (int32_t)d.ps);
   }
   if (lane == 0) {
     st->wbase = d.wbase;
@@ -729,7 +790,7 @@ __device__ void issue_chunk(const CopyCtx& c, const ChunkDesc& d, CopyStage* st,
     st->vbeg = (uint32_t)(c.out_base + d.rs - d.wbase);
     st->vend = (uint32_t)(c.out_base + d.re - d.wbase);
     st->np = (uint32_t)d.np;
-    st->pstart[d.np] = (uint32_t)(c.out_base + d.re - d.wbase);
+    st->pstart[d.np] = (uint16_t)(c.out_base + d.re - d.wbase);
   }
   __syncwarp();
   fence_proxy_async_smem();   // earlier generic accesses of this stage before async writes
@@ -774,10 +835,21 @@ __device__ void emit_range(const CopyStage* st, uint32_t cw, int lane) {
       const uint32_t wr = w * 16u;
       const uint32_t lo = wr > vbeg ? wr : vbeg;
       const uint32_t hi = (wr + 16u < vend) ? wr + 16u : vend;
+      // the piece holding byte lo: the warp's last piece or the next (large
+      // pieces), else a search of the rest (many small pieces per chunk)
       uint32_t pe = st->pstart[i + 1];
-      while (pe <= lo) {
+      if (pe <= lo) {
         ++i;
         pe = st->pstart[i + 1];
+        if (pe <= lo) {
+          uint32_t ia = i + 1, ib = np;   // pstart[ia] <= lo < pstart[np]
+          while (ib - ia > 1) {
+            const uint32_t m = (ia + ib) >> 1;
+            if (st->pstart[m] <= lo) ia = m; else ib = m;
+          }
+          i = ia;
+          pe = st->pstart[i + 1];
+        }
       }
       // bytes [lo, pe) come from piece i; a word that reaches further takes
       // the rest from the following pieces, one boundary at a time

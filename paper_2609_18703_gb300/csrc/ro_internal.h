@@ -28,9 +28,13 @@ constexpr int AC_THREADS = 256;                               // 2 producer + 6 
 constexpr int AC_PRODUCERS = 2, AC_CONSUMERS = AC_THREADS / 32 - AC_PRODUCERS;
 constexpr int AC_STAGES = 3;                                  // chunks staged per CTA
 constexpr uint64_t AC_CHUNK = 16384;                          // output bytes per copy chunk (relative)
-constexpr uint32_t AC_PIECES = 256;                           // member pieces staged per chunk
-constexpr uint32_t AC_BUF = 16384 + 32 * AC_PIECES;           // staged source bytes per chunk (fits any
-                                                              // AC_PIECES pieces: each adds < 32)
+// A chunk is staged when it has at most AC_PIECES member pieces whose
+// 16-byte-aligned source blocks fit AC_BUF bytes (each piece adds < 32 bytes
+// of alignment to its payload); other chunks are copied directly.  Packed
+// records of 32 bytes or more start on 16-byte boundaries and fit.
+constexpr uint32_t AC_PIECES = 1024;
+constexpr uint32_t AC_BUF = 24576;
+constexpr uint32_t AC_SMALL = 64;   // pieces of at most this many staged bytes: cp.async, not a bulk copy
 
 // kernel entry points for occupancy queries and per-kernel timing
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CFINISH, K_APARENTS,
