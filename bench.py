@@ -43,7 +43,7 @@ K_ACOPY = 8
 # full-size bench is too large to capture with the full section set, so the
 # per-launch traffic reported here scales that ratio by the bytes a launch
 # assembles.
-COPY_TRAFFIC_RATIO = 0.990
+COPY_TRAFFIC_RATIO = 0.987
 
 
 def parse():
@@ -410,7 +410,9 @@ def run_ours(args, rank, world, local_rank):
     hbm_peak, peak_kind = peaks()
     if args.workload == "skew":
         from workload import skew
-        lv = skew(salt=rank).top
+        # --parents scales the config (same 1-in-10,000 share of 100k-child parents)
+        P = args.parents if args.parents != 1_000_000 else 10_000_000
+        lv = skew(parents=P, heavy=max(1, P // 10_000), salt=rank).top
     else:
         lv = docpage(parents=args.parents, waves=args.waves, salt=rank).top
     stream = torch.cuda.Stream()

@@ -158,7 +158,8 @@ enum {
   RO_K_COMMIT_SCATTER = 4, RO_K_COMMIT_FINISH = 5, RO_K_ASM_PARENTS = 6, RO_K_ASM_MEMBERS = 7,
   RO_K_ASM_COPY = 8, RO_K_RETRY_CLAIM = 9, RO_K_RETRY_SCATTER = 10, RO_K_PB_KEYS = 11,
   RO_K_PB_HIST = 12, RO_K_PB_ROWSCAN = 13, RO_K_PB_SORT = 14, RO_K_PB_BOUNDS = 15,
-  RO_K_PB_HEADS = 16, RO_K_PB_MARK = 17, RO_K_PB_SCAN = 18, RO_K_PB_EMIT = 19, RO_K_COUNT = 20
+  RO_K_PB_HEADS = 16, RO_K_PB_MARK = 17, RO_K_PB_SCAN = 18, RO_K_PB_EMIT = 19,
+  RO_K_COMMIT_FIX = 20, RO_K_COUNT = 21
 };
 /* Tracing (no counterpart in the paper; it instruments the path).  Every
  * kernel launch is counted; kernels whose bit (1 << RO_K_*) is set in

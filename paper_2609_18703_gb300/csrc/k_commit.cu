@@ -53,8 +53,6 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
   // verdict counts: accept, invalid, not in flight, stale, -, barrier,
   // duplicate candidates, accepted GroupFailures
   __shared__ unsigned long long s_cnt[8];
-  __shared__ unsigned long long s_fix[2];
-  __shared__ uint32_t s_last;
   DevScalars* ds = a.ds;
   if (threadIdx.x < 8) s_cnt[threadIdx.x] = 0;
   __syncthreads();
@@ -159,24 +157,30 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
     if (s_cnt[5]) atomicAdd(&ds->stats[7], s_cnt[5]);
     if (s_cnt[6]) atomicAdd(&ds->cm_conflicts, s_cnt[6]);
     if (s_cnt[7]) atomicAdd(&ds->cm_gf, s_cnt[7]);
-    s_last = ticket(&ds->cm_scatter_ticket) == gridDim.x - 1;
-    if (s_last) {
-      s_fix[0] = ld_relaxed_u64(&ds->cm_conflicts);
-      s_fix[1] = ld_relaxed_u64(&ds->cm_gf);
-    }
+  }
+}
+
+// One CTA after the scatter, on the same stream: reports of one Grain that
+// met in this call are ordered and GroupFailure barriers applied (rare; it
+// returns at once otherwise), so the next commit and the completion scan
+// (which may run on another stream) see final outcomes.  Kept out of the
+// scatter so that the scatter's registers and shared memory stay small.
+__global__ void __launch_bounds__(CM_THREADS) commit_fix_kernel(CommitArgs a) {
+  wait_predecessor();
+  DevScalars* ds = a.ds;
+  __shared__ unsigned long long s_fix[2];
+  if (threadIdx.x == 0) {
+    s_fix[0] = ds->cm_conflicts;
+    s_fix[1] = ds->cm_gf;
   }
   __syncthreads();
-  if (!s_last) return;
-  // The last CTA out: reports of one Grain that met in this call are ordered
-  // and GroupFailure barriers are applied before the call ends, so the next
-  // commit (and the completion scan, which may run on another stream) sees
-  // final outcomes.
+  if (s_fix[0] == 0ull && s_fix[1] == 0ull) return;
+  const uint64_t n = commit_count(a);
   if (s_fix[0]) resolve_duplicates(a, n);
   if (s_fix[1]) resolve_barriers(a, n);
   if (threadIdx.x == 0) {
     ds->cm_conflicts = 0ull;
     ds->cm_gf = 0ull;
-    ds->cm_scatter_ticket = 0u;
   }
 }
 
@@ -639,6 +643,7 @@ void launch_commit_scatter(const LaunchCfg& L, const CommitArgs& a) {
       (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(warps, CM_THREADS / 32),
                                                     (uint64_t)L.grid_commit));
   launch_k(L, K_COMMIT, commit_scatter_kernel, grid, CM_THREADS, 0, a);
+  launch_k(L, K_CFIX, commit_fix_kernel, 1, CM_THREADS, 0, a);
 }
 
 void launch_commit_finish(const LaunchCfg& L, const CommitArgs& a) {
@@ -648,6 +653,7 @@ void launch_commit_finish(const LaunchCfg& L, const CommitArgs& a) {
 }
 
 const void* kernel_ptr_commit(int which) {
+  if (which == K_CFIX) return (const void*)commit_fix_kernel;
   return which == K_COMMIT ? (const void*)commit_scatter_kernel : (const void*)commit_finish_kernel;
 }
 

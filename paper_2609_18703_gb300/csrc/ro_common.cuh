@@ -111,7 +111,7 @@ struct DevScalars {
   // chunk (no flush), totals, the admission's bad candidates, refusal
   unsigned long long pb_Q, pb_head, pb_old_tail, pb_stop, pb_npop, pb_nb, pb_R, pb_bad;
   uint32_t pb_err, pb_pad;
-  uint32_t cm_scatter_ticket, cm_pad;
+  uint32_t cm_pad0, cm_pad1;
   // ro_assemble
   unsigned long long as_bytes;    // bytes of the latest assemble (host read-back)
   unsigned long long as_elems;    // list entries of the latest assemble (host read-back)

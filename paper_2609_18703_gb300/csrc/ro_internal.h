@@ -40,7 +40,7 @@ constexpr uint32_t AC_SMALL = 64;   // pieces of at most this many staged bytes:
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CFINISH, K_APARENTS,
                 K_AMEMBERS, K_ACOPY, K_RT_CLAIM, K_RT_SCATTER, K_PB_KEYS, K_PB_HIST,
                 K_PB_ROWSCAN, K_PB_SORT, K_PB_BOUNDS, K_PB_HEADS, K_PB_MARK, K_PB_SCAN, K_PB_EMIT,
-                K_COUNT };
+                K_CFIX, K_COUNT };
 
 // Launch counter and optional CUDA-event timing of selected kernels, on the
 // stream they are launched on (see ro_ctx_profile in the C ABI).
