@@ -18,7 +18,7 @@
 //                first byte;
 //   asm_copy     per chunk: two producer warps stage chunks' member pieces
 //                in shared memory with cp.async.bulk (a ring of AC_STAGES
-//                stages, mbarrier completion, bounded waits) while six
+//                stages, mbarrier completion, bounded waits) while eight
 //                consumer warps turn staged chunks into aligned 16-byte
 //                stores; source and destination alignments may differ
 //                arbitrarily.
@@ -152,7 +152,7 @@ __global__ void __launch_bounds__(AP_THREADS) asm_parents_kernel(AssembleArgs a)
 
 // ---------------------------------------------------------------------------
 // asm_members: list -> plan (relative offsets and member positions).
-__global__ void __launch_bounds__(AM_THREADS) asm_members_kernel(AssembleArgs a) {
+__global__ void __maxnreg__(56) asm_members_kernel(AssembleArgs a) {
   wait_predecessor();
   __shared__ uint32_t s_mb[AM_SMEM_CAP];
   __shared__ uint32_t s_coff[AM_SMEM_CAP];
@@ -898,10 +898,11 @@ __device__ void emit_direct(const CopyCtx& c, const CopyStage* st, uint32_t cw, 
 // into a ring of AC_STAGES stages (producer p takes the CTA's chunks i with
 // i % AC_PRODUCERS == p), the other warps write them out in order; full
 // and empty mbarriers per stage hand the stages back and forth.
-// Sized to leave room beside it: two CTAs per SM take 2 x 256 threads x 80
-// registers and 2 x 3 stages of shared memory, so the commit kernels of later
-// waves (other streams) can be resident on the same SMs while a copy runs.
-__global__ void __launch_bounds__(AC_THREADS, 3) asm_copy_kernel(AssembleArgs a) {
+// Sized to leave room beside it: two CTAs per SM take 2 x 320 threads x 80
+// registers and 2 x 3 stages of shared memory, so a planning CTA (56
+// registers) of a later wave (another stream) can be resident on the same SM
+// while a copy runs.
+__global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
   wait_predecessor();
   extern __shared__ __align__(128) unsigned char ac_smem[];
   __shared__ __align__(8) uint64_t full_bar[AC_STAGES];

@@ -18,13 +18,13 @@ constexpr int CM_THREADS = 256;
 constexpr int CF_THREADS = 256;                               // bitmap words per tile (1 each)
 constexpr int MB_ITEMS = 8;                                   // members per lane per step
 constexpr int AP_THREADS = 256, AP_ITEMS = 4;                 // listed parents per tile: 1024
-// members per tile: 1024.  At 64 registers and 17 KB of shared memory a CTA
-// fits beside two asm_copy CTAs on one SM, so the next waves' planning runs
-// while a copy is in flight.
+// members per tile: 1024.  At 56 registers and 17 KB of shared memory a CTA
+// fits beside two asm_copy CTAs on one SM (2 x 320 x 80 + 256 x 56 = 65,536
+// registers), so the next waves' planning runs while a copy is in flight.
 constexpr int AM_THREADS = 256, AM_ITEMS = 4;
 constexpr uint32_t AM_TILE = AM_THREADS * AM_ITEMS;
 constexpr uint32_t AM_SMEM_CAP = 2048;                        // listed parents staged per tile
-constexpr int AC_THREADS = 256;                               // 2 producer + 6 consumer warps
+constexpr int AC_THREADS = 320;                               // 2 producer + 8 consumer warps
 constexpr int AC_PRODUCERS = 2, AC_CONSUMERS = AC_THREADS / 32 - AC_PRODUCERS;
 constexpr int AC_STAGES = 3;                                  // chunks staged per CTA
 constexpr uint64_t AC_CHUNK = 16384;                          // output bytes per copy chunk (relative)
