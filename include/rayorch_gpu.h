@@ -137,7 +137,7 @@ ro_status ro_ctx_sync(ro_ctx* ctx);
  * context's stream, the context also creates a stream of its own for the
  * commits' completion scans (destroyed with the context), so one commit's
  * completed-parent list is built while the next commit's reports are
- * applied (two completion bitmaps per expansion, alternating).  The
+ * applied (four completion bitmaps per expansion, taken in turn).  The
  * context's stream first waits for the old streams.  The caller keeps the streams alive until ro_ctx_destroy
  * or the next ro_ctx_set_streams. */
 ro_status ro_ctx_set_streams(ro_ctx* ctx, void* plan_stream, void* copy_stream);

@@ -22,7 +22,7 @@
 //                 bitmap words of (popcount, word total)) and clears it; the
 //                 list is what ro_assemble(NULL) plans and copies.  It reads
 //                 only the bitmap, the per-parent member counts and offsets,
-//                 so with two bitmaps (alternate commits) it can run on its
+//                 so with several bitmaps (commits take them in turn) it runs on its
 //                 own stream while the next commit's scatter runs.
 #include <algorithm>
 

@@ -37,7 +37,7 @@ namespace {
 constexpr int MAX_EXPANSIONS = 64;
 constexpr int N_TS = 8;    // tile-status slots (TS_* in ro_common.cuh)
 constexpr int RING = 3;    // list / plan slots per expansion
-constexpr int BM_SLOTS = 2;   // completion bitmaps per expansion (commits alternate)
+constexpr int BM_SLOTS = 4;   // completion bitmaps per expansion (commits take them in turn)
 
 struct DevBuf {
   void* p = nullptr;
