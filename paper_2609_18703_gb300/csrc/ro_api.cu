@@ -463,7 +463,9 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_commit = grid_for(kernel_ptr_commit(K_COMMIT), CM_THREADS, s, 8);
   c->L.grid_cfinish = grid_for(kernel_ptr_commit(K_CFINISH), CF_THREADS, s, 4);
   c->L.grid_aparents = grid_for(kernel_ptr_assemble(K_APARENTS), AP_THREADS, s, 4);
-  c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 1);
+  // up to 4 planning CTAs per SM: large waves (100k-member parents) get the
+  // parallelism; beside a running copy only one fits and the rest wait
+  c->L.grid_amembers = grid_for(kernel_ptr_assemble(K_AMEMBERS), AM_THREADS, s, 4);
   c->L.grid_acopy = grid_for(kernel_ptr_assemble(K_ACOPY), AC_THREADS, s, 2, asm_copy_smem());
   c->L.grid_retry = grid_for(kernel_ptr_retry(K_RT_SCATTER), RT_THREADS, s, 4);
   c->L.grid_pb = grid_for(kernel_ptr_parent(K_PB_HEADS), PB_THREADS, s, 8);
