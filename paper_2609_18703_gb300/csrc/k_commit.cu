@@ -31,7 +31,24 @@
 namespace ro {
 
 constexpr uint8_t V_WIN_SEALER = 7, V_WIN_CAND = 8, V_LOSE_SEALER = 9, V_LOSE_CAND = 10;
-constexpr uint32_t GB_NONE = 0xFFFFFFFFu;
+// The GroupFailure barrier table: per parent (seq << 32) | ~r, r the lowest
+// accepted GroupFailure report of commit seq (atomicMax keeps the lowest r of
+// the newest commit); an entry of an older commit means no barrier, so the
+// table never needs clearing.
+__device__ __forceinline__ unsigned long long gb_tag(uint32_t seq, uint32_t r) {
+  return ((unsigned long long)seq << 32) | (unsigned long long)(uint32_t)~r;
+}
+__device__ __forceinline__ bool gb_get(const CommitArgs& a, uint32_t p, uint32_t* r) {
+  const unsigned long long v = __ldcg(a.gb + p);
+  if ((uint32_t)(v >> 32) != a.seq) return false;
+  *r = ~(uint32_t)v;
+  return true;
+}
+__device__ __forceinline__ uint32_t fix_slot(const CommitArgs& a) { return a.seq & 1u; }
+__device__ __forceinline__ void stat_add(unsigned long long* s, unsigned long long d) {
+  if (d) atomicAdd(s, d);   // d may be a negative delta in two's complement
+}
+
 
 // record word read past L1 (other threads update it with atomics at L2)
 __device__ __forceinline__ uint64_t ld_w(const Rec* rc) {
@@ -46,6 +63,8 @@ __device__ __forceinline__ uint64_t commit_count(const CommitArgs& a) {
 
 __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n);
 __device__ void resolve_barriers(const CommitArgs& a, uint64_t n);
+__device__ void seal_open(const CommitArgs& a, uint32_t pp, int lane, unsigned long long* n_wait,
+                          unsigned long long* n_fly);
 
 __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a) {
   wait_predecessor();
@@ -59,6 +78,10 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
   const uint64_t n = commit_count(a);
   if (a.d_n && *a.d_n > a.n_host && blockIdx.x == 0 && threadIdx.x == 0)
     atomicOr(&ds->err, ERR_INVAL);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {   // the next commit's slot (its last reader is done)
+    ds->cm_conflicts[fix_slot(a) ^ 1u] = 0ull;
+    ds->cm_gf[fix_slot(a) ^ 1u] = 0ull;
+  }
   const int lane = threadIdx.x & 31;
   const uint64_t warp_global = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
@@ -102,7 +125,7 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
                                         ((uint64_t)outcome << W_STATE_SHIFT)));
           p = par;
           bad = (s == ST_FAILED || s == ST_SUPPRESSED || s == ST_GROUP_FAILURE);
-          if (s == ST_GROUP_FAILURE) atomicMin(a.gb + par, (uint32_t)r);   // barrier: commit_finish
+          if (s == ST_GROUP_FAILURE) atomicMax(a.gb + par, gb_tag(a.seq, (uint32_t)r));   // barrier
         } else if ((cur & 3u) == PH_WAITING || (cur & 3u) == PH_READY) {
           v = V_NOT_INFLIGHT;
         } else if ((cur >> 2) != g) {
@@ -155,33 +178,108 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
     for (int k = 0; k < 4; ++k)
       if (s_cnt[k]) atomicAdd(&ds->stats[k], s_cnt[k]);
     if (s_cnt[5]) atomicAdd(&ds->stats[7], s_cnt[5]);
-    if (s_cnt[6]) atomicAdd(&ds->cm_conflicts, s_cnt[6]);
-    if (s_cnt[7]) atomicAdd(&ds->cm_gf, s_cnt[7]);
+    if (s_cnt[6]) atomicAdd(&ds->cm_conflicts[fix_slot(a)], s_cnt[6]);
+    if (s_cnt[7]) atomicAdd(&ds->cm_gf[fix_slot(a)], s_cnt[7]);
   }
 }
 
-// One CTA after the scatter, on the same stream: reports of one Grain that
-// met in this call are ordered and GroupFailure barriers applied (rare; it
-// returns at once otherwise), so the next commit and the completion scan
-// (which may run on another stream) see final outcomes.  Kept out of the
-// scatter so that the scatter's registers and shared memory stay small.
+// The barriers of a call without repeated reports, spread over the grid:
+// each CTA takes tiles of FX_TILE reports.  A report after its parent's
+// barrier report (table gb) is rejected: an accepted one's Grain becomes
+// Suppressed by the barrier, one that met a WAITING or READY Grain meets a
+// sealed one (the fence compares generations); and the warp holding a
+// barrier's own GroupFailure report seals that parent's open siblings.  The
+// two touch disjoint Grains (sealed by this call vs still open), and the
+// parent's counters are only added to, so no order between them is needed;
+// the result equals the one-CTA pass in array order.
+constexpr uint32_t FX_TILE = 2048;
+__device__ void apply_barriers_grid(const CommitArgs& a, uint64_t n) {
+  DevScalars* ds = a.ds;
+  __shared__ unsigned long long s_d[7];   // as in resolve_barriers
+  if (threadIdx.x < 7) s_d[threadIdx.x] = 0;
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const uint64_t tiles = ceil_div(n, (uint64_t)FX_TILE);
+  for (uint64_t t = blockIdx.x; t < tiles; t += gridDim.x) {
+    for (uint64_t base = t * FX_TILE; base < (t + 1) * FX_TILE; base += blockDim.x) {
+      const uint64_t r = base + threadIdx.x;
+      uint32_t p = 0, b = 0;
+      bool under = false, trig = false;
+      uint8_t v = V_INVALID;
+      uint64_t c = 0;
+      if (r < n) {
+        v = a.code[r];
+        if (v == V_ACCEPT || v == V_NOT_INFLIGHT) {
+          c = a.child[r];
+          p = a.rec[c].parent;
+          if (gb_get(a, p, &b)) {
+            under = r > b;
+            trig = r == b;   // the barrier's own (accepted) GroupFailure report
+          }
+        }
+      }
+      if (under) {
+        if (v == V_ACCEPT) {
+          Rec* rc = a.rec + c;
+          const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
+          rc->len = 0u;
+          rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
+          const uint8_t st = a.state[r];
+          if (!(st == ST_FAILED || st == ST_SUPPRESSED || st == ST_GROUP_FAILURE))
+            atomicAdd(a.pw + p, 1ull << 32);   // its outcome class is now bad
+          a.code[r] = V_BARRIER;
+          atomicAdd(&s_d[0], ~0ull);
+          atomicAdd(&s_d[4], 1ull);
+          atomicAdd(&s_d[6], 1ull);
+        } else {
+          const uint32_t ph = __ldcg(a.phase + c);
+          const uint32_t gen_c = ((ph & 3u) == PH_WAITING) ? 0u : (ph >> 2);
+          const uint32_t g = a.gen ? a.gen[r] : 0u;
+          const bool same = g == gen_c;
+          a.code[r] = same ? V_BARRIER : V_STALE;
+          atomicAdd(&s_d[1], ~0ull);
+          atomicAdd(&s_d[same ? 4 : 2], 1ull);
+        }
+      }
+      unsigned m = __ballot_sync(0xffffffffu, trig);
+      while (m) {
+        const int src = __ffs(m) - 1;
+        m &= m - 1;
+        seal_open(a, __shfl_sync(0xffffffffu, p, src), lane, &s_d[5], &s_d[6]);
+      }
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    stat_add(&ds->stats[0], s_d[0]);
+    stat_add(&ds->stats[2], s_d[1]);
+    stat_add(&ds->stats[3], s_d[2]);
+    stat_add(&ds->stats[7], s_d[4]);
+    stat_add(&ds->stats[8], s_d[5]);
+    stat_add(&ds->stats[9], s_d[6]);
+  }
+}
+
+// After the scatter, on the same stream: reports of one Grain that met in
+// this call are ordered (one CTA, array order) and GroupFailure barriers
+// applied (one CTA after an ordering, else the whole grid), so the next
+// commit and the completion scan (which may run on another stream) see
+// final outcomes.  Returns at once when the scatter saw neither.  Kept out
+// of the scatter so that the scatter's registers and shared memory stay small.
 __global__ void __launch_bounds__(CM_THREADS) commit_fix_kernel(CommitArgs a) {
   wait_predecessor();
   DevScalars* ds = a.ds;
-  __shared__ unsigned long long s_fix[2];
-  if (threadIdx.x == 0) {
-    s_fix[0] = ds->cm_conflicts;
-    s_fix[1] = ds->cm_gf;
-  }
-  __syncthreads();
-  if (s_fix[0] == 0ull && s_fix[1] == 0ull) return;
+  const unsigned long long dups = ds->cm_conflicts[fix_slot(a)], gfs = ds->cm_gf[fix_slot(a)];
+  if (dups == 0ull && gfs == 0ull) return;
   const uint64_t n = commit_count(a);
-  if (s_fix[0]) resolve_duplicates(a, n);
-  if (s_fix[1]) resolve_barriers(a, n);
-  if (threadIdx.x == 0) {
-    ds->cm_conflicts = 0ull;
-    ds->cm_gf = 0ull;
+  if (dups) {
+    if (blockIdx.x == 0) {
+      resolve_duplicates(a, n);
+      if (gfs) resolve_barriers(a, n);
+    }
+    return;
   }
+  apply_barriers_grid(a, n);
 }
 
 // Make the lowest-index report of each Grain that was reported more than once
@@ -268,8 +366,45 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
   __syncthreads();
 }
 
-__device__ __forceinline__ void stat_add(unsigned long long* s, unsigned long long d) {
-  if (d) atomicAdd(s, d);   // d may be a negative delta in two's complement
+
+// A barrier seals every sibling of parent pp that is still open (a whole
+// warp, lane = its lane): Suppressed, barrier bit set, counted down at the
+// parent; the parent then completes (with a failed member it gathers
+// nothing).  Siblings sealed while WAITING or READY and while IN-FLIGHT are
+// added to *n_wait and *n_fly (shared counters of the CTA).
+__device__ void seal_open(const CommitArgs& a, uint32_t pp, int lane, unsigned long long* n_wait,
+                          unsigned long long* n_fly) {
+  const uint64_t c0 = a.offsets[pp], c1 = a.offsets[pp + 1];
+  uint32_t k_wait = 0, k_fly = 0;
+  for (uint64_t d = c0 + lane; d < c1; d += 32) {
+    const uint32_t ph = __ldcg(a.phase + d);
+    const uint32_t f = ph & 3u;
+    if (f == PH_SEALED) continue;
+    const uint32_t gen_d = (f == PH_WAITING) ? 0u : (ph >> 2);
+    a.phase[d] = ph_make(PH_SEALED, gen_d);
+    Rec* rc = a.rec + d;
+    const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
+    rc->len = 0u;
+    rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
+    if (f == PH_INFLIGHT) ++k_fly; else ++k_wait;
+  }
+  for (int sh = 16; sh > 0; sh >>= 1) {
+    k_wait += __shfl_down_sync(0xffffffffu, k_wait, sh);
+    k_fly += __shfl_down_sync(0xffffffffu, k_fly, sh);
+  }
+  if (lane == 0) {
+    const unsigned long long k = (unsigned long long)k_wait + k_fly;
+    if (k) {
+      const unsigned long long old = atomicAdd(a.pw + pp, (k << 32) - k);
+      if ((uint32_t)old == k) {   // the barrier completes the parent
+        a.pm[pp] = 0u;
+        atomicOr(a.bitmap + (pp >> 5), 1u << (pp & 31));
+      }
+    }
+    atomicAdd(n_wait, (unsigned long long)k_wait);
+    atomicAdd(n_fly, (unsigned long long)k_fly);
+  }
+  __syncwarp();
 }
 
 // GroupFailure barriers (Section 4.4) of this call, applied as if the
@@ -331,14 +466,15 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
   // 1: barrier index per parent from the final verdicts (a GroupFailure can
   //    have lost to an earlier duplicate of its Grain)
   if (fast) {
-    for (uint32_t i = threadIdx.x; i < nf; i += blockDim.x) a.gb[s_gp[i]] = GB_NONE;
+    for (uint32_t i = threadIdx.x; i < nf; i += blockDim.x) a.gb[s_gp[i]] = 0ull;
     __syncthreads();
     for (uint32_t i = threadIdx.x; i < nf; i += blockDim.x)
-      if (a.code[s_gr[i]] == V_ACCEPT) atomicMin(a.gb + s_gp[i], s_gr[i]);
+      if (a.code[s_gr[i]] == V_ACCEPT) atomicMax(a.gb + s_gp[i], gb_tag(a.seq, s_gr[i]));
     __syncthreads();
     for (uint32_t i = threadIdx.x; i < nf; i += blockDim.x) {
       const uint32_t r = s_gr[i], p = s_gp[i];
-      if (a.code[r] != V_ACCEPT || __ldcg(a.gb + p) != r) continue;
+      uint32_t br;
+      if (a.code[r] != V_ACCEPT || !gb_get(a, p, &br) || br != r) continue;
       const uint32_t k = atomicAdd(&s_ng, 1u);
       s_p[k] = p;
       s_b[k] = r;
@@ -348,13 +484,13 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
   } else {
     for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
       uint32_t p;
-      if (a.state[r] == ST_GROUP_FAILURE && parent_of(r, &p)) a.gb[p] = GB_NONE;
+      if (a.state[r] == ST_GROUP_FAILURE && parent_of(r, &p)) a.gb[p] = 0ull;
     }
     __syncthreads();
     for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
       uint32_t p;
       if (a.state[r] == ST_GROUP_FAILURE && a.code[r] == V_ACCEPT && parent_of(r, &p))
-        atomicMin(a.gb + p, (uint32_t)r);
+        atomicMax(a.gb + p, gb_tag(a.seq, (uint32_t)r));
     }
   }
   __syncthreads();
@@ -388,8 +524,8 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
       return true;
     }
     const uint32_t pp = a.rec[c].parent;
-    const uint32_t bb = __ldcg(a.gb + pp);
-    if (bb == GB_NONE) return false;
+    uint32_t bb;
+    if (!gb_get(a, pp, &bb)) return false;
     *p = pp;
     *b = bb;
     return true;
@@ -438,7 +574,7 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
   __syncthreads();
   // 3: duplicates after a barrier of a Grain whose accepted report (2) just
   //    turned into a barrier rejection (only if this call had duplicates)
-  const bool had_dups = ds->cm_conflicts != 0;
+  const bool had_dups = ds->cm_conflicts[fix_slot(a)] != 0;
   for (uint64_t base = (uint64_t)threadIdx.x * RB_GROUP; had_dups && base < n;
        base += (uint64_t)blockDim.x * RB_GROUP) {
     uint8_t cv[RB_GROUP];
@@ -461,63 +597,21 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
   //    barrier (the parent then completes; it has a failed member, so it
   //    gathers nothing)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  auto seal_open = [&](uint32_t pp) {
-    const uint64_t c0 = a.offsets[pp], c1 = a.offsets[pp + 1];
-    uint32_t k_wait = 0, k_fly = 0;
-    for (uint64_t d = c0 + lane; d < c1; d += 32) {
-      const uint32_t ph = __ldcg(a.phase + d);
-      const uint32_t f = ph & 3u;
-      if (f == PH_SEALED) continue;
-      const uint32_t gen_d = (f == PH_WAITING) ? 0u : (ph >> 2);
-      a.phase[d] = ph_make(PH_SEALED, gen_d);
-      Rec* rc = a.rec + d;
-      const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
-      rc->len = 0u;
-      rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
-      if (f == PH_INFLIGHT) ++k_fly; else ++k_wait;
-    }
-    for (int sh = 16; sh > 0; sh >>= 1) {
-      k_wait += __shfl_down_sync(0xffffffffu, k_wait, sh);
-      k_fly += __shfl_down_sync(0xffffffffu, k_fly, sh);
-    }
-    if (lane == 0) {
-      const unsigned long long k = (unsigned long long)k_wait + k_fly;
-      if (k) {
-        const unsigned long long old = atomicAdd(a.pw + pp, (k << 32) - k);
-        if ((uint32_t)old == k) {   // the barrier completes the parent
-          a.pm[pp] = 0u;
-          atomicOr(a.bitmap + (pp >> 5), 1u << (pp & 31));
-        }
-      }
-      atomicAdd(&s_d[5], (unsigned long long)k_wait);
-      atomicAdd(&s_d[6], (unsigned long long)k_fly);
-    }
-    __syncwarp();
-  };
   if (fast) {
-    for (uint32_t i = warp; i < ng; i += nw) seal_open(s_sp[i]);
+    for (uint32_t i = warp; i < ng; i += nw) seal_open(a, s_sp[i], lane, &s_d[5], &s_d[6]);
   } else {
     for (uint64_t base = (uint64_t)warp * 32; base < n; base += (uint64_t)nw * 32) {
       const uint64_t r = base + lane;
       uint32_t p = 0;
+      uint32_t br = 0;
       const bool trig = r < n && a.state[r] == ST_GROUP_FAILURE && a.code[r] == V_ACCEPT &&
-                        parent_of(r, &p) && __ldcg(a.gb + p) == (uint32_t)r;
+                        parent_of(r, &p) && gb_get(a, p, &br) && br == (uint32_t)r;
       unsigned m = __ballot_sync(0xffffffffu, trig);
       while (m) {
         const int src = __ffs(m) - 1;
         m &= m - 1;
-        seal_open(__shfl_sync(0xffffffffu, p, src));
+        seal_open(a, __shfl_sync(0xffffffffu, p, src), lane, &s_d[5], &s_d[6]);
       }
-    }
-  }
-  __syncthreads();
-  // 5: this call's barrier indices are spent
-  if (fast) {
-    for (uint32_t i = threadIdx.x; i < nf; i += blockDim.x) a.gb[s_gp[i]] = GB_NONE;
-  } else {
-    for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
-      uint32_t p;
-      if (a.state[r] == ST_GROUP_FAILURE && parent_of(r, &p)) a.gb[p] = GB_NONE;
     }
   }
   __syncthreads();
@@ -643,7 +737,11 @@ void launch_commit_scatter(const LaunchCfg& L, const CommitArgs& a) {
       (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(warps, CM_THREADS / 32),
                                                     (uint64_t)L.grid_commit));
   launch_k(L, K_COMMIT, commit_scatter_kernel, grid, CM_THREADS, 0, a);
-  launch_k(L, K_CFIX, commit_fix_kernel, 1, CM_THREADS, 0, a);
+  // the fix returns at once unless the scatter flagged the call; a grid for
+  // the barriers of calls without repeated reports
+  const int grid_fix = (int)std::max<uint64_t>(
+      1, std::min<uint64_t>(ceil_div(a.n_host, (uint64_t)FX_TILE), (uint64_t)L.grid_commit));
+  launch_k(L, K_CFIX, commit_fix_kernel, grid_fix, CM_THREADS, 0, a);
 }
 
 void launch_commit_finish(const LaunchCfg& L, const CommitArgs& a) {

@@ -140,6 +140,7 @@ struct ro_ctx {
   cudaStream_t fin_stream = nullptr;    // completion scans (commit_finish)
   cudaStream_t own_fin = nullptr;       // created for fin_stream, destroyed with the context
   uint32_t n_calls = 1;
+  uint32_t commit_seq = 0;              // commits issued on this context
   int num_sms = 0;
   LaunchCfg L{}, Lp{}, Lc{}, Lf{};
   DevScalars* ds = nullptr;
@@ -679,7 +680,7 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   RO_TRY(ensure(c, S.bitmap, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), "completion bitmaps"));
   RO_TRY(ensure(c, S.pm, P * sizeof(uint32_t), "parent member counts"));
   RO_TRY(ensure(c, S.wm, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), "word member counts"));
-  RO_TRY(ensure(c, S.gb, P * sizeof(uint32_t), "GroupFailure barriers"));
+  RO_TRY(ensure(c, S.gb, P * sizeof(unsigned long long), "GroupFailure barriers"));
   for (auto& l : S.lists) {
     RO_TRY(ensure(c, l.done, P * sizeof(uint32_t), "completed parents"));
     RO_TRY(ensure(c, l.status, P, "completed parents"));
@@ -696,7 +697,7 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   }
   cudaMemsetAsync(S.bitmap.p, 0, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), c->stream);
   cudaMemsetAsync(S.wm.p, 0, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), c->stream);
-  cudaMemsetAsync(S.gb.p, 0xFF, P * sizeof(uint32_t), c->stream);   // no barrier pending
+  cudaMemsetAsync(S.gb.p, 0, P * sizeof(unsigned long long), c->stream);   // no barrier (commit 0)
   ExpandFillArgs fa{};
   fa.offsets = (const uint64_t*)S.offsets.p;
   fa.P = P;
@@ -939,7 +940,8 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.bitmap = (uint32_t*)S.bitmap.p + bs * n_words;
   ca.pm = (uint32_t*)S.pm.p;
   ca.wm = (uint32_t*)S.wm.p + bs * n_words;
-  ca.gb = (uint32_t*)S.gb.p;
+  ca.gb = (unsigned long long*)S.gb.p;
+  ca.seq = ++c->commit_seq;   // from 1: 0 in the barrier table means no barrier
   if (d_code) {
     ca.code = d_code;
   } else {

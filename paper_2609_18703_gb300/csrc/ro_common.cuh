@@ -104,7 +104,11 @@ struct DevScalars {
   unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
   uint32_t rb_ticket, rb_err;
   // ro_gather_commit
-  unsigned long long cm_n, cm_conflicts, cm_n_done, cm_gf;
+  unsigned long long cm_n, cm_n_done;
+  // per commit, in two slots (commit sequence & 1): duplicate candidates and
+  // accepted GroupFailures the scatter saw; the next commit's scatter clears
+  // the slot after this one
+  unsigned long long cm_conflicts[2], cm_gf[2];
   // ro_retry
   unsigned long long rt_done;
   // ro_batch_ready_parent: the queue window after admission, the first short

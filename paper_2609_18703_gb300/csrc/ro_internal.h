@@ -222,8 +222,9 @@ struct CommitArgs {
   uint32_t* bitmap;
   uint32_t* pm;               // per parent: members to gather once complete (0: Suppressed)
   uint32_t* wm;               // per bitmap word: sum of pm of the parents completed in this call
-  uint32_t* gb;               // per parent: lowest accepted GroupFailure report of this call
-                              // (all ones: none); reset by commit_finish
+  unsigned long long* gb;     // per parent: (seq << 32) | ~r for the lowest accepted
+                              // GroupFailure report r of commit seq; older seq: none
+  uint32_t seq;               // this commit's sequence number in the context (from 1)
   uint8_t* code;              // user's or internal
   uint32_t* done_user;        // optional
   uint32_t* done_int;         // the list (a ring slot)
