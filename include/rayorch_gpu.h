@@ -313,6 +313,9 @@ ro_status ro_retry(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* d_ch
  *   With separate streams set, d_done_parents and d_n_done are written on
  *   the context's completion-scan stream (see the conventions above);
  *   ro_assemble orders itself after them.
+ * Capture: a captured commit keeps the context's commit number it was
+ * captured with; replay a captured sequence of commits on a fresh expansion
+ * (ro_expand clears the GroupFailure barrier table), as a new microbatch.
  */
 ro_status ro_gather_commit(ro_ctx* ctx, int32_t xid, uint64_t n, const uint64_t* d_n,
                            const uint32_t* d_child, const uint8_t* d_state,

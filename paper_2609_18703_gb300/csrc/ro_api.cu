@@ -941,7 +941,12 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.pm = (uint32_t*)S.pm.p;
   ca.wm = (uint32_t*)S.wm.p + bs * n_words;
   ca.gb = (unsigned long long*)S.gb.p;
-  ca.seq = ++c->commit_seq;   // from 1: 0 in the barrier table means no barrier
+  if (++c->commit_seq == 0) {   // wrapped: old tags could look current again
+    for (auto& sl : c->slots)
+      if (sl.gb.p) cudaMemsetAsync(sl.gb.p, 0, sl.gb.cap, c->stream);
+    c->commit_seq = 1;
+  }
+  ca.seq = c->commit_seq;   // from 1: 0 in the barrier table means no barrier
   if (d_code) {
     ca.code = d_code;
   } else {
