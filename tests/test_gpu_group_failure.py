@@ -134,6 +134,38 @@ def test_random_group_failures_many_calls(seed):
         ls.check_stats()
 
 
+@pytest.mark.parametrize("seed", range(3))
+def test_random_group_failures_without_repeats(seed):
+    """Calls with GroupFailures but no repeated report of a Grain take the
+    barrier pass spread over the grid: every reserved child reports once, in
+    random order, some as GroupFailure, some with a stale generation; plus
+    reports for children that were never dispatched."""
+    rng = np.random.default_rng(6000 + seed)
+    P = 20000
+    counts = rng.integers(0, 40, P).astype(np.uint32)
+    calls = rng.integers(0, 2, P).astype(np.uint8)
+    N = int(counts.sum())
+    arena = rng.integers(0, 256, N * 16 + 64).astype(np.uint8)
+    with Lockstep(n_calls=2) as ls:
+        x = ls.expand(counts, parent_call=calls)["xid"]
+        ad = _arena_dev(arena)
+        perm = rng.permutation(N).astype(np.uint32)
+        for w, cand in enumerate(np.array_split(perm, 5)):
+            got = np.concatenate([ls.batch_ready(x, c, cand, 64, flush=True)["batched"] for c in range(2)])
+            spare = np.setdiff1d(perm[: (w + 1) * N // 5], got)[: got.size // 8]   # not dispatched now
+            ch = np.concatenate([got, spare]).astype(np.uint32)
+            ch = ch[rng.permutation(ch.size)]
+            st = rng.choice([PRESENT] * 30 + [FAILED, GF], ch.size).astype(np.uint8)
+            gen = (rng.random(ch.size) < 0.02).astype(np.uint32) * 5   # a few stale
+            ln = rng.integers(0, 16, ch.size).astype(np.uint32)
+            cm = ls.commit(x, ch, st, ln, ch.astype(np.uint64) * 16, gen=gen, arena_bytes=arena.size)
+            ls.assemble(x, arena, ad, parents=None, n_parents=max(cm["n_done"], 1))
+        for c in range(2):
+            ls.batch_ready(x, c, None, 7, flush=True)
+        ls.check_stats()
+        assert ls.o.stats()["barrier_in_flight"] > 0
+
+
 def test_rq4_analog_streaming_docpage():
     """Section 6 RQ4 on a document->page level: readiness in waves, reports
     per wave in a seeded order, GroupFailure at ordinal 0 of the 99 largest
