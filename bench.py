@@ -43,7 +43,7 @@ K_ACOPY = 8
 # full-size bench is too large to capture with the full section set, so the
 # per-launch traffic reported here scales that ratio by the bytes a launch
 # assembles.
-COPY_TRAFFIC_RATIO = 0.987
+COPY_TRAFFIC_RATIO = 0.986
 
 
 def parse():
