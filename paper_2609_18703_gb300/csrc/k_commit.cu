@@ -13,17 +13,19 @@
 //                 That add also tells whether a member Failed or was
 //                 Suppressed, so the same thread records how many members the
 //                 parent will gather (0 if Suppressed) and adds it to its
-//                 bitmap word's total.  When the call carried two reports for
-//                 one Grain or a GroupFailure (rare), the last CTA to finish
-//                 orders them, so the result equals applying the reports one
-//                 by one in array order, before the call ends.
+//                 bitmap word's total.
+// commit_fix      after the scatter, on the same stream: when the call
+//                 carried two reports for one Grain or a GroupFailure (rare)
+//                 it orders the repeats and applies the barriers, so the
+//                 result equals applying the reports one by one in array
+//                 order; otherwise it returns at once.
 // commit_finish   turns the bitmap into the ascending list of completed
 //                 parents and their member bases (one single-pass scan over
 //                 bitmap words of (popcount, word total)) and clears it; the
 //                 list is what ro_assemble(NULL) plans and copies.  It reads
 //                 only the bitmap, the per-parent member counts and offsets,
-//                 so with several bitmaps (commits take them in turn) it runs on its
-//                 own stream while the next commit's scatter runs.
+//                 so with several bitmaps (commits take them in turn) it runs
+//                 on its own stream while the next commits' scatters run.
 #include <algorithm>
 
 #include "ro_internal.h"
@@ -134,7 +136,7 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
           v = V_BARRIER;   // suppressed by a sibling's GroupFailure in an earlier call
         } else {
           // SEALED at this generation: a duplicate, possibly of a report of
-          // this same call with a higher index (ordered by commit_finish)
+          // this same call with a higher index (ordered by commit_fix)
           v = V_DUP_CANDIDATE;
           atomicOr((unsigned long long*)&a.rec[c].w, (unsigned long long)W_CONFLICT_BIT);
         }
