@@ -52,9 +52,11 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="docpage", choices=["docpage", "skew"],
+    ap.add_argument("--workload", default="docpage", choices=["docpage", "skew", "streaming"],
                     help="docpage: the 1M-document config (default); skew: 10M parents, "
-                         "1,000 of them with 100k children, 32-byte results, one wave")
+                         "1,000 of them with 100k children, 32-byte results, one wave; "
+                         "streaming: 4 Calls, 50M children, 1,000 readiness waves")
+    ap.add_argument("--batch", type=int, default=256, help="streaming: batch size (32, 256, 2048)")
     ap.add_argument("--parents", type=int, default=1_000_000)
     ap.add_argument("--profile-all", action="store_true",
                     help="time every kernel (CUDA events) in the kernel-timing steps")
@@ -820,6 +822,164 @@ def run_rq4(args, local_rank):
     ro.ro_ctx_destroy(ctx)
 
 
+def streaming_plan(lv, B):
+    """Host-side schedule of the streaming pass: per readiness wave, the
+    candidates, and the children each Call's FIFO queue reserves in that wave
+    (whole batches of B, everything on the last wave), ordered by the
+    per-child key.  Only the workload's own draws are used: each Call's queue
+    is its children in readiness order, and wave w reserves the whole batches
+    its queue holds after admitting wave w's children."""
+    W = lv.ready_bounds.size - 1
+    call_of = lv.parent_call[np.repeat(np.arange(lv.n_parents), lv.counts.astype(np.int64))]
+    per_call = [lv.readiness[call_of[lv.readiness] == c] for c in range(lv.n_calls)]
+    wave_of = np.empty(lv.n_children, np.int64)
+    for w in range(W):
+        wave_of[lv.readiness[lv.ready_bounds[w]:lv.ready_bounds[w + 1]]] = w
+    # children of Call c admitted by the end of wave w (its queue is in readiness order)
+    ends = [np.searchsorted(wave_of[q], np.arange(W), side="right") for q in per_call]
+    reports = []
+    taken = [0] * lv.n_calls
+    for w in range(W):
+        got = []
+        for c in range(lv.n_calls):
+            q, admitted = per_call[c], int(ends[c][w])
+            upto = admitted if w == W - 1 else (admitted // B) * B
+            got.append(q[taken[c]:upto])
+            taken[c] = upto
+        g = np.concatenate(got)
+        reports.append(g[np.argsort(lv.key[g], kind="stable")].astype(np.uint32))
+    return reports
+
+
+def run_streaming(args, local_rank):
+    """The streaming multi-Call configuration (4 Calls, 50M children of 1 KB,
+    2 % FAILED, 1,000 readiness waves): per wave, each Call admits the wave's
+    ready children into its FIFO queue and reserves whole batches of B; the
+    reserved children's results arrive in that wave (ordered by a per-child
+    key) and are committed; the parents they complete are assembled.  The
+    wave loop is captured once in a CUDA graph and replayed; every input is
+    resident.  One JSON line: children/s over the whole pass."""
+    import torch
+    import __graft_entry__
+    import paper_2609_18703_gb300 as ro
+    from workload import streaming
+    from workload.device import fill_payload
+
+    torch.cuda.set_device(local_rank)
+    __graft_entry__.build()
+    hbm_peak, peak_kind = peaks()
+    B = args.batch
+    lv = streaming(batch_size=B).top
+    N, P, W = lv.n_children, lv.n_parents, lv.ready_bounds.size - 1
+    reports = streaming_plan(lv, B)
+    assert sum(r.size for r in reports) == N
+    dev = torch.device("cuda", local_rank)
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
+    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).to(dev)
+    i64 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int64)).to(dev)
+    u8 = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    counts = i32(lv.counts)
+    calls = u8(lv.parent_call)
+    cand = i32(lv.readiness)
+    rep_all = np.concatenate(reports)
+    rb = np.concatenate([[0], np.cumsum([r.size for r in reports])]).astype(np.int64)
+    r_child, r_state = i32(rep_all), u8(lv.state[rep_all])
+    r_len, r_off = i32(lv.length[rep_all]), i64(lv.arena_off[rep_all])
+    arena = torch.empty(max(int(lv.arena_bytes), 16), dtype=torch.uint8, device=dev)
+    fill_payload(arena, i64(lv.arena_off), i32(lv.length), lv.payload_seed, stream)
+    out_cap = int(lv.arena_bytes) + 64
+    out = torch.empty(out_cap, dtype=torch.uint8, device=dev)
+    offsets = torch.empty(P + 1, dtype=torch.int64, device=dev)
+    cp = torch.empty(N, dtype=torch.int32, device=dev)
+    co = torch.empty(N, dtype=torch.int32, device=dev)
+    batched = torch.empty(N + B, dtype=torch.int32, device=dev)
+    status = torch.empty(P, dtype=torch.uint8, device=dev)
+    out_off = torch.empty(P + 1, dtype=torch.int64, device=dev)
+    out_len = torch.empty(P, dtype=torch.int32, device=dev)
+    cursor = torch.zeros(1, dtype=torch.int64, device=dev)
+    torch.cuda.synchronize()
+    ctx = ro.ro_ctx_create(local_rank, stream, lv.n_calls)
+    ro.ro_ctx_set_streams(ctx, torch.cuda.Stream(), torch.cuda.Stream())
+    L = ro.load()
+
+    def expand():
+        ro.ro_ctx_reset(ctx)
+        st, n, _, xid = ro.ro_expand(ctx, -1, counts, P, calls, offsets, cp, co, N, None)
+        if st != 0 or n != N:
+            raise RuntimeError(f"ro_expand: {st} {ro.ro_last_error(ctx)}")
+        return xid
+
+    def waves(xid):
+        bad = 0
+        cursor.zero_()
+        for w in range(W):
+            c0, c1 = int(lv.ready_bounds[w]), int(lv.ready_bounds[w + 1])
+            for c in range(lv.n_calls):
+                bad |= L.ro_batch_ready(ctx, xid, c, cand.data_ptr() + 4 * c0, c1 - c0, B,
+                                        int(w == W - 1), batched.data_ptr(), N + B, None, None, None)
+            s, e = int(rb[w]), int(rb[w + 1])
+            bad |= L.ro_gather_commit(ctx, xid, e - s, None, r_child.data_ptr() + 4 * s,
+                                      r_state.data_ptr() + s, r_len.data_ptr() + 4 * s,
+                                      r_off.data_ptr() + 8 * s, None, int(lv.arena_bytes), None,
+                                      None, 0, None, None)
+            bad |= L.ro_assemble(ctx, xid, arena.data_ptr(), int(lv.arena_bytes), None, P, None,
+                                 status.data_ptr(), out_off.data_ptr(), out_len.data_ptr(),
+                                 out.data_ptr(), out_cap, cursor.data_ptr(), None, None)
+        bad |= L.ro_ctx_join(ctx)
+        if bad:
+            raise RuntimeError(f"wave loop: {bad}: {ro.ro_last_error(ctx)}")
+
+    for _ in range(max(1, args.warmup)):
+        waves(expand())
+    stream.synchronize()
+    if ro.ro_ctx_sync(ctx) != 0:
+        raise RuntimeError(ro.ro_last_error(ctx))
+    stats = ro.ro_ctx_stats(ctx)
+    xid = expand()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        waves(xid)
+    for _ in range(args.warmup):
+        expand()
+        g.replay()
+    torch.cuda.synchronize()
+    steps = max(1, args.steps)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    ms = []
+    for k in range(steps):
+        expand()   # synchronises (host counts); timed per pass below, expansion included
+        ev[k].record(stream)
+        g.replay()
+        ev[k + 1].record(stream)
+        torch.cuda.synchronize()
+        ms.append(ev[k].elapsed_time(ev[k + 1]))
+    clk = clocks.stop()
+    if ro.ro_ctx_sync(ctx) != 0:
+        raise RuntimeError(ro.ro_last_error(ctx))
+    S = int(cursor.item())
+    ms.sort()
+    med = ms[len(ms) // 2]
+    line = {
+        "metric": "children/s, streaming multi-Call pass (admission, batching, commit, assembly)",
+        "value": round(N / (med * 1e-3), 1), "unit": "children/s", "n_gpus": 1, "steps": steps,
+        "warmup": args.warmup, "ms_per_step_median": round(med, 3), "ms_per_step_best": round(ms[0], 3),
+        "higher_is_better": True, "dtype": "u8/u32/u64", "data": "synthetic",
+        "config": {"workload": f"streaming: {lv.n_calls} Calls, {P} parents, {N} children of 1 KB, "
+                               f"2 % FAILED, {W} readiness waves, batch {B}",
+                   "assembled_bytes": S, "kernels_per_wave": 4 * 2 + 3 + 2,
+                   "timed": "the captured wave loop (expansion outside)"},
+        "payload_gbs": round(2.0 * S / (med * 1e-3) / 1e9, 1),
+        "payload_frac_of_hbm": round(2.0 * S / (med * 1e-3) / 1e9 / hbm_peak, 4),
+        "accepted_per_pass": stats["accepted"] // max(1, args.warmup),
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    ro.ro_ctx_destroy(ctx)
+
+
 def run_retry_bench(args, local_rank):
     """Throughput of ro_retry (Section 4.4, Eq. 2's retry edge): every child of
     the document->page level is dispatched, then a seeded random 1/16 of them
@@ -888,6 +1048,9 @@ def main():
         return
     if args.rq4:
         run_rq4(args, int(os.environ.get("LOCAL_RANK", "0")))
+        return
+    if args.workload == "streaming" and args.impl != "reference":
+        run_streaming(args, int(os.environ.get("LOCAL_RANK", "0")))
         return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
