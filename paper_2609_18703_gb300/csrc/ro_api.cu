@@ -154,6 +154,18 @@ struct ro_ctx {
   DevBuf pb_key[2], pb_val[2], pb_child, pb_hist, pb_dtot, pb_first, pb_endp, pb_hsz, pb_left,
       pb_hoff, pb_rem;
   Ev fork, x_planned, join_plan, join_copy, fin_fork, fin_join, fin_plan;
+  // Caller memory written by the copies issued since the context's stream
+  // last waited for the copy stream: a later call's planning (another
+  // stream) may run while they do, so planning that writes any of it waits
+  // for them (copy_done follows the latest copy).  Past MAX_SPANS ranges
+  // every such planning waits.
+  struct Span {
+    uintptr_t lo, hi;
+  };
+  static constexpr size_t MAX_SPANS = 4096;
+  std::vector<Span> copy_spans;
+  bool copy_spans_full = false;
+  Ev copy_done;
   Profiler prof;
   ro_status sticky = RO_OK;
   std::string err;
@@ -288,6 +300,9 @@ ro_status join(ro_ctx* c) {
   RO_TRY(order(c, c->fin_join, c->fin_stream, c->stream));
   RO_TRY(order(c, c->join_plan, c->plan_stream, c->stream));
   if (c->copy_stream != c->plan_stream) RO_TRY(order(c, c->join_copy, c->copy_stream, c->stream));
+  // planning forks from the context's stream: it now follows every copy
+  c->copy_spans.clear();
+  c->copy_spans_full = false;
   return RO_OK;
 }
 
@@ -516,7 +531,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
                     &c->pb_hoff, &c->pb_rem})
     free_buf(*b);
   free_ev(c->fork); free_ev(c->x_planned); free_ev(c->join_plan); free_ev(c->join_copy);
-  free_ev(c->fin_fork); free_ev(c->fin_join); free_ev(c->fin_plan);
+  free_ev(c->fin_fork); free_ev(c->fin_join); free_ev(c->fin_plan); free_ev(c->copy_done);
   if (c->own_fin) cudaStreamDestroy(c->own_fin);
   for (cudaEvent_t e : c->prof.pool) cudaEventDestroy(e);
   cudaFree(c->ds);
@@ -1134,6 +1149,30 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   RO_TRY(order(c, c->fork, c->stream, c->plan_stream));
   RO_TRY(order(c, c->fin_plan, c->fin_stream, c->plan_stream));   // the commit's completion list
   RO_TRY(ev_wait(c, PS.freed, c->plan_stream));
+  if (c->plan_stream != c->copy_stream) {
+    // caller memory planning writes (list structure; a caller's list's
+    // outcomes) against what copies still in flight write
+    ro_ctx::Span pw[5];
+    int npw = 0;
+    auto span = [](const void* p, uint64_t bytes) {
+      return ro_ctx::Span{(uintptr_t)p, (uintptr_t)p + (uintptr_t)bytes};
+    };
+    if (d_parents) pw[npw++] = span(d_status, n_parents);
+    if (eo) {
+      pw[npw++] = span(eo->base, (n_parents + 1) * sizeof(uint64_t));
+      pw[npw++] = span(eo->state, eo->cap);
+      pw[npw++] = span(eo->off, eo->cap * sizeof(uint64_t));
+      pw[npw++] = span(eo->len, eo->cap * sizeof(uint32_t));
+    }
+    bool meet = npw > 0 && c->copy_spans_full;
+    for (int i = 0; i < npw && !meet; ++i)
+      for (const auto& b : c->copy_spans)
+        if (pw[i].lo < pw[i].hi && pw[i].lo < b.hi && b.lo < pw[i].hi) {
+          meet = true;
+          break;
+        }
+    if (meet) RO_TRY(ev_wait(c, c->copy_done, c->plan_stream));
+  }
   launch_assemble_plan(c->Lp, aa);
   RO_TRY(check_launch(c, "assemble (plan)"));
   if (!LS && c->plan_stream != c->stream) {
@@ -1144,7 +1183,24 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   RO_TRY(order(c, PS.ready, c->plan_stream, c->copy_stream));
   launch_assemble_copy(c->Lc, aa);
   RO_TRY(check_launch(c, "assemble (copy)"));
-  if (c->copy_stream != c->plan_stream) RO_TRY(ev_record(c, PS.freed, c->copy_stream));
+  if (c->copy_stream != c->plan_stream) {
+    RO_TRY(ev_record(c, PS.freed, c->copy_stream));
+    RO_TRY(ev_record(c, c->copy_done, c->copy_stream));
+    // what this copy writes of the caller's memory (the bytes of d_out are
+    // written by copies only)
+    auto add = [&](const void* p, uint64_t bytes) {
+      if (!p || !bytes) return;
+      if (c->copy_spans.size() >= ro_ctx::MAX_SPANS) {
+        c->copy_spans_full = true;
+        return;
+      }
+      c->copy_spans.push_back({(uintptr_t)p, (uintptr_t)p + (uintptr_t)bytes});
+    };
+    if (!d_parents) add(d_status, n_parents);
+    add(d_out_off, (n_parents + 1) * sizeof(uint64_t));
+    add(d_out_len, n_parents * sizeof(uint32_t));
+    if (eo) add(eo->off, eo->cap * sizeof(uint64_t));
+  }
   // the copy reads the list's outcomes: the slot is free once it is done
   if (LS && c->copy_stream != c->stream) RO_TRY(ev_record(c, LS->freed, c->copy_stream));
   x->assembles += 1;

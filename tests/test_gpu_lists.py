@@ -19,7 +19,8 @@ def _built():
     __graft_entry__.build()
 
 
-from tests.lockstep import Lockstep, dev  # noqa: E402
+import paper_2609_18703_gb300 as ro  # noqa: E402
+from tests.lockstep import Lockstep, dev, empty, host  # noqa: E402
 from tests.pipeline import host_arena  # noqa: E402
 from workload import DROPPED, FAILED, PRESENT, SUPPRESSED, docpage, tiny  # noqa: E402
 
@@ -89,3 +90,53 @@ def test_present_empty_list():
         assert list(r["parent_status"]) == [PRESENT, PRESENT, SUPPRESSED, PRESENT]
         assert list(r["elem_base"]) == [0, 3, 5, 5, 8]
         ls.check_stats()
+
+
+@pytest.mark.parametrize("second_list", [True, False])
+def test_back_to_back_calls_reusing_outputs_on_streams(second_list):
+    """Two list assemblies issued without waiting, on a context with
+    planning and copy streams, into the same caller arrays: the second
+    call's planning writes the list structure (and a caller list's
+    outcomes) while the first call's copy may still be writing the same
+    arrays.  The arrays end with the second call's values, as in stream
+    order."""
+    lv = docpage(parents=4000, waves=1).top
+    a = host_arena(lv)
+    ad = _arena_dev(a)
+    rng = np.random.default_rng(77)
+    with Lockstep(streams=True) as ls:
+        x = ls.expand(lv.counts)["xid"]
+        ls.batch_ready(x, 0, None, lv.batch_size, flush=True)
+        ch, st, ln, of = lv.reports(lv.wave(0))
+        cm = ls.commit(x, ch, st, ln, of, arena_bytes=lv.arena_bytes)
+        P, N = lv.n_parents, ls.N[x]
+        cap = int(lv.arena_bytes) + 64
+        first = np.arange(P, dtype=np.uint32)[::-1].copy()   # every parent: a long copy
+        second = rng.choice(P, 300, replace=False).astype(np.uint32) if second_list else None
+        n2 = second.size if second_list else max(cm["n_done"], 1)
+        r2 = ls.o.assemble_list(x, a, parents=second, n_parents=n2, out_cap=cap, cursor=None,
+                                elem_cap=N, check=False)
+        assert r2["status"] == 0
+        d_status, d_off, d_len = empty(P, np.uint8), empty(P + 1, np.uint64), empty(P, np.uint32)
+        d_eb = empty(P + 1, np.uint64)
+        d_es, d_eo, d_el = empty(N, np.uint8), empty(N, np.uint64), empty(N, np.uint32)
+        out = torch.zeros(cap, dtype=torch.uint8, device="cuda")
+        keep = []
+        for par, n in ((first, P), (second, n2)):
+            d_par = None if par is None else dev(par, np.uint32)
+            keep.append(d_par)
+            st, _, _ = ro.ro_assemble_list(ls.ctx, x, ad, ad.numel(), d_par, n, None, d_status, d_off,
+                                           d_len, out, cap, None, None, d_eb, d_es, d_eo, d_el, N,
+                                           None, want_host=False)
+            assert st == ro.RO_OK, ro.ro_last_error(ls.ctx)
+        assert ro.ro_ctx_join(ls.ctx) == ro.RO_OK
+        torch.cuda.synchronize()
+        k, m, ob = r2["n_assembled"], r2["n_elems"], r2["out_bytes"]
+        assert np.array_equal(host(d_status, np.uint8, k), r2["parent_status"])
+        assert np.array_equal(host(d_off, np.uint64, k + 1), r2["out_off"])
+        assert np.array_equal(host(d_len, np.uint32, k), r2["out_len"])
+        assert np.array_equal(host(d_eb, np.uint64, k + 1), r2["elem_base"])
+        assert np.array_equal(host(d_es, np.uint8, m), r2["elem_state"])
+        assert np.array_equal(host(d_eo, np.uint64, m), r2["elem_off"])
+        assert np.array_equal(host(d_el, np.uint32, m), r2["elem_len"])
+        assert np.array_equal(out[:ob].cpu().numpy(), r2["out"][:ob])
