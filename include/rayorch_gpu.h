@@ -364,6 +364,9 @@ ro_status ro_gather_commit(ro_ctx* ctx, int32_t xid, uint64_t n, const uint64_t*
  * (see ro_ctx_set_streams); the outputs (d_status, d_out_off, d_out_len,
  * d_out, the cursor, d_out_bytes) are written there.  Read them after
  * ro_ctx_join in stream order, or after any synchronising call.
+ * Consecutive calls may pass the same output arrays: their writes land in
+ * call order (a call whose planning writes caller memory that an earlier
+ * call's copy is still writing waits for that copy).
  */
 ro_status ro_assemble(ro_ctx* ctx, int32_t xid, const uint8_t* d_arena, uint64_t arena_bytes,
                       const uint32_t* d_parents, uint64_t n_parents, const uint64_t* d_n_parents,
