@@ -1,10 +1,14 @@
-"""The 1,000,000-document configuration at full size (16.4M children,
+"""Full-size configurations.  The 1,000,000-document configuration (16.4M children,
 38.8 GB arena, 256 arrival waves, batch 256), in the launch configuration
 bench.py times, against the oracle on every output: lineage arrays, the
 reserved batches, every wave's verdicts, completed-parent list, statuses,
 offsets, lengths and all ~12 GB of assembled bytes.  The CUDA-graph replay of
 the wave loop (what the benchmark runs) is then checked byte for byte
-against the eager run.  Needs ~70 GB of host memory and ~60 GB on the GPU."""
+against the eager run.  Needs ~70 GB of host memory and ~60 GB on the GPU.
+The extreme-skew (110M children), video -> clip -> frame (100,000 videos,
+nested) and streaming (four Calls, 50M children, 1,000 readiness waves)
+configurations run at full size too, each compared with the oracle call by
+call."""
 import numpy as np
 import pytest
 
@@ -160,3 +164,106 @@ def test_docpage_full_size(setup):
             assert torch.equal(out_d[:total], eager)
     assert ro.ro_ctx_sync(ctx) == 0
     ro.ro_ctx_destroy(ctx)
+
+
+def _arena_dev(a):
+    from tests.lockstep import dev
+    return dev(a if a.size else np.zeros(1, np.uint8), np.uint8)
+
+
+def test_skew_full_size():
+    """The extreme-skew configuration at full size: 10,000,000 parents, 1,000
+    of them with 100,000 children (109,999,000 children of 32 bytes), one
+    arrival wave, batch 256: lineage arrays, reserved batches, every
+    verdict, the completed list, statuses, offsets, lengths and all 3.5 GB
+    of assembled bytes equal the oracle's."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from tests.lockstep import Lockstep
+    from tests.pipeline import host_arena
+    from workload import skew
+    lv = skew().top
+    assert lv.n_children == 109_999_000
+    a = host_arena(lv)
+    with Lockstep() as ls:
+        x = ls.expand(lv.counts)["xid"]
+        ls.batch_ready(x, 0, None, lv.batch_size, flush=True)
+        ch, st, ln, of = lv.reports(lv.wave(0))
+        cm = ls.commit(x, ch, st, ln, of, arena_bytes=lv.arena_bytes)
+        assert cm["n_done"] == lv.n_parents
+        r = ls.assemble(x, a, _arena_dev(a), parents=None, n_parents=cm["n_done"])
+        assert r["out_bytes"] == lv.arena_bytes   # no failures: every byte is assembled
+        ls.check_stats()
+
+
+def test_video_nested_full_size():
+    """The video -> clip -> frame configuration at full size: 100,000 videos,
+    their clips and frames (512-byte records), frames gathered into clips,
+    the clips' assembled results committed as the reports of the videos'
+    expansion and gathered again; every output of both levels equal to the
+    oracle's."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from tests.lockstep import Lockstep
+    from tests.pipeline import host_arena
+    from workload import video
+    top, leaf = video().levels
+    assert top.n_parents == 100_000
+    a = host_arena(leaf)
+    with Lockstep() as ls:
+        x0 = ls.expand(top.counts)["xid"]
+        ls.batch_ready(x0, 0, None, top.batch_size, flush=True)
+        x1 = ls.expand(leaf.counts, parent_xid=x0)["xid"]
+        ls.batch_ready(x1, 0, None, leaf.batch_size, flush=True)
+        ch, st, ln, of = leaf.reports(leaf.wave(0))
+        cm1 = ls.commit(x1, ch, st, ln, of, arena_bytes=leaf.arena_bytes)
+        assert cm1["n_done"] == leaf.n_parents
+        a1 = ls.assemble(x1, a, _arena_dev(a), parents=None, n_parents=cm1["n_done"])
+        del a
+        r1 = a1["r"]
+        level1 = a1["out"][:a1["out_bytes"]].cpu().numpy()
+        cm0 = ls.commit(x0, cm1["done"], r1["parent_status"], r1["out_len"], r1["out_off"][:-1],
+                        arena_bytes=a1["out_bytes"])
+        assert cm0["n_done"] == top.n_parents
+        ls.assemble(x0, level1, _arena_dev(level1), parents=None, n_parents=cm0["n_done"])
+        ls.check_stats()
+
+
+def test_streaming_full_size():
+    """The streaming configuration at full size and the benchmark's default
+    batch: four Calls, 50,000,050 children of 1 KB, 1,000 readiness waves;
+    per wave every Call admits the wave's ready children and reserves whole
+    batches (the last wave flushes), the reserved children's results are
+    committed in their key order and the completed parents assembled.  Every
+    Call's reservation, every verdict, completed list, status, offset and
+    length equal the oracle's; the assembled bytes of one wave in 25 and of
+    the last wave are compared in full, and the total byte count of all."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from tests.lockstep import Lockstep
+    from tests.pipeline import host_arena
+    from workload import streaming
+    lv = streaming().top
+    assert lv.n_children == 50_000_050
+    a = host_arena(lv)
+    ad = _arena_dev(a)
+    B = lv.batch_size
+    total = 0
+    with Lockstep(n_calls=4) as ls:
+        x = ls.expand(lv.counts, parent_call=lv.parent_call)["xid"]
+        n_ready = lv.ready_bounds.size - 1
+        for w in range(n_ready):
+            cand = lv.readiness[lv.ready_bounds[w]:lv.ready_bounds[w + 1]]
+            last = w == n_ready - 1
+            reserved = [ls.batch_ready(x, c, cand, B, flush=last)["batched"] for c in range(4)]
+            got = np.concatenate(reserved)
+            got = got[np.argsort(lv.key[got], kind="stable")]
+            ch, st, ln, of = lv.reports(got)
+            cm = ls.commit(x, ch, st, ln, of, arena_bytes=lv.arena_bytes)
+            # the oracle assembles (and the test compares) bytes only when given the arena
+            r = ls.assemble(x, a if (w % 25 == 0 or last) else None, ad, parents=None,
+                            n_parents=max(cm["n_done"], 1))
+            total += r["out_bytes"]
+        ls.check_stats()
+        assert ls.o.stats()["ready_bad_candidates"] == 0
+    assert total > 0
