@@ -52,6 +52,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--one-call-stream", action="store_true",
+                    help="streaming: every Call admits on the context's stream (no Call streams)")
     ap.add_argument("--workload", default="docpage", choices=["docpage", "skew", "streaming"],
                     help="docpage: the 1M-document config (default); skew: 10M parents, "
                          "1,000 of them with 100k children, 32-byte results, one wave; "
@@ -893,7 +895,8 @@ def run_streaming(args, local_rank):
     offsets = torch.empty(P + 1, dtype=torch.int64, device=dev)
     cp = torch.empty(N, dtype=torch.int32, device=dev)
     co = torch.empty(N, dtype=torch.int32, device=dev)
-    batched = torch.empty(N + B, dtype=torch.int32, device=dev)
+    # each Call admits on a stream of its own, into a batch list of its own
+    batched = [torch.empty(N + B, dtype=torch.int32, device=dev) for _ in range(lv.n_calls)]
     status = torch.empty(P, dtype=torch.uint8, device=dev)
     out_off = torch.empty(P + 1, dtype=torch.int64, device=dev)
     out_len = torch.empty(P, dtype=torch.int32, device=dev)
@@ -901,6 +904,8 @@ def run_streaming(args, local_rank):
     torch.cuda.synchronize()
     ctx = ro.ro_ctx_create(local_rank, stream, lv.n_calls)
     ro.ro_ctx_set_streams(ctx, torch.cuda.Stream(), torch.cuda.Stream())
+    call_streams = [torch.cuda.Stream() for _ in range(lv.n_calls)] if not args.one_call_stream else []
+    ro.ro_ctx_set_call_streams(ctx, call_streams)
     L = ro.load()
 
     def expand():
@@ -917,7 +922,8 @@ def run_streaming(args, local_rank):
             c0, c1 = int(lv.ready_bounds[w]), int(lv.ready_bounds[w + 1])
             for c in range(lv.n_calls):
                 bad |= L.ro_batch_ready(ctx, xid, c, cand.data_ptr() + 4 * c0, c1 - c0, B,
-                                        int(w == W - 1), batched.data_ptr(), N + B, None, None, None)
+                                        int(w == W - 1), batched[c].data_ptr(), N + B, None, None,
+                                        None)
             s, e = int(rb[w]), int(rb[w + 1])
             bad |= L.ro_gather_commit(ctx, xid, e - s, None, r_child.data_ptr() + 4 * s,
                                       r_state.data_ptr() + s, r_len.data_ptr() + 4 * s,
@@ -970,6 +976,8 @@ def run_streaming(args, local_rank):
         "config": {"workload": f"streaming: {lv.n_calls} Calls, {P} parents, {N} children of 1 KB, "
                                f"2 % FAILED, {W} readiness waves, batch {B}",
                    "assembled_bytes": S, "kernels_per_wave": 4 * 2 + 3 + 2,
+                   "admissions": "on the context's stream" if args.one_call_stream
+                                 else "one stream per Call",
                    "timed": "the captured wave loop (expansion outside)"},
         "payload_gbs": round(2.0 * S / (med * 1e-3) / 1e9, 1),
         "payload_frac_of_hbm": round(2.0 * S / (med * 1e-3) / 1e9 / hbm_peak, 4),

@@ -24,12 +24,14 @@
  *   library never keeps a caller pointer beyond the call (except the arena,
  *   see ro_gather_commit).  A context owns its internal lineage state
  *   (phase words, result slots, parent counters, queues, scratch).
- * - Work is issued on the context's stream, in call order, except assembly
- *   and completion lists: ro_assemble plans on the context's plan stream and
- *   copies on its copy stream, and with separate streams set
+ * - Work is issued on the context's stream, in call order, except assembly,
+ *   completion lists and admissions: ro_assemble plans on the context's plan
+ *   stream and copies on its copy stream, with separate streams set
  *   (ro_ctx_set_streams) ro_gather_commit builds its completed-parent list
- *   on a stream the context owns.  Each assembly is ordered after all work
- *   the caller issued on the context before it; the caller's ro_assemble
+ *   on a stream the context owns, and with Call streams set
+ *   (ro_ctx_set_call_streams) ro_batch_ready runs on its Call's stream.
+ *   Each assembly is ordered after all work the caller issued on the
+ *   context before it; the caller's ro_assemble
  *   outputs and ro_gather_commit's d_done_parents / d_n_done are complete
  *   once ro_ctx_join has made the context's stream wait for the others (or
  *   once any call synchronises).  Calls return without waiting for the
@@ -141,8 +143,27 @@ ro_status ro_ctx_sync(ro_ctx* ctx);
  * context's stream first waits for the old streams.  The caller keeps the streams alive until ro_ctx_destroy
  * or the next ro_ctx_set_streams. */
 ro_status ro_ctx_set_streams(ro_ctx* ctx, void* plan_stream, void* copy_stream);
+/* Streams for the Calls' admissions (Section 4.3: each Call has its own
+ * Ready Queue, and the queues are independent).  streams[k] (a cudaStream_t
+ * on the context's device, or NULL for the context's stream) runs
+ * ro_batch_ready for Call k, k < n; Calls from n on use the context's
+ * stream.  An admission on a Call's stream follows everything issued on
+ * the context's stream before it, so the admissions of several Calls
+ * issued one after another run at the same time; the context's stream
+ * waits for them before its next launch (any other call that works on the
+ * expansion: ro_expand, ro_gather_commit, ro_retry, ro_batch_ready_parent,
+ * ro_assemble) and in ro_ctx_join.  Each Call's outputs (d_batched,
+ * d_n_batched) are written on its stream: give Calls that run at the same
+ * time outputs of their own.  ro_batch_ready_parent always runs on the
+ * context's stream.  The context's stream first waits for the old streams;
+ * the caller keeps the streams alive until ro_ctx_destroy or the next call
+ * of this function.
+ * Errors: RO_E_INVAL if n exceeds the context's Calls or streams is NULL
+ * with n > 0. */
+ro_status ro_ctx_set_call_streams(ro_ctx* ctx, void* const* streams, uint32_t n);
 /* Make the context's stream wait (on the GPU) for all work issued so far on
- * the plan and copy streams and the completion-scan stream.  Call it before reading assembly outputs in
+ * the plan and copy streams, the completion-scan stream and the Calls'
+ * streams.  Call it before reading assembly outputs in
  * stream order, before starting a capture of the context's stream, and
  * before ending one (a captured assembly forks onto the other streams, and a
  * capture must join them back).  Nothing waits on the host. */

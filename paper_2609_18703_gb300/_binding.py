@@ -30,7 +30,7 @@ STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFL
                 4: "RO_E_STATE", 5: "RO_E_OOM", 6: "RO_E_CUDA", 7: "RO_E_TIMEOUT"}
 
 EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro_ctx_stats",
-           "ro_ctx_set_streams", "ro_ctx_join", "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
+           "ro_ctx_set_streams", "ro_ctx_set_call_streams", "ro_ctx_join", "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
            "ro_retry", "ro_batch_ready_parent", "ro_gather_commit", "ro_assemble", "ro_assemble_list", "ro_filter_reports",
            "ro_expand_noalloc")
 
@@ -79,6 +79,7 @@ def load(path: Optional[str] = None):
     L.ro_ctx_sync.argtypes = [_vp]
     L.ro_ctx_stats.argtypes = [_vp, C.POINTER(_Stats)]
     L.ro_ctx_set_streams.argtypes = [_vp, _vp, _vp]
+    L.ro_ctx_set_call_streams.argtypes = [_vp, C.POINTER(_vp), _u32]
     L.ro_ctx_join.argtypes = [_vp]
     L.ro_last_error.argtypes = [_vp]
     L.ro_last_error.restype = C.c_char_p
@@ -162,8 +163,17 @@ def ro_ctx_set_streams(ctx, plan_stream=None, copy_stream=None) -> int:
     return _check("ro_ctx_set_streams", st, ctx)
 
 
+def ro_ctx_set_call_streams(ctx, streams) -> int:
+    """Streams for the Calls' admissions: streams[k] (torch.cuda.Stream, raw
+    handle or None) runs ro_batch_ready for Call k."""
+    handles = (_vp * max(len(streams), 1))(*[_stream_handle(s) for s in streams])
+    st = load().ro_ctx_set_call_streams(ctx, handles, len(streams))
+    return _check("ro_ctx_set_call_streams", st, ctx)
+
+
 def ro_ctx_join(ctx) -> int:
-    """The context's stream waits (on the GPU) for the plan and copy streams."""
+    """The context's stream waits (on the GPU) for the plan, copy, completion
+    scan and Call streams."""
     return _check("ro_ctx_join", load().ro_ctx_join(ctx), ctx)
 
 

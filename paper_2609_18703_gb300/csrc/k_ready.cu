@@ -26,6 +26,14 @@ namespace ro {
 __device__ __forceinline__ bool call_ok(const ReadyArgs& a, uint64_t c) {
   return !a.check_call || w_call(a.rec[c].w) == a.call;
 }
+// A phase word holding claim i (a WAITING child whose first occurrence in
+// the candidate list is position i) was claimed by this call.  When other
+// Calls' admissions may run at the same time (Call streams), possibly with
+// the same candidate list, that holds only for this Call's children; one
+// at a time, every other Call's claims are settled before this call starts.
+__device__ __forceinline__ bool claimed_here(const ReadyArgs& a, uint64_t c, uint32_t w, uint64_t i) {
+  return w == ((uint32_t)i << 2) && (!a.calls_concurrent || call_ok(a, c));
+}
 
 __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
   wait_predecessor();
@@ -33,6 +41,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
   __shared__ unsigned long long s_scan[33];
   __shared__ uint32_t s_last;
   DevScalars* ds = a.ds;
+  ReadyScalars* rs = a.rs;
   unsigned long long kept = 0, bad = 0;
   const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
   for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < a.n_cand; i += stride) {
@@ -75,9 +84,9 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
       k += s_red[0][j];
       b += s_red[1][j];
     }
-    if (k) atomicAdd(&ds->rb_kept, k);
-    if (b) atomicAdd(&ds->rb_bad, b);
-    s_last = ticket(&ds->rb_ticket) == gridDim.x - 1;
+    if (k) atomicAdd(&rs->rb_kept, k);
+    if (b) atomicAdd(&rs->rb_bad, b);
+    s_last = ticket(&rs->rb_ticket) == gridDim.x - 1;
   }
   __syncthreads();
   if (!s_last) return;
@@ -111,11 +120,11 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
   if (threadIdx.x == 0) {
     {
       // plan the reservation
-      if (tail0 != tail) ds->stats[10] += tail0 - tail;
+      if (tail0 != tail) atomicAdd(&ds->stats[10], tail0 - tail);   // Calls may run at once
       a.qstate[0] = head;
       a.qstate[1] = tail;
       a.qstate[2] = 0;
-      const unsigned long long K = ld_relaxed_u64(&ds->rb_kept);
+      const unsigned long long K = ld_relaxed_u64(&rs->rb_kept);
       const unsigned long long L = tail - head, T = L + K;
       // parent-bound reservation takes nothing here: everything admitted is
       // queued and the window [head, head + T) goes to launch_parent
@@ -126,28 +135,28 @@ __global__ void __launch_bounds__(RB_THREADS) ready_count_kernel(ReadyArgs a) {
         ds->pb_head = head;
         ds->pb_old_tail = tail;
         ds->pb_stop = ~0ull;
-        ds->pb_bad = ld_relaxed_u64(&ds->rb_bad);
+        ds->pb_bad = ld_relaxed_u64(&rs->rb_bad);
         ds->pb_err = 0u;
       }
-      ds->rb_npop = npop;
-      ds->rb_n_batches = (npop + a.batch_size - 1) / a.batch_size;
+      rs->rb_npop = npop;
+      rs->rb_n_batches = (npop + a.batch_size - 1) / a.batch_size;
       if (a.n_batched_out) *a.n_batched_out = npop;
       if (npop > a.cap) {
-        ds->rb_err = 1u;
+        rs->rb_err = 1u;
         atomicOr(&ds->err, ERR_CAPACITY);
       } else {
-        ds->rb_err = 0u;
-        ds->rb_L = L;
-        ds->rb_k = K;
-        ds->rb_head = head;
-        ds->rb_tail = tail;
+        rs->rb_err = 0u;
+        rs->rb_L = L;
+        rs->rb_k = K;
+        rs->rb_head = head;
+        rs->rb_tail = tail;
         a.qstate[0] = head + npop;
         a.qstate[1] = tail + K;
-        if (!a.parent_bound) ds->stats[5] += ld_relaxed_u64(&ds->rb_bad);
+        if (!a.parent_bound) atomicAdd(&ds->stats[5], ld_relaxed_u64(&rs->rb_bad));
       }
-      ds->rb_kept = 0;
-      ds->rb_bad = 0;
-      ds->rb_ticket = 0u;
+      rs->rb_kept = 0;
+      rs->rb_bad = 0;
+      rs->rb_ticket = 0u;
     }
   }
 }
@@ -158,8 +167,9 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
   __shared__ uint32_t s_tile;
   __shared__ unsigned long long s_prefix;
   DevScalars* ds = a.ds;
-  const bool failed = ds->rb_err != 0u;
-  const unsigned long long L = ds->rb_L, npop = ds->rb_npop, head = ds->rb_head;
+  ReadyScalars* rs = a.rs;
+  const bool failed = rs->rb_err != 0u;
+  const unsigned long long L = rs->rb_L, npop = rs->rb_npop, head = rs->rb_head;
 
   if (failed) {
     // release the claims taken by the first pass; nothing else changes
@@ -167,7 +177,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
       const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
       for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < a.n_cand; i += stride) {
         const uint64_t c = a.cand[i];
-        if (c < a.N && a.phase[c] == ((uint32_t)i << 2)) a.phase[c] = WAIT_UNCLAIMED;
+        if (c < a.N && claimed_here(a, c, a.phase[c], i)) a.phase[c] = WAIT_UNCLAIMED;
       }
     }
     return;   // no tile counter was touched
@@ -191,7 +201,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
   }
 
   for (;;) {
-    if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_READY]);
+    if (threadIdx.x == 0) s_tile = claim_tile(&rs->tile_ctr);
     __syncthreads();
     const uint32_t tile = s_tile;
     __syncthreads();
@@ -208,7 +218,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
       const uint64_t c = a.cand ? (uint64_t)a.cand[i] : i;
       if (c >= a.N) continue;
       const uint32_t w = a.phase[c];
-      const bool keep = a.cand ? (w == ((uint32_t)i << 2)) : (w == WAIT_UNCLAIMED && call_ok(a, c));
+      const bool keep = a.cand ? claimed_here(a, c, w, i) : (w == WAIT_UNCLAIMED && call_ok(a, c));
       if (keep) {
         flags |= 1u << k;
         cs[k] = (uint32_t)c;
@@ -218,7 +228,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
     unsigned long long total;
     unsigned long long excl = block_excl_scan(cnt, s_scan, &total);
     if (threadIdx.x < 32) {  // one warp looks back
-      const auto pfx = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_READY], &ds->err);
+      const auto pfx = lookback_exclusive(a.ts, tile, total, rs->epoch, &ds->err);
       if (threadIdx.x == 0) s_prefix = pfx;
     }
     __syncthreads();
@@ -238,7 +248,11 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
       ++rank;
     }
   }
-  if (threadIdx.x == 0) retire_cta(ds, TS_READY, n_part);
+  if (threadIdx.x == 0 && ticket(&rs->exit_ctr) == n_part - 1) {
+    rs->tile_ctr = 0u;
+    rs->exit_ctr = 0u;
+    rs->epoch += 1ull;
+  }
 }
 
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a) {

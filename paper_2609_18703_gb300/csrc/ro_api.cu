@@ -145,6 +145,16 @@ struct ro_ctx {
   LaunchCfg L{}, Lp{}, Lc{}, Lf{};
   DevScalars* ds = nullptr;
   DevScalars* hs = nullptr;   // pinned mirror
+  ReadyScalars* rs = nullptr;   // per Call, device
+  ReadyScalars* hrs = nullptr;  // per Call, pinned mirror
+  // Streams of the Calls' admissions (ro_ctx_set_call_streams; the
+  // context's stream when unset).  An admission on a Call's stream follows
+  // the context's stream (call_fork); the context's stream waits for it
+  // (call_join) before its next launch of its own.
+  std::vector<cudaStream_t> call_stream;
+  std::vector<Ev> call_fork, call_join;
+  std::vector<char> call_pending;
+  std::vector<TsBuf> ts_call;   // the admission scans' tile status, per Call
   std::vector<ExpSlot> slots;
   std::vector<Expansion> exps;
   TsBuf ts[N_TS];
@@ -226,6 +236,8 @@ void sync_all_streams(ro_ctx* c) {
   if (c->plan_stream != c->stream) cudaStreamSynchronize(c->plan_stream);
   if (c->copy_stream != c->stream) cudaStreamSynchronize(c->copy_stream);
   if (c->fin_stream != c->stream) cudaStreamSynchronize(c->fin_stream);
+  for (cudaStream_t s : c->call_stream)
+    if (s != c->stream) cudaStreamSynchronize(s);
 }
 
 // Grow-only device buffer, zeroed when (re)allocated.  Growth needs a
@@ -296,7 +308,19 @@ ro_status order(ro_ctx* c, Ev& ev, cudaStream_t from, cudaStream_t to) {
 }
 
 // The context's stream waits for the plan and copy streams.
+// The context's stream waits for the admissions still pending on the Calls'
+// streams; every launch of its own (and every fork from it) comes after.
+ro_status settle_calls(ro_ctx* c) {
+  for (size_t k = 0; k < c->call_pending.size(); ++k) {
+    if (!c->call_pending[k]) continue;
+    RO_TRY(order(c, c->call_join[k], c->call_stream[k], c->stream));
+    c->call_pending[k] = 0;
+  }
+  return RO_OK;
+}
+
 ro_status join(ro_ctx* c) {
+  RO_TRY(settle_calls(c));
   RO_TRY(order(c, c->fin_join, c->fin_stream, c->stream));
   RO_TRY(order(c, c->join_plan, c->plan_stream, c->stream));
   if (c->copy_stream != c->plan_stream) RO_TRY(order(c, c->join_copy, c->copy_stream, c->stream));
@@ -309,8 +333,7 @@ ro_status join(ro_ctx* c) {
 // Tile-status arrays of one scan slot (flags start zeroed: epoch 0, nothing
 // published; kernels keep their epochs on the device).
 template <class T>
-ro_status tile_status(ro_ctx* c, int slot, size_t tiles, TileStatus<T>* out) {
-  TsBuf& t = c->ts[slot];
+ro_status tile_status_buf(ro_ctx* c, TsBuf& t, size_t tiles, TileStatus<T>* out) {
   tiles = std::max<size_t>(tiles, 1);
   RO_TRY(ensure(c, t.flag, tiles * sizeof(unsigned long long), "scan flags"));
   RO_TRY(ensure(c, t.agg, tiles * sizeof(Pair64), "scan aggregates"));
@@ -319,6 +342,10 @@ ro_status tile_status(ro_ctx* c, int slot, size_t tiles, TileStatus<T>* out) {
   out->agg = (T*)t.agg.p;
   out->inc = (T*)t.inc.p;
   return RO_OK;
+}
+template <class T>
+ro_status tile_status(ro_ctx* c, int slot, size_t tiles, TileStatus<T>* out) {
+  return tile_status_buf(c, c->ts[slot], tiles, out);
 }
 
 ro_status check_launch(ro_ctx* c, const char* what) {
@@ -432,6 +459,17 @@ ro_status queue_ready(ro_ctx* c, QueueBufs& Q, uint64_t N) {
   return RO_OK;
 }
 
+void free_scalars(ro_ctx* c) {
+  if (c->ds) cudaFree(c->ds);
+  if (c->hs) cudaFreeHost(c->hs);
+  if (c->rs) cudaFree(c->rs);
+  if (c->hrs) cudaFreeHost(c->hrs);
+  c->ds = nullptr;
+  c->hs = nullptr;
+  c->rs = nullptr;
+  c->hrs = nullptr;
+}
+
 }  // namespace
 
 extern "C" {
@@ -455,18 +493,26 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->n_calls = n_calls;
   cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
   if (cudaMalloc(&c->ds, sizeof(DevScalars)) != cudaSuccess ||
-      cudaMallocHost(&c->hs, sizeof(DevScalars)) != cudaSuccess) {
+      cudaMallocHost(&c->hs, sizeof(DevScalars)) != cudaSuccess ||
+      cudaMalloc(&c->rs, n_calls * sizeof(ReadyScalars)) != cudaSuccess ||
+      cudaMallocHost(&c->hrs, n_calls * sizeof(ReadyScalars)) != cudaSuccess) {
     cudaGetLastError();
-    if (c->ds) cudaFree(c->ds);
+    free_scalars(c);
     delete c;
     return RO_E_OOM;
   }
   cudaMemsetAsync(c->ds, 0, sizeof(DevScalars), c->stream);
+  cudaMemsetAsync(c->rs, 0, n_calls * sizeof(ReadyScalars), c->stream);
   std::memset(c->hs, 0, sizeof(DevScalars));
+  std::memset(c->hrs, 0, n_calls * sizeof(ReadyScalars));
+  c->call_stream.assign(n_calls, c->stream);
+  c->call_fork.resize(n_calls);
+  c->call_join.resize(n_calls);
+  c->call_pending.assign(n_calls, 0);
+  c->ts_call.resize(n_calls);
   if (prepare_assemble_kernels() != cudaSuccess) {
     cudaGetLastError();
-    cudaFree(c->ds);
-    cudaFreeHost(c->hs);
+    free_scalars(c);
     delete c;
     return RO_E_CUDA;
   }
@@ -491,8 +537,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->Lf = c->L;
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) {
-    cudaFree(c->ds);
-    cudaFreeHost(c->hs);
+    free_scalars(c);
     delete c;
     return RO_E_CUDA;
   }
@@ -534,8 +579,12 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   free_ev(c->fin_fork); free_ev(c->fin_join); free_ev(c->fin_plan); free_ev(c->copy_done);
   if (c->own_fin) cudaStreamDestroy(c->own_fin);
   for (cudaEvent_t e : c->prof.pool) cudaEventDestroy(e);
-  cudaFree(c->ds);
-  cudaFreeHost(c->hs);
+  for (auto& t : c->ts_call) {
+    free_buf(t.flag); free_buf(t.agg); free_buf(t.inc);
+  }
+  for (auto& e : c->call_fork) free_ev(e);
+  for (auto& e : c->call_join) free_ev(e);
+  free_scalars(c);
   delete c;
   return RO_OK;
 }
@@ -573,6 +622,17 @@ ro_status ro_ctx_set_streams(ro_ctx* c, void* plan_stream, void* copy_stream) {
   c->Lp.stream = c->plan_stream;
   c->Lc.stream = c->copy_stream;
   c->Lf.stream = c->fin_stream;
+  return RO_OK;
+}
+
+ro_status ro_ctx_set_call_streams(ro_ctx* c, void* const* streams, uint32_t n) {
+  RO_TRY(enter(c));
+  if (n > c->n_calls) return fail(c, RO_E_INVAL, "ro_ctx_set_call_streams: %u streams for %u Calls", n, c->n_calls);
+  if (n && !streams) return fail(c, RO_E_INVAL, "ro_ctx_set_call_streams: NULL stream list");
+  DeviceGuard g(c->device);
+  RO_TRY(join(c));   // pending admissions on the old streams first
+  for (uint32_t k = 0; k < c->n_calls; ++k)
+    c->call_stream[k] = (k < n && streams[k]) ? (cudaStream_t)streams[k] : c->stream;
   return RO_OK;
 }
 
@@ -656,6 +716,7 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
                   (unsigned long long)n_parents, (unsigned long long)px->N);
   }
   DeviceGuard g(c->device);
+  RO_TRY(settle_calls(c));   // after the Calls' pending admissions
   const size_t slot = c->exps.size();
   if (c->slots.size() <= slot) c->slots.resize(slot + 1);
   ExpSlot& S = c->slots[slot];
@@ -771,13 +832,31 @@ ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* 
   ra.batched = d_batched;
   ra.n_batched_out = d_n_batched;
   ra.ds = c->ds;
-  RO_TRY(tile_status(c, TS_READY, ceil_div(ra.n_cand, (uint64_t)RB_THREADS * RB_ITEMS), &ra.ts));
-  launch_ready(c->L, ra);
+  ra.rs = c->rs + call;
+  for (cudaStream_t s : c->call_stream) ra.calls_concurrent |= (s != c->stream);
+  ra.calls_concurrent &= ra.check_call;
+  RO_TRY(tile_status_buf(c, c->ts_call[call], ceil_div(ra.n_cand, (uint64_t)RB_THREADS * RB_ITEMS),
+                         &ra.ts));
+  // on the Call's stream when it has one, after everything issued on the
+  // context's stream so far; the context's stream waits for it before its
+  // next launch
+  LaunchCfg Lr = c->L;
+  const cudaStream_t cs = c->call_stream[call];
+  if (cs != c->stream) {
+    RO_TRY(order(c, c->call_fork[call], c->stream, cs));
+    Lr.stream = cs;
+  }
+  launch_ready(Lr, ra);
   RO_TRY(check_launch(c, "batch_ready"));
+  if (cs != c->stream) c->call_pending[call] = 1;
   if (h_n_batched || h_n_batches) {
     ro_status st = sync_and_check(c);
-    if (h_n_batched) *h_n_batched = c->hs->rb_npop;
-    if (h_n_batches) *h_n_batches = c->hs->rb_n_batches;
+    cudaError_t e = cudaMemcpyAsync(c->hrs + call, c->rs + call, sizeof(ReadyScalars),
+                                    cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "synchronise");
+    if (h_n_batched) *h_n_batched = c->hrs[call].rb_npop;
+    if (h_n_batches) *h_n_batches = c->hrs[call].rb_n_batches;
     return st;
   }
   return RO_OK;
@@ -800,6 +879,7 @@ ro_status ro_batch_ready_parent(ro_ctx* c, int32_t xid, uint32_t call, const uin
   if (d_cand && n_cand > MAX_CAND)
     return fail(c, RO_E_INVAL, "%s: more than 2^30-2 candidates in one call", fn);
   DeviceGuard g(c->device);
+  RO_TRY(settle_calls(c));   // after the Calls' pending admissions
   ExpSlot& S = c->slots[xid];
   QueueBufs& Q = S.queues[call];
   RO_TRY(queue_ready(c, Q, x->N));
@@ -832,7 +912,9 @@ ro_status ro_batch_ready_parent(ro_ctx* c, int32_t xid, uint32_t call, const uin
   ra.n_batched_out = nullptr;
   ra.parent_bound = 1;
   ra.ds = c->ds;
-  RO_TRY(tile_status(c, TS_READY, ceil_div(ra.n_cand, (uint64_t)RB_THREADS * RB_ITEMS), &ra.ts));
+  ra.rs = c->rs + call;
+  RO_TRY(tile_status_buf(c, c->ts_call[call], ceil_div(ra.n_cand, (uint64_t)RB_THREADS * RB_ITEMS),
+                         &ra.ts));
 
   ParentArgs pa{};
   pa.N = N;
@@ -890,6 +972,7 @@ ro_status ro_retry(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* d_chil
   if (n && !d_children) return fail(c, RO_E_INVAL, "ro_retry: NULL d_children");
   if (n >= 0xFFFFFFFFull) return fail(c, RO_E_OVERFLOW, "ro_retry: 2^32-1 entries or more");
   DeviceGuard g(c->device);
+  RO_TRY(settle_calls(c));   // after the Calls' pending admissions
   ExpSlot& S = c->slots[xid];
   if (h_n_retried) *h_n_retried = 0;
   if (n == 0) return RO_OK;
@@ -933,6 +1016,7 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   if (d_done_parents && done_cap < std::min<uint64_t>(n, x->P))
     return fail(c, RO_E_INVAL, "ro_gather_commit: done_cap below min(n, parents)");
   DeviceGuard g(c->device);
+  RO_TRY(settle_calls(c));   // after the Calls' pending admissions
   ExpSlot& S = c->slots[xid];
   const int ls = (int)(x->commits % RING);
   ListSlot& LS = S.lists[ls];
@@ -1069,6 +1153,7 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   if (n_parents >= (1ull << 32)) return fail(c, RO_E_OVERFLOW, "ro_assemble: list of 2^32 or more");
   if (arena_bytes >= MAX_ARENA) return fail(c, RO_E_OVERFLOW, "ro_assemble: arena of 2^48 bytes or more");
   DeviceGuard g(c->device);
+  RO_TRY(settle_calls(c));   // after the Calls' pending admissions
   // The arena and the output may be pinned host memory (read and written in
   // place by the copy, no staging copies); pageable host memory is refused.
   int arena_host = 0;

@@ -100,9 +100,6 @@ struct DevScalars {
   unsigned long long stats[13];  // same order as ro_stats
   // ro_expand
   unsigned long long n_children, n_empty, last_nonempty_parent;
-  // ro_batch_ready
-  unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
-  uint32_t rb_ticket, rb_err;
   // ro_gather_commit
   unsigned long long cm_n, cm_n_done;
   // per commit, in two slots (commit sequence & 1): duplicate candidates and
@@ -124,8 +121,19 @@ struct DevScalars {
   uint32_t exit_ctr[8];
   unsigned long long epoch[8];
 };
-enum TileSlot { TS_EXPAND = 0, TS_READY = 1, TS_COMMIT = 2, TS_ASM_PARENTS = 3, TS_ASM_MEMBERS = 4,
-                TS_RETRY = 6, TS_PARENT = 7 };   // 5: asm_copy's exit ticket
+// Admission scalars of one Call (ro_batch_ready): the first pass's counts,
+// its exit ticket and the reservation it plans, and the scatter pass's tile
+// counter, exit ticket and scan epoch.  One per Call, so that admissions of
+// different Calls can run at the same time on streams of their own.
+struct alignas(128) ReadyScalars {
+  unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
+  unsigned long long epoch;
+  uint32_t rb_ticket, rb_err, tile_ctr, exit_ctr;
+};
+// Slot 1 is unused (each Call's admission counts in its ReadyScalars);
+// 5: asm_copy's exit ticket.
+enum TileSlot { TS_EXPAND = 0, TS_COMMIT = 2, TS_ASM_PARENTS = 3, TS_ASM_MEMBERS = 4,
+                TS_RETRY = 6, TS_PARENT = 7 };
 
 // Wait until the grid this launch depends on (programmatic dependent launch)
 // has completed and its memory is visible; a no-op without a dependency.

@@ -112,6 +112,7 @@ struct ReadyArgs {
   uint32_t* phase;
   const Rec* rec;             // read for the Call when the expansion has several
   int check_call;
+  int calls_concurrent;       // other Calls' admissions may run at the same time
   uint32_t call, batch_size;
   int flush;
   uint64_t cap;
@@ -122,7 +123,8 @@ struct ReadyArgs {
   uint64_t* n_batched_out;    // optional device output
   int parent_bound;           // admit only: the window is reserved by launch_parent
   DevScalars* ds;
-  TileStatus<unsigned long long> ts;
+  ReadyScalars* rs;           // this Call's
+  TileStatus<unsigned long long> ts;   // this Call's
 };
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a);
 // ---- ro_batch_ready_parent ---------------------------------------------------------

@@ -36,13 +36,16 @@ def host(t: torch.Tensor, dtype, n: Optional[int] = None) -> np.ndarray:
 
 
 class Lockstep:
-    def __init__(self, n_calls: int = 1, streams: bool = False):
+    def __init__(self, n_calls: int = 1, streams: bool = False, call_streams: bool = False):
         self.o = OracleCtx(n_calls)
         self.stream = torch.cuda.current_stream()
         self.ctx = ro.ro_ctx_create(0, self.stream, n_calls)
         if streams:   # assembly planning and copies on streams of their own
             self.side = (torch.cuda.Stream(), torch.cuda.Stream())
             ro.ro_ctx_set_streams(self.ctx, *self.side)
+        if call_streams:   # each Call's admissions on a stream of its own
+            self.call_side = [torch.cuda.Stream() for _ in range(n_calls)]
+            ro.ro_ctx_set_call_streams(self.ctx, self.call_side)
         self.N = {}
         self.P = {}
 

@@ -245,3 +245,71 @@ def test_set_streams_back_to_one_stream():
         ps.check(ref, total)
     finally:
         ro.ro_ctx_destroy(ctx)
+
+
+@pytest.mark.parametrize("B", [32, 256])
+def test_call_admissions_on_streams_of_their_own(B):
+    """Four Calls, each admitting on a stream of its own
+    (ro_ctx_set_call_streams).  Per readiness wave the four admissions are
+    issued without waiting, from one candidate list (each Call keeps its
+    own children), so they run at the same time; every Call's reserved
+    batches, the commit of their results and the assembly equal the
+    oracle's, wave by wave."""
+    from tests.lockstep import Lockstep
+    from workload import streaming
+    lv = streaming(total_children=80000, batch_size=B, ready_waves=20).top
+    a = host_arena(lv)
+    ad = dev(a if a.size else np.zeros(1, np.uint8), np.uint8)
+    with Lockstep(n_calls=4, call_streams=True) as ls:
+        x = ls.expand(lv.counts, parent_call=lv.parent_call)["xid"]
+        N = ls.N[x]
+        d_b = [empty(N + B, np.uint32) for _ in range(4)]
+        d_nb = [empty(1, np.uint64) for _ in range(4)]
+        n_ready = lv.ready_bounds.size - 1
+        for w in range(n_ready):
+            cand = lv.readiness[lv.ready_bounds[w]:lv.ready_bounds[w + 1]]
+            last = w == n_ready - 1
+            d_cand = dev(cand, np.uint32)
+            for c in range(4):
+                st, _, _ = ro.ro_batch_ready(ls.ctx, x, c, d_cand, cand.size, B, last, d_b[c], N + B,
+                                             d_nb[c], want_host=False)
+                assert st == ro.RO_OK, ro.ro_last_error(ls.ctx)
+            assert ro.ro_ctx_sync(ls.ctx) == ro.RO_OK
+            got = []
+            for c in range(4):
+                r = ls.o.batch_ready(x, c, cand, B, last, cap=N + B, check=False)
+                nb = int(host(d_nb[c], np.uint64, 1)[0])
+                assert nb == r["n_batched"]
+                assert np.array_equal(host(d_b[c], np.uint32, nb), r["batched"])
+                got.append(r["batched"])
+            got = np.concatenate(got)
+            got = got[np.argsort(lv.key[got], kind="stable")]
+            ch, st, ln, of = lv.reports(got)
+            cm = ls.commit(x, ch, st, ln, of, arena_bytes=lv.arena_bytes)
+            ls.assemble(x, a, ad, parents=None, n_parents=max(cm["n_done"], 1))
+        ls.check_stats()
+
+
+def test_call_streams_with_failures_retries_and_capacity():
+    """Call streams with the rest of the path in between: a GroupFailure
+    commit, a retry and a refused admission (capacity) of one Call while the
+    others admit; all equal the oracle's."""
+    from tests.lockstep import Lockstep
+    rng = np.random.default_rng(41)
+    P = 3000
+    counts = rng.integers(1, 9, P).astype(np.uint32)
+    calls = (np.arange(P) % 3).astype(np.uint8)
+    with Lockstep(n_calls=3, call_streams=True) as ls:
+        x = ls.expand(counts, parent_call=calls)["xid"]
+        N = ls.N[x]
+        cand = rng.permutation(N).astype(np.uint32)
+        r = [ls.batch_ready(x, c, cand[: N // 2], 4) for c in range(3)]
+        # a GroupFailure from the first reserved child of Call 0
+        ch = np.array([r[0]["batched"][0]], np.uint32)
+        ls.commit(x, ch, np.array([5], np.uint8), np.array([8], np.uint32), np.array([0], np.uint64),
+                  arena_bytes=64)
+        ls.retry(x, 1, r[1]["batched"][:8])
+        ls.batch_ready(x, 2, cand[N // 2:], 4, cap=3)          # refused: nothing changes
+        for c in range(3):
+            ls.batch_ready(x, c, cand[N // 2:], 4, flush=True)
+        ls.check_stats()
