@@ -313,3 +313,110 @@ def test_call_streams_with_failures_retries_and_capacity():
         for c in range(3):
             ls.batch_ready(x, c, cand[N // 2:], 4, flush=True)
         ls.check_stats()
+
+
+def test_call_streams_captured_in_a_graph():
+    """The streaming configuration's wave loop (four Calls, each admitting on
+    a stream of its own; commit of the reserved children's results in key
+    order; assembly at a running cursor on plan and copy streams) captured
+    in a CUDA graph and replayed: every Call's reservation of every wave and
+    every assembled output equal the oracle's."""
+    from workload import streaming
+    B = 64
+    lv = streaming(total_children=60000, batch_size=B, ready_waves=16).top
+    a = host_arena(lv)
+    P, N, W, C = lv.n_parents, lv.n_children, lv.ready_bounds.size - 1, lv.n_calls
+    # the oracle's pass: reservations per (wave, Call), then reports, commit, assembly
+    o = OracleCtx(C)
+    x = o.expand(lv.counts, parent_call=lv.parent_call)["xid"]
+    ref, reports, cursor = [], [], 0
+    for w in range(W):
+        cand = lv.readiness[lv.ready_bounds[w]:lv.ready_bounds[w + 1]]
+        res = [o.batch_ready(x, c, cand, B, w == W - 1, cap=N + B)["batched"] for c in range(C)]
+        got = np.concatenate(res)
+        got = got[np.argsort(lv.key[got], kind="stable")]
+        ch, st, ln, of = lv.reports(got)
+        reports.append((ch.size, dev(ch, np.uint32), dev(st, np.uint8), dev(ln, np.uint32),
+                        dev(of, np.uint64)))
+        cm = o.gather_commit(x, ch, st, ln, of, arena_bytes=max(lv.arena_bytes, 1))
+        asm = o.assemble(x, a, n_parents=max(cm["n_done"], 1), cursor=cursor)
+        ref.append(dict(res=res, status=asm["parent_status"], off=asm["out_off"],
+                        bytes=asm["out_bytes"], base=cursor,
+                        out=asm["out"][cursor:cursor + asm["out_bytes"]].copy()))
+        cursor = asm["cursor"]
+    o.close()
+    counts, pc = dev(lv.counts, np.uint32), dev(lv.parent_call, np.uint8)
+    offsets, cp, co = empty(P + 1, np.uint64), empty(N, np.uint32), empty(N, np.uint32)
+    cands = [dev(lv.readiness[lv.ready_bounds[w]:lv.ready_bounds[w + 1]], np.uint32) for w in range(W)]
+    batched = [[empty(N + B, np.uint32) for _ in range(C)] for _ in range(W)]
+    nb = [[empty(1, np.uint64) for _ in range(C)] for _ in range(W)]
+    status = [empty(P, np.uint8) for _ in range(W)]
+    off = [empty(P + 1, np.uint64) for _ in range(W)]
+    ad = dev(a if a.size else np.zeros(1, np.uint8), np.uint8)
+    out_cap = int(lv.arena_bytes) + 64
+    out = torch.zeros(out_cap, dtype=torch.uint8, device="cuda")
+    cur = empty(1, np.uint64)
+    stream = torch.cuda.Stream()
+
+    def waves(ctx, xid):
+        cur.zero_()
+        for w in range(W):
+            n_c = int(lv.ready_bounds[w + 1] - lv.ready_bounds[w])
+            for c in range(C):
+                st, _, _ = ro.ro_batch_ready(ctx, xid, c, cands[w], n_c, B, w == W - 1, batched[w][c],
+                                             N + B, nb[w][c], want_host=False)
+                assert st == ro.RO_OK
+            n, ch, stt, ln, of = reports[w]
+            st, _ = ro.ro_gather_commit(ctx, xid, n, None, ch, stt, ln, of, None,
+                                        max(int(lv.arena_bytes), 1), None, None, 0, None,
+                                        want_host=False)
+            assert st == ro.RO_OK
+            st, _ = ro.ro_assemble(ctx, xid, ad, ad.numel(), None, P, None, status[w], off[w], None,
+                                   out, out_cap, cur, None, want_host=False)
+            assert st == ro.RO_OK
+        assert ro.ro_ctx_join(ctx) == ro.RO_OK
+
+    def expand(ctx):
+        st, n, _, xid = ro.ro_expand(ctx, -1, counts, P, pc, offsets, cp, co, N, None)
+        assert st == ro.RO_OK and n == N
+        return xid
+
+    def check():
+        torch.cuda.synchronize()
+        for w, r in enumerate(ref):
+            for c in range(C):
+                k = int(host(nb[w][c], np.uint64, 1)[0])
+                assert np.array_equal(host(batched[w][c], np.uint32, k), r["res"][c]), (w, c)
+            k = r["status"].size
+            assert np.array_equal(host(status[w], np.uint8, k), r["status"]), w
+            assert np.array_equal(host(off[w], np.uint64, k + 1), r["off"]), w
+            got = out[r["base"]:r["base"] + r["bytes"]].cpu().numpy()
+            assert np.array_equal(got, r["out"]), w
+        assert int(host(cur, np.uint64, 1)[0]) == cursor
+
+    with torch.cuda.stream(stream):
+        ctx = ro.ro_ctx_create(0, stream, C)
+        side = (torch.cuda.Stream(), torch.cuda.Stream())
+        call_side = [torch.cuda.Stream() for _ in range(C)]
+        ro.ro_ctx_set_streams(ctx, *side)
+        ro.ro_ctx_set_call_streams(ctx, call_side)
+        try:
+            waves(ctx, expand(ctx))   # sizes every buffer
+            assert ro.ro_ctx_sync(ctx) == ro.RO_OK, ro.ro_last_error(ctx)
+            check()
+            ro.ro_ctx_reset(ctx)
+            xid = expand(ctx)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                waves(ctx, xid)
+            for _ in range(2):
+                out.zero_()
+                for t in status + off + [b for row in batched for b in row]:
+                    t.zero_()
+                ro.ro_ctx_reset(ctx)
+                expand(ctx)
+                g.replay()
+                assert ro.ro_ctx_sync(ctx) == ro.RO_OK, ro.ro_last_error(ctx)
+                check()
+        finally:
+            ro.ro_ctx_destroy(ctx)
