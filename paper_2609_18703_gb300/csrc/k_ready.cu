@@ -260,7 +260,13 @@ void launch_ready(const LaunchCfg& L, const ReadyArgs& a) {
   const int grid_count =
       (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(a.n_cand, per), (uint64_t)L.grid_rb));
   launch_k(L, K_RB_COUNT, ready_count_kernel, grid_count, RB_THREADS, 0, a);
-  launch_k(L, K_RB_SCATTER, ready_scatter_kernel, L.grid_rb, RB_THREADS, 0, a);
+  // one CTA per tile of candidates; CTAs past them only help move the
+  // entries earlier calls queued (a grid-stride loop), for which one per SM
+  // is plenty
+  const uint64_t tiles = ceil_div(a.n_cand, (uint64_t)RB_THREADS * RB_ITEMS);
+  const int grid_scatter = (int)std::min<uint64_t>(
+      (uint64_t)L.grid_rb, std::max<uint64_t>(tiles, std::max(1, L.grid_rb / 8)));
+  launch_k(L, K_RB_SCATTER, ready_scatter_kernel, grid_scatter, RB_THREADS, 0, a);
 }
 
 const void* kernel_ptr_ready(int which) {
