@@ -420,3 +420,108 @@ def test_call_streams_captured_in_a_graph():
                 check()
         finally:
             ro.ro_ctx_destroy(ctx)
+
+
+def test_captured_commits_with_repeats_and_group_failures():
+    """A wave loop with repeated reports in some waves and GroupFailure
+    reports in others (the commit's fix-up then orders the repeats and
+    applies the barriers), captured in a CUDA graph and replayed, gives every
+    verdict, completed list, status, offset and byte the oracle gives."""
+    lv = docpage(parents=1500, waves=10).top
+    a = host_arena(lv)
+    rng = np.random.default_rng(5)
+    W, P, N = lv.n_waves, lv.n_parents, lv.n_children
+    reps = []
+    for w in range(W):
+        ch, st, ln, of = lv.reports(lv.wave(w))
+        if w in (2, 5):   # repeats of some reports of this wave, later in the array
+            idx = rng.choice(ch.size, 25, replace=False)
+            ch, st = np.concatenate([ch, ch[idx]]), np.concatenate([st, st[idx]])
+            ln, of = np.concatenate([ln, ln[idx]]), np.concatenate([of, of[idx]])
+        if w in (3, 7):   # GroupFailures
+            st = st.copy()
+            st[rng.choice(ch.size, 4, replace=False)] = 5
+        reps.append((ch, st, ln, of))
+    o = OracleCtx(1)
+    x = o.expand(lv.counts)["xid"]
+    o.batch_ready(x, 0, None, lv.batch_size, True, cap=N + lv.batch_size)
+    ref, cursor = [], 0
+    for w in range(W):
+        cm = o.gather_commit(x, *reps[w], arena_bytes=max(lv.arena_bytes, 1))
+        asm = o.assemble(x, a, n_parents=max(cm["n_done"], 1), cursor=cursor)
+        ref.append(dict(code=cm["code"], done=cm["done"], status=asm["parent_status"],
+                        off=asm["out_off"], bytes=asm["out_bytes"], base=cursor,
+                        out=asm["out"][cursor:cursor + asm["out_bytes"]].copy()))
+        cursor = asm["cursor"]
+    o.close()
+    counts = dev(lv.counts, np.uint32)
+    offsets, cp, co = empty(P + 1, np.uint64), empty(N, np.uint32), empty(N, np.uint32)
+    batched = empty(N + lv.batch_size, np.uint32)
+    dr = [tuple(dev(v, t) for v, t in zip(r, (np.uint32, np.uint8, np.uint32, np.uint64))) for r in reps]
+    code = [empty(r[0].size, np.uint8) for r in reps]
+    done = [empty(P, np.uint32) for _ in range(W)]
+    status = [empty(P, np.uint8) for _ in range(W)]
+    off = [empty(P + 1, np.uint64) for _ in range(W)]
+    ad = dev(a if a.size else np.zeros(1, np.uint8), np.uint8)
+    out_cap = int(lv.arena_bytes) + 64
+    out = torch.zeros(out_cap, dtype=torch.uint8, device="cuda")
+    cur = empty(1, np.uint64)
+    stream = torch.cuda.Stream()
+
+    def expand(ctx):
+        st, n, _, xid = ro.ro_expand(ctx, -1, counts, P, None, offsets, cp, co, N, None)
+        assert st == ro.RO_OK and n == N
+        return xid
+
+    def waves(ctx, xid):
+        st, _, _ = ro.ro_batch_ready(ctx, xid, 0, None, 0, lv.batch_size, 1, batched, N + lv.batch_size,
+                                     None, want_host=False)
+        assert st == ro.RO_OK
+        cur.zero_()
+        for w in range(W):
+            ch, stt, ln, of = dr[w]
+            st, _ = ro.ro_gather_commit(ctx, xid, reps[w][0].size, None, ch, stt, ln, of, None,
+                                        max(int(lv.arena_bytes), 1), code[w], done[w], P, None,
+                                        want_host=False)
+            assert st == ro.RO_OK
+            st, _ = ro.ro_assemble(ctx, xid, ad, ad.numel(), None, P, None, status[w], off[w], None,
+                                   out, out_cap, cur, None, want_host=False)
+            assert st == ro.RO_OK
+        assert ro.ro_ctx_join(ctx) == ro.RO_OK
+
+    def check():
+        torch.cuda.synchronize()
+        for w, r in enumerate(ref):
+            assert np.array_equal(host(code[w], np.uint8, r["code"].size), r["code"]), w
+            k = r["done"].size
+            assert np.array_equal(host(done[w], np.uint32, k), r["done"]), w
+            assert np.array_equal(host(status[w], np.uint8, k), r["status"]), w
+            assert np.array_equal(host(off[w], np.uint64, k + 1), r["off"]), w
+            got = out[r["base"]:r["base"] + r["bytes"]].cpu().numpy()
+            assert np.array_equal(got, r["out"]), w
+        assert int(host(cur, np.uint64, 1)[0]) == cursor
+
+    with torch.cuda.stream(stream):
+        ctx = ro.ro_ctx_create(0, stream, 1)
+        side = (torch.cuda.Stream(), torch.cuda.Stream())
+        ro.ro_ctx_set_streams(ctx, *side)
+        try:
+            waves(ctx, expand(ctx))
+            assert ro.ro_ctx_sync(ctx) == ro.RO_OK, ro.ro_last_error(ctx)
+            check()
+            ro.ro_ctx_reset(ctx)
+            xid = expand(ctx)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                waves(ctx, xid)
+            for _ in range(2):
+                out.zero_()
+                for t in code + done + status + off:
+                    t.zero_()
+                ro.ro_ctx_reset(ctx)
+                expand(ctx)
+                g.replay()
+                assert ro.ro_ctx_sync(ctx) == ro.RO_OK, ro.ro_last_error(ctx)
+                check()
+        finally:
+            ro.ro_ctx_destroy(ctx)
