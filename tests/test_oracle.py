@@ -172,6 +172,43 @@ def test_batch_ready_calls_partition():
         assert np.array_equal(r["batched"], np.flatnonzero(calls[cp] == call))
 
 
+def test_calls_admit_independently_of_their_order():
+    """Each Call admits only its own children (Section 4.3: one Ready Queue
+    per Call), so with one shared candidate list, duplicates included, the
+    Calls' reservations do not depend on the order the Calls run in, and each
+    Call's batches over all waves (the last one flushing) are the candidate-
+    order sequence of first occurrences of that Call's children."""
+    rng = np.random.default_rng(9)
+    P, C, B = 400, 4, 5
+    counts = rng.integers(0, 6, P).astype(np.uint32)
+    calls = rng.integers(0, C, P).astype(np.uint8)
+    N = int(counts.sum())
+    cp = np.repeat(np.arange(P), counts.astype(np.int64))
+    cand = rng.integers(0, N, 3 * N).astype(np.uint32)
+    waves = np.array_split(cand, 3)
+    runs = []
+    for order in ((0, 1, 2, 3), (3, 1, 0, 2)):
+        o = OracleCtx(n_calls=C)
+        x = o.expand(counts, parent_call=calls)["xid"]
+        got = {c: [] for c in range(C)}
+        for k, wv in enumerate(waves):
+            for c in order:
+                r = o.batch_ready(x, c, wv, B, flush=(k == len(waves) - 1))
+                assert k == len(waves) - 1 or r["n_batched"] % B == 0
+                got[c].append(r["batched"])
+        o.close()
+        runs.append(got)
+    for c in range(C):
+        for u, v in zip(runs[0][c], runs[1][c]):
+            assert np.array_equal(u, v)
+        seen, seq = set(), []
+        for v in cand.tolist():
+            if calls[cp[v]] == c and v not in seen:
+                seen.add(v)
+                seq.append(v)
+        assert np.array_equal(np.concatenate(runs[0][c]), np.array(seq, np.uint32))
+
+
 def test_batch_ready_capacity_leaves_state():
     o = OracleCtx()
     ex = o.expand([4, 4])
