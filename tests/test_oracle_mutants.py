@@ -15,6 +15,7 @@ MUTANTS = {
     "flush_ignored": ("uint64_t take = flush ? queued : (queued / batch_size) * batch_size;",
                       "uint64_t take = (queued / batch_size) * batch_size;"),
     "readmits_queued": ("if (x->phase[c] != OR_WAITING) continue;", ";"),
+    "admits_other_calls": ("    if (x->child_call[c] != call) continue;\n", "\n"),
     "fence_ignores_generation": ("} else if (g != x->gen[c]) {", "} else if (0) {"),
     "completion_off_by_one": ("if (x->terminal[p] == member_count(x, p)) x->last_done[k++] = p;",
                               "if (x->terminal[p] + 1 == member_count(x, p)) x->last_done[k++] = p;"),
