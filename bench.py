@@ -38,8 +38,7 @@ sys.path.insert(0, ROOT)
 METRIC = "children/sec expand->gather->assemble at 1 GB300; payload GB/s as % of HBM peak"
 K_ACOPY = 8
 # DRAM bytes (read + write) per algorithmic byte of asm_copy, from the ncu
-# capture summarised in profiles/asm_copy_docpage_60k_parents.md (the
-# largest wave of a 60,000-parent document->page pass, same code).  The
+# capture of the largest wave of a 60,000-parent document->page pass.  The
 # full-size bench is too large to capture with the full section set, so the
 # per-launch traffic reported here scales that ratio by the bytes a launch
 # assembles.
@@ -162,17 +161,16 @@ def max_over_ranks(x: float) -> float:
 
 
 # ------------------------------------------------------------------ CPU oracle
-def cpu_oracle_sample(parents: int, waves: int, min_seconds: float = 10.0, max_passes: int = 8):
+def cpu_oracle_sample(parents: int, waves: int, salt: int = 0, min_seconds: float = 10.0, max_passes: int = 8):
     """Time the oracle (single-threaded C) on a bounded sample of the same
     workload: the first `parents` documents of the same distribution, one
     full pass (expand, batch_ready, every wave's commit and assembly with its
     payload bytes), repeated until `min_seconds` of CPU work have run.
     Returns (children/s, seconds, children per pass, bytes per pass, passes)."""
     from oracle import OracleCtx
-    from tests.pipeline import host_arena
-    from workload import docpage
-    lv = docpage(parents=parents, waves=waves, salt=1).top
-    arena = host_arena(lv)
+    from workload import docpage, level_arena
+    lv = docpage(parents=parents, waves=waves, salt=salt).top
+    arena = level_arena(lv)
     reports = [lv.reports(lv.wave(w)) for w in range(lv.n_waves)]
     passes, total, dt = 0, 0, 0.0
     # one core, as a single-threaded baseline; the affinity is restored after
@@ -227,10 +225,9 @@ def run_reference(args, rank):
     if rank != 0:
         return
     from oracle import OracleCtx
-    from tests.pipeline import host_arena
-    from workload import docpage
-    lv = docpage(parents=args.ref_parents, waves=args.waves, salt=1).top
-    arena = host_arena(lv)
+    from workload import docpage, level_arena
+    lv = docpage(parents=args.ref_parents, waves=args.waves, salt=0).top
+    arena = level_arena(lv)
     reports = [lv.reports(lv.wave(w)) for w in range(lv.n_waves)]
 
     def one_pass():
@@ -545,7 +542,7 @@ def run_ours(args, rank, world, local_rank):
 
     cpu = None
     if rank == 0 and not args.no_cpu:
-        v_cpu, dt_cpu, n_cpu, _, p_cpu, core = cpu_oracle_sample(args.cpu_parents, args.waves)
+        v_cpu, dt_cpu, n_cpu, _, p_cpu, core = cpu_oracle_sample(args.cpu_parents, args.waves, salt=rank)
         cpu = {"value": round(v_cpu, 1), "unit": "children/s", "cores": 1, "kind": "oracle",
                "pinned_core": core, "host": host_cpu(),
                "sample": f"document->page, first {args.cpu_parents} parents ({n_cpu} children) "

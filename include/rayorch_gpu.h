@@ -455,11 +455,17 @@ ro_status ro_filter_reports(ro_ctx* ctx, uint8_t* d_state, const uint8_t* d_keep
  *   d_child_parent / d_child_ordinal uint32[child_cap], d_empty_parents
  *   uint32[P] or NULL), on `stream` (a cudaStream_t, NULL = legacy default
  *   stream) of the current device.  h_n_children (required) and h_n_empty
- *   (optional) receive N and the number of empty parents; the call
- *   synchronises the stream.
+ *   (optional) receive N and the number of empty parents.  The call
+ *   returns only after all of its work on `stream` has finished (it
+ *   synchronises the stream after the scan and again after the fill), so
+ *   its outputs are complete on return and the scratch is free for the
+ *   next call.
  *   Limits: at most 16,777,216 parents and 134,217,728 children, else
  *   RO_E_CAPACITY (beyond the static scratch; nothing is launched when the
  *   parent count is too large).  RO_E_CAPACITY also when N > child_cap.
+ *   When the children are refused (too many for the scratch or for
+ *   child_cap) the scan has run: d_offsets, d_empty_parents and the counts
+ *   are written, the child arrays are not, and the next call is unaffected.
  *   The first call on a device looks up the scratch's device address; make
  *   that first call before any stream capture.  All calls share the one
  *   scratch array: calls that overlap on the GPU (other streams, other host

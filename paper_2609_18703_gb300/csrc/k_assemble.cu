@@ -986,6 +986,9 @@ __global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
         k = blockIdx.x + (uint64_t)i * n_part;
         if (k < n_chunks) describe_chunk(c, k, d, lane);
       }
+      // this lane's cp.async copies of small pieces land before the CTA can
+      // exit (on an abort nobody else waits for them)
+      asm volatile("cp.async.wait_all;" ::: "memory");
     } else {
       const uint32_t cw = (uint32_t)(warp - AC_PRODUCERS);
       for (uint32_t i = 0;; ++i) {
@@ -1007,8 +1010,11 @@ __global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
     if (s_abort && threadIdx.x == 0) {
       for (int s = 0; s < AC_STAGES; ++s) {
         if (!s_issued[s]) continue;
-        for (uint32_t t = 0; t < (1u << 20); ++t)
-          if (mbar_try_wait(&full_bar[s], (s_issued[s] - 1u) & 1u)) break;
+        bool landed = false;
+        for (uint32_t t = 0; t < (1u << 20) && !landed; ++t)
+          landed = mbar_try_wait(&full_bar[s], (s_issued[s] - 1u) & 1u);
+        // bulk copies still in flight as the CTA exits: recorded apart
+        if (!landed) atomicOr(&ds->err, ERR_DRAIN);
       }
     }
   }

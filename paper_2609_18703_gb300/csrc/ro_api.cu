@@ -364,7 +364,11 @@ ro_status sync_and_check(ro_ctx* c) {
   const uint32_t err = c->hs->err;
   if (!err) return RO_OK;
   cudaMemsetAsync(&c->ds->err, 0, sizeof(uint32_t), c->stream);
-  if (err & ERR_TIMEOUT) return fail(c, RO_E_TIMEOUT, "a device-side wait timed out");
+  if (err & ERR_TIMEOUT)
+    return fail(c, RO_E_TIMEOUT, (err & ERR_DRAIN)
+                                     ? "a device-side wait timed out (a copy CTA exited with bulk "
+                                       "copies still in flight)"
+                                     : "a device-side wait timed out");
   if (err & ERR_OVERFLOW) return fail(c, RO_E_OVERFLOW, "an assembled parent exceeds 2^32-1 bytes");
   if (err & ERR_CAPACITY) return fail(c, RO_E_CAPACITY, "an output buffer is too small");
   return fail(c, RO_E_INVAL, "a device count or arena offset exceeded its bound");

@@ -70,6 +70,9 @@ enum : uint32_t {
   ERR_TIMEOUT = 2u,
   ERR_OVERFLOW = 4u,
   ERR_INVAL = 8u,
+  // a copy CTA that gave up waiting exited with bulk copies into its shared
+  // memory possibly still in flight (only after ERR_TIMEOUT)
+  ERR_DRAIN = 16u,
 };
 
 // Header of a list of completed parents to assemble (see ListBufs).

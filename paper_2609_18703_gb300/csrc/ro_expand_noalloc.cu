@@ -211,6 +211,7 @@ extern "C" ro_status ro_expand_noalloc(const uint32_t* d_counts, uint64_t n_pare
   }
   expand_scan_noalloc_kernel<<<sms * 2, EXP_THREADS, 0, s>>>(d_counts, n_parents, d_offsets,
                                                             d_empty_parents, scratch);
+  if (cudaGetLastError() != cudaSuccess) return RO_E_CUDA;   // not launched: the header is stale
   NaHeader hh{};
   cudaError_t e = cudaMemcpyAsync(&hh, scratch, sizeof(NaHeader), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
@@ -232,5 +233,12 @@ extern "C" ro_status ro_expand_noalloc(const uint32_t* d_counts, uint64_t n_pare
   expand_fill_noalloc_kernel<<<grid, FILL_THREADS, 0, s>>>(d_offsets, n_parents, N, d_child_parent,
                                                           d_child_ordinal, scratch);
   if (cudaGetLastError() != cudaSuccess) return RO_E_CUDA;
+  // The fill reads the shared scratch (its per-tile parent table): return
+  // only once it is done, so that a caller who takes the return as
+  // completion may start the next call from any stream or thread.
+  if (cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return RO_E_CUDA;
+  }
   return RO_OK;
 }

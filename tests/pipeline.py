@@ -8,13 +8,9 @@ from __future__ import annotations
 
 import numpy as np
 
-from workload import FAILED, PRESENT, SUPPRESSED, Level, fill_host_arena, record_bytes
+from workload import FAILED, PRESENT, SUPPRESSED, Level, level_arena, record_bytes
 
-
-def host_arena(lv: Level) -> np.ndarray:
-    n = lv.n_children
-    return fill_host_arena(lv.payload_seed, np.arange(n, dtype=np.uint64), lv.arena_off,
-                           lv.length, lv.arena_bytes)
+host_arena = level_arena   # the level's host result arena (input generation)
 
 
 def closed_form_lineage(counts: np.ndarray):

@@ -5,10 +5,10 @@ readiness orders, and fills result payload bytes from a counter-based hash.
 """
 from .configs import (CONFIGS, FAILED, DROPPED, PRESENT, SUPPRESSED, Level, Workload,
                       docpage, skew, streaming, tiny, video)
-from .payload import fill_host_arena, mix64, record_bytes, records_concat
+from .payload import fill_host_arena, level_arena, mix64, record_bytes, records_concat
 
 __all__ = [
     "CONFIGS", "PRESENT", "DROPPED", "FAILED", "SUPPRESSED", "Level", "Workload",
     "tiny", "docpage", "video", "skew", "streaming",
-    "fill_host_arena", "mix64", "record_bytes", "records_concat",
+    "fill_host_arena", "level_arena", "mix64", "record_bytes", "records_concat",
 ]

@@ -132,3 +132,11 @@ def fill_host_arena(seed: int, children: np.ndarray, offsets: np.ndarray,
         arena[dst] = by[valid]
         start = end
     return arena
+
+
+def level_arena(lv) -> np.ndarray:
+    """The host result arena of a workload level: every child's record at
+    its arena offset (FAILED children have none)."""
+    n = lv.n_children
+    return fill_host_arena(lv.payload_seed, np.arange(n, dtype=np.uint64), lv.arena_off,
+                           lv.length, lv.arena_bytes)
