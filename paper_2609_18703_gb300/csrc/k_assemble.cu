@@ -4,7 +4,7 @@
 // otherwise Present with the Present members' payloads concatenated by
 // ordinal (Dropped members add nothing).  The work is a segmented byte gather
 // from the result arena in three steps:
-//   asm_parents  (caller's lists only; commit_finish does this for the
+//   asm_parents  (caller's lists only; commit_plan does this for the
 //                parents a commit completed) per listed parent: outcome,
 //                members to gather (0 unless Present), their exclusive scan
 //                (member bases), and for every AM_TILE-member tile the parent
@@ -173,6 +173,7 @@ __global__ void __maxnreg__(56) asm_members_kernel(AssembleArgs a) {
       pl.hdr->nnz = 0;
       pl.hdr->M = M;
       pl.hdr->incomplete = 0;
+      pl.hdr->max_end = 0;
       pl.hdr->err = 1u;
       L.hdr->incomplete = 0;   // spent (asm_parents adds to it)
       if (elems_too_many) atomicOr(&ds->err, ERR_CAPACITY);
@@ -199,6 +200,7 @@ __global__ void __maxnreg__(56) asm_members_kernel(AssembleArgs a) {
       pl.hdr->nnz = 0;
       pl.hdr->M = 0;
       pl.hdr->incomplete = lh.incomplete;
+      pl.hdr->max_end = 0;
       pl.hdr->err = 0u;
       pl.hdr->chunks_ok = 1u;
       L.hdr->incomplete = 0;   // spent (asm_parents adds to it)
@@ -352,6 +354,7 @@ __global__ void __maxnreg__(56) asm_members_kernel(AssembleArgs a) {
       pl.hdr->nnz = run.b;
       pl.hdr->M = M;
       pl.hdr->incomplete = lh.incomplete;
+      pl.hdr->max_end = 0;   // checked here, member by member
       pl.hdr->chunks_ok = ceil_div(run.a, AC_CHUNK) <= pl.ctfp_cap ? 1u : 0u;
     }
     __syncthreads();
@@ -916,6 +919,10 @@ __global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
   const uint64_t base = a.cursor ? *a.cursor : 0ull;
   // conditions every CTA sees the same way
   bool failed = hdr.err != 0u;
+  if (!failed && hdr.max_end > a.arena_bytes) {   // the arena passed here must hold what was accepted
+    failed = true;
+    if (threadIdx.x == 0) atomicOr(&ds->err, ERR_INVAL);
+  }
   const bool too_many = !a.user_list && n > a.n_host;   // outputs hold fewer parents
   const bool too_big = base + S > a.out_cap;
   if (!failed && (too_many || too_big)) {

@@ -19,13 +19,9 @@
 //                 it orders the repeats and applies the barriers, so the
 //                 result equals applying the reports one by one in array
 //                 order; otherwise it returns at once.
-// commit_finish   turns the bitmap into the ascending list of completed
-//                 parents and their member bases (one single-pass scan over
-//                 bitmap words of (popcount, word total)) and clears it; the
-//                 list is what ro_assemble(NULL) plans and copies.  It reads
-//                 only the bitmap, the per-parent member counts and offsets,
-//                 so with several bitmaps (commits take them in turn) it runs
-//                 on its own stream while the next commits' scatters run.
+// The completed list and its copy plan come next, from commit_plan
+// (k_complete.cu), which may run on another stream while later commits'
+// scatters run (commits take completion bitmaps in turn).
 #include <algorithm>
 
 #include "ro_internal.h"
@@ -629,110 +625,6 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
   __syncthreads();
 }
 
-// Completed-parent list, ascending, with each parent's outcome, first child
-// and member base, and the member-tile table asm_members works from.
-__global__ void __launch_bounds__(CF_THREADS) commit_finish_kernel(CommitArgs a) {
-  wait_predecessor();
-  __shared__ Pair64 s_scan[33];
-  __shared__ uint32_t s_tile;
-  __shared__ Pair64 s_prefix;
-  DevScalars* ds = a.ds;
-  const ListBufs& L = a.list;
-  const uint64_t n_words = ceil_div(a.P, 32);
-  const uint64_t n_tiles = ceil_div(n_words, (uint64_t)CF_THREADS);
-  if (n_tiles == 0) {
-    if (blockIdx.x == 0 && threadIdx.x == 0) {
-      ds->cm_n_done = 0;
-      L.hdr->n = 0;
-      L.hdr->M = 0;
-      L.hdr->err = 0u;
-      L.hdr->incomplete = 0;
-      L.mb[0] = 0;
-      if (a.n_done_out) *a.n_done_out = 0;
-    }
-    return;
-  }
-  const uint32_t n_part = participants(n_tiles);
-  if (blockIdx.x >= n_part) return;
-
-  for (;;) {
-    if (threadIdx.x == 0) s_tile = claim_tile(&ds->tile_ctr[TS_COMMIT]);
-    __syncthreads();
-    const uint32_t tile = s_tile;
-    __syncthreads();
-    if (tile >= n_tiles) break;
-    const uint64_t w = (uint64_t)tile * CF_THREADS + threadIdx.x;
-    const uint32_t bits = (w < n_words) ? __ldcg(a.bitmap + w) : 0u;
-    const uint32_t wsum0 = (w < n_words) ? __ldcg(a.wm + w) : 0u;   // loaded alongside the bits
-    const uint32_t wsum = bits ? wsum0 : 0u;
-    Pair64 total;
-    const Pair64 excl = block_excl_scan_pair(Pair64{(unsigned long long)__popc(bits), wsum}, s_scan, &total);
-    if (threadIdx.x < 32) {  // one warp looks back
-      const auto pfx = lookback_exclusive(a.ts, tile, total, ds->epoch[TS_COMMIT], &ds->err);
-      if (threadIdx.x == 0) s_prefix = pfx;
-    }
-    __syncthreads();
-    Pair64 run = s_prefix + excl;   // (completed parents, members) before my word
-    if (bits) {
-      uint32_t b = bits;
-      while (b) {
-        // up to four completed parents at a time: their loads first, then
-        // the writes (a load after a store would wait for it)
-        constexpr int G = 4;
-        uint32_t par[G], m[G], cf[G];
-        int cnt = 0;
-#pragma unroll
-        for (int u = 0; u < G; ++u) {
-          if (b) {
-            par[u] = (uint32_t)(w * 32 + (__ffs(b) - 1));
-            b &= b - 1;
-            cnt = u + 1;
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < G; ++u) {
-          if (u < cnt) {
-            m[u] = __ldcg(a.pm + par[u]);
-            cf[u] = (uint32_t)__ldg(a.offsets + par[u]);
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < G; ++u) {
-          if (u >= cnt) break;
-          const unsigned long long i = run.a;
-          a.done_int[i] = par[u];
-          if (a.done_user) a.done_user[i] = par[u];
-          L.status[i] = m[u] ? ST_PRESENT : ST_SUPPRESSED;
-          L.mb[i] = (uint32_t)run.b;
-          L.coff[i] = cf[u];
-          for (uint64_t t = ceil_div(run.b, AM_TILE); t * AM_TILE < run.b + m[u] && t < L.mtfp_cap; ++t)
-            L.mtfp[t] = (uint32_t)i;
-          run.a += 1;
-          run.b += m[u];
-        }
-      }
-      a.bitmap[w] = 0u;
-      a.wm[w] = 0u;
-    }
-    if (tile == n_tiles - 1 && threadIdx.x == CF_THREADS - 1) {
-      ds->cm_n_done = run.a;
-      L.hdr->n = run.a;
-      L.hdr->M = run.b;
-      L.hdr->err = 0u;
-      L.hdr->incomplete = 0;
-      L.mb[run.a] = (uint32_t)run.b;
-      if (a.n_done_out) *a.n_done_out = run.a;
-    }
-  }
-  if (threadIdx.x == 0) {
-    if (ticket(&ds->exit_ctr[TS_COMMIT]) == n_part - 1) {
-      ds->tile_ctr[TS_COMMIT] = 0u;
-      ds->exit_ctr[TS_COMMIT] = 0u;
-      ds->epoch[TS_COMMIT] += 1ull;
-    }
-  }
-}
-
 void launch_commit_scatter(const LaunchCfg& L, const CommitArgs& a) {
   const uint64_t warps = ceil_div(a.n_host, 32);
   const int grid =
@@ -746,15 +638,8 @@ void launch_commit_scatter(const LaunchCfg& L, const CommitArgs& a) {
   launch_k(L, K_CFIX, commit_fix_kernel, grid_fix, CM_THREADS, 0, a);
 }
 
-void launch_commit_finish(const LaunchCfg& L, const CommitArgs& a) {
-  const uint64_t n_tiles = ceil_div(ceil_div(a.P, 32), (uint64_t)CF_THREADS);
-  const int grid_f = (int)std::max<uint64_t>(1, std::min<uint64_t>(n_tiles, (uint64_t)L.grid_cfinish));
-  launch_k(L, K_CFINISH, commit_finish_kernel, grid_f, CF_THREADS, 0, a);
-}
-
 const void* kernel_ptr_commit(int which) {
-  if (which == K_CFIX) return (const void*)commit_fix_kernel;
-  return which == K_COMMIT ? (const void*)commit_scatter_kernel : (const void*)commit_finish_kernel;
+  return which == K_CFIX ? (const void*)commit_fix_kernel : (const void*)commit_scatter_kernel;
 }
 
 }  // namespace ro

@@ -25,6 +25,7 @@ size_t asm_copy_smem();
 const void* kernel_ptr_expand(int which);
 const void* kernel_ptr_ready(int which);
 const void* kernel_ptr_commit(int which);
+const void* kernel_ptr_complete();
 const void* kernel_ptr_assemble(int which);
 const void* kernel_ptr_retry(int which);
 const void* kernel_ptr_parent(int which);
@@ -56,10 +57,14 @@ struct QueueBufs {
   bool ready = false;   // state zeroed for the current expansion
 };
 
-// A list of completed parents (written by a commit, read by planning).
+// A list of completed parents with its copy plan (written by a commit's
+// commit_plan; read by the copy, or by planning for an explicit assembly).
 struct ListSlot {
   DevBuf done, status, mb, coff, mtfp, hdr;
-  Ev freed;   // the assembly that read it is done
+  DevBuf poff, pcpos, pcsrc, pctfp, phdr;   // the copy plan
+  uint64_t pctfp_cap = 0;
+  Ev freed;     // the assembly that read it is done
+  Ev planned;   // the commit_plan that wrote it is done (the next writer may run on the other stream)
 };
 // An assembly plan (written by planning, read by the copy).
 struct PlanSlot {
@@ -137,12 +142,16 @@ struct ro_ctx {
   cudaStream_t stream = nullptr;        // expansion, admission, commit
   cudaStream_t plan_stream = nullptr;   // assembly planning
   cudaStream_t copy_stream = nullptr;   // assembly copies
-  cudaStream_t fin_stream = nullptr;    // completion scans (commit_finish)
-  cudaStream_t own_fin = nullptr;       // created for fin_stream, destroyed with the context
+  // Completion lists and their plans (commit_plan): with separate streams,
+  // commits of even and odd sequence alternate between two streams, so the
+  // plans of consecutive commits run at the same time.
+  cudaStream_t fin_stream[2] = {nullptr, nullptr};
+  cudaStream_t own_fin[2] = {nullptr, nullptr};   // created for fin_stream, destroyed with the context
+  int last_fin = 0;                     // the stream of the latest commit's plan
   uint32_t n_calls = 1;
   uint32_t commit_seq = 0;              // commits issued on this context
   int num_sms = 0;
-  LaunchCfg L{}, Lp{}, Lc{}, Lf{};
+  LaunchCfg L{}, Lp{}, Lc{}, Lf[2]{};
   DevScalars* ds = nullptr;
   DevScalars* hs = nullptr;   // pinned mirror
   ReadyScalars* rs = nullptr;   // per Call, device
@@ -163,7 +172,7 @@ struct ro_ctx {
   // parent-bound reservation scratch (see ParentArgs)
   DevBuf pb_key[2], pb_val[2], pb_child, pb_hist, pb_dtot, pb_first, pb_endp, pb_hsz, pb_left,
       pb_hoff, pb_rem;
-  Ev fork, x_planned, join_plan, join_copy, fin_fork, fin_join, fin_plan;
+  Ev fork, x_planned, join_plan, join_copy, fin_fork[2], fin_join[2], fin_plan;
   // Caller memory written by the copies issued since the context's stream
   // last waited for the copy stream: a later call's planning (another
   // stream) may run while they do, so planning that writes any of it waits
@@ -235,7 +244,8 @@ void sync_all_streams(ro_ctx* c) {
   cudaStreamSynchronize(c->stream);
   if (c->plan_stream != c->stream) cudaStreamSynchronize(c->plan_stream);
   if (c->copy_stream != c->stream) cudaStreamSynchronize(c->copy_stream);
-  if (c->fin_stream != c->stream) cudaStreamSynchronize(c->fin_stream);
+  for (cudaStream_t s : c->fin_stream)
+    if (s != c->stream) cudaStreamSynchronize(s);
   for (cudaStream_t s : c->call_stream)
     if (s != c->stream) cudaStreamSynchronize(s);
 }
@@ -321,7 +331,7 @@ ro_status settle_calls(ro_ctx* c) {
 
 ro_status join(ro_ctx* c) {
   RO_TRY(settle_calls(c));
-  RO_TRY(order(c, c->fin_join, c->fin_stream, c->stream));
+  for (int k = 0; k < 2; ++k) RO_TRY(order(c, c->fin_join[k], c->fin_stream[k], c->stream));
   RO_TRY(order(c, c->join_plan, c->plan_stream, c->stream));
   if (c->copy_stream != c->plan_stream) RO_TRY(order(c, c->join_copy, c->copy_stream, c->stream));
   // planning forks from the context's stream: it now follows every copy
@@ -335,9 +345,10 @@ ro_status join(ro_ctx* c) {
 template <class T>
 ro_status tile_status_buf(ro_ctx* c, TsBuf& t, size_t tiles, TileStatus<T>* out) {
   tiles = std::max<size_t>(tiles, 1);
+  const size_t el = std::max(sizeof(T), sizeof(Pair64));
   RO_TRY(ensure(c, t.flag, tiles * sizeof(unsigned long long), "scan flags"));
-  RO_TRY(ensure(c, t.agg, tiles * sizeof(Pair64), "scan aggregates"));
-  RO_TRY(ensure(c, t.inc, tiles * sizeof(Pair64), "scan prefixes"));
+  RO_TRY(ensure(c, t.agg, tiles * el, "scan aggregates"));
+  RO_TRY(ensure(c, t.inc, tiles * el, "scan prefixes"));
   out->flag = (unsigned long long*)t.flag.p;
   out->agg = (T*)t.agg.p;
   out->inc = (T*)t.inc.p;
@@ -418,6 +429,18 @@ ListBufs list_bufs(ListSlot& s, uint64_t mtfp_cap) {
   return l;
 }
 
+PlanBufs list_plan_bufs(ListSlot& s, uint64_t member_cap) {
+  PlanBufs p;
+  p.off = (uint64_t*)s.poff.p;
+  p.cpos = (uint64_t*)s.pcpos.p;
+  p.csrc = (uint64_t*)s.pcsrc.p;
+  p.member_cap = member_cap;
+  p.ctfp = (uint32_t*)s.pctfp.p;
+  p.ctfp_cap = s.pctfp_cap;
+  p.hdr = (PlanHdr*)s.phdr.p;
+  return p;
+}
+
 PlanBufs plan_bufs(PlanSlot& s, uint64_t member_cap) {
   PlanBufs p;
   p.off = (uint64_t*)s.off.p;
@@ -493,7 +516,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->stream = (cudaStream_t)stream;
   c->plan_stream = c->stream;
   c->copy_stream = c->stream;
-  c->fin_stream = c->stream;
+  c->fin_stream[0] = c->fin_stream[1] = c->stream;
   c->n_calls = n_calls;
   cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
   if (cudaMalloc(&c->ds, sizeof(DevScalars)) != cudaSuccess ||
@@ -527,7 +550,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_fill = grid_for(kernel_ptr_expand(K_FILL), FILL_THREADS, s, 8);
   c->L.grid_rb = grid_for(kernel_ptr_ready(K_RB_SCATTER), RB_THREADS, s, 8);
   c->L.grid_commit = grid_for(kernel_ptr_commit(K_COMMIT), CM_THREADS, s, 8);
-  c->L.grid_cfinish = grid_for(kernel_ptr_commit(K_CFINISH), CF_THREADS, s, 4);
+  c->L.grid_cplan = grid_for(kernel_ptr_complete(), CP_THREADS, s, 4);
   c->L.grid_aparents = grid_for(kernel_ptr_assemble(K_APARENTS), AP_THREADS, s, 4);
   // up to 4 planning CTAs per SM: large waves (100k-member parents) get the
   // parallelism; beside a running copy only one fits and the rest wait
@@ -538,7 +561,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_pb_sort = grid_for(kernel_ptr_parent(K_PB_SORT), PB_THREADS, s, 8);
   c->Lp = c->L;
   c->Lc = c->L;
-  c->Lf = c->L;
+  c->Lf[0] = c->Lf[1] = c->L;
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) {
     free_scalars(c);
@@ -559,7 +582,8 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
     for (auto& e : s.bm_free) free_ev(e);
     for (auto& l : s.lists) {
       free_buf(l.done); free_buf(l.status); free_buf(l.mb); free_buf(l.coff); free_buf(l.mtfp);
-      free_buf(l.hdr); free_ev(l.freed);
+      free_buf(l.hdr); free_buf(l.poff); free_buf(l.pcpos); free_buf(l.pcsrc); free_buf(l.pctfp);
+      free_buf(l.phdr); free_ev(l.freed); free_ev(l.planned);
     }
     for (auto& p : s.plans) {
       free_buf(p.off); free_buf(p.cpos); free_buf(p.csrc); free_buf(p.ctfp);
@@ -580,8 +604,12 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
                     &c->pb_hoff, &c->pb_rem})
     free_buf(*b);
   free_ev(c->fork); free_ev(c->x_planned); free_ev(c->join_plan); free_ev(c->join_copy);
-  free_ev(c->fin_fork); free_ev(c->fin_join); free_ev(c->fin_plan); free_ev(c->copy_done);
-  if (c->own_fin) cudaStreamDestroy(c->own_fin);
+  for (int k = 0; k < 2; ++k) {
+    free_ev(c->fin_fork[k]);
+    free_ev(c->fin_join[k]);
+    if (c->own_fin[k]) cudaStreamDestroy(c->own_fin[k]);
+  }
+  free_ev(c->fin_plan); free_ev(c->copy_done);
   for (cudaEvent_t e : c->prof.pool) cudaEventDestroy(e);
   for (auto& t : c->ts_call) {
     free_buf(t.flag); free_buf(t.agg); free_buf(t.inc);
@@ -609,23 +637,25 @@ ro_status ro_ctx_set_streams(ro_ctx* c, void* plan_stream, void* copy_stream) {
   c->plan_stream = plan_stream ? (cudaStream_t)plan_stream : c->stream;
   c->copy_stream = copy_stream ? (cudaStream_t)copy_stream : c->stream;
   // with streams of its own for assembly, the context also runs the
-  // completion scans on a stream of its own, so a commit's scan overlaps the
-  // next commit's scatter
+  // completion lists and plans on two streams of its own, so a commit's plan
+  // overlaps the next commits' scatters and the next commit's plan
   if (c->plan_stream != c->stream) {
-    if (!c->own_fin) {
-      cudaError_t e = cudaStreamCreateWithFlags(&c->own_fin, cudaStreamNonBlocking);
-      if (e != cudaSuccess) {
-        c->own_fin = nullptr;
-        return cuda_fail(c, e, "cudaStreamCreate");
+    for (int k = 0; k < 2; ++k) {
+      if (!c->own_fin[k]) {
+        cudaError_t e = cudaStreamCreateWithFlags(&c->own_fin[k], cudaStreamNonBlocking);
+        if (e != cudaSuccess) {
+          c->own_fin[k] = nullptr;
+          return cuda_fail(c, e, "cudaStreamCreate");
+        }
       }
+      c->fin_stream[k] = c->own_fin[k];
     }
-    c->fin_stream = c->own_fin;
   } else {
-    c->fin_stream = c->stream;
+    c->fin_stream[0] = c->fin_stream[1] = c->stream;
   }
   c->Lp.stream = c->plan_stream;
   c->Lc.stream = c->copy_stream;
-  c->Lf.stream = c->fin_stream;
+  for (int k = 0; k < 2; ++k) c->Lf[k].stream = c->fin_stream[k];
   return RO_OK;
 }
 
@@ -768,6 +798,10 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
     RO_TRY(ensure(c, l.coff, P * sizeof(uint32_t), "member bases"));
     RO_TRY(ensure(c, l.mtfp, mtfp_cap * sizeof(uint32_t), "member tiles"));
     RO_TRY(ensure(c, l.hdr, sizeof(ListHdr), "list header"));
+    RO_TRY(ensure(c, l.poff, (P + 1) * sizeof(uint64_t), "assembly plan"));
+    RO_TRY(ensure(c, l.pcpos, N * sizeof(uint64_t), "assembly plan"));
+    RO_TRY(ensure(c, l.pcsrc, N * sizeof(uint64_t), "assembly plan"));
+    RO_TRY(ensure(c, l.phdr, sizeof(PlanHdr), "assembly plan"));
   }
   for (auto& p : S.plans) {
     RO_TRY(ensure(c, p.off, (P + 1) * sizeof(uint64_t), "assembly plan"));
@@ -1061,24 +1095,42 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.n_done_out = d_n_done;
   ca.offsets = (const uint64_t*)S.offsets.p;
   ca.list = list_bufs(LS, ceil_div(x->N, AM_TILE) + 2);
+  // the chunk table of the plan: one entry per 16 KB of the arena the
+  // reports reference (a plan that needs more makes the copy search instead)
+  const uint64_t want_chunks = std::min<uint64_t>(ceil_div(arena_bytes, AC_CHUNK) + 2, 1ull << 31);
+  if (LS.pctfp_cap < want_chunks) {
+    RO_TRY(ensure(c, LS.pctfp, want_chunks * sizeof(uint32_t), "chunk table"));
+    LS.pctfp_cap = LS.pctfp.cap / sizeof(uint32_t);
+  }
+  ca.plan = list_plan_bufs(LS, std::max<uint64_t>(x->N, 1));
   ca.ds = c->ds;
-  RO_TRY(tile_status(c, TS_COMMIT, ceil_div(ceil_div(x->P, 32), (uint64_t)CF_THREADS), &ca.ts));
+  // consecutive commits plan on alternate streams, each with a scan slot of its own
+  const int pf = (int)(c->commit_seq & 1u);
+  ca.pslot = pf;
+  RO_TRY(tile_status(c, pf ? TS_COMMIT_ODD : TS_COMMIT, ceil_div(ceil_div(x->P, 32), (uint64_t)CP_WORDS),
+                     &ca.tsq));
   // the bitmap slot is free once the completion scan BM_SLOTS commits ago is done
   RO_TRY(ev_wait(c, S.bm_free[bs], c->stream));
   launch_commit_scatter(c->L, ca);
-  // the completion scan follows the scatter (on its own stream when the
-  // context has one); the list slot is free once the assembly that read it
-  // (RING commits ago) is done
-  RO_TRY(order(c, c->fin_fork, c->stream, c->fin_stream));
-  RO_TRY(ev_wait(c, LS.freed, c->fin_stream));
-  launch_commit_finish(c->Lf, ca);
-  if (c->fin_stream != c->stream) RO_TRY(ev_record(c, S.bm_free[bs], c->fin_stream));
+  // the completed list and its plan follow the scatter (on their own stream
+  // when the context has one); the list slot is free once the assembly that
+  // read it (RING commits ago) is done
+  const cudaStream_t fs = c->fin_stream[pf];
+  RO_TRY(order(c, c->fin_fork[pf], c->stream, fs));
+  RO_TRY(ev_wait(c, LS.freed, fs));
+  RO_TRY(ev_wait(c, LS.planned, fs));
+  launch_commit_plan(c->Lf[pf], ca);
+  if (fs != c->stream) {
+    RO_TRY(ev_record(c, S.bm_free[bs], fs));
+    RO_TRY(ev_record(c, LS.planned, fs));
+  }
+  c->last_fin = pf;
   RO_TRY(check_launch(c, "gather_commit"));
   x->last_list = ls;
   x->commits += 1;
   if (h_n_done) {
     ro_status st = sync_and_check(c);
-    *h_n_done = c->hs->cm_n_done;
+    *h_n_done = c->hs->cm_n_done[pf];
     return st;
   }
   return RO_OK;
@@ -1173,12 +1225,17 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   ExpSlot& S = c->slots[xid];
   const uint64_t member_cap = std::max<uint64_t>(x->N, 1);
   const uint64_t mtfp_cap = ceil_div(member_cap, AM_TILE) + 2;
+  // The commit's own list without list structure was planned by the commit
+  // (commit_plan): only the copy runs.  Otherwise plan here, into a plan slot.
+  const bool planned = !d_parents && !eo;
   PlanSlot& PS = S.plans[x->assembles % RING];
-  // chunk table: one entry per 16 KB of output (the copy searches beyond it)
-  const uint64_t want_chunks = std::min<uint64_t>(ceil_div(out_cap, AC_CHUNK) + 2, 1ull << 31);
-  if (PS.ctfp_cap < want_chunks) {
-    RO_TRY(ensure(c, PS.ctfp, want_chunks * sizeof(uint32_t), "chunk table"));
-    PS.ctfp_cap = PS.ctfp.cap / sizeof(uint32_t);
+  if (!planned) {
+    // chunk table: one entry per 16 KB of output (the copy searches beyond it)
+    const uint64_t want_chunks = std::min<uint64_t>(ceil_div(out_cap, AC_CHUNK) + 2, 1ull << 31);
+    if (PS.ctfp_cap < want_chunks) {
+      RO_TRY(ensure(c, PS.ctfp, want_chunks * sizeof(uint32_t), "chunk table"));
+      PS.ctfp_cap = PS.ctfp.cap / sizeof(uint32_t);
+    }
   }
   AssembleArgs aa{};
   aa.user_list = d_parents;
@@ -1210,7 +1267,15 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   aa.plan = plan_bufs(PS, member_cap);
   aa.ds = c->ds;
   ListSlot* LS = nullptr;
-  if (d_parents) {
+  if (planned) {
+    LS = &S.lists[x->last_list];
+    aa.list = list_bufs(*LS, mtfp_cap);
+    aa.plan = list_plan_bufs(*LS, member_cap);
+    // the copy follows the context's stream (the caller's cursor and
+    // outputs) and the commit's plan
+    RO_TRY(order(c, c->fork, c->stream, c->copy_stream));
+    RO_TRY(order(c, c->fin_plan, c->fin_stream[c->last_fin], c->copy_stream));
+  } else if (d_parents) {
     // a caller's list may be longer than the expansion's parents (repeats)
     RO_TRY(ensure(c, PS.off, (n_parents + 1) * sizeof(uint64_t), "assembly plan"));
     aa.plan.off = (uint64_t*)PS.off.p;
@@ -1231,49 +1296,51 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
     LS = &S.lists[x->last_list];
     aa.list = list_bufs(*LS, mtfp_cap);
   }
-  RO_TRY(tile_status(c, TS_ASM_MEMBERS, ceil_div(member_cap, (uint64_t)AM_TILE), &aa.ts_members));
+  if (!planned) {
+    RO_TRY(tile_status(c, TS_ASM_MEMBERS, ceil_div(member_cap, (uint64_t)AM_TILE), &aa.ts_members));
 
-  // planning follows everything enqueued on the context's stream so far,
-  // and the copy that last read this plan slot
-  RO_TRY(order(c, c->fork, c->stream, c->plan_stream));
-  RO_TRY(order(c, c->fin_plan, c->fin_stream, c->plan_stream));   // the commit's completion list
-  RO_TRY(ev_wait(c, PS.freed, c->plan_stream));
-  if (c->plan_stream != c->copy_stream) {
-    // caller memory planning writes (list structure; a caller's list's
-    // outcomes) against what copies still in flight write
-    ro_ctx::Span pw[5];
-    int npw = 0;
-    auto span = [](const void* p, uint64_t bytes) {
-      return ro_ctx::Span{(uintptr_t)p, (uintptr_t)p + (uintptr_t)bytes};
-    };
-    if (d_parents) pw[npw++] = span(d_status, n_parents);
-    if (eo) {
-      pw[npw++] = span(eo->base, (n_parents + 1) * sizeof(uint64_t));
-      pw[npw++] = span(eo->state, eo->cap);
-      pw[npw++] = span(eo->off, eo->cap * sizeof(uint64_t));
-      pw[npw++] = span(eo->len, eo->cap * sizeof(uint32_t));
+    // planning follows everything enqueued on the context's stream so far,
+    // and the copy that last read this plan slot
+    RO_TRY(order(c, c->fork, c->stream, c->plan_stream));
+    RO_TRY(order(c, c->fin_plan, c->fin_stream[c->last_fin], c->plan_stream));   // the commit's list
+    RO_TRY(ev_wait(c, PS.freed, c->plan_stream));
+    if (c->plan_stream != c->copy_stream) {
+      // caller memory planning writes (list structure; a caller's list's
+      // outcomes) against what copies still in flight write
+      ro_ctx::Span pw[5];
+      int npw = 0;
+      auto span = [](const void* p, uint64_t bytes) {
+        return ro_ctx::Span{(uintptr_t)p, (uintptr_t)p + (uintptr_t)bytes};
+      };
+      if (d_parents) pw[npw++] = span(d_status, n_parents);
+      if (eo) {
+        pw[npw++] = span(eo->base, (n_parents + 1) * sizeof(uint64_t));
+        pw[npw++] = span(eo->state, eo->cap);
+        pw[npw++] = span(eo->off, eo->cap * sizeof(uint64_t));
+        pw[npw++] = span(eo->len, eo->cap * sizeof(uint32_t));
+      }
+      bool meet = npw > 0 && c->copy_spans_full;
+      for (int i = 0; i < npw && !meet; ++i)
+        for (const auto& b : c->copy_spans)
+          if (pw[i].lo < pw[i].hi && pw[i].lo < b.hi && b.lo < pw[i].hi) {
+            meet = true;
+            break;
+          }
+      if (meet) RO_TRY(ev_wait(c, c->copy_done, c->plan_stream));
     }
-    bool meet = npw > 0 && c->copy_spans_full;
-    for (int i = 0; i < npw && !meet; ++i)
-      for (const auto& b : c->copy_spans)
-        if (pw[i].lo < pw[i].hi && pw[i].lo < b.hi && b.lo < pw[i].hi) {
-          meet = true;
-          break;
-        }
-    if (meet) RO_TRY(ev_wait(c, c->copy_done, c->plan_stream));
+    launch_assemble_plan(c->Lp, aa);
+    RO_TRY(check_launch(c, "assemble (plan)"));
+    if (!LS && c->plan_stream != c->stream) {
+      // a caller's list is classified against the parents' counters as they
+      // are now: later commits wait for that
+      RO_TRY(order(c, c->x_planned, c->plan_stream, c->stream));
+    }
+    RO_TRY(order(c, PS.ready, c->plan_stream, c->copy_stream));
   }
-  launch_assemble_plan(c->Lp, aa);
-  RO_TRY(check_launch(c, "assemble (plan)"));
-  if (!LS && c->plan_stream != c->stream) {
-    // a caller's list is classified against the parents' counters as they
-    // are now: later commits wait for that
-    RO_TRY(order(c, c->x_planned, c->plan_stream, c->stream));
-  }
-  RO_TRY(order(c, PS.ready, c->plan_stream, c->copy_stream));
   launch_assemble_copy(c->Lc, aa);
   RO_TRY(check_launch(c, "assemble (copy)"));
   if (c->copy_stream != c->plan_stream) {
-    RO_TRY(ev_record(c, PS.freed, c->copy_stream));
+    if (!planned) RO_TRY(ev_record(c, PS.freed, c->copy_stream));
     RO_TRY(ev_record(c, c->copy_done, c->copy_stream));
     // what this copy writes of the caller's memory (the bytes of d_out are
     // written by copies only)

@@ -92,6 +92,8 @@ struct PlanHdr {
   uint32_t chunks_ok;        // the chunk table covers every chunk
   unsigned long long M;      // list entries (members of the listed Present parents)
   unsigned long long incomplete;   // listed entries that are not complete parents
+  unsigned long long max_end;      // largest arena end of a planned member, when the
+                                   // plan did not check it against the arena (else 0)
 };
 
 // Counters and small results that kernels hand to later kernels and to the
@@ -104,7 +106,7 @@ struct DevScalars {
   // ro_expand
   unsigned long long n_children, n_empty, last_nonempty_parent;
   // ro_gather_commit
-  unsigned long long cm_n, cm_n_done;
+  unsigned long long cm_n, cm_n_done[2];   // completed parents, per plan slot
   // per commit, in two slots (commit sequence & 1): duplicate candidates and
   // accepted GroupFailures the scatter saw; the next commit's scatter clears
   // the slot after this one
@@ -133,10 +135,11 @@ struct alignas(128) ReadyScalars {
   unsigned long long epoch;
   uint32_t rb_ticket, rb_err, tile_ctr, exit_ctr;
 };
-// Slot 1 is unused (each Call's admission counts in its ReadyScalars);
+// TS_COMMIT and TS_COMMIT_ODD: the completion lists and plans of commits of
+// even and odd sequence (they may run at the same time, on two streams);
 // 5: asm_copy's exit ticket.
-enum TileSlot { TS_EXPAND = 0, TS_COMMIT = 2, TS_ASM_PARENTS = 3, TS_ASM_MEMBERS = 4,
-                TS_RETRY = 6, TS_PARENT = 7 };
+enum TileSlot { TS_EXPAND = 0, TS_COMMIT_ODD = 1, TS_COMMIT = 2, TS_ASM_PARENTS = 3,
+                TS_ASM_MEMBERS = 4, TS_RETRY = 6, TS_PARENT = 7 };
 
 // Wait until the grid this launch depends on (programmatic dependent launch)
 // has completed and its memory is visible; a no-op without a dependency.
@@ -171,11 +174,22 @@ struct Pair64 {
   __device__ __forceinline__ Pair64 operator+(const Pair64& o) const { return {a + o.a, b + o.b}; }
 };
 
+// Four 64-bit values carried together; the fourth combines by maximum.
+struct Quad64 {
+  unsigned long long a, b, c, d;
+  __device__ __forceinline__ Quad64 operator+(const Quad64& o) const {
+    return {a + o.a, b + o.b, c + o.c, d > o.d ? d : o.d};
+  }
+};
+
 __device__ __forceinline__ unsigned long long load_cg(const unsigned long long* p) {
   return __ldcg(p);
 }
 __device__ __forceinline__ Pair64 load_cg(const Pair64* p) {
   return Pair64{__ldcg(&p->a), __ldcg(&p->b)};
+}
+__device__ __forceinline__ Quad64 load_cg(const Quad64* p) {
+  return Quad64{__ldcg(&p->a), __ldcg(&p->b), __ldcg(&p->c), __ldcg(&p->d)};
 }
 
 // Spin limit of every device-side wait: ~2^22 polls with a short sleep each
@@ -217,6 +231,18 @@ __device__ __forceinline__ void ts_publish(const TileStatus<T>& ts, uint32_t til
 __device__ __forceinline__ unsigned long long warp_sum(unsigned long long v) {
 #pragma unroll
   for (int d = 16; d > 0; d >>= 1) v += __shfl_xor_sync(0xffffffffu, v, d);
+  return v;
+}
+__device__ __forceinline__ Quad64 warp_sum(Quad64 v) {
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) {
+    Quad64 o;
+    o.a = __shfl_xor_sync(0xffffffffu, v.a, d);
+    o.b = __shfl_xor_sync(0xffffffffu, v.b, d);
+    o.c = __shfl_xor_sync(0xffffffffu, v.c, d);
+    o.d = __shfl_xor_sync(0xffffffffu, v.d, d);
+    v = v + o;
+  }
   return v;
 }
 __device__ __forceinline__ Pair64 warp_sum(Pair64 v) {

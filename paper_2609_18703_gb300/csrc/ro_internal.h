@@ -15,7 +15,20 @@ constexpr int FILL_THREADS = 256;
 constexpr uint32_t FILL_SMEM_CAP = FILL_TILE + 256;           // offsets staged per fill tile
 constexpr int RB_THREADS = 256, RB_ITEMS = 8;                 // candidates per tile: 2048
 constexpr int CM_THREADS = 256;
-constexpr int CF_THREADS = 256;                               // bitmap words per tile (1 each)
+// commit_plan: a tile of CP_WORDS bitmap words (32 parents each, one word
+// per thread; CP_WORDS <= CP_THREADS); at most CP_CAP completed parents staged in shared memory at a
+// time, members in rounds of CP_ROUND.  At CP_MAXREG registers and ~27 KB of
+// shared memory a CTA fits beside two asm_copy CTAs on one SM.
+#ifndef RO_CP_WORDS
+#define RO_CP_WORDS 256
+#endif
+constexpr int CP_THREADS = 256;
+constexpr uint32_t CP_WORDS = RO_CP_WORDS;
+static_assert(CP_WORDS <= (uint32_t)CP_THREADS, "one bitmap word per thread at most");
+constexpr uint32_t CP_CAP = 2048;
+constexpr int CP_ITEMS = 4;
+constexpr uint32_t CP_ROUND = CP_THREADS * CP_ITEMS;
+#define CP_MAXREG 56
 constexpr int MB_ITEMS = 8;                                   // members per lane per step
 constexpr int AP_THREADS = 256, AP_ITEMS = 4;                 // listed parents per tile: 1024
 // members per tile: 1024.  At 56 registers and 17 KB of shared memory a CTA
@@ -37,7 +50,7 @@ constexpr uint32_t AC_BUF = 24576;
 constexpr uint32_t AC_SMALL = 64;   // pieces of at most this many staged bytes: cp.async, not a bulk copy
 
 // kernel entry points for occupancy queries and per-kernel timing
-enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CFINISH, K_APARENTS,
+enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CPLAN, K_APARENTS,
                 K_AMEMBERS, K_ACOPY, K_RT_CLAIM, K_RT_SCATTER, K_PB_KEYS, K_PB_HIST,
                 K_PB_ROWSCAN, K_PB_SORT, K_PB_BOUNDS, K_PB_HEADS, K_PB_MARK, K_PB_SCAN, K_PB_EMIT,
                 K_CFIX, K_COUNT };
@@ -51,7 +64,7 @@ void prof_end(Profiler* p, cudaStream_t s, int kid);
 struct LaunchCfg {
   cudaStream_t stream;
   Profiler* prof;
-  int grid_expand_scan, grid_fill, grid_rb, grid_commit, grid_cfinish, grid_aparents,
+  int grid_expand_scan, grid_fill, grid_rb, grid_commit, grid_cplan, grid_aparents,
       grid_amembers, grid_acopy, grid_retry, grid_pb, grid_pb_sort;
 };
 
@@ -183,7 +196,7 @@ void launch_retry(const LaunchCfg& L, const RetryArgs& a);
 
 // ---- lists and plans -------------------------------------------------------------------
 // A list of parents to assemble with its member bases: produced by
-// commit_finish (the parents a commit completed) or by asm_parents (a
+// commit_plan (the parents a commit completed) or by asm_parents (a
 // caller's list), consumed by asm_members.
 struct ListBufs {
   const uint32_t* parents;    // listed parent ids
@@ -195,8 +208,8 @@ struct ListBufs {
   ListHdr* hdr;
 };
 // The assembly plan of a list: everything the copy needs, with positions
-// relative to the start of that call's output.  Produced by asm_members,
-// consumed by asm_copy.
+// relative to the start of that call's output.  Produced by asm_members, or
+// by commit_plan for the commit's own list; consumed by asm_copy.
 struct PlanBufs {
   uint64_t* off;              // relative output offset per listed parent (+ total at [n])
   uint64_t* cpos;             // relative output position of each contributing member
@@ -233,14 +246,16 @@ struct CommitArgs {
   uint64_t* n_done_out;       // optional device output
   const uint64_t* offsets;
   ListBufs list;              // written: the completed parents with member bases
+  PlanBufs plan;              // written: the copy plan of that list
+  int pslot;                  // commit_plan's scan slot (0 / 1, alternating by commit)
   DevScalars* ds;
-  TileStatus<Pair64> ts;
+  TileStatus<Quad64> tsq;     // commit_plan's look-back
 };
-// the scatter (with the ordering of repeated reports and GroupFailure
-// barriers in its last CTA) and the completion scan, which may run on
+// the scatter (then the fix-up of repeated reports and GroupFailure
+// barriers) and the completion list with its copy plan, which may run on
 // different streams
 void launch_commit_scatter(const LaunchCfg& L, const CommitArgs& a);
-void launch_commit_finish(const LaunchCfg& L, const CommitArgs& a);
+void launch_commit_plan(const LaunchCfg& L, const CommitArgs& a);
 
 // ---- ro_assemble ---------------------------------------------------------------------
 struct AssembleArgs {

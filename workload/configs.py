@@ -216,6 +216,63 @@ def streaming(total_children: int = 50_000_000, batch_size: int = 256,
     return Workload(f"streaming {n_calls} Calls ({n} children, batch {batch_size})", [lv])
 
 
+def _restrict_order(order: np.ndarray, bounds: np.ndarray, keep_below: int):
+    """The entries of `order` below `keep_below`, in order, with the bounds of
+    the waves they fell in."""
+    n_w = bounds.size - 1
+    wave = np.repeat(np.arange(n_w, dtype=np.int64), np.diff(bounds))
+    keep = order < keep_below
+    kept = order[keep]
+    per = np.bincount(wave[keep], minlength=n_w)
+    return kept.astype(np.uint32), np.concatenate([[0], np.cumsum(per)]).astype(np.int64)
+
+
+def _repack(lv: Level, order: np.ndarray) -> None:
+    """Lay the PRESENT records out back to back in `order` (no padding)."""
+    ordered_len = lv.length[order].astype(np.uint64)
+    starts = np.cumsum(ordered_len) - ordered_len
+    off = np.zeros(lv.n_children, dtype=np.uint64)
+    off[order] = starts
+    lv.arena_off = np.where(lv.length > 0, off, 0).astype(np.uint64)
+    lv.arena_bytes = int(ordered_len.sum())
+
+
+def _head_level(lv: Level, parents: int) -> Level:
+    counts = lv.counts[:parents].copy()
+    n = int(counts.sum(dtype=np.uint64))
+    out = Level(counts=counts, n_children=n, batch_size=lv.batch_size, n_calls=lv.n_calls,
+                parent_call=None if lv.parent_call is None else lv.parent_call[:parents].copy(),
+                payload_seed=lv.payload_seed)
+    if lv.state is not None:
+        out.state = lv.state[:n].copy()
+        out.length = lv.length[:n].copy()
+    if lv.key is not None:
+        out.key = lv.key[:n].copy()
+    if lv.arrival is not None:
+        out.arrival, out.wave_bounds = _restrict_order(lv.arrival, lv.wave_bounds, n)
+    if lv.readiness is not None:
+        out.readiness, out.ready_bounds = _restrict_order(lv.readiness, lv.ready_bounds, n)
+    if out.length is not None:
+        # arrival order when there is one (configs 1-4), else child order
+        _repack(out, out.arrival if out.arrival is not None else np.arange(n, dtype=np.uint32))
+    return out
+
+
+def subset(wl: Workload, parents: int) -> Workload:
+    """The first `parents` top-level parents of a drawn workload with all
+    their descendants: the same draws (counts, outcomes, lengths, payload
+    seed, arrival and readiness orders restricted to the kept children, wave
+    by wave), the records packed into a smaller arena in the same order."""
+    levels = []
+    keep = parents
+    for lv in wl.levels:
+        keep = min(keep, lv.n_parents)
+        h = _head_level(lv, keep)
+        levels.append(h)
+        keep = h.n_children   # the next level's parents are these children
+    return Workload(f"{wl.name}, first {parents} parents", levels, wl.description)
+
+
 CONFIGS = {
     "tiny": tiny,
     "docpage": docpage,
