@@ -31,6 +31,9 @@
 namespace ro {
 
 constexpr int TS_ASM_COPY = 5;
+#ifndef RO_COPY_DYNAMIC
+#define RO_COPY_DYNAMIC 1
+#endif
 
 template <class V>
 __device__ __forceinline__ uint32_t last_le_u(const V* v, uint32_t lo, uint32_t hi, uint64_t x) {
@@ -529,9 +532,17 @@ __device__ __forceinline__ void cp_async_track(uint64_t* bar) {
 
 // Bounded wait on a stage barrier for the phase of parity `parity`; false
 // (recording ERR_TIMEOUT and raising the CTA's abort flag) if it gave up or
-// another warp of the CTA already did.
+// another warp of the CTA already did.  Called by every lane of a warp; the
+// answer is the same for the whole warp (false if any lane gave up), so the
+// warp's collective operations after it never see a split warp.
+__device__ __forceinline__ bool stage_wait_lane(uint64_t* bar, uint32_t parity, uint32_t* err,
+                                                volatile uint32_t* abort);
 __device__ __forceinline__ bool stage_wait2(uint64_t* bar, uint32_t parity, uint32_t* err,
                                             volatile uint32_t* abort) {
+  return __all_sync(0xffffffffu, stage_wait_lane(bar, parity, err, abort));
+}
+__device__ __forceinline__ bool stage_wait_lane(uint64_t* bar, uint32_t parity, uint32_t* err,
+                                                volatile uint32_t* abort) {
   // at most 2^20 polls of up to ~1 us each
   for (uint32_t i = 0; i < (1u << 20); ++i) {
     if (mbar_try_wait_sleep(bar, parity, 1000u)) return true;
@@ -566,6 +577,7 @@ struct CopyStage {
   __align__(16) unsigned char buf[AC_BUF + 32];
 };
 constexpr uint32_t AC_FALLBACK = 0xFFFFFFFFu;
+constexpr uint32_t AC_DONE = 0xFFFFFFFEu;      // no chunk: the consumers stop at this stage
 
 size_t asm_copy_smem() { return AC_STAGES * sizeof(CopyStage); }
 
@@ -912,6 +924,7 @@ __global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
   __shared__ __align__(8) uint64_t empty_bar[AC_STAGES];
   __shared__ uint32_t s_issued[AC_STAGES];
   __shared__ uint32_t s_abort;
+  __shared__ uint32_t s_round[2];   // the current and next claimed rounds (dynamic chunks)
   CopyStage* stages = reinterpret_cast<CopyStage*>(ac_smem);
   DevScalars* ds = a.ds;
   const PlanHdr hdr = *a.plan.hdr;
@@ -977,6 +990,76 @@ __global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
     }
     __syncthreads();
     volatile uint32_t* abort = &s_abort;
+#if RO_COPY_DYNAMIC
+    if (warp < AC_PRODUCERS) {
+      // Chunks are claimed in rounds of AC_PRODUCERS from a counter the grid
+      // shares, so a CTA that starts late (its SM busy with another stream's
+      // work) takes fewer: producer 0 claims the next round while this one
+      // is staged and hands each round to the other producer at a named
+      // barrier; stage index AC_PRODUCERS * r + warp holds chunk base_r +
+      // warp.  Both producers leave at the same round (the barrier needs
+      // both), and the first stage index left unfilled is marked done for
+      // the consumers.
+      ChunkDesc d;
+      uint32_t next = 0;
+      if (warp == 0 && lane == 0) next = atomicAdd(&ds->tile_ctr[TS_ASM_COPY], (uint32_t)AC_PRODUCERS);
+      uint32_t r = 0;
+      for (;; ++r) {
+        if (warp == 0 && lane == 0) {
+          // a wait that gave up stops both producers at the same round
+          s_round[r & 1u] = *abort ? 0xFFFFFFFFu : next;
+          if ((uint64_t)next < n_chunks)   // the claim of the following round, ahead
+            next = atomicAdd(&ds->tile_ctr[TS_ASM_COPY], (uint32_t)AC_PRODUCERS);
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(AC_PRODUCERS * 32) : "memory");
+        const uint64_t base_r = s_round[r & 1u];
+        if (base_r >= n_chunks) break;
+        const uint64_t k = base_r + (uint64_t)warp;
+        const uint32_t i = AC_PRODUCERS * r + (uint32_t)warp;
+        const uint32_t s = i % AC_STAGES, u = i / AC_STAGES;
+        if (k < n_chunks) describe_chunk(c, k, d, lane);
+        if (u > 0 && !stage_wait2(&empty_bar[s], (u - 1u) & 1u, &ds->err, abort)) continue;
+        if (k < n_chunks) {
+          issue_chunk(c, d, &stages[s], &full_bar[s], lane);
+        } else if (lane == 0) {   // the last round is short: the consumers stop here
+          stages[s].np = AC_DONE;
+          mbar_arrive(&full_bar[s]);
+        }
+        if (lane == 0) s_issued[s] = u + 1u;
+        __syncwarp();
+      }
+      const bool aborted = __any_sync(0xffffffffu, *abort != 0u);
+      if (warp == 0 && !aborted) {   // the first stage index left unfilled
+        const uint32_t i = AC_PRODUCERS * r;
+        const uint32_t s = i % AC_STAGES, u = i / AC_STAGES;
+        if (u == 0 || stage_wait2(&empty_bar[s], (u - 1u) & 1u, &ds->err, abort)) {
+          if (lane == 0) {
+            stages[s].np = AC_DONE;
+            mbar_arrive(&full_bar[s]);
+            s_issued[s] = u + 1u;
+          }
+        }
+        __syncwarp();
+      }
+      // this lane's cp.async copies of small pieces land before the CTA can
+      // exit (on an abort nobody else waits for them)
+      asm volatile("cp.async.wait_all;" ::: "memory");
+    } else {
+      const uint32_t cw = (uint32_t)(warp - AC_PRODUCERS);
+      for (uint32_t i = 0;; ++i) {
+        const uint32_t s = i % AC_STAGES, u = i / AC_STAGES;
+        if (!stage_wait2(&full_bar[s], u & 1u, &ds->err, abort)) break;
+        const uint32_t np = stages[s].np;
+        if (np == AC_DONE) break;
+        if (np == AC_FALLBACK)
+          emit_direct(c, &stages[s], cw, lane);
+        else
+          emit_range(&stages[s], cw, lane);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty_bar[s]);
+      }
+    }
+#else
     if (warp < AC_PRODUCERS) {
       // each chunk is described before its stage frees up: the loads of
       // chunk i+AC_PRODUCERS overlap the copies and the writing of chunk i
@@ -1011,6 +1094,7 @@ __global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
         if (lane == 0) mbar_arrive(&empty_bar[s]);
       }
     }
+#endif
     __syncthreads();
     // a wait that gave up: give the copies still in flight a bounded chance
     // to land before the CTA's shared memory is released
@@ -1034,6 +1118,7 @@ __global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
       ds->as_bytes = S;
       ds->as_elems = hdr.M;
       a.plan.hdr->err = 0u;   // the plan is consumed
+      ds->tile_ctr[TS_ASM_COPY] = 0u;   // the chunk counter, for the next copy
       ds->exit_ctr[TS_ASM_COPY] = 0u;
     }
   }

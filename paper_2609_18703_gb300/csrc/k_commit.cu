@@ -266,6 +266,7 @@ __device__ void apply_barriers_grid(const CommitArgs& a, uint64_t n) {
 // of the scatter so that the scatter's registers and shared memory stay small.
 __global__ void __launch_bounds__(CM_THREADS) commit_fix_kernel(CommitArgs a) {
   wait_predecessor();
+  allow_successor();   // the next commit's scatter launches now and waits for this grid
   DevScalars* ds = a.ds;
   const unsigned long long dups = ds->cm_conflicts[fix_slot(a)], gfs = ds->cm_gf[fix_slot(a)];
   if (dups == 0ull && gfs == 0ull) return;

@@ -55,6 +55,7 @@ enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CPL
                 K_PB_ROWSCAN, K_PB_SORT, K_PB_BOUNDS, K_PB_HEADS, K_PB_MARK, K_PB_SCAN, K_PB_EMIT,
                 K_CFIX, K_COUNT };
 
+
 // Launch counter and optional CUDA-event timing of selected kernels, on the
 // stream they are launched on (see ro_ctx_profile in the C ABI).
 struct Profiler;
