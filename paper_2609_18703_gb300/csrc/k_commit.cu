@@ -9,11 +9,8 @@
 //                 the same parent are merged first (__match_any_sync), so a
 //                 hot parent sees one atomic per warp.  The add that takes
 //                 `remaining` to zero completes the parent and sets its bit in
-//                 a completion bitmap.
-//                 That add also tells whether a member Failed or was
-//                 Suppressed, so the same thread records how many members the
-//                 parent will gather (0 if Suppressed) and adds it to its
-//                 bitmap word's total.
+//                 a completion bitmap (the counter's high half then tells
+//                 whether a member Failed or was Suppressed).
 // commit_fix      after the scatter, on the same stream: when the call
 //                 carried two reports for one Grain or a GroupFailure (rare)
 //                 it orders the repeats and applies the barriers, so the
@@ -64,7 +61,29 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n);
 __device__ void seal_open(const CommitArgs& a, uint32_t pp, int lane, unsigned long long* n_wait,
                           unsigned long long* n_fly);
 
+// Warm L2 with the lines of this warp's first 32 reports while the previous
+// kernel drains (addresses inside the report arrays' host-given length; L2 is
+// coherent, so nothing read later can be stale).
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+__device__ __forceinline__ void prefetch_reports(const CommitArgs& a) {
+  const int lane = threadIdx.x & 31;
+  const uint64_t r0 = (((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * 32;
+  if (r0 >= a.n_host) return;
+  switch (lane) {
+    case 0: prefetch_l2(a.child + r0); break;
+    case 1: prefetch_l2(a.len + r0); break;
+    case 2: prefetch_l2(a.off + r0); break;
+    case 3: if (r0 + 16 < a.n_host) prefetch_l2(a.off + r0 + 16); break;
+    case 4: prefetch_l2(a.state + r0); break;
+    case 5: if (a.gen) prefetch_l2(a.gen + r0); break;
+    default: break;
+  }
+}
+
 __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a) {
+  prefetch_reports(a);
   wait_predecessor();
   allow_successor();
   // verdict counts: accept, invalid, not in flight, stale, -, barrier,
@@ -148,15 +167,9 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
         const unsigned n_tot = __popc(grp), n_bad = __popc(grp & badm);
         const unsigned long long delta =
             ((unsigned long long)n_bad << 32) - (unsigned long long)n_tot;
-        // the parent's size, loaded alongside the count (used if it completes)
-        const uint32_t size = (uint32_t)(__ldg(a.offsets + p + 1) - __ldg(a.offsets + p));
         const unsigned long long old = atomicAdd(a.pw + p, delta);
-        if ((uint32_t)old == n_tot) {   // the last members: the parent is complete
-          const uint32_t m = (pw_bad(old) + n_bad) ? 0u : size;
-          a.pm[p] = m;
-          if (m) atomicAdd(a.wm + (p >> 5), m);
+        if ((uint32_t)old == n_tot)   // the last members: the parent is complete
           atomicOr(a.bitmap + (p >> 5), 1u << (p & 31));
-        }
       }
     }
     if (v <= V_DUP_CANDIDATE) cnt[v] += 1;
@@ -346,18 +359,11 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
     }
   }
   __syncthreads();
-  // E: a parent whose outcome class moved and that is complete gets its
-  //    member count to gather redone; then the verdicts become final
+  // E: the verdicts become final (a parent's outcome class moved with its
+  //    counter in D; the completion list reads it from there)
   for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
     const uint8_t v = a.code[r];
     if (v < V_WIN_SEALER || v > V_LOSE_CAND) continue;
-    const uint32_t p = a.rec[a.child[r]].parent;
-    const unsigned long long pv = __ldcg(a.pw + p);
-    if (pw_remaining(pv) == 0u) {
-      const uint32_t m = pw_bad(pv) ? 0u : (uint32_t)(a.offsets[p + 1] - a.offsets[p]);
-      const uint32_t old = atomicExch(a.pm + p, m);
-      if (old != m) atomicAdd(a.wm + (p >> 5), m - old);
-    }
     a.code[r] = (v == V_WIN_SEALER || v == V_WIN_CAND) ? V_ACCEPT : V_DUPLICATE;
   }
   __syncthreads();
@@ -395,10 +401,8 @@ __device__ void seal_open(const CommitArgs& a, uint32_t pp, int lane, unsigned l
     const unsigned long long k = (unsigned long long)k_wait + k_fly;
     if (k) {
       const unsigned long long old = atomicAdd(a.pw + pp, (k << 32) - k);
-      if ((uint32_t)old == k) {   // the barrier completes the parent
-        a.pm[pp] = 0u;
+      if ((uint32_t)old == k)   // the barrier completes the parent
         atomicOr(a.bitmap + (pp >> 5), 1u << (pp & 31));
-      }
     }
     atomicAdd(n_wait, (unsigned long long)k_wait);
     atomicAdd(n_fly, (unsigned long long)k_fly);

@@ -6,8 +6,9 @@
 // commit_plan  runs after a commit's scatter (and its fix-up), one pass over
 //              the commit's completion bitmap in tiles of CP_WORDS words
 //              (32 parents per word).  Per tile it finds the parents this
-//              commit completed, their members to gather (0 when
-//              Suppressed) and those members' records, then takes ONE
+//              commit completed, their members to gather (the parent's size
+//              from the offsets, or 0 when its counter records a Failed or
+//              Suppressed member) and those members' records, then takes ONE
 //              decoupled look-back over the tuple (parents | members << 32,
 //              payload bytes, contributing members, largest arena end).
 //              With that prefix it writes, in ascending parent order:
@@ -69,6 +70,42 @@ __device__ __forceinline__ void block_reduce3(unsigned long long& a, unsigned lo
   __syncthreads();
 }
 
+// A completed parent's members to gather (its size, or 0 when a member
+// Failed or was Suppressed: the parent is then Suppressed) and first child.
+__device__ __forceinline__ void parent_info(const CommitArgs& a, uint32_t p, uint32_t* m,
+                                            uint32_t* first) {
+  const unsigned long long v = __ldcg(a.pw + p);
+  const uint64_t o0 = __ldg(a.offsets + p), o1 = __ldg(a.offsets + p + 1);
+  *m = pw_bad(v) ? 0u : (uint32_t)(o1 - o0);
+  *first = (uint32_t)o0;
+}
+
+// Members gathered by the completed parents of bitmap word w (loads issued
+// four parents at a time, so they overlap).
+__device__ __forceinline__ uint32_t word_members(const CommitArgs& a, uint64_t w, uint32_t bits) {
+  uint32_t sum = 0;
+  while (bits) {
+    constexpr int G = 4;
+    uint32_t p[G], m[G], cf[G];
+    int cnt = 0;
+#pragma unroll
+    for (int u = 0; u < G; ++u) {
+      if (bits) {
+        p[u] = (uint32_t)(w * 32 + (uint32_t)(__ffs(bits) - 1));
+        bits &= bits - 1;
+        cnt = u + 1;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < G; ++u)
+      if (u < cnt) parent_info(a, p[u], &m[u], &cf[u]);
+#pragma unroll
+    for (int u = 0; u < G; ++u)
+      if (u < cnt) sum += m[u];
+  }
+  return sum;
+}
+
 struct CpShared {
   Pair64 scan[33];
   uint32_t wp[CP_WORDS + 1];    // per word: local list index of its first completed parent
@@ -107,12 +144,8 @@ __device__ void stage_group(const CommitArgs& a, CpShared& sh, uint64_t w, uint3
       }
     }
 #pragma unroll
-    for (int u = 0; u < G; ++u) {
-      if (u < cnt) {
-        m[u] = __ldcg(a.pm + p[u]);
-        cf[u] = (uint32_t)__ldg(a.offsets + p[u]);
-      }
-    }
+    for (int u = 0; u < G; ++u)
+      if (u < cnt) parent_info(a, p[u], &m[u], &cf[u]);
 #pragma unroll
     for (int u = 0; u < G; ++u) {
       if (u >= cnt) break;
@@ -220,12 +253,9 @@ __global__ void __maxnreg__(CP_MAXREG) commit_plan_kernel(CommitArgs a) {
     __syncthreads();
     if (tile >= n_tiles) break;
     const uint64_t w = (uint64_t)tile * CP_WORDS + threadIdx.x;
-    uint32_t bits = 0, wsum = 0;
-    if (threadIdx.x < CP_WORDS && w < n_words) {
-      bits = __ldcg(a.bitmap + w);
-      wsum = __ldcg(a.wm + w);   // loaded alongside the bits
-    }
-    if (!bits) wsum = 0;
+    uint32_t bits = 0;
+    if (threadIdx.x < CP_WORDS && w < n_words) bits = __ldcg(a.bitmap + w);
+    const uint32_t wsum = word_members(a, w, bits);
     Pair64 tot;
     const Pair64 ex = block_excl_scan_pair(Pair64{(unsigned long long)__popc(bits), wsum}, sh.scan, &tot);
     if (threadIdx.x < CP_WORDS) {
@@ -390,10 +420,7 @@ __global__ void __maxnreg__(CP_MAXREG) commit_plan_kernel(CommitArgs a) {
         if (sh.pmb[k] == mhi) pl.off[gp + g0 + k] = gb + carry_b;
       __syncthreads();   // the next group restages
     }
-    if (bits) {   // the bitmap slot is clean for its next commit
-      a.bitmap[w] = 0u;
-      a.wm[w] = 0u;
-    }
+    if (bits) a.bitmap[w] = 0u;   // the bitmap slot is clean for its next commit
   }
   if (threadIdx.x == 0) retire_cta(ds, slot, n_part);
 }

@@ -75,7 +75,7 @@ struct PlanSlot {
 
 // Device buffers of one expansion slot, kept across ro_ctx_reset and reused.
 struct ExpSlot {
-  DevBuf offsets, pw, phase, rec, bitmap, tfp, pm, wm, gb;   // bitmap, wm: two slots each
+  DevBuf offsets, pw, phase, rec, bitmap, tfp, gb;   // bitmap: BM_SLOTS slots
   Ev bm_free[BM_SLOTS];   // the completion scan that read a bitmap slot is done
   ListSlot lists[RING];
   PlanSlot plans[RING];
@@ -578,7 +578,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   sync_all_streams(c);
   for (auto& s : c->slots) {
     free_buf(s.offsets); free_buf(s.pw); free_buf(s.phase); free_buf(s.rec); free_buf(s.bitmap);
-    free_buf(s.tfp); free_buf(s.pm); free_buf(s.wm); free_buf(s.gb);
+    free_buf(s.tfp); free_buf(s.gb);
     for (auto& e : s.bm_free) free_ev(e);
     for (auto& l : s.lists) {
       free_buf(l.done); free_buf(l.status); free_buf(l.mb); free_buf(l.coff); free_buf(l.mtfp);
@@ -788,8 +788,6 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   RO_TRY(ensure(c, S.phase, N * sizeof(uint32_t), "phase words"));
   RO_TRY(ensure(c, S.rec, N * sizeof(Rec), "result records"));
   RO_TRY(ensure(c, S.bitmap, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), "completion bitmaps"));
-  RO_TRY(ensure(c, S.pm, P * sizeof(uint32_t), "parent member counts"));
-  RO_TRY(ensure(c, S.wm, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), "word member counts"));
   RO_TRY(ensure(c, S.gb, P * sizeof(unsigned long long), "GroupFailure barriers"));
   for (auto& l : S.lists) {
     RO_TRY(ensure(c, l.done, P * sizeof(uint32_t), "completed parents"));
@@ -810,7 +808,6 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
     RO_TRY(ensure(c, p.hdr, sizeof(PlanHdr), "assembly plan"));
   }
   cudaMemsetAsync(S.bitmap.p, 0, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), c->stream);
-  cudaMemsetAsync(S.wm.p, 0, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), c->stream);
   cudaMemsetAsync(S.gb.p, 0, P * sizeof(unsigned long long), c->stream);   // no barrier (commit 0)
   ExpandFillArgs fa{};
   fa.offsets = (const uint64_t*)S.offsets.p;
@@ -1075,8 +1072,6 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   const int bs = (int)(x->commits % BM_SLOTS);   // bitmap slot of this commit
   const uint64_t n_words = ceil_div(x->P, 32);
   ca.bitmap = (uint32_t*)S.bitmap.p + bs * n_words;
-  ca.pm = (uint32_t*)S.pm.p;
-  ca.wm = (uint32_t*)S.wm.p + bs * n_words;
   ca.gb = (unsigned long long*)S.gb.p;
   if (++c->commit_seq == 0) {   // wrapped: old tags could look current again
     for (auto& sl : c->slots)

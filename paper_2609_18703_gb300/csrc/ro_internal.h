@@ -235,9 +235,7 @@ struct CommitArgs {
   uint32_t* phase;
   Rec* rec;
   unsigned long long* pw;
-  uint32_t* bitmap;
-  uint32_t* pm;               // per parent: members to gather once complete (0: Suppressed)
-  uint32_t* wm;               // per bitmap word: sum of pm of the parents completed in this call
+  uint32_t* bitmap;           // parents this call completed
   unsigned long long* gb;     // per parent: (seq << 32) | ~r for the lowest accepted
                               // GroupFailure report r of commit seq; older seq: none
   uint32_t seq;               // this commit's sequence number in the context (from 1)
