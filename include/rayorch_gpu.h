@@ -28,7 +28,8 @@
  *   completion lists and admissions: ro_assemble plans on the context's plan
  *   stream and copies on its copy stream, with separate streams set
  *   (ro_ctx_set_streams) ro_gather_commit builds its completed-parent list
- *   on a stream the context owns, and with Call streams set
+ *   and that list's copy plan on one of two streams the context owns
+ *   (commits alternate between them), and with Call streams set
  *   (ro_ctx_set_call_streams) ro_batch_ready runs on its Call's stream.
  *   Each assembly is ordered after all work the caller issued on the
  *   context before it; the caller's ro_assemble
@@ -136,11 +137,12 @@ ro_status ro_ctx_sync(ro_ctx* ctx);
  * and commits; up to three commits and assemblies per expansion may be in
  * flight at once (the context keeps three list and plan slots per expansion
  * and orders their reuse with events).  With a plan stream other than the
- * context's stream, the context also creates a stream of its own for the
- * commits' completion scans (destroyed with the context), so one commit's
- * completed-parent list is built while the next commit's reports are
- * applied (four completion bitmaps per expansion, taken in turn).  The
- * context's stream first waits for the old streams.  The caller keeps the streams alive until ro_ctx_destroy
+ * context's stream, the context also creates two streams of its own
+ * (destroyed with the context) for the commits' completed-parent lists and
+ * their copy plans, which consecutive commits take in turn: one commit's
+ * list is built while the next commits' reports are applied and the next
+ * commit's list is built (four completion bitmaps per expansion, taken in
+ * turn).  The context's stream first waits for the old streams.  The caller keeps the streams alive until ro_ctx_destroy
  * or the next ro_ctx_set_streams. */
 ro_status ro_ctx_set_streams(ro_ctx* ctx, void* plan_stream, void* copy_stream);
 /* Streams for the Calls' admissions (Section 4.3: each Call has its own
@@ -162,8 +164,8 @@ ro_status ro_ctx_set_streams(ro_ctx* ctx, void* plan_stream, void* copy_stream);
  * with n > 0. */
 ro_status ro_ctx_set_call_streams(ro_ctx* ctx, void* const* streams, uint32_t n);
 /* Make the context's stream wait (on the GPU) for all work issued so far on
- * the plan and copy streams, the completion-scan stream and the Calls'
- * streams.  Call it before reading assembly outputs in
+ * the plan and copy streams, the context's two completion streams and the
+ * Calls' streams.  Call it before reading assembly outputs in
  * stream order, before starting a capture of the context's stream, and
  * before ending one (a captured assembly forks onto the other streams, and a
  * capture must join them back).  Nothing waits on the host. */
@@ -332,8 +334,10 @@ ro_status ro_retry(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t* d_ch
  *               call, ascending.  done_cap must be >= min(n, parents of xid).
  *   d_n_done (device) / h_n_done (host, synchronises) out or NULL.
  *   With separate streams set, d_done_parents and d_n_done are written on
- *   the context's completion-scan stream (see the conventions above);
- *   ro_assemble orders itself after them.
+ *   one of the context's completion streams (see the conventions above);
+ *   ro_assemble orders itself after them.  The same pass plans the copy of
+ *   the completed parents, so ro_assemble of this list (d_parents NULL,
+ *   without list structure) runs only the copy.
  * Capture: a captured commit keeps the context's commit number it was
  * captured with; replay a captured sequence of commits on a fresh expansion
  * (ro_expand clears the GroupFailure barrier table), as a new microbatch.
@@ -381,9 +385,12 @@ ro_status ro_gather_commit(ro_ctx* ctx, int32_t xid, uint64_t n, const uint64_t*
  * as the results of the level above (nested expansions).
  * Errors: RO_E_CAPACITY when base + bytes > out_cap or the list is longer
  * than n_parents (nothing is copied).
- * Streams: planning runs on the plan stream and the copy on the copy stream
- * (see ro_ctx_set_streams); the outputs (d_status, d_out_off, d_out_len,
- * d_out, the cursor, d_out_bytes) are written there.  Read them after
+ * Streams: the latest commit's list (d_parents NULL) was planned by the
+ * commit, so only the copy runs, on the copy stream; an explicit list is
+ * planned on the plan stream first (see ro_ctx_set_streams).  The outputs
+ * (d_status, d_out_off, d_out_len, d_out, the cursor, d_out_bytes) are
+ * written by the copy.  A d_arena smaller than the accepted reports'
+ * ranges is refused on the GPU (RO_E_INVAL, nothing copied).  Read them after
  * ro_ctx_join in stream order, or after any synchronising call.
  * Consecutive calls may pass the same output arrays: their writes land in
  * call order (a call whose planning writes caller memory that an earlier

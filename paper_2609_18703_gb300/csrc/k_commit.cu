@@ -7,10 +7,13 @@
 //                 counts the member down at its parent with one 64-bit atomic
 //                 add on (remaining | bad << 32).  Lanes of a warp that hit
 //                 the same parent are merged first (__match_any_sync), so a
-//                 hot parent sees one atomic per warp.  The add that takes
-//                 `remaining` to zero completes the parent and sets its bit in
-//                 a completion bitmap (the counter's high half then tells
-//                 whether a member Failed or was Suppressed).
+//                 hot parent sees one atomic per warp.  Members of heavy
+//                 parents (>= HEAVY_CHILDREN children, whose reports seldom
+//                 share a warp) are first summed per CTA in a shared-memory
+//                 table and added to the parent once per CTA.  The add that
+//                 takes `remaining` to zero completes the parent and sets its
+//                 bit in a completion bitmap (the counter's high half then
+//                 tells whether a member Failed or was Suppressed).
 // commit_fix      after the scatter, on the same stream: when the call
 //                 carried two reports for one Grain or a GroupFailure (rare)
 //                 it orders the repeats and applies the barriers, so the
@@ -82,10 +85,53 @@ __device__ __forceinline__ void prefetch_reports(const CommitArgs& a) {
   }
 }
 
+// Per-CTA table of heavy parents' member counts (open addressing on the
+// parent id): value = bad members << 32 | members, added to the parent's
+// counter (as bad << 32 - members) when the CTA is done.
+constexpr int HT_SIZE = 2048;
+constexpr int HT_PROBES = 32;
+constexpr uint32_t HT_EMPTY = 0xFFFFFFFFu;   // no parent has this id (P < 2^32)
+struct HeavyTable {
+  uint32_t key[HT_SIZE];
+  unsigned long long val[HT_SIZE];
+};
+size_t commit_scatter_smem(int heavy) { return heavy ? sizeof(HeavyTable) : 0; }
+
+// Count n_tot members (n_bad of them Failed or Suppressed) down at parent p;
+// the add that takes `remaining` to zero completes the parent.
+__device__ __forceinline__ void count_down(const CommitArgs& a, uint32_t p, uint32_t n_tot, uint32_t n_bad) {
+  const unsigned long long delta = ((unsigned long long)n_bad << 32) - (unsigned long long)n_tot;
+  const unsigned long long old = atomicAdd(a.pw + p, delta);
+  if ((uint32_t)old == n_tot)   // the last members: the parent is complete
+    atomicOr(a.bitmap + (p >> 5), 1u << (p & 31));
+}
+
+// Add to heavy parent p's entry of the CTA's table; false when no entry was
+// found within HT_PROBES slots (the caller counts down directly).
+__device__ __forceinline__ bool table_add(HeavyTable* t, uint32_t p, unsigned long long v) {
+  uint32_t h = (p * 2654435761u) >> (32 - 11);   // HT_SIZE = 2^11
+  for (int i = 0; i < HT_PROBES; ++i) {
+    const uint32_t k = atomicCAS(&t->key[h], HT_EMPTY, p);
+    if (k == HT_EMPTY || k == p) {
+      atomicAdd(&t->val[h], v);
+      return true;
+    }
+    h = (h + 1) & (HT_SIZE - 1);
+  }
+  return false;
+}
+
 __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a) {
   prefetch_reports(a);
   wait_predecessor();
   allow_successor();
+  extern __shared__ __align__(16) unsigned char cm_smem[];
+  HeavyTable* ht = reinterpret_cast<HeavyTable*>(cm_smem);
+  if (a.heavy)
+    for (int i = threadIdx.x; i < HT_SIZE; i += blockDim.x) {
+      ht->key[i] = HT_EMPTY;
+      ht->val[i] = 0ull;
+    }
   // verdict counts: accept, invalid, not in flight, stale, -, barrier,
   // duplicate candidates, accepted GroupFailures
   __shared__ unsigned long long s_cnt[8];
@@ -107,7 +153,7 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
     const uint64_t r = base + lane;
     uint8_t v = 255;   // inactive lane
     uint32_t p = 0;
-    bool bad = false;
+    bool bad = false, heavy = false;
     if (r < n) {
       const uint64_t c = a.child[r];
       const uint8_t s = a.state[r];
@@ -119,7 +165,15 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
       if (c >= a.N || !valid_state || !in_bounds) {
         v = V_INVALID;
       } else {
-        const uint32_t par = a.rec[c].parent;   // immutable: read alongside the fence
+        // parent and heavy flag, immutable: read alongside the fence
+        uint32_t par;
+        if (a.heavy) {
+          const ulonglong2 rv = *reinterpret_cast<const ulonglong2*>(a.rec + c);
+          par = (uint32_t)rv.x;
+          heavy = (rv.y & W_HEAVY_BIT) != 0ull;
+        } else {
+          par = a.rec[c].parent;
+        }
         // Eq. (3): accept iff IN-FLIGHT at the report's generation
         const uint32_t want = ph_make(PH_INFLIGHT, g);
         uint32_t cur;
@@ -165,11 +219,8 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
       const unsigned grp = __match_any_sync(acc, p);
       if (lane == __ffs(grp) - 1) {
         const unsigned n_tot = __popc(grp), n_bad = __popc(grp & badm);
-        const unsigned long long delta =
-            ((unsigned long long)n_bad << 32) - (unsigned long long)n_tot;
-        const unsigned long long old = atomicAdd(a.pw + p, delta);
-        if ((uint32_t)old == n_tot)   // the last members: the parent is complete
-          atomicOr(a.bitmap + (p >> 5), 1u << (p & 31));
+        if (!(heavy && table_add(ht, p, ((unsigned long long)n_bad << 32) | n_tot)))
+          count_down(a, p, n_tot, n_bad);
       }
     }
     if (v <= V_DUP_CANDIDATE) cnt[v] += 1;
@@ -185,6 +236,13 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
     if (lane == 0 && x) atomicAdd(&s_cnt[k], (unsigned long long)x);
   }
   __syncthreads();
+  if (a.heavy)   // the CTA's heavy-parent counts, one add per parent
+    for (int i = threadIdx.x; i < HT_SIZE; i += blockDim.x) {
+      const uint32_t p = ht->key[i];
+      if (p == HT_EMPTY) continue;
+      const unsigned long long v = ht->val[i];
+      count_down(a, p, (uint32_t)v, (uint32_t)(v >> 32));
+    }
   if (threadIdx.x == 0) {
     for (int k = 0; k < 4; ++k)
       if (s_cnt[k]) atomicAdd(&ds->stats[k], s_cnt[k]);
@@ -635,7 +693,7 @@ void launch_commit_scatter(const LaunchCfg& L, const CommitArgs& a) {
   const int grid =
       (int)std::max<uint64_t>(1, std::min<uint64_t>(ceil_div(warps, CM_THREADS / 32),
                                                     (uint64_t)L.grid_commit));
-  launch_k(L, K_COMMIT, commit_scatter_kernel, grid, CM_THREADS, 0, a);
+  launch_k(L, K_COMMIT, commit_scatter_kernel, grid, CM_THREADS, commit_scatter_smem(a.heavy), a);
   // the fix returns at once unless the scatter flagged the call; a grid for
   // the barriers of calls without repeated reports
   const int grid_fix = (int)std::max<uint64_t>(

@@ -55,6 +55,11 @@ __global__ void __launch_bounds__(EXP_THREADS) expand_scan_kernel(ExpandScanArgs
       mine.a += cnt[k];
       mine.b += (p < a.P && cnt[k] == 0u) ? 1ull : 0ull;
     }
+    uint32_t heavy = 0;
+#pragma unroll
+    for (int k = 0; k < EXP_ITEMS; ++k) heavy += cnt[k] >= HEAVY_CHILDREN ? 1u : 0u;
+    heavy = __reduce_add_sync(0xffffffffu, heavy);
+    if ((threadIdx.x & 31) == 0 && heavy) atomicAdd(&ds->n_heavy, (unsigned long long)heavy);
     Pair64 total;
     Pair64 excl = block_excl_scan_pair(mine, s_scan, &total);
     if (threadIdx.x < 32) {  // one warp looks back
@@ -119,11 +124,12 @@ __global__ void __launch_bounds__(FILL_THREADS) expand_fill_kernel(ExpandFillArg
     }
     __syncthreads();
     for (uint64_t c = c0 + threadIdx.x; c < c1; c += blockDim.x) {
-      uint64_t p, base;
+      uint64_t p, base, end;
       if (staged) {
         const uint32_t k = last_le(s_off, 0u, (uint32_t)R - 1u, c);
         p = p_lo + k;
         base = s_off[k];
+        end = s_off[k + 1];
       } else {
         // many empty parents inside one tile: search the global offsets
         uint64_t lo = p_lo, hi = p_hi + 1;
@@ -136,6 +142,7 @@ __global__ void __launch_bounds__(FILL_THREADS) expand_fill_kernel(ExpandFillArg
         }
         p = lo;
         base = a.offsets[lo];
+        end = a.offsets[lo + 1];
       }
       const uint32_t call = a.parent_call ? (uint32_t)a.parent_call[p] : 0u;
       a.child_parent[c] = (uint32_t)p;
@@ -144,7 +151,7 @@ __global__ void __launch_bounds__(FILL_THREADS) expand_fill_kernel(ExpandFillArg
       Rec r;
       r.parent = (uint32_t)p;
       r.len = 0u;
-      r.w = (uint64_t)call << W_CALL_SHIFT;
+      r.w = ((uint64_t)call << W_CALL_SHIFT) | (end - base >= HEAVY_CHILDREN ? W_HEAVY_BIT : 0ull);
       a.rec[c] = r;
     }
     __syncthreads();

@@ -87,6 +87,7 @@ struct Expansion {
   uint64_t P = 0, N = 0;
   uint64_t commits = 0, assembles = 0;
   int last_list = -1;   // list slot written by the latest commit
+  bool heavy = false;   // some parent has at least HEAVY_CHILDREN children
 };
 
 struct TsBuf {
@@ -771,6 +772,7 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   sa.tfp_cap = tfp_entries;
   sa.ds = c->ds;
   RO_TRY(tile_status(c, TS_EXPAND, ceil_div(P, (uint64_t)EXP_THREADS * EXP_ITEMS), &sa.ts));
+  cudaMemsetAsync(&c->ds->n_heavy, 0, sizeof(unsigned long long), c->stream);
   launch_expand_scan(c->L, sa);
   RO_TRY(check_launch(c, "expand_scan"));
   RO_TRY(sync_and_check(c));
@@ -828,6 +830,7 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   x.parent_xid = parent_xid;
   x.P = P;
   x.N = N;
+  x.heavy = c->hs->n_heavy != 0;
   c->exps.push_back(x);
   *xid = (int32_t)slot;
   return RO_OK;
@@ -1072,6 +1075,7 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   const int bs = (int)(x->commits % BM_SLOTS);   // bitmap slot of this commit
   const uint64_t n_words = ceil_div(x->P, 32);
   ca.bitmap = (uint32_t*)S.bitmap.p + bs * n_words;
+  ca.heavy = x->heavy ? 1 : 0;
   ca.gb = (unsigned long long*)S.gb.p;
   if (++c->commit_seq == 0) {   // wrapped: old tags could look current again
     for (auto& sl : c->slots)

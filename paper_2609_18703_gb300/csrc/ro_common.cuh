@@ -7,7 +7,8 @@
 //             attempt generation (Eq. 3).
 //   rec[c]    16-byte record: immediate parent, payload length and one word
 //             packing the arena offset (48 bits), the published outcome
-//             (3 bits), two commit bookkeeping flags and the Call (8 bits).
+//             (3 bits), whether the parent is heavy (at least HEAVY_CHILDREN
+//             children), commit bookkeeping flags and the Call (8 bits).
 // Per-parent state: pw[p] = remaining unsealed members (low 32 bits) plus the
 // number of Failed/Suppressed members (high 32 bits), so one 64-bit atomic add
 // both counts a member down and records its outcome class.
@@ -43,16 +44,22 @@ constexpr uint8_t V_DUP_CANDIDATE = 6;
 struct __align__(16) Rec {
   uint32_t parent;
   uint32_t len;
-  uint64_t w;   // off (0-47) | state (48-50) | barrier (53) | sealer-seen (54) | conflict (55) | call (56-63)
+  uint64_t w;   // off (0-47) | state (48-50) | heavy parent (52) | barrier (53) | sealer-seen (54) |
+                // conflict (55) | call (56-63)
 };
 constexpr uint64_t W_OFF_MASK = (1ull << 48) - 1;
 constexpr int W_STATE_SHIFT = 48;
 constexpr uint64_t W_STATE_MASK = 7ull << W_STATE_SHIFT;
+constexpr uint64_t W_HEAVY_BIT = 1ull << 52;     // the parent has >= HEAVY_CHILDREN children (set at expand)
 constexpr uint64_t W_BARRIER_BIT = 1ull << 53;   // sealed by a sibling's GroupFailure
 constexpr uint64_t W_SEALER_BIT = 1ull << 54;
 constexpr uint64_t W_CONFLICT_BIT = 1ull << 55;
 constexpr int W_CALL_SHIFT = 56;
 constexpr uint64_t MAX_ARENA = 1ull << 48;
+// A parent with at least this many children is heavy: a commit counts its
+// members down in shared memory per CTA and adds them to the parent's
+// counter once per CTA (its reports seldom share a warp).
+constexpr uint32_t HEAVY_CHILDREN = 4096;
 
 __device__ __forceinline__ uint8_t w_state(uint64_t w) {
   return (uint8_t)((w >> W_STATE_SHIFT) & 7u);
@@ -104,7 +111,7 @@ struct DevScalars {
   uint32_t pad0;
   unsigned long long stats[13];  // same order as ro_stats
   // ro_expand
-  unsigned long long n_children, n_empty, last_nonempty_parent;
+  unsigned long long n_children, n_empty, last_nonempty_parent, n_heavy;
   // ro_gather_commit
   unsigned long long cm_n, cm_n_done[2];   // completed parents, per plan slot
   // per commit, in two slots (commit sequence & 1): duplicate candidates and

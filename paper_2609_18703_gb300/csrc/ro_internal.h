@@ -236,6 +236,7 @@ struct CommitArgs {
   Rec* rec;
   unsigned long long* pw;
   uint32_t* bitmap;           // parents this call completed
+  int heavy;                  // the expansion has heavy parents: count them per CTA first
   unsigned long long* gb;     // per parent: (seq << 32) | ~r for the lowest accepted
                               // GroupFailure report r of commit seq; older seq: none
   uint32_t seq;               // this commit's sequence number in the context (from 1)

@@ -29,7 +29,7 @@ def _built():
 
 from tests.lockstep import Lockstep, dev  # noqa: E402
 from tests.pipeline import host_arena  # noqa: E402
-from workload import FAILED, PRESENT, docpage, streaming  # noqa: E402
+from workload import DROPPED, FAILED, PRESENT, SUPPRESSED, docpage, streaming  # noqa: E402
 
 GF = 5   # report kind GroupFailure
 
@@ -204,4 +204,35 @@ def test_barrier_on_a_100k_child_parent():
         ls.commit(x, *_rep([3, 4, 0, 5], [PRESENT, PRESENT, PRESENT, GF]), arena_bytes=arena.size)
         ls.assemble(x, arena, ad, parents=None, n_parents=3)
         ls.batch_ready(x, 0, None, 1000, flush=True)
+        ls.check_stats()
+
+
+@pytest.mark.parametrize("seed", range(2))
+def test_heavy_parents_with_repeats_failures_and_barriers(seed):
+    """Parents of 4,096 children or more (their members are counted down per
+    CTA in shared memory, then once per parent) mixed with light ones, over
+    several commits carrying repeated reports, failures, Dropped results and
+    GroupFailures: every verdict, completion and assembled byte equals the
+    oracle's (a report's order inside a call still decides)."""
+    rng = np.random.default_rng(7100 + seed)
+    counts = rng.integers(0, 6, 4000).astype(np.uint32)
+    heavy = rng.choice(counts.size, 6, replace=False)
+    counts[heavy] = [4096, 5000, 9000, 4095, 12000, 20000]   # one just below the threshold
+    N = int(counts.sum())
+    arena = rng.integers(0, 256, N * 8 + 64).astype(np.uint8)
+    with Lockstep() as ls:
+        x = ls.expand(counts)["xid"]
+        ad = _arena_dev(arena)
+        ls.batch_ready(x, 0, None, 256, flush=True)
+        perm = rng.permutation(N).astype(np.uint32)
+        for w, chunk in enumerate(np.array_split(perm, 5)):
+            rep = rng.choice(chunk, size=chunk.size // 8)
+            ch = np.concatenate([chunk, rep])
+            ch = ch[rng.permutation(ch.size)].astype(np.uint32)
+            st = rng.choice([PRESENT] * 40 + [DROPPED, FAILED, SUPPRESSED] + ([GF] if w >= 2 else []),
+                            ch.size).astype(np.uint8)
+            ln = rng.integers(0, 9, ch.size).astype(np.uint32)
+            of = ch.astype(np.uint64) * 8
+            cm = ls.commit(x, ch, st, ln, of, arena_bytes=arena.size)
+            ls.assemble(x, arena, ad, parents=None, n_parents=max(cm["n_done"], 1))
         ls.check_stats()
