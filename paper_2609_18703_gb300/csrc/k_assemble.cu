@@ -908,6 +908,35 @@ __device__ void emit_direct(const CopyCtx& c, const CopyStage* st, uint32_t cw, 
   }
 }
 
+// A copy of at most AC_SMALL_CHUNKS chunks is latency-bound: every warp of
+// the participating CTAs takes 2 KB slices of the output in turn and copies
+// the member pieces inside each straight from the arena (no claims, staging
+// or barriers), the slice's first member found from the chunk table and one
+// warp-wide probe of the next 32 members.
+constexpr uint64_t AC_SLICE = 2048;
+__device__ void copy_small(const CopyCtx& c, uint64_t gw, uint64_t n_w, int lane) {
+  const uint64_t n_sl = ceil_div(c.S, AC_SLICE);
+  for (uint64_t sl = gw; sl < n_sl; sl += n_w) {
+    uint64_t ra = sl * AC_SLICE;
+    const uint64_t rb = (ra + AC_SLICE < c.S) ? ra + AC_SLICE : c.S;
+    uint64_t k;
+    if (c.ctfp) {   // the member holding the chunk's first byte holds or precedes ra
+      const uint64_t k0 = c.ctfp[ra / AC_CHUNK], probe = k0 + (uint64_t)lane;
+      const unsigned m = __ballot_sync(0xffffffffu, probe < c.Mnz && c.cpos[probe] <= ra);
+      k = (m == 0xffffffffu) ? warp_search(c.cpos, c.Mnz, ra, lane) : k0 + (uint64_t)(__popc(m) - 1);
+    } else {
+      k = warp_search(c.cpos, c.Mnz, ra, lane);
+    }
+    for (; ra < rb; ++k) {
+      const uint64_t pk = c.cpos[k], pn = cpos_at(c, k + 1);
+      const uint64_t e = pn < rb ? pn : rb;
+      warp_copy(c.a->out + (c.out_base - (uint64_t)(uintptr_t)c.a->out) + ra,
+                c.a->arena + c.csrc[k] + (ra - pk), e - ra, lane);
+      ra = e;
+    }
+  }
+}
+
 // The copy: per-parent outputs, then the chunks of the call's output, each
 // CTA taking every n_part-th chunk.  Warps 0..AC_PRODUCERS-1 stage chunks
 // into a ring of AC_STAGES stages (producer p takes the CTA's chunks i with
@@ -979,6 +1008,10 @@ __global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
         }
       }
     }
+    if (n_chunks <= a.small_chunks) {
+      copy_small(c, (uint64_t)blockIdx.x * (AC_THREADS / 32) + warp, (uint64_t)n_part * (AC_THREADS / 32),
+                 lane);
+    } else {
     if (threadIdx.x == 0) {
       for (int s = 0; s < AC_STAGES; ++s) {
         mbar_init(&full_bar[s], 1);
@@ -1108,7 +1141,11 @@ __global__ void __maxnreg__(80) asm_copy_kernel(AssembleArgs a) {
         if (!landed) atomicOr(&ds->err, ERR_DRAIN);
       }
     }
+    }
   }
+  // this CTA's bytes are done: the next copy on the stream may be scheduled
+  // into the space it leaves (it waits for this grid before it reads anything)
+  allow_successor();
   if (threadIdx.x == 0) {
     if (ticket(&ds->exit_ctr[TS_ASM_COPY]) == n_part - 1) {
       if (!failed && a.cursor) *a.cursor = base + S;

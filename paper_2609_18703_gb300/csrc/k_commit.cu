@@ -26,6 +26,10 @@
 
 #include "ro_internal.h"
 
+#ifndef RO_FIX_EARLY
+#define RO_FIX_EARLY 0
+#endif
+
 namespace ro {
 
 constexpr uint8_t V_WIN_SEALER = 7, V_WIN_CAND = 8, V_LOSE_SEALER = 9, V_LOSE_CAND = 10;
@@ -336,8 +340,15 @@ __device__ void apply_barriers_grid(const CommitArgs& a, uint64_t n) {
 // final outcomes.  Returns at once when the scatter saw neither.  Kept out
 // of the scatter so that the scatter's registers and shared memory stay small.
 __global__ void __launch_bounds__(CM_THREADS) commit_fix_kernel(CommitArgs a) {
+#if RO_FIX_EARLY
+  // the next commit's scatter launches now (it waits for this grid before it
+  // touches lineage state, and warms L2 with its reports meanwhile)
+  allow_successor();
   wait_predecessor();
-  allow_successor();   // the next commit's scatter launches now and waits for this grid
+#else
+  wait_predecessor();
+  allow_successor();
+#endif
   DevScalars* ds = a.ds;
   const unsigned long long dups = ds->cm_conflicts[fix_slot(a)], gfs = ds->cm_gf[fix_slot(a)];
   if (dups == 0ull && gfs == 0ull) return;

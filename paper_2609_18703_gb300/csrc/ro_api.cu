@@ -12,6 +12,7 @@
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -38,7 +39,16 @@ namespace {
 constexpr int MAX_EXPANSIONS = 64;
 constexpr int N_TS = 8;    // tile-status slots (TS_* in ro_common.cuh)
 constexpr int RING = 3;    // list / plan slots per expansion
-constexpr int BM_SLOTS = 4;   // completion bitmaps per expansion (commits take them in turn)
+// Completion bitmaps per expansion, taken in turn by its commits.  A commit
+// may reuse a slot once the plan that read it (BM_SLOTS commits earlier) is
+// done; the context's stream waits for that only every BM_WAIT commits (for
+// all plans at least BM_WAIT + 1 commits old), so a scatter seldom depends
+// on anything but the previous kernel on its stream and launches early.
+#ifndef RO_BM_SLOTS
+#define RO_BM_SLOTS 32
+#endif
+constexpr int BM_SLOTS = RO_BM_SLOTS;
+constexpr int BM_WAIT = BM_SLOTS / 2;
 
 struct DevBuf {
   void* p = nullptr;
@@ -76,7 +86,8 @@ struct PlanSlot {
 // Device buffers of one expansion slot, kept across ro_ctx_reset and reused.
 struct ExpSlot {
   DevBuf offsets, pw, phase, rec, bitmap, tfp, gb;   // bitmap: BM_SLOTS slots
-  Ev bm_free[BM_SLOTS];   // the completion scan that read a bitmap slot is done
+  Ev bm_free[BM_SLOTS];   // the plan that read a bitmap slot is done
+  int bm_stream[BM_SLOTS] = {};   // the completion stream that plan ran on
   ListSlot lists[RING];
   PlanSlot plans[RING];
   std::vector<QueueBufs> queues;
@@ -151,6 +162,7 @@ struct ro_ctx {
   int last_fin = 0;                     // the stream of the latest commit's plan
   uint32_t n_calls = 1;
   uint32_t commit_seq = 0;              // commits issued on this context
+  uint64_t copy_small_chunks = AC_SMALL_CHUNKS;   // copies this small go direct
   int num_sms = 0;
   LaunchCfg L{}, Lp{}, Lc{}, Lf[2]{};
   DevScalars* ds = nullptr;
@@ -519,6 +531,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->copy_stream = c->stream;
   c->fin_stream[0] = c->fin_stream[1] = c->stream;
   c->n_calls = n_calls;
+  if (const char* e = std::getenv("RO_COPY_SMALL_CHUNKS")) c->copy_small_chunks = std::strtoull(e, nullptr, 10);
   cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
   if (cudaMalloc(&c->ds, sizeof(DevScalars)) != cudaSuccess ||
       cudaMallocHost(&c->hs, sizeof(DevScalars)) != cudaSuccess ||
@@ -1108,8 +1121,23 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.pslot = pf;
   RO_TRY(tile_status(c, pf ? TS_COMMIT_ODD : TS_COMMIT, ceil_div(ceil_div(x->P, 32), (uint64_t)CP_WORDS),
                      &ca.tsq));
-  // the bitmap slot is free once the completion scan BM_SLOTS commits ago is done
-  RO_TRY(ev_wait(c, S.bm_free[bs], c->stream));
+  // The bitmap slots of this commit and the next BM_WAIT - 1 are free once
+  // every plan up to commit w - BM_WAIT - 1 is done: wait for the latest such
+  // plan of each completion stream (a stream runs its plans in order).
+  if (x->commits % BM_WAIT == 0 && x->commits > (uint64_t)BM_WAIT) {
+    const uint64_t w = x->commits;
+    bool seen[2] = {false, false};
+    // (commits w - BM_SLOTS .. w - BM_WAIT - 1: the slot of commit w - BM_SLOTS
+    // is this commit's, and its event is not overwritten yet)
+    for (uint64_t j = w - BM_WAIT - 1; j + BM_SLOTS >= w && !(seen[0] && seen[1]); --j) {
+      const int k = S.bm_stream[j % BM_SLOTS];
+      if (!seen[k]) {
+        RO_TRY(ev_wait(c, S.bm_free[j % BM_SLOTS], c->stream));
+        seen[k] = true;
+      }
+      if (j == 0) break;
+    }
+  }
   launch_commit_scatter(c->L, ca);
   // the completed list and its plan follow the scatter (on their own stream
   // when the context has one); the list slot is free once the assembly that
@@ -1121,6 +1149,7 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   launch_commit_plan(c->Lf[pf], ca);
   if (fs != c->stream) {
     RO_TRY(ev_record(c, S.bm_free[bs], fs));
+    S.bm_stream[bs] = pf;
     RO_TRY(ev_record(c, LS.planned, fs));
   }
   c->last_fin = pf;
@@ -1248,6 +1277,7 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   aa.arena = d_arena;
   aa.arena_bytes = arena_bytes;
   aa.arena_host = arena_host;
+  aa.small_chunks = c->copy_small_chunks;
   aa.status = d_status;
   aa.out_off = d_out_off;
   aa.out_len = d_out_len;

@@ -48,6 +48,9 @@ constexpr uint64_t AC_CHUNK = 16384;                          // output bytes pe
 constexpr uint32_t AC_PIECES = 1024;
 constexpr uint32_t AC_BUF = 24576;
 constexpr uint32_t AC_SMALL = 64;   // pieces of at most this many staged bytes: cp.async, not a bulk copy
+// copies of at most this many chunks take the direct path (RO_COPY_SMALL_CHUNKS
+// in the environment at context creation overrides it; 0 stages every copy)
+constexpr uint64_t AC_SMALL_CHUNKS = 256;
 
 // kernel entry points for occupancy queries and per-kernel timing
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CPLAN, K_APARENTS,
@@ -269,6 +272,7 @@ struct AssembleArgs {
   const uint8_t* arena;
   uint64_t arena_bytes;
   int arena_host;             // the arena is pinned host memory: no bulk (TMA) copies from it
+  uint64_t small_chunks;      // copies of at most this many chunks go direct (no staging)
   uint8_t* status;
   uint64_t* out_off;
   uint32_t* out_len;          // optional
