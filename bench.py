@@ -638,6 +638,7 @@ def kernel_alg_bytes(info: dict) -> dict:
         "expand_scan": 4 * P + 8 * (P + info["levels"]),     # counts in, offsets out
         "expand_fill": 8 * N,                                  # parent and ordinal per child
         "ready_scatter": 4 * N,                                # the batch list
+        "ready_fused": 4 * N,                                  # the same, one-pass admission
         "commit_scatter": 21 * R,                              # report (17) + lineage (4)
         "commit_plan": 13 * P + 16 * M + 16 * Z,               # list + records in + plan out
         "asm_members": 16 * M + 16 * Z,                        # records in, plan out (lists)
@@ -650,7 +651,7 @@ def kernel_alg_bytes(info: dict) -> dict:
 # sha256 (first 16 hex digits) of the kernel's source file at capture time;
 # a source that has changed since makes the bench report traffic as null.
 KERNEL_SOURCE = {"expand_scan": "k_expand.cu", "expand_fill": "k_expand.cu",
-                 "ready_count": "k_ready.cu", "ready_scatter": "k_ready.cu",
+                 "ready_count": "k_ready.cu", "ready_scatter": "k_ready.cu", "ready_fused": "k_ready.cu",
                  "commit_scatter": "k_commit.cu", "commit_fix": "k_commit.cu",
                  "commit_plan": "k_complete.cu", "asm_members": "k_assemble.cu",
                  "asm_copy": "k_assemble.cu"}
@@ -1317,7 +1318,8 @@ def run_streaming(args, rank, world, local_rank):
     ro.ro_ctx_profile(ctx, 0)
     tot = level_totals([lv])
     alg = kernel_alg_bytes({"P": P, "N": N, "R": N, "S": S, "levels": 1, **tot})
-    alg["ready_scatter"] += 4 * N * lv.n_calls   # every Call reads every candidate list
+    for k in ("ready_scatter", "ready_fused"):   # every Call reads every candidate list
+        alg[k] += 4 * N * lv.n_calls
     kernel_ms = {k: round(v[2], 4) for k, v in prof.items() if v[1]}
     dom = max((k for k in alg if k in kernel_ms), key=lambda k: alg[k])
     n_launch = prof[dom][0]

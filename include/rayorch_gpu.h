@@ -121,6 +121,11 @@ typedef struct {
  * ordered gathering are scoped to one input microbatch).  `stream` is a
  * cudaStream_t (NULL = legacy default stream) on device `device`; n_calls in
  * [1, 256] is the number of Calls whose Ready Queues the context keeps.
+ * Two environment variables, read here, tune the context: RO_COPY_SMALL_CHUNKS
+ * (copies of at most this many 16 KB chunks take the direct path; default
+ * 256, 0 stages every copy) and RO_ADMIT_TWO_PASS (non-zero: every
+ * admission takes the two-pass path instead of the one-pass cooperative
+ * kernel that lists of up to a few thousand tiles of 2,048 candidates use).
  */
 ro_status ro_ctx_create(ro_ctx** ctx, int32_t device, void* stream, uint32_t n_calls);
 ro_status ro_ctx_destroy(ro_ctx* ctx);
@@ -178,11 +183,11 @@ const char* ro_last_error(const ro_ctx* ctx);
 /* Kernel ids for the profiling calls below, in launch order of the path. */
 enum {
   RO_K_EXPAND_SCAN = 0, RO_K_EXPAND_FILL = 1, RO_K_READY_COUNT = 2, RO_K_READY_SCATTER = 3,
-  RO_K_COMMIT_SCATTER = 4, RO_K_COMMIT_FINISH = 5, RO_K_ASM_PARENTS = 6, RO_K_ASM_MEMBERS = 7,
+  RO_K_COMMIT_SCATTER = 4, RO_K_COMMIT_PLAN = 5, RO_K_ASM_PARENTS = 6, RO_K_ASM_MEMBERS = 7,
   RO_K_ASM_COPY = 8, RO_K_RETRY_CLAIM = 9, RO_K_RETRY_SCATTER = 10, RO_K_PB_KEYS = 11,
   RO_K_PB_HIST = 12, RO_K_PB_ROWSCAN = 13, RO_K_PB_SORT = 14, RO_K_PB_BOUNDS = 15,
   RO_K_PB_HEADS = 16, RO_K_PB_MARK = 17, RO_K_PB_SCAN = 18, RO_K_PB_EMIT = 19,
-  RO_K_COMMIT_FIX = 20, RO_K_COUNT = 21
+  RO_K_COMMIT_FIX = 20, RO_K_READY_FUSED = 21, RO_K_COUNT = 22
 };
 /* Tracing (no counterpart in the paper; it instruments the path).  Every
  * kernel launch is counted; kernels whose bit (1 << RO_K_*) is set in

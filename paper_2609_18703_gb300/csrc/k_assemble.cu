@@ -276,11 +276,11 @@ __global__ void __maxnreg__(56) asm_members_kernel(AssembleArgs a) {
       }
     }
     // all record loads first (no store in between), so they overlap
-    Rec rr[AM_ITEMS];
+    Slot rr[AM_ITEMS];
 #pragma unroll
     for (int k = 0; k < AM_ITEMS; ++k) {
       if (ridx[k] != NONE) {
-        rr[k] = a.rec[ridx[k]];
+        rr[k] = a.slot[ridx[k]];
       } else {
         rr[k].len = 0;
         rr[k].w = 0;
@@ -293,7 +293,7 @@ __global__ void __maxnreg__(56) asm_members_kernel(AssembleArgs a) {
     for (int k = 0; k < AM_ITEMS; ++k) {
       contrib[k] = 0;
       src[k] = 0;
-      const Rec r = rr[k];
+      const Slot r = rr[k];
       if (w_state(r.w) == ST_PRESENT && r.len) {
         contrib[k] = r.len;
         src[k] = w_off(r.w);

@@ -53,7 +53,7 @@ __device__ __forceinline__ void stat_add(unsigned long long* s, unsigned long lo
 
 
 // record word read past L1 (other threads update it with atomics at L2)
-__device__ __forceinline__ uint64_t ld_w(const Rec* rc) {
+__device__ __forceinline__ uint64_t ld_w(const Slot* rc) {
   return __ldcg((const unsigned long long*)&rc->w);
 }
 
@@ -169,23 +169,28 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
       if (c >= a.N || !valid_state || !in_bounds) {
         v = V_INVALID;
       } else {
-        // parent and heavy flag, immutable: read alongside the fence
+        // the parent, immutable.  A fill tile of FILL_TILE children that
+        // starts with the same parent as the next one is one heavy parent's
+        // (it has more than HEAVY_CHILDREN children): the small fill-tile
+        // table, resident in L2, names it, and the report touches no sector
+        // but its slot's.  Otherwise it is read alongside the fence.
         uint32_t par;
-        if (a.heavy) {
-          const ulonglong2 rv = *reinterpret_cast<const ulonglong2*>(a.rec + c);
-          par = (uint32_t)rv.x;
-          heavy = (rv.y & W_HEAVY_BIT) != 0ull;
+        const uint64_t t = c / FILL_TILE;
+        if (a.heavy && t + 1 < a.n_fill_tiles) {
+          const uint32_t f0 = __ldg(a.tfp + t), f1 = __ldg(a.tfp + t + 1);
+          heavy = f0 == f1;
+          par = heavy ? f0 : a.par[c];
         } else {
-          par = a.rec[c].parent;
+          par = a.par[c];
         }
         // Eq. (3): accept iff IN-FLIGHT at the report's generation
         const uint32_t want = ph_make(PH_INFLIGHT, g);
         uint32_t cur;
         bool won = false;
         if (g >> 30) {
-          cur = a.phase[c];   // no Grain ever reaches such a generation
+          cur = a.slot[c].phase;   // no Grain ever reaches such a generation
         } else {
-          cur = atomicCAS(a.phase + c, want, ph_make(PH_SEALED, g));
+          cur = atomicCAS(&a.slot[c].phase, want, ph_make(PH_SEALED, g));
           won = cur == want;
         }
         if (won) {
@@ -193,7 +198,7 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
           const bool present = s == ST_PRESENT;
           // a GroupFailure's own Grain failed
           const uint8_t outcome = (s == ST_GROUP_FAILURE) ? ST_FAILED : s;
-          Rec* rc = a.rec + c;
+          Slot* rc = a.slot + c;
           rc->len = present ? l : 0u;
           atomicOr((unsigned long long*)&rc->w,
                    (unsigned long long)((present ? (o & W_OFF_MASK) : 0ull) |
@@ -205,13 +210,13 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
           v = V_NOT_INFLIGHT;
         } else if ((cur >> 2) != g) {
           v = V_STALE;
-        } else if (ld_w(a.rec + c) & W_BARRIER_BIT) {
+        } else if (ld_w(a.slot + c) & W_BARRIER_BIT) {
           v = V_BARRIER;   // suppressed by a sibling's GroupFailure in an earlier call
         } else {
           // SEALED at this generation: a duplicate, possibly of a report of
           // this same call with a higher index (ordered by commit_fix)
           v = V_DUP_CANDIDATE;
-          atomicOr((unsigned long long*)&a.rec[c].w, (unsigned long long)W_CONFLICT_BIT);
+          atomicOr((unsigned long long*)&a.slot[c].w, (unsigned long long)W_CONFLICT_BIT);
         }
       }
       a.code[r] = v;
@@ -284,7 +289,7 @@ __device__ void apply_barriers_grid(const CommitArgs& a, uint64_t n) {
         v = a.code[r];
         if (v == V_ACCEPT || v == V_NOT_INFLIGHT) {
           c = a.child[r];
-          p = a.rec[c].parent;
+          p = a.par[c];
           if (gb_get(a, p, &b)) {
             under = r > b;
             trig = r == b;   // the barrier's own (accepted) GroupFailure report
@@ -293,7 +298,7 @@ __device__ void apply_barriers_grid(const CommitArgs& a, uint64_t n) {
       }
       if (under) {
         if (v == V_ACCEPT) {
-          Rec* rc = a.rec + c;
+          Slot* rc = a.slot + c;
           const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
           rc->len = 0u;
           rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
@@ -305,7 +310,7 @@ __device__ void apply_barriers_grid(const CommitArgs& a, uint64_t n) {
           atomicAdd(&s_d[4], 1ull);
           atomicAdd(&s_d[6], 1ull);
         } else {
-          const uint32_t ph = __ldcg(a.phase + c);
+          const uint32_t ph = __ldcg(&a.slot[c].phase);
           const uint32_t gen_c = ((ph & 3u) == PH_WAITING) ? 0u : (ph >> 2);
           const uint32_t g = a.gen ? a.gen[r] : 0u;
           const bool same = g == gen_c;
@@ -375,7 +380,7 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
   //    minimum-index election in the record's len field with its own index
   for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
     if (a.code[r] != V_ACCEPT) continue;
-    Rec* rc = a.rec + a.child[r];
+    Slot* rc = a.slot + a.child[r];
     if (ld_w(rc) & W_CONFLICT_BIT) {
       rc->len = (uint32_t)r;
       atomicOr((unsigned long long*)&rc->w, (unsigned long long)W_SEALER_BIT);
@@ -386,7 +391,7 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
   //    duplicates of an earlier call's publication
   for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
     if (a.code[r] != V_DUP_CANDIDATE) continue;
-    Rec* rc = a.rec + a.child[r];
+    Slot* rc = a.slot + a.child[r];
     if (ld_w(rc) & W_SEALER_BIT) {
       atomicMin(&rc->len, (uint32_t)r);
     } else {
@@ -400,7 +405,7 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
   for (uint64_t r = threadIdx.x; r < n; r += blockDim.x) {
     const uint8_t v = a.code[r];
     if (v != V_ACCEPT && v != V_DUP_CANDIDATE) continue;
-    const Rec* rc = a.rec + a.child[r];
+    const Slot* rc = a.slot + a.child[r];
     if (!(ld_w(rc) & W_SEALER_BIT)) continue;
     const bool win = __ldcg(&rc->len) == (uint32_t)r;
     a.code[r] = (v == V_ACCEPT) ? (win ? V_WIN_SEALER : V_LOSE_SEALER)
@@ -413,8 +418,9 @@ __device__ void resolve_duplicates(const CommitArgs& a, uint64_t n) {
     if (v < V_WIN_SEALER || v > V_LOSE_CAND) continue;
     const uint8_t s = a.state[r];
     const bool bad = (s == ST_FAILED || s == ST_SUPPRESSED || s == ST_GROUP_FAILURE);
-    Rec* rc = a.rec + a.child[r];
-    const uint32_t p = rc->parent;
+    const uint64_t c = a.child[r];
+    Slot* rc = a.slot + c;
+    const uint32_t p = a.par[c];
     if (v == V_WIN_SEALER || v == V_WIN_CAND) {
       const bool present = s == ST_PRESENT;
       const uint8_t outcome = (s == ST_GROUP_FAILURE) ? ST_FAILED : s;
@@ -451,15 +457,17 @@ __device__ void seal_open(const CommitArgs& a, uint32_t pp, int lane, unsigned l
   const uint64_t c0 = a.offsets[pp], c1 = a.offsets[pp + 1];
   uint32_t k_wait = 0, k_fly = 0;
   for (uint64_t d = c0 + lane; d < c1; d += 32) {
-    const uint32_t ph = __ldcg(a.phase + d);
+    Slot* rc = a.slot + d;
+    const uint32_t ph = __ldcg(&rc->phase);
     const uint32_t f = ph & 3u;
     if (f == PH_SEALED) continue;
     const uint32_t gen_d = (f == PH_WAITING) ? 0u : (ph >> 2);
-    a.phase[d] = ph_make(PH_SEALED, gen_d);
-    Rec* rc = a.rec + d;
-    const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
-    rc->len = 0u;
-    rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
+    Slot sl;   // the whole slot in one store
+    sl.phase = ph_make(PH_SEALED, gen_d);
+    sl.len = 0u;
+    sl.w = (ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK)) | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) |
+           W_BARRIER_BIT;
+    *rc = sl;
     if (f == PH_INFLIGHT) ++k_fly; else ++k_wait;
   }
   for (int sh = 16; sh > 0; sh >>= 1) {
@@ -513,7 +521,7 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
   auto parent_of = [&](uint64_t r, uint32_t* p) -> bool {
     const uint64_t c = a.child[r];
     if (c >= a.N) return false;
-    *p = a.rec[c].parent;
+    *p = a.par[c];
     return true;
   };
   // 0: the call's GroupFailure reports (with a valid child)
@@ -595,7 +603,7 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
       *b = s_sb[lo];
       return true;
     }
-    const uint32_t pp = a.rec[c].parent;
+    const uint32_t pp = a.par[c];
     uint32_t bb;
     if (!gb_get(a, pp, &bb)) return false;
     *p = pp;
@@ -621,7 +629,7 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
       uint32_t p, b;
       if (!barrier_of(c, &p, &b) || r <= b) continue;
       if (v == V_ACCEPT) {
-        Rec* rc = a.rec + c;
+        Slot* rc = a.slot + c;
         const uint64_t keep = ld_w(rc) & ~(W_OFF_MASK | W_STATE_MASK);
         rc->len = 0u;
         rc->w = keep | ((uint64_t)ST_SUPPRESSED << W_STATE_SHIFT) | W_BARRIER_BIT;
@@ -633,7 +641,7 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
         atomicAdd(&s_d[4], 1ull);
         atomicAdd(&s_d[6], 1ull);
       } else {
-        const uint32_t ph = __ldcg(a.phase + c);
+        const uint32_t ph = __ldcg(&a.slot[c].phase);
         const uint32_t gen_c = ((ph & 3u) == PH_WAITING) ? 0u : (ph >> 2);
         const uint32_t g = a.gen ? a.gen[r] : 0u;
         const bool same = g == gen_c;
@@ -658,7 +666,7 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n) {
       const uint64_t r = base + j, c = a.child[r];
       uint32_t p, b;
       if (!barrier_of(c, &p, &b) || r <= b) continue;
-      if (!(ld_w(a.rec + c) & W_BARRIER_BIT)) continue;   // sealed before the barrier
+      if (!(ld_w(a.slot + c) & W_BARRIER_BIT)) continue;   // sealed before the barrier
       a.code[r] = V_BARRIER;
       atomicAdd(&s_d[3], ~0ull);
       atomicAdd(&s_d[4], 1ull);

@@ -193,12 +193,12 @@ __device__ __forceinline__ MemberMap map_members(const CpShared& sh, uint32_t cn
 }
 
 __device__ __forceinline__ void load_records(const CommitArgs& a, const CpShared& sh, const MemberMap& mm,
-                                             uint64_t gt, Rec* rr) {
+                                             uint64_t gt, Slot* rr) {
 #pragma unroll
   for (int k = 0; k < CP_ITEMS; ++k) {
     if (mm.valid & (1u << k)) {
       const uint32_t i = mm.par[k];
-      rr[k] = a.rec[(uint64_t)sh.coff[i] + (gt + k - sh.pmb[i])];
+      rr[k] = a.slot[(uint64_t)sh.coff[i] + (gt + k - sh.pmb[i])];
     } else {
       rr[k].len = 0;
       rr[k].w = 0;
@@ -206,7 +206,7 @@ __device__ __forceinline__ void load_records(const CommitArgs& a, const CpShared
   }
 }
 
-__device__ __forceinline__ uint32_t contrib_of(const Rec& r) {
+__device__ __forceinline__ uint32_t contrib_of(const Slot& r) {
   return (w_state(r.w) == ST_PRESENT) ? r.len : 0u;
 }
 
@@ -283,7 +283,7 @@ __global__ void __maxnreg__(CP_MAXREG) commit_plan_kernel(CommitArgs a) {
       for (uint64_t r0 = mlo; r0 < mhi; r0 += CP_ROUND) {
         const uint64_t gt = r0 + (uint64_t)threadIdx.x * CP_ITEMS;
         const MemberMap mm = map_members(sh, cnt, gt, mhi);
-        Rec rr[CP_ITEMS];
+        Slot rr[CP_ITEMS];
         load_records(a, sh, mm, gt, rr);
 #pragma unroll
         for (int k = 0; k < CP_ITEMS; ++k) {
@@ -373,7 +373,7 @@ __global__ void __maxnreg__(CP_MAXREG) commit_plan_kernel(CommitArgs a) {
             csrc[k] = sh.csrc[threadIdx.x * CP_ITEMS + k];
           }
         } else {
-          Rec rr[CP_ITEMS];
+          Slot rr[CP_ITEMS];
           load_records(a, sh, mm, gt, rr);
 #pragma unroll
           for (int k = 0; k < CP_ITEMS; ++k) {

@@ -55,11 +55,11 @@ __global__ void __launch_bounds__(EXP_THREADS) expand_scan_kernel(ExpandScanArgs
       mine.a += cnt[k];
       mine.b += (p < a.P && cnt[k] == 0u) ? 1ull : 0ull;
     }
-    uint32_t heavy = 0;
+    unsigned long long heavy = 0;   // children of heavy parents
 #pragma unroll
-    for (int k = 0; k < EXP_ITEMS; ++k) heavy += cnt[k] >= HEAVY_CHILDREN ? 1u : 0u;
-    heavy = __reduce_add_sync(0xffffffffu, heavy);
-    if ((threadIdx.x & 31) == 0 && heavy) atomicAdd(&ds->n_heavy, (unsigned long long)heavy);
+    for (int k = 0; k < EXP_ITEMS; ++k) heavy += cnt[k] >= HEAVY_CHILDREN ? cnt[k] : 0u;
+    for (int d = 16; d > 0; d >>= 1) heavy += __shfl_xor_sync(0xffffffffu, heavy, d);
+    if ((threadIdx.x & 31) == 0 && heavy) atomicAdd(&ds->n_heavy, heavy);
     Pair64 total;
     Pair64 excl = block_excl_scan_pair(mine, s_scan, &total);
     if (threadIdx.x < 32) {  // one warp looks back
@@ -124,12 +124,11 @@ __global__ void __launch_bounds__(FILL_THREADS) expand_fill_kernel(ExpandFillArg
     }
     __syncthreads();
     for (uint64_t c = c0 + threadIdx.x; c < c1; c += blockDim.x) {
-      uint64_t p, base, end;
+      uint64_t p, base;
       if (staged) {
         const uint32_t k = last_le(s_off, 0u, (uint32_t)R - 1u, c);
         p = p_lo + k;
         base = s_off[k];
-        end = s_off[k + 1];
       } else {
         // many empty parents inside one tile: search the global offsets
         uint64_t lo = p_lo, hi = p_hi + 1;
@@ -142,17 +141,16 @@ __global__ void __launch_bounds__(FILL_THREADS) expand_fill_kernel(ExpandFillArg
         }
         p = lo;
         base = a.offsets[lo];
-        end = a.offsets[lo + 1];
       }
       const uint32_t call = a.parent_call ? (uint32_t)a.parent_call[p] : 0u;
       a.child_parent[c] = (uint32_t)p;
       a.child_ordinal[c] = (uint32_t)(c - base);
-      a.phase[c] = WAIT_UNCLAIMED;
-      Rec r;
-      r.parent = (uint32_t)p;
-      r.len = 0u;
-      r.w = ((uint64_t)call << W_CALL_SHIFT) | (end - base >= HEAVY_CHILDREN ? W_HEAVY_BIT : 0ull);
-      a.rec[c] = r;
+      a.par[c] = (uint32_t)p;
+      Slot sl;
+      sl.phase = WAIT_UNCLAIMED;
+      sl.len = 0u;
+      sl.w = (uint64_t)call << W_CALL_SHIFT;
+      a.slot[c] = sl;
     }
     __syncthreads();
   }

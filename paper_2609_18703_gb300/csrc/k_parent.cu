@@ -48,7 +48,7 @@ __global__ void __launch_bounds__(PB_THREADS) pb_keys_kernel(ParentArgs a) {
       c[u] = j < Q ? a.queue[head + j] : 0u;
     }
 #pragma unroll
-    for (int u = 0; u < U; ++u) p[u] = j0 + u * stride < Q ? a.rec[c[u]].parent : 0u;
+    for (int u = 0; u < U; ++u) p[u] = j0 + u * stride < Q ? a.par[c[u]] : 0u;
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const uint64_t j = j0 + u * stride;
@@ -325,7 +325,7 @@ __global__ void __launch_bounds__(PB_THREADS) pb_emit_kernel(ParentArgs a) {
   if (ds->pb_err) {
     // refused: the admitted Grains go back to WAITING, the tail back
     const uint64_t t0 = ds->pb_old_tail, t1 = head + Q;
-    for (uint64_t t = t0 + g; t < t1; t += stride) a.phase[a.queue[t]] = WAIT_UNCLAIMED;
+    for (uint64_t t = t0 + g; t < t1; t += stride) a.slot[a.queue[t]].phase = WAIT_UNCLAIMED;
     if (g == 0) a.qstate[1] = t0;
     return;
   }
@@ -342,7 +342,7 @@ __global__ void __launch_bounds__(PB_THREADS) pb_emit_kernel(ParentArgs a) {
     if (hw >= stop) continue;
     const uint32_t c = a.child[val[s]];
     a.batched[a.hoff[hw] + k] = c;
-    a.phase[c] = (a.phase[c] & ~3u) | PH_INFLIGHT;
+    a.slot[c].phase = (a.slot[c].phase & ~3u) | PH_INFLIGHT;
   }
   for (uint64_t j = g; j < R; j += stride) a.queue[head + npop + j] = a.rem[j];
   if (g == 0) {

@@ -17,13 +17,19 @@
 
 namespace ro {
 
-__device__ __forceinline__ bool retry_target(const RetryArgs& a, uint64_t c, uint32_t* ph) {
-  if (c >= a.N) return false;
-  const uint32_t w = a.phase[c];
-  if ((w & 3u) != PH_INFLIGHT) return false;
-  if (a.check_call && w_call(a.rec[c].w) != a.call) return false;
-  *ph = w;
-  return true;
+// Grain c is a target: IN-FLIGHT and of the Call (from its slot v, read
+// whole: phase word, len and w share one sector).
+__device__ __forceinline__ bool retry_target(const RetryArgs& a, const Slot& v) {
+  if ((v.phase & 3u) != PH_INFLIGHT) return false;
+  return !a.check_call || w_call(v.w) == a.call;
+}
+__device__ __forceinline__ Slot load_slot(const Slot* p) {
+  const ulonglong2 v = __ldcg(reinterpret_cast<const ulonglong2*>(p));
+  Slot s;
+  s.phase = (uint32_t)v.x;
+  s.len = (uint32_t)(v.x >> 32);
+  s.w = v.y;
+  return s;
 }
 
 __global__ void __launch_bounds__(RT_THREADS) retry_claim_kernel(RetryArgs a) {
@@ -31,8 +37,7 @@ __global__ void __launch_bounds__(RT_THREADS) retry_claim_kernel(RetryArgs a) {
   const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
   for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < a.n; i += stride) {
     const uint64_t c = a.children[i];
-    uint32_t ph;
-    if (retry_target(a, c, &ph)) atomicMax(&a.rec[c].len, ~(uint32_t)i);
+    if (c < a.N && retry_target(a, load_slot(a.slot + c))) atomicMax(&a.slot[c].len, ~(uint32_t)i);
   }
 }
 
@@ -55,26 +60,25 @@ __global__ void __launch_bounds__(RT_THREADS) retry_scatter_kernel(RetryArgs a) 
     __syncthreads();
     if (tile >= n_tiles) break;
     const uint64_t i0 = tile * TILE + (uint64_t)threadIdx.x * RT_ITEMS;
+    // the group's entries, then their slots, every load in flight at once
     uint32_t cs[RT_ITEMS], phs[RT_ITEMS];
+#pragma unroll
+    for (int k = 0; k < RT_ITEMS; ++k) cs[k] = i0 + k < a.n ? a.children[i0 + k] : 0u;
     uint32_t flags = 0;
-    unsigned long long cnt = 0;
 #pragma unroll
     for (int k = 0; k < RT_ITEMS; ++k) {
-      const uint64_t i = i0 + k;
-      cs[k] = 0;
       phs[k] = 0;
-      if (i >= a.n) continue;
-      const uint64_t c = a.children[i];
-      uint32_t ph;
-      // the winner still sees its own claim; a later entry for the same
-      // Grain sees another claim or the cleared one
-      if (retry_target(a, c, &ph) && a.rec[c].len == ~(uint32_t)i) {
-        flags |= 1u << k;
-        cs[k] = (uint32_t)c;
-        phs[k] = ph;
-        ++cnt;
+      if (i0 + k < a.n && cs[k] < a.N) {
+        const Slot v = load_slot(a.slot + cs[k]);
+        // the winner still sees its own claim; a later entry for the same
+        // Grain sees another claim or the cleared one
+        if (retry_target(a, v) && v.len == ~(uint32_t)(i0 + k)) {
+          flags |= 1u << k;
+          phs[k] = v.phase;
+        }
       }
     }
+    const unsigned long long cnt = __popc(flags);
     unsigned long long total;
     const unsigned long long excl = block_excl_scan(cnt, s_scan, &total);
     if (threadIdx.x < 32) {  // one warp looks back
@@ -88,8 +92,8 @@ __global__ void __launch_bounds__(RT_THREADS) retry_scatter_kernel(RetryArgs a) 
       if (!(flags & (1u << k))) continue;
       const uint32_t c = cs[k];
       a.rq[rlen + rank] = c;
-      a.rec[c].len = 0u;
-      a.phase[c] = ph_make(PH_READY, (phs[k] >> 2) + 1u);
+      a.slot[c].len = 0u;
+      a.slot[c].phase = ph_make(PH_READY, (phs[k] >> 2) + 1u);
       ++rank;
     }
     if (tile == n_tiles - 1 && threadIdx.x == RT_THREADS - 1) {

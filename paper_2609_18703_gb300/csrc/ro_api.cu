@@ -85,7 +85,7 @@ struct PlanSlot {
 
 // Device buffers of one expansion slot, kept across ro_ctx_reset and reused.
 struct ExpSlot {
-  DevBuf offsets, pw, phase, rec, bitmap, tfp, gb;   // bitmap: BM_SLOTS slots
+  DevBuf offsets, pw, slot, par, bitmap, tfp, gb;   // bitmap: BM_SLOTS slots
   Ev bm_free[BM_SLOTS];   // the plan that read a bitmap slot is done
   int bm_stream[BM_SLOTS] = {};   // the completion stream that plan ran on
   ListSlot lists[RING];
@@ -98,7 +98,7 @@ struct Expansion {
   uint64_t P = 0, N = 0;
   uint64_t commits = 0, assembles = 0;
   int last_list = -1;   // list slot written by the latest commit
-  bool heavy = false;   // some parent has at least HEAVY_CHILDREN children
+  bool heavy = false;   // parents of at least HEAVY_CHILDREN children hold >= N/4 children
 };
 
 struct TsBuf {
@@ -563,6 +563,15 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_expand_scan = grid_for(kernel_ptr_expand(K_EXPAND_SCAN), EXP_THREADS, s, 4);
   c->L.grid_fill = grid_for(kernel_ptr_expand(K_FILL), FILL_THREADS, s, 8);
   c->L.grid_rb = grid_for(kernel_ptr_ready(K_RB_SCATTER), RB_THREADS, s, 8);
+  {
+    int coop = 0;
+    cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, device);
+    c->L.grid_rb_coop = coop ? grid_for(kernel_ptr_ready(K_RB_FUSED), RB_THREADS, s, 64) : 0;
+    // RO_ADMIT_TWO_PASS=1 in the environment at context creation keeps every
+    // admission on the two-pass path
+    if (const char* e = std::getenv("RO_ADMIT_TWO_PASS"))
+      if (std::strtoul(e, nullptr, 10) != 0) c->L.grid_rb_coop = 0;
+  }
   c->L.grid_commit = grid_for(kernel_ptr_commit(K_COMMIT), CM_THREADS, s, 8);
   c->L.grid_cplan = grid_for(kernel_ptr_complete(), CP_THREADS, s, 4);
   c->L.grid_aparents = grid_for(kernel_ptr_assemble(K_APARENTS), AP_THREADS, s, 4);
@@ -591,7 +600,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   DeviceGuard g(c->device);
   sync_all_streams(c);
   for (auto& s : c->slots) {
-    free_buf(s.offsets); free_buf(s.pw); free_buf(s.phase); free_buf(s.rec); free_buf(s.bitmap);
+    free_buf(s.offsets); free_buf(s.pw); free_buf(s.slot); free_buf(s.par); free_buf(s.bitmap);
     free_buf(s.tfp); free_buf(s.gb);
     for (auto& e : s.bm_free) free_ev(e);
     for (auto& l : s.lists) {
@@ -800,8 +809,8 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
     return fail(c, RO_E_INVAL, "ro_expand: NULL child arrays");
 
   const uint64_t mtfp_cap = ceil_div(N, AM_TILE) + 2;
-  RO_TRY(ensure(c, S.phase, N * sizeof(uint32_t), "phase words"));
-  RO_TRY(ensure(c, S.rec, N * sizeof(Rec), "result records"));
+  RO_TRY(ensure(c, S.slot, N * sizeof(Slot), "child slots"));
+  RO_TRY(ensure(c, S.par, N * sizeof(uint32_t), "child parents"));
   RO_TRY(ensure(c, S.bitmap, BM_SLOTS * ceil_div(P, 32) * sizeof(uint32_t), "completion bitmaps"));
   RO_TRY(ensure(c, S.gb, P * sizeof(unsigned long long), "GroupFailure barriers"));
   for (auto& l : S.lists) {
@@ -832,8 +841,8 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   fa.parent_call = d_parent_call;
   fa.child_parent = d_child_parent;
   fa.child_ordinal = d_child_ordinal;
-  fa.phase = (uint32_t*)S.phase.p;
-  fa.rec = (Rec*)S.rec.p;
+  fa.slot = (Slot*)S.slot.p;
+  fa.par = (uint32_t*)S.par.p;
   launch_expand_fill(c->L, fa);
   RO_TRY(check_launch(c, "expand_fill"));
   if (S.queues.size() < c->n_calls) S.queues.resize(c->n_calls);
@@ -843,7 +852,7 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
   x.parent_xid = parent_xid;
   x.P = P;
   x.N = N;
-  x.heavy = c->hs->n_heavy != 0;
+  x.heavy = c->hs->n_heavy != 0 && 4 * c->hs->n_heavy >= x.N;
   c->exps.push_back(x);
   *xid = (int32_t)slot;
   return RO_OK;
@@ -870,8 +879,7 @@ ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* 
   ra.cand = d_cand;
   ra.n_cand = d_cand ? n_cand : x->N;
   ra.N = x->N;
-  ra.phase = (uint32_t*)S.phase.p;
-  ra.rec = (const Rec*)S.rec.p;
+  ra.slot = (Slot*)S.slot.p;
   ra.check_call = c->n_calls > 1;
   ra.call = call;
   ra.batch_size = batch_size;
@@ -949,8 +957,7 @@ ro_status ro_batch_ready_parent(ro_ctx* c, int32_t xid, uint32_t call, const uin
   ra.cand = d_cand;
   ra.n_cand = d_cand ? n_cand : N;
   ra.N = N;
-  ra.phase = (uint32_t*)S.phase.p;
-  ra.rec = (const Rec*)S.rec.p;
+  ra.slot = (Slot*)S.slot.p;
   ra.check_call = c->n_calls > 1;
   ra.call = call;
   ra.batch_size = batch_size;
@@ -975,8 +982,8 @@ ro_status ro_batch_ready_parent(ro_ctx* c, int32_t xid, uint32_t call, const uin
   int bits = 0;
   while (bits < 32 && P > 1 && ((P - 1) >> bits) != 0) ++bits;
   pa.passes = (bits + 7) / 8;
-  pa.rec = (const Rec*)S.rec.p;
-  pa.phase = (uint32_t*)S.phase.p;
+  pa.par = (const uint32_t*)S.par.p;
+  pa.slot = (Slot*)S.slot.p;
   pa.queue = (uint32_t*)Q.q.p;
   pa.qstate = (unsigned long long*)Q.state.p;
   pa.batched = d_batched;
@@ -1033,8 +1040,7 @@ ro_status ro_retry(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* d_chil
   ta.children = d_children;
   ta.n = n;
   ta.N = x->N;
-  ta.phase = (uint32_t*)S.phase.p;
-  ta.rec = (Rec*)S.rec.p;
+  ta.slot = (Slot*)S.slot.p;
   ta.check_call = c->n_calls > 1;
   ta.call = call;
   ta.rq = (uint32_t*)Q.rq.p;
@@ -1082,13 +1088,15 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   ca.arena_bytes = arena_bytes;
   ca.N = x->N;
   ca.P = x->P;
-  ca.phase = (uint32_t*)S.phase.p;
-  ca.rec = (Rec*)S.rec.p;
+  ca.slot = (Slot*)S.slot.p;
+  ca.par = (const uint32_t*)S.par.p;
   ca.pw = (unsigned long long*)S.pw.p;
   const int bs = (int)(x->commits % BM_SLOTS);   // bitmap slot of this commit
   const uint64_t n_words = ceil_div(x->P, 32);
   ca.bitmap = (uint32_t*)S.bitmap.p + bs * n_words;
   ca.heavy = x->heavy ? 1 : 0;
+  ca.tfp = (const uint32_t*)S.tfp.p;
+  ca.n_fill_tiles = ceil_div(x->N, FILL_TILE);
   ca.gb = (unsigned long long*)S.gb.p;
   if (++c->commit_seq == 0) {   // wrapped: old tags could look current again
     for (auto& sl : c->slots)
@@ -1273,7 +1281,7 @@ ro_status assemble_impl(ro_ctx* c, int32_t xid, const uint8_t* d_arena, uint64_t
   aa.N = x->N;
   aa.offsets = (const uint64_t*)S.offsets.p;
   aa.pw = (const unsigned long long*)S.pw.p;
-  aa.rec = (const Rec*)S.rec.p;
+  aa.slot = (const Slot*)S.slot.p;
   aa.arena = d_arena;
   aa.arena_bytes = arena_bytes;
   aa.arena_host = arena_host;

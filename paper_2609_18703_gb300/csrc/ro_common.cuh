@@ -1,14 +1,17 @@
 // ro_common.cuh — layouts and device helpers shared by the lineage kernels.
 //
 // Per-child state of an expansion lives in two arrays:
-//   phase[c]  uint32 Grain phase word (Eq. 2): bits 0-1 phase; for WAITING the
-//             upper 30 bits hold the admission claim of the current
-//             ro_batch_ready call (all ones = unclaimed), otherwise the
-//             attempt generation (Eq. 3).
-//   rec[c]    16-byte record: immediate parent, payload length and one word
-//             packing the arena offset (48 bits), the published outcome
-//             (3 bits), whether the parent is heavy (at least HEAVY_CHILDREN
-//             children), commit bookkeeping flags and the Call (8 bits).
+//   slot[c]   16 bytes, one 32-byte sector holds it whole:
+//             phase  uint32 Grain phase word (Eq. 2): bits 0-1 phase; for
+//                    WAITING the upper 30 bits hold the admission claim of
+//                    the current ro_batch_ready call (all ones = unclaimed),
+//                    otherwise the attempt generation (Eq. 3);
+//             len    payload length of the published result;
+//             w      the arena offset (48 bits), the published outcome
+//                    (3 bits), commit bookkeeping flags and the Call (8 bits).
+//             The fence CAS, the Call check and the publish of a result
+//             touch this one sector.
+//   par[c]    uint32 immediate parent, written once at expansion.
 // Per-parent state: pw[p] = remaining unsealed members (low 32 bits) plus the
 // number of Failed/Suppressed members (high 32 bits), so one 64-bit atomic add
 // both counts a member down and records its outcome class.
@@ -40,25 +43,26 @@ constexpr uint8_t V_ACCEPT = 0, V_INVALID = 1, V_NOT_INFLIGHT = 2, V_STALE = 3,
 // ACCEPT or DUPLICATE by the commit's ordering pass
 constexpr uint8_t V_DUP_CANDIDATE = 6;
 
-// ---- result record ----------------------------------------------------------
-struct __align__(16) Rec {
-  uint32_t parent;
+// ---- per-child slot -----------------------------------------------------------
+struct __align__(16) Slot {
+  uint32_t phase;
   uint32_t len;
-  uint64_t w;   // off (0-47) | state (48-50) | heavy parent (52) | barrier (53) | sealer-seen (54) |
-                // conflict (55) | call (56-63)
+  uint64_t w;   // off (0-47) | state (48-50) | barrier (53) | sealer-seen (54) | conflict (55) |
+                // call (56-63)
 };
 constexpr uint64_t W_OFF_MASK = (1ull << 48) - 1;
 constexpr int W_STATE_SHIFT = 48;
 constexpr uint64_t W_STATE_MASK = 7ull << W_STATE_SHIFT;
-constexpr uint64_t W_HEAVY_BIT = 1ull << 52;     // the parent has >= HEAVY_CHILDREN children (set at expand)
 constexpr uint64_t W_BARRIER_BIT = 1ull << 53;   // sealed by a sibling's GroupFailure
 constexpr uint64_t W_SEALER_BIT = 1ull << 54;
 constexpr uint64_t W_CONFLICT_BIT = 1ull << 55;
 constexpr int W_CALL_SHIFT = 56;
 constexpr uint64_t MAX_ARENA = 1ull << 48;
-// A parent with at least this many children is heavy: a commit counts its
+// A parent with at least this many children is heavy.  When heavy parents
+// hold a quarter of an expansion's children or more, a commit counts their
 // members down in shared memory per CTA and adds them to the parent's
-// counter once per CTA (its reports seldom share a warp).
+// counter once per CTA (their reports seldom share a warp), and takes their
+// parent from the fill-tile table instead of the per-child parent array.
 constexpr uint32_t HEAVY_CHILDREN = 4096;
 
 __device__ __forceinline__ uint8_t w_state(uint64_t w) {
@@ -111,7 +115,8 @@ struct DevScalars {
   uint32_t pad0;
   unsigned long long stats[13];  // same order as ro_stats
   // ro_expand
-  unsigned long long n_children, n_empty, last_nonempty_parent, n_heavy;
+  unsigned long long n_children, n_empty, last_nonempty_parent,
+      n_heavy;   // children of parents with at least HEAVY_CHILDREN children
   // ro_gather_commit
   unsigned long long cm_n, cm_n_done[2];   // completed parents, per plan slot
   // per commit, in two slots (commit sequence & 1): duplicate candidates and
@@ -134,13 +139,16 @@ struct DevScalars {
   unsigned long long epoch[8];
 };
 // Admission scalars of one Call (ro_batch_ready): the first pass's counts,
-// its exit ticket and the reservation it plans, and the scatter pass's tile
-// counter, exit ticket and scan epoch.  One per Call, so that admissions of
+// its exit ticket and the reservation it plans, the scatter pass's tile
+// counter, exit ticket and scan epoch, and the one-pass admission's grid
+// barrier.  One per Call, so that admissions of
 // different Calls can run at the same time on streams of their own.
 struct alignas(128) ReadyScalars {
   unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
   unsigned long long epoch;
   uint32_t rb_ticket, rb_err, tile_ctr, exit_ctr;
+  // grid barrier of the one-pass admission: arrivals, generation
+  uint32_t bar_count, bar_gen;
 };
 // TS_COMMIT and TS_COMMIT_ODD: the completion lists and plans of commits of
 // even and odd sequence (they may run at the same time, on two streams);

@@ -56,7 +56,7 @@ constexpr uint64_t AC_SMALL_CHUNKS = 256;
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CPLAN, K_APARENTS,
                 K_AMEMBERS, K_ACOPY, K_RT_CLAIM, K_RT_SCATTER, K_PB_KEYS, K_PB_HIST,
                 K_PB_ROWSCAN, K_PB_SORT, K_PB_BOUNDS, K_PB_HEADS, K_PB_MARK, K_PB_SCAN, K_PB_EMIT,
-                K_CFIX, K_COUNT };
+                K_CFIX, K_RB_FUSED, K_COUNT };
 
 
 // Launch counter and optional CUDA-event timing of selected kernels, on the
@@ -70,6 +70,8 @@ struct LaunchCfg {
   Profiler* prof;
   int grid_expand_scan, grid_fill, grid_rb, grid_commit, grid_cplan, grid_aparents,
       grid_amembers, grid_acopy, grid_retry, grid_pb, grid_pb_sort;
+  // CTAs of the one-pass admission the device holds at once (0: no cooperative launch)
+  int grid_rb_coop;
 };
 
 // Launch one kernel between the profiler's marks, with programmatic
@@ -88,6 +90,26 @@ inline void launch_k(const LaunchCfg& L, int kid, void (*kern)(Arg), int grid, i
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, kern, a);
+  prof_end(L.prof, L.stream, kid);
+}
+
+// The same for a kernel whose CTAs wait for one another (grid barriers): a
+// cooperative launch, so that every CTA of the grid is resident at once (the
+// grid must not exceed what the device holds; see LaunchCfg::grid_rb_coop).
+// No programmatic dependent launch: the kernel starts after its predecessor.
+template <typename Arg>
+inline void launch_coop(const LaunchCfg& L, int kid, void (*kern)(Arg), int grid, int block, const Arg& a) {
+  prof_begin(L.prof, L.stream, kid);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3((unsigned)block);
+  cfg.stream = L.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cudaLaunchKernelEx(&cfg, kern, a);
@@ -116,8 +138,8 @@ struct ExpandFillArgs {
   const uint8_t* parent_call;  // optional
   uint32_t* child_parent;
   uint32_t* child_ordinal;
-  uint32_t* phase;
-  Rec* rec;
+  Slot* slot;
+  uint32_t* par;
 };
 void launch_expand_fill(const LaunchCfg& L, const ExpandFillArgs& a);
 
@@ -126,8 +148,7 @@ struct ReadyArgs {
   const uint32_t* cand;       // NULL: all children in id order
   uint64_t n_cand;
   uint64_t N;
-  uint32_t* phase;
-  const Rec* rec;             // read for the Call when the expansion has several
+  Slot* slot;                 // phase word; the Call (w) when the expansion has several
   int check_call;
   int calls_concurrent;       // other Calls' admissions may run at the same time
   uint32_t call, batch_size;
@@ -154,8 +175,8 @@ struct ParentArgs {
   int flush;
   int passes;                 // 8-bit digit passes covering the largest parent id
   int pass;                   // the sort pass of this launch
-  const Rec* rec;
-  uint32_t* phase;
+  const uint32_t* par;
+  Slot* slot;
   uint32_t* queue;
   unsigned long long* qstate;
   uint32_t* batched;
@@ -187,8 +208,7 @@ struct RetryArgs {
   const uint32_t* children;
   uint64_t n;
   uint64_t N;
-  uint32_t* phase;
-  Rec* rec;                   // len of an IN-FLIGHT Grain holds the claim (~index) meanwhile
+  Slot* slot;                 // len of an IN-FLIGHT Grain holds the claim (~index) meanwhile
   int check_call;
   uint32_t call;
   uint32_t* rq;               // recovery queue storage
@@ -235,11 +255,13 @@ struct CommitArgs {
   const uint32_t* gen;        // optional
   uint64_t arena_bytes;
   uint64_t N, P;
-  uint32_t* phase;
-  Rec* rec;
+  Slot* slot;
+  const uint32_t* par;
   unsigned long long* pw;
   uint32_t* bitmap;           // parents this call completed
-  int heavy;                  // the expansion has heavy parents: count them per CTA first
+  int heavy;                  // heavy parents hold a quarter of the children: count them per CTA first
+  const uint32_t* tfp;        // fill tile -> parent of its first child (expand_fill's table)
+  uint64_t n_fill_tiles;      // tiles of FILL_TILE children written in tfp
   unsigned long long* gb;     // per parent: (seq << 32) | ~r for the lowest accepted
                               // GroupFailure report r of commit seq; older seq: none
   uint32_t seq;               // this commit's sequence number in the context (from 1)
@@ -268,7 +290,7 @@ struct AssembleArgs {
   uint64_t P, N;
   const uint64_t* offsets;
   const unsigned long long* pw;
-  const Rec* rec;
+  const Slot* slot;
   const uint8_t* arena;
   uint64_t arena_bytes;
   int arena_host;             // the arena is pinned host memory: no bulk (TMA) copies from it

@@ -229,27 +229,29 @@ def test_video_nested_full_size():
         ls.check_stats()
 
 
-def test_streaming_full_size():
-    """The streaming configuration at full size and the benchmark's default
-    batch: four Calls, 50,000,050 children of 1 KB, 1,000 readiness waves;
-    per wave every Call admits the wave's ready children and reserves whole
+@pytest.mark.parametrize("B", [32, 256, 2048])
+def test_streaming_full_size(B):
+    """The streaming configuration at full size, at each batch size the
+    benchmark sweeps, with the bench's default streams (assembly planning and
+    copies on streams of their own, each Call's admissions on a stream of its
+    own): four Calls, 50,000,050 children of 1 KB, 1,000 readiness waves; per
+    wave every Call admits the wave's ready children and reserves whole
     batches (the last wave flushes), the reserved children's results are
     committed in their key order and the completed parents assembled.  Every
-    Call's reservation, every verdict, completed list, status, offset and
-    length equal the oracle's; the assembled bytes of one wave in 25 and of
-    the last wave are compared in full, and the total byte count of all."""
+    Call's reservation, every verdict, completed list, status, offset, length
+    and every wave's assembled bytes equal the oracle's (compared wave by
+    wave, so host memory stays bounded)."""
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     from tests.lockstep import Lockstep
     from tests.pipeline import host_arena
     from workload import streaming
-    lv = streaming().top
+    lv = streaming(batch_size=B).top
     assert lv.n_children == 50_000_050
     a = host_arena(lv)
     ad = _arena_dev(a)
-    B = lv.batch_size
     total = 0
-    with Lockstep(n_calls=4) as ls:
+    with Lockstep(n_calls=4, streams=True, call_streams=True) as ls:
         x = ls.expand(lv.counts, parent_call=lv.parent_call)["xid"]
         n_ready = lv.ready_bounds.size - 1
         for w in range(n_ready):
@@ -260,9 +262,7 @@ def test_streaming_full_size():
             got = got[np.argsort(lv.key[got], kind="stable")]
             ch, st, ln, of = lv.reports(got)
             cm = ls.commit(x, ch, st, ln, of, arena_bytes=lv.arena_bytes)
-            # the oracle assembles (and the test compares) bytes only when given the arena
-            r = ls.assemble(x, a if (w % 25 == 0 or last) else None, ad, parents=None,
-                            n_parents=max(cm["n_done"], 1))
+            r = ls.assemble(x, a, ad, parents=None, n_parents=max(cm["n_done"], 1))
             total += r["out_bytes"]
         ls.check_stats()
         assert ls.o.stats()["ready_bad_candidates"] == 0
