@@ -60,8 +60,9 @@ def parse(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="docpage", choices=WORKLOADS)
-    ap.add_argument("--one-call-stream", action="store_true",
-                    help="streaming: every Call admits on the context's stream (no Call streams)")
+    ap.add_argument("--admissions", default="calls", choices=["calls", "call-streams", "one-stream"],
+                    help="streaming: one ro_batch_ready_calls per wave (default), or one "
+                         "ro_batch_ready per Call on streams of their own, or on the context's stream")
     ap.add_argument("--batch", type=int, default=256, help="streaming: batch size (32, 256, 2048)")
     ap.add_argument("--children", type=int, default=50_000_000, help="streaming: children in total")
     ap.add_argument("--parents", type=int, default=1_000_000,
@@ -1238,9 +1239,14 @@ def run_streaming(args, rank, world, local_rank):
     torch.cuda.synchronize()
     ctx = ro.ro_ctx_create(local_rank, stream, lv.n_calls)
     ro.ro_ctx_set_streams(ctx, torch.cuda.Stream(), torch.cuda.Stream())
-    call_streams = [torch.cuda.Stream() for _ in range(lv.n_calls)] if not args.one_call_stream else []
+    call_streams = [torch.cuda.Stream() for _ in range(lv.n_calls)] if args.admissions == "call-streams" else []
     ro.ro_ctx_set_call_streams(ctx, call_streams)
     L = ro.load()
+    import ctypes
+    n_calls = lv.n_calls
+    c_calls = (ctypes.c_uint32 * n_calls)(*range(n_calls))
+    c_batched = (ctypes.c_void_p * n_calls)(*[b.data_ptr() for b in batched])
+    c_caps = (ctypes.c_uint64 * n_calls)(*([N + B] * n_calls))
 
     def expand():
         ro.ro_ctx_reset(ctx)
@@ -1256,10 +1262,14 @@ def run_streaming(args, rank, world, local_rank):
         cursor.zero_()
         for w in range(W):
             c0, c1 = int(lv.ready_bounds[w]), int(lv.ready_bounds[w + 1])
-            for c in range(lv.n_calls):
-                bad |= L.ro_batch_ready(ctx, xid, c, cand.data_ptr() + 4 * c0, c1 - c0, B,
-                                        int(w == W - 1), batched[c].data_ptr(), N + B, None, None,
-                                        None)
+            if args.admissions == "calls":   # every Call's admission in one launch
+                bad |= L.ro_batch_ready_calls(ctx, xid, n_calls, c_calls, cand.data_ptr() + 4 * c0, c1 - c0,
+                                              B, int(w == W - 1), c_batched, c_caps, None)
+            else:
+                for c in range(n_calls):
+                    bad |= L.ro_batch_ready(ctx, xid, c, cand.data_ptr() + 4 * c0, c1 - c0, B,
+                                            int(w == W - 1), batched[c].data_ptr(), N + B, None, None,
+                                            None)
             s, e = int(rb[w]), int(rb[w + 1])
             bad |= L.ro_gather_commit(ctx, xid, e - s, None, r_child.data_ptr() + 4 * s,
                                       r_state.data_ptr() + s, r_len.data_ptr() + 4 * s,
@@ -1345,9 +1355,11 @@ def run_streaming(args, rank, world, local_rank):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8/u32/u64",
             "data": "synthetic", "config": cfg,
             "parallelism": f"replicas x{world} (one microbatch per GPU)",
-            "run": {"kernels_per_wave": lv.n_calls * 2 + 4, "cuda_graph": True,
-                    "admissions": "on the context's stream" if args.one_call_stream
-                                  else "one stream per Call"},
+            "run": {"cuda_graph": True,
+                    "admissions": {"calls": "all Calls in one launch (ro_batch_ready_calls)",
+                                   "call-streams": "one ro_batch_ready per Call, each on a stream of its own",
+                                   "one-stream": "one ro_batch_ready per Call, on the context's stream"}[args.admissions],
+                    "kernels_per_wave": round(per_replay / W, 2)},
             "assembled_bytes": S,
             "payload_gbs": round(payload_gbs, 1),
             "payload_frac_of_hbm": round(payload_gbs / hbm_peak, 4),
@@ -1458,10 +1470,10 @@ def run_retry_bench(args, local_rank):
     assert stats["retried"] == (args.warmup + args.steps) * lst.numel()
     ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
     k = lst.numel()
-    # algorithmic bytes per retried Grain: list entry 4 read, phase word read
-    # and rewritten (8), record word read for the Call (8) and len claimed and
-    # cleared (12), recovery-queue entry 4 written
-    alg = 36.0 * k
+    # algorithmic bytes per retried Grain: list entry 4 read, its 16-byte slot
+    # read (phase word, claim in len, Call), phase word and len rewritten (8),
+    # recovery-queue entry 4 written
+    alg = 32.0 * k
     print(json.dumps({"retry": {
         "workload": f"document->page: {N} children in flight; one failed attempt of {k} Grains "
                     f"(random order) retried per call",

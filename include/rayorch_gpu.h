@@ -257,6 +257,34 @@ ro_status ro_batch_ready(ro_ctx* ctx, int32_t xid, uint32_t call, const uint32_t
                          uint64_t* h_n_batched, uint64_t* h_n_batches);
 
 /* ------------------------------------------------------------------------
+ * ro_batch_ready_calls — the admissions of n Calls from one candidate list
+ * (Section 4.3: each Call keeps a Ready Queue of its own), in one launch.
+ *
+ * The result equals ro_batch_ready(ctx, xid, calls[k], d_cand, n_cand,
+ * batch_size, flush, d_batched[k], batched_cap[k], d_n_batched[k], NULL,
+ * NULL) for k = 0 .. n-1 in turn (each Call admits only its own children,
+ * into its own queue, so the Calls' admissions are independent).  Runs on
+ * the context's stream, after the Calls' pending admissions on their own
+ * streams: one cooperative kernel over all n Calls when the list's tiles fit
+ * the device at once (n times (n_cand / 2048 + 1) CTAs), else one admission
+ * after another.
+ *
+ *   calls        host uint32[n]: distinct Calls, n in [1, 8].
+ *   d_batched    host array of n device pointers (uint32[batched_cap[k]] out).
+ *   batched_cap  host uint64[n].
+ *   d_n_batched  host array of n device pointers (uint64 out, each may be
+ *                NULL), or NULL.
+ * Errors: RO_E_INVAL (n out of range, a Call named twice or out of range,
+ * NULL arrays) with no side effects; a reservation larger than a Call's
+ * capacity refuses that Call's admission only (RO_E_CAPACITY at the next
+ * synchronising call; that Call's queue and phases unchanged).
+ */
+ro_status ro_batch_ready_calls(ro_ctx* ctx, int32_t xid, uint32_t n, const uint32_t* calls,
+                               const uint32_t* d_cand, uint64_t n_cand, uint32_t batch_size,
+                               int32_t flush, uint32_t* const* d_batched,
+                               const uint64_t* batched_cap, uint64_t* const* d_n_batched);
+
+/* ------------------------------------------------------------------------
  * ro_batch_ready_parent — admission into the per-Call FIFO Ready Queue and
  * parent-bound reservation (Section 4.3, Eq. 2).
  *

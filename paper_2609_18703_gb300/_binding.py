@@ -31,7 +31,7 @@ STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFL
 
 EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro_ctx_stats",
            "ro_ctx_set_streams", "ro_ctx_set_call_streams", "ro_ctx_join", "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
-           "ro_retry", "ro_batch_ready_parent", "ro_gather_commit", "ro_assemble", "ro_assemble_list", "ro_filter_reports",
+           "ro_batch_ready_calls", "ro_retry", "ro_batch_ready_parent", "ro_gather_commit", "ro_assemble", "ro_assemble_list", "ro_filter_reports",
            "ro_expand_noalloc")
 
 # kernel ids (RO_K_*), in launch order of the path
@@ -87,6 +87,8 @@ def load(path: Optional[str] = None):
     L.ro_ctx_profile_read.argtypes = [_vp, _pu64, _pu64, C.POINTER(C.c_double), _u32]
     L.ro_expand.argtypes = [_vp, _i32, _vp, _u64, _vp, _vp, _vp, _vp, _u64, _vp, _pu64, _pu64, _pi32]
     L.ro_batch_ready.argtypes = [_vp, _i32, _u32, _vp, _u64, _u32, _i32, _vp, _u64, _vp, _pu64, _pu64]
+    L.ro_batch_ready_calls.argtypes = [_vp, _i32, _u32, C.POINTER(C.c_uint32), _vp, _u64, _u32, _i32,
+                                       C.POINTER(_vp), _pu64, C.POINTER(_vp)]
     L.ro_retry.argtypes = [_vp, _i32, _u32, _vp, _u64, _pu64]
     L.ro_gather_commit.argtypes = [_vp, _i32, _u64, _vp, _vp, _vp, _vp, _vp, _vp, _u64, _vp, _vp, _u64,
                                    _vp, _pu64]
@@ -222,6 +224,20 @@ def ro_batch_ready(ctx, xid, call, d_cand, n_cand, batch_size, flush, d_batched,
                                C.byref(nb) if want_host else None,
                                C.byref(nbt) if want_host else None)
     return (st, nb.value, nbt.value) if want_host else (st, None, None)
+
+
+def ro_batch_ready_calls(ctx, xid, calls, d_cand, n_cand, batch_size, flush, d_batched, batched_cap,
+                         d_n_batched=None):
+    """Admissions of several Calls from one candidate list (one launch);
+    d_batched, batched_cap and d_n_batched are per-Call sequences.  Returns
+    the status."""
+    n = len(calls)
+    c_calls = (C.c_uint32 * n)(*calls)
+    c_b = (_vp * n)(*[_ptr(d) for d in d_batched])
+    c_cap = (C.c_uint64 * n)(*batched_cap)
+    c_nb = (_vp * n)(*[_ptr(d) for d in d_n_batched]) if d_n_batched is not None else None
+    return load().ro_batch_ready_calls(ctx, xid, n, c_calls, _ptr(d_cand), n_cand, batch_size,
+                                       int(flush), c_b, c_cap, c_nb)
 
 
 def ro_retry(ctx, xid, call, d_children, n, want_host: bool = True):

@@ -68,7 +68,12 @@ __device__ void resolve_barriers(const CommitArgs& a, uint64_t n);
 __device__ void seal_open(const CommitArgs& a, uint32_t pp, int lane, unsigned long long* n_wait,
                           unsigned long long* n_fly);
 
-// Warm L2 with the lines of this warp's first 32 reports while the previous
+#ifndef RO_CM_GROUPS
+#define RO_CM_GROUPS 1
+#endif
+constexpr int CM_GROUPS = RO_CM_GROUPS;   // groups of 32 reports a warp has in flight per step (2 and 4 measured slower)
+
+// Warm L2 with the lines of this warp's first CM_GROUPS groups of 32 reports while the previous
 // kernel drains (addresses inside the report arrays' host-given length; L2 is
 // coherent, so nothing read later can be stale).
 __device__ __forceinline__ void prefetch_l2(const void* p) {
@@ -76,16 +81,18 @@ __device__ __forceinline__ void prefetch_l2(const void* p) {
 }
 __device__ __forceinline__ void prefetch_reports(const CommitArgs& a) {
   const int lane = threadIdx.x & 31;
-  const uint64_t r0 = (((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * 32;
+  if (lane >= 6 * CM_GROUPS) return;
+  const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
+  const uint64_t w = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const uint64_t r0 = (w + (uint64_t)(lane / 6) * n_warps) * 32;   // this lane's group
   if (r0 >= a.n_host) return;
-  switch (lane) {
+  switch (lane % 6) {
     case 0: prefetch_l2(a.child + r0); break;
     case 1: prefetch_l2(a.len + r0); break;
     case 2: prefetch_l2(a.off + r0); break;
     case 3: if (r0 + 16 < a.n_host) prefetch_l2(a.off + r0 + 16); break;
     case 4: prefetch_l2(a.state + r0); break;
-    case 5: if (a.gen) prefetch_l2(a.gen + r0); break;
-    default: break;
+    default: if (a.gen) prefetch_l2(a.gen + r0); break;
   }
 }
 
@@ -125,7 +132,8 @@ __device__ __forceinline__ bool table_add(HeavyTable* t, uint32_t p, unsigned lo
   return false;
 }
 
-__global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a) {
+// at most 56 registers: a CTA (256 threads) fits beside two copy CTAs
+__global__ void __maxnreg__(56) commit_scatter_kernel(CommitArgs a) {
   prefetch_reports(a);
   wait_predecessor();
   allow_successor();
@@ -153,88 +161,113 @@ __global__ void __launch_bounds__(CM_THREADS) commit_scatter_kernel(CommitArgs a
   const uint64_t warp_global = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
   uint32_t cnt[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-  for (uint64_t base = warp_global * 32; base < n; base += n_warps * 32) {
-    const uint64_t r = base + lane;
-    uint8_t v = 255;   // inactive lane
-    uint32_t p = 0;
-    bool bad = false, heavy = false;
-    if (r < n) {
-      const uint64_t c = a.child[r];
-      const uint8_t s = a.state[r];
-      const uint32_t l = a.len[r];
-      const uint64_t o = a.off[r];
-      const uint32_t g = a.gen ? a.gen[r] : 0u;
+  // Each warp takes CM_GROUPS groups of 32 reports per step (group q at
+  // base + q * stride): their loads, parents and fence CASes are all in flight
+  // before the first verdict is used.
+  const uint64_t stride = n_warps * 32;
+  for (uint64_t base = warp_global * 32; base < n; base += CM_GROUPS * stride) {
+    uint64_t c[CM_GROUPS], o[CM_GROUPS];
+    uint32_t l[CM_GROUPS], g[CM_GROUPS], par[CM_GROUPS], cur[CM_GROUPS];
+    uint8_t st[CM_GROUPS], v[CM_GROUPS];
+    bool heavy[CM_GROUPS], won[CM_GROUPS];
+#pragma unroll
+    for (int q = 0; q < CM_GROUPS; ++q) {
+      const uint64_t r = base + q * stride + lane;
+      v[q] = 255;   // inactive lane
+      if (r < n) {
+        c[q] = a.child[r];
+        st[q] = a.state[r];
+        l[q] = a.len[r];
+        o[q] = a.off[r];
+        g[q] = a.gen ? a.gen[r] : 0u;
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < CM_GROUPS; ++q) {
+      const uint64_t r = base + q * stride + lane;
+      heavy[q] = won[q] = false;
+      par[q] = cur[q] = 0u;
+      if (r >= n) continue;
+      const uint8_t s = st[q];
       const bool valid_state = s >= ST_PRESENT && s <= ST_GROUP_FAILURE;
-      const bool in_bounds = s != ST_PRESENT || (o <= a.arena_bytes && (uint64_t)l <= a.arena_bytes - o);
-      if (c >= a.N || !valid_state || !in_bounds) {
-        v = V_INVALID;
+      const bool in_bounds =
+          s != ST_PRESENT || (o[q] <= a.arena_bytes && (uint64_t)l[q] <= a.arena_bytes - o[q]);
+      if (c[q] >= a.N || !valid_state || !in_bounds) {
+        v[q] = V_INVALID;
+        continue;
+      }
+      v[q] = 254;   // decided below
+      // the parent, immutable.  A fill tile of FILL_TILE children that
+      // starts with the same parent as the next one is one heavy parent's
+      // (it has more than HEAVY_CHILDREN children): the small fill-tile
+      // table, resident in L2, names it, and the report touches no sector
+      // but its slot's.  Otherwise it is read alongside the fence.
+      const uint64_t t = c[q] / FILL_TILE;
+      if (a.heavy && t + 1 < a.n_fill_tiles) {
+        const uint32_t f0 = __ldg(a.tfp + t), f1 = __ldg(a.tfp + t + 1);
+        heavy[q] = f0 == f1;
+        par[q] = heavy[q] ? f0 : a.par[c[q]];
       } else {
-        // the parent, immutable.  A fill tile of FILL_TILE children that
-        // starts with the same parent as the next one is one heavy parent's
-        // (it has more than HEAVY_CHILDREN children): the small fill-tile
-        // table, resident in L2, names it, and the report touches no sector
-        // but its slot's.  Otherwise it is read alongside the fence.
-        uint32_t par;
-        const uint64_t t = c / FILL_TILE;
-        if (a.heavy && t + 1 < a.n_fill_tiles) {
-          const uint32_t f0 = __ldg(a.tfp + t), f1 = __ldg(a.tfp + t + 1);
-          heavy = f0 == f1;
-          par = heavy ? f0 : a.par[c];
-        } else {
-          par = a.par[c];
-        }
-        // Eq. (3): accept iff IN-FLIGHT at the report's generation
-        const uint32_t want = ph_make(PH_INFLIGHT, g);
-        uint32_t cur;
-        bool won = false;
-        if (g >> 30) {
-          cur = a.slot[c].phase;   // no Grain ever reaches such a generation
-        } else {
-          cur = atomicCAS(&a.slot[c].phase, want, ph_make(PH_SEALED, g));
-          won = cur == want;
-        }
-        if (won) {
-          v = V_ACCEPT;
+        par[q] = a.par[c[q]];
+      }
+      // Eq. (3): accept iff IN-FLIGHT at the report's generation
+      const uint32_t want = ph_make(PH_INFLIGHT, g[q]);
+      if (g[q] >> 30) {
+        cur[q] = a.slot[c[q]].phase;   // no Grain ever reaches such a generation
+      } else {
+        cur[q] = atomicCAS(&a.slot[c[q]].phase, want, ph_make(PH_SEALED, g[q]));
+        won[q] = cur[q] == want;
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < CM_GROUPS; ++q) {
+      const uint64_t r = base + q * stride + lane;
+      uint32_t p = 0;
+      bool bad = false;
+      if (v[q] == 254) {
+        const uint8_t s = st[q];
+        if (won[q]) {
+          v[q] = V_ACCEPT;
           const bool present = s == ST_PRESENT;
           // a GroupFailure's own Grain failed
           const uint8_t outcome = (s == ST_GROUP_FAILURE) ? ST_FAILED : s;
-          Slot* rc = a.slot + c;
-          rc->len = present ? l : 0u;
+          Slot* rc = a.slot + c[q];
+          rc->len = present ? l[q] : 0u;
           atomicOr((unsigned long long*)&rc->w,
-                   (unsigned long long)((present ? (o & W_OFF_MASK) : 0ull) |
+                   (unsigned long long)((present ? (o[q] & W_OFF_MASK) : 0ull) |
                                         ((uint64_t)outcome << W_STATE_SHIFT)));
-          p = par;
+          p = par[q];
           bad = (s == ST_FAILED || s == ST_SUPPRESSED || s == ST_GROUP_FAILURE);
-          if (s == ST_GROUP_FAILURE) atomicMax(a.gb + par, gb_tag(a.seq, (uint32_t)r));   // barrier
-        } else if ((cur & 3u) == PH_WAITING || (cur & 3u) == PH_READY) {
-          v = V_NOT_INFLIGHT;
-        } else if ((cur >> 2) != g) {
-          v = V_STALE;
-        } else if (ld_w(a.slot + c) & W_BARRIER_BIT) {
-          v = V_BARRIER;   // suppressed by a sibling's GroupFailure in an earlier call
+          if (s == ST_GROUP_FAILURE) atomicMax(a.gb + p, gb_tag(a.seq, (uint32_t)r));   // barrier
+        } else if ((cur[q] & 3u) == PH_WAITING || (cur[q] & 3u) == PH_READY) {
+          v[q] = V_NOT_INFLIGHT;
+        } else if ((cur[q] >> 2) != g[q]) {
+          v[q] = V_STALE;
+        } else if (ld_w(a.slot + c[q]) & W_BARRIER_BIT) {
+          v[q] = V_BARRIER;   // suppressed by a sibling's GroupFailure in an earlier call
         } else {
           // SEALED at this generation: a duplicate, possibly of a report of
           // this same call with a higher index (ordered by commit_fix)
-          v = V_DUP_CANDIDATE;
-          atomicOr((unsigned long long*)&a.slot[c].w, (unsigned long long)W_CONFLICT_BIT);
+          v[q] = V_DUP_CANDIDATE;
+          atomicOr((unsigned long long*)&a.slot[c[q]].w, (unsigned long long)W_CONFLICT_BIT);
         }
       }
-      a.code[r] = v;
-    }
-    // merge the accepted lanes of this warp by parent, one atomic per parent
-    const unsigned acc = __ballot_sync(0xffffffffu, v == V_ACCEPT);
-    const unsigned badm = __ballot_sync(0xffffffffu, v == V_ACCEPT && bad);
-    if (v == V_ACCEPT) {
-      const unsigned grp = __match_any_sync(acc, p);
-      if (lane == __ffs(grp) - 1) {
-        const unsigned n_tot = __popc(grp), n_bad = __popc(grp & badm);
-        if (!(heavy && table_add(ht, p, ((unsigned long long)n_bad << 32) | n_tot)))
-          count_down(a, p, n_tot, n_bad);
+      if (r < n) a.code[r] = v[q];
+      // merge the accepted lanes of this warp by parent, one atomic per parent
+      const unsigned acc = __ballot_sync(0xffffffffu, v[q] == V_ACCEPT);
+      const unsigned badm = __ballot_sync(0xffffffffu, v[q] == V_ACCEPT && bad);
+      if (v[q] == V_ACCEPT) {
+        const unsigned grp = __match_any_sync(acc, p);
+        if (lane == __ffs(grp) - 1) {
+          const unsigned n_tot = __popc(grp), n_bad = __popc(grp & badm);
+          if (!(heavy[q] && table_add(ht, p, ((unsigned long long)n_bad << 32) | n_tot)))
+            count_down(a, p, n_tot, n_bad);
+        }
       }
+      if (v[q] <= V_DUP_CANDIDATE) cnt[v[q]] += 1;
+      // any GroupFailure report (it may still win an ordering of duplicates)
+      if (r < n && v[q] != V_INVALID && st[q] == ST_GROUP_FAILURE) cnt[7] += 1;
     }
-    if (v <= V_DUP_CANDIDATE) cnt[v] += 1;
-    // any GroupFailure report (it may still win an ordering of duplicates)
-    if (r < n && v != V_INVALID && a.state[r] == ST_GROUP_FAILURE) cnt[7] += 1;
   }
   // statistics: accepted, invalid, not in flight, stale, barrier (duplicates
   // are counted by the finish pass), candidates for ordering, GroupFailures

@@ -121,6 +121,68 @@ __device__ __forceinline__ uint32_t claim_group(const ReadyArgs& a, uint64_t bas
   return firsts;
 }
 
+// The same claims for the one-pass admission: *won = the candidates whose
+// claim this thread took (they stand unless a child is named twice).
+// Returns whether any claim met another one (a repeat somewhere in the list).
+__device__ __forceinline__ bool claim_group_won(const ReadyArgs& a, uint64_t base, const CandGroup& g,
+                                                uint32_t elig, uint32_t* won) {
+  uint32_t old[RB_ITEMS], w = 0u;
+  bool conflict = false;
+#pragma unroll
+  for (int k = 0; k < RB_ITEMS; ++k) {
+    old[k] = g.ph[k];
+    if (!((elig >> k) & 1u)) continue;
+    const uint32_t i = (uint32_t)cand_pos(base, k);
+    if ((g.ph[k] >> 2) != CLAIM_NONE) conflict = true;   // claimed before this attempt
+    if ((g.ph[k] >> 2) > i) old[k] = atomicCAS(&a.slot[g.c[k]].phase, g.ph[k], i << 2);
+  }
+#pragma unroll
+  for (int k = 0; k < RB_ITEMS; ++k) {
+    if (!((elig >> k) & 1u)) continue;
+    const uint32_t i = (uint32_t)cand_pos(base, k), mine = i << 2;
+    if ((g.ph[k] >> 2) <= i) continue;   // a lower position holds it
+    uint32_t cur = g.ph[k], o = old[k];
+    bool ok = o == cur;
+    while (!ok) {   // another claim got there first
+      conflict = true;
+      cur = o;
+      if ((cur & 3u) != PH_WAITING || (cur >> 2) <= i) break;
+      o = atomicCAS(&a.slot[g.c[k]].phase, cur, mine);
+      ok = o == cur;
+    }
+    if (ok) w |= 1u << k;
+  }
+  *won = w;
+  return conflict;
+}
+
+// A tile's admitted and bad counts, summed over the CTA, into the per-tile
+// arrays (the look-back buffers' value arrays) for the other CTAs.
+__device__ __forceinline__ void publish_counts(const ReadyArgs& a, uint32_t tile, uint32_t flags, const CandGroup& g,
+                                               unsigned long long (*s_red)[RB_THREADS / 32]) {
+  unsigned long long kept = __popc(flags), bad = __popc(g.in_range & ~g.valid);
+  for (int d = 16; d > 0; d >>= 1) {
+    kept += __shfl_down_sync(0xffffffffu, kept, d);
+    bad += __shfl_down_sync(0xffffffffu, bad, d);
+  }
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  if (lane == 0) {
+    s_red[0][wid] = kept;
+    s_red[1][wid] = bad;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long k = 0, b = 0;
+    for (int j = 0; j < RB_THREADS / 32; ++j) {
+      k += s_red[0][j];
+      b += s_red[1][j];
+    }
+    a.ts.agg[tile] = k;
+    a.ts.inc[tile] = b;
+  }
+  __syncthreads();
+}
+
 // Eligible candidates of a group: naming a WAITING child of this Call.
 __device__ __forceinline__ uint32_t eligible(const ReadyArgs& a, const CandGroup& g) {
   uint32_t elig = 0u;
@@ -427,73 +489,69 @@ __device__ void grid_barrier(ReadyScalars* rs, uint32_t* err) {
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(RB_THREADS) ready_fused_kernel(ReadyArgs a) {
+// The one-pass admission of Call a by CTA b of the Call's T + 1 (T tiles,
+// then the window).  gs holds the grid's barrier, launch sequence and
+// conflict tag (one set per launch, the first Call's); seq_owner advances the
+// sequence when done.  Every CTA of the grid meets at the same barriers.
+__device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint32_t b, ReadyScalars* gs,
+                                            bool seq_owner) {
   __shared__ unsigned long long s_scan[33];
   __shared__ uint32_t s_rows[RB_ITEMS * (RB_THREADS / 32) + 1];
   __shared__ unsigned long long s_red[2][RB_THREADS / 32];
   __shared__ unsigned long long s_tot[3];   // prefix of this tile, admitted, bad
   DevScalars* ds = a.ds;
   ReadyScalars* rs = a.rs;
-  const uint32_t T = gridDim.x - 1u;   // candidate tiles
-  const bool window = blockIdx.x == T;
-  const uint64_t base = (uint64_t)blockIdx.x * RB_THREADS * RB_ITEMS;
-  // per-tile counts (admitted, bad) go through the look-back buffers' value arrays
+  const bool window = b == T;
+  const uint64_t base = (uint64_t)b * RB_THREADS * RB_ITEMS;
+  // per-tile counts (admitted, bad), in the look-back buffers' value arrays
   unsigned long long* cnt_kept = a.ts.agg;
   unsigned long long* cnt_bad = a.ts.inc;
   CandGroup g;
   uint32_t flags = 0u, elig = 0u;
   unsigned long long head = 0, tail = 0, tail0 = 0;
 
-  // A: candidates, slots and claims; the window is compacted meanwhile
+  // this launch's tag for the conflict word (the sequence owner advances the
+  // sequence when done; every CTA reads it first)
+  const uint32_t tag = ld_acquire(&gs->adm_seq) + 1u;
+
+  // A: candidates, slots and claims; the window is compacted meanwhile.  A
+  // claim that met another one (a child named twice) marks the call; without
+  // any, every claim taken stands and the tile counts below are final.
   if (!window) {
     load_group(a, base, g);
     elig = eligible(a, g);
-    if (a.cand)
-      claim_group(a, base, g, elig);
-    else
+    if (a.cand) {
+      if (claim_group_won(a, base, g, elig, &flags) && ld_acquire(&gs->adm_conflict) != tag)
+        atomicExch(&gs->adm_conflict, tag);
+    } else {
       flags = elig;   // ids are distinct
+    }
+    publish_counts(a, b, flags, g, s_red);
   } else {
     compact_window(a, s_scan, &head, &tail, &tail0);
+    if (threadIdx.x == 0) {
+      rs->rb_head = head;   // the window, for the other CTAs
+      rs->rb_L = tail - head;
+    }
   }
-  if (a.cand) grid_barrier(rs, &ds->err);
+  grid_barrier(gs, &ds->err);
 
-  // B: with every claim settled, a candidate is admitted iff its child holds
-  // its claim; tile counts
-  if (!window) {
-    if (a.cand) {
+  // B (repeats only): with every claim settled, a candidate is admitted iff
+  // its child holds its claim; the tile counts again
+  if (a.cand && __ldcg(&gs->adm_conflict) == tag) {
+    if (!window) {
       uint32_t ph[RB_ITEMS];
 #pragma unroll
       for (int k = 0; k < RB_ITEMS; ++k)
         ph[k] = ((elig >> k) & 1u) ? __ldcg(&a.slot[g.c[k]].phase) : 0u;
+      flags = 0u;
 #pragma unroll
       for (int k = 0; k < RB_ITEMS; ++k)
         if (((elig >> k) & 1u) && ph[k] == ((uint32_t)cand_pos(base, k) << 2)) flags |= 1u << k;
+      publish_counts(a, b, flags, g, s_red);
     }
-    unsigned long long kept = __popc(flags), bad = __popc(g.in_range & ~g.valid);
-    for (int d = 16; d > 0; d >>= 1) {
-      kept += __shfl_down_sync(0xffffffffu, kept, d);
-      bad += __shfl_down_sync(0xffffffffu, bad, d);
-    }
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    if (lane == 0) {
-      s_red[0][wid] = kept;
-      s_red[1][wid] = bad;
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      unsigned long long k = 0, b = 0;
-      for (int j = 0; j < RB_THREADS / 32; ++j) {
-        k += s_red[0][j];
-        b += s_red[1][j];
-      }
-      cnt_kept[blockIdx.x] = k;
-      cnt_bad[blockIdx.x] = b;
-    }
-  } else if (threadIdx.x == 0) {
-    rs->rb_head = head;   // the window, for the other CTAs
-    rs->rb_L = tail - head;
+    grid_barrier(gs, &ds->err);
   }
-  grid_barrier(rs, &ds->err);
 
   // C: prefix of this tile, number admitted and bad (one warp)
   if (threadIdx.x < 32) {
@@ -501,7 +559,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_fused_kernel(ReadyArgs a) {
     for (uint32_t t = threadIdx.x; t < T; t += 32) {
       const unsigned long long k = __ldcg(cnt_kept + t);
       K += k;
-      if (t < blockIdx.x) pre += k;
+      if (t < b) pre += k;
       bad += __ldcg(cnt_bad + t);
     }
     for (int d = 16; d > 0; d >>= 1) {
@@ -529,6 +587,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_fused_kernel(ReadyArgs a) {
         if (a.cand && ((flags >> k) & 1u)) a.slot[g.c[k]].phase = WAIT_UNCLAIMED;
     } else if (threadIdx.x == 0) {
       plan_reservation(a, head, tail, tail0, K, s_tot[2]);   // records the refusal
+      if (seq_owner) st_release(&gs->adm_seq, tag);
     }
     return;
   }
@@ -558,6 +617,19 @@ __global__ void __launch_bounds__(RB_THREADS) ready_fused_kernel(ReadyArgs a) {
     }
     if (threadIdx.x == 0) plan_reservation(a, head, tail, tail0, K, s_tot[2]);
   }
+  if (seq_owner && threadIdx.x == 0) st_release(&gs->adm_seq, tag);   // every CTA has read it
+}
+
+__global__ void __launch_bounds__(RB_THREADS) ready_fused_kernel(ReadyArgs a) {
+  fused_admit(a, gridDim.x - 1u, blockIdx.x, a.rs, blockIdx.x == gridDim.x - 1u);
+}
+
+// Several Calls' admissions from one candidate list: the grid holds each
+// Call's T tiles and its window CTA in turn.
+__global__ void __launch_bounds__(RB_THREADS) ready_fused_calls_kernel(MultiReadyArgs m) {
+  const uint32_t per = gridDim.x / m.n;   // CTAs per Call
+  const uint32_t k = blockIdx.x / per, b = blockIdx.x % per;
+  fused_admit(m.a[k], per - 1u, b, m.a[0].rs, k == 0 && b == per - 1u);
 }
 
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a) {
@@ -579,7 +651,13 @@ void launch_ready(const LaunchCfg& L, const ReadyArgs& a) {
   launch_k(L, K_RB_SCATTER, ready_scatter_kernel, grid_scatter, RB_THREADS, 0, a);
 }
 
+void launch_ready_calls(const LaunchCfg& L, const MultiReadyArgs& m) {
+  const uint64_t per = ceil_div(m.a[0].n_cand, (uint64_t)RB_THREADS * RB_ITEMS) + 1;
+  launch_coop(L, K_RB_FUSED, ready_fused_calls_kernel, (int)(per * m.n), RB_THREADS, m);
+}
+
 const void* kernel_ptr_ready(int which) {
+  if (which == K_RB_FUSED_CALLS) return (const void*)ready_fused_calls_kernel;
   if (which == K_RB_FUSED) return (const void*)ready_fused_kernel;
   return which == K_RB_COUNT ? (const void*)ready_count_kernel : (const void*)ready_scatter_kernel;
 }

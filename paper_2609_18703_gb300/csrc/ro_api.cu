@@ -567,10 +567,11 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
     int coop = 0;
     cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, device);
     c->L.grid_rb_coop = coop ? grid_for(kernel_ptr_ready(K_RB_FUSED), RB_THREADS, s, 64) : 0;
+    c->L.grid_rb_coop_calls = coop ? grid_for(kernel_ptr_ready(K_RB_FUSED_CALLS), RB_THREADS, s, 64) : 0;
     // RO_ADMIT_TWO_PASS=1 in the environment at context creation keeps every
     // admission on the two-pass path
     if (const char* e = std::getenv("RO_ADMIT_TWO_PASS"))
-      if (std::strtoul(e, nullptr, 10) != 0) c->L.grid_rb_coop = 0;
+      if (std::strtoul(e, nullptr, 10) != 0) c->L.grid_rb_coop = c->L.grid_rb_coop_calls = 0;
   }
   c->L.grid_commit = grid_for(kernel_ptr_commit(K_COMMIT), CM_THREADS, s, 8);
   c->L.grid_cplan = grid_for(kernel_ptr_complete(), CP_THREADS, s, 4);
@@ -859,19 +860,11 @@ ro_status ro_expand(ro_ctx* c, int32_t parent_xid, const uint32_t* d_counts, uin
 }
 
 // ---------------------------------------------------------------------------
-ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* d_cand,
-                         uint64_t n_cand, uint32_t batch_size, int32_t flush, uint32_t* d_batched,
-                         uint64_t batched_cap, uint64_t* d_n_batched, uint64_t* h_n_batched,
-                         uint64_t* h_n_batches) {
-  RO_TRY(enter(c));
+// The admission arguments of one Call (queue, scan slot, outputs).
+ro_status ready_args(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* d_cand, uint64_t n_cand,
+                     uint32_t batch_size, int32_t flush, uint32_t* d_batched, uint64_t batched_cap,
+                     uint64_t* d_n_batched, ReadyArgs* out) {
   Expansion* x = get_exp(c, xid);
-  if (!x) return fail(c, RO_E_STATE, "ro_batch_ready: unknown expansion %d", xid);
-  if (call >= c->n_calls) return fail(c, RO_E_INVAL, "ro_batch_ready: call %u out of range", call);
-  if (batch_size == 0) return fail(c, RO_E_INVAL, "ro_batch_ready: batch_size is 0");
-  if (batched_cap && !d_batched) return fail(c, RO_E_INVAL, "ro_batch_ready: NULL d_batched");
-  if (d_cand && n_cand > MAX_CAND)
-    return fail(c, RO_E_INVAL, "ro_batch_ready: more than 2^30-2 candidates in one call");
-  DeviceGuard g(c->device);
   ExpSlot& S = c->slots[xid];
   QueueBufs& Q = S.queues[call];
   RO_TRY(queue_ready(c, Q, x->N));
@@ -892,10 +885,30 @@ ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* 
   ra.n_batched_out = d_n_batched;
   ra.ds = c->ds;
   ra.rs = c->rs + call;
-  for (cudaStream_t s : c->call_stream) ra.calls_concurrent |= (s != c->stream);
-  ra.calls_concurrent &= ra.check_call;
   RO_TRY(tile_status_buf(c, c->ts_call[call], ceil_div(ra.n_cand, (uint64_t)RB_THREADS * RB_ITEMS),
                          &ra.ts));
+  *out = ra;
+  return RO_OK;
+}
+
+ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* d_cand,
+                         uint64_t n_cand, uint32_t batch_size, int32_t flush, uint32_t* d_batched,
+                         uint64_t batched_cap, uint64_t* d_n_batched, uint64_t* h_n_batched,
+                         uint64_t* h_n_batches) {
+  RO_TRY(enter(c));
+  Expansion* x = get_exp(c, xid);
+  if (!x) return fail(c, RO_E_STATE, "ro_batch_ready: unknown expansion %d", xid);
+  if (call >= c->n_calls) return fail(c, RO_E_INVAL, "ro_batch_ready: call %u out of range", call);
+  if (batch_size == 0) return fail(c, RO_E_INVAL, "ro_batch_ready: batch_size is 0");
+  if (batched_cap && !d_batched) return fail(c, RO_E_INVAL, "ro_batch_ready: NULL d_batched");
+  if (d_cand && n_cand > MAX_CAND)
+    return fail(c, RO_E_INVAL, "ro_batch_ready: more than 2^30-2 candidates in one call");
+  DeviceGuard g(c->device);
+  ReadyArgs ra{};
+  RO_TRY(ready_args(c, xid, call, d_cand, n_cand, batch_size, flush, d_batched, batched_cap,
+                    d_n_batched, &ra));
+  for (cudaStream_t s : c->call_stream) ra.calls_concurrent |= (s != c->stream);
+  ra.calls_concurrent &= ra.check_call;
   // on the Call's stream when it has one, after everything issued on the
   // context's stream so far; the context's stream waits for it before its
   // next launch
@@ -919,6 +932,42 @@ ro_status ro_batch_ready(ro_ctx* c, int32_t xid, uint32_t call, const uint32_t* 
     return st;
   }
   return RO_OK;
+}
+
+// ---------------------------------------------------------------------------
+ro_status ro_batch_ready_calls(ro_ctx* c, int32_t xid, uint32_t n, const uint32_t* calls,
+                               const uint32_t* d_cand, uint64_t n_cand, uint32_t batch_size,
+                               int32_t flush, uint32_t* const* d_batched,
+                               const uint64_t* batched_cap, uint64_t* const* d_n_batched) {
+  RO_TRY(enter(c));
+  const char* fn = "ro_batch_ready_calls";
+  Expansion* x = get_exp(c, xid);
+  if (!x) return fail(c, RO_E_STATE, "%s: unknown expansion %d", fn, xid);
+  if (n == 0 || n > RB_CALLS_MAX) return fail(c, RO_E_INVAL, "%s: %u Calls (1 to %u)", fn, n, RB_CALLS_MAX);
+  if (!calls || !d_batched || !batched_cap) return fail(c, RO_E_INVAL, "%s: NULL argument", fn);
+  if (batch_size == 0) return fail(c, RO_E_INVAL, "%s: batch_size is 0", fn);
+  if (d_cand && n_cand > MAX_CAND)
+    return fail(c, RO_E_INVAL, "%s: more than 2^30-2 candidates in one call", fn);
+  for (uint32_t k = 0; k < n; ++k) {
+    if (calls[k] >= c->n_calls) return fail(c, RO_E_INVAL, "%s: call %u out of range", fn, calls[k]);
+    if (batched_cap[k] && !d_batched[k]) return fail(c, RO_E_INVAL, "%s: NULL d_batched", fn);
+    for (uint32_t j = 0; j < k; ++j)
+      if (calls[j] == calls[k]) return fail(c, RO_E_INVAL, "%s: call %u named twice", fn, calls[k]);
+  }
+  DeviceGuard g(c->device);
+  RO_TRY(settle_calls(c));   // after the Calls' pending admissions on their streams
+  MultiReadyArgs m{};
+  m.n = n;
+  for (uint32_t k = 0; k < n; ++k)
+    RO_TRY(ready_args(c, xid, calls[k], d_cand, n_cand, batch_size, flush, d_batched[k], batched_cap[k],
+                      d_n_batched ? d_n_batched[k] : nullptr, &m.a[k]));
+  const uint64_t per = ceil_div(m.a[0].n_cand, (uint64_t)RB_THREADS * RB_ITEMS) + 1;
+  if (per * n <= (uint64_t)c->L.grid_rb_coop_calls) {
+    launch_ready_calls(c->L, m);
+  } else {   // too long a list for one grid: one admission after another
+    for (uint32_t k = 0; k < n; ++k) launch_ready(c->L, m.a[k]);
+  }
+  return check_launch(c, "batch_ready_calls");
 }
 
 // ---------------------------------------------------------------------------

@@ -147,8 +147,9 @@ struct alignas(128) ReadyScalars {
   unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
   unsigned long long epoch;
   uint32_t rb_ticket, rb_err, tile_ctr, exit_ctr;
-  // grid barrier of the one-pass admission: arrivals, generation
-  uint32_t bar_count, bar_gen;
+  // one-pass admission: grid barrier (arrivals, generation), launch
+  // sequence and the tag of the latest launch that met a repeated child
+  uint32_t bar_count, bar_gen, adm_seq, adm_conflict;
 };
 // TS_COMMIT and TS_COMMIT_ODD: the completion lists and plans of commits of
 // even and odd sequence (they may run at the same time, on two streams);
@@ -270,13 +271,18 @@ __device__ __forceinline__ Pair64 warp_sum(Pair64 v) {
 }
 
 // Exclusive prefix of tile `tile` given its local aggregate (decoupled
-// look-back), computed by one whole warp: each step inspects the 32 nearest
-// predecessors not yet summed at once (lane l the l-th nearest), adds the
-// aggregates up to the nearest inclusive prefix and stops there, else moves
-// 32 tiles back.  Tiles are claimed in increasing order by running CTAs, so
+// look-back), computed by one whole warp: each step inspects the
+// 32 * LB_PER_LANE nearest predecessors not yet summed at once (lane l the
+// LB_PER_LANE after lane l - 1's), waits until every one up to the nearest
+// inclusive prefix is published, adds the aggregates up to that prefix and
+// stops there, else moves 32 * LB_PER_LANE tiles back.  Tiles are claimed in increasing order by running CTAs, so
 // every predecessor is resident or done and each wait ends; the waits are
 // bounded anyway (SPIN_LIMIT) and record ERR_TIMEOUT.  Every lane returns
 // the prefix.
+#ifndef RO_LB_PER_LANE
+#define RO_LB_PER_LANE 1
+#endif
+constexpr int LB_PER_LANE = RO_LB_PER_LANE;   // predecessors each lane inspects per step (4 measured slower: its polls cost more than the shorter walks save)
 template <class T>
 __device__ T lookback_exclusive(const TileStatus<T>& ts, uint32_t tile, const T& local,
                                 unsigned long long epoch, uint32_t* err) {
@@ -290,18 +296,38 @@ __device__ T lookback_exclusive(const TileStatus<T>& ts, uint32_t tile, const T&
   T excl{};
   int64_t j = (int64_t)tile - 1;   // nearest predecessor not summed yet
   for (;;) {
-    const int64_t mine = j - lane;
-    unsigned long long f = 0;
+    // lane l inspects predecessors j - LB_PER_LANE * l - q, nearest first;
+    // those past tile 0 count as an inclusive prefix of zero
+    const int64_t m0 = j - (int64_t)lane * LB_PER_LANE;
+    unsigned long long f[LB_PER_LANE];
     uint32_t spins = 0;
     bool gave_up = false;
+    int stop = 32, qi = LB_PER_LANE;
     for (;;) {
-      const bool ready = mine < 0 || (((f = ld_acquire_u64(ts.flag + mine)) >> 2) == epoch && (f & 3ull) != 0ull);
-      if (__all_sync(0xffffffffu, ready)) break;
+      // per lane, nearest first: the first predecessor not published yet
+      // (nr) and the first inclusive prefix (qi)
+      int nr = LB_PER_LANE;
+      qi = LB_PER_LANE;
+#pragma unroll
+      for (int q = LB_PER_LANE - 1; q >= 0; --q) {
+        f[q] = 2ull;
+        if (m0 - q >= 0) f[q] = ld_acquire_u64(ts.flag + (m0 - q));
+        const bool ready = m0 - q < 0 || ((f[q] >> 2) == epoch && (f[q] & 3ull) != 0ull);
+        if (!ready) nr = q;
+        else if ((f[q] & 3ull) == 2ull) qi = q;
+      }
+      if (qi > nr) qi = LB_PER_LANE;   // an inclusive prefix behind an unpublished tile
+      // go on once every predecessor up to the nearest inclusive prefix is in
+      const unsigned bm = __ballot_sync(0xffffffffu, nr < LB_PER_LANE && qi == LB_PER_LANE);
+      const unsigned sm = __ballot_sync(0xffffffffu, qi < LB_PER_LANE);
+      stop = sm ? __ffs(sm) - 1 : 32;
+      const int blocked = bm ? __ffs(bm) - 1 : 32;
+      if (stop < blocked || blocked == 32) break;
       ++spins;
-      bool stop = spins > SPIN_LIMIT;
+      bool give = spins > SPIN_LIMIT;
       // once any wait of this context has given up, stop waiting at once
-      if ((spins & 1023u) == 0u && lane == 0 && (ld_acquire(err) & ERR_TIMEOUT)) stop = true;
-      if (__any_sync(0xffffffffu, stop)) {
+      if ((spins & 1023u) == 0u && lane == 0 && (ld_acquire(err) & ERR_TIMEOUT)) give = true;
+      if (__any_sync(0xffffffffu, give)) {
         gave_up = true;
         break;
       }
@@ -311,18 +337,21 @@ __device__ T lookback_exclusive(const TileStatus<T>& ts, uint32_t tile, const T&
       if (lane == 0) atomicOr(err, ERR_TIMEOUT);
       break;
     }
-    // lanes past tile 0 count as an inclusive prefix of zero
-    const bool inclusive = mine < 0 || (f & 3ull) == 2ull;
-    const unsigned im = __ballot_sync(0xffffffffu, inclusive);
-    const int stop = im ? __ffs(im) - 1 : 32;
     T v{};
-    if (mine >= 0) {
-      if (lane < stop) v = load_cg(ts.agg + mine);
-      else if (lane == stop) v = load_cg(ts.inc + mine);
+    if (lane <= stop) {
+      const int na = lane < stop ? LB_PER_LANE : qi;   // aggregates before it
+#pragma unroll
+      for (int q = 0; q < LB_PER_LANE; ++q) {
+        if (m0 - q < 0) continue;
+        if (q < na)
+          v = v + load_cg(ts.agg + (m0 - q));
+        else if (q == na && lane == stop)
+          v = v + load_cg(ts.inc + (m0 - q));
+      }
     }
     excl = excl + warp_sum(v);
     if (stop < 32) break;
-    j -= 32;
+    j -= 32 * LB_PER_LANE;
   }
   if (lane == 0) ts_publish(ts, tile, excl + local, 2ull, epoch);
   __syncwarp();

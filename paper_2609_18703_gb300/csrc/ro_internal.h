@@ -56,7 +56,8 @@ constexpr uint64_t AC_SMALL_CHUNKS = 256;
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CPLAN, K_APARENTS,
                 K_AMEMBERS, K_ACOPY, K_RT_CLAIM, K_RT_SCATTER, K_PB_KEYS, K_PB_HIST,
                 K_PB_ROWSCAN, K_PB_SORT, K_PB_BOUNDS, K_PB_HEADS, K_PB_MARK, K_PB_SCAN, K_PB_EMIT,
-                K_CFIX, K_RB_FUSED, K_COUNT };
+                K_CFIX, K_RB_FUSED, K_COUNT,
+                K_RB_FUSED_CALLS = 100 };   // occupancy query only (profiled as K_RB_FUSED)
 
 
 // Launch counter and optional CUDA-event timing of selected kernels, on the
@@ -70,8 +71,9 @@ struct LaunchCfg {
   Profiler* prof;
   int grid_expand_scan, grid_fill, grid_rb, grid_commit, grid_cplan, grid_aparents,
       grid_amembers, grid_acopy, grid_retry, grid_pb, grid_pb_sort;
-  // CTAs of the one-pass admission the device holds at once (0: no cooperative launch)
-  int grid_rb_coop;
+  // CTAs of the one-pass admission (one Call; several) the device holds at
+  // once (0: no cooperative launch)
+  int grid_rb_coop, grid_rb_coop_calls;
 };
 
 // Launch one kernel between the profiler's marks, with programmatic
@@ -165,6 +167,14 @@ struct ReadyArgs {
   TileStatus<unsigned long long> ts;   // this Call's
 };
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a);
+// the admissions of up to RB_CALLS_MAX Calls from one candidate list, one
+// cooperative launch (the caller checks that the grid fits: LaunchCfg::grid_rb_coop_calls)
+constexpr uint32_t RB_CALLS_MAX = 8;
+struct MultiReadyArgs {
+  ReadyArgs a[RB_CALLS_MAX];
+  uint32_t n;
+};
+void launch_ready_calls(const LaunchCfg& L, const MultiReadyArgs& m);
 // ---- ro_batch_ready_parent ---------------------------------------------------------
 constexpr int PB_THREADS = 256, PB_ITEMS = 8;                 // queue entries per tile: 2048
 constexpr uint32_t PB_TILE = PB_THREADS * PB_ITEMS;

@@ -116,6 +116,35 @@ class Lockstep:
             assert np.array_equal(got, r["batched"])
         return dict(status=st, batched=r["batched"], n_batched=nb)
 
+    def batch_ready_calls(self, xid: int, calls, cand, batch_size: int = 1, flush: bool = False,
+                          caps=None) -> list:
+        """ro_batch_ready_calls (several Calls, one launch) against the
+        oracle's admissions of the same Calls in turn.  Returns each Call's
+        reserved children (None where its reservation was refused)."""
+        cand = np.asarray(cand, dtype=np.uint32)
+        if caps is None:
+            caps = [self.N[xid] + batch_size] * len(calls)
+        d_cand = dev(cand, np.uint32)
+        d_b = [empty(max(int(c), 1), np.uint32) for c in caps]
+        d_nb = [empty(1, np.uint64) for _ in calls]
+        st = ro.ro_batch_ready_calls(self.ctx, xid, list(calls), d_cand, cand.size, batch_size, flush,
+                                     d_b, [int(c) for c in caps], d_nb)
+        assert st == ro.RO_OK, ro.ro_last_error(self.ctx)
+        sync = ro.ro_ctx_sync(self.ctx)
+        out, refused = [], False
+        for k, c in enumerate(calls):
+            r = self.o.batch_ready(xid, c, cand, batch_size, flush, cap=int(caps[k]), check=False)
+            if r["status"] == ro.RO_E_CAPACITY:
+                refused = True
+                out.append(None)
+                continue
+            nb = int(host(d_nb[k], np.uint64, 1)[0])
+            assert nb == r["n_batched"], (c, nb, r["n_batched"])
+            assert np.array_equal(host(d_b[k], np.uint32, nb), r["batched"])
+            out.append(r["batched"])
+        assert sync == (ro.RO_E_CAPACITY if refused else ro.RO_OK), ro.ro_last_error(self.ctx)
+        return out
+
     def batch_ready_parent(self, xid: int, call: int = 0, cand=None, batch_size: int = 1,
                            flush: bool = False, cap: Optional[int] = None,
                            off_cap: Optional[int] = None) -> dict:

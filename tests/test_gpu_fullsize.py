@@ -229,12 +229,15 @@ def test_video_nested_full_size():
         ls.check_stats()
 
 
-@pytest.mark.parametrize("B", [32, 256, 2048])
-def test_streaming_full_size(B):
+@pytest.mark.parametrize("B,admissions", [(32, "calls"), (256, "calls"), (2048, "calls"),
+                                          (256, "call-streams")])
+def test_streaming_full_size(B, admissions):
     """The streaming configuration at full size, at each batch size the
     benchmark sweeps, with the bench's default streams (assembly planning and
-    copies on streams of their own, each Call's admissions on a stream of its
-    own): four Calls, 50,000,050 children of 1 KB, 1,000 readiness waves; per
+    copies on streams of their own) and its default admission (every Call's
+    in one ro_batch_ready_calls per wave), and at B = 256 also with each
+    Call's admissions on a stream of its own: four Calls, 50,000,050
+    children of 1 KB, 1,000 readiness waves; per
     wave every Call admits the wave's ready children and reserves whole
     batches (the last wave flushes), the reserved children's results are
     committed in their key order and the completed parents assembled.  Every
@@ -251,13 +254,16 @@ def test_streaming_full_size(B):
     a = host_arena(lv)
     ad = _arena_dev(a)
     total = 0
-    with Lockstep(n_calls=4, streams=True, call_streams=True) as ls:
+    with Lockstep(n_calls=4, streams=True, call_streams=admissions == "call-streams") as ls:
         x = ls.expand(lv.counts, parent_call=lv.parent_call)["xid"]
         n_ready = lv.ready_bounds.size - 1
         for w in range(n_ready):
             cand = lv.readiness[lv.ready_bounds[w]:lv.ready_bounds[w + 1]]
             last = w == n_ready - 1
-            reserved = [ls.batch_ready(x, c, cand, B, flush=last)["batched"] for c in range(4)]
+            if admissions == "calls":
+                reserved = ls.batch_ready_calls(x, [0, 1, 2, 3], cand, B, flush=last)
+            else:
+                reserved = [ls.batch_ready(x, c, cand, B, flush=last)["batched"] for c in range(4)]
             got = np.concatenate(reserved)
             got = got[np.argsort(lv.key[got], kind="stable")]
             ch, st, ln, of = lv.reports(got)
