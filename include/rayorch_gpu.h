@@ -175,6 +175,19 @@ ro_status ro_ctx_set_call_streams(ro_ctx* ctx, void* const* streams, uint32_t n)
  * before ending one (a captured assembly forks onto the other streams, and a
  * capture must join them back).  Nothing waits on the host. */
 ro_status ro_ctx_join(ro_ctx* ctx);
+/* Self-test of the bounded device-side waits.  Every wait of the lineage
+ * kernels gives up after a bounded number of polls (about two seconds),
+ * records the time-out in the context and returns, so that a wait that can
+ * never end (a lost dependency) turns into RO_E_TIMEOUT instead of a hung
+ * GPU.  This call runs one such wait that nothing releases, on scratch state
+ * of its own: kind 0 a decoupled look-back whose predecessor tile never
+ * publishes, kind 1 a grid barrier of two CTAs one of which never arrives.
+ * It synchronises and returns RO_E_TIMEOUT when the wait gave up and was
+ * reported (the expected outcome), RO_OK if it was not (a defect).  Lineage
+ * state is untouched; the context stays usable.
+ * Errors: RO_E_INVAL for another kind; an earlier call's pending device
+ * error is returned first. */
+ro_status ro_ctx_selftest_timeout(ro_ctx* ctx, uint32_t kind);
 /* Synchronise and copy the cumulative counters. */
 ro_status ro_ctx_stats(ro_ctx* ctx, ro_stats* out);
 /* Text of the last error on this context ("" if none).  Valid until the next call. */

@@ -8,7 +8,7 @@ from ._binding import (EXPORTS, KERNELS, ro_ctx_profile, ro_ctx_profile_read, RO
                        RO_E_OOM, RO_E_OVERFLOW, RO_E_STATE, RO_E_TIMEOUT, RO_FAILED, RO_GROUP_FAILURE, RO_OK,
                        RO_PENDING, RO_PRESENT, RO_REJ_BARRIER, RO_REJ_DUPLICATE, RO_REJ_INVALID,
                        RO_REJ_NOT_INFLIGHT, RO_REJ_STALE_GEN, RO_SUPPRESSED, RoError, load,
-                       ro_assemble, ro_assemble_list, ro_batch_ready, ro_batch_ready_calls, ro_batch_ready_parent, ro_filter_reports, ro_ctx_create, ro_ctx_destroy, ro_ctx_reset,
+                       ro_assemble, ro_assemble_list, ro_batch_ready, ro_batch_ready_calls, ro_batch_ready_parent, ro_ctx_selftest_timeout, ro_filter_reports, ro_ctx_create, ro_ctx_destroy, ro_ctx_reset,
                        ro_ctx_set_streams, ro_ctx_set_call_streams, ro_ctx_join, ro_ctx_stats, ro_ctx_sync, ro_expand, ro_expand_noalloc, ro_gather_commit, ro_retry,
                        ro_last_error)
 

@@ -30,7 +30,7 @@ STATUS_NAMES = {0: "RO_OK", 1: "RO_E_INVAL", 2: "RO_E_CAPACITY", 3: "RO_E_OVERFL
                 4: "RO_E_STATE", 5: "RO_E_OOM", 6: "RO_E_CUDA", 7: "RO_E_TIMEOUT"}
 
 EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro_ctx_stats",
-           "ro_ctx_set_streams", "ro_ctx_set_call_streams", "ro_ctx_join", "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
+           "ro_ctx_set_streams", "ro_ctx_set_call_streams", "ro_ctx_join", "ro_ctx_selftest_timeout", "ro_last_error", "ro_ctx_profile", "ro_ctx_profile_read", "ro_expand", "ro_batch_ready",
            "ro_batch_ready_calls", "ro_retry", "ro_batch_ready_parent", "ro_gather_commit", "ro_assemble", "ro_assemble_list", "ro_filter_reports",
            "ro_expand_noalloc")
 
@@ -81,6 +81,7 @@ def load(path: Optional[str] = None):
     L.ro_ctx_set_streams.argtypes = [_vp, _vp, _vp]
     L.ro_ctx_set_call_streams.argtypes = [_vp, C.POINTER(_vp), _u32]
     L.ro_ctx_join.argtypes = [_vp]
+    L.ro_ctx_selftest_timeout.argtypes = [_vp, _u32]
     L.ro_last_error.argtypes = [_vp]
     L.ro_last_error.restype = C.c_char_p
     L.ro_ctx_profile.argtypes = [_vp, _u32]
@@ -224,6 +225,12 @@ def ro_batch_ready(ctx, xid, call, d_cand, n_cand, batch_size, flush, d_batched,
                                C.byref(nb) if want_host else None,
                                C.byref(nbt) if want_host else None)
     return (st, nb.value, nbt.value) if want_host else (st, None, None)
+
+
+def ro_ctx_selftest_timeout(ctx, kind: int) -> int:
+    """Runs one bounded device-side wait that nothing releases; returns the
+    status (RO_E_TIMEOUT expected)."""
+    return load().ro_ctx_selftest_timeout(ctx, kind)
 
 
 def ro_batch_ready_calls(ctx, xid, calls, d_cand, n_cand, batch_size, flush, d_batched, batched_cap,

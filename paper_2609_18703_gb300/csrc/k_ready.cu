@@ -463,42 +463,14 @@ __global__ void __launch_bounds__(RB_THREADS) ready_scatter_kernel(ReadyArgs a) 
 // its tile's prefix, the number admitted, the window's live length and so
 // the reservation, and writes; no second launch and no look-back.
 
-// All CTAs of the grid meet here.  Arrivals count up; the last one resets
-// the count and advances the generation the others wait on (bounded: a wait
-// that gives up records ERR_TIMEOUT and the call's results are void).
-__device__ void grid_barrier(ReadyScalars* rs, uint32_t* err) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    const uint32_t gen = ld_acquire(&rs->bar_gen);
-    __threadfence();
-    if (atomicAdd(&rs->bar_count, 1u) == gridDim.x - 1u) {
-      rs->bar_count = 0u;
-      st_release(&rs->bar_gen, gen + 1u);
-    } else {
-      uint32_t spins = 0;
-      while (ld_acquire(&rs->bar_gen) == gen) {
-        if (++spins > SPIN_LIMIT) {
-          atomicOr(err, ERR_TIMEOUT);
-          break;
-        }
-        __nanosleep(32);
-      }
-    }
-    __threadfence();
-  }
-  __syncthreads();
-}
-
 // The one-pass admission of Call a by CTA b of the Call's T + 1 (T tiles,
-// then the window).  gs holds the grid's barrier, launch sequence and
-// conflict tag (one set per launch, the first Call's); seq_owner advances the
-// sequence when done.  Every CTA of the grid meets at the same barriers.
-__device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint32_t b, ReadyScalars* gs,
-                                            bool seq_owner) {
+// then the window).  gs holds the grid's barrier (one per launch, the first
+// Call's); every CTA of the grid meets at the same barriers.
+__device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint32_t b, ReadyScalars* gs) {
   __shared__ unsigned long long s_scan[33];
   __shared__ uint32_t s_rows[RB_ITEMS * (RB_THREADS / 32) + 1];
   __shared__ unsigned long long s_red[2][RB_THREADS / 32];
-  __shared__ unsigned long long s_tot[3];   // prefix of this tile, admitted, bad
+  __shared__ unsigned long long s_tot[5];   // prefix of this tile, admitted, bad, window length, head
   DevScalars* ds = a.ds;
   ReadyScalars* rs = a.rs;
   const bool window = b == T;
@@ -510,19 +482,29 @@ __device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint3
   uint32_t flags = 0u, elig = 0u;
   unsigned long long head = 0, tail = 0, tail0 = 0;
 
-  // this launch's tag for the conflict word (the sequence owner advances the
-  // sequence when done; every CTA reads it first)
-  const uint32_t tag = ld_acquire(&gs->adm_seq) + 1u;
+  // The candidate list is the caller's input: warm L2 with this CTA's
+  // lines while the previous kernel drains, then wait for it (lineage state
+  // may still change until then), and let the next kernel launch.
+  if (!window && a.cand && threadIdx.x < RB_THREADS * RB_ITEMS / 32) {   // one 128-byte line each
+    const uint64_t i = base + (uint64_t)threadIdx.x * 32;
+    if (i < a.n_cand) asm volatile("prefetch.global.L2 [%0];" ::"l"(a.cand + i));
+  }
+  wait_predecessor();
+  allow_successor();
+  // the barrier generation, read with the first loads (no barrier of this
+  // launch completes before this CTA arrives)
+  const uint32_t gen0 = __ldcg(&gs->bar_gen) & ~BAR_FLAG;
+  bool conflict = false;
 
   // A: candidates, slots and claims; the window is compacted meanwhile.  A
-  // claim that met another one (a child named twice) marks the call; without
-  // any, every claim taken stands and the tile counts below are final.
+  // claim that met another one (a child named twice) is reported at the
+  // barrier; without any, every claim taken stands and the tile counts
+  // below are final.
   if (!window) {
     load_group(a, base, g);
     elig = eligible(a, g);
     if (a.cand) {
-      if (claim_group_won(a, base, g, elig, &flags) && ld_acquire(&gs->adm_conflict) != tag)
-        atomicExch(&gs->adm_conflict, tag);
+      conflict = __syncthreads_or(claim_group_won(a, base, g, elig, &flags)) != 0;
     } else {
       flags = elig;   // ids are distinct
     }
@@ -534,11 +516,11 @@ __device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint3
       rs->rb_L = tail - head;
     }
   }
-  grid_barrier(gs, &ds->err);
+  const bool repeats = grid_barrier(gs, (gen0 + 1u) & ~BAR_FLAG, &ds->err, conflict);
 
   // B (repeats only): with every claim settled, a candidate is admitted iff
   // its child holds its claim; the tile counts again
-  if (a.cand && __ldcg(&gs->adm_conflict) == tag) {
+  if (repeats) {
     if (!window) {
       uint32_t ph[RB_ITEMS];
 #pragma unroll
@@ -550,12 +532,17 @@ __device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint3
         if (((elig >> k) & 1u) && ph[k] == ((uint32_t)cand_pos(base, k) << 2)) flags |= 1u << k;
       publish_counts(a, b, flags, g, s_red);
     }
-    grid_barrier(gs, &ds->err);
+    grid_barrier(gs, (gen0 + 2u) & ~BAR_FLAG, &ds->err);
   }
 
-  // C: prefix of this tile, number admitted and bad (one warp)
+  // C: prefix of this tile, number admitted and bad, and the window (one
+  // warp; all its loads in flight together)
   if (threadIdx.x < 32) {
-    unsigned long long pre = 0, K = 0, bad = 0;
+    unsigned long long pre = 0, K = 0, bad = 0, wL = 0, wH = 0;
+    if (threadIdx.x == 0 && !window) {
+      wL = __ldcg(&rs->rb_L);
+      wH = __ldcg(&rs->rb_head);
+    }
     for (uint32_t t = threadIdx.x; t < T; t += 32) {
       const unsigned long long k = __ldcg(cnt_kept + t);
       K += k;
@@ -571,12 +558,13 @@ __device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint3
       s_tot[0] = pre;
       s_tot[1] = K;
       s_tot[2] = bad;
+      s_tot[3] = window ? tail - head : wL;
+      s_tot[4] = window ? head : wH;
     }
   }
   __syncthreads();
   const unsigned long long K = s_tot[1];
-  const unsigned long long L = window ? tail - head : __ldcg(&rs->rb_L);
-  const unsigned long long qhead = window ? head : __ldcg(&rs->rb_head);
+  const unsigned long long L = s_tot[3], qhead = s_tot[4];
   const unsigned long long Tq = L + K;
   const unsigned long long npop = a.flush ? Tq : (Tq / a.batch_size) * a.batch_size;
   if (npop > a.cap) {
@@ -587,7 +575,6 @@ __device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint3
         if (a.cand && ((flags >> k) & 1u)) a.slot[g.c[k]].phase = WAIT_UNCLAIMED;
     } else if (threadIdx.x == 0) {
       plan_reservation(a, head, tail, tail0, K, s_tot[2]);   // records the refusal
-      if (seq_owner) st_release(&gs->adm_seq, tag);
     }
     return;
   }
@@ -617,11 +604,10 @@ __device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint3
     }
     if (threadIdx.x == 0) plan_reservation(a, head, tail, tail0, K, s_tot[2]);
   }
-  if (seq_owner && threadIdx.x == 0) st_release(&gs->adm_seq, tag);   // every CTA has read it
 }
 
 __global__ void __launch_bounds__(RB_THREADS) ready_fused_kernel(ReadyArgs a) {
-  fused_admit(a, gridDim.x - 1u, blockIdx.x, a.rs, blockIdx.x == gridDim.x - 1u);
+  fused_admit(a, gridDim.x - 1u, blockIdx.x, a.rs);
 }
 
 // Several Calls' admissions from one candidate list: the grid holds each
@@ -629,7 +615,7 @@ __global__ void __launch_bounds__(RB_THREADS) ready_fused_kernel(ReadyArgs a) {
 __global__ void __launch_bounds__(RB_THREADS) ready_fused_calls_kernel(MultiReadyArgs m) {
   const uint32_t per = gridDim.x / m.n;   // CTAs per Call
   const uint32_t k = blockIdx.x / per, b = blockIdx.x % per;
-  fused_admit(m.a[k], per - 1u, b, m.a[0].rs, k == 0 && b == per - 1u);
+  fused_admit(m.a[k], per - 1u, b, m.a[0].rs);
 }
 
 void launch_ready(const LaunchCfg& L, const ReadyArgs& a) {

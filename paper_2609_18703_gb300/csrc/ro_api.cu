@@ -181,6 +181,7 @@ struct ro_ctx {
   std::vector<Expansion> exps;
   TsBuf ts[N_TS];
   DevBuf code;
+  DevBuf selftest;                      // ro_ctx_selftest_timeout scratch
   DevBuf x_mb, x_coff, x_mtfp, x_hdr;   // explicit-list assembly scratch
   // parent-bound reservation scratch (see ParentArgs)
   DevBuf pb_key[2], pb_val[2], pb_child, pb_hist, pb_dtot, pb_first, pb_endp, pb_hsz, pb_left,
@@ -622,7 +623,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   for (auto& t : c->ts) {
     free_buf(t.flag); free_buf(t.agg); free_buf(t.inc);
   }
-  free_buf(c->code); free_buf(c->x_mb); free_buf(c->x_coff); free_buf(c->x_mtfp); free_buf(c->x_hdr);
+  free_buf(c->code); free_buf(c->selftest); free_buf(c->x_mb); free_buf(c->x_coff); free_buf(c->x_mtfp); free_buf(c->x_hdr);
   for (DevBuf* b : {&c->pb_key[0], &c->pb_key[1], &c->pb_val[0], &c->pb_val[1], &c->pb_child,
                     &c->pb_hist, &c->pb_dtot, &c->pb_first, &c->pb_endp, &c->pb_hsz, &c->pb_left,
                     &c->pb_hoff, &c->pb_rem})
@@ -968,6 +969,30 @@ ro_status ro_batch_ready_calls(ro_ctx* c, int32_t xid, uint32_t n, const uint32_
     for (uint32_t k = 0; k < n; ++k) launch_ready(c->L, m.a[k]);
   }
   return check_launch(c, "batch_ready_calls");
+}
+
+// ---------------------------------------------------------------------------
+ro_status ro_ctx_selftest_timeout(ro_ctx* c, uint32_t kind) {
+  RO_TRY(enter(c));
+  if (kind > 1) return fail(c, RO_E_INVAL, "ro_ctx_selftest_timeout: kind %u (0 or 1)", kind);
+  DeviceGuard g(c->device);
+  RO_TRY(sync_and_check(c));   // earlier work settled, its errors reported first
+  const size_t flags = 2 * sizeof(unsigned long long), vals = 2 * 16;
+  RO_TRY(ensure(c, c->selftest, flags + 2 * vals + sizeof(ReadyScalars), "self-test scratch"));
+  char* base = (char*)c->selftest.p;
+  cudaError_t e = cudaMemsetAsync(base, 0, flags + 2 * vals + sizeof(ReadyScalars), c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "self-test scratch");
+  SelftestArgs a{};
+  a.kind = kind;
+  a.ts.flag = (unsigned long long*)base;
+  a.ts.agg = (unsigned long long*)(base + flags);
+  a.ts.inc = (unsigned long long*)(base + flags + vals);
+  a.epoch = 1ull;   // the zeroed flags hold epoch 0
+  a.rs = (ReadyScalars*)(base + flags + 2 * vals);
+  a.err = &c->ds->err;
+  launch_selftest(c->stream, a);
+  RO_TRY(check_launch(c, "selftest"));
+  return sync_and_check(c);
 }
 
 // ---------------------------------------------------------------------------

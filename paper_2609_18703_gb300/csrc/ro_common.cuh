@@ -147,9 +147,8 @@ struct alignas(128) ReadyScalars {
   unsigned long long rb_kept, rb_bad, rb_L, rb_k, rb_npop, rb_head, rb_tail, rb_n_batches;
   unsigned long long epoch;
   uint32_t rb_ticket, rb_err, tile_ctr, exit_ctr;
-  // one-pass admission: grid barrier (arrivals, generation), launch
-  // sequence and the tag of the latest launch that met a repeated child
-  uint32_t bar_count, bar_gen, adm_seq, adm_conflict;
+  // one-pass admission: grid barrier (arrivals, generation)
+  uint32_t bar_count, bar_gen;
 };
 // TS_COMMIT and TS_COMMIT_ODD: the completion lists and plans of commits of
 // even and odd sequence (they may run at the same time, on two streams);
@@ -356,6 +355,44 @@ __device__ T lookback_exclusive(const TileStatus<T>& ts, uint32_t tile, const T&
   if (lane == 0) ts_publish(ts, tile, excl + local, 2ull, epoch);
   __syncwarp();
   return excl;
+}
+
+// All CTAs of the grid meet here.  Arrivals count up in the low 16 bits of
+// the count (a CTA passing `flag` also adds 1 << 16); the last one resets the
+// count and advances the generation to `target` (the launch's first
+// generation plus the barrier's number, read before any CTA could arrive),
+// with bit 31 set when any CTA passed `flag`.  The others wait for it
+// (bounded: a wait that gives up records ERR_TIMEOUT and the call's results
+// are void).  Returns whether any CTA passed `flag`, to every thread.
+constexpr uint32_t BAR_FLAG = 1u << 31;
+__device__ __forceinline__ bool grid_barrier(ReadyScalars* rs, uint32_t target, uint32_t* err,
+                                             bool flag = false) {
+  __shared__ uint32_t s_flag;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const uint32_t add = 1u + (flag ? (1u << 16) : 0u);
+    const uint32_t old = atomicAdd(&rs->bar_count, add);
+    if ((old & 0xFFFFu) == gridDim.x - 1u) {
+      const bool any = ((old + add) >> 16) != 0u;
+      rs->bar_count = 0u;
+      st_release(&rs->bar_gen, target | (any ? BAR_FLAG : 0u));
+      s_flag = any;
+    } else {
+      uint32_t spins = 0, g;
+      while (((g = ld_acquire(&rs->bar_gen)) & ~BAR_FLAG) != target) {
+        if (++spins > SPIN_LIMIT) {
+          atomicOr(err, ERR_TIMEOUT);
+          break;
+        }
+        __nanosleep(32);
+      }
+      s_flag = (g & BAR_FLAG) != 0u;
+    }
+    __threadfence();
+  }
+  __syncthreads();
+  return s_flag;
 }
 
 // Claim the next tile of a dynamically scheduled (persistent) kernel.

@@ -100,8 +100,8 @@ inline void launch_k(const LaunchCfg& L, int kid, void (*kern)(Arg), int grid, i
 
 // The same for a kernel whose CTAs wait for one another (grid barriers): a
 // cooperative launch, so that every CTA of the grid is resident at once (the
-// grid must not exceed what the device holds; see LaunchCfg::grid_rb_coop).
-// No programmatic dependent launch: the kernel starts after its predecessor.
+// grid must not exceed what the device holds; see LaunchCfg::grid_rb_coop),
+// with programmatic dependent launch as above.
 template <typename Arg>
 inline void launch_coop(const LaunchCfg& L, int kid, void (*kern)(Arg), int grid, int block, const Arg& a) {
   prof_begin(L.prof, L.stream, kid);
@@ -109,14 +109,26 @@ inline void launch_coop(const LaunchCfg& L, int kid, void (*kern)(Arg), int grid
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3((unsigned)block);
   cfg.stream = L.stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeCooperative;
   attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   cudaLaunchKernelEx(&cfg, kern, a);
   prof_end(L.prof, L.stream, kid);
 }
+
+// ---- self-test of the bounded waits ---------------------------------------------------
+struct SelftestArgs {
+  uint32_t kind;              // 0: look-back on an unpublished tile; 1: grid barrier missing an arrival
+  TileStatus<unsigned long long> ts;   // two tiles, flags zero
+  unsigned long long epoch;   // an epoch no flag holds
+  ReadyScalars* rs;           // barrier scratch, zeroed
+  uint32_t* err;
+};
+void launch_selftest(cudaStream_t s, const SelftestArgs& a);
 
 // ---- ro_expand ----------------------------------------------------------------
 struct ExpandScanArgs {
