@@ -243,7 +243,7 @@ __global__ void __maxnreg__(CP_MAXREG) commit_plan_kernel(CommitArgs a) {
   }
   const uint32_t n_part = participants(n_tiles);
   if (blockIdx.x >= n_part) return;
-  const int slot = a.pslot ? TS_COMMIT_ODD : TS_COMMIT;
+  const int slot = commit_slot(a.pslot);
   const unsigned long long epoch = ds->epoch[slot];
 
   for (;;) {

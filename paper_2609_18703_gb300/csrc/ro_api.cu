@@ -37,8 +37,8 @@ using namespace ro;
 namespace {
 
 constexpr int MAX_EXPANSIONS = 64;
-constexpr int N_TS = 8;    // tile-status slots (TS_* in ro_common.cuh)
-constexpr int RING = 3;    // list / plan slots per expansion
+constexpr int N_TS = N_TILE_SLOTS;    // tile-status slots (TS_* in ro_common.cuh)
+constexpr int RING = FIN_STREAMS + 1 > 3 ? FIN_STREAMS + 1 : 3;   // list / plan slots per expansion
 // Completion bitmaps per expansion, taken in turn by its commits.  A commit
 // may reuse a slot once the plan that read it (BM_SLOTS commits earlier) is
 // done; the context's stream waits for that only every BM_WAIT commits (for
@@ -157,14 +157,14 @@ struct ro_ctx {
   // Completion lists and their plans (commit_plan): with separate streams,
   // commits of even and odd sequence alternate between two streams, so the
   // plans of consecutive commits run at the same time.
-  cudaStream_t fin_stream[2] = {nullptr, nullptr};
-  cudaStream_t own_fin[2] = {nullptr, nullptr};   // created for fin_stream, destroyed with the context
+  cudaStream_t fin_stream[FIN_STREAMS] = {};
+  cudaStream_t own_fin[FIN_STREAMS] = {};   // created for fin_stream, destroyed with the context
   int last_fin = 0;                     // the stream of the latest commit's plan
   uint32_t n_calls = 1;
   uint32_t commit_seq = 0;              // commits issued on this context
   uint64_t copy_small_chunks = AC_SMALL_CHUNKS;   // copies this small go direct
   int num_sms = 0;
-  LaunchCfg L{}, Lp{}, Lc{}, Lf[2]{};
+  LaunchCfg L{}, Lp{}, Lc{}, Lf[FIN_STREAMS]{};
   DevScalars* ds = nullptr;
   DevScalars* hs = nullptr;   // pinned mirror
   ReadyScalars* rs = nullptr;   // per Call, device
@@ -186,7 +186,7 @@ struct ro_ctx {
   // parent-bound reservation scratch (see ParentArgs)
   DevBuf pb_key[2], pb_val[2], pb_child, pb_hist, pb_dtot, pb_first, pb_endp, pb_hsz, pb_left,
       pb_hoff, pb_rem;
-  Ev fork, x_planned, join_plan, join_copy, fin_fork[2], fin_join[2], fin_plan;
+  Ev fork, x_planned, join_plan, join_copy, fin_fork[FIN_STREAMS], fin_join[FIN_STREAMS], fin_plan;
   // Caller memory written by the copies issued since the context's stream
   // last waited for the copy stream: a later call's planning (another
   // stream) may run while they do, so planning that writes any of it waits
@@ -345,7 +345,7 @@ ro_status settle_calls(ro_ctx* c) {
 
 ro_status join(ro_ctx* c) {
   RO_TRY(settle_calls(c));
-  for (int k = 0; k < 2; ++k) RO_TRY(order(c, c->fin_join[k], c->fin_stream[k], c->stream));
+  for (int k = 0; k < FIN_STREAMS; ++k) RO_TRY(order(c, c->fin_join[k], c->fin_stream[k], c->stream));
   RO_TRY(order(c, c->join_plan, c->plan_stream, c->stream));
   if (c->copy_stream != c->plan_stream) RO_TRY(order(c, c->join_copy, c->copy_stream, c->stream));
   // planning forks from the context's stream: it now follows every copy
@@ -530,7 +530,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->stream = (cudaStream_t)stream;
   c->plan_stream = c->stream;
   c->copy_stream = c->stream;
-  c->fin_stream[0] = c->fin_stream[1] = c->stream;
+  for (auto& f : c->fin_stream) f = c->stream;
   c->n_calls = n_calls;
   if (const char* e = std::getenv("RO_COPY_SMALL_CHUNKS")) c->copy_small_chunks = std::strtoull(e, nullptr, 10);
   cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
@@ -586,7 +586,7 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   c->L.grid_pb_sort = grid_for(kernel_ptr_parent(K_PB_SORT), PB_THREADS, s, 8);
   c->Lp = c->L;
   c->Lc = c->L;
-  c->Lf[0] = c->Lf[1] = c->L;
+  for (auto& f : c->Lf) f = c->L;
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) {
     free_scalars(c);
@@ -629,7 +629,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
                     &c->pb_hoff, &c->pb_rem})
     free_buf(*b);
   free_ev(c->fork); free_ev(c->x_planned); free_ev(c->join_plan); free_ev(c->join_copy);
-  for (int k = 0; k < 2; ++k) {
+  for (int k = 0; k < FIN_STREAMS; ++k) {
     free_ev(c->fin_fork[k]);
     free_ev(c->fin_join[k]);
     if (c->own_fin[k]) cudaStreamDestroy(c->own_fin[k]);
@@ -662,10 +662,10 @@ ro_status ro_ctx_set_streams(ro_ctx* c, void* plan_stream, void* copy_stream) {
   c->plan_stream = plan_stream ? (cudaStream_t)plan_stream : c->stream;
   c->copy_stream = copy_stream ? (cudaStream_t)copy_stream : c->stream;
   // with streams of its own for assembly, the context also runs the
-  // completion lists and plans on two streams of its own, so a commit's plan
-  // overlaps the next commits' scatters and the next commit's plan
+  // completion lists and plans on FIN_STREAMS streams of its own, so a
+  // commit's plan overlaps the next commits' scatters and plans
   if (c->plan_stream != c->stream) {
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < FIN_STREAMS; ++k) {
       if (!c->own_fin[k]) {
         cudaError_t e = cudaStreamCreateWithFlags(&c->own_fin[k], cudaStreamNonBlocking);
         if (e != cudaSuccess) {
@@ -676,11 +676,11 @@ ro_status ro_ctx_set_streams(ro_ctx* c, void* plan_stream, void* copy_stream) {
       c->fin_stream[k] = c->own_fin[k];
     }
   } else {
-    c->fin_stream[0] = c->fin_stream[1] = c->stream;
+    for (auto& f : c->fin_stream) f = c->stream;
   }
   c->Lp.stream = c->plan_stream;
   c->Lc.stream = c->copy_stream;
-  for (int k = 0; k < 2; ++k) c->Lf[k].stream = c->fin_stream[k];
+  for (int k = 0; k < FIN_STREAMS; ++k) c->Lf[k].stream = c->fin_stream[k];
   return RO_OK;
 }
 
@@ -1198,24 +1198,25 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   }
   ca.plan = list_plan_bufs(LS, std::max<uint64_t>(x->N, 1));
   ca.ds = c->ds;
-  // consecutive commits plan on alternate streams, each with a scan slot of its own
-  const int pf = (int)(c->commit_seq & 1u);
+  // consecutive commits plan on the completion streams in turn, each with a scan slot of its own
+  const int pf = (int)(c->commit_seq % FIN_STREAMS);
   ca.pslot = pf;
-  RO_TRY(tile_status(c, pf ? TS_COMMIT_ODD : TS_COMMIT, ceil_div(ceil_div(x->P, 32), (uint64_t)CP_WORDS),
-                     &ca.tsq));
+  RO_TRY(tile_status(c, commit_slot(pf), ceil_div(ceil_div(x->P, 32), (uint64_t)CP_WORDS), &ca.tsq));
   // The bitmap slots of this commit and the next BM_WAIT - 1 are free once
   // every plan up to commit w - BM_WAIT - 1 is done: wait for the latest such
   // plan of each completion stream (a stream runs its plans in order).
   if (x->commits % BM_WAIT == 0 && x->commits > (uint64_t)BM_WAIT) {
     const uint64_t w = x->commits;
-    bool seen[2] = {false, false};
+    bool seen[FIN_STREAMS] = {};
+    int n_seen = 0;
     // (commits w - BM_SLOTS .. w - BM_WAIT - 1: the slot of commit w - BM_SLOTS
     // is this commit's, and its event is not overwritten yet)
-    for (uint64_t j = w - BM_WAIT - 1; j + BM_SLOTS >= w && !(seen[0] && seen[1]); --j) {
+    for (uint64_t j = w - BM_WAIT - 1; j + BM_SLOTS >= w && n_seen < FIN_STREAMS; --j) {
       const int k = S.bm_stream[j % BM_SLOTS];
       if (!seen[k]) {
         RO_TRY(ev_wait(c, S.bm_free[j % BM_SLOTS], c->stream));
         seen[k] = true;
+        ++n_seen;
       }
       if (j == 0) break;
     }

@@ -22,6 +22,16 @@
 
 namespace ro {
 
+// Completion streams a context plans its commits on (consecutive commits
+// take them in turn), at most FIN_MAX; tile-status slots of the scans.
+#ifndef RO_FIN_STREAMS
+#define RO_FIN_STREAMS 3
+#endif
+constexpr int FIN_MAX = 4;
+constexpr int FIN_STREAMS = RO_FIN_STREAMS;
+static_assert(FIN_STREAMS >= 1 && FIN_STREAMS <= FIN_MAX, "1 to 4 completion streams");
+constexpr int N_TILE_SLOTS = 10;
+
 // ---- Grain phases (Eq. 2) -------------------------------------------------
 constexpr uint32_t PH_WAITING = 0u, PH_READY = 1u, PH_INFLIGHT = 2u, PH_SEALED = 3u;
 constexpr uint32_t CLAIM_NONE = 0x3FFFFFFFu;              // unclaimed WAITING
@@ -118,7 +128,7 @@ struct DevScalars {
   unsigned long long n_children, n_empty, last_nonempty_parent,
       n_heavy;   // children of parents with at least HEAVY_CHILDREN children
   // ro_gather_commit
-  unsigned long long cm_n, cm_n_done[2];   // completed parents, per plan slot
+  unsigned long long cm_n, cm_n_done[FIN_MAX];   // completed parents, per plan slot
   // per commit, in two slots (commit sequence & 1): duplicate candidates and
   // accepted GroupFailures the scatter saw; the next commit's scatter clears
   // the slot after this one
@@ -134,9 +144,9 @@ struct DevScalars {
   unsigned long long as_bytes;    // bytes of the latest assemble (host read-back)
   unsigned long long as_elems;    // list entries of the latest assemble (host read-back)
   // dynamic tile counters / exit tickets / scan epochs, one per look-back kernel
-  uint32_t tile_ctr[8];
-  uint32_t exit_ctr[8];
-  unsigned long long epoch[8];
+  uint32_t tile_ctr[N_TILE_SLOTS];
+  uint32_t exit_ctr[N_TILE_SLOTS];
+  unsigned long long epoch[N_TILE_SLOTS];
 };
 // Admission scalars of one Call (ro_batch_ready): the first pass's counts,
 // its exit ticket and the reservation it plans, the scatter pass's tile
@@ -150,11 +160,15 @@ struct alignas(128) ReadyScalars {
   // one-pass admission: grid barrier (arrivals, generation)
   uint32_t bar_count, bar_gen;
 };
-// TS_COMMIT and TS_COMMIT_ODD: the completion lists and plans of commits of
-// even and odd sequence (they may run at the same time, on two streams);
+// TS_COMMIT, TS_COMMIT_ODD, TS_COMMIT_2, TS_COMMIT_3: the completion lists
+// and plans of commits whose sequence number is 0, 1, 2, 3 modulo the
+// completion streams (they may run at the same time, one per stream);
 // 5: asm_copy's exit ticket.
 enum TileSlot { TS_EXPAND = 0, TS_COMMIT_ODD = 1, TS_COMMIT = 2, TS_ASM_PARENTS = 3,
-                TS_ASM_MEMBERS = 4, TS_RETRY = 6, TS_PARENT = 7 };
+                TS_ASM_MEMBERS = 4, TS_RETRY = 6, TS_PARENT = 7, TS_COMMIT_2 = 8, TS_COMMIT_3 = 9 };
+__host__ __device__ constexpr int commit_slot(int pslot) {
+  return pslot == 0 ? TS_COMMIT : pslot == 1 ? TS_COMMIT_ODD : pslot == 2 ? TS_COMMIT_2 : TS_COMMIT_3;
+}
 
 // Wait until the grid this launch depends on (programmatic dependent launch)
 // has completed and its memory is visible; a no-op without a dependency.

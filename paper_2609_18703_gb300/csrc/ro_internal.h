@@ -294,7 +294,7 @@ struct CommitArgs {
   const uint64_t* offsets;
   ListBufs list;              // written: the completed parents with member bases
   PlanBufs plan;              // written: the copy plan of that list
-  int pslot;                  // commit_plan's scan slot (0 / 1, alternating by commit)
+  int pslot;                  // commit_plan's scan slot (commit sequence modulo FIN_STREAMS)
   DevScalars* ds;
   TileStatus<Quad64> tsq;     // commit_plan's look-back
 };
