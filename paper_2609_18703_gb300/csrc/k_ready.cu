@@ -578,6 +578,18 @@ __device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint3
     }
     return;
   }
+  // entries queued by earlier calls leave first: the Call's T + 1 CTAs take
+  // a slice each (positions below L, apart from the new entries' L and up)
+  {
+    const unsigned long long n_old = L < npop ? L : npop;
+    const unsigned long long per = (n_old + T) / (T + 1), j0 = (unsigned long long)b * per;
+    const unsigned long long j1 = j0 + per < n_old ? j0 + per : n_old;
+    for (unsigned long long j = j0 + threadIdx.x; j < j1; j += RB_THREADS) {
+      const uint32_t c = a.queue[qhead + j];
+      a.batched[j] = c;
+      a.slot[c].phase = (a.slot[c].phase & ~3u) | PH_INFLIGHT;
+    }
+  }
   if (!window) {
     uint32_t rowpfx[RB_ITEMS];
     rank_rows(flags, s_rows, rowpfx);
@@ -594,15 +606,8 @@ __device__ __forceinline__ void fused_admit(const ReadyArgs a, uint32_t T, uint3
         a.slot[c].phase = ph_make(PH_READY, 0u);
       }
     }
-  } else {
-    // entries queued by earlier calls leave first
-    const unsigned long long n_old = L < npop ? L : npop;
-    for (unsigned long long j = threadIdx.x; j < n_old; j += RB_THREADS) {
-      const uint32_t c = a.queue[head + j];
-      a.batched[j] = c;
-      a.slot[c].phase = (a.slot[c].phase & ~3u) | PH_INFLIGHT;
-    }
-    if (threadIdx.x == 0) plan_reservation(a, head, tail, tail0, K, s_tot[2]);
+  } else if (threadIdx.x == 0) {
+    plan_reservation(a, head, tail, tail0, K, s_tot[2]);
   }
 }
 
