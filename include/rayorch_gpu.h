@@ -28,8 +28,8 @@
  *   completion lists and admissions: ro_assemble plans on the context's plan
  *   stream and copies on its copy stream, with separate streams set
  *   (ro_ctx_set_streams) ro_gather_commit builds its completed-parent list
- *   and that list's copy plan on one of two streams the context owns
- *   (commits alternate between them), and with Call streams set
+ *   and that list's copy plan on one of three streams the context owns
+ *   (commits take them in turn), and with Call streams set
  *   (ro_ctx_set_call_streams) ro_batch_ready runs on its Call's stream.
  *   Each assembly is ordered after all work the caller issued on the
  *   context before it; the caller's ro_assemble
@@ -139,15 +139,15 @@ ro_status ro_ctx_sync(ro_ctx* ctx);
  * plan_stream and copy_stream are cudaStream_t handles on the context's
  * device, NULL for the context's stream.  With separate streams the planning
  * and copy of one wave's completed parents overlap the next waves' admission
- * and commits; up to three commits and assemblies per expansion may be in
- * flight at once (the context keeps three list and plan slots per expansion
+ * and commits; up to four commits and assemblies per expansion may be in
+ * flight at once (the context keeps four list and plan slots per expansion
  * and orders their reuse with events).  With a plan stream other than the
- * context's stream, the context also creates two streams of its own
+ * context's stream, the context also creates three streams of its own
  * (destroyed with the context) for the commits' completed-parent lists and
  * their copy plans, which consecutive commits take in turn: one commit's
  * list is built while the next commits' reports are applied and the next
- * commit's list is built (four completion bitmaps per expansion, taken in
- * turn).  The context's stream first waits for the old streams.  The caller keeps the streams alive until ro_ctx_destroy
+ * two commits' lists are built (32 completion bitmaps per expansion, taken
+ * in turn).  The context's stream first waits for the old streams.  The caller keeps the streams alive until ro_ctx_destroy
  * or the next ro_ctx_set_streams. */
 ro_status ro_ctx_set_streams(ro_ctx* ctx, void* plan_stream, void* copy_stream);
 /* Streams for the Calls' admissions (Section 4.3: each Call has its own
@@ -169,7 +169,7 @@ ro_status ro_ctx_set_streams(ro_ctx* ctx, void* plan_stream, void* copy_stream);
  * with n > 0. */
 ro_status ro_ctx_set_call_streams(ro_ctx* ctx, void* const* streams, uint32_t n);
 /* Make the context's stream wait (on the GPU) for all work issued so far on
- * the plan and copy streams, the context's two completion streams and the
+ * the plan and copy streams, the context's three completion streams and the
  * Calls' streams.  Call it before reading assembly outputs in
  * stream order, before starting a capture of the context's stream, and
  * before ending one (a captured assembly forks onto the other streams, and a

@@ -155,8 +155,8 @@ struct ro_ctx {
   cudaStream_t plan_stream = nullptr;   // assembly planning
   cudaStream_t copy_stream = nullptr;   // assembly copies
   // Completion lists and their plans (commit_plan): with separate streams,
-  // commits of even and odd sequence alternate between two streams, so the
-  // plans of consecutive commits run at the same time.
+  // consecutive commits take FIN_STREAMS streams in turn, so the plans of
+  // consecutive commits run at the same time.
   cudaStream_t fin_stream[FIN_STREAMS] = {};
   cudaStream_t own_fin[FIN_STREAMS] = {};   // created for fin_stream, destroyed with the context
   int last_fin = 0;                     // the stream of the latest commit's plan
