@@ -1198,10 +1198,16 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
   }
   ca.plan = list_plan_bufs(LS, std::max<uint64_t>(x->N, 1));
   ca.ds = c->ds;
-  // consecutive commits plan on the completion streams in turn, each with a scan slot of its own
+  // consecutive commits plan on the completion streams in turn, each with a
+  // scan slot of its own; every slot is sized together, so that a capture of
+  // later commits finds its slot grown whichever stream the first calls took
   const int pf = (int)(c->commit_seq % FIN_STREAMS);
   ca.pslot = pf;
-  RO_TRY(tile_status(c, commit_slot(pf), ceil_div(ceil_div(x->P, 32), (uint64_t)CP_WORDS), &ca.tsq));
+  for (int k = 0; k < FIN_STREAMS; ++k) {
+    TileStatus<Quad64> t;
+    RO_TRY(tile_status(c, commit_slot(k), ceil_div(ceil_div(x->P, 32), (uint64_t)CP_WORDS), &t));
+    if (k == pf) ca.tsq = t;
+  }
   // The bitmap slots of this commit and the next BM_WAIT - 1 are free once
   // every plan up to commit w - BM_WAIT - 1 is done: wait for the latest such
   // plan of each completion stream (a stream runs its plans in order).

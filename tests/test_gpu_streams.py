@@ -207,6 +207,41 @@ def test_async_waves_captured_in_a_graph():
             ro.ro_ctx_destroy(ctx)
 
 
+def test_one_wave_captured_after_one_eager_commit():
+    """A one-wave pass run once eagerly (its commit takes one completion
+    stream), then captured and replayed twice (the captured commits take the
+    next streams in turn): every stream's scan slot was sized by the eager
+    call, so the capture never needs to grow a buffer, and each replay
+    equals the oracle."""
+    lv = docpage(parents=3000, waves=1).top
+    a = host_arena(lv)
+    ref, total = oracle_waves(lv, a)
+    ps = AsyncPass(lv, a)
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        ctx = ro.ro_ctx_create(0, stream, 1)
+        ro.ro_ctx_set_streams(ctx, torch.cuda.Stream(), torch.cuda.Stream())
+        try:
+            ps.waves(ctx, ps.expand(ctx))
+            assert ro.ro_ctx_sync(ctx) == ro.RO_OK
+            for _ in range(2):
+                ro.ro_ctx_reset(ctx)
+                x = ps.expand(ctx)
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    ps.waves(ctx, x)
+                ps.out.zero_()
+                for t in ps.status + ps.off + ps.len + ps.done:
+                    t.zero_()
+                ro.ro_ctx_reset(ctx)
+                ps.expand(ctx)
+                g.replay()
+                assert ro.ro_ctx_sync(ctx) == ro.RO_OK, ro.ro_last_error(ctx)
+                ps.check(ref, total)
+        finally:
+            ro.ro_ctx_destroy(ctx)
+
+
 def test_explicit_lists_between_commits_see_exactly_the_earlier_commits():
     lv = docpage(parents=2500, waves=10).top
     rng = np.random.default_rng(21)
