@@ -104,3 +104,42 @@ def test_bad_arguments_change_nothing():
         for c in range(2):
             ls.batch_ready(x, c, np.arange(7, dtype=np.uint32), 4, flush=True)
         ls.check_stats()
+
+
+def test_empty_lists_flush_exact_and_short_capacities():
+    """Edge cases of one launch over several Calls: an empty candidate list
+    (one id past the expansion: only the windows earlier calls left move,
+    on flush), a capacity exactly
+    equal to a Call's reservation (admitted) and one entry short of it
+    (refused, that Call alone), and a single Call through the same entry
+    point; each against the oracle's admissions in turn.  The exact sizes
+    come from a second context with the same history."""
+    rng = np.random.default_rng(515)
+    P = 2500
+    counts = rng.integers(1, 7, P).astype(np.uint32)
+    calls = (np.arange(P) % 3).astype(np.uint8)
+    B = 16
+
+    def history(ls):
+        x = ls.expand(counts, parent_call=calls)["xid"]
+        N = ls.N[x]
+        perm = np.random.default_rng(516).permutation(N).astype(np.uint32)
+        _admit_all(ls, x, [0, 1, 2], perm[:3001], B, False, [N + B] * 3)   # partial batches stay
+        none = np.array([N + 5], np.uint32)   # one id past the expansion: admits nothing
+        _admit_all(ls, x, [2, 0, 1], none, B, False, [N + B] * 3)       # nothing moves
+        return x, N, perm
+
+    with Lockstep(n_calls=3) as probe:
+        x, N, perm = history(probe)
+        sizes = [b.size for b in _admit_all(probe, x, [0, 1, 2], perm[3001:6001], B, False, [N + B] * 3)]
+    assert sizes[0] > 0 and sizes[2] > 0
+    with Lockstep(n_calls=3) as ls:
+        x, N, perm = history(ls)
+        got = _admit_all(ls, x, [0, 1, 2], perm[3001:6001], B, False, [sizes[0], N + B, sizes[2] - 1])
+        assert got[0] is not None and got[0].size == sizes[0]
+        assert got[1] is not None and got[2] is None   # refused alone
+        _admit_all(ls, x, [1, 2, 0], np.array([N + 5], np.uint32), B, True, [N + B] * 3)   # the windows flush
+        _admit_all(ls, x, [1], perm[6001:], B, True, [N + B])           # one Call
+        for c in range(3):
+            ls.batch_ready(x, c, None, B, flush=True)
+        ls.check_stats()
