@@ -7,12 +7,15 @@
 // keeps the smallest claim.  Lists of up to a few thousand tiles of 2,048
 // candidates take one kernel:
 //   ready_fused   cooperative launch, one CTA per tile plus one for the
-//                 queue window: claims, a grid barrier, per-tile admitted
-//                 counts, a grid barrier, then every CTA knows its tile's
+//                 queue window: claims and per-tile admitted counts, a grid
+//                 barrier (and, only when some child was named twice, a
+//                 recount and a second one), then every CTA knows its tile's
 //                 prefix and the reservation and writes its children into the
 //                 reserved batches (IN-FLIGHT) or behind the queue's tail
-//                 (READY); the window's CTA compacts the window meanwhile and
-//                 moves the entries earlier calls queued, which leave first.
+//                 (READY); the window's CTA compacts the window meanwhile,
+//                 and the entries earlier calls queued leave first, a slice
+//                 per CTA.  ready_fused_calls runs several Calls' admissions
+//                 from one candidate list in one such grid.
 // Longer lists (and every list with RO_ADMIT_TWO_PASS set) take two:
 //   ready_count   decides admission.  Counting the claims' transitions out of
 //                 "unclaimed" gives the exact number admitted.  The last CTA
@@ -275,7 +278,8 @@ __device__ void compact_window(const ReadyArgs& a, unsigned long long* s_scan, u
 // batches leave (all with flush); parent-bound: nothing here, the window
 // goes to launch_parent.  A reservation larger than the output capacity
 // fails the call (rb_err): the queue keeps its (compacted) window and the
-// second pass releases the claims.
+// claims are released (by the scatter pass, or in the one-pass admission
+// by the CTAs that took them).
 __device__ void plan_reservation(const ReadyArgs& a, unsigned long long head, unsigned long long tail,
                                  unsigned long long tail0, unsigned long long K, unsigned long long bad) {
   DevScalars* ds = a.ds;
