@@ -648,17 +648,19 @@ def kernel_alg_bytes(info: dict) -> dict:
 
 
 # ncu DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch
-# of a kernel, from one capture of the named workload and command, with the
-# sha256 (first 16 hex digits) of the kernel's source file at capture time;
-# a source that has changed since makes the bench report traffic as null.
+# of a kernel, from one capture of the workload named by its description (the
+# line's config.workload) run with the default options, with the sha256
+# (first 16 hex digits) of the kernel's source file at capture time; another
+# workload or size, a non-default run option, or a source that has changed
+# since makes the bench report traffic as null.
 KERNEL_SOURCE = {"expand_scan": "k_expand.cu", "expand_fill": "k_expand.cu",
                  "ready_count": "k_ready.cu", "ready_scatter": "k_ready.cu", "ready_fused": "k_ready.cu",
                  "commit_scatter": "k_commit.cu", "commit_fix": "k_commit.cu",
                  "commit_plan": "k_complete.cu", "asm_members": "k_assemble.cu",
                  "asm_copy": "k_assemble.cu"}
-# (workload, kernel) -> (bytes per launch, source sha16, how it was captured)
+# (workload description, kernel) -> (bytes per launch, source sha16, how it was captured)
 TRAFFIC = {
-    ("docpage", "asm_copy"): (
+    ("document->page: 1000000 parents, 16399843 children, 256 arrival waves, batch 256", "asm_copy"): (
         82359700, "17d3df01e8ba8a81",
         "ncu dram__bytes_read.sum + dram__bytes_write.sum (one pass) of all 256 asm_copy launches "
         "of one full-size 1M-document step, averaged per launch: 12.99 GB read, 8.09 GB written "
@@ -674,9 +676,9 @@ def source_sha16(kernel: str):
         return hashlib.sha256(fh.read()).hexdigest()[:16]
 
 
-def measured_traffic(workload: str, kernel: str):
-    t = TRAFFIC.get((workload, kernel))
-    if not t or t[1] != source_sha16(kernel):
+def measured_traffic(workload_desc: str, kernel: str, default_run: bool = True):
+    t = TRAFFIC.get((workload_desc, kernel))
+    if not default_run or not t or t[1] != source_sha16(kernel):
         return None, None
     return t[0], t[2]
 
@@ -821,7 +823,9 @@ def run_ours(args, rank, world, local_rank):
     n_launch = prof[dom][0] // kt_steps
     dom_ms = kernel_ms[dom]
     achieved = alg[dom] / (dom_ms * 1e-3) / 1e9 if dom_ms > 0 else 0.0
-    traffic, traffic_src = measured_traffic(args.workload, dom)
+    default_run = not (ps.parent_bound or ps.lists or ps.keep is not None or args.one_stream
+                       or graph is None)
+    traffic, traffic_src = measured_traffic(cfg["workload"], dom, default_run)
     pass_alg = 33.0 * ps.N + 25.0 * ps.P + 2.0 * S
     n_entries = int(ps.n_elems.sum().item()) if ps.lists else 0
     if ps.lists:   # per entry: state, offset, length; per listed parent: its range start
@@ -1341,7 +1345,7 @@ def run_streaming(args, rank, world, local_rank):
     dom = max((k for k in alg if k in kernel_ms), key=lambda k: alg[k])
     n_launch = prof[dom][0]
     achieved = alg[dom] / (kernel_ms[dom] * 1e-3) / 1e9 if kernel_ms[dom] > 0 else 0.0
-    traffic, traffic_src = measured_traffic("streaming", dom)
+    traffic, traffic_src = measured_traffic(cfg["workload"], dom)
     pass_alg = 33.0 * N + 25.0 * P + 2.0 * S + 4.0 * N * lv.n_calls
 
     # end to end in place: candidates and reports copied per wave from pinned
