@@ -26,3 +26,17 @@ def test_plan_matches_oracle_reservations(B):
         assert np.array_equal(got, plan[w]), w
         o.gather_commit(x, *lv.reports(got), arena_bytes=lv.arena_bytes)
     o.close()
+
+
+def test_copy_traffic_only_for_the_captured_workload_and_run():
+    """The bench's roofline `traffic` is an ncu figure for one workload at one
+    size and the default run options; any other run reports it as null."""
+    import bench
+    full = "document->page: 1000000 parents, 16399843 children, 256 arrival waves, batch 256"
+    t, src = bench.measured_traffic(full, "asm_copy")
+    captured = bench.TRAFFIC[(full, "asm_copy")][1] == bench.source_sha16("asm_copy")
+    assert (t is not None and bool(src)) == captured   # null once the kernel's source changed
+    assert bench.measured_traffic(full, "asm_copy", default_run=False) == (None, None)
+    assert bench.measured_traffic(full, "commit_scatter") == (None, None)
+    small = "document->page: 60000 parents, 979486 children, 16 arrival waves, batch 256"
+    assert bench.measured_traffic(small, "asm_copy") == (None, None)
