@@ -42,3 +42,14 @@ def test_create_without_gpu_fails_cleanly():
     h = ctypes.c_void_p()
     st = pkg.load().ro_ctx_create(ctypes.byref(h), 0, None, 1)
     assert st == pkg.RO_E_CUDA and not h.value
+
+
+def test_binding_kernel_names_follow_the_header_ids():
+    """The binding's kernel names (profiling) are the header's RO_K_* ids in order."""
+    from paper_2609_18703_gb300._binding import KERNELS
+    src = open(os.path.join(ROOT, "include", "rayorch_gpu.h")).read()
+    block = re.search(r"enum \{\s*(RO_K_EXPAND_SCAN.*?)\};", src, re.S).group(1)
+    ids = {n: int(v) for n, v in re.findall(r"RO_K_(\w+)\s*=\s*(\d+)", block)}
+    count = ids.pop("COUNT")
+    assert sorted(ids.values()) == list(range(count))
+    assert [n.lower() for n, _ in sorted(ids.items(), key=lambda kv: kv[1])] == list(KERNELS)
