@@ -121,16 +121,11 @@ typedef struct {
  * ordered gathering are scoped to one input microbatch).  `stream` is a
  * cudaStream_t (NULL = legacy default stream) on device `device`; n_calls in
  * [1, 256] is the number of Calls whose Ready Queues the context keeps.
- * Three environment variables, read here, tune the context:
- * RO_COPY_SMALL_CHUNKS (copies of at most this many 16 KB chunks take the
- * direct path; default 256, 0 stages every copy), RO_ADMIT_TWO_PASS
- * (non-zero: every admission takes the two-pass path instead of the
- * one-pass cooperative kernel that lists of up to a few thousand tiles of
- * 2,048 candidates use) and RO_COMMIT_PARTITION_MIN (ro_gather_commit calls
- * of at least this many reports first group them by child range, keeping
- * each parent's reports in array order, so that the fence works on one
- * range's lineage state at a time; default 2^24; the results are the same
- * either way).
+ * Two environment variables, read here, tune the context: RO_COPY_SMALL_CHUNKS
+ * (copies of at most this many 16 KB chunks take the direct path; default
+ * 256, 0 stages every copy) and RO_ADMIT_TWO_PASS (non-zero: every
+ * admission takes the two-pass path instead of the one-pass cooperative
+ * kernel that lists of up to a few thousand tiles of 2,048 candidates use).
  */
 ro_status ro_ctx_create(ro_ctx** ctx, int32_t device, void* stream, uint32_t n_calls);
 ro_status ro_ctx_destroy(ro_ctx* ctx);
@@ -205,8 +200,7 @@ enum {
   RO_K_ASM_COPY = 8, RO_K_RETRY_CLAIM = 9, RO_K_RETRY_SCATTER = 10, RO_K_PB_KEYS = 11,
   RO_K_PB_HIST = 12, RO_K_PB_ROWSCAN = 13, RO_K_PB_SORT = 14, RO_K_PB_BOUNDS = 15,
   RO_K_PB_HEADS = 16, RO_K_PB_MARK = 17, RO_K_PB_SCAN = 18, RO_K_PB_EMIT = 19,
-  RO_K_COMMIT_FIX = 20, RO_K_READY_FUSED = 21, RO_K_PART_HIST = 22, RO_K_PART_SCAN = 23,
-  RO_K_PART_SCATTER = 24, RO_K_PART_UNPERMUTE = 25, RO_K_COUNT = 26
+  RO_K_COMMIT_FIX = 20, RO_K_READY_FUSED = 21, RO_K_COUNT = 22
 };
 /* Tracing (no counterpart in the paper; it instruments the path).  Every
  * kernel launch is counted; kernels whose bit (1 << RO_K_*) is set in

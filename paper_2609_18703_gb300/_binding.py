@@ -38,8 +38,7 @@ EXPORTS = ("ro_ctx_create", "ro_ctx_destroy", "ro_ctx_reset", "ro_ctx_sync", "ro
 KERNELS = ("expand_scan", "expand_fill", "ready_count", "ready_scatter", "commit_scatter",
            "commit_plan", "asm_parents", "asm_members", "asm_copy", "retry_claim", "retry_scatter",
            "pb_keys", "pb_hist", "pb_rowscan", "pb_sort", "pb_bounds", "pb_heads", "pb_mark",
-           "pb_scan", "pb_emit", "commit_fix", "ready_fused", "part_hist", "part_scan",
-           "part_scatter", "part_unpermute")
+           "pb_scan", "pb_emit", "commit_fix", "ready_fused")
 
 
 class RoError(RuntimeError):

@@ -163,7 +163,6 @@ struct ro_ctx {
   uint32_t n_calls = 1;
   uint32_t commit_seq = 0;              // commits issued on this context
   uint64_t copy_small_chunks = AC_SMALL_CHUNKS;   // copies this small go direct
-  uint64_t part_min = PT_MIN_REPORTS;             // commits this large are grouped by child range first
   int num_sms = 0;
   LaunchCfg L{}, Lp{}, Lc{}, Lf[FIN_STREAMS]{};
   DevScalars* ds = nullptr;
@@ -182,8 +181,6 @@ struct ro_ctx {
   std::vector<Expansion> exps;
   TsBuf ts[N_TS];
   DevBuf code;
-  // a large commit's reports grouped by child range (see PartArgs)
-  DevBuf pt_child, pt_state, pt_len, pt_off, pt_gen, pt_rix, pt_hist, pt_pfx, pt_btot, pt_edges;
   DevBuf selftest;                      // ro_ctx_selftest_timeout scratch
   DevBuf x_mb, x_coff, x_mtfp, x_hdr;   // explicit-list assembly scratch
   // parent-bound reservation scratch (see ParentArgs)
@@ -536,7 +533,6 @@ ro_status ro_ctx_create(ro_ctx** out, int32_t device, void* stream, uint32_t n_c
   for (auto& f : c->fin_stream) f = c->stream;
   c->n_calls = n_calls;
   if (const char* e = std::getenv("RO_COPY_SMALL_CHUNKS")) c->copy_small_chunks = std::strtoull(e, nullptr, 10);
-  if (const char* e = std::getenv("RO_COMMIT_PARTITION_MIN")) c->part_min = std::strtoull(e, nullptr, 10);
   cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
   if (cudaMalloc(&c->ds, sizeof(DevScalars)) != cudaSuccess ||
       cudaMallocHost(&c->hs, sizeof(DevScalars)) != cudaSuccess ||
@@ -630,8 +626,7 @@ ro_status ro_ctx_destroy(ro_ctx* c) {
   free_buf(c->code); free_buf(c->selftest); free_buf(c->x_mb); free_buf(c->x_coff); free_buf(c->x_mtfp); free_buf(c->x_hdr);
   for (DevBuf* b : {&c->pb_key[0], &c->pb_key[1], &c->pb_val[0], &c->pb_val[1], &c->pb_child,
                     &c->pb_hist, &c->pb_dtot, &c->pb_first, &c->pb_endp, &c->pb_hsz, &c->pb_left,
-                    &c->pb_hoff, &c->pb_rem, &c->pt_child, &c->pt_state, &c->pt_len, &c->pt_off,
-                    &c->pt_gen, &c->pt_rix, &c->pt_hist, &c->pt_pfx, &c->pt_btot, &c->pt_edges})
+                    &c->pb_hoff, &c->pb_rem})
     free_buf(*b);
   free_ev(c->fork); free_ev(c->x_planned); free_ev(c->join_plan); free_ev(c->join_copy);
   for (int k = 0; k < FIN_STREAMS; ++k) {
@@ -1183,57 +1178,12 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
     c->commit_seq = 1;
   }
   ca.seq = c->commit_seq;   // from 1: 0 in the barrier table means no barrier
-  // A commit of many reports groups them by child range first (k_partition.cu):
-  // the scatter then works on one range's slots and counters at a time.
-  const bool part = n > 0 && n >= c->part_min;
-  PartArgs pa{};
-  if (part) {
-    const uint64_t nt = ceil_div(n, (uint64_t)PT_TILE);
-    RO_TRY(ensure(c, c->pt_child, n * sizeof(uint32_t), "grouped reports"));
-    RO_TRY(ensure(c, c->pt_state, n, "grouped reports"));
-    RO_TRY(ensure(c, c->pt_len, n * sizeof(uint32_t), "grouped reports"));
-    RO_TRY(ensure(c, c->pt_off, n * sizeof(uint64_t), "grouped reports"));
-    if (d_gen) RO_TRY(ensure(c, c->pt_gen, n * sizeof(uint32_t), "grouped reports"));
-    if (d_code) RO_TRY(ensure(c, c->pt_rix, n * sizeof(uint32_t), "grouped reports"));
-    RO_TRY(ensure(c, c->pt_hist, PT_BUCKETS * nt * sizeof(uint32_t), "report grouping"));
-    RO_TRY(ensure(c, c->pt_pfx, PT_BUCKETS * nt * sizeof(uint32_t), "report grouping"));
-    RO_TRY(ensure(c, c->pt_btot, PT_BUCKETS * sizeof(uint32_t), "report grouping"));
-    RO_TRY(ensure(c, c->pt_edges, PT_BUCKETS * sizeof(uint32_t), "report grouping"));
-    pa.n_host = n;
-    pa.d_n = d_n;
-    pa.child = d_child;
-    pa.state = d_state;
-    pa.len = d_len;
-    pa.off = d_arena_off;
-    pa.gen = d_gen;
-    pa.child_p = (uint32_t*)c->pt_child.p;
-    pa.state_p = (uint8_t*)c->pt_state.p;
-    pa.len_p = (uint32_t*)c->pt_len.p;
-    pa.off_p = (uint64_t*)c->pt_off.p;
-    pa.gen_p = d_gen ? (uint32_t*)c->pt_gen.p : nullptr;
-    pa.rix_p = d_code ? (uint32_t*)c->pt_rix.p : nullptr;
-    pa.tfp = (const uint32_t*)S.tfp.p;
-    pa.n_fill_tiles = ceil_div(x->N, FILL_TILE);
-    pa.offsets = (const uint64_t*)S.offsets.p;
-    pa.edges = (uint32_t*)c->pt_edges.p;
-    pa.hist = (uint32_t*)c->pt_hist.p;
-    pa.pfx = (uint32_t*)c->pt_pfx.p;
-    pa.btot = (uint32_t*)c->pt_btot.p;
-    pa.n_tiles = nt;
-    ca.child = pa.child_p;
-    ca.state = pa.state_p;
-    ca.len = pa.len_p;
-    ca.off = pa.off_p;
-    ca.gen = pa.gen_p;
-  }
-  if (d_code && !part) {
+  if (d_code) {
     ca.code = d_code;
-  } else {   // verdicts in grouped order go back to the caller's order afterwards
+  } else {
     RO_TRY(ensure(c, c->code, n, "report verdicts"));
     ca.code = (uint8_t*)c->code.p;
   }
-  pa.code_p = ca.code;
-  pa.code_out = d_code;
   ca.done_user = d_done_parents;
   ca.done_int = (uint32_t*)LS.done.p;
   ca.n_done_out = d_n_done;
@@ -1277,18 +1227,12 @@ ro_status ro_gather_commit(ro_ctx* c, int32_t xid, uint64_t n, const uint64_t* d
       if (j == 0) break;
     }
   }
-  if (part) {
-    cudaError_t e = cudaMemsetAsync(pa.btot, 0, PT_BUCKETS * sizeof(uint32_t), c->stream);
-    if (e != cudaSuccess) return cuda_fail(c, e, "cudaMemsetAsync");
-    launch_partition(c->L, pa);
-  }
   launch_commit_scatter(c->L, ca);
   // the completed list and its plan follow the scatter (on their own stream
   // when the context has one); the list slot is free once the assembly that
   // read it (RING commits ago) is done
   const cudaStream_t fs = c->fin_stream[pf];
   RO_TRY(order(c, c->fin_fork[pf], c->stream, fs));
-  if (part && d_code) launch_unpermute(c->L, pa);   // the plan does not wait for it
   RO_TRY(ev_wait(c, LS.freed, fs));
   RO_TRY(ev_wait(c, LS.planned, fs));
   launch_commit_plan(c->Lf[pf], ca);

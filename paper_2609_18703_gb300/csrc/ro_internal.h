@@ -56,7 +56,7 @@ constexpr uint64_t AC_SMALL_CHUNKS = 256;
 enum KernelId { K_EXPAND_SCAN, K_FILL, K_RB_COUNT, K_RB_SCATTER, K_COMMIT, K_CPLAN, K_APARENTS,
                 K_AMEMBERS, K_ACOPY, K_RT_CLAIM, K_RT_SCATTER, K_PB_KEYS, K_PB_HIST,
                 K_PB_ROWSCAN, K_PB_SORT, K_PB_BOUNDS, K_PB_HEADS, K_PB_MARK, K_PB_SCAN, K_PB_EMIT,
-                K_CFIX, K_RB_FUSED, K_PT_HIST, K_PT_SCAN, K_PT_SCATTER, K_PT_UNPERM, K_COUNT,
+                K_CFIX, K_RB_FUSED, K_COUNT,
                 K_RB_FUSED_CALLS = 100 };   // occupancy query only (profiled as K_RB_FUSED)
 
 
@@ -303,42 +303,6 @@ struct CommitArgs {
 // different streams
 void launch_commit_scatter(const LaunchCfg& L, const CommitArgs& a);
 void launch_commit_plan(const LaunchCfg& L, const CommitArgs& a);
-
-// ---- a large commit's reports grouped by child range (k_partition.cu) -------------
-constexpr int PT_THREADS = 256;
-constexpr int PT_BUCKETS = 256;        // child ranges
-constexpr uint32_t PT_TILE = 2048;     // reports per tile of the grouping passes
-// commits of at least this many reports are grouped first
-// (RO_COMMIT_PARTITION_MIN in the environment at context creation overrides it)
-constexpr uint64_t PT_MIN_REPORTS = 1ull << 24;
-struct PartArgs {
-  uint64_t n_host;
-  const uint64_t* d_n;        // optional device count
-  const uint32_t* child;      // the caller's reports
-  const uint8_t* state;
-  const uint32_t* len;
-  const uint64_t* off;
-  const uint32_t* gen;        // optional
-  uint32_t* child_p;          // the same, grouped
-  uint8_t* state_p;
-  uint32_t* len_p;
-  uint64_t* off_p;
-  uint32_t* gen_p;            // when gen
-  uint32_t* rix_p;            // optional: each grouped report's index in the caller's arrays
-  const uint32_t* tfp;        // the expansion's fill-tile table and offsets (range edges)
-  uint64_t n_fill_tiles;
-  const uint64_t* offsets;
-  uint32_t* edges;            // PT_BUCKETS
-  uint32_t* hist;             // PT_BUCKETS x n_tiles: reports of range b in tile t
-  uint32_t* pfx;              // PT_BUCKETS x n_tiles: where they go
-  uint32_t* btot;             // PT_BUCKETS, zeroed before the launch
-  uint64_t n_tiles;           // ceil(n_host / PT_TILE)
-  const uint8_t* code_p;      // verdicts in grouped order
-  uint8_t* code_out;          // the caller's, in its order
-};
-// hist, scan, scatter on the context's stream
-void launch_partition(const LaunchCfg& L, const PartArgs& a);
-void launch_unpermute(const LaunchCfg& L, const PartArgs& a);
 
 // ---- ro_assemble ---------------------------------------------------------------------
 struct AssembleArgs {
